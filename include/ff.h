@@ -1,0 +1,211 @@
+/*
+ * ff.h -- C ABI of the GB300 (sm_103a) rollout denoising step of a
+ * flow-matching DiT under Flow-GRPO-style reinforcement learning.
+ *
+ * The step (paper Sec. 3.1, Eq. 1 and Table 1; Sec. 2.3 "advantage
+ * computation"):
+ *   1. v = v_theta(x_t, t)                        ff_dit_velocity
+ *   2. x_{t+dt} = Eq. 1 update, log p(x_{t+dt}|x_t) ff_sde_step_logprob
+ *   3. A = group-normalised reward                 ff_group_advantage
+ *   4. clipped-ratio policy loss over (b, step)    ff_grpo_loss
+ *
+ * Conventions for every entry point:
+ *   - Returns an int status: FF_OK or one of the FF_ERR_* codes below.  On
+ *     error nothing is launched and ff_last_error() (thread-local) says why.
+ *   - Array arguments are DEVICE pointers owned by the caller, unless the
+ *     comment says "host".  They must be 16-byte aligned (128-bit vector
+ *     access) and must not alias unless stated.
+ *   - Work is enqueued on the caller's stream; results are valid once that
+ *     stream has been synchronised.  No entry point synchronises the device,
+ *     and none allocates device memory: scratch space is a caller-owned
+ *     workspace whose size comes from the matching *_workspace_size query.
+ *   - Errors found inside a kernel (a bounded wait that ran out) set a device
+ *     status word; ff_check_device_status() reads and clears it.
+ */
+#ifndef FF_H
+#define FF_H
+
+#include <stddef.h>
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes ------------------------------------------------------ */
+#define FF_OK 0
+#define FF_ERR_INVALID_ARG 1   /* null pointer, bad size, misalignment, bad enum */
+#define FF_ERR_UNSUPPORTED 2   /* shape outside what the kernels handle        */
+#define FF_ERR_WORKSPACE 3     /* workspace missing or too small               */
+#define FF_ERR_CUDA 4          /* a CUDA runtime/driver call or launch failed  */
+#define FF_ERR_DEVICE_CHECK 5  /* a kernel reported an error via status word   */
+
+/* ---- enums ------------------------------------------------------------- */
+#define FF_SDE_SAMPLE 0   /* draw x_next = mean + std * eps and write it     */
+#define FF_SDE_EVAL 1     /* read the given x_next and only score it        */
+#define FF_LP_SUM 0       /* log-prob summed over the D elements of a sample */
+#define FF_LP_MEAN 1      /* ... divided by D                                */
+
+#define FF_SCHED_FLOW_SDE 0   /* Table 1: sigma_t = eta sqrt(t/(1-t))       */
+#define FF_SCHED_DANCE_SDE 1  /* Table 1: sigma_t = eta                     */
+#define FF_SCHED_ODE 2        /* Table 1: sigma_t = 0                       */
+
+#define FF_ARCH_MMDIT 0   /* Flux / Qwen-Image style double + single stream */
+
+/* Last error message of the calling thread ("" if none). */
+const char* ff_last_error(void);
+
+/* Library version, major*10000 + minor*100 + patch. */
+int ff_version(void);
+
+/* Reads and clears the device status word of the current device (0 = no
+ * kernel-reported error).  Synchronises the given stream first. */
+int ff_check_device_status(cudaStream_t stream, int* status_out);
+
+/* ------------------------------------------------------------------------
+ * Optional launch timing (off by default).  While enabled, every kernel the
+ * library launches is bracketed by two CUDA events recorded on its stream,
+ * and the record keeps the kernel's name and its algorithmic work (flops and
+ * bytes that the operation must do, not what the kernel happens to move).
+ * ff_prof_enable creates the events up front (host-side; no device memory);
+ * launches beyond max_records are not timed.  ff_prof_read synchronises on
+ * record i's end event.  Not for use under stream capture.
+ * ------------------------------------------------------------------------ */
+int ff_prof_enable(int max_records);
+int ff_prof_disable(void);
+int ff_prof_reset(void);
+int ff_prof_count(int* n);
+int ff_prof_read(int i, char* name, int name_cap, float* ms, double* flops, double* bytes);
+
+/* ------------------------------------------------------------------------
+ * Sampler schedule (host only).  Paper Table 1 and Eq. 1.
+ *   t_out[0..n_steps]: t_k = 1 - k/n_steps, mapped by the time shift
+ *     t' = shift t / (1 + (shift - 1) t) when shift != 1  (host array).
+ *   sigma_out[0..n_steps-1]: sigma at each step's start time t_k; for
+ *     FF_SCHED_FLOW_SDE t is clamped to t_clamp inside the square root
+ *     (the formula is singular at t = 1).  Host array.
+ * ------------------------------------------------------------------------ */
+int ff_sde_schedule(int kind, int n_steps, double shift, double eta, double t_clamp,
+                    double* t_out, double* sigma_out);
+
+/* ------------------------------------------------------------------------
+ * SDE step + Gaussian transition log-probability.  Paper Eq. 1, Table 1.
+ * Time runs from 1 (noise) to 0 (data); with Delta = t - t_next > 0,
+ *   mean = x - [v + sigma^2/(2t) (x + (1-t) v)] Delta,   std = sigma sqrt(Delta)
+ *   SAMPLE: x_next = mean + std * eps (written);  EVAL: x_next is read.
+ *   logp[b * ld] = sum_j -(x_next_j - mean_j)^2/(2 std^2) - D ln std - D/2 ln 2pi
+ *   (divided by D for FF_LP_MEAN).  A sample with std == 0 (ODE step) gets
+ *   x_next = mean and logp = 0.
+ *
+ * B samples of D fp32 elements each, row-major [B, D]; D % 4 == 0.
+ *   x_t, v:      [B, D] fp32, read.
+ *   eps:         [B, D] fp32, read in SAMPLE mode; may be NULL in EVAL mode.
+ *   x_next:      [B, D] fp32, written (SAMPLE) or read (EVAL).  May alias x_t
+ *                in SAMPLE mode (in-place update).
+ *   t, t_next, sigma: [B] fp32 each (device), per-sample times and sigma;
+ *                require 0 < t, t_next < t, sigma >= 0 (not checked on the
+ *                host: device values).
+ *   logp:        fp32, logp[b * ld] written for b < B; ld >= 1.
+ *   ws:          workspace of at least ff_sde_workspace_size(B, D) bytes.
+ * ------------------------------------------------------------------------ */
+int ff_sde_workspace_size(int B, int64_t D, size_t* bytes);
+int ff_sde_step_logprob(int B, int64_t D, const float* x_t, const float* v,
+                        const float* eps, float* x_next, const float* t,
+                        const float* t_next, const float* sigma, int mode, int reduce,
+                        float* logp, int ld, void* ws, size_t ws_bytes,
+                        cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Group-relative advantage (paper Sec. 2.3, advantage computation of the
+ * GRPO trainer).  Samples form contiguous groups of G (one prompt each):
+ *   A[g*G + i] = (r[g*G + i] - mean_g) / (std_g + eps_A),  std_g population.
+ * rewards, adv: [n_groups * G] fp32.  G in [1, 4096].  adv may alias rewards.
+ * ------------------------------------------------------------------------ */
+int ff_group_advantage(int n_groups, int G, const float* rewards, float eps_A,
+                       float* adv, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Clipped-ratio policy loss of Flow-GRPO (paper Sec. 3.1; PPO-style clip):
+ *   rho = exp(lp_new - lp_old),
+ *   loss = -1/(B T) sum_{b,k} min(rho A_b, clip(rho, 1 - clip_lo, 1 + clip_hi) A_b)
+ *   grad_lp_new[b,k] = -A_b rho / (B T) where the unclipped term is the
+ *   minimum (ties: unclipped), else 0.
+ * lp_new, lp_old: [B, T] fp32 row-major; adv: [B] fp32; loss: [1] fp32
+ * (written); grad_lp_new: [B, T] fp32 or NULL.
+ * ws: workspace of at least ff_grpo_loss_workspace_size(B, T) bytes.
+ * ------------------------------------------------------------------------ */
+int ff_grpo_loss_workspace_size(int B, int T, size_t* bytes);
+int ff_grpo_loss(int B, int T, const float* lp_new, const float* lp_old,
+                 const float* adv, float clip_lo, float clip_hi, float* loss,
+                 float* grad_lp_new, void* ws, size_t ws_bytes, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
+ * DiT velocity v_theta(x_t, t) (the network of Eq. 1 and Eq. 3).
+ *
+ * Architecture (MMDiT, Flux / Qwen-Image style): timestep embedding MLP and
+ * all adaLN modulations from one GEMM; patch and text embeddings; n_double
+ * double-stream blocks (per-stream weights, joint attention over
+ * [text; image]); n_single single-stream blocks; final LN-modulate + linear.
+ * LayerNorm has no affine and eps 1e-6; q and k get a per-head RMSNorm with a
+ * learned scale (eps 1e-6) and RoPE over (frame, row, col) slices of the head
+ * dim (rope_axes, sum = head_dim; pair (2j, 2j+1) of a slice of width a turns
+ * by pos * theta^(-2j/a)); text tokens sit at position (0, 0, 0); GELU is the
+ * tanh form; attention scale is 1/sqrt(d).
+ *
+ * Weights live in ONE caller-owned bf16 device blob; ff_dit_weight_layout
+ * gives every tensor's name, element offset and shape (nn.Linear [out, in]).
+ * ------------------------------------------------------------------------ */
+typedef struct ff_dit_config {
+    int arch;          /* FF_ARCH_MMDIT */
+    int hidden;        /* H, multiple of 64 */
+    int heads;         /* h */
+    int head_dim;      /* d: 64 or 128; h * d == H */
+    int mlp;           /* F, multiple of 64 */
+    int n_double;      /* double-stream blocks */
+    int n_single;      /* single-stream blocks */
+    int patch_dim;     /* P, latent token width (64), multiple of 16 */
+    int txt_dim;       /* D_txt, multiple of 64 */
+    int n_txt;         /* N_t text tokens per sample */
+    int grid_f, grid_h, grid_w;  /* latent token grid; N_i = f*h*w */
+    int rope_axes[3];  /* head-dim slice per (frame, row, col); even; sum = d */
+    float rope_theta;  /* 10000 */
+    int time_freq_dim; /* sinusoid features of 1000 t (256), multiple of 64 */
+} ff_dit_config;
+
+typedef struct ff_tensor_desc {
+    char name[64];     /* e.g. "double.0.img.qkv.w" */
+    int64_t offset;    /* in bf16 elements from the blob start (multiple of 64) */
+    int ndim;          /* 1 or 2 */
+    int64_t shape[2];  /* [out, in] for matrices, [n] for vectors */
+} ff_tensor_desc;
+
+typedef struct ff_dit ff_dit;
+
+/* Fills out[0..min(capacity, count)-1] (out may be NULL to query), sets
+ * *count and *total_elems (blob size in bf16 elements). */
+int ff_dit_weight_layout(const ff_dit_config* cfg, ff_tensor_desc* out, int capacity,
+                         int* count, int64_t* total_elems);
+
+/* Validates cfg and records the blob pointer (no copy, no device
+ * allocation).  The blob must stay alive and unchanged until destroy. */
+int ff_dit_create(const ff_dit_config* cfg, const void* weights_dev, ff_dit** out);
+int ff_dit_destroy(ff_dit* model);
+
+/* Workspace bytes for a velocity call on a batch of B samples. */
+int ff_dit_workspace_size(const ff_dit* model, int B, size_t* bytes);
+
+/* v_out[b, n, :] = v_theta(x_t[b], t[b], txt[b]).
+ *   x_t:   [B, N_i, P] fp32 latent tokens (row-major grid order)
+ *   txt:   [B, N_t, D_txt] bf16 cached text embeddings
+ *   t:     [B] fp32 times in (0, 1]
+ *   v_out: [B, N_i, P] fp32 (must not alias x_t)
+ *   ws:    at least ff_dit_workspace_size(model, B) bytes, 256-byte aligned */
+int ff_dit_velocity(const ff_dit* model, int B, const float* x_t, const void* txt,
+                    const float* t, float* v_out, void* ws, size_t ws_bytes,
+                    cudaStream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* FF_H */

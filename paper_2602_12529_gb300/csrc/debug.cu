@@ -1,0 +1,76 @@
+// debug.cu -- exported per-kernel entry points (include/ff_debug.h) used by
+// the stage-wise parity tests.  They only marshal arguments to the same
+// launchers ff_dit_velocity uses.
+#include "../../include/ff_debug.h"
+#include "internal.h"
+
+extern "C" {
+
+int ff_debug_gemm(int M, int N, int K, const void* A, int64_t lda, const void* B, int64_t ldb, const void* bias,
+                  int act, int out_f32, void* out, int64_t ldo, cudaStream_t stream) {
+    using namespace ff;
+    if (act < FF_ACT_NONE || act > FF_ACT_SILU) return set_error(FF_ERR_INVALID_ARG, "bad act %d", act);
+    GemmEpilogue e;
+    e.act = act;
+    e.out_f32 = out_f32 ? 1 : 0;
+    e.bias = static_cast<const __nv_bfloat16*>(bias);
+    e.out0 = out;
+    e.ld0 = ldo;
+    return gemm_bf16(A, lda, B, ldb, M, N, K, e, stream);
+}
+
+int ff_debug_gemm_gated(int M, int N, int K, const void* A, int64_t lda, const void* B, int64_t ldb, const void* bias,
+                        float* resid, int64_t ld_resid, const float* gate, int64_t ld_gate, int rows_per_sample,
+                        cudaStream_t stream) {
+    using namespace ff;
+    GemmEpilogue e;
+    e.epi = EPI_GATED_RESIDUAL;
+    e.bias = static_cast<const __nv_bfloat16*>(bias);
+    e.resid = resid;
+    e.ld_resid = ld_resid;
+    e.gate = gate;
+    e.ld_gate = ld_gate;
+    e.rows_per_sample = rows_per_sample;
+    return gemm_bf16(A, lda, B, ldb, M, N, K, e, stream);
+}
+
+int ff_debug_attention(int B, int heads, int head_dim, int n0, const void* qkv0, int64_t ld0, void* out0,
+                       int64_t ldo0, int n1, const void* qkv1, int64_t ld1, void* out1, int64_t ldo1,
+                       cudaStream_t stream) {
+    using namespace ff;
+    AttnSegment s0{static_cast<const __nv_bfloat16*>(qkv0), ld0, static_cast<__nv_bfloat16*>(out0), ldo0, n0};
+    AttnSegment s1{static_cast<const __nv_bfloat16*>(qkv1), ld1, static_cast<__nv_bfloat16*>(out1), ldo1, n1};
+    return attention(s0, s1, B, heads, head_dim, heads * head_dim, stream);
+}
+
+int ff_debug_ln_modulate(int rows, int H, const float* x, const float* mods, int64_t ld_mods, int shift_off,
+                         int scale_off, int tokens_per_sample, void* out, cudaStream_t stream) {
+    using namespace ff;
+    if (!x || !mods || !out || rows < 0 || H <= 0 || tokens_per_sample <= 0)
+        return set_error(FF_ERR_INVALID_ARG, "ln_modulate: bad arguments");
+    LnModArgs a{};
+    a.x = x; a.ldx = H; a.out = static_cast<__nv_bfloat16*>(out); a.ldo = H; a.rows = rows; a.H = H;
+    a.rows_txt = 0; a.n_txt = 1; a.n_img = tokens_per_sample; a.mods = mods; a.ld_mods = ld_mods;
+    a.shift_txt = a.shift_img = shift_off;
+    a.scale_txt = a.scale_img = scale_off;
+    return ln_modulate(a, stream);
+}
+
+int ff_debug_qk_norm_rope(int rows, int rows_txt, int heads, int head_dim, void* qkv, int64_t ld, const void* q_scale,
+                          const void* k_scale, int grid_f, int grid_h, int grid_w, const int* rope_axes,
+                          float rope_theta, cudaStream_t stream) {
+    using namespace ff;
+    if (!qkv || !q_scale || !k_scale || !rope_axes || rows < 0 || rows_txt < 0 || rows_txt > rows)
+        return set_error(FF_ERR_INVALID_ARG, "qk_norm_rope: bad arguments");
+    if (rope_axes[0] + rope_axes[1] + rope_axes[2] != head_dim)
+        return set_error(FF_ERR_INVALID_ARG, "qk_norm_rope: rope_axes must sum to head_dim");
+    QkNormRopeArgs a{};
+    a.qkv = static_cast<__nv_bfloat16*>(qkv); a.ld = ld; a.rows = rows; a.heads = heads; a.head_dim = head_dim;
+    a.rows_txt = rows_txt; a.n_img = grid_f * grid_h * grid_w; a.grid_f = grid_f; a.grid_h = grid_h; a.grid_w = grid_w;
+    a.axes0 = rope_axes[0]; a.axes1 = rope_axes[1]; a.axes2 = rope_axes[2]; a.theta = rope_theta;
+    a.q_scale_txt = a.q_scale_img = static_cast<const __nv_bfloat16*>(q_scale);
+    a.k_scale_txt = a.k_scale_img = static_cast<const __nv_bfloat16*>(k_scale);
+    return qk_norm_rope(a, stream);
+}
+
+}  // extern "C"

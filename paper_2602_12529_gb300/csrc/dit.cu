@@ -1,0 +1,365 @@
+// dit.cu -- the DiT velocity entry points: weight-blob layout, model handle,
+// workspace plan, and the launch sequence of one velocity call.
+//
+// Activation layout in the workspace (R_t = B N_t text rows, R_i = B N_i
+// image rows, R = R_t + R_i): every per-token buffer is "stream-major" --
+// rows [0, R_t) are the text tokens of samples 0..B-1 (sample-major), rows
+// [R_t, R) the image tokens.  A double-stream block runs each stream's GEMMs
+// on its contiguous row range with its own weights; a single-stream block
+// runs one GEMM over all R rows (row order is irrelevant to a Linear); only
+// attention (segments per sample) and the adaLN vectors (sample per row) need
+// the split.
+//
+//   mods  fp32 [B, W_mod]      all adaLN vectors (one GEMM per call)
+//   x     fp32 [R, H]          residual stream
+//   h     bf16 [R, H]          LN-modulated GEMM operand
+//   qkv   bf16 [R, 3H]         q | k | v (RMSNorm + RoPE applied in place)
+//   o     bf16 [R, H]          attention output (double-stream blocks)
+//   u     bf16 [R, H + F]      MLP hidden [R, F] (double) or [attn | GELU(mlp)] (single)
+#include <string.h>
+
+#include <string>
+#include <unordered_map>
+#include <vector>
+
+#include "internal.h"
+
+struct ff_dit {
+    ff_dit_config cfg;
+    const __nv_bfloat16* w;
+    std::unordered_map<std::string, int64_t> off;
+    int64_t mod_width;
+};
+
+namespace ff {
+namespace {
+
+struct Spec {
+    std::string name;
+    int ndim;
+    int64_t s0, s1;
+};
+
+int64_t mod_width(const ff_dit_config& c) {
+    const int64_t H = c.hidden;
+    return c.n_double * 12 * H + c.n_single * 3 * H + 2 * H;
+}
+
+// Same order and names as the oracle's parameter list.
+std::vector<Spec> specs(const ff_dit_config& c) {
+    const int64_t H = c.hidden, F = c.mlp, P = c.patch_dim, d = c.head_dim;
+    std::vector<Spec> s;
+    auto mat = [&](const std::string& n, int64_t o, int64_t i) { s.push_back({n, 2, o, i}); };
+    auto vec = [&](const std::string& n, int64_t o) { s.push_back({n, 1, o, 0}); };
+    mat("t_embed.fc1.w", H, c.time_freq_dim); vec("t_embed.fc1.b", H);
+    mat("t_embed.fc2.w", H, H); vec("t_embed.fc2.b", H);
+    mat("mod.w", mod_width(c), H); vec("mod.b", mod_width(c));
+    mat("img_in.w", H, P); vec("img_in.b", H);
+    mat("txt_in.w", H, c.txt_dim); vec("txt_in.b", H);
+    for (int l = 0; l < c.n_double; ++l) {
+        for (const char* st : {"img", "txt"}) {
+            const std::string p = "double." + std::to_string(l) + "." + st + ".";
+            mat(p + "qkv.w", 3 * H, H); vec(p + "qkv.b", 3 * H);
+            vec(p + "q_norm.scale", d); vec(p + "k_norm.scale", d);
+            mat(p + "proj.w", H, H); vec(p + "proj.b", H);
+            mat(p + "mlp1.w", F, H); vec(p + "mlp1.b", F);
+            mat(p + "mlp2.w", H, F); vec(p + "mlp2.b", H);
+        }
+    }
+    for (int l = 0; l < c.n_single; ++l) {
+        const std::string p = "single." + std::to_string(l) + ".";
+        mat(p + "linear1.w", 3 * H + F, H); vec(p + "linear1.b", 3 * H + F);
+        vec(p + "q_norm.scale", d); vec(p + "k_norm.scale", d);
+        mat(p + "linear2.w", H, H + F); vec(p + "linear2.b", H);
+    }
+    mat("final.w", P, H); vec("final.b", P);
+    return s;
+}
+
+int validate(const ff_dit_config* c) {
+    if (!c) return set_error(FF_ERR_INVALID_ARG, "config is null");
+    if (c->arch != FF_ARCH_MMDIT) return set_error(FF_ERR_UNSUPPORTED, "arch %d not supported", c->arch);
+    if (c->hidden <= 0 || c->hidden % 128) return set_error(FF_ERR_UNSUPPORTED, "hidden %d must be a multiple of 128", c->hidden);
+    if (c->head_dim != 64 && c->head_dim != 128) return set_error(FF_ERR_UNSUPPORTED, "head_dim %d", c->head_dim);
+    if (c->heads * c->head_dim != c->hidden) return set_error(FF_ERR_INVALID_ARG, "heads * head_dim != hidden");
+    if (c->mlp <= 0 || c->mlp % 64) return set_error(FF_ERR_UNSUPPORTED, "mlp %d must be a multiple of 64", c->mlp);
+    if (c->n_double < 0 || c->n_single < 0 || c->n_double + c->n_single < 1)
+        return set_error(FF_ERR_INVALID_ARG, "need at least one block");
+    if (c->patch_dim <= 0 || c->patch_dim % 32) return set_error(FF_ERR_UNSUPPORTED, "patch_dim %d", c->patch_dim);
+    if (c->txt_dim <= 0 || c->txt_dim % 8) return set_error(FF_ERR_UNSUPPORTED, "txt_dim %d", c->txt_dim);
+    if (c->n_txt <= 0) return set_error(FF_ERR_UNSUPPORTED, "n_txt must be positive");
+    if (c->grid_f <= 0 || c->grid_h <= 0 || c->grid_w <= 0) return set_error(FF_ERR_INVALID_ARG, "bad latent grid");
+    if (c->rope_axes[0] % 2 || c->rope_axes[1] % 2 || c->rope_axes[2] % 2 || c->rope_axes[0] < 0 ||
+        c->rope_axes[1] < 0 || c->rope_axes[2] < 0 ||
+        c->rope_axes[0] + c->rope_axes[1] + c->rope_axes[2] != c->head_dim)
+        return set_error(FF_ERR_INVALID_ARG, "rope_axes must be even and sum to head_dim");
+    if (!(c->rope_theta > 1.0f)) return set_error(FF_ERR_INVALID_ARG, "rope_theta must be > 1");
+    if (c->time_freq_dim <= 0 || c->time_freq_dim % 64) return set_error(FF_ERR_UNSUPPORTED, "time_freq_dim %d", c->time_freq_dim);
+    return FF_OK;
+}
+
+constexpr size_t kAlign = 256;
+size_t up(size_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
+
+struct Workspace {
+    float* mods;
+    __nv_bfloat16 *temb, *th, *tc;
+    float* x;
+    __nv_bfloat16 *xb, *h, *qkv, *o, *u;
+    size_t bytes;
+};
+
+Workspace plan(const ff_dit_config& c, int B, uint8_t* base) {
+    const size_t H = c.hidden, F = c.mlp;
+    const size_t Ni = static_cast<size_t>(c.grid_f) * c.grid_h * c.grid_w;
+    const size_t R = static_cast<size_t>(B) * (c.n_txt + Ni);
+    size_t o = 0;
+    Workspace w{};
+    auto take = [&](size_t bytes) { uint8_t* p = base ? base + o : nullptr; o += up(bytes); return p; };
+    w.mods = reinterpret_cast<float*>(take(static_cast<size_t>(B) * mod_width(c) * 4));
+    w.temb = reinterpret_cast<__nv_bfloat16*>(take(static_cast<size_t>(B) * c.time_freq_dim * 2));
+    w.th = reinterpret_cast<__nv_bfloat16*>(take(B * H * 2));
+    w.tc = reinterpret_cast<__nv_bfloat16*>(take(B * H * 2));
+    w.x = reinterpret_cast<float*>(take(R * H * 4));
+    w.xb = reinterpret_cast<__nv_bfloat16*>(take(B * Ni * c.patch_dim * 2));
+    w.h = reinterpret_cast<__nv_bfloat16*>(take(R * H * 2));
+    w.qkv = reinterpret_cast<__nv_bfloat16*>(take(R * 3 * H * 2));
+    w.o = reinterpret_cast<__nv_bfloat16*>(take(R * H * 2));
+    w.u = reinterpret_cast<__nv_bfloat16*>(take(R * (H + F) * 2));
+    w.bytes = o;
+    return w;
+}
+
+#define FF_TRY(expr)                \
+    do {                            \
+        const int rc_ = (expr);     \
+        if (rc_ != FF_OK) return rc_; \
+    } while (0)
+
+}  // namespace
+}  // namespace ff
+
+extern "C" {
+
+int ff_dit_weight_layout(const ff_dit_config* cfg, ff_tensor_desc* out, int capacity, int* count,
+                         int64_t* total_elems) {
+    using namespace ff;
+    FF_TRY(validate(cfg));
+    if (!count || !total_elems) return set_error(FF_ERR_INVALID_ARG, "count/total_elems is null");
+    const std::vector<Spec> s = specs(*cfg);
+    int64_t off = 0;
+    for (size_t i = 0; i < s.size(); ++i) {
+        const int64_t n = s[i].ndim == 2 ? s[i].s0 * s[i].s1 : s[i].s0;
+        if (out && static_cast<int>(i) < capacity) {
+            memset(&out[i], 0, sizeof(ff_tensor_desc));
+            strncpy(out[i].name, s[i].name.c_str(), sizeof(out[i].name) - 1);
+            out[i].offset = off;
+            out[i].ndim = s[i].ndim;
+            out[i].shape[0] = s[i].s0;
+            out[i].shape[1] = s[i].ndim == 2 ? s[i].s1 : 0;
+        }
+        off += (n + 63) / 64 * 64;   // every tensor starts on a 128-byte boundary
+    }
+    *count = static_cast<int>(s.size());
+    *total_elems = off;
+    return FF_OK;
+}
+
+int ff_dit_create(const ff_dit_config* cfg, const void* weights_dev, ff_dit** out) {
+    using namespace ff;
+    FF_TRY(validate(cfg));
+    if (!weights_dev || !out) return set_error(FF_ERR_INVALID_ARG, "weights/out is null");
+    if (!aligned16(weights_dev)) return set_error(FF_ERR_INVALID_ARG, "weight blob must be 16-byte aligned");
+    ff_dit* m = new ff_dit();
+    m->cfg = *cfg;
+    m->w = static_cast<const __nv_bfloat16*>(weights_dev);
+    m->mod_width = mod_width(*cfg);
+    int64_t off = 0;
+    for (const Spec& s : specs(*cfg)) {
+        m->off[s.name] = off;
+        const int64_t n = s.ndim == 2 ? s.s0 * s.s1 : s.s0;
+        off += (n + 63) / 64 * 64;
+    }
+    *out = m;
+    return FF_OK;
+}
+
+int ff_dit_destroy(ff_dit* m) {
+    delete m;
+    return FF_OK;
+}
+
+int ff_dit_workspace_size(const ff_dit* m, int B, size_t* bytes) {
+    using namespace ff;
+    if (!m || !bytes) return set_error(FF_ERR_INVALID_ARG, "model/bytes is null");
+    if (B <= 0) return set_error(FF_ERR_INVALID_ARG, "B=%d must be positive", B);
+    *bytes = plan(m->cfg, B, nullptr).bytes;
+    return FF_OK;
+}
+
+int ff_dit_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, const float* t, float* v_out, void* ws,
+                    size_t ws_bytes, cudaStream_t stream) {
+    using namespace ff;
+    if (!m) return set_error(FF_ERR_INVALID_ARG, "model is null");
+    if (B <= 0) return set_error(FF_ERR_INVALID_ARG, "B=%d must be positive", B);
+    if (!x_t || !txt || !t || !v_out || !ws) return set_error(FF_ERR_INVALID_ARG, "null pointer argument");
+    if (!aligned16(x_t) || !aligned16(txt) || !aligned16(v_out) || (reinterpret_cast<uintptr_t>(ws) % kAlign))
+        return set_error(FF_ERR_INVALID_ARG, "misaligned pointer (arrays 16 B, workspace 256 B)");
+    const ff_dit_config& c = m->cfg;
+    const Workspace w = plan(c, B, static_cast<uint8_t*>(ws));
+    if (ws_bytes < w.bytes) return set_error(FF_ERR_WORKSPACE, "workspace %zu B < %zu B needed", ws_bytes, w.bytes);
+
+    const int H = c.hidden, F = c.mlp, P = c.patch_dim, d = c.head_dim;
+    const int Nt = c.n_txt, Ni = c.grid_f * c.grid_h * c.grid_w;
+    const int Rt = B * Nt, Ri = B * Ni, R = Rt + Ri;
+    const int64_t Wm = m->mod_width;
+    auto W = [&](const std::string& n) { return m->w + m->off.at(n); };
+
+    // ---- timestep embedding MLP and every adaLN vector
+    FF_TRY(timestep_embed(t, B, c.time_freq_dim, w.temb, stream));
+    {
+        GemmEpilogue e;
+        e.act = ACT_SILU; e.bias = W("t_embed.fc1.b"); e.out0 = w.th; e.ld0 = H;
+        FF_TRY(gemm_bf16(w.temb, c.time_freq_dim, W("t_embed.fc1.w"), c.time_freq_dim, B, H, c.time_freq_dim, e, stream));
+    }
+    {
+        GemmEpilogue e;   // SiLU(c): only the modulation GEMM consumes c
+        e.act = ACT_SILU; e.bias = W("t_embed.fc2.b"); e.out0 = w.tc; e.ld0 = H;
+        FF_TRY(gemm_bf16(w.th, H, W("t_embed.fc2.w"), H, B, H, H, e, stream));
+    }
+    {
+        GemmEpilogue e;
+        e.out_f32 = 1; e.bias = W("mod.b"); e.out0 = w.mods; e.ld0 = Wm;
+        FF_TRY(gemm_bf16(w.tc, H, W("mod.w"), H, B, static_cast<int>(Wm), H, e, stream));
+    }
+
+    // ---- patch and text embeddings into the residual stream
+    FF_TRY(f32_to_bf16(x_t, w.xb, static_cast<int64_t>(Ri) * P, stream));
+    {
+        GemmEpilogue e;
+        e.out_f32 = 1; e.bias = W("img_in.b"); e.out0 = w.x + static_cast<int64_t>(Rt) * H; e.ld0 = H;
+        FF_TRY(gemm_bf16(w.xb, P, W("img_in.w"), P, Ri, H, P, e, stream));
+    }
+    {
+        GemmEpilogue e;
+        e.out_f32 = 1; e.bias = W("txt_in.b"); e.out0 = w.x; e.ld0 = H;
+        FF_TRY(gemm_bf16(txt, c.txt_dim, W("txt_in.w"), c.txt_dim, Rt, H, c.txt_dim, e, stream));
+    }
+
+    QkNormRopeArgs qa{};
+    qa.qkv = w.qkv; qa.ld = 3 * H; qa.rows = R; qa.heads = c.heads; qa.head_dim = d;
+    qa.rows_txt = Rt; qa.n_img = Ni; qa.grid_f = c.grid_f; qa.grid_h = c.grid_h; qa.grid_w = c.grid_w;
+    qa.axes0 = c.rope_axes[0]; qa.axes1 = c.rope_axes[1]; qa.axes2 = c.rope_axes[2]; qa.theta = c.rope_theta;
+
+    LnModArgs la{};
+    la.x = w.x; la.ldx = H; la.out = w.h; la.ldo = H; la.rows = R; la.H = H;
+    la.rows_txt = Rt; la.n_txt = Nt; la.n_img = Ni; la.mods = w.mods; la.ld_mods = Wm;
+
+    struct Stream { const char* name; int row0, rows, tokens; int64_t mod; };
+
+    // ---- double-stream blocks
+    for (int l = 0; l < c.n_double; ++l) {
+        const int64_t base = static_cast<int64_t>(l) * 12 * H;
+        const Stream st[2] = {{"txt", 0, Rt, Nt, base + 6 * H}, {"img", Rt, Ri, Ni, base}};
+        const std::string pre = "double." + std::to_string(l) + ".";
+        // LN-modulate 1
+        la.shift_txt = static_cast<int>(st[0].mod); la.scale_txt = static_cast<int>(st[0].mod + H);
+        la.shift_img = static_cast<int>(st[1].mod); la.scale_img = static_cast<int>(st[1].mod + H);
+        FF_TRY(ln_modulate(la, stream));
+        // QKV per stream
+        for (const Stream& s : st) {
+            const std::string p = pre + s.name + ".";
+            GemmEpilogue e;
+            e.bias = W(p + "qkv.b"); e.out0 = w.qkv + static_cast<int64_t>(s.row0) * 3 * H; e.ld0 = 3 * H;
+            FF_TRY(gemm_bf16(w.h + static_cast<int64_t>(s.row0) * H, H, W(p + "qkv.w"), H, s.rows, 3 * H, H, e, stream));
+        }
+        qa.q_scale_txt = W(pre + "txt.q_norm.scale"); qa.k_scale_txt = W(pre + "txt.k_norm.scale");
+        qa.q_scale_img = W(pre + "img.q_norm.scale"); qa.k_scale_img = W(pre + "img.k_norm.scale");
+        FF_TRY(qk_norm_rope(qa, stream));
+        {
+            AttnSegment a0{w.qkv, 3 * H, w.o, H, Nt};
+            AttnSegment a1{w.qkv + static_cast<int64_t>(Rt) * 3 * H, 3 * H, w.o + static_cast<int64_t>(Rt) * H, H, Ni};
+            FF_TRY(attention(a0, a1, B, c.heads, d, H, stream));
+        }
+        // projection + gated residual (gate1)
+        for (const Stream& s : st) {
+            const std::string p = pre + s.name + ".";
+            GemmEpilogue e;
+            e.epi = EPI_GATED_RESIDUAL; e.bias = W(p + "proj.b");
+            e.resid = w.x + static_cast<int64_t>(s.row0) * H; e.ld_resid = H;
+            e.gate = w.mods + s.mod + 2 * H; e.ld_gate = Wm; e.rows_per_sample = s.tokens;
+            FF_TRY(gemm_bf16(w.o + static_cast<int64_t>(s.row0) * H, H, W(p + "proj.w"), H, s.rows, H, H, e, stream));
+        }
+        // LN-modulate 2
+        la.shift_txt = static_cast<int>(st[0].mod + 3 * H); la.scale_txt = static_cast<int>(st[0].mod + 4 * H);
+        la.shift_img = static_cast<int>(st[1].mod + 3 * H); la.scale_img = static_cast<int>(st[1].mod + 4 * H);
+        FF_TRY(ln_modulate(la, stream));
+        // MLP
+        for (const Stream& s : st) {
+            const std::string p = pre + s.name + ".";
+            GemmEpilogue e;
+            e.act = ACT_GELU; e.bias = W(p + "mlp1.b"); e.out0 = w.u + static_cast<int64_t>(s.row0) * F; e.ld0 = F;
+            FF_TRY(gemm_bf16(w.h + static_cast<int64_t>(s.row0) * H, H, W(p + "mlp1.w"), H, s.rows, F, H, e, stream));
+        }
+        for (const Stream& s : st) {
+            const std::string p = pre + s.name + ".";
+            GemmEpilogue e;
+            e.epi = EPI_GATED_RESIDUAL; e.bias = W(p + "mlp2.b");
+            e.resid = w.x + static_cast<int64_t>(s.row0) * H; e.ld_resid = H;
+            e.gate = w.mods + s.mod + 5 * H; e.ld_gate = Wm; e.rows_per_sample = s.tokens;
+            FF_TRY(gemm_bf16(w.u + static_cast<int64_t>(s.row0) * F, F, W(p + "mlp2.w"), F, s.rows, H, F, e, stream));
+        }
+    }
+
+    // ---- single-stream blocks on the joint sequence
+    for (int l = 0; l < c.n_single; ++l) {
+        const int64_t off = static_cast<int64_t>(c.n_double) * 12 * H + static_cast<int64_t>(l) * 3 * H;
+        const std::string p = "single." + std::to_string(l) + ".";
+        la.shift_txt = la.shift_img = static_cast<int>(off);
+        la.scale_txt = la.scale_img = static_cast<int>(off + H);
+        FF_TRY(ln_modulate(la, stream));
+        {
+            GemmEpilogue e;   // [q k v] -> qkv ; GELU(mlp) -> u[:, H:]
+            e.bias = W(p + "linear1.b");
+            e.out0 = w.qkv; e.ld0 = 3 * H;
+            e.split_n = 3 * H; e.out1 = w.u; e.ld1 = H + F; e.col1 = H;
+            e.act = ACT_GELU; e.act_from = 3 * H;
+            FF_TRY(gemm_bf16(w.h, H, W(p + "linear1.w"), H, R, 3 * H + F, H, e, stream));
+        }
+        qa.q_scale_txt = qa.q_scale_img = W(p + "q_norm.scale");
+        qa.k_scale_txt = qa.k_scale_img = W(p + "k_norm.scale");
+        FF_TRY(qk_norm_rope(qa, stream));
+        {
+            AttnSegment a0{w.qkv, 3 * H, w.u, H + F, Nt};
+            AttnSegment a1{w.qkv + static_cast<int64_t>(Rt) * 3 * H, 3 * H, w.u + static_cast<int64_t>(Rt) * (H + F),
+                           H + F, Ni};
+            FF_TRY(attention(a0, a1, B, c.heads, d, H, stream));
+        }
+        // linear2 + gated residual, per segment (sample index differs)
+        const Stream st[2] = {{"txt", 0, Rt, Nt, off}, {"img", Rt, Ri, Ni, off}};
+        for (const Stream& s : st) {
+            GemmEpilogue e;
+            e.epi = EPI_GATED_RESIDUAL; e.bias = W(p + "linear2.b");
+            e.resid = w.x + static_cast<int64_t>(s.row0) * H; e.ld_resid = H;
+            e.gate = w.mods + off + 2 * H; e.ld_gate = Wm; e.rows_per_sample = s.tokens;
+            FF_TRY(gemm_bf16(w.u + static_cast<int64_t>(s.row0) * (H + F), H + F, W(p + "linear2.w"), H + F, s.rows,
+                             H, H + F, e, stream));
+        }
+    }
+
+    // ---- final layer on image tokens -> v (fp32)
+    {
+        const int64_t off = static_cast<int64_t>(c.n_double) * 12 * H + static_cast<int64_t>(c.n_single) * 3 * H;
+        LnModArgs f = la;
+        f.x = w.x + static_cast<int64_t>(Rt) * H; f.rows = Ri; f.rows_txt = 0;
+        f.shift_img = f.shift_txt = static_cast<int>(off);
+        f.scale_img = f.scale_txt = static_cast<int>(off + H);
+        FF_TRY(ln_modulate(f, stream));
+        GemmEpilogue e;
+        e.out_f32 = 1; e.bias = W("final.b"); e.out0 = v_out; e.ld0 = P;
+        FF_TRY(gemm_bf16(w.h, H, W("final.w"), H, Ri, P, H, e, stream));
+    }
+    return FF_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,211 @@
+// elementwise.cu -- the row-wise kernels of the DiT velocity:
+//   * ln_modulate: LayerNorm (no affine, eps 1e-6) then x (1 + scale) + shift
+//     with the sample's adaLN vectors, fp32 in -> bf16 GEMM operand out;
+//   * qk_norm_rope: per-head RMSNorm of q and k (learned scale, eps 1e-6)
+//     and the rotary embedding over (frame, row, col) slices of the head
+//     dim, in place on the bf16 qkv buffer;
+//   * timestep_embed: [cos | sin] of 1000 t times the sinusoid frequencies;
+//   * f32_to_bf16: operand conversion of the fp32 latent tokens.
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace ff {
+namespace {
+
+constexpr float kLnEps = 1e-6f;
+constexpr float kRmsEps = 1e-6f;
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// One warp per row; H % 128 == 0 so every lane owns H/128 float4s.  The row
+// is read three times (sum, centred sum of squares, output); the second and
+// third reads hit L1.
+__global__ void __launch_bounds__(256) ln_modulate_kernel(LnModArgs a) {
+    const int row = (blockIdx.x * 256 + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (row >= a.rows) return;
+    int b, sh, sc;
+    if (row < a.rows_txt) {
+        b = row / a.n_txt;
+        sh = a.shift_txt;
+        sc = a.scale_txt;
+    } else {
+        b = (row - a.rows_txt) / a.n_img;
+        sh = a.shift_img;
+        sc = a.scale_img;
+    }
+    const float4* x = reinterpret_cast<const float4*>(a.x + static_cast<int64_t>(row) * a.ldx);
+    const int nv = a.H >> 2;
+    float s = 0.f;
+    for (int i = lane; i < nv; i += 32) {
+        const float4 v = x[i];
+        s += (v.x + v.y) + (v.z + v.w);
+    }
+    const float mean = warp_sum(s) / a.H;
+    float q = 0.f;
+    for (int i = lane; i < nv; i += 32) {
+        const float4 v = x[i];
+        const float d0 = v.x - mean, d1 = v.y - mean, d2 = v.z - mean, d3 = v.w - mean;
+        q += (d0 * d0 + d1 * d1) + (d2 * d2 + d3 * d3);
+    }
+    const float rstd = rsqrtf(warp_sum(q) / a.H + kLnEps);
+    const float4* shift = reinterpret_cast<const float4*>(a.mods + static_cast<int64_t>(b) * a.ld_mods + sh);
+    const float4* scale = reinterpret_cast<const float4*>(a.mods + static_cast<int64_t>(b) * a.ld_mods + sc);
+    uint2* out = reinterpret_cast<uint2*>(a.out + static_cast<int64_t>(row) * a.ldo);
+    for (int i = lane; i < nv; i += 32) {
+        const float4 v = x[i];
+        const float4 h = shift[i];
+        const float4 c = scale[i];
+        const float y0 = (v.x - mean) * rstd * (1.f + c.x) + h.x;
+        const float y1 = (v.y - mean) * rstd * (1.f + c.y) + h.y;
+        const float y2 = (v.z - mean) * rstd * (1.f + c.z) + h.z;
+        const float y3 = (v.w - mean) * rstd * (1.f + c.w) + h.w;
+        out[i] = make_uint2(pack_bf16x2(y0, y1), pack_bf16x2(y2, y3));
+    }
+}
+
+// One warp per (row, head): lane owns E = d/32 consecutive elements (2 or 4),
+// i.e. whole rotation pairs.
+template <int E>
+__global__ void __launch_bounds__(256) qk_norm_rope_kernel(QkNormRopeArgs a) {
+    const int64_t gw = (static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (gw >= static_cast<int64_t>(a.rows) * a.heads) return;
+    const int row = static_cast<int>(gw / a.heads);
+    const int head = static_cast<int>(gw - static_cast<int64_t>(row) * a.heads);
+    const bool img = row >= a.rows_txt;
+    const int H = a.heads * a.head_dim;
+    const int c0 = lane * E;
+    const __nv_bfloat16* qs = img ? a.q_scale_img : a.q_scale_txt;
+    const __nv_bfloat16* ks = img ? a.k_scale_img : a.k_scale_txt;
+
+    // rotation of this lane's pairs (identity for text tokens at position 0)
+    float cs[E / 2], sn[E / 2];
+    if (img) {
+        const int n = (row - a.rows_txt) % a.n_img;
+        const int hw = a.grid_h * a.grid_w;
+        const float pos[3] = {static_cast<float>(n / hw), static_cast<float>((n / a.grid_w) % a.grid_h),
+                              static_cast<float>(n % a.grid_w)};
+        const float log2_theta = log2f(a.theta);
+#pragma unroll
+        for (int p = 0; p < E / 2; ++p) {
+            const int pair = c0 / 2 + p;
+            int axis, j, width;
+            if (pair < a.axes0 / 2) {
+                axis = 0; j = pair; width = a.axes0;
+            } else if (pair < (a.axes0 + a.axes1) / 2) {
+                axis = 1; j = pair - a.axes0 / 2; width = a.axes1;
+            } else {
+                axis = 2; j = pair - (a.axes0 + a.axes1) / 2; width = a.axes2;
+            }
+            const float freq = exp2f(-(2.0f * j / width) * log2_theta);
+            sincosf(pos[axis] * freq, &sn[p], &cs[p]);
+        }
+    } else {
+#pragma unroll
+        for (int p = 0; p < E / 2; ++p) { cs[p] = 1.f; sn[p] = 0.f; }
+    }
+
+#pragma unroll
+    for (int which = 0; which < 2; ++which) {
+        __nv_bfloat16* ptr = a.qkv + static_cast<int64_t>(row) * a.ld + which * H + head * a.head_dim + c0;
+        const __nv_bfloat16* sc = (which == 0 ? qs : ks) + c0;
+        float v[E];
+        if (E == 4) {
+            const uint2 u = *reinterpret_cast<const uint2*>(ptr);
+            const float2 f0 = unpack_bf16x2(u.x), f1 = unpack_bf16x2(u.y);
+            v[0] = f0.x; v[1] = f0.y; v[2 % E] = f1.x; v[3 % E] = f1.y;
+        } else {
+            const float2 f0 = unpack_bf16x2(*reinterpret_cast<const uint32_t*>(ptr));
+            v[0] = f0.x; v[1 % E] = f0.y;
+        }
+        float ss = 0.f;
+#pragma unroll
+        for (int i = 0; i < E; ++i) ss += v[i] * v[i];
+        const float r = rsqrtf(warp_sum(ss) / a.head_dim + kRmsEps);
+#pragma unroll
+        for (int i = 0; i < E; ++i) v[i] = v[i] * r * __bfloat162float(sc[i]);
+        float o[E];
+#pragma unroll
+        for (int p = 0; p < E / 2; ++p) {
+            o[2 * p] = v[2 * p] * cs[p] - v[2 * p + 1] * sn[p];
+            o[2 * p + 1] = v[2 * p] * sn[p] + v[2 * p + 1] * cs[p];
+        }
+        if (E == 4) {
+            *reinterpret_cast<uint2*>(ptr) = make_uint2(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2 % E], o[3 % E]));
+        } else {
+            *reinterpret_cast<uint32_t*>(ptr) = pack_bf16x2(o[0], o[1 % E]);
+        }
+    }
+}
+
+__global__ void timestep_embed_kernel(const float* t, int B, int dim, __nv_bfloat16* out) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= B * dim) return;
+    const int b = i / dim;
+    const int j = i - b * dim;
+    const int half = dim / 2;
+    const int f = j < half ? j : j - half;
+    const double freq = exp(-9.210340371976184 * static_cast<double>(f) / half);   // ln(1e4)
+    const double arg = 1000.0 * static_cast<double>(t[b]) * freq;
+    out[i] = __float2bfloat16_rn(static_cast<float>(j < half ? cos(arg) : sin(arg)));
+}
+
+__global__ void f32_to_bf16_kernel(const float4* in, uint2* out, int64_t n4) {
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n4;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const float4 v = __ldcs(in + i);
+        out[i] = make_uint2(pack_bf16x2(v.x, v.y), pack_bf16x2(v.z, v.w));
+    }
+}
+
+}  // namespace
+
+int ln_modulate(const LnModArgs& a, cudaStream_t stream) {
+    if (a.rows <= 0) return FF_OK;
+    if (a.H % 128 || a.ldx % 4 || a.ldo % 4 || a.ld_mods % 4 || (a.shift_txt | a.scale_txt | a.shift_img | a.scale_img) % 4)
+        return set_error(FF_ERR_UNSUPPORTED, "ln_modulate: H=%d must be a multiple of 128", a.H);
+    const int grid = (a.rows + 7) / 8;
+    ProfScope prof(stream, "ln_modulate", 0.0, static_cast<double>(a.rows) * a.H * 6.0);
+    ln_modulate_kernel<<<grid, 256, 0, stream>>>(a);
+    return check_launch("ln_modulate_kernel");
+}
+
+int qk_norm_rope(const QkNormRopeArgs& a, cudaStream_t stream) {
+    if (a.rows <= 0) return FF_OK;
+    const int64_t warps = static_cast<int64_t>(a.rows) * a.heads;
+    const int64_t grid = (warps + 7) / 8;
+    if (grid > 0x7fffffff) return set_error(FF_ERR_UNSUPPORTED, "qk_norm_rope: too many rows");
+    ProfScope prof(stream, "qk_norm_rope", 0.0, static_cast<double>(a.rows) * a.heads * a.head_dim * 8.0);
+    if (a.head_dim == 128)
+        qk_norm_rope_kernel<4><<<static_cast<unsigned>(grid), 256, 0, stream>>>(a);
+    else if (a.head_dim == 64)
+        qk_norm_rope_kernel<2><<<static_cast<unsigned>(grid), 256, 0, stream>>>(a);
+    else
+        return set_error(FF_ERR_UNSUPPORTED, "qk_norm_rope: head_dim %d", a.head_dim);
+    return check_launch("qk_norm_rope_kernel");
+}
+
+int timestep_embed(const float* t, int B, int dim, __nv_bfloat16* out, cudaStream_t stream) {
+    const int n = B * dim;
+    ProfScope prof(stream, "timestep_embed", 0.0, 4.0 * B + 2.0 * n);
+    timestep_embed_kernel<<<(n + 255) / 256, 256, 0, stream>>>(t, B, dim, out);
+    return check_launch("timestep_embed_kernel");
+}
+
+int f32_to_bf16(const float* in, __nv_bfloat16* out, int64_t n, cudaStream_t stream) {
+    if (n % 4) return set_error(FF_ERR_UNSUPPORTED, "f32_to_bf16: n %% 4 != 0");
+    const int64_t n4 = n / 4;
+    int64_t grid = (n4 + 255) / 256;
+    if (grid > 4 * num_sms() * 8) grid = 4 * num_sms() * 8;
+    ProfScope prof(stream, "f32_to_bf16", 0.0, 6.0 * n);
+    f32_to_bf16_kernel<<<static_cast<unsigned>(grid), 256, 0, stream>>>(reinterpret_cast<const float4*>(in),
+                                                                        reinterpret_cast<uint2*>(out), n4);
+    return check_launch("f32_to_bf16_kernel");
+}
+
+}  // namespace ff

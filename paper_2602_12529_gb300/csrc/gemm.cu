@@ -1,0 +1,333 @@
+// gemm.cu -- persistent, warp-specialised tcgen05 GEMM for sm_103a.
+//
+//   D[M, N] = A[M, K] * B[N, K]^T      (bf16 operands, fp32 accumulation)
+//
+// Every Linear of the DiT (nn.Linear weights [out, in], activations [tokens,
+// in]) runs through this kernel.  Layout per CTA (one CTA per SM):
+//   warp 0      TMA producer: 128x64 A tile + BNx64 B tile per stage, 128-byte
+//               swizzle, STAGES-deep mbarrier ring.
+//   warp 1      TMEM allocator; lane 0 issues tcgen05.mma (M=128, N=BN, K=16
+//               per instruction) into one of two TMEM accumulators.
+//   warps 2..5  epilogue: tcgen05.ld of the accumulator (one TMEM lane = one
+//               output row per thread), then the fused tail -- bias, GELU or
+//               SiLU, and either a bf16/fp32 store (optionally split over two
+//               outputs by column) or the adaLN gated residual update
+//               x += gate[b] * (acc + bias) on the fp32 residual stream.
+// The two TMEM accumulators let the epilogue of tile i overlap the main loop
+// of tile i+1.  Tiles are visited in groups of 16 M-blocks so that the A and
+// B panels being read at any moment stay resident in L2.
+//
+// Every wait is bounded (ptx.cuh); on a timeout the kernel records
+// kStatusWaitTimeout in the device status word, drains its own tensor-core
+// work, frees TMEM and returns.
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace ff {
+namespace {
+
+constexpr int BM = 128;
+constexpr int BK = 64;
+constexpr int kThreads = 192;
+constexpr int kGroupM = 16;
+
+template <int BN>
+struct Cfg {
+    static constexpr int kStages = BN == 256 ? 4 : (BN == 128 ? 6 : 8);
+    static constexpr int kABytes = BM * BK * 2;
+    static constexpr int kBBytes = BN * BK * 2;
+    static constexpr int kStageBytes = kABytes + kBBytes;
+    static constexpr int kTmemCols = 2 * BN;
+    static constexpr int kBarrierBytes = 256;
+    static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + kBarrierBytes;
+};
+
+__device__ __forceinline__ void tile_coords(int tile, int num_m, int num_n, int& mb, int& nb) {
+    const int group_tiles = kGroupM * num_n;
+    const int group = tile / group_tiles;
+    const int first_m = group * kGroupM;
+    const int gm = min(num_m - first_m, kGroupM);
+    const int local = tile - group * group_tiles;
+    mb = first_m + local % gm;
+    nb = local / gm;
+}
+
+__device__ __forceinline__ void bias_add8(float* v, const __nv_bfloat16* b) {
+    const uint4 u = *reinterpret_cast<const uint4*>(b);
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const float2 f = unpack_bf16x2(w[i]);
+        v[2 * i] += f.x;
+        v[2 * i + 1] += f.y;
+    }
+}
+
+// Fused tail for one 32-column chunk of one output row held by this thread.
+__device__ __forceinline__ void epilogue_chunk(const GemmEpilogue& e, int M, int row, int n, float (&v)[32]) {
+    if (e.bias) {
+#pragma unroll
+        for (int j = 0; j < 4; ++j) bias_add8(v + 8 * j, e.bias + n + 8 * j);
+    }
+    if (e.act != ACT_NONE && n >= e.act_from) {
+        if (e.act == ACT_GELU) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = gelu_tanh(v[i]);
+        } else {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = silu(v[i]);
+        }
+    }
+    if (row >= M) return;
+    if (e.epi == EPI_GATED_RESIDUAL) {
+        const int b = row / e.rows_per_sample;
+        const float4* g = reinterpret_cast<const float4*>(e.gate + static_cast<int64_t>(b) * e.ld_gate + n);
+        float4* x = reinterpret_cast<float4*>(e.resid + static_cast<int64_t>(row) * e.ld_resid + n);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            const float4 gv = g[j];
+            float4 xv = x[j];
+            xv.x += gv.x * v[4 * j];
+            xv.y += gv.y * v[4 * j + 1];
+            xv.z += gv.z * v[4 * j + 2];
+            xv.w += gv.w * v[4 * j + 3];
+            x[j] = xv;
+        }
+        return;
+    }
+    void* base;
+    int64_t ld;
+    int col;
+    if (n < e.split_n) {
+        base = e.out0; ld = e.ld0; col = n;
+    } else {
+        base = e.out1; ld = e.ld1; col = n - e.split_n + e.col1;
+    }
+    if (e.out_f32) {
+        float4* o = reinterpret_cast<float4*>(static_cast<float*>(base) + static_cast<int64_t>(row) * ld + col);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) o[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+    } else {
+        uint4* o = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(base) + static_cast<int64_t>(row) * ld + col);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const float* s = v + 8 * j;
+            o[j] = make_uint4(pack_bf16x2(s[0], s[1]), pack_bf16x2(s[2], s[3]), pack_bf16x2(s[4], s[5]),
+                              pack_bf16x2(s[6], s[7]));
+        }
+    }
+}
+
+template <int BN>
+__global__ void __launch_bounds__(kThreads, 1)
+gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b, int M,
+                    int N, int K, const GemmEpilogue epi, int* status) {
+    using C = Cfg<BN>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint64_t* full_bar = reinterpret_cast<uint64_t*>(smem + C::kStages * C::kStageBytes);
+    uint64_t* empty_bar = full_bar + C::kStages;
+    uint64_t* tfull_bar = empty_bar + C::kStages;   // [2]
+    uint64_t* tempty_bar = tfull_bar + 2;           // [2]
+    uint64_t* drain_bar = tempty_bar + 2;           // [1]
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_bar + 1);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < C::kStages; ++s) {
+            mbar_init(&full_bar[s], 1);
+            mbar_init(&empty_bar[s], 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(&tfull_bar[a], 1);
+            mbar_init(&tempty_bar[a], 4);
+        }
+        mbar_init(drain_bar, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+        prefetch_tmap(&tm_a);
+        prefetch_tmap(&tm_b);
+    }
+    if (warp == 1) {
+        tmem_alloc(tmem_slot, C::kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+
+    const int num_m = (M + BM - 1) / BM;
+    const int num_n = (N + BN - 1) / BN;
+    const int num_tiles = num_m * num_n;
+    const int num_k = (K + BK - 1) / BK;
+
+    if (warp == 0 && lane == 0) {
+        // ---------------- TMA producer
+        int stage = 0;
+        uint32_t phase = 0;
+        for (int tile = blockIdx.x; tile < num_tiles && !*abort_flag; tile += gridDim.x) {
+            int mb, nb;
+            tile_coords(tile, num_m, num_n, mb, nb);
+            for (int kb = 0; kb < num_k; ++kb) {
+                if (!mbar_wait(&empty_bar[stage], phase ^ 1)) {
+                    report_status(status, kStatusWaitTimeout);
+                    *abort_flag = 1;
+                    break;
+                }
+                uint8_t* sa = smem + stage * C::kStageBytes;
+                uint8_t* sb = sa + C::kABytes;
+                mbar_arrive_expect_tx(&full_bar[stage], C::kStageBytes);
+                tma_load_2d(sa, &tm_a, &full_bar[stage], kb * BK, mb * BM);
+                tma_load_2d(sb, &tm_b, &full_bar[stage], kb * BK, nb * BN);
+                if (++stage == C::kStages) { stage = 0; phase ^= 1; }
+            }
+        }
+    } else if (warp == 1 && lane == 0) {
+        // ---------------- MMA issuer
+        constexpr uint32_t idesc = idesc_bf16_f32(BM, BN);
+        int stage = 0;
+        uint32_t phase = 0;
+        int acc = 0;
+        uint32_t acc_phase = 0;
+        for (int tile = blockIdx.x; tile < num_tiles && !*abort_flag; tile += gridDim.x) {
+            if (!mbar_wait(&tempty_bar[acc], acc_phase ^ 1)) {
+                report_status(status, kStatusWaitTimeout);
+                *abort_flag = 1;
+                break;
+            }
+            tc_fence_after();
+            const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
+            bool ok = true;
+            for (int kb = 0; kb < num_k; ++kb) {
+                if (!mbar_wait(&full_bar[stage], phase)) {
+                    report_status(status, kStatusWaitTimeout);
+                    *abort_flag = 1;
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t sa = smem_u32(smem + stage * C::kStageBytes);
+                const uint32_t sb = sa + C::kABytes;
+                const uint64_t da = smem_desc_k_sw128(sa);
+                const uint64_t db = smem_desc_k_sw128(sb);
+#pragma unroll
+                for (int k = 0; k < BK / 16; ++k) {
+                    // +32 bytes per 16-element K step (encoded >> 4)
+                    tc_mma_bf16(d_tmem, da + static_cast<uint64_t>(2 * k), db + static_cast<uint64_t>(2 * k), idesc,
+                                (kb | k) != 0 ? 1u : 0u);
+                }
+                tc_commit(&empty_bar[stage]);
+                if (++stage == C::kStages) { stage = 0; phase ^= 1; }
+            }
+            if (!ok) break;
+            tc_commit(&tfull_bar[acc]);
+            if (++acc == 2) { acc = 0; acc_phase ^= 1; }
+        }
+        // all tensor-core work of this thread finished before TMEM is freed
+        tc_commit(drain_bar);
+        if (!mbar_wait(drain_bar, 0)) report_status(status, kStatusWaitTimeout);
+    } else if (warp >= 2) {
+        // ---------------- epilogue (4 warps; warp w reads TMEM lanes 32*(w%4)..)
+        const int q = warp & 3;
+        int acc = 0;
+        uint32_t acc_phase = 0;
+        for (int tile = blockIdx.x; tile < num_tiles && !*abort_flag; tile += gridDim.x) {
+            int mb, nb;
+            tile_coords(tile, num_m, num_n, mb, nb);
+            if (!mbar_wait(&tfull_bar[acc], acc_phase)) {
+                report_status(status, kStatusWaitTimeout);
+                *abort_flag = 1;
+                break;
+            }
+            tc_fence_after();
+            const int row = mb * BM + q * 32 + lane;
+            const uint32_t t_acc = tmem_base + static_cast<uint32_t>(acc * BN) + (static_cast<uint32_t>(q * 32) << 16);
+#pragma unroll 1
+            for (int c = 0; c < BN; c += 32) {
+                uint32_t r[32];
+                tmem_ld_x32(t_acc + c, r);
+                tmem_ld_wait();
+                const int n = nb * BN + c;
+                if (n >= N) continue;
+                float v[32];
+#pragma unroll
+                for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+                epilogue_chunk(epi, M, row, n, v);
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&tempty_bar[acc]);
+            if (++acc == 2) { acc = 0; acc_phase ^= 1; }
+        }
+    }
+
+    if (*abort_flag) {
+        // let bulk copies already in flight land before the CTA exits
+        const uint64_t t0 = global_timer_ns();
+        while (global_timer_ns() - t0 < 50000ull) {
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem_base, C::kTmemCols);
+    }
+}
+
+template <int BN>
+int launch(const void* A, int64_t lda, const void* B, int64_t ldb, int M, int N, int K, const GemmEpilogue& epi,
+           cudaStream_t stream) {
+    using C = Cfg<BN>;
+    if (cudaFuncSetAttribute(gemm_tcgen05_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes) !=
+        cudaSuccess)
+        return set_error(FF_ERR_CUDA, "gemm: cannot set shared memory size (%d B)", C::kSmemBytes);
+    CUtensorMap ta, tb;
+    int rc = make_tmap_bf16(&ta, A, M, K, lda, BM);
+    if (rc) return rc;
+    rc = make_tmap_bf16(&tb, B, N, K, ldb, BN);
+    if (rc) return rc;
+    const int tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN);
+    const int grid = tiles < num_sms() ? tiles : num_sms();
+    const double mn = static_cast<double>(M) * N;
+    const double out_bytes = epi.epi == EPI_GATED_RESIDUAL ? mn * 8.0 : mn * (epi.out_f32 ? 4.0 : 2.0);
+    ProfScope prof(stream, "gemm_bf16", 2.0 * mn * K, 2.0 * (static_cast<double>(M) + N) * K + out_bytes);
+    gemm_tcgen05_kernel<BN><<<grid, kThreads, C::kSmemBytes, stream>>>(ta, tb, M, N, K, epi, device_status_ptr());
+    return check_launch("gemm_tcgen05_kernel");
+}
+
+}  // namespace
+
+int gemm_bf16(const void* A, int64_t lda, const void* B, int64_t ldb, int M, int N, int K, const GemmEpilogue& e,
+              cudaStream_t stream) {
+    if (!A || !B) return set_error(FF_ERR_INVALID_ARG, "gemm: null operand");
+    if (M <= 0 || N <= 0 || K <= 0) return set_error(FF_ERR_INVALID_ARG, "gemm: bad shape %d x %d x %d", M, N, K);
+    if (N % 32 != 0) return set_error(FF_ERR_UNSUPPORTED, "gemm: N=%d not a multiple of 32", N);
+    if (K % 8 != 0 || lda % 8 != 0 || ldb % 8 != 0 || lda < K || ldb < K)
+        return set_error(FF_ERR_UNSUPPORTED, "gemm: K/ld must be multiples of 8 (K=%d lda=%lld ldb=%lld)", K,
+                         (long long)lda, (long long)ldb);
+    if (e.bias && !aligned16(e.bias)) return set_error(FF_ERR_INVALID_ARG, "gemm: bias not 16-byte aligned");
+    if (e.epi == EPI_GATED_RESIDUAL) {
+        if (!e.resid || !e.gate || e.rows_per_sample <= 0 || !aligned16(e.resid) || !aligned16(e.gate) ||
+            e.ld_resid % 4 || e.ld_gate % 4)
+            return set_error(FF_ERR_INVALID_ARG, "gemm: bad gated-residual epilogue");
+    } else {
+        if (!e.out0 || !aligned16(e.out0)) return set_error(FF_ERR_INVALID_ARG, "gemm: bad output");
+        const int vec = e.out_f32 ? 4 : 8;
+        if (e.ld0 % vec) return set_error(FF_ERR_INVALID_ARG, "gemm: output ld not vector aligned");
+        if (e.split_n < N) {
+            if (e.split_n % 32 || !e.out1 || !aligned16(e.out1) || e.ld1 % vec || e.col1 % vec)
+                return set_error(FF_ERR_INVALID_ARG, "gemm: bad split output");
+        }
+    }
+    if (e.act != ACT_NONE && e.act_from % 32) return set_error(FF_ERR_INVALID_ARG, "gemm: act_from % 32 != 0");
+    if (N <= 64) return launch<64>(A, lda, B, ldb, M, N, K, e, stream);
+    if (N <= 128) return launch<128>(A, lda, B, ldb, M, N, K, e, stream);
+    return launch<256>(A, lda, B, ldb, M, N, K, e, stream);
+}
+
+}  // namespace ff

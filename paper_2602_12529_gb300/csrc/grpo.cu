@@ -1,0 +1,146 @@
+// grpo.cu -- group-relative advantage and the clipped-ratio policy loss of
+// Flow-GRPO (paper Sec. 2.3 "advantage computation", Sec. 3.1).
+//
+// Advantage: one warp per group of G contiguous samples; mean and population
+// std in fp64 (two passes over the group held in L1), then
+// A = (r - mean) / (std + eps_A).
+//
+// Loss: rho = exp(lp_new - lp_old) per (sample, step);
+//   obj = min(rho A, clip(rho, 1 - lo, 1 + hi) A), loss = -sum(obj) / (B T),
+//   grad_lp_new = -A rho / (B T) where the unclipped term is the minimum.
+// Pass 1 writes one fp64 partial per block (grid size depends only on B T, so
+// the summation order is fixed); pass 2 adds the partials in order.
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace ff {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kElemsPerBlock = kThreads * 4;
+constexpr int kMaxLossBlocks = 1024;
+
+__global__ void __launch_bounds__(kThreads) group_advantage_kernel(int n_groups, int G, const float* r, float eps,
+                                                                   float* adv) {
+    const int warp = (blockIdx.x * kThreads + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (warp >= n_groups) return;
+    const float* rg = r + static_cast<int64_t>(warp) * G;
+    double s = 0.0;
+    for (int i = lane; i < G; i += 32) s += rg[i];
+#pragma unroll
+    for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    const double mean = s / G;
+    double q = 0.0;
+    for (int i = lane; i < G; i += 32) {
+        const double d = rg[i] - mean;
+        q += d * d;
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) q += __shfl_xor_sync(0xffffffffu, q, o);
+    const double denom = sqrt(q / G) + static_cast<double>(eps);
+    float* ag = adv + static_cast<int64_t>(warp) * G;
+    // each lane rewrites only the elements it reads itself, after the
+    // reductions above, so adv may alias r
+    for (int i = lane; i < G; i += 32) ag[i] = static_cast<float>((static_cast<double>(rg[i]) - mean) / denom);
+}
+
+__global__ void __launch_bounds__(kThreads) grpo_loss_partial_kernel(int64_t n, int T, const float* lp_new,
+                                                                     const float* lp_old, const float* adv,
+                                                                     float lo, float hi, float inv_n,
+                                                                     float* grad, double* partial) {
+    __shared__ double red[kThreads / 32];
+    double s = 0.0;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; i < n;
+         i += static_cast<int64_t>(gridDim.x) * kThreads) {
+        const float a = adv[i / T];
+        const float rho = expf(lp_new[i] - lp_old[i]);
+        const float unclipped = rho * a;
+        const float clipped = fminf(fmaxf(rho, 1.0f - lo), 1.0f + hi) * a;
+        const bool take = unclipped <= clipped;
+        s += static_cast<double>(take ? unclipped : clipped);
+        if (grad) grad[i] = take ? -a * rho * inv_n : 0.0f;
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double t = 0.0;
+        for (int w = 0; w < kThreads / 32; ++w) t += red[w];
+        partial[blockIdx.x] = t;
+    }
+}
+
+__global__ void grpo_loss_finalize_kernel(int nblocks, const double* partial, double inv_n, float* loss) {
+    __shared__ double red[kThreads / 32];
+    double s = 0.0;
+    for (int i = threadIdx.x; i < nblocks; i += blockDim.x) s += partial[i];
+#pragma unroll
+    for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double t = 0.0;
+        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += red[w];
+        *loss = static_cast<float>(-t * inv_n);
+    }
+}
+
+int loss_blocks(int64_t n) {
+    const int64_t b = (n + kElemsPerBlock - 1) / kElemsPerBlock;
+    return static_cast<int>(b < kMaxLossBlocks ? b : kMaxLossBlocks);
+}
+
+}  // namespace
+}  // namespace ff
+
+extern "C" {
+
+int ff_group_advantage(int n_groups, int G, const float* rewards, float eps_A, float* adv, cudaStream_t stream) {
+    using namespace ff;
+    if (n_groups <= 0 || G <= 0) return set_error(FF_ERR_INVALID_ARG, "advantage: n_groups=%d G=%d", n_groups, G);
+    if (G > 4096) return set_error(FF_ERR_UNSUPPORTED, "advantage: G=%d > 4096", G);
+    if (!rewards || !adv) return set_error(FF_ERR_INVALID_ARG, "advantage: null pointer");
+    if (!(eps_A >= 0.0f)) return set_error(FF_ERR_INVALID_ARG, "advantage: eps_A must be >= 0");
+    const int warps_per_block = kThreads / 32;
+    const int grid = (n_groups + warps_per_block - 1) / warps_per_block;
+    ProfScope prof(stream, "group_advantage", 0.0, 8.0 * n_groups * G);
+    group_advantage_kernel<<<grid, kThreads, 0, stream>>>(n_groups, G, rewards, eps_A, adv);
+    return check_launch("group_advantage_kernel");
+}
+
+int ff_grpo_loss_workspace_size(int B, int T, size_t* bytes) {
+    if (!bytes) return ff::set_error(FF_ERR_INVALID_ARG, "bytes is null");
+    if (B <= 0 || T <= 0) return ff::set_error(FF_ERR_INVALID_ARG, "B=%d T=%d must be positive", B, T);
+    *bytes = static_cast<size_t>(ff::loss_blocks(static_cast<int64_t>(B) * T)) * sizeof(double);
+    return FF_OK;
+}
+
+int ff_grpo_loss(int B, int T, const float* lp_new, const float* lp_old, const float* adv, float clip_lo,
+                 float clip_hi, float* loss, float* grad_lp_new, void* ws, size_t ws_bytes, cudaStream_t stream) {
+    using namespace ff;
+    if (B <= 0 || T <= 0) return set_error(FF_ERR_INVALID_ARG, "loss: B=%d T=%d must be positive", B, T);
+    if (!lp_new || !lp_old || !adv || !loss) return set_error(FF_ERR_INVALID_ARG, "loss: null pointer");
+    if (!(clip_lo >= 0.0f && clip_lo < 1.0f && clip_hi >= 0.0f))
+        return set_error(FF_ERR_INVALID_ARG, "loss: clip range must satisfy 0 <= lo < 1, hi >= 0");
+    const int64_t n = static_cast<int64_t>(B) * T;
+    const int nb = loss_blocks(n);
+    const size_t need = static_cast<size_t>(nb) * sizeof(double);
+    if (!ws || ws_bytes < need || (reinterpret_cast<uintptr_t>(ws) & 7))
+        return set_error(FF_ERR_WORKSPACE, "loss: workspace %zu B < %zu B needed (or misaligned)", ws_bytes, need);
+    double* partial = static_cast<double*>(ws);
+    {
+    ProfScope prof(stream, "grpo_loss", 0.0, static_cast<double>(n) * (grad_lp_new ? 12.0 : 8.0) + 4.0 * B);
+    grpo_loss_partial_kernel<<<nb, kThreads, 0, stream>>>(n, T, lp_new, lp_old, adv, clip_lo, clip_hi,
+                                                          static_cast<float>(1.0 / static_cast<double>(n)),
+                                                          grad_lp_new, partial);
+    }
+    int rc = check_launch("grpo_loss_partial_kernel");
+    if (rc) return rc;
+    ProfScope prof(stream, "grpo_loss_finalize", 0.0, nb * 8.0 + 4.0);
+    grpo_loss_finalize_kernel<<<1, kThreads, 0, stream>>>(nb, partial, 1.0 / static_cast<double>(n), loss);
+    return check_launch("grpo_loss_finalize_kernel");
+}
+
+}  // extern "C"

@@ -1,0 +1,207 @@
+// sde.cu -- fused Flow-SDE step and Gaussian transition log-probability
+// (paper Eq. 1 and Table 1).
+//
+// Per sample b (Delta = t - t_next > 0, a = sigma^2 / (2 t)):
+//   mean = x - Delta (v + a (x + (1 - t) v)) = cx x + cv v,
+//          cx = 1 - Delta a,  cv = -Delta (1 + a (1 - t))
+//   std  = sigma sqrt(Delta)
+//   SAMPLE: x_next = mean + std eps;  EVAL: x_next given
+//   logp = -sum (x_next - mean)^2 / (2 std^2) - D ln std - D/2 ln 2 pi
+// The per-sample coefficients are formed in fp64 once per thread; the
+// elementwise work is fp32 FMAs over 128-bit streaming loads.  Pass 1 writes
+// one fp64 partial sum of squared residuals per 4096-element chunk; pass 2
+// (one block per sample) adds the partials in a fixed order, so the result
+// does not depend on scheduling.
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace ff {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kVecPerThread = 4;                              // float4 per thread per chunk
+constexpr int kChunk = kThreads * kVecPerThread * 4;          // 4096 elements
+
+struct StepCoef {
+    float cx, cv, std;
+};
+
+__device__ __forceinline__ StepCoef step_coef(const float* t, const float* t_next, const float* sigma, int b) {
+    const double tt = t[b];
+    const double tn = t_next[b];
+    const double sg = sigma[b];
+    const double delta = tt - tn;
+    const double a = sg * sg / (2.0 * tt);
+    StepCoef c;
+    c.cx = static_cast<float>(1.0 - delta * a);
+    c.cv = static_cast<float>(-delta * (1.0 + a * (1.0 - tt)));
+    c.std = static_cast<float>(sg * sqrt(delta));
+    return c;
+}
+
+__device__ __forceinline__ double block_sum(double v, double* red) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    const int w = threadIdx.x >> 5;
+    if ((threadIdx.x & 31) == 0) red[w] = v;
+    __syncthreads();
+    double s = 0.0;
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < (int)(blockDim.x >> 5); ++i) s += red[i];
+    }
+    return s;   // valid in thread 0
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(kThreads) sde_step_partial_kernel(int64_t D, int nchunk, const float* x,
+                                                                    const float* v, const float* eps, float* x_next,
+                                                                    const float* t, const float* t_next,
+                                                                    const float* sigma, double* partial) {
+    __shared__ double red[kThreads / 32];
+    const int b = blockIdx.y;
+    const int chunk = blockIdx.x;
+    const StepCoef c = step_coef(t, t_next, sigma, b);
+    const int64_t row = static_cast<int64_t>(b) * D;
+    const int64_t base = static_cast<int64_t>(chunk) * kChunk;
+    const float4* x4 = reinterpret_cast<const float4*>(x + row);
+    const float4* v4 = reinterpret_cast<const float4*>(v + row);
+    const float4* e4 = reinterpret_cast<const float4*>(eps + (MODE == FF_SDE_SAMPLE ? row : 0));
+    float4* n4 = reinterpret_cast<float4*>(x_next + row);
+    const int64_t nvec = D >> 2;
+
+    float4 xv[kVecPerThread], vv[kVecPerThread], ev[kVecPerThread];
+#pragma unroll
+    for (int j = 0; j < kVecPerThread; ++j) {
+        const int64_t i = (base >> 2) + threadIdx.x + j * kThreads;
+        if (i < nvec) {
+            xv[j] = __ldcs(x4 + i);
+            vv[j] = __ldcs(v4 + i);
+            ev[j] = MODE == FF_SDE_SAMPLE ? __ldcs(e4 + i) : __ldcs(reinterpret_cast<const float4*>(n4) + i);
+        }
+    }
+    float ss = 0.f;
+#pragma unroll
+    for (int j = 0; j < kVecPerThread; ++j) {
+        const int64_t i = (base >> 2) + threadIdx.x + j * kThreads;
+        if (i < nvec) {
+            float m[4] = {fmaf(c.cx, xv[j].x, c.cv * vv[j].x), fmaf(c.cx, xv[j].y, c.cv * vv[j].y),
+                          fmaf(c.cx, xv[j].z, c.cv * vv[j].z), fmaf(c.cx, xv[j].w, c.cv * vv[j].w)};
+            float o[4];
+            if (MODE == FF_SDE_SAMPLE) {
+                o[0] = fmaf(c.std, ev[j].x, m[0]);
+                o[1] = fmaf(c.std, ev[j].y, m[1]);
+                o[2] = fmaf(c.std, ev[j].z, m[2]);
+                o[3] = fmaf(c.std, ev[j].w, m[3]);
+                __stcs(n4 + i, make_float4(o[0], o[1], o[2], o[3]));
+            } else {
+                o[0] = ev[j].x; o[1] = ev[j].y; o[2] = ev[j].z; o[3] = ev[j].w;
+            }
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const float r = o[k] - m[k];
+                ss = fmaf(r, r, ss);
+            }
+        }
+    }
+    const double s = block_sum(static_cast<double>(ss), red);
+    if (threadIdx.x == 0) partial[static_cast<int64_t>(b) * nchunk + chunk] = s;
+}
+
+__global__ void __launch_bounds__(kThreads) sde_logprob_finalize_kernel(int64_t D, int nchunk, const double* partial,
+                                                                        const float* t, const float* t_next,
+                                                                        const float* sigma, int reduce, float* logp,
+                                                                        int ld) {
+    __shared__ double red[kThreads / 32];
+    const int b = blockIdx.x;
+    double s = 0.0;
+    for (int i = threadIdx.x; i < nchunk; i += kThreads) s += partial[static_cast<int64_t>(b) * nchunk + i];
+    s = block_sum(s, red);
+    if (threadIdx.x == 0) {
+        const double delta = static_cast<double>(t[b]) - static_cast<double>(t_next[b]);
+        const double sd = static_cast<double>(sigma[b]) * sqrt(delta);
+        double lp = 0.0;
+        if (sd > 0.0) {
+            const double dd = static_cast<double>(D);
+            lp = -0.5 * s / (sd * sd) - dd * log(sd) - 0.5 * dd * log(2.0 * 3.14159265358979323846);
+            if (reduce == FF_LP_MEAN) lp /= dd;
+        }
+        logp[static_cast<int64_t>(b) * ld] = static_cast<float>(lp);
+    }
+}
+
+int nchunks(int64_t D) { return static_cast<int>((D + kChunk - 1) / kChunk); }
+
+}  // namespace
+}  // namespace ff
+
+extern "C" {
+
+int ff_sde_workspace_size(int B, int64_t D, size_t* bytes) {
+    if (!bytes) return ff::set_error(FF_ERR_INVALID_ARG, "bytes is null");
+    if (B <= 0 || D <= 0) return ff::set_error(FF_ERR_INVALID_ARG, "B and D must be positive");
+    *bytes = static_cast<size_t>(B) * static_cast<size_t>(ff::nchunks(D)) * sizeof(double);
+    return FF_OK;
+}
+
+int ff_sde_step_logprob(int B, int64_t D, const float* x_t, const float* v, const float* eps, float* x_next,
+                        const float* t, const float* t_next, const float* sigma, int mode, int reduce, float* logp,
+                        int ld, void* ws, size_t ws_bytes, cudaStream_t stream) {
+    using namespace ff;
+    if (B <= 0 || D <= 0) return set_error(FF_ERR_INVALID_ARG, "sde: B=%d D=%lld must be positive", B, (long long)D);
+    if (D % 4) return set_error(FF_ERR_UNSUPPORTED, "sde: D=%lld not a multiple of 4", (long long)D);
+    if (mode != FF_SDE_SAMPLE && mode != FF_SDE_EVAL) return set_error(FF_ERR_INVALID_ARG, "sde: bad mode %d", mode);
+    if (reduce != FF_LP_SUM && reduce != FF_LP_MEAN) return set_error(FF_ERR_INVALID_ARG, "sde: bad reduce %d", reduce);
+    if (!x_t || !v || !x_next || !t || !t_next || !sigma || !logp || (mode == FF_SDE_SAMPLE && !eps))
+        return set_error(FF_ERR_INVALID_ARG, "sde: null pointer");
+    if (!aligned16(x_t) || !aligned16(v) || !aligned16(x_next) || (mode == FF_SDE_SAMPLE && !aligned16(eps)))
+        return set_error(FF_ERR_INVALID_ARG, "sde: arrays must be 16-byte aligned");
+    if (ld < 1) return set_error(FF_ERR_INVALID_ARG, "sde: ld=%d < 1", ld);
+    if (B > 65535) return set_error(FF_ERR_UNSUPPORTED, "sde: B=%d > 65535", B);
+    const int nc = nchunks(D);
+    const size_t need = static_cast<size_t>(B) * nc * sizeof(double);
+    if (!ws || ws_bytes < need || (reinterpret_cast<uintptr_t>(ws) & 7))
+        return set_error(FF_ERR_WORKSPACE, "sde: workspace %zu B < %zu B needed (or misaligned)", ws_bytes, need);
+    double* partial = static_cast<double*>(ws);
+    const dim3 grid(nc, B);
+    {
+    ProfScope prof(stream, "sde_step", 0.0, static_cast<double>(B) * D * (mode == FF_SDE_SAMPLE ? 16.0 : 12.0));
+    if (mode == FF_SDE_SAMPLE)
+        sde_step_partial_kernel<FF_SDE_SAMPLE><<<grid, kThreads, 0, stream>>>(D, nc, x_t, v, eps, x_next, t, t_next,
+                                                                              sigma, partial);
+    else
+        sde_step_partial_kernel<FF_SDE_EVAL><<<grid, kThreads, 0, stream>>>(D, nc, x_t, v, eps, x_next, t, t_next,
+                                                                            sigma, partial);
+    }
+    int rc = check_launch("sde_step_partial_kernel");
+    if (rc) return rc;
+    ProfScope prof(stream, "sde_finalize", 0.0, static_cast<double>(B) * nc * 8.0 + B * 16.0);
+    sde_logprob_finalize_kernel<<<B, kThreads, 0, stream>>>(D, nc, partial, t, t_next, sigma, reduce, logp, ld);
+    return check_launch("sde_logprob_finalize_kernel");
+}
+
+}  // extern "C"
+
+extern "C" int ff_sde_schedule(int kind, int n_steps, double shift, double eta, double t_clamp, double* t_out,
+                               double* sigma_out) {
+    using namespace ff;
+    if (n_steps <= 0 || !t_out || !sigma_out) return set_error(FF_ERR_INVALID_ARG, "schedule: bad arguments");
+    if (!(shift > 0.0)) return set_error(FF_ERR_INVALID_ARG, "schedule: shift must be > 0");
+    if (kind != FF_SCHED_FLOW_SDE && kind != FF_SCHED_DANCE_SDE && kind != FF_SCHED_ODE)
+        return set_error(FF_ERR_INVALID_ARG, "schedule: bad kind %d", kind);
+    if (kind == FF_SCHED_FLOW_SDE && !(t_clamp > 0.0 && t_clamp < 1.0))
+        return set_error(FF_ERR_INVALID_ARG, "schedule: t_clamp must lie in (0, 1)");
+    for (int k = 0; k <= n_steps; ++k) {
+        const double t = 1.0 - static_cast<double>(k) / n_steps;
+        t_out[k] = shift == 1.0 ? t : shift * t / (1.0 + (shift - 1.0) * t);
+    }
+    for (int k = 0; k < n_steps; ++k) {
+        const double t = t_out[k] < t_clamp ? t_out[k] : t_clamp;
+        if (kind == FF_SCHED_FLOW_SDE)
+            sigma_out[k] = eta * sqrt(t / (1.0 - t));
+        else if (kind == FF_SCHED_DANCE_SDE)
+            sigma_out[k] = eta;
+        else
+            sigma_out[k] = 0.0;
+    }
+    return FF_OK;
+}

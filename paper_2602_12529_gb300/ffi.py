@@ -1,0 +1,287 @@
+"""ctypes binding of libff.so (include/ff.h, include/ff_debug.h).
+
+Argument marshalling only: torch tensors supply device memory and the CUDA
+stream; every computation runs in the library's kernels.  The functions keep
+the C names.  If the library is not built, or a GPU call is made without a
+CUDA device, they raise -- there is no fallback path.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+
+from .build import LIB
+
+FF_OK = 0
+FF_SDE_SAMPLE, FF_SDE_EVAL = 0, 1
+FF_LP_SUM, FF_LP_MEAN = 0, 1
+FF_SCHED_FLOW_SDE, FF_SCHED_DANCE_SDE, FF_SCHED_ODE = 0, 1, 2
+FF_ARCH_MMDIT = 0
+FF_ACT_NONE, FF_ACT_GELU, FF_ACT_SILU = 0, 1, 2
+
+
+class FFError(RuntimeError):
+    def __init__(self, func: str, code: int, msg: str):
+        super().__init__(f"{func} failed with status {code}: {msg}")
+        self.code = code
+
+
+class DitConfig(C.Structure):
+    _fields_ = [("arch", C.c_int), ("hidden", C.c_int), ("heads", C.c_int), ("head_dim", C.c_int),
+                ("mlp", C.c_int), ("n_double", C.c_int), ("n_single", C.c_int), ("patch_dim", C.c_int),
+                ("txt_dim", C.c_int), ("n_txt", C.c_int), ("grid_f", C.c_int), ("grid_h", C.c_int),
+                ("grid_w", C.c_int), ("rope_axes", C.c_int * 3), ("rope_theta", C.c_float),
+                ("time_freq_dim", C.c_int)]
+
+
+class TensorDesc(C.Structure):
+    _fields_ = [("name", C.c_char * 64), ("offset", C.c_int64), ("ndim", C.c_int), ("shape", C.c_int64 * 2)]
+
+
+_P = C.c_void_p
+_I = C.c_int
+_I64 = C.c_int64
+_F = C.c_float
+_D = C.c_double
+_SZ = C.c_size_t
+
+_SIGS = {
+    "ff_last_error": ([], C.c_char_p),
+    "ff_version": ([], _I),
+    "ff_check_device_status": ([_P, C.POINTER(_I)], _I),
+    "ff_sde_schedule": ([_I, _I, _D, _D, _D, C.POINTER(_D), C.POINTER(_D)], _I),
+    "ff_sde_workspace_size": ([_I, _I64, C.POINTER(_SZ)], _I),
+    "ff_sde_step_logprob": ([_I, _I64, _P, _P, _P, _P, _P, _P, _P, _I, _I, _P, _I, _P, _SZ, _P], _I),
+    "ff_group_advantage": ([_I, _I, _P, _F, _P, _P], _I),
+    "ff_grpo_loss_workspace_size": ([_I, _I, C.POINTER(_SZ)], _I),
+    "ff_grpo_loss": ([_I, _I, _P, _P, _P, _F, _F, _P, _P, _P, _SZ, _P], _I),
+    "ff_dit_weight_layout": ([C.POINTER(DitConfig), C.POINTER(TensorDesc), _I, C.POINTER(_I), C.POINTER(_I64)], _I),
+    "ff_dit_create": ([C.POINTER(DitConfig), _P, C.POINTER(_P)], _I),
+    "ff_dit_destroy": ([_P], _I),
+    "ff_dit_workspace_size": ([_P, _I, C.POINTER(_SZ)], _I),
+    "ff_dit_velocity": ([_P, _I, _P, _P, _P, _P, _P, _SZ, _P], _I),
+    "ff_debug_gemm": ([_I, _I, _I, _P, _I64, _P, _I64, _P, _I, _I, _P, _I64, _P], _I),
+    "ff_debug_gemm_gated": ([_I, _I, _I, _P, _I64, _P, _I64, _P, _P, _I64, _P, _I64, _I, _P], _I),
+    "ff_debug_attention": ([_I, _I, _I, _I, _P, _I64, _P, _I64, _I, _P, _I64, _P, _I64, _P], _I),
+    "ff_debug_ln_modulate": ([_I, _I, _P, _P, _I64, _I, _I, _I, _P, _P], _I),
+    "ff_debug_qk_norm_rope": ([_I, _I, _I, _I, _P, _I64, _P, _P, _I, _I, _I, C.POINTER(_I), _F, _P], _I),
+}
+
+_lib = None
+
+
+def lib() -> C.CDLL:
+    """The loaded libff.so (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB):
+            raise RuntimeError(f"libff.so not found at {LIB}; build it with paper_2602_12529_gb300.build.build()")
+        L = C.CDLL(LIB)
+        for name, (args, res) in _SIGS.items():
+            f = getattr(L, name)
+            f.argtypes = args
+            f.restype = res
+        _lib = L
+    return _lib
+
+
+def _call(name: str, *args) -> None:
+    rc = getattr(lib(), name)(*args)
+    if rc != FF_OK:
+        raise FFError(name, rc, lib().ff_last_error().decode())
+
+
+# ----------------------------------------------------------------- helpers
+
+def _ptr(t) -> int | None:
+    """Device address of a CUDA tensor (None for None)."""
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("expected a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError("expected a contiguous tensor")
+    return t.data_ptr()
+
+
+def _stream(stream) -> int:
+    import torch
+    s = torch.cuda.current_stream() if stream is None else stream
+    return s.cuda_stream
+
+
+def _check(t, dtype, name):
+    if t.dtype != dtype:
+        raise TypeError(f"{name}: expected {dtype}, got {t.dtype}")
+
+
+# ------------------------------------------------------------ host queries
+
+def ff_version() -> int:
+    return lib().ff_version()
+
+
+def ff_sde_schedule(kind: int, n_steps: int, shift: float = 1.0, eta: float = 0.7, t_clamp: float = 0.96):
+    """Host-only: (t[0..S], sigma[0..S-1]) as Python lists of float."""
+    t = (_D * (n_steps + 1))()
+    s = (_D * n_steps)()
+    _call("ff_sde_schedule", kind, n_steps, shift, eta, t_clamp, t, s)
+    return list(t), list(s)
+
+
+def ff_sde_workspace_size(B: int, D: int) -> int:
+    n = _SZ()
+    _call("ff_sde_workspace_size", B, D, C.byref(n))
+    return n.value
+
+
+def ff_grpo_loss_workspace_size(B: int, T: int) -> int:
+    n = _SZ()
+    _call("ff_grpo_loss_workspace_size", B, T, C.byref(n))
+    return n.value
+
+
+def make_config(cfg: dict) -> DitConfig:
+    c = DitConfig()
+    c.arch = FF_ARCH_MMDIT
+    for k in ("hidden", "heads", "head_dim", "mlp", "n_double", "n_single", "patch_dim", "txt_dim", "n_txt",
+              "time_freq_dim"):
+        setattr(c, k, int(cfg[k]))
+    c.grid_f, c.grid_h, c.grid_w = (int(v) for v in cfg["grid"])
+    for i, a in enumerate(cfg["rope_axes"]):
+        c.rope_axes[i] = int(a)
+    c.rope_theta = float(cfg["rope_theta"])
+    return c
+
+
+def ff_dit_weight_layout(cfg: dict):
+    """[(name, offset_elems, shape)], total_elems for a workload dict."""
+    c = make_config(cfg)
+    n = _I()
+    total = _I64()
+    _call("ff_dit_weight_layout", C.byref(c), None, 0, C.byref(n), C.byref(total))
+    descs = (TensorDesc * n.value)()
+    _call("ff_dit_weight_layout", C.byref(c), descs, n.value, C.byref(n), C.byref(total))
+    out = []
+    for d in descs:
+        shape = (d.shape[0], d.shape[1]) if d.ndim == 2 else (d.shape[0],)
+        out.append((d.name.decode(), int(d.offset), shape))
+    return out, int(total.value)
+
+
+# --------------------------------------------------------------- GPU calls
+
+def ff_sde_step_logprob(x_t, v, eps, x_next, t, t_next, sigma, logp, mode=FF_SDE_SAMPLE, reduce=FF_LP_SUM,
+                        ld=1, ws=None, stream=None):
+    import torch
+    B = x_t.shape[0]
+    D = x_t.numel() // B
+    for n_, a in (("x_t", x_t), ("v", v), ("x_next", x_next), ("t", t), ("t_next", t_next), ("sigma", sigma),
+                  ("logp", logp)):
+        _check(a, torch.float32, n_)
+    if ws is None:
+        ws = torch.empty(ff_sde_workspace_size(B, D), dtype=torch.uint8, device=x_t.device)
+    _call("ff_sde_step_logprob", B, D, _ptr(x_t), _ptr(v), _ptr(eps), _ptr(x_next), _ptr(t), _ptr(t_next),
+          _ptr(sigma), mode, reduce, _ptr(logp), ld, _ptr(ws), ws.numel(), _stream(stream))
+
+
+def ff_group_advantage(rewards, G: int, eps_A: float, adv, stream=None):
+    import torch
+    _check(rewards, torch.float32, "rewards")
+    _check(adv, torch.float32, "adv")
+    n = rewards.numel()
+    if n % G:
+        raise ValueError("rewards.numel() must be a multiple of G")
+    _call("ff_group_advantage", n // G, G, _ptr(rewards), eps_A, _ptr(adv), _stream(stream))
+
+
+def ff_grpo_loss(lp_new, lp_old, adv, clip_lo: float, clip_hi: float, loss, grad_lp_new=None, ws=None,
+                 stream=None):
+    import torch
+    B, T = lp_new.shape
+    for n_, a in (("lp_new", lp_new), ("lp_old", lp_old), ("adv", adv), ("loss", loss)):
+        _check(a, torch.float32, n_)
+    if ws is None:
+        ws = torch.empty(ff_grpo_loss_workspace_size(B, T), dtype=torch.uint8, device=lp_new.device)
+    _call("ff_grpo_loss", B, T, _ptr(lp_new), _ptr(lp_old), _ptr(adv), clip_lo, clip_hi, _ptr(loss),
+          _ptr(grad_lp_new), _ptr(ws), ws.numel(), _stream(stream))
+
+
+class Dit:
+    """Handle of a DiT over a caller-owned bf16 weight blob (torch tensor)."""
+
+    def __init__(self, cfg: dict, blob):
+        self.cfg = dict(cfg)
+        self._c = make_config(cfg)
+        self.blob = blob
+        h = _P()
+        _call("ff_dit_create", C.byref(self._c), _ptr(blob), C.byref(h))
+        self._h = h
+
+    def close(self):
+        if self._h is not None and self._h.value:
+            lib().ff_dit_destroy(self._h)
+        self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def workspace_size(self, B: int) -> int:
+        n = _SZ()
+        _call("ff_dit_workspace_size", self._h, B, C.byref(n))
+        return n.value
+
+    def ff_dit_velocity(self, x_t, txt, t, v_out, ws, stream=None):
+        import torch
+        _check(x_t, torch.float32, "x_t")
+        _check(txt, torch.bfloat16, "txt")
+        _check(t, torch.float32, "t")
+        _check(v_out, torch.float32, "v_out")
+        B = x_t.shape[0]
+        _call("ff_dit_velocity", self._h, B, _ptr(x_t), _ptr(txt), _ptr(t), _ptr(v_out), _ptr(ws), ws.numel(),
+              _stream(stream))
+
+
+def ff_check_device_status(stream=None) -> int:
+    st = _I()
+    rc = lib().ff_check_device_status(_stream(stream), C.byref(st))
+    if rc not in (FF_OK, 5):
+        raise FFError("ff_check_device_status", rc, lib().ff_last_error().decode())
+    return st.value
+
+
+# ------------------------------------------------------------- debug hooks
+
+def ff_debug_gemm(A, B, bias, out, act=FF_ACT_NONE, stream=None):
+    M, K = A.shape
+    N = B.shape[0]
+    import torch
+    _call("ff_debug_gemm", M, N, K, _ptr(A), A.stride(0), _ptr(B), B.stride(0), _ptr(bias), act,
+          1 if out.dtype == torch.float32 else 0, _ptr(out), out.stride(0), _stream(stream))
+
+
+def ff_debug_gemm_gated(A, B, bias, resid, gate, rows_per_sample, stream=None):
+    M, K = A.shape
+    N = B.shape[0]
+    _call("ff_debug_gemm_gated", M, N, K, _ptr(A), A.stride(0), _ptr(B), B.stride(0), _ptr(bias), _ptr(resid),
+          resid.stride(0), _ptr(gate), gate.stride(0), rows_per_sample, _stream(stream))
+
+
+def ff_debug_attention(B, heads, head_dim, qkv0, out0, n0, qkv1, out1, n1, stream=None):
+    _call("ff_debug_attention", B, heads, head_dim, n0, _ptr(qkv0), qkv0.shape[-1], _ptr(out0), out0.shape[-1],
+          n1, _ptr(qkv1), qkv1.shape[-1], _ptr(out1), out1.shape[-1], _stream(stream))
+
+
+def ff_debug_ln_modulate(x, mods, shift_off, scale_off, tokens_per_sample, out, stream=None):
+    rows, H = x.shape
+    _call("ff_debug_ln_modulate", rows, H, _ptr(x), _ptr(mods), mods.shape[-1], shift_off, scale_off,
+          tokens_per_sample, _ptr(out), _stream(stream))
+
+
+def ff_debug_qk_norm_rope(qkv, rows_txt, heads, head_dim, q_scale, k_scale, grid, rope_axes, theta, stream=None):
+    axes = (_I * 3)(*rope_axes)
+    _call("ff_debug_qk_norm_rope", qkv.shape[0], rows_txt, heads, head_dim, _ptr(qkv), qkv.shape[-1],
+          _ptr(q_scale), _ptr(k_scale), grid[0], grid[1], grid[2], axes, theta, _stream(stream))

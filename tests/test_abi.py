@@ -1,0 +1,124 @@
+"""CPU checks of the C ABI: the library builds and loads, exports every symbol
+the headers declare, and its host-only entry points (schedule, weight layout,
+workspace queries, argument validation) behave without a GPU."""
+import ctypes as C
+import os
+import re
+
+import numpy as np
+import pytest
+
+import synth
+from oracle import dit as odit
+from oracle import sde as osde
+from paper_2602_12529_gb300 import build, ffi
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def L():
+    build.build()
+    return ffi.lib()
+
+
+def _declared():
+    names = set()
+    for h in os.listdir(os.path.join(ROOT, "include")):
+        src = open(os.path.join(ROOT, "include", h)).read()
+        names |= set(re.findall(r"^\s*(?:const\s+char\s*\*|int)\s+(ff_\w+)\s*\(", src, re.M))
+    return names
+
+
+def test_exports_every_declared_symbol(L):
+    declared = _declared()
+    assert len(declared) >= 19
+    for name in declared:
+        assert hasattr(L, name), name
+    assert set(ffi._SIGS) >= declared
+
+
+def test_version_and_error_string(L):
+    assert ffi.ff_version() >= 100
+    assert isinstance(L.ff_last_error(), bytes)
+
+
+@pytest.mark.parametrize("steps,shift", [(4, 1.0), (10, 3.0), (1, 3.0)])
+def test_schedule_matches_oracle(L, steps, shift):
+    t, s = ffi.ff_sde_schedule(ffi.FF_SCHED_FLOW_SDE, steps, shift, 0.7, 0.96)
+    np.testing.assert_allclose(t, osde.time_grid(steps, shift), rtol=0, atol=1e-15)
+    np.testing.assert_allclose(s, osde.sigma_flow_sde(np.array(t[:-1]), 0.7, 0.96), rtol=1e-15)
+    _, s2 = ffi.ff_sde_schedule(ffi.FF_SCHED_DANCE_SDE, steps, shift, 0.3, 0.96)
+    assert s2 == [0.3] * steps
+    _, s3 = ffi.ff_sde_schedule(ffi.FF_SCHED_ODE, steps, shift, 0.3, 0.96)
+    assert s3 == [0.0] * steps
+
+
+def test_schedule_rejects_bad_arguments(L):
+    with pytest.raises(ffi.FFError):
+        ffi.ff_sde_schedule(7, 4)
+    with pytest.raises(ffi.FFError):
+        ffi.ff_sde_schedule(ffi.FF_SCHED_FLOW_SDE, 0)
+    with pytest.raises(ffi.FFError):
+        ffi.ff_sde_schedule(ffi.FF_SCHED_FLOW_SDE, 4, 1.0, 0.7, 1.0)
+
+
+@pytest.mark.parametrize("name", list(synth.CONFIGS))
+def test_weight_layout_matches_oracle_parameters(L, name):
+    cfg = synth.config(name)
+    if cfg["arch"] != "mmdit":
+        pytest.skip("layout covers the MMDiT family")
+    specs, total = ffi.ff_dit_weight_layout(cfg)
+    want = odit.param_specs(cfg)
+    assert [(n, tuple(s)) for n, _, s in specs] == [(n, tuple(s)) for n, s in want]
+    offs = [o for _, o, _ in specs]
+    assert all(o % 64 == 0 for o in offs)
+    assert offs == sorted(offs)
+    last_n, last_o, last_s = specs[-1]
+    assert total >= last_o + int(np.prod(last_s))
+
+
+def test_workspace_queries(L):
+    n1 = ffi.ff_sde_workspace_size(4, 262144)
+    assert n1 == 4 * 64 * 8
+    assert ffi.ff_grpo_loss_workspace_size(32, 10) == 8
+    assert ffi.ff_grpo_loss_workspace_size(1 << 20, 64) == 1024 * 8
+    with pytest.raises(ffi.FFError):
+        ffi.ff_sde_workspace_size(0, 16)
+
+
+def test_host_validation_without_gpu(L):
+    # every one of these is rejected before any CUDA call is made
+    rc = L.ff_sde_step_logprob(0, 16, None, None, None, None, None, None, None, 0, 0, None, 1, None, 0, None)
+    assert rc == 1
+    rc = L.ff_sde_step_logprob(2, 18, 16, 16, 16, 16, 16, 16, 16, 0, 0, 16, 1, 16, 1 << 20, None)
+    assert rc == 2   # D % 4 != 0
+    rc = L.ff_sde_step_logprob(2, 16, 16, 16, 16, 16, 16, 16, 16, 5, 0, 16, 1, 16, 1 << 20, None)
+    assert rc == 1   # bad mode
+    rc = L.ff_sde_step_logprob(2, 16, 16, 16, 16, 16, 16, 16, 16, 0, 0, 16, 1, 16, 8, None)
+    assert rc == 3   # workspace too small
+    assert L.ff_group_advantage(0, 4, 16, 1e-4, 16, None) == 1
+    assert L.ff_group_advantage(1, 5000, 16, 1e-4, 16, None) == 2
+    assert L.ff_grpo_loss(4, 1, None, 16, 16, 0.2, 0.2, 16, None, 16, 64, None) == 1
+    assert L.ff_grpo_loss(4, 1, 16, 16, 16, 1.5, 0.2, 16, None, 16, 64, None) == 1
+    assert L.ff_grpo_loss(4, 1, 16, 16, 16, 0.2, 0.2, 16, None, 16, 0, None) == 3
+    assert b"workspace" in L.ff_last_error()
+
+
+def test_dit_handle_and_config_validation(L):
+    cfg = synth.config("tiny_mmdit")
+    c = ffi.make_config(cfg)
+    h = C.c_void_p()
+    assert L.ff_dit_create(C.byref(c), C.c_void_p(256), C.byref(h)) == 0
+    n = C.c_size_t()
+    assert L.ff_dit_workspace_size(h, 4, C.byref(n)) == 0
+    R = 4 * (32 + 64)
+    assert n.value >= R * 256 * (4 + 2 + 6 + 2) + R * (256 + 1024) * 2
+    # a velocity call with a too-small workspace is rejected on the host
+    assert L.ff_dit_velocity(h, 4, 16, 16, 16, 16, 256, 1024, None) == 3
+    assert L.ff_dit_velocity(h, 4, 16, 16, 16, 16, 255, n.value, None) == 1
+    assert L.ff_dit_destroy(h) == 0
+    bad = ffi.make_config(dict(cfg, rope_axes=(8, 28, 30)))
+    assert L.ff_dit_create(C.byref(bad), C.c_void_p(256), C.byref(h)) == 1
+    bad = ffi.make_config(dict(cfg, head_dim=32, heads=8))
+    assert L.ff_dit_create(C.byref(bad), C.c_void_p(256), C.byref(h)) == 2
