@@ -39,7 +39,8 @@ struct Cfg {
     static constexpr int kStageBytes = kABytes + kBBytes;
     static constexpr int kTmemCols = 2 * BN;
     static constexpr int kBarrierBytes = 256;
-    static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + kBarrierBytes;
+    static constexpr int kStageFloats = 32 * 33;   // per epilogue warp: 32x32 fp32 transpose tile
+    static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + kBarrierBytes + 4 * kStageFloats * 4;
 };
 
 __device__ __forceinline__ void tile_coords(int tile, int num_m, int num_n, int& mb, int& nb) {
@@ -63,6 +64,53 @@ __device__ __forceinline__ void bias_add8(float* v, const __nv_bfloat16* b) {
     }
 }
 
+// Gated residual x[row, n..n+31] += gate[b(row), n..] * v for the 32 rows of
+// one epilogue warp.  The accumulator arrives one row per lane; it is
+// transposed through a padded 32x33 shared tile, and the global
+// read-modify-write runs on float4 row segments: lane = (row offset rs in
+// 0..3, column quad cq in 0..7), rows rs + 4j, so one warp instruction
+// covers 4 full 128-byte row segments.  The residual and gate of the next
+// chunk are loaded while the current one is finished (software pipeline).
+struct GatedRegs {
+    float4 x[8];
+    float4 g[8];
+};
+
+__device__ __forceinline__ void gated_load(const GemmEpilogue& e, int M, int row0, int n, int lane, GatedRegs& R) {
+    const int col = n + 4 * (lane & 7);
+    const int rs = lane >> 3;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        const int row = row0 + rs + 4 * j;
+        if (row < M) {
+            const int b = row / e.rows_per_sample;
+            R.g[j] = *reinterpret_cast<const float4*>(e.gate + static_cast<int64_t>(b) * e.ld_gate + col);
+            R.x[j] = *reinterpret_cast<const float4*>(e.resid + static_cast<int64_t>(row) * e.ld_resid + col);
+        }
+    }
+}
+
+__device__ __forceinline__ void gated_store(const GemmEpilogue& e, int M, int row0, int n, int lane,
+                                            const GatedRegs& R, const float* st) {
+    const int cq = lane & 7;
+    const int rs = lane >> 3;
+    const int col = n + 4 * cq;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        const int r = rs + 4 * j;
+        const int row = row0 + r;
+        if (row < M) {
+            const float* a = st + r * 33 + 4 * cq;
+            float4 o = R.x[j];
+            o.x += R.g[j].x * a[0];
+            o.y += R.g[j].y * a[1];
+            o.z += R.g[j].z * a[2];
+            o.w += R.g[j].w * a[3];
+            *reinterpret_cast<float4*>(e.resid + static_cast<int64_t>(row) * e.ld_resid + col) = o;
+        }
+    }
+}
+
 // Fused tail for one 32-column chunk of one output row held by this thread.
 __device__ __forceinline__ void epilogue_chunk(const GemmEpilogue& e, int M, int row, int n, float (&v)[32]) {
     if (e.bias) {
@@ -79,22 +127,6 @@ __device__ __forceinline__ void epilogue_chunk(const GemmEpilogue& e, int M, int
         }
     }
     if (row >= M) return;
-    if (e.epi == EPI_GATED_RESIDUAL) {
-        const int b = row / e.rows_per_sample;
-        const float4* g = reinterpret_cast<const float4*>(e.gate + static_cast<int64_t>(b) * e.ld_gate + n);
-        float4* x = reinterpret_cast<float4*>(e.resid + static_cast<int64_t>(row) * e.ld_resid + n);
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            const float4 gv = g[j];
-            float4 xv = x[j];
-            xv.x += gv.x * v[4 * j];
-            xv.y += gv.y * v[4 * j + 1];
-            xv.z += gv.z * v[4 * j + 2];
-            xv.w += gv.w * v[4 * j + 3];
-            x[j] = xv;
-        }
-        return;
-    }
     void* base;
     int64_t ld;
     int col;
@@ -132,6 +164,7 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_const
     uint64_t* drain_bar = tempty_bar + 2;           // [1]
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_bar + 1);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    float* stage_f = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(full_bar) + C::kBarrierBytes);
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -246,17 +279,45 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_const
             tc_fence_after();
             const int row = mb * BM + q * 32 + lane;
             const uint32_t t_acc = tmem_base + static_cast<uint32_t>(acc * BN) + (static_cast<uint32_t>(q * 32) << 16);
-#pragma unroll 1
-            for (int c = 0; c < BN; c += 32) {
-                uint32_t r[32];
-                tmem_ld_x32(t_acc + c, r);
-                tmem_ld_wait();
-                const int n = nb * BN + c;
-                if (n >= N) continue;
-                float v[32];
+            if (epi.epi == EPI_GATED_RESIDUAL) {
+                float* st = stage_f + (warp - 2) * C::kStageFloats;
+                const int row0 = mb * BM + q * 32;
+                GatedRegs R[2];
+                gated_load(epi, M, row0, nb * BN, lane, R[0]);
 #pragma unroll
-                for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
-                epilogue_chunk(epi, M, row, n, v);
+                for (int c = 0; c < BN / 32; ++c) {
+                    const int n = nb * BN + c * 32;
+                    if (c + 1 < BN / 32 && n + 32 < N) gated_load(epi, M, row0, n + 32, lane, R[(c + 1) & 1]);
+                    uint32_t r[32];
+                    tmem_ld_x32(t_acc + c * 32, r);
+                    tmem_ld_wait();
+                    if (n >= N) continue;
+                    float v[32];
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+                    if (epi.bias) {
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) bias_add8(v + 8 * j, epi.bias + n + 8 * j);
+                    }
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) st[lane * 33 + i] = v[i];
+                    __syncwarp();
+                    gated_store(epi, M, row0, n, lane, R[c & 1], st);
+                    __syncwarp();
+                }
+            } else {
+#pragma unroll 1
+                for (int c = 0; c < BN; c += 32) {
+                    uint32_t r[32];
+                    tmem_ld_x32(t_acc + c, r);
+                    tmem_ld_wait();
+                    const int n = nb * BN + c;
+                    if (n >= N) continue;
+                    float v[32];
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+                    epilogue_chunk(epi, M, row, n, v);
+                }
             }
             tc_fence_before();
             __syncwarp();

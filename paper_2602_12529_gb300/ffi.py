@@ -49,6 +49,11 @@ _SIGS = {
     "ff_last_error": ([], C.c_char_p),
     "ff_version": ([], _I),
     "ff_check_device_status": ([_P, C.POINTER(_I)], _I),
+    "ff_prof_enable": ([_I], _I),
+    "ff_prof_disable": ([], _I),
+    "ff_prof_reset": ([], _I),
+    "ff_prof_count": ([C.POINTER(_I)], _I),
+    "ff_prof_read": ([_I, C.c_char_p, _I, C.POINTER(_F), C.POINTER(_D), C.POINTER(_D)], _I),
     "ff_sde_schedule": ([_I, _I, _D, _D, _D, C.POINTER(_D), C.POINTER(_D)], _I),
     "ff_sde_workspace_size": ([_I, _I64, C.POINTER(_SZ)], _I),
     "ff_sde_step_logprob": ([_I, _I64, _P, _P, _P, _P, _P, _P, _P, _I, _I, _P, _I, _P, _SZ, _P], _I),
@@ -251,6 +256,33 @@ def ff_check_device_status(stream=None) -> int:
     if rc not in (FF_OK, 5):
         raise FFError("ff_check_device_status", rc, lib().ff_last_error().decode())
     return st.value
+
+
+# ------------------------------------------------------------ launch timing
+
+def ff_prof_enable(max_records: int) -> None:
+    _call("ff_prof_enable", max_records)
+
+
+def ff_prof_disable() -> None:
+    _call("ff_prof_disable")
+
+
+def ff_prof_reset() -> None:
+    _call("ff_prof_reset")
+
+
+def ff_prof_records():
+    """[(kernel name, ms, algorithmic flops, algorithmic bytes)] of the timed launches."""
+    n = _I()
+    _call("ff_prof_count", C.byref(n))
+    out = []
+    buf = C.create_string_buffer(64)
+    for i in range(n.value):
+        ms, fl, by = _F(), _D(), _D()
+        _call("ff_prof_read", i, buf, 64, C.byref(ms), C.byref(fl), C.byref(by))
+        out.append((buf.value.decode(), float(ms.value), float(fl.value), float(by.value)))
+    return out
 
 
 # ------------------------------------------------------------- debug hooks
