@@ -117,6 +117,35 @@ int ff_sde_step_logprob(int B, int64_t D, const float* x_t, const float* v,
                         cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
+ * ff_sde_step_logprob_noalloc -- the SDE step + log-prob above, for callers
+ * that cannot allocate device memory: for example a plug-in running inside a
+ * host application that owns every device allocation itself (its own pool,
+ * its own accounting), where an extra cudaMalloc would fragment that pool,
+ * bypass its limits, or stall the device at a moment the host does not
+ * control.  The paper has no counterpart; this is a deployment convenience.
+ *
+ * Same arguments and results as ff_sde_step_logprob, minus the workspace.
+ * The caller still passes every input and output.  The scratch is a fixed
+ * 512 KiB array of fp64 partial sums built into the library, held on every
+ * GPU that loads the library until the process exits.  Limit:
+ * B * ceil(D / 4096) <= 65536 (for example B = 32 samples of up to 8.3 M
+ * elements); larger calls are rejected with FF_ERR_UNSUPPORTED and a message
+ * naming the limit.  Nothing here calls cudaMalloc, cudaFree or any other
+ * allocating routine.
+ *
+ * The first call on each device looks up the array's device address
+ * (cudaGetSymbolAddress, with that device current) and caches it; make that
+ * first call before any stream capture begins.  Every call on a device uses
+ * the same array, and each call rewrites every slot it reads, so no clearing
+ * is needed; but calls whose kernels overlap on the GPU (different streams,
+ * no ordering between them) race on the array and must not be issued.
+ * ------------------------------------------------------------------------ */
+int ff_sde_step_logprob_noalloc(int B, int64_t D, const float* x_t, const float* v,
+                                const float* eps, float* x_next, const float* t,
+                                const float* t_next, const float* sigma, int mode, int reduce,
+                                float* logp, int ld, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
  * Group-relative advantage (paper Sec. 2.3, advantage computation of the
  * GRPO trainer).  Samples form contiguous groups of G (one prompt each):
  *   A[g*G + i] = (r[g*G + i] - mean_g) / (std_g + eps_A),  std_g population.

@@ -205,3 +205,82 @@ extern "C" int ff_sde_schedule(int kind, int n_steps, double shift, double eta, 
     }
     return FF_OK;
 }
+
+// ---------------------------------------------------------------------------
+// ff_sde_step_logprob_noalloc: the same step for callers that cannot hand the
+// library any device memory of their own (see include/ff.h).  The per-chunk
+// partial sums live in a fixed array in the library's device image instead
+// of a caller workspace.
+// ---------------------------------------------------------------------------
+#include <mutex>
+
+namespace ff {
+namespace {
+
+constexpr int kNoAllocMaxPartials = 65536;   // 512 KiB of fp64 partial sums on every device
+
+// Shared by every call on a device; each call overwrites every slot it later
+// reads, so nothing has to start at zero.
+static __device__ __align__(256) double g_sde_scratch[kNoAllocMaxPartials];
+
+constexpr int kNoAllocMaxDevices = 64;
+double* g_sde_scratch_addr[kNoAllocMaxDevices] = {};
+std::mutex g_sde_scratch_mu;
+
+// Device address of g_sde_scratch on the current device, looked up once per
+// device with that device current (host code cannot use the symbol itself).
+int sde_scratch_address(double** out) {
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kNoAllocMaxDevices)
+        return set_error(FF_ERR_CUDA, "sde (no-alloc): no usable current device");
+    std::lock_guard<std::mutex> lk(g_sde_scratch_mu);
+    if (!g_sde_scratch_addr[dev]) {
+        void* p = nullptr;
+        const cudaError_t e = cudaGetSymbolAddress(&p, g_sde_scratch);
+        if (e != cudaSuccess || !p)
+            return set_error(FF_ERR_CUDA, "sde (no-alloc): cudaGetSymbolAddress failed: %s", cudaGetErrorString(e));
+        g_sde_scratch_addr[dev] = static_cast<double*>(p);
+    }
+    *out = g_sde_scratch_addr[dev];
+    return FF_OK;
+}
+
+}  // namespace
+}  // namespace ff
+
+extern "C" int ff_sde_step_logprob_noalloc(int B, int64_t D, const float* x_t, const float* v, const float* eps,
+                                           float* x_next, const float* t, const float* t_next, const float* sigma,
+                                           int mode, int reduce, float* logp, int ld, cudaStream_t stream) {
+    using namespace ff;
+    if (B <= 0 || D <= 0) return set_error(FF_ERR_INVALID_ARG, "sde (no-alloc): B=%d D=%lld must be positive", B, (long long)D);
+    if (D % 4) return set_error(FF_ERR_UNSUPPORTED, "sde (no-alloc): D=%lld not a multiple of 4", (long long)D);
+    if (mode != FF_SDE_SAMPLE && mode != FF_SDE_EVAL) return set_error(FF_ERR_INVALID_ARG, "sde (no-alloc): bad mode %d", mode);
+    if (reduce != FF_LP_SUM && reduce != FF_LP_MEAN)
+        return set_error(FF_ERR_INVALID_ARG, "sde (no-alloc): bad reduce %d", reduce);
+    if (!x_t || !v || !x_next || !t || !t_next || !sigma || !logp || (mode == FF_SDE_SAMPLE && !eps))
+        return set_error(FF_ERR_INVALID_ARG, "sde (no-alloc): null pointer");
+    if (!aligned16(x_t) || !aligned16(v) || !aligned16(x_next) || (mode == FF_SDE_SAMPLE && !aligned16(eps)))
+        return set_error(FF_ERR_INVALID_ARG, "sde (no-alloc): arrays must be 16-byte aligned");
+    if (ld < 1) return set_error(FF_ERR_INVALID_ARG, "sde (no-alloc): ld=%d < 1", ld);
+    if (B > 65535) return set_error(FF_ERR_UNSUPPORTED, "sde (no-alloc): B=%d > 65535", B);
+    const int nc = nchunks(D);
+    if (static_cast<int64_t>(B) * nc > kNoAllocMaxPartials)
+        return set_error(FF_ERR_UNSUPPORTED,
+                         "sde (no-alloc): B * ceil(D / %d) = %lld partial sums exceed the built-in scratch of %d; "
+                         "use ff_sde_step_logprob with a workspace",
+                         kChunk, (long long)B * nc, kNoAllocMaxPartials);
+    double* partial = nullptr;
+    const int rc0 = sde_scratch_address(&partial);
+    if (rc0) return rc0;
+    const dim3 grid(nc, B);
+    if (mode == FF_SDE_SAMPLE)
+        sde_step_partial_kernel<FF_SDE_SAMPLE><<<grid, kThreads, 0, stream>>>(D, nc, x_t, v, eps, x_next, t, t_next,
+                                                                              sigma, partial);
+    else
+        sde_step_partial_kernel<FF_SDE_EVAL><<<grid, kThreads, 0, stream>>>(D, nc, x_t, v, eps, x_next, t, t_next,
+                                                                            sigma, partial);
+    int rc = check_launch("sde_step_partial_kernel (no-alloc)");
+    if (rc) return rc;
+    sde_logprob_finalize_kernel<<<B, kThreads, 0, stream>>>(D, nc, partial, t, t_next, sigma, reduce, logp, ld);
+    return check_launch("sde_logprob_finalize_kernel (no-alloc)");
+}

@@ -57,6 +57,7 @@ _SIGS = {
     "ff_sde_schedule": ([_I, _I, _D, _D, _D, C.POINTER(_D), C.POINTER(_D)], _I),
     "ff_sde_workspace_size": ([_I, _I64, C.POINTER(_SZ)], _I),
     "ff_sde_step_logprob": ([_I, _I64, _P, _P, _P, _P, _P, _P, _P, _I, _I, _P, _I, _P, _SZ, _P], _I),
+    "ff_sde_step_logprob_noalloc": ([_I, _I64, _P, _P, _P, _P, _P, _P, _P, _I, _I, _P, _I, _P], _I),
     "ff_group_advantage": ([_I, _I, _P, _F, _P, _P], _I),
     "ff_grpo_loss_workspace_size": ([_I, _I, C.POINTER(_SZ)], _I),
     "ff_grpo_loss": ([_I, _I, _P, _P, _P, _F, _F, _P, _P, _P, _SZ, _P], _I),
@@ -188,6 +189,20 @@ def ff_sde_step_logprob(x_t, v, eps, x_next, t, t_next, sigma, logp, mode=FF_SDE
         ws = torch.empty(ff_sde_workspace_size(B, D), dtype=torch.uint8, device=x_t.device)
     _call("ff_sde_step_logprob", B, D, _ptr(x_t), _ptr(v), _ptr(eps), _ptr(x_next), _ptr(t), _ptr(t_next),
           _ptr(sigma), mode, reduce, _ptr(logp), ld, _ptr(ws), ws.numel(), _stream(stream))
+
+
+def ff_sde_step_logprob_noalloc(x_t, v, eps, x_next, t, t_next, sigma, logp, mode=FF_SDE_SAMPLE,
+                                reduce=FF_LP_SUM, ld=1, stream=None):
+    """ff_sde_step_logprob without a workspace: scratch is the library's own
+    fixed device array (for callers that cannot allocate device memory)."""
+    import torch
+    B = x_t.shape[0]
+    D = x_t.numel() // B
+    for n_, a in (("x_t", x_t), ("v", v), ("x_next", x_next), ("t", t), ("t_next", t_next), ("sigma", sigma),
+                  ("logp", logp)):
+        _check(a, torch.float32, n_)
+    _call("ff_sde_step_logprob_noalloc", B, D, _ptr(x_t), _ptr(v), _ptr(eps), _ptr(x_next), _ptr(t), _ptr(t_next),
+          _ptr(sigma), mode, reduce, _ptr(logp), ld, _stream(stream))
 
 
 def ff_group_advantage(rewards, G: int, eps_A: float, adv, stream=None):
