@@ -69,6 +69,9 @@ def load_peaks():
         return 6800.0, 1900.0, 1700.0, "fallback"
 
 
+KERNEL_SOURCES = {"gemm_bf16": ["gemm.cu"], "attention": ["attention.cu"], "sde_step": ["sde.cu"]}
+
+
 def profile_traffic(kernel, workload):
     """DRAM bytes per launch recorded from an ncu capture, if the kernel's
     source has not changed since (source hash recorded with the number)."""
@@ -79,17 +82,18 @@ def profile_traffic(kernel, workload):
         return None
     m = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", txt)
     h = re.search(r"source_sha256:\s*([0-9a-f]+)", txt)
-    if not m or not h:
+    if not m or not h or kernel not in KERNEL_SOURCES:
         return None
-    if h.group(1) != kernel_source_hash():
+    if h.group(1) != kernel_source_hash(kernel):
         return None
     return float(m.group(1))
 
 
-def kernel_source_hash():
+def kernel_source_hash(kernel):
+    """Hash of the files that define a kernel (its .cu plus the shared headers)."""
     d = os.path.join(ROOT, "paper_2602_12529_gb300", "csrc")
     sha = hashlib.sha256()
-    for f in sorted(os.listdir(d)):
+    for f in KERNEL_SOURCES[kernel] + ["ptx.cuh", "internal.h"]:
         with open(os.path.join(d, f), "rb") as fh:
             sha.update(f.encode() + fh.read())
     return sha.hexdigest()[:16]
