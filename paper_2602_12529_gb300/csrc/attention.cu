@@ -6,23 +6,27 @@
 // h*d, k at H + h*d, v at 2H + h*d) by TMA; the segments may live in
 // different buffers.
 //
-// One CTA = 128 query rows of one segment of one (sample, head); two CTAs
-// share an SM.  Warp roles (6 warps):
-//   warp 0      TMA producer: the Q tile once, then 64-token K/V tiles into a
-//               2-deep ring (K/V tiles never straddle the segment boundary;
-//               rows past the segment end are masked).
-//   warp 1      TMEM allocator; lane 0 issues the MMAs:
-//                 S_j = Q K_j^T   (M 128, N 64, K d)  into TMEM buffer j % 2
-//                 O  += P_j V_j   (M 128, N d,  K 64) into the TMEM O tile,
-//               issuing S_{j+1} before O += P_j V_j so the tensor core works
-//               while the softmax warps process S_j.
-//   warps 2..5  softmax: thread = query row = TMEM lane.  Reads S_j,
-//               updates the running max / sum in base 2 (log2 e folded into
-//               the scale), writes P_j = exp2(S - m) as bf16 into a
-//               128-byte-swizzled shared tile (the A operand of P V), and
-//               rescales the O rows in TMEM only when the running max grows
-//               by more than 8 (2^8 headroom in fp32/bf16), which makes
-//               corrections rare.  Finally O / l goes out as bf16.
+// One CTA = two 128-row query tiles (256 query rows) of one segment of one
+// (sample, head), sharing every K/V tile.  Warp roles (10 warps):
+//   warp 0      TMA producer: both Q tiles once, then 128-token K/V tiles
+//               into a 2-deep ring (K/V tiles never straddle the segment
+//               boundary; rows past the segment end are masked).
+//   warp 1      TMEM allocator (all 512 columns); lane 0 issues the MMAs.
+//               Per query tile t the order is S_t,j = Q_t K_j^T (M 128, N 128,
+//               A and B from shared memory) -> softmax -> O_t += P_t,j V_j
+//               (M 128, N d, A = P from TMEM, B = V from shared memory) ->
+//               S_t,j+1; the two tiles alternate, so the tensor core works on
+//               one tile while the other tile's softmax runs.  Keeping P in
+//               TMEM halves the shared-memory operand traffic of P V, which
+//               is what bounds narrow MMAs.
+//   warps 2..9  two softmax warpgroups, one per query tile: thread = query
+//               row = TMEM lane.  Reads its S row, keeps the running max /
+//               sum in base 2 (log2 e folded into the scale), writes
+//               P = exp2(S - m) as bf16 pairs over the S columns, and
+//               rescales its O row in TMEM only when the running max grows by
+//               more than 8 (2^8 headroom), which makes corrections rare.
+//               Part of the exponentials run on the FMA pipe (exp2_poly2).
+//               Finally O / l goes out as bf16.
 // Every wait is bounded; on a timeout the kernel records the status word,
 // drains its tensor-core work, frees TMEM and returns.
 #include "internal.h"
@@ -31,26 +35,29 @@
 namespace ff {
 namespace {
 
-constexpr int kBM = 128;         // query rows per CTA
-constexpr int kBN = 64;          // tokens per K/V tile
+constexpr int kBM = 128;         // query rows per query tile (two tiles per CTA)
+constexpr int kBN = 128;         // tokens per K/V tile
 constexpr int kStages = 2;
-constexpr int kThreads = 192;
+constexpr int kThreads = 320;    // producer, MMA, 2 x 4 softmax warps
 constexpr float kRescaleThreshold = 8.0f;   // log2 units
+constexpr int kSwExp = 40;       // of every 128 scores, this many use the software exp2
 
 template <int HD>
 struct ACfg {
-    static constexpr int kQBytes = kBM * HD * 2;
+    static constexpr int kQBytes = kBM * HD * 2;        // one query tile
     static constexpr int kKBytes = kBN * HD * 2;
     static constexpr int kStageBytes = 2 * kKBytes;     // K + V
-    static constexpr int kPBytes = kBM * kBN * 2;
-    static constexpr int kSmemBytes = kQBytes + kStages * kStageBytes + kPBytes + 256;
-    static constexpr int kTmemCols = 256;               // S0 | S1 | O
-    static constexpr int kColS0 = 0, kColS1 = kBN, kColO = 2 * kBN;
+    static constexpr int kBarBytes = 256;
+    static constexpr int kSmemBytes = 2 * kQBytes + kStages * kStageBytes + kBarBytes;
+    static constexpr int kTmemCols = 512;
+    // TMEM columns of query tile t: S (fp32, kBN columns) at t*256, with P
+    // (bf16 pairs, kBN/2 columns) written over its first half; O at t*256+128
+    static constexpr int kColO = kBN;
 };
 
 struct AttnParams {
     int n[2];            // tokens per sample in each segment
-    int qtiles0;         // query tiles of segment 0 (then segment 1's follow)
+    int qpairs0;         // 256-row query blocks of segment 0 (segment 1's follow)
     int H;
     float scale_log2;
     __nv_bfloat16* out[2];
@@ -63,7 +70,37 @@ __device__ __forceinline__ float ex2(float x) {
     return y;
 }
 
-__device__ __forceinline__ void tmem_st_x32(uint32_t taddr, const uint32_t (&r)[32]) {
+__device__ __forceinline__ float max3(float a, float b, float c) {
+    float y;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(y) : "f"(a), "f"(b), "f"(c));
+    return y;
+}
+
+// Software 2^x for a pair of arguments, on the FMA pipe (the MUFU unit alone
+// cannot keep up with the tensor core at d = 128).  Range reduction: n =
+// round(x) via the 1.5 * 2^23 shifter, f = x - n in [-1/2, 1/2]; 2^f from a
+// degree-3 minimax polynomial (Remez exchange on the relative error,
+// coefficients from csrc/fit_exp2.py; max relative error 7.5e-5, below the
+// bf16 rounding that P receives); 2^n is added into the exponent field.
+// Arguments are clamped at -126: p(f) >= 2^-1/2 has biased exponent >= 126,
+// so adding n >= -126 never wraps the exponent field (at n = -127 a p(0)
+// just below 1 would wrap to a NaN); 2^-126 is zero for every use here.
+__device__ __forceinline__ float2 exp2_poly2(float2 x) {
+    constexpr float kShift = 12582912.0f;   // 1.5 * 2^23
+    x.x = fmaxf(x.x, -126.0f);
+    x.y = fmaxf(x.y, -126.0f);
+    const float2 t = __fadd2_rn(x, make_float2(kShift, kShift));
+    const float2 n = __fadd2_rn(t, make_float2(-kShift, -kShift));
+    const float2 f = __ffma2_rn(n, make_float2(-1.0f, -1.0f), x);
+    float2 q = __ffma2_rn(make_float2(5.517166853e-02f, 5.517166853e-02f), f,
+                          make_float2(2.426111251e-01f, 2.426111251e-01f));
+    q = __ffma2_rn(q, f, make_float2(6.932609677e-01f, 6.932609677e-01f));
+    q = __ffma2_rn(q, f, make_float2(9.999280572e-01f, 9.999280572e-01f));
+    return make_float2(__uint_as_float(__float_as_uint(q.x) + (__float_as_uint(t.x) << 23)),
+                       __uint_as_float(__float_as_uint(q.y) + (__float_as_uint(t.y) << 23)));
+}
+
+__device__ __forceinline__ void tmem_st_x32(uint32_t taddr, const uint32_t* r) {
     asm volatile(
         "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
         "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, "
@@ -75,6 +112,17 @@ __device__ __forceinline__ void tmem_st_x32(uint32_t taddr, const uint32_t (&r)[
         : "memory");
 }
 __device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+
+// D[tmem] (+)= A[tmem] * B[smem]: the P V product with P held in TMEM.
+__device__ __forceinline__ void tc_mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                               uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}\n"
+        ::"r"(d_tmem), "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
 
 // B operand stored MN-major with 128-byte swizzle (V: rows = K = tokens,
 // 64 contiguous d per 128-byte row): leading byte offset = distance between
@@ -89,69 +137,72 @@ __device__ __forceinline__ uint64_t smem_desc_mn_sw128(uint32_t saddr, uint32_t 
     return d;
 }
 
+// Barriers.  Per query tile the chain S -> softmax -> P -> O += P V -> next S
+// is strictly ordered, so no waiter can lag two phases behind a parity wait.
+struct Bars {
+    uint64_t q_full;
+    uint64_t kv_full[kStages];
+    uint64_t kv_empty[kStages];
+    uint64_t s_full[2];       // [query tile] MMA -> softmax: S_t,j is in TMEM (and O += P V_{j-1} done)
+    uint64_t p_full[2];       //              softmax -> MMA: P_t,j is in TMEM, O rescaled
+    uint64_t o_last[2];       //              MMA -> softmax: the last O += P V has landed
+    uint64_t drain;
+    uint32_t tmem_slot;
+    int abort_flag;
+};
+
 template <int HD>
-__global__ void __launch_bounds__(kThreads, 2)
+__global__ void __launch_bounds__(kThreads, 1)
 attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_constant__ CUtensorMap tm_q1,
                     const __grid_constant__ CUtensorMap tm_kv0, const __grid_constant__ CUtensorMap tm_kv1,
                     const AttnParams p, int* status) {
     using C = ACfg<HD>;
+    static_assert(sizeof(Bars) <= C::kBarBytes, "barrier block too small");
     extern __shared__ __align__(1024) uint8_t smem[];
-    uint8_t* sQ = smem;
-    uint8_t* sKV = smem + C::kQBytes;
-    uint8_t* sP = sKV + kStages * C::kStageBytes;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(sP + C::kPBytes);
-    uint64_t* q_full = bars;                 // [1]
-    uint64_t* kv_full = bars + 1;            // [kStages]
-    uint64_t* kv_empty = kv_full + kStages;  // [kStages]
-    uint64_t* s_full = kv_empty + kStages;   // [2]
-    uint64_t* s_free = s_full + 2;           // [2]
-    uint64_t* p_full = s_free + 2;           // [1]
-    uint64_t* o_done = p_full + 1;           // [1]
-    uint64_t* drain = o_done + 1;            // [1]
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
-    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    uint8_t* sQ = smem;                                   // [2][kQBytes]
+    uint8_t* sKV = smem + 2 * C::kQBytes;                 // [kStages][K | V]
+    Bars& bar = *reinterpret_cast<Bars*>(sKV + kStages * C::kStageBytes);
+    volatile int* abort_flag = &bar.abort_flag;
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     const int b = blockIdx.z;
     const int h = blockIdx.y;
-    const int seg = blockIdx.x < p.qtiles0 ? 0 : 1;
-    const int q0 = (blockIdx.x - (seg ? p.qtiles0 : 0)) * kBM;   // first query row within the segment
+    const int seg = blockIdx.x < p.qpairs0 ? 0 : 1;
+    const int q0 = (blockIdx.x - (seg ? p.qpairs0 : 0)) * (2 * kBM);   // first query row within the segment
     const int nt0 = (p.n[0] + kBN - 1) / kBN;
     const int ntiles = nt0 + (p.n[1] + kBN - 1) / kBN;
 
     if (threadIdx.x == 0) {
+        *abort_flag = 0;
         if (smem_u32(smem) & 1023u) {   // the swizzled tiles need 1024-byte alignment
             report_status(status, kStatusBadArgument);
             *abort_flag = 1;
-        } else {
-            *abort_flag = 0;
         }
-        mbar_init(q_full, 1);
+        mbar_init(&bar.q_full, 1);
         for (int s = 0; s < kStages; ++s) {
-            mbar_init(&kv_full[s], 1);
-            mbar_init(&kv_empty[s], 1);
+            mbar_init(&bar.kv_full[s], 1);
+            mbar_init(&bar.kv_empty[s], 1);
         }
-        for (int s = 0; s < 2; ++s) {
-            mbar_init(&s_full[s], 1);
-            mbar_init(&s_free[s], 4);
+        for (int t = 0; t < 2; ++t) {
+            mbar_init(&bar.s_full[t], 1);
+            mbar_init(&bar.p_full[t], 4);
+            mbar_init(&bar.o_last[t], 1);
         }
-        mbar_init(p_full, 4);
-        mbar_init(o_done, 1);
-        mbar_init(drain, 1);
+        mbar_init(&bar.drain, 1);
         fence_mbar_init();
         prefetch_tmap(seg ? &tm_q1 : &tm_q0);
         prefetch_tmap(&tm_kv0);
         prefetch_tmap(&tm_kv1);
     }
     if (warp == 1) {
-        tmem_alloc(tmem_slot, C::kTmemCols);
+        tmem_alloc(&bar.tmem_slot, C::kTmemCols);
         tmem_relinquish();
     }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    const uint32_t tmem = *tmem_slot;
+    const uint32_t tmem = bar.tmem_slot;
     const bool aborted_at_start = *abort_flag;
 
     auto fail = [&]() {
@@ -164,55 +215,40 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
     } else if (warp == 0 && lane == 0) {
         // ------------------------------------------------------------ producer
         const CUtensorMap* tq = seg ? &tm_q1 : &tm_q0;
-        mbar_arrive_expect_tx(q_full, C::kQBytes);
-        for (int c = 0; c < HD / 64; ++c)
-            tma_load_2d(sQ + c * (kBM * 128), tq, q_full, h * HD + c * 64, b * p.n[seg] + q0);
+        mbar_arrive_expect_tx(&bar.q_full, 2 * C::kQBytes);
+        for (int t = 0; t < 2; ++t)
+            for (int c = 0; c < HD / 64; ++c)
+                tma_load_2d(sQ + t * C::kQBytes + c * (kBM * 128), tq, &bar.q_full, h * HD + c * 64,
+                            b * p.n[seg] + q0 + t * kBM);
         for (int j = 0; j < ntiles && !*abort_flag; ++j) {
             const int s = j % kStages;
-            const uint32_t ph = (j / kStages) & 1;
-            if (!mbar_wait(&kv_empty[s], ph ^ 1)) { fail(); break; }
+            if (!mbar_wait(&bar.kv_empty[s], ((j / kStages) & 1) ^ 1)) { fail(); break; }
             const int ks = j < nt0 ? 0 : 1;
             const int row = b * p.n[ks] + (j - (ks ? nt0 : 0)) * kBN;
             const CUtensorMap* tkv = ks ? &tm_kv1 : &tm_kv0;
             uint8_t* dk = sKV + s * C::kStageBytes;
             uint8_t* dv = dk + C::kKBytes;
-            mbar_arrive_expect_tx(&kv_full[s], C::kStageBytes);
+            mbar_arrive_expect_tx(&bar.kv_full[s], C::kStageBytes);
             for (int c = 0; c < HD / 64; ++c) {
-                tma_load_2d(dk + c * (kBN * 128), tkv, &kv_full[s], p.H + h * HD + c * 64, row);
-                tma_load_2d(dv + c * (kBN * 128), tkv, &kv_full[s], 2 * p.H + h * HD + c * 64, row);
+                tma_load_2d(dk + c * (kBN * 128), tkv, &bar.kv_full[s], p.H + h * HD + c * 64, row);
+                tma_load_2d(dv + c * (kBN * 128), tkv, &bar.kv_full[s], 2 * p.H + h * HD + c * 64, row);
             }
         }
     } else if (warp == 1 && lane == 0) {
         // ------------------------------------------------------------ MMA issuer
+        // Order per query tile t: S_t,0 ; then for each j: O_t += P_t,j V_j ;
+        // S_t,j+1.  The two tiles interleave so one tile's MMAs run while the
+        // other tile's softmax works.  tcgen05.mma from one thread executes in
+        // issue order, so S_t,j+1 overwrites the columns of P_t,j only after
+        // O_t += P_t,j V_j has read them.
         constexpr uint32_t idesc_s = idesc_bf16_f32(kBM, kBN);
         constexpr uint32_t idesc_o = idesc_bf16_f32(kBM, HD) | (1u << 16);   // B (V) is MN-major
-        const uint32_t aQ = smem_u32(sQ);
-        const uint32_t aP = smem_u32(sP);
-        bool ok = mbar_wait(q_full, 0);
+        bool ok = mbar_wait(&bar.q_full, 0);
         if (!ok) fail();
-        auto issue_pv = [&](int j) -> bool {
-            // O += P_j V_j once the softmax has published P_j
-            if (!mbar_wait(p_full, j & 1)) return false;
-            tc_fence_after();
-            const int s = j % kStages;
-            const uint32_t aV = smem_u32(sKV + s * C::kStageBytes + C::kKBytes);
-#pragma unroll
-            for (int k = 0; k < kBN / 16; ++k) {
-                const uint64_t da = smem_desc_k_sw128(aP) + static_cast<uint64_t>(2 * k);
-                const uint64_t db = smem_desc_mn_sw128(aV + k * 2048, kBN * 128);
-                tc_mma_bf16(tmem + C::kColO, da, db, idesc_o, (j | k) != 0 ? 1u : 0u);
-            }
-            tc_commit(o_done);
-            tc_commit(&kv_empty[s]);
-            return true;
-        };
-        for (int j = 0; ok && j < ntiles && !*abort_flag; ++j) {
-            const int s = j % kStages;
-            if (!mbar_wait(&kv_full[s], (j / kStages) & 1)) { fail(); ok = false; break; }
-            if (!mbar_wait(&s_free[j & 1], ((j >> 1) & 1) ^ 1)) { fail(); ok = false; break; }
-            tc_fence_after();
-            const uint32_t aK = smem_u32(sKV + s * C::kStageBytes);
-            const uint32_t dS = tmem + ((j & 1) ? C::kColS1 : C::kColS0);
+        auto issue_s = [&](int t, int j) {
+            const uint32_t aQ = smem_u32(sQ + t * C::kQBytes);
+            const uint32_t aK = smem_u32(sKV + (j % kStages) * C::kStageBytes);
+            const uint32_t dS = tmem + t * 256;
 #pragma unroll
             for (int k = 0; k < HD / 16; ++k) {
                 const uint32_t off_q = (k / 4) * (kBM * 128) + (k % 4) * 32;
@@ -220,105 +256,141 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
                 tc_mma_bf16(dS, smem_desc_k_sw128(aQ + off_q), smem_desc_k_sw128(aK + off_k), idesc_s,
                             k != 0 ? 1u : 0u);
             }
-            tc_commit(&s_full[j & 1]);
-            if (j >= 1 && !issue_pv(j - 1)) { fail(); ok = false; break; }
+            tc_commit(&bar.s_full[t]);
+        };
+        auto issue_pv = [&](int t, int j) -> bool {
+            if (!mbar_wait(&bar.p_full[t], j & 1)) return false;
+            tc_fence_after();
+            const uint32_t aV = smem_u32(sKV + (j % kStages) * C::kStageBytes + C::kKBytes);
+            const uint32_t dO = tmem + t * 256 + C::kColO;
+            const uint32_t aP = tmem + t * 256;
+#pragma unroll
+            for (int k = 0; k < kBN / 16; ++k) {
+                const uint64_t db = smem_desc_mn_sw128(aV + k * 2048, kBN * 128);
+                tc_mma_bf16_ts(dO, aP + k * 8, db, idesc_o, (j | k) != 0 ? 1u : 0u);
+            }
+            return true;
+        };
+        if (ok && ntiles > 0) {
+            if (!mbar_wait(&bar.kv_full[0], 0)) { fail(); ok = false; }
+            else {
+                tc_fence_after();
+                issue_s(0, 0);
+                issue_s(1, 0);
+            }
         }
-        if (ok && !*abort_flag && ntiles > 0 && !issue_pv(ntiles - 1)) fail();
-        tc_commit(drain);
-        if (!mbar_wait(drain, 0)) report_status(status, kStatusWaitTimeout);
+        for (int j = 0; ok && j < ntiles && !*abort_flag; ++j) {
+            const bool more = j + 1 < ntiles;
+            for (int t = 0; t < 2; ++t) {
+                if (!issue_pv(t, j)) { fail(); ok = false; break; }
+                if (more) {
+                    if (t == 0 && !mbar_wait(&bar.kv_full[(j + 1) % kStages], ((j + 1) / kStages) & 1)) {
+                        fail(); ok = false; break;
+                    }
+                    tc_fence_after();
+                    issue_s(t, j + 1);
+                }
+            }
+            if (!ok) break;
+            tc_commit(&bar.kv_empty[j % kStages]);
+        }
+        if (ok) {
+            tc_commit(&bar.o_last[0]);
+            tc_commit(&bar.o_last[1]);
+        }
+        tc_commit(&bar.drain);
+        if (!mbar_wait(&bar.drain, 0)) report_status(status, kStatusWaitTimeout);
     } else if (warp >= 2) {
         // ------------------------------------------------------------ softmax
-        const int q = warp & 3;
+        const int t = (warp - 2) >> 2;                   // query tile of this warpgroup
+        const int q = warp & 3;                          // TMEM lane quarter of this warp
         const int r = q * 32 + lane;                     // query row within the tile = TMEM lane
-        const uint32_t lane_base = static_cast<uint32_t>(q * 32) << 16;
+        const uint32_t tS = tmem + (static_cast<uint32_t>(q * 32) << 16) + t * 256;
+        const uint32_t tO = tS + C::kColO;
         float m_used = -INFINITY;
         float l = 0.f;
         bool ok = true;
         for (int j = 0; j < ntiles; ++j) {
             if (*abort_flag) { ok = false; break; }
-            if (!mbar_wait(&s_full[j & 1], (j >> 1) & 1)) { fail(); ok = false; break; }
+            // S_t,j ready; O_t += P_t,j-1 V_j-1 has completed as well
+            if (!mbar_wait(&bar.s_full[t], j & 1)) { fail(); ok = false; break; }
             tc_fence_after();
             uint32_t sr[kBN];
-            {
-                uint32_t (&a)[32] = *reinterpret_cast<uint32_t(*)[32]>(&sr[0]);
-                uint32_t (&c)[32] = *reinterpret_cast<uint32_t(*)[32]>(&sr[32]);
-                const uint32_t ts = tmem + lane_base + ((j & 1) ? C::kColS1 : C::kColS0);
-                tmem_ld_x32(ts, a);
-                tmem_ld_x32(ts + 32, c);
-                tmem_ld_wait();
-            }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&s_free[j & 1]);
+#pragma unroll
+            for (int c = 0; c < kBN; c += 32) tmem_ld_x32(tS + c, *reinterpret_cast<uint32_t(*)[32]>(&sr[c]));
+            tmem_ld_wait();
 
             const int ks = j < nt0 ? 0 : 1;
             const int valid = p.n[ks] - (j - (ks ? nt0 : 0)) * kBN;   // columns < valid are real tokens
-            float mx = -INFINITY;
+            if (valid < kBN) {
 #pragma unroll
-            for (int i = 0; i < kBN; ++i) {
-                const float v = i < valid ? __uint_as_float(sr[i]) * p.scale_log2 : -INFINITY;
-                sr[i] = __float_as_uint(v);
-                mx = fmaxf(mx, v);
+                for (int i = 0; i < kBN; ++i)
+                    if (i >= valid) sr[i] = __float_as_uint(-INFINITY);
             }
+            float mc[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+            for (int i = 0; i < kBN; i += 8) {
+#pragma unroll
+                for (int k = 0; k < 4; ++k)
+                    mc[k] = max3(mc[k], __uint_as_float(sr[i + 2 * k]), __uint_as_float(sr[i + 2 * k + 1]));
+            }
+            const float mx = max3(mc[0], mc[1], fmaxf(mc[2], mc[3])) * p.scale_log2;
             const bool grow = mx > m_used + kRescaleThreshold;
             const float m_new = grow ? mx : m_used;
             const float alpha = ex2(m_used - m_new);   // 0 on the first tile, 1 without growth
-            uint32_t pk[kBN / 2];
-            float sum = 0.f;
+            const float2 c2 = make_float2(p.scale_log2, p.scale_log2);
+            const float2 nm2 = make_float2(-m_new, -m_new);
+            float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                             make_float2(0.f, 0.f)};
 #pragma unroll
             for (int i = 0; i < kBN; i += 2) {
-                const float e0 = ex2(__uint_as_float(sr[i]) - m_new);
-                const float e1 = ex2(__uint_as_float(sr[i + 1]) - m_new);
-                sum += e0 + e1;
-                pk[i / 2] = pack_bf16x2(e0, e1);
+                const float2 x = __ffma2_rn(make_float2(__uint_as_float(sr[i]), __uint_as_float(sr[i + 1])), c2, nm2);
+                float2 e;
+                if (i < kSwExp) {
+                    e = exp2_poly2(x);
+                } else {
+                    e.x = ex2(x.x);
+                    e.y = ex2(x.y);
+                }
+                acc[(i >> 1) & 3] = __fadd2_rn(acc[(i >> 1) & 3], e);
+                sr[i / 2] = pack_bf16x2(e.x, e.y);   // P packed over the front of the S registers
             }
-            l = l * alpha + sum;
+            const float2 a01 = __fadd2_rn(acc[0], acc[1]);
+            const float2 a23 = __fadd2_rn(acc[2], acc[3]);
+            l = l * alpha + ((a01.x + a01.y) + (a23.x + a23.y));
             m_used = m_new;
-
-            // P buffer and O are free once O += P_{j-1} V_{j-1} has completed
-            if (j >= 1) {
-                if (!mbar_wait(o_done, (j - 1) & 1)) { fail(); ok = false; break; }
-                tc_fence_after();
-                if (__any_sync(0xffffffffu, grow)) {
-                    // rescale this warp's O rows (alpha = 1 for rows whose max held)
+            // a grown max rescales this warp's O rows (O is stable: its last
+            // update completed before S_t,j was published)
+            if (j >= 1 && __any_sync(0xffffffffu, grow)) {
 #pragma unroll 1
-                    for (int c = 0; c < HD; c += 32) {
-                        uint32_t o[32];
-                        const uint32_t to = tmem + lane_base + C::kColO + c;
-                        tmem_ld_x32(to, o);
-                        tmem_ld_wait();
+                for (int c = 0; c < HD; c += 32) {
+                    uint32_t o[32];
+                    tmem_ld_x32(tO + c, o);
+                    tmem_ld_wait();
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
-                        tmem_st_x32(to, o);
-                    }
-                    tmem_st_wait();
+                    for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+                    tmem_st_x32(tO + c, o);
                 }
             }
-            // P row r: 64 bf16 = one 128-byte swizzle row, 8 chunks of 16 bytes
-            {
-                uint8_t* prow = sP + (r >> 3) * 1024 + (r & 7) * 128;
+            // P_t,j (bf16 pairs) over the first kBN/2 columns of S_t
 #pragma unroll
-                for (int c = 0; c < 8; ++c) {
-                    *reinterpret_cast<uint4*>(prow + ((c ^ (r & 7)) << 4)) =
-                        make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
-                }
-            }
-            fence_proxy_async_smem();
+            for (int c = 0; c < kBN / 2; c += 32) tmem_st_x32(tS + c, &sr[c]);
+            tmem_st_wait();
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(p_full);
+            if (lane == 0) mbar_arrive(&bar.p_full[t]);
         }
-        // ---- epilogue: O / l -> bf16
-        if (ok && ntiles > 0 && mbar_wait(o_done, (ntiles - 1) & 1)) {
+        // ---- epilogue: O / l -> bf16, after the last O += P V
+        if (ok && ntiles > 0 && mbar_wait(&bar.o_last[t], 0)) {
             tc_fence_after();
             const float inv = 1.f / l;
-            const int row = q0 + r;
+            const int row = q0 + t * kBM + r;
             const bool live = row < p.n[seg];
             __nv_bfloat16* dst = p.out[seg] + (static_cast<int64_t>(b) * p.n[seg] + row) * p.ldo[seg] + h * HD;
 #pragma unroll 1
             for (int c = 0; c < HD; c += 32) {
                 uint32_t o[32];
-                tmem_ld_x32(tmem + lane_base + C::kColO + c, o);
+                tmem_ld_x32(tO + c, o);
                 tmem_ld_wait();
                 if (live) {
 #pragma unroll
@@ -348,6 +420,12 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
     }
 }
 
+__global__ void exp2_poly_kernel(const float2* x, float2* y, int64_t n2) {
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n2;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x)
+        y[i] = exp2_poly2(x[i]);
+}
+
 template <int HD>
 int launch_attn(const AttnSegment& s0, const AttnSegment& s1, int B, int heads, int H, cudaStream_t stream) {
     using C = ACfg<HD>;
@@ -368,7 +446,7 @@ int launch_attn(const AttnSegment& s0, const AttnSegment& s1, int B, int heads, 
     AttnParams p;
     p.n[0] = s0.n;
     p.n[1] = s1.n;
-    p.qtiles0 = (s0.n + kBM - 1) / kBM;
+    p.qpairs0 = (s0.n + 2 * kBM - 1) / (2 * kBM);
     p.H = H;
     p.scale_log2 = static_cast<float>(1.4426950408889634 / sqrt(static_cast<double>(HD)));
     p.out[0] = s0.out;
@@ -376,7 +454,7 @@ int launch_attn(const AttnSegment& s0, const AttnSegment& s1, int B, int heads, 
     p.ldo[0] = s0.ldo;
     p.ldo[1] = s1.ldo;
     const int N = s0.n + s1.n;
-    const dim3 grid(p.qtiles0 + (s1.n + kBM - 1) / kBM, heads, B);
+    const dim3 grid(p.qpairs0 + (s1.n + 2 * kBM - 1) / (2 * kBM), heads, B);
     const double nn = static_cast<double>(N) * N;
     ProfScope prof(stream, "attention", 4.0 * B * heads * nn * HD, 8.0 * B * static_cast<double>(N) * H);
     attn_tcgen05_kernel<HD><<<grid, kThreads, C::kSmemBytes, stream>>>(tq[0], tq[1], tkv[0], tkv[1], p,
@@ -404,3 +482,15 @@ int attention(const AttnSegment& s0, const AttnSegment& s1, int B, int heads, in
 }
 
 }  // namespace ff
+
+extern "C" int ff_debug_exp2(const float* x, float* y, int64_t n, cudaStream_t stream) {
+    using namespace ff;
+    if (!x || !y || n <= 0 || n % 2 || !aligned16(x) || !aligned16(y))
+        return set_error(FF_ERR_INVALID_ARG, "exp2: bad arguments (n even, 16-byte aligned arrays)");
+    const int64_t n2 = n / 2;
+    int64_t grid = (n2 + 255) / 256;
+    if (grid > 4096) grid = 4096;
+    exp2_poly_kernel<<<static_cast<unsigned>(grid), 256, 0, stream>>>(reinterpret_cast<const float2*>(x),
+                                                                       reinterpret_cast<float2*>(y), n2);
+    return check_launch("exp2_poly_kernel");
+}

@@ -386,7 +386,11 @@ int gemm_bf16(const void* A, int64_t lda, const void* B, int64_t ldb, int M, int
         }
     }
     if (e.act != ACT_NONE && e.act_from % 32) return set_error(FF_ERR_INVALID_ARG, "gemm: act_from % 32 != 0");
-    if (N <= 64) return launch<64>(A, lda, B, ldb, M, N, K, e, stream);
+    // narrow tiles when wide ones would leave most SMs idle (e.g. the
+    // batch-row time-embedding GEMMs)
+    const int64_t mblocks = (M + BM - 1) / BM;
+    const bool few = mblocks * ((N + 255) / 256) < num_sms() / 2;
+    if (N <= 64 || few) return launch<64>(A, lda, B, ldb, M, N, K, e, stream);
     if (N <= 128) return launch<128>(A, lda, B, ldb, M, N, K, e, stream);
     return launch<256>(A, lda, B, ldb, M, N, K, e, stream);
 }
