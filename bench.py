@@ -48,6 +48,7 @@ def parse_args():
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default=WORKLOAD)
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-sweep", action="store_true", help="skip the HBM bandwidth sweep of the memory-bound kernels")
     return p.parse_args()
 
 
@@ -245,6 +246,76 @@ def run_reference(args):
 # the CUDA path
 # ---------------------------------------------------------------------------
 
+def hbm_sweep(ffi, dev, hbm_peak, l2_bytes=129 * 2 ** 20):
+    """Bandwidth of the memory-bound kernels at sizes well beyond L2, with
+    enough rotating buffer sets that every launch reads from HBM."""
+    import torch
+
+    def timeit(fns, reps=10):
+        for f in fns[:3]:
+            f()
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for i in range(reps):
+            fns[i % len(fns)]()
+        e1.record()
+        torch.cuda.synchronize(dev)
+        return e0.elapsed_time(e1) / reps / 1e3
+
+    def nsets(nbytes):
+        return max(1, -(-4 * l2_bytes // nbytes))
+
+    out = {}
+    rows = []
+    for n in (1 << 24, 1 << 26, 1 << 28):
+        B, D = 4, n // 4
+        per = 16 * n
+        sets = []
+        for _ in range(nsets(per)):
+            x = torch.randn(B, D, device=dev)
+            sets.append((x, torch.randn_like(x), torch.randn_like(x), torch.empty_like(x)))
+        t = torch.full((B,), 0.75, device=dev)
+        tn = torch.full((B,), 0.5, device=dev)
+        sg = torch.full((B,), 0.7, device=dev)
+        lp = torch.empty(B, device=dev)
+        ws = torch.empty(ffi.ff_sde_workspace_size(B, D), dtype=torch.uint8, device=dev)
+        fns = [lambda s_=s_: ffi.ff_sde_step_logprob(s_[0], s_[1], s_[2], s_[3], t, tn, sg, lp, ws=ws) for s_ in sets]
+        sec = timeit(fns)
+        rows.append({"elements": n, "bytes": per, "gbs": per / sec / 1e9, "frac": per / sec / 1e9 / hbm_peak,
+                     "sets": len(sets)})
+        del sets
+    out["sde_step"] = rows
+    rows = []
+    for n in (1 << 22, 1 << 24, 1 << 26):
+        Bq, T = n // 16, 16
+        per = 12 * n + 4 * Bq
+        sets = []
+        for _ in range(nsets(per)):
+            a = torch.randn(Bq, T, device=dev)
+            sets.append((a, a + 0.01 * torch.randn_like(a), torch.randn(Bq, device=dev), torch.empty_like(a)))
+        loss = torch.empty(1, device=dev)
+        ws = torch.empty(ffi.ff_grpo_loss_workspace_size(Bq, T), dtype=torch.uint8, device=dev)
+        fns = [lambda s_=s_: ffi.ff_grpo_loss(s_[0], s_[1], s_[2], 0.2, 0.2, loss, s_[3], ws=ws) for s_ in sets]
+        sec = timeit(fns)
+        rows.append({"elements": n, "bytes": per, "gbs": per / sec / 1e9, "frac": per / sec / 1e9 / hbm_peak,
+                     "sets": len(sets)})
+        del sets
+    out["grpo_loss"] = rows
+    rows = []
+    for n in (1 << 22, 1 << 24, 1 << 26):
+        per = 8 * n
+        sets = [(torch.rand(n, device=dev), torch.empty(n, device=dev)) for _ in range(nsets(per))]
+        fns = [lambda s_=s_: ffi.ff_group_advantage(s_[0], 16, 1e-4, s_[1]) for s_ in sets]
+        sec = timeit(fns)
+        rows.append({"elements": n, "group": 16, "bytes": per, "gbs": per / sec / 1e9,
+                     "frac": per / sec / 1e9 / hbm_peak, "sets": len(sets)})
+        del sets
+    out["group_advantage"] = rows
+    torch.cuda.empty_cache()
+    return out
+
+
 def run_ours(args):
     import numpy as np
     import torch
@@ -406,6 +477,7 @@ def run_ours(args):
     e2e_step()
     ms_e2e = timed(e2e_step, args.steps) / args.steps
     e2e_value = world * tokens_per_step / (ms_e2e / 1e3)
+    sweep = hbm_sweep(ffi, dev, hbm) if rank == 0 and not args.no_sweep else None
     clk = clocks.stop() if clocks else None
     status = ffi.ff_check_device_status()
 
@@ -430,6 +502,7 @@ def run_ours(args):
                 "cpu_baseline": cpu,
                 "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                         "ms_per_step": ms_e2e},
+                "hbm_sweep": sweep,
                 "gpu_launches": launches,
                 "clocks": clk,
                 "device_status": status}

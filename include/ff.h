@@ -128,9 +128,9 @@ int ff_sde_step_logprob(int B, int64_t D, const float* x_t, const float* v,
  * The caller still passes every input and output.  The scratch is a fixed
  * 512 KiB array of fp64 partial sums built into the library, held on every
  * GPU that loads the library until the process exits.  Limit:
- * B * ceil(D / 4096) <= 65536 (for example B = 32 samples of up to 8.3 M
- * elements); larger calls are rejected with FF_ERR_UNSUPPORTED and a message
- * naming the limit.  Nothing here calls cudaMalloc, cudaFree or any other
+ * B * min(ceil(D / 4096), 1024) <= 65536 partial sums, which holds for any
+ * D when B <= 64; larger calls are rejected with FF_ERR_UNSUPPORTED and a
+ * message naming the limit.  Nothing here calls cudaMalloc, cudaFree or any other
  * allocating routine.
  *
  * The first call on each device looks up the array's device address

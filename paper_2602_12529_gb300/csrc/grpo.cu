@@ -17,53 +17,98 @@ namespace ff {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kElemsPerBlock = kThreads * 4;
-constexpr int kMaxLossBlocks = 1024;
+constexpr int kElemsPerBlock = kThreads * 16;
+constexpr int kMaxLossBlocks = 1216;   // 8 blocks of 256 threads on each of 152 SMs
 
+// G in {4, 8, 16, 32, 64, 128}: each lane owns 4 consecutive samples (one
+// float4) and a group spans G / 4 lanes; the reductions shuffle within those
+// lanes.  fp32 sums over at most 128 values (the tests bound them against
+// fp64).
+__global__ void __launch_bounds__(kThreads) group_advantage_vec_kernel(int64_t n4, int G, const float4* r, float eps,
+                                                                       float4* adv) {
+    const int64_t i = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x;
+    const bool live = i < n4;
+    const float4 x = live ? r[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+    const int lanes = G >> 2;
+    float s = (x.x + x.y) + (x.z + x.w);
+    for (int o = 1; o < lanes; o <<= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    const float mean = s / G;
+    const float d0 = x.x - mean, d1 = x.y - mean, d2 = x.z - mean, d3 = x.w - mean;
+    float q = (d0 * d0 + d1 * d1) + (d2 * d2 + d3 * d3);
+    for (int o = 1; o < lanes; o <<= 1) q += __shfl_xor_sync(0xffffffffu, q, o);
+    const float inv = 1.0f / (sqrtf(q / G) + eps);
+    if (live) adv[i] = make_float4(d0 * inv, d1 * inv, d2 * inv, d3 * inv);
+}
+
+// Any G: one warp per group, the group re-read from L1 for the second pass.
 __global__ void __launch_bounds__(kThreads) group_advantage_kernel(int n_groups, int G, const float* r, float eps,
                                                                    float* adv) {
     const int warp = (blockIdx.x * kThreads + threadIdx.x) >> 5;
     const int lane = threadIdx.x & 31;
     if (warp >= n_groups) return;
     const float* rg = r + static_cast<int64_t>(warp) * G;
-    double s = 0.0;
+    float s = 0.f;
     for (int i = lane; i < G; i += 32) s += rg[i];
 #pragma unroll
     for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-    const double mean = s / G;
-    double q = 0.0;
+    const float mean = s / G;
+    float q = 0.f;
     for (int i = lane; i < G; i += 32) {
-        const double d = rg[i] - mean;
+        const float d = rg[i] - mean;
         q += d * d;
     }
 #pragma unroll
     for (int o = 16; o; o >>= 1) q += __shfl_xor_sync(0xffffffffu, q, o);
-    const double denom = sqrt(q / G) + static_cast<double>(eps);
+    const float denom = sqrtf(q / G) + eps;
     float* ag = adv + static_cast<int64_t>(warp) * G;
     // each lane rewrites only the elements it reads itself, after the
     // reductions above, so adv may alias r
-    for (int i = lane; i < G; i += 32) ag[i] = static_cast<float>((static_cast<double>(rg[i]) - mean) / denom);
+    for (int i = lane; i < G; i += 32) ag[i] = (rg[i] - mean) / denom;
 }
 
+// One fp32 partial per thread over float4 groups (sample index b = i / T in
+// 32-bit arithmetic), fp64 only for the block and cross-block sums.
 __global__ void __launch_bounds__(kThreads) grpo_loss_partial_kernel(int64_t n, int T, const float* lp_new,
                                                                      const float* lp_old, const float* adv,
                                                                      float lo, float hi, float inv_n,
                                                                      float* grad, double* partial) {
     __shared__ double red[kThreads / 32];
-    double s = 0.0;
-    for (int64_t i = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; i < n;
-         i += static_cast<int64_t>(gridDim.x) * kThreads) {
-        const float a = adv[i / T];
-        const float rho = expf(lp_new[i] - lp_old[i]);
+    float s = 0.f;
+    const int64_t n4 = n >> 2;
+    const float4* a4 = reinterpret_cast<const float4*>(lp_new);
+    const float4* b4 = reinterpret_cast<const float4*>(lp_old);
+    const uint32_t Tu = static_cast<uint32_t>(T);
+    auto term = [&](float ln, float lo_, uint32_t idx, float& g) {
+        const float a = adv[idx / Tu];
+        const float rho = __expf(ln - lo_);
         const float unclipped = rho * a;
         const float clipped = fminf(fmaxf(rho, 1.0f - lo), 1.0f + hi) * a;
         const bool take = unclipped <= clipped;
-        s += static_cast<double>(take ? unclipped : clipped);
-        if (grad) grad[i] = take ? -a * rho * inv_n : 0.0f;
+        g = take ? -a * rho * inv_n : 0.0f;
+        return take ? unclipped : clipped;
+    };
+    for (int64_t v = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; v < n4;
+         v += static_cast<int64_t>(gridDim.x) * kThreads) {
+        const float4 x = __ldcs(a4 + v);
+        const float4 y = __ldcs(b4 + v);
+        const uint32_t i0 = static_cast<uint32_t>(v << 2);
+        float4 g;
+        s += term(x.x, y.x, i0, g.x);
+        s += term(x.y, y.y, i0 + 1, g.y);
+        s += term(x.z, y.z, i0 + 2, g.z);
+        s += term(x.w, y.w, i0 + 3, g.w);
+        if (grad) __stcs(reinterpret_cast<float4*>(grad) + v, g);
     }
+    for (int64_t i = (n4 << 2) + static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; i < n;
+         i += static_cast<int64_t>(gridDim.x) * kThreads) {
+        float g;
+        s += term(lp_new[i], lp_old[i], static_cast<uint32_t>(i), g);
+        if (grad) grad[i] = g;
+    }
+    double d = s;
 #pragma unroll
-    for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
+    for (int o = 16; o; o >>= 1) d += __shfl_xor_sync(0xffffffffu, d, o);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = d;
     __syncthreads();
     if (threadIdx.x == 0) {
         double t = 0.0;
@@ -103,9 +148,17 @@ int ff_group_advantage(int n_groups, int G, const float* rewards, float eps_A, f
     if (G > 4096) return set_error(FF_ERR_UNSUPPORTED, "advantage: G=%d > 4096", G);
     if (!rewards || !adv) return set_error(FF_ERR_INVALID_ARG, "advantage: null pointer");
     if (!(eps_A >= 0.0f)) return set_error(FF_ERR_INVALID_ARG, "advantage: eps_A must be >= 0");
+    ProfScope prof(stream, "group_advantage", 0.0, 8.0 * n_groups * G);
+    if (G >= 4 && G <= 128 && (G & (G - 1)) == 0 && aligned16(rewards) && aligned16(adv)) {
+        const int64_t n4 = static_cast<int64_t>(n_groups) * G / 4;
+        const int64_t grid = (n4 + kThreads - 1) / kThreads;
+        if (grid > 0x7fffffff) return set_error(FF_ERR_UNSUPPORTED, "advantage: too many samples");
+        group_advantage_vec_kernel<<<static_cast<unsigned>(grid), kThreads, 0, stream>>>(
+            n4, G, reinterpret_cast<const float4*>(rewards), eps_A, reinterpret_cast<float4*>(adv));
+        return check_launch("group_advantage_vec_kernel");
+    }
     const int warps_per_block = kThreads / 32;
     const int grid = (n_groups + warps_per_block - 1) / warps_per_block;
-    ProfScope prof(stream, "group_advantage", 0.0, 8.0 * n_groups * G);
     group_advantage_kernel<<<grid, kThreads, 0, stream>>>(n_groups, G, rewards, eps_A, adv);
     return check_launch("group_advantage_kernel");
 }
@@ -122,6 +175,10 @@ int ff_grpo_loss(int B, int T, const float* lp_new, const float* lp_old, const f
     using namespace ff;
     if (B <= 0 || T <= 0) return set_error(FF_ERR_INVALID_ARG, "loss: B=%d T=%d must be positive", B, T);
     if (!lp_new || !lp_old || !adv || !loss) return set_error(FF_ERR_INVALID_ARG, "loss: null pointer");
+    if (!aligned16(lp_new) || !aligned16(lp_old) || (grad_lp_new && !aligned16(grad_lp_new)))
+        return set_error(FF_ERR_INVALID_ARG, "loss: lp_new, lp_old and grad_lp_new must be 16-byte aligned");
+    if (static_cast<int64_t>(B) * T >= (int64_t(1) << 32))
+        return set_error(FF_ERR_UNSUPPORTED, "loss: B * T must be below 2^32");
     if (!(clip_lo >= 0.0f && clip_lo < 1.0f && clip_hi >= 0.0f))
         return set_error(FF_ERR_INVALID_ARG, "loss: clip range must satisfy 0 <= lo < 1, hi >= 0");
     const int64_t n = static_cast<int64_t>(B) * T;

@@ -52,59 +52,66 @@ __device__ __forceinline__ double block_sum(double v, double* red) {
     return s;   // valid in thread 0
 }
 
+// Grid (blocks_per_sample, B); block k of sample b handles chunks
+// k, k + blocks_per_sample, ... and writes one fp64 partial.  The number of
+// blocks per sample depends only on D (see nblocks), so the summation order
+// is fixed.  The per-sample coefficients are formed once per block in fp64.
 template <int MODE>
-__global__ void __launch_bounds__(kThreads) sde_step_partial_kernel(int64_t D, int nchunk, const float* x,
+__global__ void __launch_bounds__(kThreads) sde_step_partial_kernel(int64_t D, int nblk, const float* x,
                                                                     const float* v, const float* eps, float* x_next,
                                                                     const float* t, const float* t_next,
                                                                     const float* sigma, double* partial) {
     __shared__ double red[kThreads / 32];
+    __shared__ StepCoef coef;
     const int b = blockIdx.y;
-    const int chunk = blockIdx.x;
-    const StepCoef c = step_coef(t, t_next, sigma, b);
+    if (threadIdx.x == 0) coef = step_coef(t, t_next, sigma, b);
+    __syncthreads();
+    const StepCoef c = coef;
     const int64_t row = static_cast<int64_t>(b) * D;
-    const int64_t base = static_cast<int64_t>(chunk) * kChunk;
     const float4* x4 = reinterpret_cast<const float4*>(x + row);
     const float4* v4 = reinterpret_cast<const float4*>(v + row);
     const float4* e4 = reinterpret_cast<const float4*>(eps + (MODE == FF_SDE_SAMPLE ? row : 0));
     float4* n4 = reinterpret_cast<float4*>(x_next + row);
     const int64_t nvec = D >> 2;
-
-    float4 xv[kVecPerThread], vv[kVecPerThread], ev[kVecPerThread];
-#pragma unroll
-    for (int j = 0; j < kVecPerThread; ++j) {
-        const int64_t i = (base >> 2) + threadIdx.x + j * kThreads;
-        if (i < nvec) {
-            xv[j] = __ldcs(x4 + i);
-            vv[j] = __ldcs(v4 + i);
-            ev[j] = MODE == FF_SDE_SAMPLE ? __ldcs(e4 + i) : __ldcs(reinterpret_cast<const float4*>(n4) + i);
-        }
-    }
     float ss = 0.f;
+    for (int64_t base = static_cast<int64_t>(blockIdx.x) * (kChunk / 4); base < nvec;
+         base += static_cast<int64_t>(nblk) * (kChunk / 4)) {
+        float4 xv[kVecPerThread], vv[kVecPerThread], ev[kVecPerThread];
 #pragma unroll
-    for (int j = 0; j < kVecPerThread; ++j) {
-        const int64_t i = (base >> 2) + threadIdx.x + j * kThreads;
-        if (i < nvec) {
-            float m[4] = {fmaf(c.cx, xv[j].x, c.cv * vv[j].x), fmaf(c.cx, xv[j].y, c.cv * vv[j].y),
-                          fmaf(c.cx, xv[j].z, c.cv * vv[j].z), fmaf(c.cx, xv[j].w, c.cv * vv[j].w)};
-            float o[4];
-            if (MODE == FF_SDE_SAMPLE) {
-                o[0] = fmaf(c.std, ev[j].x, m[0]);
-                o[1] = fmaf(c.std, ev[j].y, m[1]);
-                o[2] = fmaf(c.std, ev[j].z, m[2]);
-                o[3] = fmaf(c.std, ev[j].w, m[3]);
-                __stcs(n4 + i, make_float4(o[0], o[1], o[2], o[3]));
-            } else {
-                o[0] = ev[j].x; o[1] = ev[j].y; o[2] = ev[j].z; o[3] = ev[j].w;
+        for (int j = 0; j < kVecPerThread; ++j) {
+            const int64_t i = base + threadIdx.x + j * kThreads;
+            if (i < nvec) {
+                xv[j] = __ldcs(x4 + i);
+                vv[j] = __ldcs(v4 + i);
+                ev[j] = MODE == FF_SDE_SAMPLE ? __ldcs(e4 + i) : __ldcs(reinterpret_cast<const float4*>(n4) + i);
             }
+        }
 #pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                const float r = o[k] - m[k];
-                ss = fmaf(r, r, ss);
+        for (int j = 0; j < kVecPerThread; ++j) {
+            const int64_t i = base + threadIdx.x + j * kThreads;
+            if (i < nvec) {
+                float m[4] = {fmaf(c.cx, xv[j].x, c.cv * vv[j].x), fmaf(c.cx, xv[j].y, c.cv * vv[j].y),
+                              fmaf(c.cx, xv[j].z, c.cv * vv[j].z), fmaf(c.cx, xv[j].w, c.cv * vv[j].w)};
+                float o[4];
+                if (MODE == FF_SDE_SAMPLE) {
+                    o[0] = fmaf(c.std, ev[j].x, m[0]);
+                    o[1] = fmaf(c.std, ev[j].y, m[1]);
+                    o[2] = fmaf(c.std, ev[j].z, m[2]);
+                    o[3] = fmaf(c.std, ev[j].w, m[3]);
+                    __stcs(n4 + i, make_float4(o[0], o[1], o[2], o[3]));
+                } else {
+                    o[0] = ev[j].x; o[1] = ev[j].y; o[2] = ev[j].z; o[3] = ev[j].w;
+                }
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    const float r = o[k] - m[k];
+                    ss = fmaf(r, r, ss);
+                }
             }
         }
     }
     const double s = block_sum(static_cast<double>(ss), red);
-    if (threadIdx.x == 0) partial[static_cast<int64_t>(b) * nchunk + chunk] = s;
+    if (threadIdx.x == 0) partial[static_cast<int64_t>(b) * nblk + blockIdx.x] = s;
 }
 
 __global__ void __launch_bounds__(kThreads) sde_logprob_finalize_kernel(int64_t D, int nchunk, const double* partial,
@@ -129,7 +136,14 @@ __global__ void __launch_bounds__(kThreads) sde_logprob_finalize_kernel(int64_t 
     }
 }
 
-int nchunks(int64_t D) { return static_cast<int>((D + kChunk - 1) / kChunk); }
+constexpr int kMaxBlocksPerSample = 1024;
+
+// partial sums (blocks) per sample: one per 4096-element chunk up to 1024,
+// then every block loops over several chunks
+int nchunks(int64_t D) {
+    const int64_t c = (D + kChunk - 1) / kChunk;
+    return static_cast<int>(c < kMaxBlocksPerSample ? c : kMaxBlocksPerSample);
+}
 
 }  // namespace
 }  // namespace ff
@@ -266,9 +280,9 @@ extern "C" int ff_sde_step_logprob_noalloc(int B, int64_t D, const float* x_t, c
     const int nc = nchunks(D);
     if (static_cast<int64_t>(B) * nc > kNoAllocMaxPartials)
         return set_error(FF_ERR_UNSUPPORTED,
-                         "sde (no-alloc): B * ceil(D / %d) = %lld partial sums exceed the built-in scratch of %d; "
-                         "use ff_sde_step_logprob with a workspace",
-                         kChunk, (long long)B * nc, kNoAllocMaxPartials);
+                         "sde (no-alloc): B * min(ceil(D / %d), %d) = %lld partial sums exceed the built-in scratch "
+                         "of %d; use ff_sde_step_logprob with a workspace",
+                         kChunk, kMaxBlocksPerSample, (long long)B * nc, kNoAllocMaxPartials);
     double* partial = nullptr;
     const int rc0 = sde_scratch_address(&partial);
     if (rc0) return rc0;

@@ -82,7 +82,8 @@ def test_workspace_queries(L):
     n1 = ffi.ff_sde_workspace_size(4, 262144)
     assert n1 == 4 * 64 * 8
     assert ffi.ff_grpo_loss_workspace_size(32, 10) == 8
-    assert ffi.ff_grpo_loss_workspace_size(1 << 20, 64) == 1024 * 8
+    assert ffi.ff_grpo_loss_workspace_size(1 << 20, 64) == 1216 * 8
+    assert ffi.ff_sde_workspace_size(4, 1 << 26) == 4 * 1024 * 8
     with pytest.raises(ffi.FFError):
         ffi.ff_sde_workspace_size(0, 16)
 
