@@ -52,6 +52,7 @@ extern "C" {
 #define FF_SCHED_ODE 2        /* Table 1: sigma_t = 0                       */
 
 #define FF_ARCH_MMDIT 0   /* Flux / Qwen-Image style double + single stream */
+#define FF_ARCH_WAN 1     /* WAN-style video DiT: self-attn + text cross-attn + FFN */
 
 /* Last error message of the calling thread ("" if none). */
 const char* ff_last_error(void);
@@ -182,17 +183,27 @@ int ff_grpo_loss(int B, int T, const float* lp_new, const float* lp_old,
  * by pos * theta^(-2j/a)); text tokens sit at position (0, 0, 0); GELU is the
  * tanh form; attention scale is 1/sqrt(d).
  *
+ * WAN-style DiT (arch FF_ARCH_WAN; n_double = number of blocks, n_single =
+ * 0): text embedded by Linear-GELU-Linear; one shared projection of the
+ * timestep embedding e to six H-wide vectors plus a learned per-block bias
+ * gives each block's (shift, scale, gate) x 2; a block is LN-modulate ->
+ * QKV -> per-head RMSNorm + 3-axis RoPE -> self-attention over the latent
+ * tokens -> gated projection; affine LN -> cross-attention (RMSNorm'd q from
+ * the latent tokens, RMSNorm'd k and v from the text, no RoPE) -> projection
+ * added ungated; LN-modulate -> GELU MLP -> gated residual.  The final layer
+ * uses shift / scale = e + a learned bias.
+ *
  * Weights live in ONE caller-owned bf16 device blob; ff_dit_weight_layout
  * gives every tensor's name, element offset and shape (nn.Linear [out, in]).
  * ------------------------------------------------------------------------ */
 typedef struct ff_dit_config {
-    int arch;          /* FF_ARCH_MMDIT */
+    int arch;          /* FF_ARCH_MMDIT or FF_ARCH_WAN */
     int hidden;        /* H, multiple of 64 */
     int heads;         /* h */
     int head_dim;      /* d: 64 or 128; h * d == H */
     int mlp;           /* F, multiple of 64 */
-    int n_double;      /* double-stream blocks */
-    int n_single;      /* single-stream blocks */
+    int n_double;      /* double-stream blocks (WAN: the number of blocks) */
+    int n_single;      /* single-stream blocks (WAN: 0) */
     int patch_dim;     /* P, latent token width (64), multiple of 16 */
     int txt_dim;       /* D_txt, multiple of 64 */
     int n_txt;         /* N_t text tokens per sample */

@@ -292,3 +292,97 @@ def velocity(P, cfg, x_t, txt, t, img_rows=None):
         h = modulate(layer_norm(xi), mods[b, off:off + H], mods[b, off + H:off + 2 * H])
         outs.append(linear(h, P["final.w"], P["final.b"]))
     return np.stack(outs)
+
+
+# ---------------------------------------------------------------------------
+# WAN-style video DiT (self-attention over latent tokens with 3D RoPE,
+# cross-attention to the embedded text, gated FFN).  The paper names WAN
+# (Sec. 1) without an architecture; the definition below is the one the
+# CUDA path implements:
+#
+#   e  = Linear-SiLU-Linear(sinusoid(1000 t))                      [H]
+#   e0 = SiLU(e) W_mod^T + b_mod                                   [6H], shared
+#   txt_h = Linear(GELU(Linear(txt)))                              [N_t, H]
+#   x = Linear(x_t)                                                [N_i, H]
+#   per block l, (shift1, scale1, gate1, shift2, scale2, gate2) = e0 + b_l:
+#     h = LN(x) (1 + scale1) + shift1; q, k, v = h W_qkv^T + b
+#     q, k <- RoPE(RMSNorm_head(q, k)) over (frame, row, col) axes
+#     x += gate1 * (SelfAttn(q, k, v) W_proj^T + b)
+#     h = LN(x) * w_cn + b_cn                  (affine LN, no modulation)
+#     qc = RMSNorm_head(h W_cq^T + b);  kc, vc = txt_h W_ckv^T + b;
+#     kc = RMSNorm_head(kc)                    (no RoPE in cross-attention)
+#     x += CrossAttn(qc, kc, vc) W_cproj^T + b (no gate)
+#     h = LN(x) (1 + scale2) + shift2
+#     x += gate2 * (GELU(h W_1^T + b_1) W_2^T + b_2)
+#   final: (shift, scale) = e + b_final (each H), v = (LN(x)(1+scale)+shift) W^T + b
+# ---------------------------------------------------------------------------
+
+def wan_param_specs(cfg: dict):
+    H, F, P, d = cfg["hidden"], cfg["mlp"], cfg["patch_dim"], cfg["head_dim"]
+    tf = cfg["time_freq_dim"]
+    s = [("t_embed.fc1.w", (H, tf)), ("t_embed.fc1.b", (H,)),
+         ("t_embed.fc2.w", (H, H)), ("t_embed.fc2.b", (H,)),
+         ("mod.w", (6 * H, H)), ("mod.b", (6 * H,)),
+         ("img_in.w", (H, P)), ("img_in.b", (H,)),
+         ("txt_in.w", (H, cfg["txt_dim"])), ("txt_in.b", (H,)),
+         ("txt_in2.w", (H, H)), ("txt_in2.b", (H,))]
+    for l in range(cfg["n_double"]):
+        p = f"blocks.{l}."
+        s += [(p + "mod.b", (6 * H,)),
+              (p + "qkv.w", (3 * H, H)), (p + "qkv.b", (3 * H,)),
+              (p + "q_norm.scale", (d,)), (p + "k_norm.scale", (d,)),
+              (p + "proj.w", (H, H)), (p + "proj.b", (H,)),
+              (p + "cross_norm.scale", (H,)), (p + "cross_norm.b", (H,)),
+              (p + "cross_q.w", (H, H)), (p + "cross_q.b", (H,)), (p + "cross_q_norm.scale", (d,)),
+              (p + "cross_kv.w", (2 * H, H)), (p + "cross_kv.b", (2 * H,)), (p + "cross_k_norm.scale", (d,)),
+              (p + "cross_proj.w", (H, H)), (p + "cross_proj.b", (H,)),
+              (p + "mlp1.w", (F, H)), (p + "mlp1.b", (F,)),
+              (p + "mlp2.w", (H, F)), (p + "mlp2.b", (H,))]
+    s += [("final.mod.b", (2 * H,)), ("final.w", (P, H)), ("final.b", (P,))]
+    return s
+
+
+def wan_velocity(P, cfg, x_t, txt, t, img_rows=None):
+    """v_theta(x_t, t) of the WAN-style DiT.  Same conventions as velocity();
+    img_rows restricts the last block and the final layer to those tokens."""
+    x_t = np.asarray(x_t, dtype=np.float64)
+    txt = np.asarray(txt, dtype=np.float64)
+    B = x_t.shape[0]
+    H, nh = cfg["hidden"], cfg["heads"]
+    L = cfg["n_double"]
+    emb = timestep_embedding(t, cfg["time_freq_dim"])
+    e = linear(silu(linear(emb, P["t_embed.fc1.w"], P["t_embed.fc1.b"])), P["t_embed.fc2.w"], P["t_embed.fc2.b"])
+    e0 = linear(silu(e), P["mod.w"], P["mod.b"])
+    ang = rope_angles(image_positions(cfg["grid"]), cfg["rope_axes"], cfg["rope_theta"])
+    rows = None if img_rows is None else np.asarray(img_rows, dtype=np.int64)
+    outs = []
+    for b in range(B):
+        th = linear(gelu_tanh(linear(txt[b], P["txt_in.w"], P["txt_in.b"])), P["txt_in2.w"], P["txt_in2.b"])
+        x = linear(x_t[b], P["img_in.w"], P["img_in.b"])
+        for l in range(L):
+            p = f"blocks.{l}."
+            m = e0[b] + P[p + "mod.b"]
+            sh1, sc1, g1, sh2, sc2, g2 = (m[i * H:(i + 1) * H] for i in range(6))
+            h = modulate(layer_norm(x), sh1, sc1)
+            qkv = linear(h, P[p + "qkv.w"], P[p + "qkv.b"])
+            q = apply_rope(rms_norm(_heads(qkv[:, :H], nh), P[p + "q_norm.scale"]), ang)
+            k = apply_rope(rms_norm(_heads(qkv[:, H:2 * H], nh), P[p + "k_norm.scale"]), ang)
+            v = _heads(qkv[:, 2 * H:], nh)
+            r = np.arange(x.shape[0]) if (rows is None or l < L - 1) else rows
+            o = attention(q[r], k, v).reshape(len(r), H)
+            x = x[r] + g1 * linear(o, P[p + "proj.w"], P[p + "proj.b"])
+            h = layer_norm(x) * P[p + "cross_norm.scale"] + P[p + "cross_norm.b"]
+            qc = rms_norm(_heads(linear(h, P[p + "cross_q.w"], P[p + "cross_q.b"]), nh), P[p + "cross_q_norm.scale"])
+            kv = linear(th, P[p + "cross_kv.w"], P[p + "cross_kv.b"])
+            kc = rms_norm(_heads(kv[:, :H], nh), P[p + "cross_k_norm.scale"])
+            vc = _heads(kv[:, H:], nh)
+            x = x + linear(attention(qc, kc, vc).reshape(len(r), H), P[p + "cross_proj.w"], P[p + "cross_proj.b"])
+            h = modulate(layer_norm(x), sh2, sc2)
+            u = gelu_tanh(linear(h, P[p + "mlp1.w"], P[p + "mlp1.b"]))
+            x = x + g2 * linear(u, P[p + "mlp2.w"], P[p + "mlp2.b"])
+        if L == 0 and rows is not None:
+            x = x[rows]
+        fm = P["final.mod.b"]
+        h = modulate(layer_norm(x), e[b] + fm[:H], e[b] + fm[H:])
+        outs.append(linear(h, P["final.w"], P["final.b"]))
+    return np.stack(outs)

@@ -56,9 +56,10 @@ struct ACfg {
 };
 
 struct AttnParams {
-    int n[2];            // tokens per sample in each segment
-    int qpairs0;         // 256-row query blocks of segment 0 (segment 1's follow)
-    int H;
+    int nq[2];           // query tokens per sample in each query segment
+    int nkv[2];          // key/value tokens per sample in each key/value segment
+    int qpairs0;         // 256-row query blocks of query segment 0 (segment 1's follow)
+    int q_col, k_col, v_col;
     float scale_log2;
     __nv_bfloat16* out[2];
     int64_t ldo[2];
@@ -170,8 +171,8 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
     const int h = blockIdx.y;
     const int seg = blockIdx.x < p.qpairs0 ? 0 : 1;
     const int q0 = (blockIdx.x - (seg ? p.qpairs0 : 0)) * (2 * kBM);   // first query row within the segment
-    const int nt0 = (p.n[0] + kBN - 1) / kBN;
-    const int ntiles = nt0 + (p.n[1] + kBN - 1) / kBN;
+    const int nt0 = (p.nkv[0] + kBN - 1) / kBN;
+    const int ntiles = nt0 + (p.nkv[1] + kBN - 1) / kBN;
 
     if (threadIdx.x == 0) {
         *abort_flag = 0;
@@ -218,20 +219,20 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
         mbar_arrive_expect_tx(&bar.q_full, 2 * C::kQBytes);
         for (int t = 0; t < 2; ++t)
             for (int c = 0; c < HD / 64; ++c)
-                tma_load_2d(sQ + t * C::kQBytes + c * (kBM * 128), tq, &bar.q_full, h * HD + c * 64,
-                            b * p.n[seg] + q0 + t * kBM);
+                tma_load_2d(sQ + t * C::kQBytes + c * (kBM * 128), tq, &bar.q_full, p.q_col + h * HD + c * 64,
+                            b * p.nq[seg] + q0 + t * kBM);
         for (int j = 0; j < ntiles && !*abort_flag; ++j) {
             const int s = j % kStages;
             if (!mbar_wait(&bar.kv_empty[s], ((j / kStages) & 1) ^ 1)) { fail(); break; }
             const int ks = j < nt0 ? 0 : 1;
-            const int row = b * p.n[ks] + (j - (ks ? nt0 : 0)) * kBN;
+            const int row = b * p.nkv[ks] + (j - (ks ? nt0 : 0)) * kBN;
             const CUtensorMap* tkv = ks ? &tm_kv1 : &tm_kv0;
             uint8_t* dk = sKV + s * C::kStageBytes;
             uint8_t* dv = dk + C::kKBytes;
             mbar_arrive_expect_tx(&bar.kv_full[s], C::kStageBytes);
             for (int c = 0; c < HD / 64; ++c) {
-                tma_load_2d(dk + c * (kBN * 128), tkv, &bar.kv_full[s], p.H + h * HD + c * 64, row);
-                tma_load_2d(dv + c * (kBN * 128), tkv, &bar.kv_full[s], 2 * p.H + h * HD + c * 64, row);
+                tma_load_2d(dk + c * (kBN * 128), tkv, &bar.kv_full[s], p.k_col + h * HD + c * 64, row);
+                tma_load_2d(dv + c * (kBN * 128), tkv, &bar.kv_full[s], p.v_col + h * HD + c * 64, row);
             }
         }
     } else if (warp == 1 && lane == 0) {
@@ -321,7 +322,7 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
             tmem_ld_wait();
 
             const int ks = j < nt0 ? 0 : 1;
-            const int valid = p.n[ks] - (j - (ks ? nt0 : 0)) * kBN;   // columns < valid are real tokens
+            const int valid = p.nkv[ks] - (j - (ks ? nt0 : 0)) * kBN;   // columns < valid are real tokens
             if (valid < kBN) {
 #pragma unroll
                 for (int i = 0; i < kBN; ++i)
@@ -385,8 +386,8 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
             tc_fence_after();
             const float inv = 1.f / l;
             const int row = q0 + t * kBM + r;
-            const bool live = row < p.n[seg];
-            __nv_bfloat16* dst = p.out[seg] + (static_cast<int64_t>(b) * p.n[seg] + row) * p.ldo[seg] + h * HD;
+            const bool live = row < p.nq[seg];
+            __nv_bfloat16* dst = p.out[seg] + (static_cast<int64_t>(b) * p.nq[seg] + row) * p.ldo[seg] + h * HD;
 #pragma unroll 1
             for (int c = 0; c < HD; c += 32) {
                 uint32_t o[32];
@@ -427,36 +428,38 @@ __global__ void exp2_poly_kernel(const float2* x, float2* y, int64_t n2) {
 }
 
 template <int HD>
-int launch_attn(const AttnSegment& s0, const AttnSegment& s1, int B, int heads, int H, cudaStream_t stream) {
+int launch_attn(const AttnSpec& a, cudaStream_t stream) {
     using C = ACfg<HD>;
     if (cudaFuncSetAttribute(attn_tcgen05_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes) !=
         cudaSuccess)
         return set_error(FF_ERR_CUDA, "attention: cannot set shared memory size");
-    const AttnSegment* seg[2] = {&s0, &s1};
     CUtensorMap tq[2], tkv[2];
     for (int i = 0; i < 2; ++i) {
-        // a segment with no tokens still needs a valid map: point it at the other one
-        const AttnSegment& s = seg[i]->n > 0 ? *seg[i] : *seg[1 - i];
-        const int64_t rows = static_cast<int64_t>(B) * s.n;
-        int rc = make_tmap_bf16(&tq[i], s.qkv, rows, 3 * static_cast<int64_t>(H), s.ld, kBM);
+        // an empty segment still needs a valid map: point it at the other one
+        const AttnQuerySeg& q = a.q[i].n > 0 ? a.q[i] : a.q[1 - i];
+        int rc = make_tmap_bf16(&tq[i], q.buf, static_cast<int64_t>(a.B) * q.n, q.ld, q.ld, kBM);
         if (rc) return rc;
-        rc = make_tmap_bf16(&tkv[i], s.qkv, rows, 3 * static_cast<int64_t>(H), s.ld, kBN);
+        const AttnKvSeg& kv = a.kv[i].n > 0 ? a.kv[i] : a.kv[1 - i];
+        rc = make_tmap_bf16(&tkv[i], kv.buf, static_cast<int64_t>(a.B) * kv.n, kv.ld, kv.ld, kBN);
         if (rc) return rc;
     }
     AttnParams p;
-    p.n[0] = s0.n;
-    p.n[1] = s1.n;
-    p.qpairs0 = (s0.n + 2 * kBM - 1) / (2 * kBM);
-    p.H = H;
+    for (int i = 0; i < 2; ++i) {
+        p.nq[i] = a.q[i].n;
+        p.nkv[i] = a.kv[i].n;
+        p.out[i] = a.q[i].out;
+        p.ldo[i] = a.q[i].ldo;
+    }
+    p.qpairs0 = (a.q[0].n + 2 * kBM - 1) / (2 * kBM);
+    p.q_col = a.q_col;
+    p.k_col = a.k_col;
+    p.v_col = a.v_col;
     p.scale_log2 = static_cast<float>(1.4426950408889634 / sqrt(static_cast<double>(HD)));
-    p.out[0] = s0.out;
-    p.out[1] = s1.out;
-    p.ldo[0] = s0.ldo;
-    p.ldo[1] = s1.ldo;
-    const int N = s0.n + s1.n;
-    const dim3 grid(p.qpairs0 + (s1.n + 2 * kBM - 1) / (2 * kBM), heads, B);
-    const double nn = static_cast<double>(N) * N;
-    ProfScope prof(stream, "attention", 4.0 * B * heads * nn * HD, 8.0 * B * static_cast<double>(N) * H);
+    const dim3 grid(p.qpairs0 + (a.q[1].n + 2 * kBM - 1) / (2 * kBM), a.heads, a.B);
+    const double nkv = static_cast<double>(a.kv[0].n + a.kv[1].n);
+    const double nq = static_cast<double>(a.q[0].n + a.q[1].n);
+    ProfScope prof(stream, "attention", 4.0 * a.B * a.heads * nq * nkv * HD,
+                   2.0 * a.B * a.heads * HD * (2.0 * nq + 2.0 * nkv));
     attn_tcgen05_kernel<HD><<<grid, kThreads, C::kSmemBytes, stream>>>(tq[0], tq[1], tkv[0], tkv[1], p,
                                                                         device_status_ptr());
     return check_launch("attn_tcgen05_kernel");
@@ -464,21 +467,46 @@ int launch_attn(const AttnSegment& s0, const AttnSegment& s1, int B, int heads, 
 
 }  // namespace
 
+int attention_general(const AttnSpec& a, cudaStream_t stream) {
+    if (a.B <= 0 || a.heads <= 0 || a.B > 65535 || a.heads > 65535)
+        return set_error(FF_ERR_INVALID_ARG, "attention: bad batch / heads");
+    for (int i = 0; i < 2; ++i) {
+        if (a.q[i].n < 0 || a.kv[i].n < 0) return set_error(FF_ERR_INVALID_ARG, "attention: negative token count");
+        if (a.q[i].n && (!a.q[i].buf || !a.q[i].out || !aligned16(a.q[i].out) || a.q[i].ld % 8 || a.q[i].ldo % 8))
+            return set_error(FF_ERR_INVALID_ARG, "attention: bad query segment %d", i);
+        if (a.kv[i].n && (!a.kv[i].buf || a.kv[i].ld % 8))
+            return set_error(FF_ERR_INVALID_ARG, "attention: bad key/value segment %d", i);
+    }
+    if (a.q[0].n + a.q[1].n <= 0 || a.kv[0].n + a.kv[1].n <= 0)
+        return set_error(FF_ERR_INVALID_ARG, "attention: no queries or no keys");
+    if (a.q_col % 64 || a.k_col % 64 || a.v_col % 64)
+        return set_error(FF_ERR_UNSUPPORTED, "attention: column offsets must be multiples of 64");
+    const int64_t hd = static_cast<int64_t>(a.heads) * a.head_dim;
+    for (int i = 0; i < 2; ++i) {
+        if (a.q[i].n && a.q_col + hd > a.q[i].ld) return set_error(FF_ERR_INVALID_ARG, "attention: q columns exceed ld");
+        if (a.kv[i].n && (a.k_col + hd > a.kv[i].ld || a.v_col + hd > a.kv[i].ld))
+            return set_error(FF_ERR_INVALID_ARG, "attention: k/v columns exceed ld");
+    }
+    if (a.head_dim == 128) return launch_attn<128>(a, stream);
+    if (a.head_dim == 64) return launch_attn<64>(a, stream);
+    return set_error(FF_ERR_UNSUPPORTED, "attention: head_dim %d", a.head_dim);
+}
+
 int attention(const AttnSegment& s0, const AttnSegment& s1, int B, int heads, int head_dim, int H,
               cudaStream_t stream) {
-    if (B <= 0 || heads <= 0 || s0.n < 0 || s1.n < 0 || s0.n + s1.n <= 0)
-        return set_error(FF_ERR_INVALID_ARG, "attention: bad shape");
-    if (B > 65535 || heads > 65535) return set_error(FF_ERR_UNSUPPORTED, "attention: grid too large");
-    if ((s0.n && (!s0.qkv || !s0.out)) || (s1.n && (!s1.qkv || !s1.out)))
-        return set_error(FF_ERR_INVALID_ARG, "attention: null segment");
-    if (s0.ld % 8 || s1.ld % 8 || s0.ldo % 8 || s1.ldo % 8)
-        return set_error(FF_ERR_INVALID_ARG, "attention: leading dimensions must be multiples of 8");
-    if ((s0.n && !aligned16(s0.out)) || (s1.n && !aligned16(s1.out)))
-        return set_error(FF_ERR_INVALID_ARG, "attention: outputs must be 16-byte aligned");
-    if (H % 64) return set_error(FF_ERR_UNSUPPORTED, "attention: H %% 64 != 0");
-    if (head_dim == 128) return launch_attn<128>(s0, s1, B, heads, H, stream);
-    if (head_dim == 64) return launch_attn<64>(s0, s1, B, heads, H, stream);
-    return set_error(FF_ERR_UNSUPPORTED, "attention: head_dim %d", head_dim);
+    AttnSpec a;
+    const AttnSegment* seg[2] = {&s0, &s1};
+    for (int i = 0; i < 2; ++i) {
+        a.q[i] = AttnQuerySeg{seg[i]->qkv, seg[i]->ld, seg[i]->n, seg[i]->out, seg[i]->ldo};
+        a.kv[i] = AttnKvSeg{seg[i]->qkv, seg[i]->ld, seg[i]->n};
+    }
+    a.q_col = 0;
+    a.k_col = H;
+    a.v_col = 2 * H;
+    a.B = B;
+    a.heads = heads;
+    a.head_dim = head_dim;
+    return attention_general(a, stream);
 }
 
 }  // namespace ff

@@ -70,6 +70,9 @@ int ff_debug_qk_norm_rope(int rows, int rows_txt, int heads, int head_dim, void*
     a.axes0 = rope_axes[0]; a.axes1 = rope_axes[1]; a.axes2 = rope_axes[2]; a.theta = rope_theta;
     a.q_scale_txt = a.q_scale_img = static_cast<const __nv_bfloat16*>(q_scale);
     a.k_scale_txt = a.k_scale_img = static_cast<const __nv_bfloat16*>(k_scale);
+    a.col[0] = 0;
+    a.col[1] = heads * head_dim;
+    a.rope = 1;
     return qk_norm_rope(a, stream);
 }
 

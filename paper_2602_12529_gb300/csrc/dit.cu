@@ -76,9 +76,43 @@ std::vector<Spec> specs(const ff_dit_config& c) {
     return s;
 }
 
+// WAN-style DiT parameters, same order and names as the oracle's list.
+std::vector<Spec> specs_wan(const ff_dit_config& c) {
+    const int64_t H = c.hidden, F = c.mlp, P = c.patch_dim, d = c.head_dim;
+    std::vector<Spec> s;
+    auto mat = [&](const std::string& n, int64_t o, int64_t i) { s.push_back({n, 2, o, i}); };
+    auto vec = [&](const std::string& n, int64_t o) { s.push_back({n, 1, o, 0}); };
+    mat("t_embed.fc1.w", H, c.time_freq_dim); vec("t_embed.fc1.b", H);
+    mat("t_embed.fc2.w", H, H); vec("t_embed.fc2.b", H);
+    mat("mod.w", 6 * H, H); vec("mod.b", 6 * H);
+    mat("img_in.w", H, P); vec("img_in.b", H);
+    mat("txt_in.w", H, c.txt_dim); vec("txt_in.b", H);
+    mat("txt_in2.w", H, H); vec("txt_in2.b", H);
+    for (int l = 0; l < c.n_double; ++l) {
+        const std::string p = "blocks." + std::to_string(l) + ".";
+        vec(p + "mod.b", 6 * H);
+        mat(p + "qkv.w", 3 * H, H); vec(p + "qkv.b", 3 * H);
+        vec(p + "q_norm.scale", d); vec(p + "k_norm.scale", d);
+        mat(p + "proj.w", H, H); vec(p + "proj.b", H);
+        vec(p + "cross_norm.scale", H); vec(p + "cross_norm.b", H);
+        mat(p + "cross_q.w", H, H); vec(p + "cross_q.b", H); vec(p + "cross_q_norm.scale", d);
+        mat(p + "cross_kv.w", 2 * H, H); vec(p + "cross_kv.b", 2 * H); vec(p + "cross_k_norm.scale", d);
+        mat(p + "cross_proj.w", H, H); vec(p + "cross_proj.b", H);
+        mat(p + "mlp1.w", F, H); vec(p + "mlp1.b", F);
+        mat(p + "mlp2.w", H, F); vec(p + "mlp2.b", H);
+    }
+    vec("final.mod.b", 2 * H);
+    mat("final.w", P, H); vec("final.b", P);
+    return s;
+}
+
+std::vector<Spec> specs_for(const ff_dit_config& c) { return c.arch == FF_ARCH_WAN ? specs_wan(c) : specs(c); }
+
 int validate(const ff_dit_config* c) {
     if (!c) return set_error(FF_ERR_INVALID_ARG, "config is null");
-    if (c->arch != FF_ARCH_MMDIT) return set_error(FF_ERR_UNSUPPORTED, "arch %d not supported", c->arch);
+    if (c->arch != FF_ARCH_MMDIT && c->arch != FF_ARCH_WAN) return set_error(FF_ERR_UNSUPPORTED, "arch %d not supported", c->arch);
+    if (c->arch == FF_ARCH_WAN && (c->n_single != 0 || c->n_double < 1))
+        return set_error(FF_ERR_INVALID_ARG, "WAN: n_double = blocks >= 1, n_single = 0");
     if (c->hidden <= 0 || c->hidden % 128) return set_error(FF_ERR_UNSUPPORTED, "hidden %d must be a multiple of 128", c->hidden);
     if (c->head_dim != 64 && c->head_dim != 128) return set_error(FF_ERR_UNSUPPORTED, "head_dim %d", c->head_dim);
     if (c->heads * c->head_dim != c->hidden) return set_error(FF_ERR_INVALID_ARG, "heads * head_dim != hidden");
@@ -106,17 +140,24 @@ struct Workspace {
     __nv_bfloat16 *temb, *th, *tc;
     float* x;
     __nv_bfloat16 *xb, *h, *qkv, *o, *u;
+    // WAN only
+    float *e, *e0;
+    __nv_bfloat16 *txt1, *txth, *kvc;
     size_t bytes;
 };
 
 Workspace plan(const ff_dit_config& c, int B, uint8_t* base) {
     const size_t H = c.hidden, F = c.mlp;
     const size_t Ni = static_cast<size_t>(c.grid_f) * c.grid_h * c.grid_w;
-    const size_t R = static_cast<size_t>(B) * (c.n_txt + Ni);
+    const bool wan = c.arch == FF_ARCH_WAN;
+    // WAN keeps only latent tokens in the residual stream; text lives in its own buffers
+    const size_t R = static_cast<size_t>(B) * (wan ? Ni : c.n_txt + Ni);
+    const size_t Rt = static_cast<size_t>(B) * c.n_txt;
+    const size_t Wm = wan ? static_cast<size_t>(c.n_double) * 6 * H + 2 * H : static_cast<size_t>(mod_width(c));
     size_t o = 0;
     Workspace w{};
     auto take = [&](size_t bytes) { uint8_t* p = base ? base + o : nullptr; o += up(bytes); return p; };
-    w.mods = reinterpret_cast<float*>(take(static_cast<size_t>(B) * mod_width(c) * 4));
+    w.mods = reinterpret_cast<float*>(take(static_cast<size_t>(B) * Wm * 4));
     w.temb = reinterpret_cast<__nv_bfloat16*>(take(static_cast<size_t>(B) * c.time_freq_dim * 2));
     w.th = reinterpret_cast<__nv_bfloat16*>(take(B * H * 2));
     w.tc = reinterpret_cast<__nv_bfloat16*>(take(B * H * 2));
@@ -126,6 +167,13 @@ Workspace plan(const ff_dit_config& c, int B, uint8_t* base) {
     w.qkv = reinterpret_cast<__nv_bfloat16*>(take(R * 3 * H * 2));
     w.o = reinterpret_cast<__nv_bfloat16*>(take(R * H * 2));
     w.u = reinterpret_cast<__nv_bfloat16*>(take(R * (H + F) * 2));
+    if (wan) {
+        w.e = reinterpret_cast<float*>(take(B * H * 4));
+        w.e0 = reinterpret_cast<float*>(take(B * 6 * H * 4));
+        w.txt1 = reinterpret_cast<__nv_bfloat16*>(take(Rt * H * 2));
+        w.txth = reinterpret_cast<__nv_bfloat16*>(take(Rt * H * 2));
+        w.kvc = reinterpret_cast<__nv_bfloat16*>(take(Rt * 2 * H * 2));
+    }
     w.bytes = o;
     return w;
 }
@@ -135,6 +183,172 @@ Workspace plan(const ff_dit_config& c, int B, uint8_t* base) {
         const int rc_ = (expr);     \
         if (rc_ != FF_OK) return rc_; \
     } while (0)
+
+// WAN-style velocity: latent tokens only in the residual stream; the text is
+// embedded once per call and feeds every block's cross-attention keys and
+// values.
+int wan_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, const float* t, float* v_out,
+                 const Workspace& w, cudaStream_t stream) {
+    const ff_dit_config& c = m->cfg;
+    const int H = c.hidden, F = c.mlp, P = c.patch_dim, d = c.head_dim, L = c.n_double;
+    const int Nt = c.n_txt, Ni = c.grid_f * c.grid_h * c.grid_w;
+    const int Rt = B * Nt, Ri = B * Ni;
+    const int64_t Wm = m->mod_width;
+    auto W = [&](const std::string& n) { return m->w + m->off.at(n); };
+
+    // timestep embedding e (fp32), SiLU(e) (bf16), e0 = SiLU(e) W_mod^T + b, per-block modulation
+    FF_TRY(timestep_embed(t, B, c.time_freq_dim, w.temb, stream));
+    {
+        GemmEpilogue e;
+        e.act = ACT_SILU; e.bias = W("t_embed.fc1.b"); e.out0 = w.th; e.ld0 = H;
+        FF_TRY(gemm_bf16(w.temb, c.time_freq_dim, W("t_embed.fc1.w"), c.time_freq_dim, B, H, c.time_freq_dim, e, stream));
+    }
+    {
+        GemmEpilogue e;
+        e.out_f32 = 1; e.bias = W("t_embed.fc2.b"); e.out0 = w.e; e.ld0 = H;
+        FF_TRY(gemm_bf16(w.th, H, W("t_embed.fc2.w"), H, B, H, H, e, stream));
+    }
+    {
+        GemmEpilogue e;
+        e.act = ACT_SILU; e.bias = W("t_embed.fc2.b"); e.out0 = w.tc; e.ld0 = H;
+        FF_TRY(gemm_bf16(w.th, H, W("t_embed.fc2.w"), H, B, H, H, e, stream));
+    }
+    {
+        GemmEpilogue e;
+        e.out_f32 = 1; e.bias = W("mod.b"); e.out0 = w.e0; e.ld0 = 6 * H;
+        FF_TRY(gemm_bf16(w.tc, H, W("mod.w"), H, B, 6 * H, H, e, stream));
+    }
+    const int64_t stride = L > 1 ? m->off.at("blocks.1.mod.b") - m->off.at("blocks.0.mod.b") : 0;
+    FF_TRY(wan_modulation(w.e, w.e0, W("blocks.0.mod.b"), stride, L, W("final.mod.b"), B, H, w.mods, Wm, stream));
+
+    // latent tokens and text embeddings
+    FF_TRY(f32_to_bf16(x_t, w.xb, static_cast<int64_t>(Ri) * P, stream));
+    {
+        GemmEpilogue e;
+        e.out_f32 = 1; e.bias = W("img_in.b"); e.out0 = w.x; e.ld0 = H;
+        FF_TRY(gemm_bf16(w.xb, P, W("img_in.w"), P, Ri, H, P, e, stream));
+    }
+    {
+        GemmEpilogue e;
+        e.act = ACT_GELU; e.bias = W("txt_in.b"); e.out0 = w.txt1; e.ld0 = H;
+        FF_TRY(gemm_bf16(txt, c.txt_dim, W("txt_in.w"), c.txt_dim, Rt, H, c.txt_dim, e, stream));
+    }
+    {
+        GemmEpilogue e;
+        e.bias = W("txt_in2.b"); e.out0 = w.txth; e.ld0 = H;
+        FF_TRY(gemm_bf16(w.txt1, H, W("txt_in2.w"), H, Rt, H, H, e, stream));
+    }
+
+    LnModArgs la{};
+    la.x = w.x; la.ldx = H; la.out = w.h; la.ldo = H; la.rows = Ri; la.H = H;
+    la.rows_txt = 0; la.n_txt = 1; la.n_img = Ni; la.mods = w.mods; la.ld_mods = Wm;
+
+    QkNormRopeArgs qa{};
+    qa.qkv = w.qkv; qa.ld = 3 * H; qa.rows = Ri; qa.heads = c.heads; qa.head_dim = d;
+    qa.rows_txt = 0; qa.n_img = Ni; qa.grid_f = c.grid_f; qa.grid_h = c.grid_h; qa.grid_w = c.grid_w;
+    qa.axes0 = c.rope_axes[0]; qa.axes1 = c.rope_axes[1]; qa.axes2 = c.rope_axes[2]; qa.theta = c.rope_theta;
+    qa.col[0] = 0; qa.col[1] = H; qa.rope = 1;
+
+    __nv_bfloat16* qc = w.qkv;   // cross-attention queries reuse the QKV buffer ([Ri, H])
+    for (int l = 0; l < L; ++l) {
+        const std::string p = "blocks." + std::to_string(l) + ".";
+        const int base = l * 6 * H;
+        // self-attention
+        la.aff_w = la.aff_b = nullptr;
+        la.shift_txt = la.shift_img = base;
+        la.scale_txt = la.scale_img = base + H;
+        FF_TRY(ln_modulate(la, stream));
+        {
+            GemmEpilogue e;
+            e.bias = W(p + "qkv.b"); e.out0 = w.qkv; e.ld0 = 3 * H;
+            FF_TRY(gemm_bf16(w.h, H, W(p + "qkv.w"), H, Ri, 3 * H, H, e, stream));
+        }
+        qa.qkv = w.qkv; qa.ld = 3 * H; qa.rows = Ri; qa.col[1] = H; qa.rope = 1;
+        qa.q_scale_txt = qa.q_scale_img = W(p + "q_norm.scale");
+        qa.k_scale_txt = qa.k_scale_img = W(p + "k_norm.scale");
+        FF_TRY(qk_norm_rope(qa, stream));
+        {
+            AttnSpec a{};
+            a.q[0] = AttnQuerySeg{nullptr, 0, 0, nullptr, 0};
+            a.q[1] = AttnQuerySeg{w.qkv, 3 * H, Ni, w.o, H};
+            a.kv[0] = AttnKvSeg{nullptr, 0, 0};
+            a.kv[1] = AttnKvSeg{w.qkv, 3 * H, Ni};
+            a.q_col = 0; a.k_col = H; a.v_col = 2 * H;
+            a.B = B; a.heads = c.heads; a.head_dim = d;
+            FF_TRY(attention_general(a, stream));
+        }
+        {
+            GemmEpilogue e;
+            e.epi = EPI_GATED_RESIDUAL; e.bias = W(p + "proj.b");
+            e.resid = w.x; e.ld_resid = H;
+            e.gate = w.mods + base + 2 * H; e.ld_gate = Wm; e.rows_per_sample = Ni;
+            FF_TRY(gemm_bf16(w.o, H, W(p + "proj.w"), H, Ri, H, H, e, stream));
+        }
+        // cross-attention to the text
+        la.aff_w = W(p + "cross_norm.scale");
+        la.aff_b = W(p + "cross_norm.b");
+        FF_TRY(ln_modulate(la, stream));
+        {
+            GemmEpilogue e;
+            e.bias = W(p + "cross_q.b"); e.out0 = qc; e.ld0 = H;
+            FF_TRY(gemm_bf16(w.h, H, W(p + "cross_q.w"), H, Ri, H, H, e, stream));
+        }
+        {
+            GemmEpilogue e;
+            e.bias = W(p + "cross_kv.b"); e.out0 = w.kvc; e.ld0 = 2 * H;
+            FF_TRY(gemm_bf16(w.txth, H, W(p + "cross_kv.w"), H, Rt, 2 * H, H, e, stream));
+        }
+        QkNormRopeArgs cq = qa;
+        cq.qkv = qc; cq.ld = H; cq.rows = Ri; cq.col[0] = 0; cq.col[1] = -1; cq.rope = 0;
+        cq.q_scale_txt = cq.q_scale_img = W(p + "cross_q_norm.scale");
+        FF_TRY(qk_norm_rope(cq, stream));
+        QkNormRopeArgs ck = cq;
+        ck.qkv = w.kvc; ck.ld = 2 * H; ck.rows = Rt;
+        ck.q_scale_txt = ck.q_scale_img = W(p + "cross_k_norm.scale");
+        FF_TRY(qk_norm_rope(ck, stream));
+        {
+            AttnSpec a{};
+            a.q[0] = AttnQuerySeg{nullptr, 0, 0, nullptr, 0};
+            a.q[1] = AttnQuerySeg{qc, H, Ni, w.o, H};
+            a.kv[0] = AttnKvSeg{w.kvc, 2 * H, Nt};
+            a.kv[1] = AttnKvSeg{nullptr, 0, 0};
+            a.q_col = 0; a.k_col = 0; a.v_col = H;
+            a.B = B; a.heads = c.heads; a.head_dim = d;
+            FF_TRY(attention_general(a, stream));
+        }
+        {
+            GemmEpilogue e;   // plain residual: no gate on the cross-attention branch
+            e.epi = EPI_GATED_RESIDUAL; e.bias = W(p + "cross_proj.b");
+            e.resid = w.x; e.ld_resid = H; e.gate = nullptr; e.rows_per_sample = Ni;
+            FF_TRY(gemm_bf16(w.o, H, W(p + "cross_proj.w"), H, Ri, H, H, e, stream));
+        }
+        // FFN
+        la.aff_w = la.aff_b = nullptr;
+        la.shift_txt = la.shift_img = base + 3 * H;
+        la.scale_txt = la.scale_img = base + 4 * H;
+        FF_TRY(ln_modulate(la, stream));
+        {
+            GemmEpilogue e;
+            e.act = ACT_GELU; e.bias = W(p + "mlp1.b"); e.out0 = w.u; e.ld0 = F;
+            FF_TRY(gemm_bf16(w.h, H, W(p + "mlp1.w"), H, Ri, F, H, e, stream));
+        }
+        {
+            GemmEpilogue e;
+            e.epi = EPI_GATED_RESIDUAL; e.bias = W(p + "mlp2.b");
+            e.resid = w.x; e.ld_resid = H;
+            e.gate = w.mods + base + 5 * H; e.ld_gate = Wm; e.rows_per_sample = Ni;
+            FF_TRY(gemm_bf16(w.u, F, W(p + "mlp2.w"), F, Ri, H, F, e, stream));
+        }
+    }
+    // final layer
+    la.aff_w = la.aff_b = nullptr;
+    la.shift_txt = la.shift_img = L * 6 * H;
+    la.scale_txt = la.scale_img = L * 6 * H + H;
+    FF_TRY(ln_modulate(la, stream));
+    GemmEpilogue e;
+    e.out_f32 = 1; e.bias = W("final.b"); e.out0 = v_out; e.ld0 = P;
+    return gemm_bf16(w.h, H, W("final.w"), H, Ri, P, H, e, stream);
+}
 
 }  // namespace
 }  // namespace ff
@@ -146,7 +360,7 @@ int ff_dit_weight_layout(const ff_dit_config* cfg, ff_tensor_desc* out, int capa
     using namespace ff;
     FF_TRY(validate(cfg));
     if (!count || !total_elems) return set_error(FF_ERR_INVALID_ARG, "count/total_elems is null");
-    const std::vector<Spec> s = specs(*cfg);
+    const std::vector<Spec> s = specs_for(*cfg);
     int64_t off = 0;
     for (size_t i = 0; i < s.size(); ++i) {
         const int64_t n = s[i].ndim == 2 ? s[i].s0 * s[i].s1 : s[i].s0;
@@ -173,9 +387,10 @@ int ff_dit_create(const ff_dit_config* cfg, const void* weights_dev, ff_dit** ou
     ff_dit* m = new ff_dit();
     m->cfg = *cfg;
     m->w = static_cast<const __nv_bfloat16*>(weights_dev);
-    m->mod_width = mod_width(*cfg);
+    m->mod_width = cfg->arch == FF_ARCH_WAN ? static_cast<int64_t>(cfg->n_double) * 6 * cfg->hidden + 2 * cfg->hidden
+                                            : mod_width(*cfg);
     int64_t off = 0;
-    for (const Spec& s : specs(*cfg)) {
+    for (const Spec& s : specs_for(*cfg)) {
         m->off[s.name] = off;
         const int64_t n = s.ndim == 2 ? s.s0 * s.s1 : s.s0;
         off += (n + 63) / 64 * 64;
@@ -209,6 +424,7 @@ int ff_dit_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, c
     const Workspace w = plan(c, B, static_cast<uint8_t*>(ws));
     if (ws_bytes < w.bytes) return set_error(FF_ERR_WORKSPACE, "workspace %zu B < %zu B needed", ws_bytes, w.bytes);
 
+    if (c.arch == FF_ARCH_WAN) return wan_velocity(m, B, x_t, txt, t, v_out, w, stream);
     const int H = c.hidden, F = c.mlp, P = c.patch_dim, d = c.head_dim;
     const int Nt = c.n_txt, Ni = c.grid_f * c.grid_h * c.grid_w;
     const int Rt = B * Nt, Ri = B * Ni, R = Rt + Ri;
@@ -250,6 +466,7 @@ int ff_dit_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, c
     qa.qkv = w.qkv; qa.ld = 3 * H; qa.rows = R; qa.heads = c.heads; qa.head_dim = d;
     qa.rows_txt = Rt; qa.n_img = Ni; qa.grid_f = c.grid_f; qa.grid_h = c.grid_h; qa.grid_w = c.grid_w;
     qa.axes0 = c.rope_axes[0]; qa.axes1 = c.rope_axes[1]; qa.axes2 = c.rope_axes[2]; qa.theta = c.rope_theta;
+    qa.col[0] = 0; qa.col[1] = H; qa.rope = 1;
 
     LnModArgs la{};
     la.x = w.x; la.ldx = H; la.out = w.h; la.ldo = H; la.rows = R; la.H = H;

@@ -53,9 +53,23 @@ __global__ void __launch_bounds__(256) ln_modulate_kernel(LnModArgs a) {
         q += (d0 * d0 + d1 * d1) + (d2 * d2 + d3 * d3);
     }
     const float rstd = rsqrtf(warp_sum(q) / a.H + kLnEps);
+    uint2* out = reinterpret_cast<uint2*>(a.out + static_cast<int64_t>(row) * a.ldo);
+    if (a.aff_w) {
+        // affine LayerNorm: LN(x) w + b
+        const uint2* w2 = reinterpret_cast<const uint2*>(a.aff_w);
+        const uint2* b2 = reinterpret_cast<const uint2*>(a.aff_b);
+        for (int i = lane; i < nv; i += 32) {
+            const float4 v = x[i];
+            const uint2 wu = w2[i], bu = b2[i];
+            const float2 w0 = unpack_bf16x2(wu.x), w1 = unpack_bf16x2(wu.y);
+            const float2 b0 = unpack_bf16x2(bu.x), b1 = unpack_bf16x2(bu.y);
+            out[i] = make_uint2(pack_bf16x2((v.x - mean) * rstd * w0.x + b0.x, (v.y - mean) * rstd * w0.y + b0.y),
+                                pack_bf16x2((v.z - mean) * rstd * w1.x + b1.x, (v.w - mean) * rstd * w1.y + b1.y));
+        }
+        return;
+    }
     const float4* shift = reinterpret_cast<const float4*>(a.mods + static_cast<int64_t>(b) * a.ld_mods + sh);
     const float4* scale = reinterpret_cast<const float4*>(a.mods + static_cast<int64_t>(b) * a.ld_mods + sc);
-    uint2* out = reinterpret_cast<uint2*>(a.out + static_cast<int64_t>(row) * a.ldo);
     for (int i = lane; i < nv; i += 32) {
         const float4 v = x[i];
         const float4 h = shift[i];
@@ -78,14 +92,13 @@ __global__ void __launch_bounds__(256) qk_norm_rope_kernel(QkNormRopeArgs a) {
     const int row = static_cast<int>(gw / a.heads);
     const int head = static_cast<int>(gw - static_cast<int64_t>(row) * a.heads);
     const bool img = row >= a.rows_txt;
-    const int H = a.heads * a.head_dim;
     const int c0 = lane * E;
     const __nv_bfloat16* qs = img ? a.q_scale_img : a.q_scale_txt;
     const __nv_bfloat16* ks = img ? a.k_scale_img : a.k_scale_txt;
 
     // rotation of this lane's pairs (identity for text tokens at position 0)
     float cs[E / 2], sn[E / 2];
-    if (img) {
+    if (img && a.rope) {
         const int n = (row - a.rows_txt) % a.n_img;
         const int hw = a.grid_h * a.grid_w;
         const float pos[3] = {static_cast<float>(n / hw), static_cast<float>((n / a.grid_w) % a.grid_h),
@@ -112,7 +125,8 @@ __global__ void __launch_bounds__(256) qk_norm_rope_kernel(QkNormRopeArgs a) {
 
 #pragma unroll
     for (int which = 0; which < 2; ++which) {
-        __nv_bfloat16* ptr = a.qkv + static_cast<int64_t>(row) * a.ld + which * H + head * a.head_dim + c0;
+        if (a.col[which] < 0) continue;
+        __nv_bfloat16* ptr = a.qkv + static_cast<int64_t>(row) * a.ld + a.col[which] + head * a.head_dim + c0;
         const __nv_bfloat16* sc = (which == 0 ? qs : ks) + c0;
         float v[E];
         if (E == 4) {
@@ -140,6 +154,25 @@ __global__ void __launch_bounds__(256) qk_norm_rope_kernel(QkNormRopeArgs a) {
         } else {
             *reinterpret_cast<uint32_t*>(ptr) = pack_bf16x2(o[0], o[1 % E]);
         }
+    }
+}
+
+__global__ void wan_modulation_kernel(const float* e, const float* e0, const __nv_bfloat16* bias0, int64_t stride,
+                                      int L, const __nv_bfloat16* fbias, int H, float* mods, int64_t ld_mods) {
+    const int b = blockIdx.y;
+    const int64_t n = static_cast<int64_t>(L) * 6 * H + 2 * H;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        float v;
+        if (i < static_cast<int64_t>(L) * 6 * H) {
+            const int l = static_cast<int>(i / (6 * H));
+            const int j = static_cast<int>(i - static_cast<int64_t>(l) * 6 * H);
+            v = e0[static_cast<int64_t>(b) * 6 * H + j] + __bfloat162float(bias0[l * stride + j]);
+        } else {
+            const int j = static_cast<int>(i - static_cast<int64_t>(L) * 6 * H);
+            v = e[static_cast<int64_t>(b) * H + (j % H)] + __bfloat162float(fbias[j]);
+        }
+        mods[static_cast<int64_t>(b) * ld_mods + i] = v;
     }
 }
 
@@ -206,6 +239,14 @@ int f32_to_bf16(const float* in, __nv_bfloat16* out, int64_t n, cudaStream_t str
     f32_to_bf16_kernel<<<static_cast<unsigned>(grid), 256, 0, stream>>>(reinterpret_cast<const float4*>(in),
                                                                         reinterpret_cast<uint2*>(out), n4);
     return check_launch("f32_to_bf16_kernel");
+}
+
+int wan_modulation(const float* e, const float* e0, const __nv_bfloat16* bias0, int64_t stride, int L,
+                   const __nv_bfloat16* fbias, int B, int H, float* mods, int64_t ld_mods, cudaStream_t stream) {
+    const dim3 grid(64, B);
+    ProfScope prof(stream, "wan_modulation", 0.0, static_cast<double>(B) * (L * 6.0 * H + 2.0 * H) * 10.0);
+    wan_modulation_kernel<<<grid, 256, 0, stream>>>(e, e0, bias0, stride, L, fbias, H, mods, ld_mods);
+    return check_launch("wan_modulation_kernel");
 }
 
 }  // namespace ff

@@ -84,7 +84,8 @@ __device__ __forceinline__ void gated_load(const GemmEpilogue& e, int M, int row
         const int row = row0 + rs + 4 * j;
         if (row < M) {
             const int b = row / e.rows_per_sample;
-            R.g[j] = *reinterpret_cast<const float4*>(e.gate + static_cast<int64_t>(b) * e.ld_gate + col);
+            R.g[j] = e.gate ? *reinterpret_cast<const float4*>(e.gate + static_cast<int64_t>(b) * e.ld_gate + col)
+                            : make_float4(1.f, 1.f, 1.f, 1.f);
             R.x[j] = *reinterpret_cast<const float4*>(e.resid + static_cast<int64_t>(row) * e.ld_resid + col);
         }
     }
@@ -373,7 +374,7 @@ int gemm_bf16(const void* A, int64_t lda, const void* B, int64_t ldb, int M, int
                          (long long)lda, (long long)ldb);
     if (e.bias && !aligned16(e.bias)) return set_error(FF_ERR_INVALID_ARG, "gemm: bias not 16-byte aligned");
     if (e.epi == EPI_GATED_RESIDUAL) {
-        if (!e.resid || !e.gate || e.rows_per_sample <= 0 || !aligned16(e.resid) || !aligned16(e.gate) ||
+        if (!e.resid || e.rows_per_sample <= 0 || !aligned16(e.resid) || (e.gate && !aligned16(e.gate)) ||
             e.ld_resid % 4 || e.ld_gate % 4)
             return set_error(FF_ERR_INVALID_ARG, "gemm: bad gated-residual epilogue");
     } else {

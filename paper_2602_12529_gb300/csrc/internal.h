@@ -49,7 +49,8 @@ struct GemmEpilogue {
     int64_t ld1 = 0;
     int col1 = 0;
     int split_n = 1 << 30;
-    // EPI_GATED_RESIDUAL: resid[m, n] += gate[(m / rows_per_sample) * ld_gate + n] * (acc + bias)
+    // EPI_GATED_RESIDUAL: resid[m, n] += gate[(m / rows_per_sample) * ld_gate + n] * (acc + bias);
+    // gate == nullptr means a plain residual update (gate 1)
     float* resid = nullptr;
     int64_t ld_resid = 0;
     const float* gate = nullptr;
@@ -70,11 +71,15 @@ struct LnModArgs {
     int rows_txt, n_txt, n_img;        // segment split and tokens per sample
     const float* mods; int64_t ld_mods;
     int shift_txt, scale_txt, shift_img, scale_img;  // column offsets into mods
+    // affine LayerNorm instead of modulation when aff_w is set: LN(x) w + b
+    const __nv_bfloat16* aff_w = nullptr;
+    const __nv_bfloat16* aff_b = nullptr;
 };
 int ln_modulate(const LnModArgs& a, cudaStream_t stream);
 
-// In-place per-head RMSNorm of q and k plus RoPE on a bf16 qkv buffer
-// [rows, ld] with q at column 0, k at column H.
+// In-place per-head RMSNorm plus (optionally) RoPE on up to two column
+// blocks ("q" at col[0], "k" at col[1]; -1 skips a block) of a bf16 buffer
+// [rows, ld].  Rows < rows_txt are text tokens (position 0: no rotation).
 struct QkNormRopeArgs {
     __nv_bfloat16* qkv; int64_t ld;
     int rows, heads, head_dim;
@@ -84,6 +89,8 @@ struct QkNormRopeArgs {
     float theta;
     const __nv_bfloat16* q_scale_txt; const __nv_bfloat16* k_scale_txt;
     const __nv_bfloat16* q_scale_img; const __nv_bfloat16* k_scale_img;
+    int col[2] = {0, -1};
+    int rope = 1;
 };
 int qk_norm_rope(const QkNormRopeArgs& a, cudaStream_t stream);
 
@@ -95,6 +102,26 @@ struct AttnSegment {
 };
 int attention(const AttnSegment& s0, const AttnSegment& s1, int B, int heads, int head_dim, int H,
               cudaStream_t stream);
+
+// General form: queries from up to two query segments, keys/values from up
+// to two key/value segments (concatenated per sample), head h of q / k / v
+// at columns q_col / k_col / v_col + h * d of its buffer.  Joint attention
+// uses the same buffers for both; cross-attention uses image queries and
+// text keys/values.
+struct AttnQuerySeg { const __nv_bfloat16* buf; int64_t ld; int n; __nv_bfloat16* out; int64_t ldo; };
+struct AttnKvSeg { const __nv_bfloat16* buf; int64_t ld; int n; };
+struct AttnSpec {
+    AttnQuerySeg q[2];
+    AttnKvSeg kv[2];
+    int q_col, k_col, v_col;
+    int B, heads, head_dim;
+};
+int attention_general(const AttnSpec& a, cudaStream_t stream);
+
+// mods[b, l*6H + j] = e0[b, j] + bias_l[j] (bias_l = bias0 + l*stride), and
+// mods[b, L*6H + j] = e[b, j % H] + fbias[j] for j < 2H (WAN modulation).
+int wan_modulation(const float* e, const float* e0, const __nv_bfloat16* bias0, int64_t stride, int L,
+                   const __nv_bfloat16* fbias, int B, int H, float* mods, int64_t ld_mods, cudaStream_t stream);
 
 int timestep_embed(const float* t, int B, int dim, __nv_bfloat16* out, cudaStream_t stream);
 int f32_to_bf16(const float* in, __nv_bfloat16* out, int64_t n, cudaStream_t stream);

@@ -16,7 +16,7 @@ FF_OK = 0
 FF_SDE_SAMPLE, FF_SDE_EVAL = 0, 1
 FF_LP_SUM, FF_LP_MEAN = 0, 1
 FF_SCHED_FLOW_SDE, FF_SCHED_DANCE_SDE, FF_SCHED_ODE = 0, 1, 2
-FF_ARCH_MMDIT = 0
+FF_ARCH_MMDIT, FF_ARCH_WAN = 0, 1
 FF_ACT_NONE, FF_ACT_GELU, FF_ACT_SILU = 0, 1, 2
 
 
@@ -150,7 +150,7 @@ def ff_grpo_loss_workspace_size(B: int, T: int) -> int:
 
 def make_config(cfg: dict) -> DitConfig:
     c = DitConfig()
-    c.arch = FF_ARCH_MMDIT
+    c.arch = FF_ARCH_WAN if cfg.get("arch", "mmdit") == "wan" else FF_ARCH_MMDIT
     for k in ("hidden", "heads", "head_dim", "mlp", "n_double", "n_single", "patch_dim", "txt_dim", "n_txt",
               "time_freq_dim"):
         setattr(c, k, int(cfg[k]))

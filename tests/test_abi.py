@@ -66,10 +66,8 @@ def test_schedule_rejects_bad_arguments(L):
 @pytest.mark.parametrize("name", list(synth.CONFIGS))
 def test_weight_layout_matches_oracle_parameters(L, name):
     cfg = synth.config(name)
-    if cfg["arch"] != "mmdit":
-        pytest.skip("layout covers the MMDiT family")
     specs, total = ffi.ff_dit_weight_layout(cfg)
-    want = odit.param_specs(cfg)
+    want = odit.wan_param_specs(cfg) if cfg["arch"] == "wan" else odit.param_specs(cfg)
     assert [(n, tuple(s)) for n, _, s in specs] == [(n, tuple(s)) for n, s in want]
     offs = [o for _, o, _ in specs]
     assert all(o % 64 == 0 for o in offs)

@@ -88,3 +88,31 @@ def test_velocity_flux_block_sampled_rows(cuda):
                              img_rows=rows)[0]
         err = rms_rel(v[b, rows], want)
         assert err <= V_TOL, (b, err)
+
+
+WAN_SMALL = dict(name="wan_small", arch="wan", hidden=256, heads=4, head_dim=64, mlp=512, n_double=2, n_single=0,
+                 patch_dim=64, txt_dim=256, n_txt=20, grid=(3, 4, 6), rope_axes=(24, 20, 20), rope_theta=10000.0,
+                 time_freq_dim=256, batch=2)
+
+
+@pytest.mark.parametrize("over", [{}, {"grid": (2, 5, 7), "n_txt": 13, "batch": 3, "n_double": 1}])
+def test_wan_velocity_small_full_parity(cuda, over):
+    cfg = dict(WAN_SMALL, **over)
+    model, W, x, txt, t, v = _setup(cfg, cuda)
+    want = odit.wan_velocity(odit.widen_params(W), cfg, x, odit.widen(txt), t.astype(np.float64))
+    err = rms_rel(v, want)
+    assert err <= V_TOL, err
+
+
+def test_wan_block_full_width_sampled_rows(cuda):
+    """One WAN block at full width (H 5120, 40 x 128 heads, MLP 13824) over
+    the full 21 x 30 x 52 = 32760-token video latent plus 512 text tokens."""
+    cfg = synth.config("wan_40", n_double=1)
+    model, W, x, txt, t, v = _setup(cfg, cuda)
+    P = odit.widen_params(W)
+    rng = np.random.default_rng(5)
+    rows = np.sort(rng.choice(synth.n_img(cfg), 24, replace=False))
+    rows[-1] = synth.n_img(cfg) - 1
+    want = odit.wan_velocity(P, cfg, x[:1], odit.widen(txt[:1]), t[:1].astype(np.float64), img_rows=rows)[0]
+    err = rms_rel(v[0, rows], want)
+    assert err <= V_TOL, err

@@ -5,10 +5,11 @@
   of each kind, and the Qwen-Image shape (256 + 4096 tokens, D_txt 3584) cut to
   one double block, compared with the fp64 oracle on sampled rows of sampled
   samples.
-* Full depth (24 and 60 blocks, weights drawn on the device): properties that
-  hold at any size -- finite output, identical results on a second call, and
-  every sample's velocity bit-identical to the one computed in a smaller batch
-  (samples never interact).
+* Full depth (24 and 60 MMDiT blocks; 40 WAN blocks over 32760 video tokens
+  at batch 2), weights drawn on the device: properties that hold at any size
+  -- finite output, identical results on a second call, and every sample's
+  velocity bit-identical to the one computed in a smaller batch (samples
+  never interact).
 """
 import numpy as np
 import pytest
@@ -92,11 +93,12 @@ def test_reduced_depth_sampled_rows(cuda, name, over, samples):
         assert err <= V_TOL, (b, err)
 
 
-@pytest.mark.parametrize("name,sub", [("flux_8d16s", 3), ("qwen_image_60d", 1)])
-def test_full_depth_properties(cuda, name, sub):
+@pytest.mark.parametrize("name,sub,batch", [("flux_8d16s", 3, None), ("qwen_image_60d", 1, None),
+                                            ("wan_40", 1, 2)])
+def test_full_depth_properties(cuda, name, sub, batch):
     import torch
     from paper_2602_12529_gb300 import ffi
-    cfg = synth.config(name)
+    cfg = synth.config(name) if batch is None else synth.config(name, batch=batch)
     blob = _blob_on_device(cfg, cuda)
     model = ffi.Dit(cfg, blob)
     B = cfg["batch"]

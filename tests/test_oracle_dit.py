@@ -186,3 +186,67 @@ def test_velocity_invariants():
     x2[:, [0, 5]] = x2[:, [5, 0]]
     v2 = dit.velocity(P, cfg, x2, txt, t)
     assert np.abs(v2[:, 0] - v[:, 5]).max() > 1e-6
+
+
+# ------------------------------------------------------------------ WAN
+
+WAN_TINY = dict(name="wan_pin", arch="wan", hidden=64, heads=2, head_dim=32, mlp=96, n_double=2, n_single=0,
+                patch_dim=16, txt_dim=40, n_txt=6, grid=(2, 3, 4), rope_axes=(12, 10, 10), rope_theta=10000.0,
+                time_freq_dim=32, batch=2)
+
+
+def _wan_params(cfg, seed=0):
+    return dit.widen_params(synth.weights(dit.wan_param_specs(cfg), seed=seed, std=0.1, bias_std=0.05,
+                                          scale_std=0.1))
+
+
+def test_wan_zero_modulation_and_cross_weights_give_closed_form():
+    # gates 0 and a zero cross-attention output projection make every block
+    # the identity, so v = final(LN-modulated embedding) with (shift, scale) = e + b_final
+    cfg = dict(WAN_TINY)
+    P = _wan_params(cfg)
+    P["mod.w"][:] = 0.0
+    P["mod.b"][:] = 0.0
+    for l in range(cfg["n_double"]):
+        P[f"blocks.{l}.mod.b"][:] = 0.0
+        P[f"blocks.{l}.cross_proj.w"][:] = 0.0
+        P[f"blocks.{l}.cross_proj.b"][:] = 0.0
+    x, txt, t = _inputs(cfg)
+    v = dit.wan_velocity(P, cfg, x, txt, t)
+    emb = dit.timestep_embedding(t, cfg["time_freq_dim"])
+    e = dit.linear(dit.silu(dit.linear(emb, P["t_embed.fc1.w"], P["t_embed.fc1.b"])), P["t_embed.fc2.w"],
+                   P["t_embed.fc2.b"])
+    H = cfg["hidden"]
+    for b in range(x.shape[0]):
+        xe = dit.linear(x[b], P["img_in.w"], P["img_in.b"])
+        h = dit.modulate(dit.layer_norm(xe), e[b] + P["final.mod.b"][:H], e[b] + P["final.mod.b"][H:])
+        np.testing.assert_allclose(v[b], dit.linear(h, P["final.w"], P["final.b"]), rtol=1e-12, atol=1e-14)
+
+
+def test_wan_invariants():
+    cfg = dict(WAN_TINY)
+    P = _wan_params(cfg)
+    x, txt, t = _inputs(cfg)
+    v = dit.wan_velocity(P, cfg, x, txt, t)
+    assert v.shape == x.shape
+    # text tokens enter only through (unrotated) cross-attention keys/values:
+    # their order does not matter
+    perm = np.random.default_rng(3).permutation(cfg["n_txt"])
+    np.testing.assert_allclose(dit.wan_velocity(P, cfg, x, txt[:, perm], t), v, rtol=1e-11, atol=1e-13)
+    v1 = dit.wan_velocity(P, cfg, x[1:], txt[1:], t[1:])
+    np.testing.assert_allclose(v1[0], v[1], rtol=1e-12, atol=1e-14)
+    rows = np.array([1, 13, 23])
+    np.testing.assert_allclose(dit.wan_velocity(P, cfg, x, txt, t, img_rows=rows), v[:, rows], rtol=1e-12,
+                               atol=1e-14)
+    # the frame axis is live: swapping two frames' tokens changes v
+    x2 = x.copy()
+    x2[:, [0, 12]] = x2[:, [12, 0]]
+    assert np.abs(dit.wan_velocity(P, cfg, x2, txt, t)[:, 0] - v[:, 12]).max() > 1e-6
+
+
+def test_wan_param_count():
+    c = synth.config("wan_40")
+    n = sum(int(np.prod(s)) for _, s in dit.wan_param_specs(c))
+    H, F = 5120, 13824
+    per_block = 8 * H * H + 2 * H * F
+    assert 40 * per_block < n < 40 * per_block * 1.02
