@@ -13,7 +13,7 @@
 //   mods  fp32 [B, W_mod]      all adaLN vectors (one GEMM per call)
 //   x     fp32 [R, H]          residual stream
 //   h     bf16 [R, H]          LN-modulated GEMM operand
-//   qkv   bf16 [R, 3H]         q | k | v (RMSNorm + RoPE applied in place)
+//   qkv   bf16 [R, 3H]         q | k | v (q, k RMSNorm'd and rotated by the QKV GEMM epilogue)
 //   o     bf16 [R, H]          attention output (double-stream blocks)
 //   u     bf16 [R, H + F]      MLP hidden [R, F] (double) or [attn | GELU(mlp)] (single)
 #include <string.h>
@@ -143,6 +143,7 @@ struct Workspace {
     // WAN only
     float *e, *e0;
     __nv_bfloat16 *txt1, *txth, *kvc;
+    float2* rope;   // cos / sin table of every rotation angle
     size_t bytes;
 };
 
@@ -167,6 +168,8 @@ Workspace plan(const ff_dit_config& c, int B, uint8_t* base) {
     w.qkv = reinterpret_cast<__nv_bfloat16*>(take(R * 3 * H * 2));
     w.o = reinterpret_cast<__nv_bfloat16*>(take(R * H * 2));
     w.u = reinterpret_cast<__nv_bfloat16*>(take(R * (H + F) * 2));
+    w.rope = reinterpret_cast<float2*>(take(static_cast<size_t>(rope_table_size(
+        c.grid_f, c.grid_h, c.grid_w, c.rope_axes[0], c.rope_axes[1], c.rope_axes[2])) * sizeof(float2)));
     if (wan) {
         w.e = reinterpret_cast<float*>(take(B * H * 4));
         w.e0 = reinterpret_cast<float*>(take(B * 6 * H * 4));
@@ -176,6 +179,24 @@ Workspace plan(const ff_dit_config& c, int B, uint8_t* base) {
     }
     w.bytes = o;
     return w;
+}
+
+// Fused per-head RMSNorm (+ RoPE when table is set) of the q | k columns.
+void set_qk_norm(GemmEpilogue& e, const ff_dit_config& c, int qk_cols, const __nv_bfloat16* qs,
+                 const __nv_bfloat16* ks, const float2* table, int rope_row0) {
+    e.qk_cols = qk_cols;
+    e.head_dim = c.head_dim;
+    e.q_scale = qs;
+    e.k_scale = ks;
+    e.rope_cs = table;
+    e.rope_row0 = rope_row0;
+    e.n_img = c.grid_f * c.grid_h * c.grid_w;
+    e.grid_f = c.grid_f;
+    e.grid_h = c.grid_h;
+    e.grid_w = c.grid_w;
+    e.axes0 = c.rope_axes[0];
+    e.axes1 = c.rope_axes[1];
+    e.axes2 = c.rope_axes[2];
 }
 
 #define FF_TRY(expr)                \
@@ -196,7 +217,9 @@ int wan_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, cons
     const int64_t Wm = m->mod_width;
     auto W = [&](const std::string& n) { return m->w + m->off.at(n); };
 
-    // timestep embedding e (fp32), SiLU(e) (bf16), e0 = SiLU(e) W_mod^T + b, per-block modulation
+    // rotation table; timestep embedding e (fp32), SiLU(e) (bf16), e0 = SiLU(e) W_mod^T + b; per-block modulation
+    FF_TRY(rope_table(w.rope, c.grid_f, c.grid_h, c.grid_w, c.rope_axes[0], c.rope_axes[1], c.rope_axes[2],
+                      c.rope_theta, stream));
     FF_TRY(timestep_embed(t, B, c.time_freq_dim, w.temb, stream));
     {
         GemmEpilogue e;
@@ -243,11 +266,6 @@ int wan_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, cons
     la.x = w.x; la.ldx = H; la.out = w.h; la.ldo = H; la.rows = Ri; la.H = H;
     la.rows_txt = 0; la.n_txt = 1; la.n_img = Ni; la.mods = w.mods; la.ld_mods = Wm;
 
-    QkNormRopeArgs qa{};
-    qa.qkv = w.qkv; qa.ld = 3 * H; qa.rows = Ri; qa.heads = c.heads; qa.head_dim = d;
-    qa.rows_txt = 0; qa.n_img = Ni; qa.grid_f = c.grid_f; qa.grid_h = c.grid_h; qa.grid_w = c.grid_w;
-    qa.axes0 = c.rope_axes[0]; qa.axes1 = c.rope_axes[1]; qa.axes2 = c.rope_axes[2]; qa.theta = c.rope_theta;
-    qa.col[0] = 0; qa.col[1] = H; qa.rope = 1;
 
     __nv_bfloat16* qc = w.qkv;   // cross-attention queries reuse the QKV buffer ([Ri, H])
     for (int l = 0; l < L; ++l) {
@@ -261,12 +279,9 @@ int wan_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, cons
         {
             GemmEpilogue e;
             e.bias = W(p + "qkv.b"); e.out0 = w.qkv; e.ld0 = 3 * H;
+            set_qk_norm(e, c, 2 * H, W(p + "q_norm.scale"), W(p + "k_norm.scale"), w.rope, 0);
             FF_TRY(gemm_bf16(w.h, H, W(p + "qkv.w"), H, Ri, 3 * H, H, e, stream));
         }
-        qa.qkv = w.qkv; qa.ld = 3 * H; qa.rows = Ri; qa.col[1] = H; qa.rope = 1;
-        qa.q_scale_txt = qa.q_scale_img = W(p + "q_norm.scale");
-        qa.k_scale_txt = qa.k_scale_img = W(p + "k_norm.scale");
-        FF_TRY(qk_norm_rope(qa, stream));
         {
             AttnSpec a{};
             a.q[0] = AttnQuerySeg{nullptr, 0, 0, nullptr, 0};
@@ -289,23 +304,17 @@ int wan_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, cons
         la.aff_b = W(p + "cross_norm.b");
         FF_TRY(ln_modulate(la, stream));
         {
-            GemmEpilogue e;
+            GemmEpilogue e;   // cross q with its RMSNorm fused (no rotation)
             e.bias = W(p + "cross_q.b"); e.out0 = qc; e.ld0 = H;
+            set_qk_norm(e, c, H, W(p + "cross_q_norm.scale"), W(p + "cross_q_norm.scale"), nullptr, 0);
             FF_TRY(gemm_bf16(w.h, H, W(p + "cross_q.w"), H, Ri, H, H, e, stream));
         }
         {
-            GemmEpilogue e;
+            GemmEpilogue e;   // cross k | v of the text, RMSNorm on k fused
             e.bias = W(p + "cross_kv.b"); e.out0 = w.kvc; e.ld0 = 2 * H;
+            set_qk_norm(e, c, H, W(p + "cross_k_norm.scale"), W(p + "cross_k_norm.scale"), nullptr, 0);
             FF_TRY(gemm_bf16(w.txth, H, W(p + "cross_kv.w"), H, Rt, 2 * H, H, e, stream));
         }
-        QkNormRopeArgs cq = qa;
-        cq.qkv = qc; cq.ld = H; cq.rows = Ri; cq.col[0] = 0; cq.col[1] = -1; cq.rope = 0;
-        cq.q_scale_txt = cq.q_scale_img = W(p + "cross_q_norm.scale");
-        FF_TRY(qk_norm_rope(cq, stream));
-        QkNormRopeArgs ck = cq;
-        ck.qkv = w.kvc; ck.ld = 2 * H; ck.rows = Rt;
-        ck.q_scale_txt = ck.q_scale_img = W(p + "cross_k_norm.scale");
-        FF_TRY(qk_norm_rope(ck, stream));
         {
             AttnSpec a{};
             a.q[0] = AttnQuerySeg{nullptr, 0, 0, nullptr, 0};
@@ -431,7 +440,9 @@ int ff_dit_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, c
     const int64_t Wm = m->mod_width;
     auto W = [&](const std::string& n) { return m->w + m->off.at(n); };
 
-    // ---- timestep embedding MLP and every adaLN vector
+    // ---- rotation table, timestep embedding MLP and every adaLN vector
+    FF_TRY(rope_table(w.rope, c.grid_f, c.grid_h, c.grid_w, c.rope_axes[0], c.rope_axes[1], c.rope_axes[2],
+                      c.rope_theta, stream));
     FF_TRY(timestep_embed(t, B, c.time_freq_dim, w.temb, stream));
     {
         GemmEpilogue e;
@@ -462,11 +473,6 @@ int ff_dit_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, c
         FF_TRY(gemm_bf16(txt, c.txt_dim, W("txt_in.w"), c.txt_dim, Rt, H, c.txt_dim, e, stream));
     }
 
-    QkNormRopeArgs qa{};
-    qa.qkv = w.qkv; qa.ld = 3 * H; qa.rows = R; qa.heads = c.heads; qa.head_dim = d;
-    qa.rows_txt = Rt; qa.n_img = Ni; qa.grid_f = c.grid_f; qa.grid_h = c.grid_h; qa.grid_w = c.grid_w;
-    qa.axes0 = c.rope_axes[0]; qa.axes1 = c.rope_axes[1]; qa.axes2 = c.rope_axes[2]; qa.theta = c.rope_theta;
-    qa.col[0] = 0; qa.col[1] = H; qa.rope = 1;
 
     LnModArgs la{};
     la.x = w.x; la.ldx = H; la.out = w.h; la.ldo = H; la.rows = R; la.H = H;
@@ -483,16 +489,14 @@ int ff_dit_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, c
         la.shift_txt = static_cast<int>(st[0].mod); la.scale_txt = static_cast<int>(st[0].mod + H);
         la.shift_img = static_cast<int>(st[1].mod); la.scale_img = static_cast<int>(st[1].mod + H);
         FF_TRY(ln_modulate(la, stream));
-        // QKV per stream
+        // QKV per stream, with q / k RMSNorm and RoPE fused into the epilogue
         for (const Stream& s : st) {
             const std::string p = pre + s.name + ".";
             GemmEpilogue e;
             e.bias = W(p + "qkv.b"); e.out0 = w.qkv + static_cast<int64_t>(s.row0) * 3 * H; e.ld0 = 3 * H;
+            set_qk_norm(e, c, 2 * H, W(p + "q_norm.scale"), W(p + "k_norm.scale"), s.row0 ? w.rope : nullptr, 0);
             FF_TRY(gemm_bf16(w.h + static_cast<int64_t>(s.row0) * H, H, W(p + "qkv.w"), H, s.rows, 3 * H, H, e, stream));
         }
-        qa.q_scale_txt = W(pre + "txt.q_norm.scale"); qa.k_scale_txt = W(pre + "txt.k_norm.scale");
-        qa.q_scale_img = W(pre + "img.q_norm.scale"); qa.k_scale_img = W(pre + "img.k_norm.scale");
-        FF_TRY(qk_norm_rope(qa, stream));
         {
             AttnSegment a0{w.qkv, 3 * H, w.o, H, Nt};
             AttnSegment a1{w.qkv + static_cast<int64_t>(Rt) * 3 * H, 3 * H, w.o + static_cast<int64_t>(Rt) * H, H, Ni};
@@ -541,11 +545,9 @@ int ff_dit_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, c
             e.out0 = w.qkv; e.ld0 = 3 * H;
             e.split_n = 3 * H; e.out1 = w.u; e.ld1 = H + F; e.col1 = H;
             e.act = ACT_GELU; e.act_from = 3 * H;
+            set_qk_norm(e, c, 2 * H, W(p + "q_norm.scale"), W(p + "k_norm.scale"), w.rope, Rt);
             FF_TRY(gemm_bf16(w.h, H, W(p + "linear1.w"), H, R, 3 * H + F, H, e, stream));
         }
-        qa.q_scale_txt = qa.q_scale_img = W(p + "q_norm.scale");
-        qa.k_scale_txt = qa.k_scale_img = W(p + "k_norm.scale");
-        FF_TRY(qk_norm_rope(qa, stream));
         {
             AttnSegment a0{w.qkv, 3 * H, w.u, H + F, Nt};
             AttnSegment a1{w.qkv + static_cast<int64_t>(Rt) * 3 * H, 3 * H, w.u + static_cast<int64_t>(Rt) * (H + F),

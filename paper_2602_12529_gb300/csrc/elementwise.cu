@@ -176,6 +176,26 @@ __global__ void wan_modulation_kernel(const float* e, const float* e0, const __n
     }
 }
 
+__global__ void rope_table_kernel(float2* table, int grid_f, int grid_h, int grid_w, int a0, int a1, int a2,
+                                  float theta, int n) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= n) return;
+    const int h0 = a0 / 2, h1 = a1 / 2, h2 = a2 / 2;
+    int pos, j, width;
+    if (i < grid_f * h0) {
+        pos = i / h0; j = i % h0; width = a0;
+    } else if (i < grid_f * h0 + grid_h * h1) {
+        const int k = i - grid_f * h0;
+        pos = k / h1; j = k % h1; width = a1;
+    } else {
+        const int k = i - grid_f * h0 - grid_h * h1;
+        pos = k / h2; j = k % h2; width = a2;
+    }
+    // angle in double: pos up to ~100 and the table feeds every rotation
+    const double ang = static_cast<double>(pos) * pow(static_cast<double>(theta), -2.0 * j / width);
+    table[i] = make_float2(static_cast<float>(cos(ang)), static_cast<float>(sin(ang)));
+}
+
 __global__ void timestep_embed_kernel(const float* t, int B, int dim, __nv_bfloat16* out) {
     const int i = blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= B * dim) return;
@@ -247,6 +267,19 @@ int wan_modulation(const float* e, const float* e0, const __nv_bfloat16* bias0, 
     ProfScope prof(stream, "wan_modulation", 0.0, static_cast<double>(B) * (L * 6.0 * H + 2.0 * H) * 10.0);
     wan_modulation_kernel<<<grid, 256, 0, stream>>>(e, e0, bias0, stride, L, fbias, H, mods, ld_mods);
     return check_launch("wan_modulation_kernel");
+}
+
+int rope_table_size(int grid_f, int grid_h, int grid_w, int a0, int a1, int a2) {
+    return grid_f * (a0 / 2) + grid_h * (a1 / 2) + grid_w * (a2 / 2);
+}
+
+int rope_table(float2* table, int grid_f, int grid_h, int grid_w, int a0, int a1, int a2, float theta,
+               cudaStream_t stream) {
+    const int n = rope_table_size(grid_f, grid_h, grid_w, a0, a1, a2);
+    if (n <= 0) return FF_OK;
+    ProfScope prof(stream, "rope_table", 0.0, 8.0 * n);
+    rope_table_kernel<<<(n + 255) / 256, 256, 0, stream>>>(table, grid_f, grid_h, grid_w, a0, a1, a2, theta, n);
+    return check_launch("rope_table_kernel");
 }
 
 }  // namespace ff

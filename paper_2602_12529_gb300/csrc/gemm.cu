@@ -112,6 +112,91 @@ __device__ __forceinline__ void gated_store(const GemmEpilogue& e, int M, int ro
     }
 }
 
+// Fused QKV tail: per-head RMSNorm of q / k (bias first, eps 1e-6, learned
+// scale), then RoPE from the cos/sin table, then the bf16 store.  Two passes
+// over each head's TMEM columns: the first sums squares, the second
+// normalises, rotates and stores.  The row is one token; its rotation pairs
+// (2j, 2j+1) lie inside each 32-column chunk.
+__device__ __forceinline__ void qk_norm_tile(const GemmEpilogue& e, int M, int row, int n0, uint32_t t_acc, int BN) {
+    const int d = e.head_dim;
+    const int half = e.qk_cols >> 1;
+    const bool rot = e.rope_cs != nullptr && row >= e.rope_row0;
+    const int h0 = e.axes0 >> 1, h1 = e.axes1 >> 1, h2 = e.axes2 >> 1;
+    // table offsets of this token's frame / row / column entries
+    int base0 = 0, base1 = 0, base2 = 0;
+    if (rot) {
+        const int n = (row - e.rope_row0) % e.n_img;
+        const int hw = e.grid_h * e.grid_w;
+        base0 = (n / hw) * h0;
+        base1 = e.grid_f * h0 + ((n / e.grid_w) % e.grid_h) * h1 - h0;
+        base2 = e.grid_f * h0 + e.grid_h * h1 + (n % e.grid_w) * h2 - h0 - h1;
+    }
+    for (int c0 = 0; c0 < BN; c0 += d) {
+        const int col = n0 + c0;                       // first column of this head
+        float ss = 0.f;
+        for (int c = 0; c < d; c += 32) {
+            uint32_t r[32];
+            tmem_ld_x32(t_acc + c0 + c, r);
+            tmem_ld_wait();
+            float v[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+            if (e.bias) {
+#pragma unroll
+                for (int j = 0; j < 4; ++j) bias_add8(v + 8 * j, e.bias + col + c + 8 * j);
+            }
+#pragma unroll
+            for (int i = 0; i < 32; ++i) ss = fmaf(v[i], v[i], ss);
+        }
+        const float rstd = rsqrtf(ss / d + 1e-6f);
+        const __nv_bfloat16* sc = col < half ? e.q_scale : e.k_scale;
+        for (int c = 0; c < d; c += 32) {
+            uint32_t r[32];
+            tmem_ld_x32(t_acc + c0 + c, r);
+            tmem_ld_wait();
+            float v[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+            if (e.bias) {
+#pragma unroll
+                for (int j = 0; j < 4; ++j) bias_add8(v + 8 * j, e.bias + col + c + 8 * j);
+            }
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const uint4 u = *reinterpret_cast<const uint4*>(sc + c + 8 * j);
+                const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const float2 f = unpack_bf16x2(w[i]);
+                    v[8 * j + 2 * i] *= rstd * f.x;
+                    v[8 * j + 2 * i + 1] *= rstd * f.y;
+                }
+            }
+            if (rot) {
+#pragma unroll
+                for (int i = 0; i < 16; ++i) {
+                    const int pair = (c >> 1) + i;
+                    const int idx = pair < h0 ? base0 + pair : (pair < h0 + h1 ? base1 + pair : base2 + pair);
+                    const float2 cs = e.rope_cs[idx];
+                    const float x0 = v[2 * i], x1 = v[2 * i + 1];
+                    v[2 * i] = x0 * cs.x - x1 * cs.y;
+                    v[2 * i + 1] = x0 * cs.y + x1 * cs.x;
+                }
+            }
+            if (row < M) {
+                uint4* o = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(e.out0) + static_cast<int64_t>(row) * e.ld0 +
+                                                    col + c);
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const float* s4 = v + 8 * j;
+                    o[j] = make_uint4(pack_bf16x2(s4[0], s4[1]), pack_bf16x2(s4[2], s4[3]), pack_bf16x2(s4[4], s4[5]),
+                                      pack_bf16x2(s4[6], s4[7]));
+                }
+            }
+        }
+    }
+}
+
 // Fused tail for one 32-column chunk of one output row held by this thread.
 __device__ __forceinline__ void epilogue_chunk(const GemmEpilogue& e, int M, int row, int n, float (&v)[32]) {
     if (e.bias) {
@@ -306,6 +391,8 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_const
                     gated_store(epi, M, row0, n, lane, R[c & 1], st);
                     __syncwarp();
                 }
+            } else if (epi.qk_cols > 0 && nb * BN < epi.qk_cols) {
+                qk_norm_tile(epi, M, row, nb * BN, t_acc, BN);
             } else {
 #pragma unroll 1
                 for (int c = 0; c < BN; c += 32) {
@@ -387,6 +474,14 @@ int gemm_bf16(const void* A, int64_t lda, const void* B, int64_t ldb, int M, int
         }
     }
     if (e.act != ACT_NONE && e.act_from % 32) return set_error(FF_ERR_INVALID_ARG, "gemm: act_from % 32 != 0");
+    if (e.qk_cols > 0) {
+        // whole heads per tile: the kernel must use 256-wide tiles with head_dim | 256 and qk_cols | 256
+        if (e.epi != EPI_STORE || e.out_f32 || (e.head_dim != 64 && e.head_dim != 128) || e.qk_cols % 256 ||
+            e.qk_cols > N || e.qk_cols > e.split_n || !e.q_scale || !e.k_scale || N <= 128 ||
+            (e.rope_cs && (e.n_img <= 0 || e.grid_h <= 0 || e.grid_w <= 0 || e.rope_row0 < 0)))
+            return set_error(FF_ERR_INVALID_ARG, "gemm: bad fused QK-norm epilogue");
+        return launch<256>(A, lda, B, ldb, M, N, K, e, stream);
+    }
     // narrow tiles when wide ones would leave most SMs idle (e.g. the
     // batch-row time-embedding GEMMs)
     const int64_t mblocks = (M + BM - 1) / BM;

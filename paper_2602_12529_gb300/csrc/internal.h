@@ -56,7 +56,26 @@ struct GemmEpilogue {
     const float* gate = nullptr;
     int64_t ld_gate = 0;
     int rows_per_sample = 1;
+    // Fused per-head RMSNorm (+ RoPE) of the q and k columns [0, qk_cols) of
+    // a bf16 EPI_STORE output (qk_cols = 2H, head width head_dim; q scale for
+    // columns < qk_cols / 2, k scale above).  Rows >= rope_row0 are latent
+    // tokens (row - rope_row0) % n_img of the (grid_f, grid_h, grid_w) grid
+    // and are rotated with the cos/sin table rope_cs (see rope_table); rows
+    // below rope_row0 are text tokens at position 0.
+    int qk_cols = 0;
+    int head_dim = 0;
+    const __nv_bfloat16* q_scale = nullptr;
+    const __nv_bfloat16* k_scale = nullptr;
+    const float2* rope_cs = nullptr;   // null: no rotation at all
+    int rope_row0 = 0, n_img = 1, grid_f = 1, grid_h = 1, grid_w = 1;
+    int axes0 = 0, axes1 = 0, axes2 = 0;
 };
+
+// cos / sin of every (axis, position, pair) rotation angle pos * theta^(-2j/a):
+// table[axis0: f * a0/2 + j | axis1: F a0/2 + r * a1/2 + j | axis2: ... + c * a2/2 + j]
+int rope_table_size(int grid_f, int grid_h, int grid_w, int a0, int a1, int a2);
+int rope_table(float2* table, int grid_f, int grid_h, int grid_w, int a0, int a1, int a2, float theta,
+               cudaStream_t stream);
 
 int gemm_bf16(const void* A, int64_t lda, const void* B, int64_t ldb, int M, int N, int K,
               const GemmEpilogue& epi, cudaStream_t stream);
