@@ -463,14 +463,13 @@ int ff_dit_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, c
     // ---- patch and text embeddings into the residual stream
     FF_TRY(f32_to_bf16(x_t, w.xb, static_cast<int64_t>(Ri) * P, stream));
     {
-        GemmEpilogue e;
-        e.out_f32 = 1; e.bias = W("img_in.b"); e.out0 = w.x + static_cast<int64_t>(Rt) * H; e.ld0 = H;
-        FF_TRY(gemm_bf16(w.xb, P, W("img_in.w"), P, Ri, H, P, e, stream));
-    }
-    {
-        GemmEpilogue e;
-        e.out_f32 = 1; e.bias = W("txt_in.b"); e.out0 = w.x; e.ld0 = H;
-        FF_TRY(gemm_bf16(txt, c.txt_dim, W("txt_in.w"), c.txt_dim, Rt, H, c.txt_dim, e, stream));
+        GemmArgs g[2];
+        g[0] = GemmArgs{w.xb, P, W("img_in.w"), P, Ri, H, P, GemmEpilogue{}};
+        g[0].epi.out_f32 = 1; g[0].epi.bias = W("img_in.b"); g[0].epi.out0 = w.x + static_cast<int64_t>(Rt) * H;
+        g[0].epi.ld0 = H;
+        g[1] = GemmArgs{txt, c.txt_dim, W("txt_in.w"), c.txt_dim, Rt, H, c.txt_dim, GemmEpilogue{}};
+        g[1].epi.out_f32 = 1; g[1].epi.bias = W("txt_in.b"); g[1].epi.out0 = w.x; g[1].epi.ld0 = H;
+        FF_TRY(gemm_bf16_group(g, 2, stream));
     }
 
 
@@ -489,13 +488,22 @@ int ff_dit_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, c
         la.shift_txt = static_cast<int>(st[0].mod); la.scale_txt = static_cast<int>(st[0].mod + H);
         la.shift_img = static_cast<int>(st[1].mod); la.scale_img = static_cast<int>(st[1].mod + H);
         FF_TRY(ln_modulate(la, stream));
-        // QKV per stream, with q / k RMSNorm and RoPE fused into the epilogue
-        for (const Stream& s : st) {
-            const std::string p = pre + s.name + ".";
-            GemmEpilogue e;
-            e.bias = W(p + "qkv.b"); e.out0 = w.qkv + static_cast<int64_t>(s.row0) * 3 * H; e.ld0 = 3 * H;
-            set_qk_norm(e, c, 2 * H, W(p + "q_norm.scale"), W(p + "k_norm.scale"), s.row0 ? w.rope : nullptr, 0);
-            FF_TRY(gemm_bf16(w.h + static_cast<int64_t>(s.row0) * H, H, W(p + "qkv.w"), H, s.rows, 3 * H, H, e, stream));
+        // Each GEMM below runs both streams in one launch: image problem
+        // first, the (smaller) text problem filling its tail.
+        const Stream* ord[2] = {&st[1], &st[0]};
+        // QKV, with q / k RMSNorm and RoPE fused into the epilogue
+        {
+            GemmArgs g[2];
+            for (int i = 0; i < 2; ++i) {
+                const Stream& s = *ord[i];
+                const std::string p = pre + s.name + ".";
+                g[i] = GemmArgs{w.h + static_cast<int64_t>(s.row0) * H, H, W(p + "qkv.w"), H, s.rows, 3 * H, H,
+                                GemmEpilogue{}};
+                GemmEpilogue& e = g[i].epi;
+                e.bias = W(p + "qkv.b"); e.out0 = w.qkv + static_cast<int64_t>(s.row0) * 3 * H; e.ld0 = 3 * H;
+                set_qk_norm(e, c, 2 * H, W(p + "q_norm.scale"), W(p + "k_norm.scale"), s.row0 ? w.rope : nullptr, 0);
+            }
+            FF_TRY(gemm_bf16_group(g, 2, stream));
         }
         {
             AttnSegment a0{w.qkv, 3 * H, w.o, H, Nt};
@@ -503,32 +511,50 @@ int ff_dit_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, c
             FF_TRY(attention(a0, a1, B, c.heads, d, H, stream));
         }
         // projection + gated residual (gate1)
-        for (const Stream& s : st) {
-            const std::string p = pre + s.name + ".";
-            GemmEpilogue e;
-            e.epi = EPI_GATED_RESIDUAL; e.bias = W(p + "proj.b");
-            e.resid = w.x + static_cast<int64_t>(s.row0) * H; e.ld_resid = H;
-            e.gate = w.mods + s.mod + 2 * H; e.ld_gate = Wm; e.rows_per_sample = s.tokens;
-            FF_TRY(gemm_bf16(w.o + static_cast<int64_t>(s.row0) * H, H, W(p + "proj.w"), H, s.rows, H, H, e, stream));
+        {
+            GemmArgs g[2];
+            for (int i = 0; i < 2; ++i) {
+                const Stream& s = *ord[i];
+                const std::string p = pre + s.name + ".";
+                g[i] = GemmArgs{w.o + static_cast<int64_t>(s.row0) * H, H, W(p + "proj.w"), H, s.rows, H, H,
+                                GemmEpilogue{}};
+                GemmEpilogue& e = g[i].epi;
+                e.epi = EPI_GATED_RESIDUAL; e.bias = W(p + "proj.b");
+                e.resid = w.x + static_cast<int64_t>(s.row0) * H; e.ld_resid = H;
+                e.gate = w.mods + s.mod + 2 * H; e.ld_gate = Wm; e.rows_per_sample = s.tokens;
+            }
+            FF_TRY(gemm_bf16_group(g, 2, stream));
         }
         // LN-modulate 2
         la.shift_txt = static_cast<int>(st[0].mod + 3 * H); la.scale_txt = static_cast<int>(st[0].mod + 4 * H);
         la.shift_img = static_cast<int>(st[1].mod + 3 * H); la.scale_img = static_cast<int>(st[1].mod + 4 * H);
         FF_TRY(ln_modulate(la, stream));
         // MLP
-        for (const Stream& s : st) {
-            const std::string p = pre + s.name + ".";
-            GemmEpilogue e;
-            e.act = ACT_GELU; e.bias = W(p + "mlp1.b"); e.out0 = w.u + static_cast<int64_t>(s.row0) * F; e.ld0 = F;
-            FF_TRY(gemm_bf16(w.h + static_cast<int64_t>(s.row0) * H, H, W(p + "mlp1.w"), H, s.rows, F, H, e, stream));
+        {
+            GemmArgs g[2];
+            for (int i = 0; i < 2; ++i) {
+                const Stream& s = *ord[i];
+                const std::string p = pre + s.name + ".";
+                g[i] = GemmArgs{w.h + static_cast<int64_t>(s.row0) * H, H, W(p + "mlp1.w"), H, s.rows, F, H,
+                                GemmEpilogue{}};
+                GemmEpilogue& e = g[i].epi;
+                e.act = ACT_GELU; e.bias = W(p + "mlp1.b"); e.out0 = w.u + static_cast<int64_t>(s.row0) * F; e.ld0 = F;
+            }
+            FF_TRY(gemm_bf16_group(g, 2, stream));
         }
-        for (const Stream& s : st) {
-            const std::string p = pre + s.name + ".";
-            GemmEpilogue e;
-            e.epi = EPI_GATED_RESIDUAL; e.bias = W(p + "mlp2.b");
-            e.resid = w.x + static_cast<int64_t>(s.row0) * H; e.ld_resid = H;
-            e.gate = w.mods + s.mod + 5 * H; e.ld_gate = Wm; e.rows_per_sample = s.tokens;
-            FF_TRY(gemm_bf16(w.u + static_cast<int64_t>(s.row0) * F, F, W(p + "mlp2.w"), F, s.rows, H, F, e, stream));
+        {
+            GemmArgs g[2];
+            for (int i = 0; i < 2; ++i) {
+                const Stream& s = *ord[i];
+                const std::string p = pre + s.name + ".";
+                g[i] = GemmArgs{w.u + static_cast<int64_t>(s.row0) * F, F, W(p + "mlp2.w"), F, s.rows, H, F,
+                                GemmEpilogue{}};
+                GemmEpilogue& e = g[i].epi;
+                e.epi = EPI_GATED_RESIDUAL; e.bias = W(p + "mlp2.b");
+                e.resid = w.x + static_cast<int64_t>(s.row0) * H; e.ld_resid = H;
+                e.gate = w.mods + s.mod + 5 * H; e.ld_gate = Wm; e.rows_per_sample = s.tokens;
+            }
+            FF_TRY(gemm_bf16_group(g, 2, stream));
         }
     }
 
@@ -554,15 +580,21 @@ int ff_dit_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, c
                            H + F, Ni};
             FF_TRY(attention(a0, a1, B, c.heads, d, H, stream));
         }
-        // linear2 + gated residual, per segment (sample index differs)
-        const Stream st[2] = {{"txt", 0, Rt, Nt, off}, {"img", Rt, Ri, Ni, off}};
-        for (const Stream& s : st) {
-            GemmEpilogue e;
-            e.epi = EPI_GATED_RESIDUAL; e.bias = W(p + "linear2.b");
-            e.resid = w.x + static_cast<int64_t>(s.row0) * H; e.ld_resid = H;
-            e.gate = w.mods + off + 2 * H; e.ld_gate = Wm; e.rows_per_sample = s.tokens;
-            FF_TRY(gemm_bf16(w.u + static_cast<int64_t>(s.row0) * (H + F), H + F, W(p + "linear2.w"), H + F, s.rows,
-                             H, H + F, e, stream));
+        // linear2 + gated residual: one launch, the two segments as two
+        // problems (the sample index of a row differs per segment)
+        {
+            const Stream st[2] = {{"img", Rt, Ri, Ni, off}, {"txt", 0, Rt, Nt, off}};
+            GemmArgs g[2];
+            for (int i = 0; i < 2; ++i) {
+                const Stream& s = st[i];
+                g[i] = GemmArgs{w.u + static_cast<int64_t>(s.row0) * (H + F), H + F, W(p + "linear2.w"), H + F,
+                                s.rows, H, H + F, GemmEpilogue{}};
+                GemmEpilogue& e = g[i].epi;
+                e.epi = EPI_GATED_RESIDUAL; e.bias = W(p + "linear2.b");
+                e.resid = w.x + static_cast<int64_t>(s.row0) * H; e.ld_resid = H;
+                e.gate = w.mods + off + 2 * H; e.ld_gate = Wm; e.rows_per_sample = s.tokens;
+            }
+            FF_TRY(gemm_bf16_group(g, 2, stream));
         }
     }
 

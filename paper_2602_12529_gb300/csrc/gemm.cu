@@ -236,10 +236,27 @@ __device__ __forceinline__ void epilogue_chunk(const GemmEpilogue& e, int M, int
     }
 }
 
+// Up to two independent GEMM problems share one persistent launch: the tile
+// space is problem 0's tiles followed by problem 1's, so a small problem
+// (the text stream of a double-stream block) fills the tail of a large one.
+struct GemmGroup {
+    int M[2], N[2], K[2];
+    int num_m[2], num_n[2];
+    int tiles0, tiles;
+    GemmEpilogue epi[2];
+};
+
+__device__ __forceinline__ void locate(const GemmGroup& g, int tile, int& pr, int& mb, int& nb) {
+    pr = tile < g.tiles0 ? 0 : 1;
+    const int local = pr ? tile - g.tiles0 : tile;
+    tile_coords(local, g.num_m[pr], g.num_n[pr], mb, nb);
+}
+
 template <int BN>
 __global__ void __launch_bounds__(kThreads, 1)
-gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b, int M,
-                    int N, int K, const GemmEpilogue epi, int* status) {
+gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_constant__ CUtensorMap tm_b0,
+                    const __grid_constant__ CUtensorMap tm_a1, const __grid_constant__ CUtensorMap tm_b1,
+                    const __grid_constant__ GemmGroup g, int* status) {
     using C = Cfg<BN>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -267,8 +284,12 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_const
         mbar_init(drain_bar, 1);
         *abort_flag = 0;
         fence_mbar_init();
-        prefetch_tmap(&tm_a);
-        prefetch_tmap(&tm_b);
+        prefetch_tmap(&tm_a0);
+        prefetch_tmap(&tm_b0);
+        if (g.tiles > g.tiles0) {
+            prefetch_tmap(&tm_a1);
+            prefetch_tmap(&tm_b1);
+        }
     }
     if (warp == 1) {
         tmem_alloc(tmem_slot, C::kTmemCols);
@@ -279,18 +300,16 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_const
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
 
-    const int num_m = (M + BM - 1) / BM;
-    const int num_n = (N + BN - 1) / BN;
-    const int num_tiles = num_m * num_n;
-    const int num_k = (K + BK - 1) / BK;
-
     if (warp == 0 && lane == 0) {
         // ---------------- TMA producer
         int stage = 0;
         uint32_t phase = 0;
-        for (int tile = blockIdx.x; tile < num_tiles && !*abort_flag; tile += gridDim.x) {
-            int mb, nb;
-            tile_coords(tile, num_m, num_n, mb, nb);
+        for (int tile = blockIdx.x; tile < g.tiles && !*abort_flag; tile += gridDim.x) {
+            int pr, mb, nb;
+            locate(g, tile, pr, mb, nb);
+            const CUtensorMap* ta = pr ? &tm_a1 : &tm_a0;
+            const CUtensorMap* tb = pr ? &tm_b1 : &tm_b0;
+            const int num_k = (g.K[pr] + BK - 1) / BK;
             for (int kb = 0; kb < num_k; ++kb) {
                 if (!mbar_wait(&empty_bar[stage], phase ^ 1)) {
                     report_status(status, kStatusWaitTimeout);
@@ -300,8 +319,8 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_const
                 uint8_t* sa = smem + stage * C::kStageBytes;
                 uint8_t* sb = sa + C::kABytes;
                 mbar_arrive_expect_tx(&full_bar[stage], C::kStageBytes);
-                tma_load_2d(sa, &tm_a, &full_bar[stage], kb * BK, mb * BM);
-                tma_load_2d(sb, &tm_b, &full_bar[stage], kb * BK, nb * BN);
+                tma_load_2d(sa, ta, &full_bar[stage], kb * BK, mb * BM);
+                tma_load_2d(sb, tb, &full_bar[stage], kb * BK, nb * BN);
                 if (++stage == C::kStages) { stage = 0; phase ^= 1; }
             }
         }
@@ -312,7 +331,9 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_const
         uint32_t phase = 0;
         int acc = 0;
         uint32_t acc_phase = 0;
-        for (int tile = blockIdx.x; tile < num_tiles && !*abort_flag; tile += gridDim.x) {
+        for (int tile = blockIdx.x; tile < g.tiles && !*abort_flag; tile += gridDim.x) {
+            const int pr = tile < g.tiles0 ? 0 : 1;
+            const int num_k = (g.K[pr] + BK - 1) / BK;
             if (!mbar_wait(&tempty_bar[acc], acc_phase ^ 1)) {
                 report_status(status, kStatusWaitTimeout);
                 *abort_flag = 1;
@@ -354,9 +375,11 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_const
         const int q = warp & 3;
         int acc = 0;
         uint32_t acc_phase = 0;
-        for (int tile = blockIdx.x; tile < num_tiles && !*abort_flag; tile += gridDim.x) {
-            int mb, nb;
-            tile_coords(tile, num_m, num_n, mb, nb);
+        for (int tile = blockIdx.x; tile < g.tiles && !*abort_flag; tile += gridDim.x) {
+            int pr, mb, nb;
+            locate(g, tile, pr, mb, nb);
+            const GemmEpilogue& epi = g.epi[pr];
+            const int M = g.M[pr], N = g.N[pr];
             if (!mbar_wait(&tfull_bar[acc], acc_phase)) {
                 report_status(status, kStatusWaitTimeout);
                 *abort_flag = 1;
@@ -429,36 +452,51 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_const
 }
 
 template <int BN>
-int launch(const void* A, int64_t lda, const void* B, int64_t ldb, int M, int N, int K, const GemmEpilogue& epi,
-           cudaStream_t stream) {
+int launch(const GemmArgs* p, int n, cudaStream_t stream) {
     using C = Cfg<BN>;
     if (cudaFuncSetAttribute(gemm_tcgen05_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes) !=
         cudaSuccess)
         return set_error(FF_ERR_CUDA, "gemm: cannot set shared memory size (%d B)", C::kSmemBytes);
-    CUtensorMap ta, tb;
-    int rc = make_tmap_bf16(&ta, A, M, K, lda, BM);
-    if (rc) return rc;
-    rc = make_tmap_bf16(&tb, B, N, K, ldb, BN);
-    if (rc) return rc;
-    const int tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN);
-    const int grid = tiles < num_sms() ? tiles : num_sms();
-    const double mn = static_cast<double>(M) * N;
-    const double out_bytes = epi.epi == EPI_GATED_RESIDUAL ? mn * 8.0 : mn * (epi.out_f32 ? 4.0 : 2.0);
-    ProfScope prof(stream, "gemm_bf16", 2.0 * mn * K, 2.0 * (static_cast<double>(M) + N) * K + out_bytes);
-    gemm_tcgen05_kernel<BN><<<grid, kThreads, C::kSmemBytes, stream>>>(ta, tb, M, N, K, epi, device_status_ptr());
+    CUtensorMap ta[2], tb[2];
+    GemmGroup g{};
+    double flops = 0.0, bytes = 0.0;
+    for (int i = 0; i < 2; ++i) {
+        const GemmArgs& a = p[i < n ? i : 0];
+        int rc = make_tmap_bf16(&ta[i], a.A, a.M, a.K, a.lda, BM);
+        if (rc) return rc;
+        rc = make_tmap_bf16(&tb[i], a.B, a.N, a.K, a.ldb, BN);
+        if (rc) return rc;
+        g.M[i] = a.M;
+        g.N[i] = a.N;
+        g.K[i] = a.K;
+        g.num_m[i] = (a.M + BM - 1) / BM;
+        g.num_n[i] = (a.N + BN - 1) / BN;
+        g.epi[i] = a.epi;
+        if (i < n) {
+            const double mn = static_cast<double>(a.M) * a.N;
+            flops += 2.0 * mn * a.K;
+            bytes += 2.0 * (static_cast<double>(a.M) + a.N) * a.K +
+                     (a.epi.epi == EPI_GATED_RESIDUAL ? mn * 8.0 : mn * (a.epi.out_f32 ? 4.0 : 2.0));
+        }
+    }
+    g.tiles0 = g.num_m[0] * g.num_n[0];
+    g.tiles = g.tiles0 + (n > 1 ? g.num_m[1] * g.num_n[1] : 0);
+    const int grid = g.tiles < num_sms() ? g.tiles : num_sms();
+    ProfScope prof(stream, "gemm_bf16", flops, bytes);
+    gemm_tcgen05_kernel<BN><<<grid, kThreads, C::kSmemBytes, stream>>>(ta[0], tb[0], ta[1], tb[1], g,
+                                                                       device_status_ptr());
     return check_launch("gemm_tcgen05_kernel");
 }
 
-}  // namespace
-
-int gemm_bf16(const void* A, int64_t lda, const void* B, int64_t ldb, int M, int N, int K, const GemmEpilogue& e,
-              cudaStream_t stream) {
-    if (!A || !B) return set_error(FF_ERR_INVALID_ARG, "gemm: null operand");
+int check_args(const GemmArgs& a) {
+    const GemmEpilogue& e = a.epi;
+    const int M = a.M, N = a.N, K = a.K;
+    if (!a.A || !a.B) return set_error(FF_ERR_INVALID_ARG, "gemm: null operand");
     if (M <= 0 || N <= 0 || K <= 0) return set_error(FF_ERR_INVALID_ARG, "gemm: bad shape %d x %d x %d", M, N, K);
     if (N % 32 != 0) return set_error(FF_ERR_UNSUPPORTED, "gemm: N=%d not a multiple of 32", N);
-    if (K % 8 != 0 || lda % 8 != 0 || ldb % 8 != 0 || lda < K || ldb < K)
+    if (K % 8 != 0 || a.lda % 8 != 0 || a.ldb % 8 != 0 || a.lda < K || a.ldb < K)
         return set_error(FF_ERR_UNSUPPORTED, "gemm: K/ld must be multiples of 8 (K=%d lda=%lld ldb=%lld)", K,
-                         (long long)lda, (long long)ldb);
+                         (long long)a.lda, (long long)a.ldb);
     if (e.bias && !aligned16(e.bias)) return set_error(FF_ERR_INVALID_ARG, "gemm: bias not 16-byte aligned");
     if (e.epi == EPI_GATED_RESIDUAL) {
         if (!e.resid || e.rows_per_sample <= 0 || !aligned16(e.resid) || (e.gate && !aligned16(e.gate)) ||
@@ -475,20 +513,44 @@ int gemm_bf16(const void* A, int64_t lda, const void* B, int64_t ldb, int M, int
     }
     if (e.act != ACT_NONE && e.act_from % 32) return set_error(FF_ERR_INVALID_ARG, "gemm: act_from % 32 != 0");
     if (e.qk_cols > 0) {
-        // whole heads per tile: the kernel must use 256-wide tiles with head_dim | 256 and qk_cols | 256
+        // whole heads per 256-wide tile: head_dim | 256 and qk_cols | 256
         if (e.epi != EPI_STORE || e.out_f32 || (e.head_dim != 64 && e.head_dim != 128) || e.qk_cols % 256 ||
             e.qk_cols > N || e.qk_cols > e.split_n || !e.q_scale || !e.k_scale || N <= 128 ||
             (e.rope_cs && (e.n_img <= 0 || e.grid_h <= 0 || e.grid_w <= 0 || e.rope_row0 < 0)))
             return set_error(FF_ERR_INVALID_ARG, "gemm: bad fused QK-norm epilogue");
-        return launch<256>(A, lda, B, ldb, M, N, K, e, stream);
     }
+    return FF_OK;
+}
+
+}  // namespace
+
+int gemm_bf16_group(const GemmArgs* p, int n, cudaStream_t stream) {
+    if (!p || n < 1 || n > 2) return set_error(FF_ERR_INVALID_ARG, "gemm: 1 or 2 problems per launch");
+    bool qk = false;
+    for (int i = 0; i < n; ++i) {
+        const int rc = check_args(p[i]);
+        if (rc) return rc;
+        qk = qk || p[i].epi.qk_cols > 0;
+    }
+    if (n == 2 || qk) {
+        for (int i = 0; i < n; ++i)
+            if (p[i].N <= 128) return set_error(FF_ERR_UNSUPPORTED, "gemm: grouped / fused problems need N > 128");
+        return launch<256>(p, n, stream);
+    }
+    const GemmArgs& a = p[0];
     // narrow tiles when wide ones would leave most SMs idle (e.g. the
     // batch-row time-embedding GEMMs)
-    const int64_t mblocks = (M + BM - 1) / BM;
-    const bool few = mblocks * ((N + 255) / 256) < num_sms() / 2;
-    if (N <= 64 || few) return launch<64>(A, lda, B, ldb, M, N, K, e, stream);
-    if (N <= 128) return launch<128>(A, lda, B, ldb, M, N, K, e, stream);
-    return launch<256>(A, lda, B, ldb, M, N, K, e, stream);
+    const int64_t mblocks = (a.M + BM - 1) / BM;
+    const bool few = mblocks * ((a.N + 255) / 256) < num_sms() / 2;
+    if (a.N <= 64 || few) return launch<64>(p, 1, stream);
+    if (a.N <= 128) return launch<128>(p, 1, stream);
+    return launch<256>(p, 1, stream);
+}
+
+int gemm_bf16(const void* A, int64_t lda, const void* B, int64_t ldb, int M, int N, int K, const GemmEpilogue& e,
+              cudaStream_t stream) {
+    const GemmArgs a{A, lda, B, ldb, M, N, K, e};
+    return gemm_bf16_group(&a, 1, stream);
 }
 
 }  // namespace ff

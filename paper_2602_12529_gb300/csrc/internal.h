@@ -80,6 +80,16 @@ int rope_table(float2* table, int grid_f, int grid_h, int grid_w, int a0, int a1
 int gemm_bf16(const void* A, int64_t lda, const void* B, int64_t ldb, int M, int N, int K,
               const GemmEpilogue& epi, cudaStream_t stream);
 
+// One or two independent GEMMs in a single persistent launch (tiles of the
+// first problem, then of the second).
+struct GemmArgs {
+    const void* A; int64_t lda;
+    const void* B; int64_t ldb;
+    int M, N, K;
+    GemmEpilogue epi;
+};
+int gemm_bf16_group(const GemmArgs* problems, int n, cudaStream_t stream);
+
 // ---- elementwise / row kernels -------------------------------------------
 // Row r of x (fp32 [rows, H]) belongs to segment txt if r < rows_txt, else img;
 // sample b = (r - seg_start) / tokens_per_sample.  out = LN(x) (1 + scale) + shift.
