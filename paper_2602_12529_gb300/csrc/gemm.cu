@@ -39,8 +39,8 @@ struct Cfg {
     static constexpr int kStageBytes = kABytes + kBBytes;
     static constexpr int kTmemCols = 2 * BN;
     static constexpr int kBarrierBytes = 256;
-    static constexpr int kStageFloats = 32 * 33;   // per epilogue warp: 32x32 fp32 transpose tile
-    static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + kBarrierBytes + 4 * kStageFloats * 4;
+    static constexpr int kResidBytes = BM * 32 * 4;   // one 128 x 32 fp32 residual chunk (two buffers)
+    static constexpr int kSmemBytes = kStages * kStageBytes + 2 * kResidBytes + 1024 + kBarrierBytes;
 };
 
 __device__ __forceinline__ void tile_coords(int tile, int num_m, int num_n, int& mb, int& nb) {
@@ -64,51 +64,38 @@ __device__ __forceinline__ void bias_add8(float* v, const __nv_bfloat16* b) {
     }
 }
 
-// Gated residual x[row, n..n+31] += gate[b(row), n..] * v for the 32 rows of
-// one epilogue warp.  The accumulator arrives one row per lane; it is
-// transposed through a padded 32x33 shared tile, and the global
-// read-modify-write runs on float4 row segments: lane = (row offset rs in
-// 0..3, column quad cq in 0..7), rows rs + 4j, so one warp instruction
-// covers 4 full 128-byte row segments.  The residual and gate of the next
-// chunk are loaded while the current one is finished (software pipeline).
-struct GatedRegs {
-    float4 x[8];
+// Gated residual, one 32-column chunk: x[row, n..n+31] += gate[b(row), n..] *
+// (acc + bias).  The residual chunk of the whole 128-row tile sits in shared
+// memory (loaded by TMA with 128-byte swizzle, 16-byte piece j of row r at
+// position j ^ (r % 8)); each thread updates its own row there, and the
+// chunk goes back by a TMA store.
+__device__ __forceinline__ void gated_update(const GemmEpilogue& e, int M, int row, int r, int n, const float (&v)[32],
+                                             uint8_t* rbuf) {
     float4 g[8];
-};
-
-__device__ __forceinline__ void gated_load(const GemmEpilogue& e, int M, int row0, int n, int lane, GatedRegs& R) {
-    const int col = n + 4 * (lane & 7);
-    const int rs = lane >> 3;
+    if (row < M) {
+        if (e.gate) {
+            const float4* gp = reinterpret_cast<const float4*>(e.gate + static_cast<int64_t>(row / e.rows_per_sample) *
+                                                                         e.ld_gate + n);
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-        const int row = row0 + rs + 4 * j;
-        if (row < M) {
-            const int b = row / e.rows_per_sample;
-            R.g[j] = e.gate ? *reinterpret_cast<const float4*>(e.gate + static_cast<int64_t>(b) * e.ld_gate + col)
-                            : make_float4(1.f, 1.f, 1.f, 1.f);
-            R.x[j] = *reinterpret_cast<const float4*>(e.resid + static_cast<int64_t>(row) * e.ld_resid + col);
+            for (int j = 0; j < 8; ++j) g[j] = gp[j];
+        } else {
+#pragma unroll
+            for (int j = 0; j < 8; ++j) g[j] = make_float4(1.f, 1.f, 1.f, 1.f);
         }
+    } else {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) g[j] = make_float4(0.f, 0.f, 0.f, 0.f);
     }
-}
-
-__device__ __forceinline__ void gated_store(const GemmEpilogue& e, int M, int row0, int n, int lane,
-                                            const GatedRegs& R, const float* st) {
-    const int cq = lane & 7;
-    const int rs = lane >> 3;
-    const int col = n + 4 * cq;
+    uint8_t* rowp = rbuf + r * 128;
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
-        const int r = rs + 4 * j;
-        const int row = row0 + r;
-        if (row < M) {
-            const float* a = st + r * 33 + 4 * cq;
-            float4 o = R.x[j];
-            o.x += R.g[j].x * a[0];
-            o.y += R.g[j].y * a[1];
-            o.z += R.g[j].z * a[2];
-            o.w += R.g[j].w * a[3];
-            *reinterpret_cast<float4*>(e.resid + static_cast<int64_t>(row) * e.ld_resid + col) = o;
-        }
+        float4* px = reinterpret_cast<float4*>(rowp + ((j ^ (r & 7)) << 4));
+        float4 x = *px;
+        x.x = fmaf(g[j].x, v[4 * j], x.x);
+        x.y = fmaf(g[j].y, v[4 * j + 1], x.y);
+        x.z = fmaf(g[j].z, v[4 * j + 2], x.z);
+        x.w = fmaf(g[j].w, v[4 * j + 3], x.w);
+        *px = x;
     }
 }
 
@@ -256,18 +243,21 @@ template <int BN>
 __global__ void __launch_bounds__(kThreads, 1)
 gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_constant__ CUtensorMap tm_b0,
                     const __grid_constant__ CUtensorMap tm_a1, const __grid_constant__ CUtensorMap tm_b1,
+                    const __grid_constant__ CUtensorMap tm_r0, const __grid_constant__ CUtensorMap tm_r1,
                     const __grid_constant__ GemmGroup g, int* status) {
     using C = Cfg<BN>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint64_t* full_bar = reinterpret_cast<uint64_t*>(smem + C::kStages * C::kStageBytes);
+    uint8_t* rbuf = smem + C::kStages * C::kStageBytes;            // [2][kResidBytes]
+    uint64_t* full_bar = reinterpret_cast<uint64_t*>(rbuf + 2 * C::kResidBytes);
     uint64_t* empty_bar = full_bar + C::kStages;
     uint64_t* tfull_bar = empty_bar + C::kStages;   // [2]
     uint64_t* tempty_bar = tfull_bar + 2;           // [2]
     uint64_t* drain_bar = tempty_bar + 2;           // [1]
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_bar + 1);
+    uint64_t* rfull_bar = drain_bar + 1;            // [2] residual chunk landed
+    uint64_t* rdone_bar = rfull_bar + 2;            // [2] all 128 epilogue threads updated the chunk
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(rdone_bar + 2);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-    float* stage_f = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(full_bar) + C::kBarrierBytes);
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -282,6 +272,10 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_cons
             mbar_init(&tempty_bar[a], 4);
         }
         mbar_init(drain_bar, 1);
+        mbar_init(&rfull_bar[0], 1);
+        mbar_init(&rfull_bar[1], 1);
+        mbar_init(&rdone_bar[0], 128);
+        mbar_init(&rdone_bar[1], 128);
         *abort_flag = 0;
         fence_mbar_init();
         prefetch_tmap(&tm_a0);
@@ -373,6 +367,8 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_cons
     } else if (warp >= 2) {
         // ---------------- epilogue (4 warps; warp w reads TMEM lanes 32*(w%4)..)
         const int q = warp & 3;
+        const bool leader = warp == 2 && lane == 0;     // issues the residual TMA traffic
+        uint32_t ruse[2] = {0, 0};                      // residual loads consumed per buffer
         int acc = 0;
         uint32_t acc_phase = 0;
         for (int tile = blockIdx.x; tile < g.tiles && !*abort_flag; tile += gridDim.x) {
@@ -380,53 +376,81 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_cons
             locate(g, tile, pr, mb, nb);
             const GemmEpilogue& epi = g.epi[pr];
             const int M = g.M[pr], N = g.N[pr];
+            const bool gated = epi.epi == EPI_GATED_RESIDUAL;
+            const CUtensorMap* tr = pr ? &tm_r1 : &tm_r0;
+            if (gated && leader) {
+                // the first two residual chunks of this tile, ahead of the accumulator
+                for (int c = 0; c < 2 && c < BN / 32; ++c) {
+                    bulk_wait_read<0>();
+                    mbar_arrive_expect_tx(&rfull_bar[c], C::kResidBytes);
+                    tma_load_2d(rbuf + c * C::kResidBytes, tr, &rfull_bar[c], nb * BN + c * 32, mb * BM);
+                }
+            }
             if (!mbar_wait(&tfull_bar[acc], acc_phase)) {
                 report_status(status, kStatusWaitTimeout);
                 *abort_flag = 1;
                 break;
             }
             tc_fence_after();
-            const int row = mb * BM + q * 32 + lane;
+            const int r = q * 32 + lane;                // row within the tile = TMEM lane
+            const int row = mb * BM + r;
             const uint32_t t_acc = tmem_base + static_cast<uint32_t>(acc * BN) + (static_cast<uint32_t>(q * 32) << 16);
-            if (epi.epi == EPI_GATED_RESIDUAL) {
-                float* st = stage_f + (warp - 2) * C::kStageFloats;
-                const int row0 = mb * BM + q * 32;
-                GatedRegs R[2];
-                gated_load(epi, M, row0, nb * BN, lane, R[0]);
-#pragma unroll
+            if (gated) {
+                bool ok = true;
                 for (int c = 0; c < BN / 32; ++c) {
                     const int n = nb * BN + c * 32;
-                    if (c + 1 < BN / 32 && n + 32 < N) gated_load(epi, M, row0, n + 32, lane, R[(c + 1) & 1]);
-                    uint32_t r[32];
-                    tmem_ld_x32(t_acc + c * 32, r);
+                    const int b = c & 1;
+                    uint32_t rr[32];
+                    tmem_ld_x32(t_acc + c * 32, rr);
                     tmem_ld_wait();
-                    if (n >= N) continue;
                     float v[32];
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+                    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(rr[i]);
                     if (epi.bias) {
 #pragma unroll
                         for (int j = 0; j < 4; ++j) bias_add8(v + 8 * j, epi.bias + n + 8 * j);
                     }
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) st[lane * 33 + i] = v[i];
-                    __syncwarp();
-                    gated_store(epi, M, row0, n, lane, R[c & 1], st);
-                    __syncwarp();
+                    if (!mbar_wait(&rfull_bar[b], ruse[b] & 1)) {
+                        report_status(status, kStatusWaitTimeout);
+                        *abort_flag = 1;
+                        ok = false;
+                    }
+                    if (ok) gated_update(epi, M, row, r, n, v, rbuf + b * C::kResidBytes);
+                    fence_proxy_async_smem();
+                    mbar_arrive(&rdone_bar[b]);
+                    // the leader stores the chunk once every thread has updated it
+                    // (an mbarrier, not bar.sync: a thread that gave up on a wait
+                    // must not be able to stall the others)
+                    if (leader && ok && !mbar_wait(&rdone_bar[b], ruse[b] & 1)) {
+                        report_status(status, kStatusWaitTimeout);
+                        *abort_flag = 1;
+                        ok = false;
+                    }
+                    ++ruse[b];
+                    if (leader && ok) {
+                        tma_store_2d(tr, rbuf + b * C::kResidBytes, n, mb * BM);
+                        bulk_commit();
+                        if (c + 2 < BN / 32) {
+                            bulk_wait_read<0>();
+                            mbar_arrive_expect_tx(&rfull_bar[b], C::kResidBytes);
+                            tma_load_2d(rbuf + b * C::kResidBytes, tr, &rfull_bar[b], n + 64, mb * BM);
+                        }
+                    }
                 }
+                if (!ok) break;
             } else if (epi.qk_cols > 0 && nb * BN < epi.qk_cols) {
                 qk_norm_tile(epi, M, row, nb * BN, t_acc, BN);
             } else {
 #pragma unroll 1
                 for (int c = 0; c < BN; c += 32) {
-                    uint32_t r[32];
-                    tmem_ld_x32(t_acc + c, r);
+                    uint32_t rr[32];
+                    tmem_ld_x32(t_acc + c, rr);
                     tmem_ld_wait();
                     const int n = nb * BN + c;
                     if (n >= N) continue;
                     float v[32];
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+                    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(rr[i]);
                     epilogue_chunk(epi, M, row, n, v);
                 }
             }
@@ -435,6 +459,7 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_cons
             if (lane == 0) mbar_arrive(&tempty_bar[acc]);
             if (++acc == 2) { acc = 0; acc_phase ^= 1; }
         }
+        if (leader) bulk_wait<0>();   // residual stores complete before the CTA's shared memory goes away
     }
 
     if (*abort_flag) {
@@ -457,7 +482,7 @@ int launch(const GemmArgs* p, int n, cudaStream_t stream) {
     if (cudaFuncSetAttribute(gemm_tcgen05_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes) !=
         cudaSuccess)
         return set_error(FF_ERR_CUDA, "gemm: cannot set shared memory size (%d B)", C::kSmemBytes);
-    CUtensorMap ta[2], tb[2];
+    CUtensorMap ta[2], tb[2], tr[2];
     GemmGroup g{};
     double flops = 0.0, bytes = 0.0;
     for (int i = 0; i < 2; ++i) {
@@ -466,6 +491,12 @@ int launch(const GemmArgs* p, int n, cudaStream_t stream) {
         if (rc) return rc;
         rc = make_tmap_bf16(&tb[i], a.B, a.N, a.K, a.ldb, BN);
         if (rc) return rc;
+        if (a.epi.epi == EPI_GATED_RESIDUAL) {
+            rc = make_tmap_f32_sw128(&tr[i], a.epi.resid, a.M, a.N, a.epi.ld_resid, BM);
+            if (rc) return rc;
+        } else {
+            tr[i] = ta[i];   // unused: the problem has no residual
+        }
         g.M[i] = a.M;
         g.N[i] = a.N;
         g.K[i] = a.K;
@@ -483,7 +514,10 @@ int launch(const GemmArgs* p, int n, cudaStream_t stream) {
     g.tiles = g.tiles0 + (n > 1 ? g.num_m[1] * g.num_n[1] : 0);
     const int grid = g.tiles < num_sms() ? g.tiles : num_sms();
     ProfScope prof(stream, "gemm_bf16", flops, bytes);
-    gemm_tcgen05_kernel<BN><<<grid, kThreads, C::kSmemBytes, stream>>>(ta[0], tb[0], ta[1], tb[1], g,
+    for (int i = 0; i < n; ++i)
+        if (p[i].epi.epi == EPI_GATED_RESIDUAL && p[i].N % BN)
+            return set_error(FF_ERR_UNSUPPORTED, "gemm: gated residual needs N (%d) to be a multiple of %d", p[i].N, BN);
+    gemm_tcgen05_kernel<BN><<<grid, kThreads, C::kSmemBytes, stream>>>(ta[0], tb[0], ta[1], tb[1], tr[0], tr[1], g,
                                                                        device_status_ptr());
     return check_launch("gemm_tcgen05_kernel");
 }

@@ -32,6 +32,8 @@ struct ProfScope {
 // 2-D bf16 row-major matrix [rows, cols] with leading dimension ld
 // (elements), box = box_rows x 64 columns, 128-byte swizzle, zero fill.
 int make_tmap_bf16(CUtensorMap* tm, const void* base, int64_t rows, int64_t cols, int64_t ld, int box_rows);
+// 2-D fp32 matrix, box = box_rows x 32 columns (128 bytes), 128-byte swizzle.
+int make_tmap_f32_sw128(CUtensorMap* tm, const void* base, int64_t rows, int64_t cols, int64_t ld, int box_rows);
 
 // ---- GEMM: D[M, N] = A[M, K] B[N, K]^T with a fused epilogue --------------
 enum GemmAct { ACT_NONE = 0, ACT_GELU = 1, ACT_SILU = 2 };
