@@ -223,22 +223,22 @@ int wan_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, cons
     FF_TRY(timestep_embed(t, B, c.time_freq_dim, w.temb, stream));
     {
         GemmEpilogue e;
-        e.act = ACT_SILU; e.bias = W("t_embed.fc1.b"); e.out0 = w.th; e.ld0 = H;
+        e.rows_gemv = 1; e.act = ACT_SILU; e.bias = W("t_embed.fc1.b"); e.out0 = w.th; e.ld0 = H;
         FF_TRY(gemm_bf16(w.temb, c.time_freq_dim, W("t_embed.fc1.w"), c.time_freq_dim, B, H, c.time_freq_dim, e, stream));
     }
     {
         GemmEpilogue e;
-        e.out_f32 = 1; e.bias = W("t_embed.fc2.b"); e.out0 = w.e; e.ld0 = H;
+        e.rows_gemv = 1; e.out_f32 = 1; e.bias = W("t_embed.fc2.b"); e.out0 = w.e; e.ld0 = H;
         FF_TRY(gemm_bf16(w.th, H, W("t_embed.fc2.w"), H, B, H, H, e, stream));
     }
     {
         GemmEpilogue e;
-        e.act = ACT_SILU; e.bias = W("t_embed.fc2.b"); e.out0 = w.tc; e.ld0 = H;
+        e.rows_gemv = 1; e.act = ACT_SILU; e.bias = W("t_embed.fc2.b"); e.out0 = w.tc; e.ld0 = H;
         FF_TRY(gemm_bf16(w.th, H, W("t_embed.fc2.w"), H, B, H, H, e, stream));
     }
     {
         GemmEpilogue e;
-        e.out_f32 = 1; e.bias = W("mod.b"); e.out0 = w.e0; e.ld0 = 6 * H;
+        e.rows_gemv = 1; e.out_f32 = 1; e.bias = W("mod.b"); e.out0 = w.e0; e.ld0 = 6 * H;
         FF_TRY(gemm_bf16(w.tc, H, W("mod.w"), H, B, 6 * H, H, e, stream));
     }
     const int64_t stride = L > 1 ? m->off.at("blocks.1.mod.b") - m->off.at("blocks.0.mod.b") : 0;
@@ -446,17 +446,17 @@ int ff_dit_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, c
     FF_TRY(timestep_embed(t, B, c.time_freq_dim, w.temb, stream));
     {
         GemmEpilogue e;
-        e.act = ACT_SILU; e.bias = W("t_embed.fc1.b"); e.out0 = w.th; e.ld0 = H;
+        e.rows_gemv = 1; e.act = ACT_SILU; e.bias = W("t_embed.fc1.b"); e.out0 = w.th; e.ld0 = H;
         FF_TRY(gemm_bf16(w.temb, c.time_freq_dim, W("t_embed.fc1.w"), c.time_freq_dim, B, H, c.time_freq_dim, e, stream));
     }
     {
         GemmEpilogue e;   // SiLU(c): only the modulation GEMM consumes c
-        e.act = ACT_SILU; e.bias = W("t_embed.fc2.b"); e.out0 = w.tc; e.ld0 = H;
+        e.rows_gemv = 1; e.act = ACT_SILU; e.bias = W("t_embed.fc2.b"); e.out0 = w.tc; e.ld0 = H;
         FF_TRY(gemm_bf16(w.th, H, W("t_embed.fc2.w"), H, B, H, H, e, stream));
     }
     {
         GemmEpilogue e;
-        e.out_f32 = 1; e.bias = W("mod.b"); e.out0 = w.mods; e.ld0 = Wm;
+        e.rows_gemv = 1; e.out_f32 = 1; e.bias = W("mod.b"); e.out0 = w.mods; e.ld0 = Wm;
         FF_TRY(gemm_bf16(w.tc, H, W("mod.w"), H, B, static_cast<int>(Wm), H, e, stream));
     }
 

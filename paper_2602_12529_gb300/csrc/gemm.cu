@@ -522,6 +522,138 @@ int launch(const GemmArgs* p, int n, cudaStream_t stream) {
     return check_launch("gemm_tcgen05_kernel");
 }
 
+// ---------------------------------------------------------------------------
+// Few-row GEMM (M <= 8: the per-sample time-embedding and modulation
+// products).  out[m, n] = act(A[m, :] . W[n, :] + bias[n]).  It is bound by
+// reading W once, so: A is staged in shared memory, each warp streams two W
+// rows with 16-byte loads (coalesced along K), keeps M accumulators per row
+// and reduces across lanes.  Persistent grid; columns are handed out in
+// groups of 16 per block.
+// ---------------------------------------------------------------------------
+constexpr int kGemvMaxRows = 8;
+constexpr int kGemvMaxK = 8192;
+constexpr int kGemvThreads = 256;
+
+constexpr int kGemvCols = 4;   // W rows (output columns) per warp
+
+template <int MR>
+__global__ void __launch_bounds__(kGemvThreads) gemv_rows_kernel(const __nv_bfloat16* A, int64_t lda, int M,
+                                                                 const __nv_bfloat16* W, int64_t ldw, int N, int K,
+                                                                 const GemmEpilogue e) {
+    extern __shared__ uint4 sA4[];   // [MR][K] bf16; rows >= M are zero
+    const int k8 = K / 8;
+    for (int i = threadIdx.x; i < MR * k8; i += kGemvThreads) {
+        const int m = i / k8, c = i - m * k8;
+        sA4[i] = m < M ? *reinterpret_cast<const uint4*>(A + static_cast<int64_t>(m) * lda + c * 8)
+                       : make_uint4(0u, 0u, 0u, 0u);
+    }
+    __syncthreads();
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    constexpr int kWarps = kGemvThreads / 32;
+    for (int n0 = (blockIdx.x * kWarps + warp) * kGemvCols; n0 < N; n0 += gridDim.x * kWarps * kGemvCols) {
+        float acc[kGemvCols][MR];
+#pragma unroll
+        for (int j = 0; j < kGemvCols; ++j)
+#pragma unroll
+            for (int m = 0; m < MR; ++m) acc[j][m] = 0.f;
+        const uint4* w[kGemvCols];
+#pragma unroll
+        for (int j = 0; j < kGemvCols; ++j)
+            w[j] = reinterpret_cast<const uint4*>(W + static_cast<int64_t>(min(n0 + j, N - 1)) * ldw);
+        // per lane: K chunks lane, lane + 32, ...; two chunks of every column
+        // in flight (8 independent 16-byte loads) before they are used
+        for (int c = lane; c < k8; c += 64) {
+            uint4 wv[2][kGemvCols];
+            const bool two = c + 32 < k8;
+#pragma unroll
+            for (int j = 0; j < kGemvCols; ++j) {
+                wv[0][j] = __ldcs(w[j] + c);
+                wv[1][j] = two ? __ldcs(w[j] + c + 32) : make_uint4(0u, 0u, 0u, 0u);
+            }
+#pragma unroll
+            for (int u = 0; u < 2; ++u) {
+                if (u == 1 && !two) break;
+#pragma unroll
+                for (int m = 0; m < MR; ++m) {
+                    const uint4 av = sA4[m * k8 + c + 32 * u];
+                    const uint32_t aw[4] = {av.x, av.y, av.z, av.w};
+#pragma unroll
+                    for (int j = 0; j < kGemvCols; ++j) {
+                        const uint32_t ww[4] = {wv[u][j].x, wv[u][j].y, wv[u][j].z, wv[u][j].w};
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) {
+                            const float2 a2 = unpack_bf16x2(aw[i]);
+                            const float2 w2 = unpack_bf16x2(ww[i]);
+                            acc[j][m] = fmaf(a2.x, w2.x, fmaf(a2.y, w2.y, acc[j][m]));
+                        }
+                    }
+                }
+            }
+        }
+#pragma unroll
+        for (int j = 0; j < kGemvCols; ++j)
+#pragma unroll
+            for (int m = 0; m < MR; ++m)
+#pragma unroll
+                for (int o = 16; o; o >>= 1) acc[j][m] += __shfl_xor_sync(0xffffffffu, acc[j][m], o);
+        if (lane < kGemvCols * MR) {
+            const int j = lane / MR, m = lane % MR;
+            const int n = n0 + j;
+            if (n < N && m < M) {
+                float v = 0.f;
+#pragma unroll
+                for (int jj = 0; jj < kGemvCols; ++jj)
+#pragma unroll
+                    for (int mm = 0; mm < MR; ++mm)
+                        if (jj == j && mm == m) v = acc[jj][mm];
+                if (e.bias) v += __bfloat162float(e.bias[n]);
+                if (e.act != ACT_NONE && n >= e.act_from) v = e.act == ACT_GELU ? gelu_tanh(v) : silu(v);
+                if (e.out_f32)
+                    static_cast<float*>(e.out0)[static_cast<int64_t>(m) * e.ld0 + n] = v;
+                else
+                    static_cast<__nv_bfloat16*>(e.out0)[static_cast<int64_t>(m) * e.ld0 + n] = __float2bfloat16_rn(v);
+            }
+        }
+    }
+}
+
+template <int MR>
+int launch_gemv(const GemmArgs& a, cudaStream_t stream) {
+    const int smem = MR * a.K * 2;
+    if (smem > 48 * 1024 &&
+        cudaFuncSetAttribute(gemv_rows_kernel<MR>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
+        return set_error(FF_ERR_CUDA, "gemv: cannot set shared memory size");
+    const int cols_per_block = (kGemvThreads / 32) * kGemvCols;
+    int grid = (a.N + cols_per_block - 1) / cols_per_block;
+    const int cap = 2 * num_sms();
+    if (grid > cap) grid = cap;
+    ProfScope prof(stream, "gemm_bf16", 2.0 * a.M * a.N * static_cast<double>(a.K),
+                   2.0 * static_cast<double>(a.N) * a.K + 2.0 * a.M * a.K);
+    gemv_rows_kernel<MR><<<grid, kGemvThreads, smem, stream>>>(static_cast<const __nv_bfloat16*>(a.A), a.lda, a.M,
+                                                               static_cast<const __nv_bfloat16*>(a.B), a.ldb, a.N,
+                                                               a.K, a.epi);
+    return check_launch("gemv_rows_kernel");
+}
+
+// Passes of at most 8 rows; a row's result is the same in every pass shape
+// (per-lane K order and the shuffle reduction do not depend on MR).
+int launch_gemv_rows(const GemmArgs& a, cudaStream_t stream) {
+    for (int m0 = 0; m0 < a.M; m0 += kGemvMaxRows) {
+        GemmArgs p = a;
+        p.M = a.M - m0 < kGemvMaxRows ? a.M - m0 : kGemvMaxRows;
+        p.A = static_cast<const __nv_bfloat16*>(a.A) + static_cast<int64_t>(m0) * a.lda;
+        p.epi.out0 = a.epi.out_f32 ? static_cast<void*>(static_cast<float*>(a.epi.out0) + m0 * a.epi.ld0)
+                                   : static_cast<void*>(static_cast<__nv_bfloat16*>(a.epi.out0) + m0 * a.epi.ld0);
+        int rc;
+        if (p.M <= 1) rc = launch_gemv<1>(p, stream);
+        else if (p.M <= 2) rc = launch_gemv<2>(p, stream);
+        else if (p.M <= 4) rc = launch_gemv<4>(p, stream);
+        else rc = launch_gemv<8>(p, stream);
+        if (rc) return rc;
+    }
+    return FF_OK;
+}
+
 int check_args(const GemmArgs& a) {
     const GemmEpilogue& e = a.epi;
     const int M = a.M, N = a.N, K = a.K;
@@ -572,8 +704,11 @@ int gemm_bf16_group(const GemmArgs* p, int n, cudaStream_t stream) {
         return launch<256>(p, n, stream);
     }
     const GemmArgs& a = p[0];
-    // narrow tiles when wide ones would leave most SMs idle (e.g. the
-    // batch-row time-embedding GEMMs)
+    const bool gemv_ok = a.K <= kGemvMaxK && a.epi.epi == EPI_STORE && a.epi.split_n >= a.N && a.epi.qk_cols == 0 &&
+                         aligned16(a.A) && aligned16(a.B) && a.lda % 8 == 0 && a.ldb % 8 == 0;
+    if (a.epi.rows_gemv && !gemv_ok) return set_error(FF_ERR_UNSUPPORTED, "gemm: rows_gemv needs K <= 8192 and a plain store");
+    if (gemv_ok && (a.epi.rows_gemv || a.M <= kGemvMaxRows)) return launch_gemv_rows(a, stream);
+    // narrow tiles when wide ones would leave most SMs idle
     const int64_t mblocks = (a.M + BM - 1) / BM;
     const bool few = mblocks * ((a.N + 255) / 256) < num_sms() / 2;
     if (a.N <= 64 || few) return launch<64>(p, 1, stream);

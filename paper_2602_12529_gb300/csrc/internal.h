@@ -64,6 +64,10 @@ struct GemmEpilogue {
     // tokens (row - rope_row0) % n_img of the (grid_f, grid_h, grid_w) grid
     // and are rotated with the cos/sin table rope_cs (see rope_table); rows
     // below rope_row0 are text tokens at position 0.
+    // Few-row products run on the GEMV kernel in passes of 8 rows whatever M
+    // is, so each row's result does not depend on how many rows share the
+    // launch (batch-invariant time embedding and modulation).
+    int rows_gemv = 0;
     int qk_cols = 0;
     int head_dim = 0;
     const __nv_bfloat16* q_scale = nullptr;

@@ -28,7 +28,10 @@ def _host_bf16(t):
 
 @pytest.mark.parametrize("M,N,K,act,f32", [
     (256, 256, 256, 0, 0), (300, 96, 72, 0, 1), (128, 64, 64, 0, 1), (4, 768, 256, 2, 0),
-    (1000, 1024, 320, 1, 0), (2048, 3072, 3072, 0, 1), (513, 512, 1024, 1, 1)])
+    (1000, 1024, 320, 1, 0), (2048, 3072, 3072, 0, 1), (513, 512, 1024, 1, 1),
+    # few-row (GEMV) path: ragged row counts, fp32 / bf16 outputs, activations
+    (3, 992, 320, 1, 1), (1, 64, 8, 0, 1), (8, 4096, 3072, 2, 0), (5, 6144, 256, 0, 1),
+    (9, 512, 256, 0, 1)])
 def test_gemm_parity(cuda, M, N, K, act, f32):
     import torch
     from paper_2602_12529_gb300 import ffi
