@@ -184,8 +184,8 @@ __device__ __forceinline__ void qk_norm_tile(const GemmEpilogue& e, int M, int r
     }
 }
 
-// Fused tail for one 32-column chunk of one output row held by this thread.
-__device__ __forceinline__ void epilogue_chunk(const GemmEpilogue& e, int M, int row, int n, float (&v)[32]) {
+// Bias and activation of one 32-column chunk of the row held by this thread.
+__device__ __forceinline__ void epilogue_values(const GemmEpilogue& e, int n, float (&v)[32]) {
     if (e.bias) {
 #pragma unroll
         for (int j = 0; j < 4; ++j) bias_add8(v + 8 * j, e.bias + n + 8 * j);
@@ -199,7 +199,13 @@ __device__ __forceinline__ void epilogue_chunk(const GemmEpilogue& e, int M, int
             for (int i = 0; i < 32; ++i) v[i] = silu(v[i]);
         }
     }
-    if (row >= M) return;
+}
+
+// Stores a warp's 32 rows x 32 columns from its transposed shared tile st
+// (row r at st[r * 33 ...]) as row segments: fp32 with 8 lanes x float4 per
+// row (4 rows per instruction), bf16 with 4 lanes x 8 values per row (8 rows
+// per instruction).
+__device__ __forceinline__ void store_rows(const GemmEpilogue& e, int M, int row0, int n, int lane, const float* st) {
     void* base;
     int64_t ld;
     int col;
@@ -209,16 +215,26 @@ __device__ __forceinline__ void epilogue_chunk(const GemmEpilogue& e, int M, int
         base = e.out1; ld = e.ld1; col = n - e.split_n + e.col1;
     }
     if (e.out_f32) {
-        float4* o = reinterpret_cast<float4*>(static_cast<float*>(base) + static_cast<int64_t>(row) * ld + col);
+        const int cq = lane & 7, rs = lane >> 3;
 #pragma unroll
-        for (int j = 0; j < 8; ++j) o[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+        for (int j = 0; j < 8; ++j) {
+            const int r = rs + 4 * j;
+            const float* a = st + r * 33 + 4 * cq;
+            if (row0 + r < M)
+                *reinterpret_cast<float4*>(static_cast<float*>(base) + static_cast<int64_t>(row0 + r) * ld + col + 4 * cq) =
+                    make_float4(a[0], a[1], a[2], a[3]);
+        }
     } else {
-        uint4* o = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(base) + static_cast<int64_t>(row) * ld + col);
+        const int cq = lane & 3, rs = lane >> 2;
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-            const float* s = v + 8 * j;
-            o[j] = make_uint4(pack_bf16x2(s[0], s[1]), pack_bf16x2(s[2], s[3]), pack_bf16x2(s[4], s[5]),
-                              pack_bf16x2(s[6], s[7]));
+            const int r = rs + 8 * j;
+            const float* a = st + r * 33 + 8 * cq;
+            if (row0 + r < M)
+                *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(base) + static_cast<int64_t>(row0 + r) * ld + col +
+                                          8 * cq) =
+                    make_uint4(pack_bf16x2(a[0], a[1]), pack_bf16x2(a[2], a[3]), pack_bf16x2(a[4], a[5]),
+                               pack_bf16x2(a[6], a[7]));
         }
     }
 }
@@ -441,6 +457,11 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_cons
             } else if (epi.qk_cols > 0 && nb * BN < epi.qk_cols) {
                 qk_norm_tile(epi, M, row, nb * BN, t_acc, BN);
             } else {
+                // plain store: bias / activation on the row held by this
+                // thread, then a transpose through this warp's 32x33 shared
+                // tile so that the global stores are whole row segments
+                float* st = reinterpret_cast<float*>(rbuf) + (warp - 2) * (32 * 33);
+                const int row0 = mb * BM + q * 32;
 #pragma unroll 1
                 for (int c = 0; c < BN; c += 32) {
                     uint32_t rr[32];
@@ -451,7 +472,12 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_cons
                     float v[32];
 #pragma unroll
                     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(rr[i]);
-                    epilogue_chunk(epi, M, row, n, v);
+                    epilogue_values(epi, n, v);
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) st[lane * 33 + i] = v[i];
+                    __syncwarp();
+                    store_rows(epi, M, row0, n, lane, st);
+                    __syncwarp();
                 }
             }
             tc_fence_before();
@@ -698,6 +724,8 @@ int gemm_bf16_group(const GemmArgs* p, int n, cudaStream_t stream) {
         if (rc) return rc;
         qk = qk || p[i].epi.qk_cols > 0;
     }
+    if (n == 2 && (p[0].epi.epi == EPI_GATED_RESIDUAL) != (p[1].epi.epi == EPI_GATED_RESIDUAL))
+        return set_error(FF_ERR_INVALID_ARG, "gemm: grouped problems must share the epilogue kind");
     if (n == 2 || qk) {
         for (int i = 0; i < n; ++i)
             if (p[i].N <= 128) return set_error(FF_ERR_UNSUPPORTED, "gemm: grouped / fused problems need N > 128");
