@@ -239,6 +239,90 @@ __device__ __forceinline__ void store_rows(const GemmEpilogue& e, int M, int row
     }
 }
 
+// One tile of the epilogue for the 128 rows m0.. held in this CTA's TMEM
+// (t_acc: this warp's lane quarter of the accumulator).  Returns false after
+// a bounded wait gave up.
+template <int BN>
+__device__ __forceinline__ bool epilogue_tile(const GemmEpilogue& epi, int M, int N, int m0, int nb, uint32_t t_acc,
+                                              int q, int lane, int warp, bool leader, const CUtensorMap* tr,
+                                              uint8_t* rbuf, uint64_t* rfull_bar, uint64_t* rdone_bar,
+                                              uint32_t (&ruse)[2], int* status, volatile int* abort_flag) {
+    using C = Cfg<BN>;
+    const bool gated = epi.epi == EPI_GATED_RESIDUAL;
+    const int r = q * 32 + lane;                // row within the tile = TMEM lane
+    const int row = m0 + r;
+    if (gated) {
+        bool ok = true;
+        for (int c = 0; c < BN / 32; ++c) {
+            const int n = nb * BN + c * 32;
+            const int b = c & 1;
+            uint32_t rr[32];
+            tmem_ld_x32(t_acc + c * 32, rr);
+            tmem_ld_wait();
+            float v[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(rr[i]);
+            if (epi.bias) {
+#pragma unroll
+                for (int j = 0; j < 4; ++j) bias_add8(v + 8 * j, epi.bias + n + 8 * j);
+            }
+            if (!mbar_wait(&rfull_bar[b], ruse[b] & 1)) {
+                report_status(status, kStatusWaitTimeout);
+                *abort_flag = 1;
+                ok = false;
+            }
+            if (ok) gated_update(epi, M, row, r, n, v, rbuf + b * C::kResidBytes);
+            fence_proxy_async_smem();
+            mbar_arrive(&rdone_bar[b]);
+            // the leader stores the chunk once every thread has updated it
+            // (an mbarrier, not bar.sync: a thread that gave up on a wait
+            // must not be able to stall the others)
+            if (leader && ok && !mbar_wait(&rdone_bar[b], ruse[b] & 1)) {
+                report_status(status, kStatusWaitTimeout);
+                *abort_flag = 1;
+                ok = false;
+            }
+            ++ruse[b];
+            if (leader && ok) {
+                tma_store_2d(tr, rbuf + b * C::kResidBytes, n, m0);
+                bulk_commit();
+                if (c + 2 < BN / 32) {
+                    bulk_wait_read<0>();
+                    mbar_arrive_expect_tx(&rfull_bar[b], C::kResidBytes);
+                    tma_load_2d(rbuf + b * C::kResidBytes, tr, &rfull_bar[b], n + 64, m0);
+                }
+            }
+        }
+        if (!ok) return false;
+    } else if (epi.qk_cols > 0 && nb * BN < epi.qk_cols) {
+        qk_norm_tile(epi, M, row, nb * BN, t_acc, BN);
+    } else {
+        // plain store: bias / activation on the row held by this
+        // thread, then a transpose through this warp's 32x33 shared
+        // tile so that the global stores are whole row segments
+        float* st = reinterpret_cast<float*>(rbuf) + (warp - 2) * (32 * 33);
+        const int row0 = m0 + q * 32;
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+            uint32_t rr[32];
+            tmem_ld_x32(t_acc + c, rr);
+            tmem_ld_wait();
+            const int n = nb * BN + c;
+            if (n >= N) continue;
+            float v[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(rr[i]);
+            epilogue_values(epi, n, v);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) st[lane * 33 + i] = v[i];
+            __syncwarp();
+            store_rows(epi, M, row0, n, lane, st);
+            __syncwarp();
+        }
+    }
+    return true;
+}
+
 // Up to two independent GEMM problems share one persistent launch: the tile
 // space is problem 0's tiles followed by problem 1's, so a small problem
 // (the text stream of a double-stream block) fills the tail of a large one.
@@ -385,6 +469,7 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_cons
         const int q = warp & 3;
         const bool leader = warp == 2 && lane == 0;     // issues the residual TMA traffic
         uint32_t ruse[2] = {0, 0};                      // residual loads consumed per buffer
+        const uint32_t t_acc_base = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
         int acc = 0;
         uint32_t acc_phase = 0;
         for (int tile = blockIdx.x; tile < g.tiles && !*abort_flag; tile += gridDim.x) {
@@ -408,78 +493,9 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_cons
                 break;
             }
             tc_fence_after();
-            const int r = q * 32 + lane;                // row within the tile = TMEM lane
-            const int row = mb * BM + r;
-            const uint32_t t_acc = tmem_base + static_cast<uint32_t>(acc * BN) + (static_cast<uint32_t>(q * 32) << 16);
-            if (gated) {
-                bool ok = true;
-                for (int c = 0; c < BN / 32; ++c) {
-                    const int n = nb * BN + c * 32;
-                    const int b = c & 1;
-                    uint32_t rr[32];
-                    tmem_ld_x32(t_acc + c * 32, rr);
-                    tmem_ld_wait();
-                    float v[32];
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(rr[i]);
-                    if (epi.bias) {
-#pragma unroll
-                        for (int j = 0; j < 4; ++j) bias_add8(v + 8 * j, epi.bias + n + 8 * j);
-                    }
-                    if (!mbar_wait(&rfull_bar[b], ruse[b] & 1)) {
-                        report_status(status, kStatusWaitTimeout);
-                        *abort_flag = 1;
-                        ok = false;
-                    }
-                    if (ok) gated_update(epi, M, row, r, n, v, rbuf + b * C::kResidBytes);
-                    fence_proxy_async_smem();
-                    mbar_arrive(&rdone_bar[b]);
-                    // the leader stores the chunk once every thread has updated it
-                    // (an mbarrier, not bar.sync: a thread that gave up on a wait
-                    // must not be able to stall the others)
-                    if (leader && ok && !mbar_wait(&rdone_bar[b], ruse[b] & 1)) {
-                        report_status(status, kStatusWaitTimeout);
-                        *abort_flag = 1;
-                        ok = false;
-                    }
-                    ++ruse[b];
-                    if (leader && ok) {
-                        tma_store_2d(tr, rbuf + b * C::kResidBytes, n, mb * BM);
-                        bulk_commit();
-                        if (c + 2 < BN / 32) {
-                            bulk_wait_read<0>();
-                            mbar_arrive_expect_tx(&rfull_bar[b], C::kResidBytes);
-                            tma_load_2d(rbuf + b * C::kResidBytes, tr, &rfull_bar[b], n + 64, mb * BM);
-                        }
-                    }
-                }
-                if (!ok) break;
-            } else if (epi.qk_cols > 0 && nb * BN < epi.qk_cols) {
-                qk_norm_tile(epi, M, row, nb * BN, t_acc, BN);
-            } else {
-                // plain store: bias / activation on the row held by this
-                // thread, then a transpose through this warp's 32x33 shared
-                // tile so that the global stores are whole row segments
-                float* st = reinterpret_cast<float*>(rbuf) + (warp - 2) * (32 * 33);
-                const int row0 = mb * BM + q * 32;
-#pragma unroll 1
-                for (int c = 0; c < BN; c += 32) {
-                    uint32_t rr[32];
-                    tmem_ld_x32(t_acc + c, rr);
-                    tmem_ld_wait();
-                    const int n = nb * BN + c;
-                    if (n >= N) continue;
-                    float v[32];
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(rr[i]);
-                    epilogue_values(epi, n, v);
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) st[lane * 33 + i] = v[i];
-                    __syncwarp();
-                    store_rows(epi, M, row0, n, lane, st);
-                    __syncwarp();
-                }
-            }
+            if (!epilogue_tile<BN>(epi, M, N, mb * BM, nb, t_acc_base + static_cast<uint32_t>(acc * BN), q, lane, warp,
+                                   leader, tr, rbuf, rfull_bar, rdone_bar, ruse, status, abort_flag))
+                break;
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&tempty_bar[acc]);
@@ -500,6 +516,251 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_cons
         tc_fence_after();
         tmem_dealloc(tmem_base, C::kTmemCols);
     }
+}
+
+// ---------------------------------------------------------------------------
+// Two-SM variant: a cluster of two CTAs computes one 256 x 256 tile with
+// tcgen05.mma.cta_group::2.  Each CTA stages its own 128 rows of A and its
+// half (128 rows) of B, so per-SM shared-memory operand traffic per FLOP
+// drops by a third against the 128 x 256 single-CTA tile.  The leader CTA
+// (rank 0) owns the stage-full barriers (both CTAs' TMA loads complete on
+// them) and the accumulator-empty barriers (both CTAs' epilogues arrive on
+// them) and issues every MMA; its commits are multicast to the same barrier
+// in both CTAs.  Each CTA's epilogue drains its own 128 accumulator rows.
+// Every wait is bounded and both CTAs always reach the closing cluster
+// barrier, so neither can leave while the other may still signal it.
+// ---------------------------------------------------------------------------
+constexpr int PBM = 256;   // rows per pair tile
+constexpr int PBN = 256;   // columns per pair tile
+constexpr int kPairStages = 6;
+
+struct PairCfg {
+    static constexpr int kABytes = 128 * BK * 2;           // this CTA's A rows
+    static constexpr int kBBytes = (PBN / 2) * BK * 2;     // this CTA's half of B
+    static constexpr int kStageBytes = kABytes + kBBytes;
+    static constexpr int kResidBytes = 128 * 32 * 4;
+    static constexpr int kBarrierBytes = 256;
+    static constexpr int kSmemBytes = kPairStages * kStageBytes + 2 * kResidBytes + 1024 + kBarrierBytes;
+};
+
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_constant__ CUtensorMap tm_b0,
+                 const __grid_constant__ CUtensorMap tm_a1, const __grid_constant__ CUtensorMap tm_b1,
+                 const __grid_constant__ CUtensorMap tm_r0, const __grid_constant__ CUtensorMap tm_r1,
+                 const __grid_constant__ GemmGroup g, int* status) {
+    using C = PairCfg;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t* rbuf = smem + kPairStages * C::kStageBytes;
+    uint64_t* full_bar = reinterpret_cast<uint64_t*>(rbuf + 2 * C::kResidBytes);   // used in the leader
+    uint64_t* empty_bar = full_bar + kPairStages;                                   // both CTAs
+    uint64_t* tfull_bar = empty_bar + kPairStages;   // [2] both CTAs
+    uint64_t* tempty_bar = tfull_bar + 2;            // [2] leader, 8 arrivals
+    uint64_t* drain_bar = tempty_bar + 2;            // [1] leader
+    uint64_t* rfull_bar = drain_bar + 1;             // [2] per CTA
+    uint64_t* rdone_bar = rfull_bar + 2;             // [2] per CTA
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(rdone_bar + 2);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_ctarank();
+    const int cluster = blockIdx.x >> 1;
+    const int nclusters = gridDim.x >> 1;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kPairStages; ++s) {
+            mbar_init(&full_bar[s], 1);
+            mbar_init(&empty_bar[s], 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(&tfull_bar[a], 1);
+            mbar_init(&tempty_bar[a], 8);
+            mbar_init(&rfull_bar[a], 1);
+            mbar_init(&rdone_bar[a], 128);
+        }
+        mbar_init(drain_bar, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+        prefetch_tmap(&tm_a0);
+        prefetch_tmap(&tm_b0);
+        if (g.tiles > g.tiles0) {
+            prefetch_tmap(&tm_a1);
+            prefetch_tmap(&tm_b1);
+        }
+    }
+    if (warp == 1) {
+        tmem_alloc_pair(tmem_slot, 2 * PBN);
+        tmem_relinquish_pair();
+    }
+    tc_fence_before();
+    cluster_sync();   // both CTAs' barriers and TMEM exist before any cross-CTA traffic
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+
+    if (warp == 0 && lane == 0) {
+        // ---------------- TMA producer (both CTAs; completion counted in the leader)
+        int stage = 0;
+        uint32_t phase = 0;
+        for (int tile = cluster; tile < g.tiles && !*abort_flag; tile += nclusters) {
+            int pr, mb, nb;
+            locate(g, tile, pr, mb, nb);
+            const CUtensorMap* ta = pr ? &tm_a1 : &tm_a0;
+            const CUtensorMap* tb = pr ? &tm_b1 : &tm_b0;
+            const int num_k = (g.K[pr] + BK - 1) / BK;
+            for (int kb = 0; kb < num_k; ++kb) {
+                if (!mbar_wait(&empty_bar[stage], phase ^ 1)) {
+                    report_status(status, kStatusWaitTimeout);
+                    *abort_flag = 1;
+                    break;
+                }
+                uint8_t* sa = smem + stage * C::kStageBytes;
+                uint8_t* sb = sa + C::kABytes;
+                const uint32_t fb = mapa_shared(smem_u32(&full_bar[stage]), 0);
+                if (rank == 0) mbar_arrive_expect_tx(&full_bar[stage], 2 * C::kStageBytes);
+                tma_load_2d_pair(sa, ta, fb, kb * BK, mb * PBM + rank * 128);
+                tma_load_2d_pair(sb, tb, fb, kb * BK, nb * PBN + rank * (PBN / 2));
+                if (++stage == kPairStages) { stage = 0; phase ^= 1; }
+            }
+        }
+    } else if (warp == 1 && lane == 0 && rank == 0) {
+        // ---------------- MMA issuer (leader only): 256 x 256 x 16 per instruction
+        constexpr uint32_t idesc = idesc_bf16_f32(PBM, PBN);
+        int stage = 0;
+        uint32_t phase = 0;
+        int acc = 0;
+        uint32_t acc_phase = 0;
+        for (int tile = cluster; tile < g.tiles && !*abort_flag; tile += nclusters) {
+            const int pr = tile < g.tiles0 ? 0 : 1;
+            const int num_k = (g.K[pr] + BK - 1) / BK;
+            if (!mbar_wait(&tempty_bar[acc], acc_phase ^ 1)) {
+                report_status(status, kStatusWaitTimeout);
+                *abort_flag = 1;
+                break;
+            }
+            tc_fence_after();
+            const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * PBN);
+            bool ok = true;
+            for (int kb = 0; kb < num_k; ++kb) {
+                if (!mbar_wait(&full_bar[stage], phase)) {
+                    report_status(status, kStatusWaitTimeout);
+                    *abort_flag = 1;
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t sa = smem_u32(smem + stage * C::kStageBytes);
+                const uint32_t sb = sa + C::kABytes;
+                const uint64_t da = smem_desc_k_sw128(sa);
+                const uint64_t db = smem_desc_k_sw128(sb);
+#pragma unroll
+                for (int k = 0; k < BK / 16; ++k)
+                    tc_mma_bf16_pair(d_tmem, da + static_cast<uint64_t>(2 * k), db + static_cast<uint64_t>(2 * k), idesc,
+                                     (kb | k) != 0 ? 1u : 0u);
+                tc_commit_pair_mc(&empty_bar[stage], 0x3);
+                if (++stage == kPairStages) { stage = 0; phase ^= 1; }
+            }
+            if (!ok) break;
+            tc_commit_pair_mc(&tfull_bar[acc], 0x3);
+            if (++acc == 2) { acc = 0; acc_phase ^= 1; }
+        }
+        tc_commit_pair_mc(drain_bar, 0x1);
+        if (!mbar_wait(drain_bar, 0)) report_status(status, kStatusWaitTimeout);
+    } else if (warp >= 2) {
+        // ---------------- epilogue (both CTAs, own 128 accumulator rows)
+        const int q = warp & 3;
+        const bool leader = warp == 2 && lane == 0;
+        uint32_t ruse[2] = {0, 0};
+        const uint32_t t_acc_base = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
+        int acc = 0;
+        uint32_t acc_phase = 0;
+        for (int tile = cluster; tile < g.tiles && !*abort_flag; tile += nclusters) {
+            int pr, mb, nb;
+            locate(g, tile, pr, mb, nb);
+            const GemmEpilogue& epi = g.epi[pr];
+            const int M = g.M[pr], N = g.N[pr];
+            const int m0 = mb * PBM + rank * 128;
+            const CUtensorMap* tr = pr ? &tm_r1 : &tm_r0;
+            if (epi.epi == EPI_GATED_RESIDUAL && leader) {
+                for (int c = 0; c < 2; ++c) {
+                    bulk_wait_read<0>();
+                    mbar_arrive_expect_tx(&rfull_bar[c], C::kResidBytes);
+                    tma_load_2d(rbuf + c * C::kResidBytes, tr, &rfull_bar[c], nb * PBN + c * 32, m0);
+                }
+            }
+            if (!mbar_wait(&tfull_bar[acc], acc_phase)) {
+                report_status(status, kStatusWaitTimeout);
+                *abort_flag = 1;
+                break;
+            }
+            tc_fence_after();
+            if (!epilogue_tile<PBN>(epi, M, N, m0, nb, t_acc_base + static_cast<uint32_t>(acc * PBN), q, lane, warp,
+                                    leader, tr, rbuf, rfull_bar, rdone_bar, ruse, status, abort_flag))
+                break;
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive_cluster(mapa_shared(smem_u32(&tempty_bar[acc]), 0));
+            if (++acc == 2) { acc = 0; acc_phase ^= 1; }
+        }
+        if (leader) bulk_wait<0>();
+    }
+
+    if (*abort_flag) {
+        const uint64_t t0 = global_timer_ns();
+        while (global_timer_ns() - t0 < 50000ull) {
+        }
+    }
+    tc_fence_before();
+    cluster_sync();   // nothing crosses the pair after this point
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc_pair(tmem_base, 2 * PBN);
+    }
+}
+
+int launch_pair(const GemmArgs* p, int n, cudaStream_t stream) {
+    using C = PairCfg;
+    if (cudaFuncSetAttribute(gemm_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes) !=
+        cudaSuccess)
+        return set_error(FF_ERR_CUDA, "gemm (pair): cannot set shared memory size (%d B)", C::kSmemBytes);
+    CUtensorMap ta[2], tb[2], tr[2];
+    GemmGroup g{};
+    double flops = 0.0, bytes = 0.0;
+    for (int i = 0; i < 2; ++i) {
+        const GemmArgs& a = p[i < n ? i : 0];
+        int rc = make_tmap_bf16(&ta[i], a.A, a.M, a.K, a.lda, 128);
+        if (rc) return rc;
+        rc = make_tmap_bf16(&tb[i], a.B, a.N, a.K, a.ldb, PBN / 2);
+        if (rc) return rc;
+        if (a.epi.epi == EPI_GATED_RESIDUAL) {
+            rc = make_tmap_f32_sw128(&tr[i], a.epi.resid, a.M, a.N, a.epi.ld_resid, 128);
+            if (rc) return rc;
+        } else {
+            tr[i] = ta[i];
+        }
+        g.M[i] = a.M;
+        g.N[i] = a.N;
+        g.K[i] = a.K;
+        g.num_m[i] = (a.M + PBM - 1) / PBM;
+        g.num_n[i] = (a.N + PBN - 1) / PBN;
+        g.epi[i] = a.epi;
+        if (i < n) {
+            const double mn = static_cast<double>(a.M) * a.N;
+            flops += 2.0 * mn * a.K;
+            bytes += 2.0 * (static_cast<double>(a.M) + a.N) * a.K +
+                     (a.epi.epi == EPI_GATED_RESIDUAL ? mn * 8.0 : mn * (a.epi.out_f32 ? 4.0 : 2.0));
+        }
+    }
+    for (int i = 0; i < n; ++i)
+        if (p[i].epi.epi == EPI_GATED_RESIDUAL && p[i].N % PBN)
+            return set_error(FF_ERR_UNSUPPORTED, "gemm (pair): gated residual needs N %% 256 == 0");
+    g.tiles0 = g.num_m[0] * g.num_n[0];
+    g.tiles = g.tiles0 + (n > 1 ? g.num_m[1] * g.num_n[1] : 0);
+    const int clusters = g.tiles < num_sms() / 2 ? g.tiles : num_sms() / 2;
+    ProfScope prof(stream, "gemm_bf16", flops, bytes);
+    gemm_pair_kernel<<<2 * clusters, kThreads, C::kSmemBytes, stream>>>(ta[0], tb[0], ta[1], tb[1], tr[0], tr[1], g,
+                                                                        device_status_ptr());
+    return check_launch("gemm_pair_kernel");
 }
 
 template <int BN>
@@ -726,6 +987,15 @@ int gemm_bf16_group(const GemmArgs* p, int n, cudaStream_t stream) {
     }
     if (n == 2 && (p[0].epi.epi == EPI_GATED_RESIDUAL) != (p[1].epi.epi == EPI_GATED_RESIDUAL))
         return set_error(FF_ERR_INVALID_ARG, "gemm: grouped problems must share the epilogue kind");
+    // two-SM 256 x 256 tiles when every problem's N is a multiple of 256 and
+    // there is enough work for them
+    bool pair = true;
+    int max_m = 0;
+    for (int i = 0; i < n; ++i) {
+        pair = pair && p[i].N % 256 == 0 && p[i].epi.rows_gemv == 0;
+        max_m = p[i].M > max_m ? p[i].M : max_m;
+    }
+    if (pair && max_m >= 512) return launch_pair(p, n, stream);
     if (n == 2 || qk) {
         for (int i = 0; i < n; ++i)
             if (p[i].N <= 128) return set_error(FF_ERR_UNSUPPORTED, "gemm: grouped / fused problems need N > 128");
