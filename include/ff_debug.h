@@ -52,11 +52,6 @@ int ff_debug_qk_norm_rope(int rows, int rows_txt, int heads, int head_dim, void*
                           const void* q_scale, const void* k_scale, int grid_f, int grid_h, int grid_w,
                           const int* rope_axes, float rope_theta, cudaStream_t stream);
 
-/* y[i] = 2^x[i] by the attention kernel's software exponential (range
- * reduction to n + f, f in [-1/2, 1/2], degree-3 minimax polynomial for 2^f,
- * n added to the exponent; arguments clamped at -126).  n even. */
-int ff_debug_exp2(const float* x, float* y, int64_t n, cudaStream_t stream);
-
 #ifdef __cplusplus
 }
 #endif

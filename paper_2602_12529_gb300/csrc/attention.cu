@@ -8,9 +8,12 @@
 //
 // One CTA = two 128-row query tiles (256 query rows) of one segment of one
 // (sample, head), sharing every K/V tile.  Warp roles (10 warps):
-//   warp 0      TMA producer: both Q tiles once, then 128-token K/V tiles
-//               into a 2-deep ring (K/V tiles never straddle the segment
-//               boundary; rows past the segment end are masked).
+//   warp 0      TMA producer: both Q tiles once, then the 128-token K and V
+//               tiles in the order K_0, V_0, K_1, V_1, ... into a ring of
+//               single-operand slots (5 at d = 128), so the operands of the
+//               next K/V step are resident a whole step before they are used
+//               (K/V tiles never straddle the segment boundary; rows past the
+//               segment end are masked).
 //   warp 1      TMEM allocator (all 512 columns); lane 0 issues the MMAs.
 //               Per query tile t the order is S_t,j = Q_t K_j^T (M 128, N 128,
 //               A and B from shared memory) -> softmax -> O_t += P_t,j V_j
@@ -25,7 +28,6 @@
 //               P = exp2(S - m) as bf16 pairs over the S columns, and
 //               rescales its O row in TMEM only when the running max grows by
 //               more than 8 (2^8 headroom), which makes corrections rare.
-//               Part of the exponentials run on the FMA pipe (exp2_poly2).
 //               Finally O / l goes out as bf16.
 // Every wait is bounded; on a timeout the kernel records the status word,
 // drains its tensor-core work, frees TMEM and returns.
@@ -37,18 +39,17 @@ namespace {
 
 constexpr int kBM = 128;         // query rows per query tile (two tiles per CTA)
 constexpr int kBN = 128;         // tokens per K/V tile
-constexpr int kStages = 2;
 constexpr int kThreads = 320;    // producer, MMA, 2 x 4 softmax warps
 constexpr float kRescaleThreshold = 8.0f;   // log2 units
-constexpr int kSwExp = 40;       // of every 128 scores, this many use the software exp2
 
 template <int HD>
 struct ACfg {
     static constexpr int kQBytes = kBM * HD * 2;        // one query tile
-    static constexpr int kKBytes = kBN * HD * 2;
-    static constexpr int kStageBytes = 2 * kKBytes;     // K + V
+    static constexpr int kKBytes = kBN * HD * 2;        // one K or V tile = one ring slot
     static constexpr int kBarBytes = 256;
-    static constexpr int kSmemBytes = 2 * kQBytes + kStages * kStageBytes + kBarBytes;
+    static constexpr int kSlots = (232448 - 2 * kQBytes - kBarBytes) / kKBytes < 8
+                                      ? (232448 - 2 * kQBytes - kBarBytes) / kKBytes : 8;
+    static constexpr int kSmemBytes = 2 * kQBytes + kSlots * kKBytes + kBarBytes;
     static constexpr int kTmemCols = 512;
     // TMEM columns of query tile t: S (fp32, kBN columns) at t*256, with P
     // (bf16 pairs, kBN/2 columns) written over its first half; O at t*256+128
@@ -77,30 +78,6 @@ __device__ __forceinline__ float max3(float a, float b, float c) {
     return y;
 }
 
-// Software 2^x for a pair of arguments, on the FMA pipe (the MUFU unit alone
-// cannot keep up with the tensor core at d = 128).  Range reduction: n =
-// round(x) via the 1.5 * 2^23 shifter, f = x - n in [-1/2, 1/2]; 2^f from a
-// degree-3 minimax polynomial (Remez exchange on the relative error,
-// coefficients from csrc/fit_exp2.py; max relative error 7.5e-5, below the
-// bf16 rounding that P receives); 2^n is added into the exponent field.
-// Arguments are clamped at -126: p(f) >= 2^-1/2 has biased exponent >= 126,
-// so adding n >= -126 never wraps the exponent field (at n = -127 a p(0)
-// just below 1 would wrap to a NaN); 2^-126 is zero for every use here.
-__device__ __forceinline__ float2 exp2_poly2(float2 x) {
-    constexpr float kShift = 12582912.0f;   // 1.5 * 2^23
-    x.x = fmaxf(x.x, -126.0f);
-    x.y = fmaxf(x.y, -126.0f);
-    const float2 t = __fadd2_rn(x, make_float2(kShift, kShift));
-    const float2 n = __fadd2_rn(t, make_float2(-kShift, -kShift));
-    const float2 f = __ffma2_rn(n, make_float2(-1.0f, -1.0f), x);
-    float2 q = __ffma2_rn(make_float2(5.517166853e-02f, 5.517166853e-02f), f,
-                          make_float2(2.426111251e-01f, 2.426111251e-01f));
-    q = __ffma2_rn(q, f, make_float2(6.932609677e-01f, 6.932609677e-01f));
-    q = __ffma2_rn(q, f, make_float2(9.999280572e-01f, 9.999280572e-01f));
-    return make_float2(__uint_as_float(__float_as_uint(q.x) + (__float_as_uint(t.x) << 23)),
-                       __uint_as_float(__float_as_uint(q.y) + (__float_as_uint(t.y) << 23)));
-}
-
 __device__ __forceinline__ void tmem_st_x32(uint32_t taddr, const uint32_t* r) {
     asm volatile(
         "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
@@ -124,7 +101,6 @@ __device__ __forceinline__ void tc_mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem,
         ::"r"(d_tmem), "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
         : "memory");
 }
-
 // B operand stored MN-major with 128-byte swizzle (V: rows = K = tokens,
 // 64 contiguous d per 128-byte row): leading byte offset = distance between
 // 64-wide d blocks, stride byte offset = distance between 8-token groups.
@@ -140,10 +116,11 @@ __device__ __forceinline__ uint64_t smem_desc_mn_sw128(uint32_t saddr, uint32_t 
 
 // Barriers.  Per query tile the chain S -> softmax -> P -> O += P V -> next S
 // is strictly ordered, so no waiter can lag two phases behind a parity wait.
+constexpr int kMaxSlots = 8;
 struct Bars {
     uint64_t q_full;
-    uint64_t kv_full[kStages];
-    uint64_t kv_empty[kStages];
+    uint64_t slot_full[kMaxSlots];    // ring item n = 2 j (K_j) or 2 j + 1 (V_j) lives in slot n % kSlots
+    uint64_t slot_empty[kMaxSlots];
     uint64_t s_full[2];       // [query tile] MMA -> softmax: S_t,j is in TMEM (and O += P V_{j-1} done)
     uint64_t p_full[2];       //              softmax -> MMA: P_t,j is in TMEM, O rescaled
     uint64_t o_last[2];       //              MMA -> softmax: the last O += P V has landed
@@ -159,10 +136,12 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
                     const AttnParams p, int* status) {
     using C = ACfg<HD>;
     static_assert(sizeof(Bars) <= C::kBarBytes, "barrier block too small");
+    static_assert(C::kSlots >= 3 && C::kSlots <= kMaxSlots, "K/V ring size");
+    constexpr int S = C::kSlots;
     extern __shared__ __align__(1024) uint8_t smem[];
     uint8_t* sQ = smem;                                   // [2][kQBytes]
-    uint8_t* sKV = smem + 2 * C::kQBytes;                 // [kStages][K | V]
-    Bars& bar = *reinterpret_cast<Bars*>(sKV + kStages * C::kStageBytes);
+    uint8_t* sKV = smem + 2 * C::kQBytes;                 // [kSlots][K or V tile]
+    Bars& bar = *reinterpret_cast<Bars*>(sKV + S * C::kKBytes);
     volatile int* abort_flag = &bar.abort_flag;
 
     const int warp = threadIdx.x >> 5;
@@ -181,9 +160,9 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
             *abort_flag = 1;
         }
         mbar_init(&bar.q_full, 1);
-        for (int s = 0; s < kStages; ++s) {
-            mbar_init(&bar.kv_full[s], 1);
-            mbar_init(&bar.kv_empty[s], 1);
+        for (int s = 0; s < S; ++s) {
+            mbar_init(&bar.slot_full[s], 1);
+            mbar_init(&bar.slot_empty[s], 1);
         }
         for (int t = 0; t < 2; ++t) {
             mbar_init(&bar.s_full[t], 1);
@@ -221,19 +200,18 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
             for (int c = 0; c < HD / 64; ++c)
                 tma_load_2d(sQ + t * C::kQBytes + c * (kBM * 128), tq, &bar.q_full, p.q_col + h * HD + c * 64,
                             b * p.nq[seg] + q0 + t * kBM);
-        for (int j = 0; j < ntiles && !*abort_flag; ++j) {
-            const int s = j % kStages;
-            if (!mbar_wait(&bar.kv_empty[s], ((j / kStages) & 1) ^ 1)) { fail(); break; }
+        for (int n = 0; n < 2 * ntiles && !*abort_flag; ++n) {
+            const int s = n % S;
+            if (!mbar_wait(&bar.slot_empty[s], ((n / S) & 1) ^ 1)) { fail(); break; }
+            const int j = n >> 1;
             const int ks = j < nt0 ? 0 : 1;
             const int row = b * p.nkv[ks] + (j - (ks ? nt0 : 0)) * kBN;
             const CUtensorMap* tkv = ks ? &tm_kv1 : &tm_kv0;
-            uint8_t* dk = sKV + s * C::kStageBytes;
-            uint8_t* dv = dk + C::kKBytes;
-            mbar_arrive_expect_tx(&bar.kv_full[s], C::kStageBytes);
-            for (int c = 0; c < HD / 64; ++c) {
-                tma_load_2d(dk + c * (kBN * 128), tkv, &bar.kv_full[s], p.k_col + h * HD + c * 64, row);
-                tma_load_2d(dv + c * (kBN * 128), tkv, &bar.kv_full[s], p.v_col + h * HD + c * 64, row);
-            }
+            const int col = ((n & 1) ? p.v_col : p.k_col) + h * HD;
+            uint8_t* dst = sKV + s * C::kKBytes;
+            mbar_arrive_expect_tx(&bar.slot_full[s], C::kKBytes);
+            for (int c = 0; c < HD / 64; ++c)
+                tma_load_2d(dst + c * (kBN * 128), tkv, &bar.slot_full[s], col + c * 64, row);
         }
     } else if (warp == 1 && lane == 0) {
         // ------------------------------------------------------------ MMA issuer
@@ -241,28 +219,35 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
         // S_t,j+1.  The two tiles interleave so one tile's MMAs run while the
         // other tile's softmax works.  tcgen05.mma from one thread executes in
         // issue order, so S_t,j+1 overwrites the columns of P_t,j only after
-        // O_t += P_t,j V_j has read them.
+        // O_t += P_t,j V_j has read them.  K_0 is released once both S_t,0 are
+        // done, V_j and K_j+1 together after step j.
         constexpr uint32_t idesc_s = idesc_bf16_f32(kBM, kBN);
         constexpr uint32_t idesc_o = idesc_bf16_f32(kBM, HD) | (1u << 16);   // B (V) is MN-major
         bool ok = mbar_wait(&bar.q_full, 0);
         if (!ok) fail();
+        auto slot_ready = [&](int n) {
+            if (!mbar_wait(&bar.slot_full[n % S], (n / S) & 1)) return false;
+            tc_fence_after();
+            return true;
+        };
         auto issue_s = [&](int t, int j) {
             const uint32_t aQ = smem_u32(sQ + t * C::kQBytes);
-            const uint32_t aK = smem_u32(sKV + (j % kStages) * C::kStageBytes);
+            const uint32_t aK = smem_u32(sKV + ((2 * j) % S) * C::kKBytes);
             const uint32_t dS = tmem + t * 256;
 #pragma unroll
             for (int k = 0; k < HD / 16; ++k) {
                 const uint32_t off_q = (k / 4) * (kBM * 128) + (k % 4) * 32;
                 const uint32_t off_k = (k / 4) * (kBN * 128) + (k % 4) * 32;
                 tc_mma_bf16(dS, smem_desc_k_sw128(aQ + off_q), smem_desc_k_sw128(aK + off_k), idesc_s,
-                            k != 0 ? 1u : 0u);
+                                k != 0 ? 1u : 0u);
             }
             tc_commit(&bar.s_full[t]);
         };
         auto issue_pv = [&](int t, int j) -> bool {
             if (!mbar_wait(&bar.p_full[t], j & 1)) return false;
             tc_fence_after();
-            const uint32_t aV = smem_u32(sKV + (j % kStages) * C::kStageBytes + C::kKBytes);
+            if (t == 0 && !slot_ready(2 * j + 1)) return false;
+            const uint32_t aV = smem_u32(sKV + ((2 * j + 1) % S) * C::kKBytes);
             const uint32_t dO = tmem + t * 256 + C::kColO;
             const uint32_t aP = tmem + t * 256;
 #pragma unroll
@@ -273,11 +258,11 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
             return true;
         };
         if (ok && ntiles > 0) {
-            if (!mbar_wait(&bar.kv_full[0], 0)) { fail(); ok = false; }
+            if (!slot_ready(0)) { fail(); ok = false; }
             else {
-                tc_fence_after();
                 issue_s(0, 0);
                 issue_s(1, 0);
+                tc_commit(&bar.slot_empty[0]);
             }
         }
         for (int j = 0; ok && j < ntiles && !*abort_flag; ++j) {
@@ -285,15 +270,13 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
             for (int t = 0; t < 2; ++t) {
                 if (!issue_pv(t, j)) { fail(); ok = false; break; }
                 if (more) {
-                    if (t == 0 && !mbar_wait(&bar.kv_full[(j + 1) % kStages], ((j + 1) / kStages) & 1)) {
-                        fail(); ok = false; break;
-                    }
-                    tc_fence_after();
+                    if (t == 0 && !slot_ready(2 * j + 2)) { fail(); ok = false; break; }
                     issue_s(t, j + 1);
                 }
             }
             if (!ok) break;
-            tc_commit(&bar.kv_empty[j % kStages]);
+            tc_commit(&bar.slot_empty[(2 * j + 1) % S]);
+            if (more) tc_commit(&bar.slot_empty[(2 * j + 2) % S]);
         }
         if (ok) {
             tc_commit(&bar.o_last[0]);
@@ -346,13 +329,7 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
 #pragma unroll
             for (int i = 0; i < kBN; i += 2) {
                 const float2 x = __ffma2_rn(make_float2(__uint_as_float(sr[i]), __uint_as_float(sr[i + 1])), c2, nm2);
-                float2 e;
-                if (i < kSwExp) {
-                    e = exp2_poly2(x);
-                } else {
-                    e.x = ex2(x.x);
-                    e.y = ex2(x.y);
-                }
+                const float2 e = make_float2(ex2(x.x), ex2(x.y));
                 acc[(i >> 1) & 3] = __fadd2_rn(acc[(i >> 1) & 3], e);
                 sr[i / 2] = pack_bf16x2(e.x, e.y);   // P packed over the front of the S registers
             }
@@ -419,12 +396,6 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
         tc_fence_after();
         tmem_dealloc(tmem, C::kTmemCols);
     }
-}
-
-__global__ void exp2_poly_kernel(const float2* x, float2* y, int64_t n2) {
-    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n2;
-         i += static_cast<int64_t>(gridDim.x) * blockDim.x)
-        y[i] = exp2_poly2(x[i]);
 }
 
 template <int HD>
@@ -510,15 +481,3 @@ int attention(const AttnSegment& s0, const AttnSegment& s1, int B, int heads, in
 }
 
 }  // namespace ff
-
-extern "C" int ff_debug_exp2(const float* x, float* y, int64_t n, cudaStream_t stream) {
-    using namespace ff;
-    if (!x || !y || n <= 0 || n % 2 || !aligned16(x) || !aligned16(y))
-        return set_error(FF_ERR_INVALID_ARG, "exp2: bad arguments (n even, 16-byte aligned arrays)");
-    const int64_t n2 = n / 2;
-    int64_t grid = (n2 + 255) / 256;
-    if (grid > 4096) grid = 4096;
-    exp2_poly_kernel<<<static_cast<unsigned>(grid), 256, 0, stream>>>(reinterpret_cast<const float2*>(x),
-                                                                       reinterpret_cast<float2*>(y), n2);
-    return check_launch("exp2_poly_kernel");
-}

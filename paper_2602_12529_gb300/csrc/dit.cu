@@ -463,12 +463,14 @@ int ff_dit_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, c
     // ---- patch and text embeddings into the residual stream
     FF_TRY(f32_to_bf16(x_t, w.xb, static_cast<int64_t>(Ri) * P, stream));
     {
+        // the long-K text product first, so its few expensive tiles start at
+        // once and the short patch-embedding tiles fill in behind them
         GemmArgs g[2];
-        g[0] = GemmArgs{w.xb, P, W("img_in.w"), P, Ri, H, P, GemmEpilogue{}};
-        g[0].epi.out_f32 = 1; g[0].epi.bias = W("img_in.b"); g[0].epi.out0 = w.x + static_cast<int64_t>(Rt) * H;
-        g[0].epi.ld0 = H;
-        g[1] = GemmArgs{txt, c.txt_dim, W("txt_in.w"), c.txt_dim, Rt, H, c.txt_dim, GemmEpilogue{}};
-        g[1].epi.out_f32 = 1; g[1].epi.bias = W("txt_in.b"); g[1].epi.out0 = w.x; g[1].epi.ld0 = H;
+        g[0] = GemmArgs{txt, c.txt_dim, W("txt_in.w"), c.txt_dim, Rt, H, c.txt_dim, GemmEpilogue{}};
+        g[0].epi.out_f32 = 1; g[0].epi.bias = W("txt_in.b"); g[0].epi.out0 = w.x; g[0].epi.ld0 = H;
+        g[1] = GemmArgs{w.xb, P, W("img_in.w"), P, Ri, H, P, GemmEpilogue{}};
+        g[1].epi.out_f32 = 1; g[1].epi.bias = W("img_in.b"); g[1].epi.out0 = w.x + static_cast<int64_t>(Rt) * H;
+        g[1].epi.ld0 = H;
         FF_TRY(gemm_bf16_group(g, 2, stream));
     }
 

@@ -11,8 +11,10 @@
 //   warps 2..5  epilogue: tcgen05.ld of the accumulator (one TMEM lane = one
 //               output row per thread), then the fused tail -- bias, GELU or
 //               SiLU, and either a bf16/fp32 store (optionally split over two
-//               outputs by column) or the adaLN gated residual update
-//               x += gate[b] * (acc + bias) on the fp32 residual stream.
+//               outputs by column; each warp stages 32 x 32 blocks in shared
+//               memory and writes them with TMA bulk stores) or the adaLN
+//               gated residual update x += gate[b] * (acc + bias) on the fp32
+//               residual stream.
 // The two TMEM accumulators let the epilogue of tile i overlap the main loop
 // of tile i+1.  Tiles are visited in groups of 16 M-blocks so that the A and
 // B panels being read at any moment stay resident in L2.
@@ -205,48 +207,44 @@ __device__ __forceinline__ void epilogue_values(const GemmEpilogue& e, int n, fl
 // (row r at st[r * 33 ...]) as row segments: fp32 with 8 lanes x float4 per
 // row (4 rows per instruction), bf16 with 4 lanes x 8 values per row (8 rows
 // per instruction).
-__device__ __forceinline__ void store_rows(const GemmEpilogue& e, int M, int row0, int n, int lane, const float* st) {
-    void* base;
-    int64_t ld;
-    int col;
-    if (n < e.split_n) {
-        base = e.out0; ld = e.ld0; col = n;
-    } else {
-        base = e.out1; ld = e.ld1; col = n - e.split_n + e.col1;
-    }
-    if (e.out_f32) {
-        const int cq = lane & 7, rs = lane >> 3;
+// Output maps of a launch: problem i stores columns [0, split_n) through
+// m[2 i] and columns [split_n, N) through m[2 i + 1] (based at out1 + col1).
+struct OutMaps {
+    CUtensorMap m[4];
+};
+
+// One 32 x 32 output block of this warp (lane = row) into its shared staging
+// buffer, in the swizzled layout of the output map: fp32 rows of 128 bytes
+// (16-byte piece j of row r at j ^ (r % 8)), bf16 rows of 64 bytes (piece j at
+// j ^ ((r / 2) % 4)).  Either way the 8 lanes of a store phase hit distinct
+// banks.
+__device__ __forceinline__ void stage_chunk(bool f32, int lane, const float (&v)[32], uint8_t* buf) {
+    if (f32) {
+        uint8_t* row = buf + lane * 128;
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            const int r = rs + 4 * j;
-            const float* a = st + r * 33 + 4 * cq;
-            if (row0 + r < M)
-                *reinterpret_cast<float4*>(static_cast<float*>(base) + static_cast<int64_t>(row0 + r) * ld + col + 4 * cq) =
-                    make_float4(a[0], a[1], a[2], a[3]);
-        }
+        for (int j = 0; j < 8; ++j)
+            *reinterpret_cast<float4*>(row + ((j ^ (lane & 7)) << 4)) =
+                make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
     } else {
-        const int cq = lane & 3, rs = lane >> 2;
+        uint8_t* row = buf + lane * 64;
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            const int r = rs + 8 * j;
-            const float* a = st + r * 33 + 8 * cq;
-            if (row0 + r < M)
-                *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(base) + static_cast<int64_t>(row0 + r) * ld + col +
-                                          8 * cq) =
-                    make_uint4(pack_bf16x2(a[0], a[1]), pack_bf16x2(a[2], a[3]), pack_bf16x2(a[4], a[5]),
-                               pack_bf16x2(a[6], a[7]));
-        }
+        for (int j = 0; j < 4; ++j)
+            *reinterpret_cast<uint4*>(row + ((j ^ ((lane >> 1) & 3)) << 4)) =
+                make_uint4(pack_bf16x2(v[8 * j], v[8 * j + 1]), pack_bf16x2(v[8 * j + 2], v[8 * j + 3]),
+                           pack_bf16x2(v[8 * j + 4], v[8 * j + 5]), pack_bf16x2(v[8 * j + 6], v[8 * j + 7]));
     }
 }
 
 // One tile of the epilogue for the 128 rows m0.. held in this CTA's TMEM
-// (t_acc: this warp's lane quarter of the accumulator).  Returns false after
-// a bounded wait gave up.
+// (t_acc: this warp's lane quarter of the accumulator).  `to` are the
+// problem's two output maps and `sc` counts this warp's output blocks (its
+// two staging buffers alternate).  Returns false after a bounded wait gave up.
 template <int BN>
 __device__ __forceinline__ bool epilogue_tile(const GemmEpilogue& epi, int M, int N, int m0, int nb, uint32_t t_acc,
                                               int q, int lane, int warp, bool leader, const CUtensorMap* tr,
-                                              uint8_t* rbuf, uint64_t* rfull_bar, uint64_t* rdone_bar,
-                                              uint32_t (&ruse)[2], int* status, volatile int* abort_flag) {
+                                              const CUtensorMap* to, uint8_t* rbuf, uint64_t* rfull_bar,
+                                              uint64_t* rdone_bar, uint32_t (&ruse)[2], uint32_t& sc, int* status,
+                                              volatile int* abort_flag) {
     using C = Cfg<BN>;
     const bool gated = epi.epi == EPI_GATED_RESIDUAL;
     const int r = q * 32 + lane;                // row within the tile = TMEM lane
@@ -297,27 +295,35 @@ __device__ __forceinline__ bool epilogue_tile(const GemmEpilogue& epi, int M, in
     } else if (epi.qk_cols > 0 && nb * BN < epi.qk_cols) {
         qk_norm_tile(epi, M, row, nb * BN, t_acc, BN);
     } else {
-        // plain store: bias / activation on the row held by this
-        // thread, then a transpose through this warp's 32x33 shared
-        // tile so that the global stores are whole row segments
-        float* st = reinterpret_cast<float*>(rbuf) + (warp - 2) * (32 * 33);
+        // plain store: bias / activation on the row held by this thread,
+        // staged as a 32 x 32 block and written by a TMA bulk store (rows
+        // past M are clipped by the map); the warp's two staging buffers
+        // alternate, so the block before last must have been read out first
+        uint8_t* stage = rbuf + (warp - 2) * 8192;
         const int row0 = m0 + q * 32;
 #pragma unroll 1
         for (int c = 0; c < BN; c += 32) {
+            const int n = nb * BN + c;
+            if (n >= N) break;
             uint32_t rr[32];
             tmem_ld_x32(t_acc + c, rr);
             tmem_ld_wait();
-            const int n = nb * BN + c;
-            if (n >= N) continue;
             float v[32];
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(rr[i]);
             epilogue_values(epi, n, v);
-#pragma unroll
-            for (int i = 0; i < 32; ++i) st[lane * 33 + i] = v[i];
+            uint8_t* buf = stage + (sc & 1) * 4096;
+            if (lane == 0) bulk_wait_read<1>();
             __syncwarp();
-            store_rows(epi, M, row0, n, lane, st);
+            stage_chunk(epi.out_f32 != 0, lane, v, buf);
+            fence_proxy_async_smem();
             __syncwarp();
+            if (lane == 0) {
+                if (n < epi.split_n) tma_store_2d(&to[0], buf, n, row0);
+                else tma_store_2d(&to[1], buf, n - epi.split_n, row0);
+                bulk_commit();
+            }
+            ++sc;
         }
     }
     return true;
@@ -344,7 +350,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_constant__ CUtensorMap tm_b0,
                     const __grid_constant__ CUtensorMap tm_a1, const __grid_constant__ CUtensorMap tm_b1,
                     const __grid_constant__ CUtensorMap tm_r0, const __grid_constant__ CUtensorMap tm_r1,
-                    const __grid_constant__ GemmGroup g, int* status) {
+                    const __grid_constant__ OutMaps om, const __grid_constant__ GemmGroup g, int* status) {
     using C = Cfg<BN>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -469,6 +475,7 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_cons
         const int q = warp & 3;
         const bool leader = warp == 2 && lane == 0;     // issues the residual TMA traffic
         uint32_t ruse[2] = {0, 0};                      // residual loads consumed per buffer
+        uint32_t sc = 0;                                // output blocks staged by this warp
         const uint32_t t_acc_base = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
         int acc = 0;
         uint32_t acc_phase = 0;
@@ -494,14 +501,15 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_cons
             }
             tc_fence_after();
             if (!epilogue_tile<BN>(epi, M, N, mb * BM, nb, t_acc_base + static_cast<uint32_t>(acc * BN), q, lane, warp,
-                                   leader, tr, rbuf, rfull_bar, rdone_bar, ruse, status, abort_flag))
+                                   leader, tr, &om.m[2 * pr], rbuf, rfull_bar, rdone_bar, ruse, sc, status,
+                                   abort_flag))
                 break;
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&tempty_bar[acc]);
             if (++acc == 2) { acc = 0; acc_phase ^= 1; }
         }
-        if (leader) bulk_wait<0>();   // residual stores complete before the CTA's shared memory goes away
+        if (lane == 0) bulk_wait<0>();   // this warp's stores complete before the CTA's shared memory goes away
     }
 
     if (*abort_flag) {
@@ -547,7 +555,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_constant__ CUtensorMap tm_b0,
                  const __grid_constant__ CUtensorMap tm_a1, const __grid_constant__ CUtensorMap tm_b1,
                  const __grid_constant__ CUtensorMap tm_r0, const __grid_constant__ CUtensorMap tm_r1,
-                 const __grid_constant__ GemmGroup g, int* status) {
+                 const __grid_constant__ OutMaps om, const __grid_constant__ GemmGroup g, int* status) {
     using C = PairCfg;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -671,6 +679,7 @@ gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_constan
         const int q = warp & 3;
         const bool leader = warp == 2 && lane == 0;
         uint32_t ruse[2] = {0, 0};
+        uint32_t sc = 0;
         const uint32_t t_acc_base = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
         int acc = 0;
         uint32_t acc_phase = 0;
@@ -695,14 +704,15 @@ gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_constan
             }
             tc_fence_after();
             if (!epilogue_tile<PBN>(epi, M, N, m0, nb, t_acc_base + static_cast<uint32_t>(acc * PBN), q, lane, warp,
-                                    leader, tr, rbuf, rfull_bar, rdone_bar, ruse, status, abort_flag))
+                                    leader, tr, &om.m[2 * pr], rbuf, rfull_bar, rdone_bar, ruse, sc, status,
+                                    abort_flag))
                 break;
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive_cluster(mapa_shared(smem_u32(&tempty_bar[acc]), 0));
             if (++acc == 2) { acc = 0; acc_phase ^= 1; }
         }
-        if (leader) bulk_wait<0>();
+        if (lane == 0) bulk_wait<0>();
     }
 
     if (*abort_flag) {
@@ -718,17 +728,43 @@ gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_constan
     }
 }
 
+// The two output maps of a store epilogue.  A gated-residual problem stores
+// through its residual map instead; its entries (and an unsplit problem's
+// second one) are copies of a valid map, so every kernel parameter is a
+// well-formed tensor map.
+int make_out_maps(const GemmArgs& a, CUtensorMap* m) {
+    const GemmEpilogue& e = a.epi;
+    if (e.epi == EPI_GATED_RESIDUAL) {
+        const int rc = make_tmap_f32_sw128(&m[0], e.resid, a.M, a.N, e.ld_resid, 128);
+        m[1] = m[0];
+        return rc;
+    }
+    const bool f32 = e.out_f32 != 0;
+    const int n0 = e.split_n < a.N ? e.split_n : a.N;
+    int rc = make_tmap_out(&m[0], e.out0, a.M, n0, e.ld0, f32);
+    if (rc) return rc;
+    if (e.split_n < a.N) {
+        const uint8_t* base1 = static_cast<const uint8_t*>(e.out1) + static_cast<int64_t>(e.col1) * (f32 ? 4 : 2);
+        return make_tmap_out(&m[1], base1, a.M, a.N - e.split_n, e.ld1, f32);
+    }
+    m[1] = m[0];
+    return FF_OK;
+}
+
 int launch_pair(const GemmArgs* p, int n, cudaStream_t stream) {
     using C = PairCfg;
     if (cudaFuncSetAttribute(gemm_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes) !=
         cudaSuccess)
         return set_error(FF_ERR_CUDA, "gemm (pair): cannot set shared memory size (%d B)", C::kSmemBytes);
     CUtensorMap ta[2], tb[2], tr[2];
+    OutMaps om;
     GemmGroup g{};
     double flops = 0.0, bytes = 0.0;
     for (int i = 0; i < 2; ++i) {
         const GemmArgs& a = p[i < n ? i : 0];
-        int rc = make_tmap_bf16(&ta[i], a.A, a.M, a.K, a.lda, 128);
+        int rc = make_out_maps(a, &om.m[2 * i]);
+        if (rc) return rc;
+        rc = make_tmap_bf16(&ta[i], a.A, a.M, a.K, a.lda, 128);
         if (rc) return rc;
         rc = make_tmap_bf16(&tb[i], a.B, a.N, a.K, a.ldb, PBN / 2);
         if (rc) return rc;
@@ -758,8 +794,8 @@ int launch_pair(const GemmArgs* p, int n, cudaStream_t stream) {
     g.tiles = g.tiles0 + (n > 1 ? g.num_m[1] * g.num_n[1] : 0);
     const int clusters = g.tiles < num_sms() / 2 ? g.tiles : num_sms() / 2;
     ProfScope prof(stream, "gemm_bf16", flops, bytes);
-    gemm_pair_kernel<<<2 * clusters, kThreads, C::kSmemBytes, stream>>>(ta[0], tb[0], ta[1], tb[1], tr[0], tr[1], g,
-                                                                        device_status_ptr());
+    gemm_pair_kernel<<<2 * clusters, kThreads, C::kSmemBytes, stream>>>(ta[0], tb[0], ta[1], tb[1], tr[0], tr[1], om,
+                                                                        g, device_status_ptr());
     return check_launch("gemm_pair_kernel");
 }
 
@@ -770,11 +806,14 @@ int launch(const GemmArgs* p, int n, cudaStream_t stream) {
         cudaSuccess)
         return set_error(FF_ERR_CUDA, "gemm: cannot set shared memory size (%d B)", C::kSmemBytes);
     CUtensorMap ta[2], tb[2], tr[2];
+    OutMaps om;
     GemmGroup g{};
     double flops = 0.0, bytes = 0.0;
     for (int i = 0; i < 2; ++i) {
         const GemmArgs& a = p[i < n ? i : 0];
-        int rc = make_tmap_bf16(&ta[i], a.A, a.M, a.K, a.lda, BM);
+        int rc = make_out_maps(a, &om.m[2 * i]);
+        if (rc) return rc;
+        rc = make_tmap_bf16(&ta[i], a.A, a.M, a.K, a.lda, BM);
         if (rc) return rc;
         rc = make_tmap_bf16(&tb[i], a.B, a.N, a.K, a.ldb, BN);
         if (rc) return rc;
@@ -804,8 +843,8 @@ int launch(const GemmArgs* p, int n, cudaStream_t stream) {
     for (int i = 0; i < n; ++i)
         if (p[i].epi.epi == EPI_GATED_RESIDUAL && p[i].N % BN)
             return set_error(FF_ERR_UNSUPPORTED, "gemm: gated residual needs N (%d) to be a multiple of %d", p[i].N, BN);
-    gemm_tcgen05_kernel<BN><<<grid, kThreads, C::kSmemBytes, stream>>>(ta[0], tb[0], ta[1], tb[1], tr[0], tr[1], g,
-                                                                       device_status_ptr());
+    gemm_tcgen05_kernel<BN><<<grid, kThreads, C::kSmemBytes, stream>>>(ta[0], tb[0], ta[1], tb[1], tr[0], tr[1], om,
+                                                                       g, device_status_ptr());
     return check_launch("gemm_tcgen05_kernel");
 }
 

@@ -34,6 +34,9 @@ struct ProfScope {
 int make_tmap_bf16(CUtensorMap* tm, const void* base, int64_t rows, int64_t cols, int64_t ld, int box_rows);
 // 2-D fp32 matrix, box = box_rows x 32 columns (128 bytes), 128-byte swizzle.
 int make_tmap_f32_sw128(CUtensorMap* tm, const void* base, int64_t rows, int64_t cols, int64_t ld, int box_rows);
+// GEMM output tile store map: box = 32 rows x 32 columns of fp32 (128-byte
+// swizzle) or bf16 (64-byte swizzle).
+int make_tmap_out(CUtensorMap* tm, const void* base, int64_t rows, int64_t cols, int64_t ld, bool f32);
 
 // ---- GEMM: D[M, N] = A[M, K] B[N, K]^T with a fused epilogue --------------
 enum GemmAct { ACT_NONE = 0, ACT_GELU = 1, ACT_SILU = 2 };

@@ -94,6 +94,29 @@ int make_tmap_f32_sw128(CUtensorMap* tm, const void* base, int64_t rows, int64_t
     return FF_OK;
 }
 
+int make_tmap_out(CUtensorMap* tm, const void* base, int64_t rows, int64_t cols, int64_t ld, bool f32) {
+    if (!g_encode) {
+        CUtensorMap dummy;
+        const int rc = make_tmap_bf16(&dummy, base, 1, 8, 8, 1);   // resolves the driver entry point
+        if (rc) return rc;
+    }
+    const int es = f32 ? 4 : 2;
+    if (!aligned16(base)) return set_error(FF_ERR_INVALID_ARG, "tensor map base not 16-byte aligned");
+    if ((ld * es) % 16) return set_error(FF_ERR_INVALID_ARG, "tensor map row pitch not a multiple of 16 bytes");
+    const cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld) * es};
+    const cuuint32_t box[2] = {32, 32};
+    const cuuint32_t estr[2] = {1, 1};
+    const CUresult r = g_encode(tm, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                                const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                                f32 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B,
+                                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS)
+        return set_error(FF_ERR_CUDA, "cuTensorMapEncodeTiled (output) failed (%d) rows=%lld cols=%lld ld=%lld",
+                         (int)r, (long long)rows, (long long)cols, (long long)ld);
+    return FF_OK;
+}
+
 int make_tmap_bf16(CUtensorMap* tm, const void* base, int64_t rows, int64_t cols, int64_t ld, int box_rows) {
     if (!g_encode) {
         std::lock_guard<std::mutex> lk(g_mu);

@@ -70,7 +70,6 @@ _SIGS = {
     "ff_debug_gemm_gated": ([_I, _I, _I, _P, _I64, _P, _I64, _P, _P, _I64, _P, _I64, _I, _P], _I),
     "ff_debug_attention": ([_I, _I, _I, _I, _P, _I64, _P, _I64, _I, _P, _I64, _P, _I64, _P], _I),
     "ff_debug_ln_modulate": ([_I, _I, _P, _P, _I64, _I, _I, _I, _P, _P], _I),
-    "ff_debug_exp2": ([_P, _P, _I64, _P], _I),
     "ff_debug_qk_norm_rope": ([_I, _I, _I, _I, _P, _I64, _P, _P, _I, _I, _I, C.POINTER(_I), _F, _P], _I),
 }
 
@@ -334,6 +333,3 @@ def ff_debug_qk_norm_rope(qkv, rows_txt, heads, head_dim, q_scale, k_scale, grid
     _call("ff_debug_qk_norm_rope", qkv.shape[0], rows_txt, heads, head_dim, _ptr(qkv), qkv.shape[-1],
           _ptr(q_scale), _ptr(k_scale), grid[0], grid[1], grid[2], axes, theta, _stream(stream))
 
-
-def ff_debug_exp2(x, y, stream=None):
-    _call("ff_debug_exp2", _ptr(x), _ptr(y), x.numel(), _stream(stream))
