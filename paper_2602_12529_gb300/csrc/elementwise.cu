@@ -1,6 +1,7 @@
 // elementwise.cu -- the row-wise kernels of the DiT velocity:
 //   * ln_modulate: LayerNorm (no affine, eps 1e-6) then x (1 + scale) + shift
-//     with the sample's adaLN vectors, fp32 in -> bf16 GEMM operand out;
+//     with the sample's adaLN vectors (or an affine LayerNorm), fp32 in ->
+//     bf16 GEMM operand out;
 //   * qk_norm_rope: per-head RMSNorm of q and k (learned scale, eps 1e-6)
 //     and the rotary embedding over (frame, row, col) slices of the head
 //     dim, in place on the bf16 qkv buffer;
@@ -21,13 +22,27 @@ __device__ __forceinline__ float warp_sum(float v) {
     return v;
 }
 
-// One warp per row; H % 128 == 0 so every lane owns H/128 float4s.  The row
-// is read three times (sum, centred sum of squares, output); the second and
-// third reads hit L1.
-__global__ void __launch_bounds__(256) ln_modulate_kernel(LnModArgs a) {
-    const int row = (blockIdx.x * 256 + threadIdx.x) >> 5;
-    const int lane = threadIdx.x & 31;
-    if (row >= a.rows) return;
+// One CTA of 256 threads per row; thread t holds the float4s t, t + 256, ...
+// of the row in registers (PER of them, H <= 1024 PER), so x is read once:
+// the mean and the centred sum of squares come from the registers, reduced
+// over the CTA through shared memory.
+constexpr int kLnThreads = 256;
+
+__device__ __forceinline__ float block_sum(float v, float* red, int lane, int w) {
+    v = warp_sum(v);
+    if (lane == 0) red[w] = v;
+    __syncthreads();
+    float t = 0.f;
+#pragma unroll
+    for (int i = 0; i < kLnThreads / 32; ++i) t += red[i];
+    return t;
+}
+
+template <int PER>
+__global__ void __launch_bounds__(kLnThreads) ln_modulate_kernel(LnModArgs a) {
+    __shared__ float red[2][kLnThreads / 32];
+    const int row = blockIdx.x;
+    const int t = threadIdx.x, lane = t & 31, w = t >> 5;
     int b, sh, sc;
     if (row < a.rows_txt) {
         b = row / a.n_txt;
@@ -40,45 +55,57 @@ __global__ void __launch_bounds__(256) ln_modulate_kernel(LnModArgs a) {
     }
     const float4* x = reinterpret_cast<const float4*>(a.x + static_cast<int64_t>(row) * a.ldx);
     const int nv = a.H >> 2;
+    float4 r[PER];
+#pragma unroll
+    for (int i = 0; i < PER; ++i) {
+        const int k = t + kLnThreads * i;
+        r[i] = k < nv ? __ldcs(x + k) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
     float s = 0.f;
-    for (int i = lane; i < nv; i += 32) {
-        const float4 v = x[i];
-        s += (v.x + v.y) + (v.z + v.w);
-    }
-    const float mean = warp_sum(s) / a.H;
+#pragma unroll
+    for (int i = 0; i < PER; ++i) s += (r[i].x + r[i].y) + (r[i].z + r[i].w);
+    const float mean = block_sum(s, red[0], lane, w) / a.H;
     float q = 0.f;
-    for (int i = lane; i < nv; i += 32) {
-        const float4 v = x[i];
-        const float d0 = v.x - mean, d1 = v.y - mean, d2 = v.z - mean, d3 = v.w - mean;
-        q += (d0 * d0 + d1 * d1) + (d2 * d2 + d3 * d3);
+#pragma unroll
+    for (int i = 0; i < PER; ++i) {
+        if (t + kLnThreads * i < nv) {
+            const float d0 = r[i].x - mean, d1 = r[i].y - mean, d2 = r[i].z - mean, d3 = r[i].w - mean;
+            q += (d0 * d0 + d1 * d1) + (d2 * d2 + d3 * d3);
+        }
     }
-    const float rstd = rsqrtf(warp_sum(q) / a.H + kLnEps);
+    const float rstd = rsqrtf(block_sum(q, red[1], lane, w) / a.H + kLnEps);
     uint2* out = reinterpret_cast<uint2*>(a.out + static_cast<int64_t>(row) * a.ldo);
     if (a.aff_w) {
         // affine LayerNorm: LN(x) w + b
         const uint2* w2 = reinterpret_cast<const uint2*>(a.aff_w);
         const uint2* b2 = reinterpret_cast<const uint2*>(a.aff_b);
-        for (int i = lane; i < nv; i += 32) {
-            const float4 v = x[i];
-            const uint2 wu = w2[i], bu = b2[i];
+#pragma unroll
+        for (int i = 0; i < PER; ++i) {
+            const int k = t + kLnThreads * i;
+            if (k >= nv) break;
+            const float4 v = r[i];
+            const uint2 wu = w2[k], bu = b2[k];
             const float2 w0 = unpack_bf16x2(wu.x), w1 = unpack_bf16x2(wu.y);
             const float2 b0 = unpack_bf16x2(bu.x), b1 = unpack_bf16x2(bu.y);
-            out[i] = make_uint2(pack_bf16x2((v.x - mean) * rstd * w0.x + b0.x, (v.y - mean) * rstd * w0.y + b0.y),
+            out[k] = make_uint2(pack_bf16x2((v.x - mean) * rstd * w0.x + b0.x, (v.y - mean) * rstd * w0.y + b0.y),
                                 pack_bf16x2((v.z - mean) * rstd * w1.x + b1.x, (v.w - mean) * rstd * w1.y + b1.y));
         }
         return;
     }
     const float4* shift = reinterpret_cast<const float4*>(a.mods + static_cast<int64_t>(b) * a.ld_mods + sh);
     const float4* scale = reinterpret_cast<const float4*>(a.mods + static_cast<int64_t>(b) * a.ld_mods + sc);
-    for (int i = lane; i < nv; i += 32) {
-        const float4 v = x[i];
-        const float4 h = shift[i];
-        const float4 c = scale[i];
+#pragma unroll
+    for (int i = 0; i < PER; ++i) {
+        const int k = t + kLnThreads * i;
+        if (k >= nv) break;
+        const float4 v = r[i];
+        const float4 h = shift[k];
+        const float4 c = scale[k];
         const float y0 = (v.x - mean) * rstd * (1.f + c.x) + h.x;
         const float y1 = (v.y - mean) * rstd * (1.f + c.y) + h.y;
         const float y2 = (v.z - mean) * rstd * (1.f + c.z) + h.z;
         const float y3 = (v.w - mean) * rstd * (1.f + c.w) + h.w;
-        out[i] = make_uint2(pack_bf16x2(y0, y1), pack_bf16x2(y2, y3));
+        out[k] = make_uint2(pack_bf16x2(y0, y1), pack_bf16x2(y2, y3));
     }
 }
 
@@ -225,9 +252,19 @@ int ln_modulate(const LnModArgs& a, cudaStream_t stream) {
     if (a.rows <= 0) return FF_OK;
     if (a.H % 128 || a.ldx % 4 || a.ldo % 4 || a.ld_mods % 4 || (a.shift_txt | a.scale_txt | a.shift_img | a.scale_img) % 4)
         return set_error(FF_ERR_UNSUPPORTED, "ln_modulate: H=%d must be a multiple of 128", a.H);
-    const int grid = (a.rows + 7) / 8;
+    const int per = (a.H / 4 + kLnThreads - 1) / kLnThreads;   // float4s per thread
     ProfScope prof(stream, "ln_modulate", 0.0, static_cast<double>(a.rows) * a.H * 6.0);
-    ln_modulate_kernel<<<grid, 256, 0, stream>>>(a);
+    switch (per) {
+        case 1: ln_modulate_kernel<1><<<a.rows, kLnThreads, 0, stream>>>(a); break;
+        case 2: ln_modulate_kernel<2><<<a.rows, kLnThreads, 0, stream>>>(a); break;
+        case 3: ln_modulate_kernel<3><<<a.rows, kLnThreads, 0, stream>>>(a); break;
+        case 4: ln_modulate_kernel<4><<<a.rows, kLnThreads, 0, stream>>>(a); break;
+        case 5: ln_modulate_kernel<5><<<a.rows, kLnThreads, 0, stream>>>(a); break;
+        case 6: ln_modulate_kernel<6><<<a.rows, kLnThreads, 0, stream>>>(a); break;
+        case 7: ln_modulate_kernel<7><<<a.rows, kLnThreads, 0, stream>>>(a); break;
+        case 8: ln_modulate_kernel<8><<<a.rows, kLnThreads, 0, stream>>>(a); break;
+        default: return set_error(FF_ERR_UNSUPPORTED, "ln_modulate: H=%d above 8192", a.H);
+    }
     return check_launch("ln_modulate_kernel");
 }
 

@@ -42,7 +42,9 @@ struct Cfg {
     static constexpr int kTmemCols = 2 * BN;
     static constexpr int kBarrierBytes = 256;
     static constexpr int kResidBytes = BM * 32 * 4;   // one 128 x 32 fp32 residual chunk (two buffers)
-    static constexpr int kSmemBytes = kStages * kStageBytes + 2 * kResidBytes + 1024 + kBarrierBytes;
+    static constexpr int kEpiBytes = 2 * kResidBytes;  // epilogue staging: residual chunks or output blocks
+    static constexpr int kStageBufs = kEpiBytes / (4 * 4096);   // 4 KB output blocks per epilogue warp
+    static constexpr int kSmemBytes = kStages * kStageBytes + kEpiBytes + 1024 + kBarrierBytes;
 };
 
 __device__ __forceinline__ void tile_coords(int tile, int num_m, int num_n, int& mb, int& nb) {
@@ -186,11 +188,25 @@ __device__ __forceinline__ void qk_norm_tile(const GemmEpilogue& e, int M, int r
     }
 }
 
+// Bias of a 32-column chunk (bf16 pairs), loaded ahead of its use.
+__device__ __forceinline__ void load_bias32(const __nv_bfloat16* bias, int n, uint4 (&u)[4]) {
+#pragma unroll
+    for (int j = 0; j < 4; ++j) u[j] = bias ? reinterpret_cast<const uint4*>(bias + n)[j] : make_uint4(0, 0, 0, 0);
+}
+
 // Bias and activation of one 32-column chunk of the row held by this thread.
-__device__ __forceinline__ void epilogue_values(const GemmEpilogue& e, int n, float (&v)[32]) {
+__device__ __forceinline__ void epilogue_values(const GemmEpilogue& e, int n, const uint4 (&bu)[4], float (&v)[32]) {
     if (e.bias) {
 #pragma unroll
-        for (int j = 0; j < 4; ++j) bias_add8(v + 8 * j, e.bias + n + 8 * j);
+        for (int j = 0; j < 4; ++j) {
+            const uint32_t w[4] = {bu[j].x, bu[j].y, bu[j].z, bu[j].w};
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const float2 f = unpack_bf16x2(w[i]);
+                v[8 * j + 2 * i] += f.x;
+                v[8 * j + 2 * i + 1] += f.y;
+            }
+        }
     }
     if (e.act != ACT_NONE && n >= e.act_from) {
         if (e.act == ACT_GELU) {
@@ -203,10 +219,6 @@ __device__ __forceinline__ void epilogue_values(const GemmEpilogue& e, int n, fl
     }
 }
 
-// Stores a warp's 32 rows x 32 columns from its transposed shared tile st
-// (row r at st[r * 33 ...]) as row segments: fp32 with 8 lanes x float4 per
-// row (4 rows per instruction), bf16 with 4 lanes x 8 values per row (8 rows
-// per instruction).
 // Output maps of a launch: problem i stores columns [0, split_n) through
 // m[2 i] and columns [split_n, N) through m[2 i + 1] (based at out1 + col1).
 struct OutMaps {
@@ -237,9 +249,10 @@ __device__ __forceinline__ void stage_chunk(bool f32, int lane, const float (&v)
 
 // One tile of the epilogue for the 128 rows m0.. held in this CTA's TMEM
 // (t_acc: this warp's lane quarter of the accumulator).  `to` are the
-// problem's two output maps and `sc` counts this warp's output blocks (its
-// two staging buffers alternate).  Returns false after a bounded wait gave up.
-template <int BN>
+// problem's two output maps; the warp owns SB staging blocks of 4 KB and `sc`
+// counts its store steps, which rotate through them.  Returns false after a
+// bounded wait gave up.
+template <int BN, int SB>
 __device__ __forceinline__ bool epilogue_tile(const GemmEpilogue& epi, int M, int N, int m0, int nb, uint32_t t_acc,
                                               int q, int lane, int warp, bool leader, const CUtensorMap* tr,
                                               const CUtensorMap* to, uint8_t* rbuf, uint64_t* rfull_bar,
@@ -296,31 +309,62 @@ __device__ __forceinline__ bool epilogue_tile(const GemmEpilogue& epi, int M, in
         qk_norm_tile(epi, M, row, nb * BN, t_acc, BN);
     } else {
         // plain store: bias / activation on the row held by this thread,
-        // staged as a 32 x 32 block and written by a TMA bulk store (rows
-        // past M are clipped by the map); the warp's two staging buffers
-        // alternate, so the block before last must have been read out first
-        uint8_t* stage = rbuf + (warp - 2) * 8192;
+        // staged as 32 x 32 blocks and written by TMA bulk stores (rows past
+        // M are clipped by the map).  A step covers CW columns (two blocks
+        // when the warp has room to double-buffer them, which halves the
+        // per-step fence / sync / issue cost); the next step's accumulator
+        // columns and bias are requested before this step is processed, and
+        // a staging buffer is reused once the store NB steps back has read it
+        // out.
+        constexpr int CW = SB >= 4 ? 64 : 32;
+        constexpr int NB = SB * 32 / CW;
+        uint8_t* stage = rbuf + (warp - 2) * (SB * 4096);
         const int row0 = m0 + q * 32;
-#pragma unroll 1
-        for (int c = 0; c < BN; c += 32) {
-            const int n = nb * BN + c;
-            if (n >= N) break;
-            uint32_t rr[32];
-            tmem_ld_x32(t_acc + c, rr);
-            tmem_ld_wait();
-            float v[32];
+        const int ncol = N - nb * BN < BN ? N - nb * BN : BN;   // a multiple of 32
+        uint32_t rr[CW];
+        uint4 bnext[CW / 8];
+        auto fetch = [&](int c) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(rr[i]);
-            epilogue_values(epi, n, v);
-            uint8_t* buf = stage + (sc & 1) * 4096;
-            if (lane == 0) bulk_wait_read<1>();
+            for (int k = 0; k < CW / 32; ++k)
+                if (c + 32 * k < ncol) {
+                    tmem_ld_x32(t_acc + c + 32 * k, *reinterpret_cast<uint32_t(*)[32]>(&rr[32 * k]));
+                    load_bias32(epi.bias, nb * BN + c + 32 * k, *reinterpret_cast<uint4(*)[4]>(&bnext[4 * k]));
+                }
+        };
+        fetch(0);
+#pragma unroll 1
+        for (int c = 0; c < ncol; c += CW) {
+            const int nblk = ncol - c < CW ? 1 : CW / 32;
+            tmem_ld_wait();
+            float v[CW];
+#pragma unroll
+            for (int i = 0; i < CW; ++i) v[i] = __uint_as_float(rr[i]);
+            uint4 bcur[CW / 8];
+#pragma unroll
+            for (int j = 0; j < CW / 8; ++j) bcur[j] = bnext[j];
+            if (c + CW < ncol) fetch(c + CW);
+            uint8_t* buf = stage + (sc % NB) * (CW / 32) * 4096;
+#pragma unroll
+            for (int k = 0; k < CW / 32; ++k)
+                if (k < nblk)
+                    epilogue_values(epi, nb * BN + c + 32 * k, *reinterpret_cast<const uint4(*)[4]>(&bcur[4 * k]),
+                                    *reinterpret_cast<float(*)[32]>(&v[32 * k]));
+            if (lane == 0) bulk_wait_read<NB - 1>();
             __syncwarp();
-            stage_chunk(epi.out_f32 != 0, lane, v, buf);
+#pragma unroll
+            for (int k = 0; k < CW / 32; ++k)
+                if (k < nblk) stage_chunk(epi.out_f32 != 0, lane, *reinterpret_cast<float(*)[32]>(&v[32 * k]),
+                                          buf + k * 4096);
             fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) {
-                if (n < epi.split_n) tma_store_2d(&to[0], buf, n, row0);
-                else tma_store_2d(&to[1], buf, n - epi.split_n, row0);
+#pragma unroll
+                for (int k = 0; k < CW / 32; ++k) {
+                    if (k >= nblk) break;
+                    const int n = nb * BN + c + 32 * k;
+                    if (n < epi.split_n) tma_store_2d(&to[0], buf + k * 4096, n, row0);
+                    else tma_store_2d(&to[1], buf + k * 4096, n - epi.split_n, row0);
+                }
                 bulk_commit();
             }
             ++sc;
@@ -355,7 +399,7 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_cons
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* rbuf = smem + C::kStages * C::kStageBytes;            // [2][kResidBytes]
-    uint64_t* full_bar = reinterpret_cast<uint64_t*>(rbuf + 2 * C::kResidBytes);
+    uint64_t* full_bar = reinterpret_cast<uint64_t*>(rbuf + C::kEpiBytes);
     uint64_t* empty_bar = full_bar + C::kStages;
     uint64_t* tfull_bar = empty_bar + C::kStages;   // [2]
     uint64_t* tempty_bar = tfull_bar + 2;           // [2]
@@ -500,7 +544,7 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_cons
                 break;
             }
             tc_fence_after();
-            if (!epilogue_tile<BN>(epi, M, N, mb * BM, nb, t_acc_base + static_cast<uint32_t>(acc * BN), q, lane, warp,
+            if (!epilogue_tile<BN, C::kStageBufs>(epi, M, N, mb * BM, nb, t_acc_base + static_cast<uint32_t>(acc * BN), q, lane, warp,
                                    leader, tr, &om.m[2 * pr], rbuf, rfull_bar, rdone_bar, ruse, sc, status,
                                    abort_flag))
                 break;
@@ -540,15 +584,17 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_cons
 // ---------------------------------------------------------------------------
 constexpr int PBM = 256;   // rows per pair tile
 constexpr int PBN = 256;   // columns per pair tile
-constexpr int kPairStages = 6;
+constexpr int kPairStages = 5;
 
 struct PairCfg {
     static constexpr int kABytes = 128 * BK * 2;           // this CTA's A rows
     static constexpr int kBBytes = (PBN / 2) * BK * 2;     // this CTA's half of B
     static constexpr int kStageBytes = kABytes + kBBytes;
     static constexpr int kResidBytes = 128 * 32 * 4;
+    static constexpr int kEpiBytes = 4 * kResidBytes;   // residual chunks, or 4 output blocks per warp
+    static constexpr int kStageBufs = kEpiBytes / (4 * 4096);
     static constexpr int kBarrierBytes = 256;
-    static constexpr int kSmemBytes = kPairStages * kStageBytes + 2 * kResidBytes + 1024 + kBarrierBytes;
+    static constexpr int kSmemBytes = kPairStages * kStageBytes + kEpiBytes + 1024 + kBarrierBytes;
 };
 
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
@@ -560,7 +606,7 @@ gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_constan
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* rbuf = smem + kPairStages * C::kStageBytes;
-    uint64_t* full_bar = reinterpret_cast<uint64_t*>(rbuf + 2 * C::kResidBytes);   // used in the leader
+    uint64_t* full_bar = reinterpret_cast<uint64_t*>(rbuf + C::kEpiBytes);   // used in the leader
     uint64_t* empty_bar = full_bar + kPairStages;                                   // both CTAs
     uint64_t* tfull_bar = empty_bar + kPairStages;   // [2] both CTAs
     uint64_t* tempty_bar = tfull_bar + 2;            // [2] leader, 8 arrivals
@@ -703,13 +749,17 @@ gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_constan
                 break;
             }
             tc_fence_after();
-            if (!epilogue_tile<PBN>(epi, M, N, m0, nb, t_acc_base + static_cast<uint32_t>(acc * PBN), q, lane, warp,
+            if (!epilogue_tile<PBN, PairCfg::kStageBufs>(epi, M, N, m0, nb, t_acc_base + static_cast<uint32_t>(acc * PBN), q, lane, warp,
                                     leader, tr, &om.m[2 * pr], rbuf, rfull_bar, rdone_bar, ruse, sc, status,
                                     abort_flag))
                 break;
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive_cluster(mapa_shared(smem_u32(&tempty_bar[acc]), 0));
+            // the leader's own warps arrive locally; the peer's through the cluster
+            if (lane == 0) {
+                if (rank == 0) mbar_arrive(&tempty_bar[acc]);
+                else mbar_arrive_cluster(mapa_shared(smem_u32(&tempty_bar[acc]), 0));
+            }
             if (++acc == 2) { acc = 0; acc_phase ^= 1; }
         }
         if (lane == 0) bulk_wait<0>();

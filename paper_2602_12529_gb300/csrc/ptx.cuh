@@ -167,8 +167,14 @@ __device__ __forceinline__ uint32_t mapa_shared(uint32_t cta_addr, uint32_t rank
 __device__ __forceinline__ void cluster_sync() {
     asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
+// Arrive on an mbarrier of the peer CTA (cluster address) with the default
+// release at CTA scope.  Used only where the arrival hands over no memory:
+// it tells the peer that this warp's TMEM reads have completed
+// (tcgen05.wait::ld returned), so the peer may overwrite those columns.  A
+// release at cluster scope would make the arriving thread wait on a
+// cluster-wide fence first, which costs more than a thousand cycles.
 __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
-    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+    asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
 }
 // TMA load into this CTA's shared memory whose completion is counted on an
 // mbarrier that may live in the peer CTA of the pair (cluster address)
