@@ -248,25 +248,34 @@ __device__ __forceinline__ void stage_chunk(bool f32, int lane, const float (&v)
 }
 
 // One tile of the epilogue for the 128 rows m0.. held in this CTA's TMEM
-// (t_acc: this warp's lane quarter of the accumulator).  `to` are the
+// (t_acc: this warp's lane quarter of the accumulator).  With EW = 8
+// epilogue warps, two warps share each lane quarter and split the tile's
+// columns in halves (column group g = (warp - 2) / 4); each group has its own
+// pair of residual buffers and barriers and its own leader.  `to` are the
 // problem's two output maps; the warp owns SB staging blocks of 4 KB and `sc`
 // counts its store steps, which rotate through them.  Returns false after a
 // bounded wait gave up.
-template <int BN, int SB>
+template <int BN, int SB, int EW>
 __device__ __forceinline__ bool epilogue_tile(const GemmEpilogue& epi, int M, int N, int m0, int nb, uint32_t t_acc,
                                               int q, int lane, int warp, bool leader, const CUtensorMap* tr,
                                               const CUtensorMap* to, uint8_t* rbuf, uint64_t* rfull_bar,
                                               uint64_t* rdone_bar, uint32_t (&ruse)[2], uint32_t& sc, int* status,
                                               volatile int* abort_flag) {
     using C = Cfg<BN>;
+    constexpr int CG = BN * 4 / EW;             // columns per column group
+    const int g = EW == 8 ? (warp - 2) >> 2 : 0;
     const bool gated = epi.epi == EPI_GATED_RESIDUAL;
     const int r = q * 32 + lane;                // row within the tile = TMEM lane
     const int row = m0 + r;
     if (gated) {
         bool ok = true;
-        for (int c = 0; c < BN / 32; ++c) {
+        rbuf += 2 * g * C::kResidBytes;
+        rfull_bar += 2 * g;
+        rdone_bar += 2 * g;
+        const int c_end = (g + 1) * (CG / 32);
+        for (int c = g * (CG / 32); c < c_end; ++c) {
             const int n = nb * BN + c * 32;
-            const int b = c & 1;
+            const int b = (c - g * (CG / 32)) & 1;
             uint32_t rr[32];
             tmem_ld_x32(t_acc + c * 32, rr);
             tmem_ld_wait();
@@ -297,7 +306,7 @@ __device__ __forceinline__ bool epilogue_tile(const GemmEpilogue& epi, int M, in
             if (leader && ok) {
                 tma_store_2d(tr, rbuf + b * C::kResidBytes, n, m0);
                 bulk_commit();
-                if (c + 2 < BN / 32) {
+                if (c + 2 < c_end) {
                     bulk_wait_read<0>();
                     mbar_arrive_expect_tx(&rfull_bar[b], C::kResidBytes);
                     tma_load_2d(rbuf + b * C::kResidBytes, tr, &rfull_bar[b], n + 64, m0);
@@ -306,7 +315,7 @@ __device__ __forceinline__ bool epilogue_tile(const GemmEpilogue& epi, int M, in
         }
         if (!ok) return false;
     } else if (epi.qk_cols > 0 && nb * BN < epi.qk_cols) {
-        qk_norm_tile(epi, M, row, nb * BN, t_acc, BN);
+        qk_norm_tile(epi, M, row, nb * BN + g * CG, t_acc + g * CG, CG);
     } else {
         // plain store: bias / activation on the row held by this thread,
         // staged as 32 x 32 blocks and written by TMA bulk stores (rows past
@@ -320,7 +329,7 @@ __device__ __forceinline__ bool epilogue_tile(const GemmEpilogue& epi, int M, in
         constexpr int NB = SB * 32 / CW;
         uint8_t* stage = rbuf + (warp - 2) * (SB * 4096);
         const int row0 = m0 + q * 32;
-        const int ncol = N - nb * BN < BN ? N - nb * BN : BN;   // a multiple of 32
+        const int ncol = N - nb * BN < (g + 1) * CG ? N - nb * BN : (g + 1) * CG;   // a multiple of 32
         uint32_t rr[CW];
         uint4 bnext[CW / 8];
         auto fetch = [&](int c) {
@@ -331,9 +340,9 @@ __device__ __forceinline__ bool epilogue_tile(const GemmEpilogue& epi, int M, in
                     load_bias32(epi.bias, nb * BN + c + 32 * k, *reinterpret_cast<uint4(*)[4]>(&bnext[4 * k]));
                 }
         };
-        fetch(0);
+        fetch(g * CG);
 #pragma unroll 1
-        for (int c = 0; c < ncol; c += CW) {
+        for (int c = g * CG; c < ncol; c += CW) {
             const int nblk = ncol - c < CW ? 1 : CW / 32;
             tmem_ld_wait();
             float v[CW];
@@ -544,7 +553,7 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_cons
                 break;
             }
             tc_fence_after();
-            if (!epilogue_tile<BN, C::kStageBufs>(epi, M, N, mb * BM, nb, t_acc_base + static_cast<uint32_t>(acc * BN), q, lane, warp,
+            if (!epilogue_tile<BN, C::kStageBufs, 4>(epi, M, N, mb * BM, nb, t_acc_base + static_cast<uint32_t>(acc * BN), q, lane, warp,
                                    leader, tr, &om.m[2 * pr], rbuf, rfull_bar, rdone_bar, ruse, sc, status,
                                    abort_flag))
                 break;
@@ -585,19 +594,20 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_cons
 constexpr int PBM = 256;   // rows per pair tile
 constexpr int PBN = 256;   // columns per pair tile
 constexpr int kPairStages = 5;
+constexpr int kPairThreads = 320;   // producer, MMA, 8 epilogue warps
 
 struct PairCfg {
     static constexpr int kABytes = 128 * BK * 2;           // this CTA's A rows
     static constexpr int kBBytes = (PBN / 2) * BK * 2;     // this CTA's half of B
     static constexpr int kStageBytes = kABytes + kBBytes;
     static constexpr int kResidBytes = 128 * 32 * 4;
-    static constexpr int kEpiBytes = 4 * kResidBytes;   // residual chunks, or 4 output blocks per warp
-    static constexpr int kStageBufs = kEpiBytes / (4 * 4096);
+    static constexpr int kEpiBytes = 4 * kResidBytes;   // 2 x 2 residual chunks, or 2 output blocks per warp
+    static constexpr int kStageBufs = kEpiBytes / (8 * 4096);
     static constexpr int kBarrierBytes = 256;
     static constexpr int kSmemBytes = kPairStages * kStageBytes + kEpiBytes + 1024 + kBarrierBytes;
 };
 
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
 gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_constant__ CUtensorMap tm_b0,
                  const __grid_constant__ CUtensorMap tm_a1, const __grid_constant__ CUtensorMap tm_b1,
                  const __grid_constant__ CUtensorMap tm_r0, const __grid_constant__ CUtensorMap tm_r1,
@@ -609,11 +619,11 @@ gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_constan
     uint64_t* full_bar = reinterpret_cast<uint64_t*>(rbuf + C::kEpiBytes);   // used in the leader
     uint64_t* empty_bar = full_bar + kPairStages;                                   // both CTAs
     uint64_t* tfull_bar = empty_bar + kPairStages;   // [2] both CTAs
-    uint64_t* tempty_bar = tfull_bar + 2;            // [2] leader, 8 arrivals
+    uint64_t* tempty_bar = tfull_bar + 2;            // [2] leader, 16 arrivals
     uint64_t* drain_bar = tempty_bar + 2;            // [1] leader
-    uint64_t* rfull_bar = drain_bar + 1;             // [2] per CTA
-    uint64_t* rdone_bar = rfull_bar + 2;             // [2] per CTA
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(rdone_bar + 2);
+    uint64_t* rfull_bar = drain_bar + 1;             // [2 groups][2] per CTA
+    uint64_t* rdone_bar = rfull_bar + 4;             // [2 groups][2] per CTA
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(rdone_bar + 4);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5;
@@ -629,7 +639,9 @@ gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_constan
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(&tfull_bar[a], 1);
-            mbar_init(&tempty_bar[a], 8);
+            mbar_init(&tempty_bar[a], 16);
+        }
+        for (int a = 0; a < 4; ++a) {
             mbar_init(&rfull_bar[a], 1);
             mbar_init(&rdone_bar[a], 128);
         }
@@ -721,9 +733,11 @@ gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_constan
         tc_commit_pair_mc(drain_bar, 0x1);
         if (!mbar_wait(drain_bar, 0)) report_status(status, kStatusWaitTimeout);
     } else if (warp >= 2) {
-        // ---------------- epilogue (both CTAs, own 128 accumulator rows)
+        // ---------------- epilogue (both CTAs, own 128 accumulator rows; two
+        // warps per TMEM lane quarter, one per column half)
         const int q = warp & 3;
-        const bool leader = warp == 2 && lane == 0;
+        const int grp = (warp - 2) >> 2;
+        const bool leader = (warp == 2 || warp == 6) && lane == 0;
         uint32_t ruse[2] = {0, 0};
         uint32_t sc = 0;
         const uint32_t t_acc_base = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
@@ -737,10 +751,12 @@ gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_constan
             const int m0 = mb * PBM + rank * 128;
             const CUtensorMap* tr = pr ? &tm_r1 : &tm_r0;
             if (epi.epi == EPI_GATED_RESIDUAL && leader) {
+                // the first two residual chunks of this group's column half
                 for (int c = 0; c < 2; ++c) {
                     bulk_wait_read<0>();
-                    mbar_arrive_expect_tx(&rfull_bar[c], C::kResidBytes);
-                    tma_load_2d(rbuf + c * C::kResidBytes, tr, &rfull_bar[c], nb * PBN + c * 32, m0);
+                    mbar_arrive_expect_tx(&rfull_bar[2 * grp + c], C::kResidBytes);
+                    tma_load_2d(rbuf + (2 * grp + c) * C::kResidBytes, tr, &rfull_bar[2 * grp + c],
+                                nb * PBN + grp * (PBN / 2) + c * 32, m0);
                 }
             }
             if (!mbar_wait(&tfull_bar[acc], acc_phase)) {
@@ -749,7 +765,7 @@ gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_constan
                 break;
             }
             tc_fence_after();
-            if (!epilogue_tile<PBN, PairCfg::kStageBufs>(epi, M, N, m0, nb, t_acc_base + static_cast<uint32_t>(acc * PBN), q, lane, warp,
+            if (!epilogue_tile<PBN, PairCfg::kStageBufs, 8>(epi, M, N, m0, nb, t_acc_base + static_cast<uint32_t>(acc * PBN), q, lane, warp,
                                     leader, tr, &om.m[2 * pr], rbuf, rfull_bar, rdone_bar, ruse, sc, status,
                                     abort_flag))
                 break;
@@ -844,7 +860,7 @@ int launch_pair(const GemmArgs* p, int n, cudaStream_t stream) {
     g.tiles = g.tiles0 + (n > 1 ? g.num_m[1] * g.num_n[1] : 0);
     const int clusters = g.tiles < num_sms() / 2 ? g.tiles : num_sms() / 2;
     ProfScope prof(stream, "gemm_bf16", flops, bytes);
-    gemm_pair_kernel<<<2 * clusters, kThreads, C::kSmemBytes, stream>>>(ta[0], tb[0], ta[1], tb[1], tr[0], tr[1], om,
+    gemm_pair_kernel<<<2 * clusters, kPairThreads, C::kSmemBytes, stream>>>(ta[0], tb[0], ta[1], tb[1], tr[0], tr[1], om,
                                                                         g, device_status_ptr());
     return check_launch("gemm_pair_kernel");
 }
