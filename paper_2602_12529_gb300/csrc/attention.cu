@@ -30,7 +30,11 @@
 //               more than 8 (2^8 headroom), which makes corrections rare.
 //               Finally O / l goes out as bf16.
 // Every wait is bounded; on a timeout the kernel records the status word,
-// drains its tensor-core work, frees TMEM and returns.
+// drains its tensor-core work, frees TMEM and returns.  The MMA and softmax
+// loops do not poll the abort flag: a role that gave up stops signalling, so
+// the others run into their own bounded waits, and a shared-memory load per
+// step would queue behind the S = Q K^T operand reads, which take nearly all
+// of the shared-memory bandwidth while they run.
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -230,16 +234,20 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
             tc_fence_after();
             return true;
         };
+        // Descriptors are built once per operand tile; stepping inside a tile
+        // adds the byte offset >> 4 to the start-address field (addresses stay
+        // below 256 KB, so the field never carries), which keeps the issue
+        // cost per MMA to a few instructions.
+        const uint64_t desc_q[2] = {smem_desc_k_sw128(smem_u32(sQ)), smem_desc_k_sw128(smem_u32(sQ + C::kQBytes))};
         auto issue_s = [&](int t, int j) {
-            const uint32_t aQ = smem_u32(sQ + t * C::kQBytes);
-            const uint32_t aK = smem_u32(sKV + ((2 * j) % S) * C::kKBytes);
+            const uint64_t dq = desc_q[t];
+            const uint64_t dk = smem_desc_k_sw128(smem_u32(sKV + ((2 * j) % S) * C::kKBytes));
             const uint32_t dS = tmem + t * 256;
 #pragma unroll
             for (int k = 0; k < HD / 16; ++k) {
-                const uint32_t off_q = (k / 4) * (kBM * 128) + (k % 4) * 32;
-                const uint32_t off_k = (k / 4) * (kBN * 128) + (k % 4) * 32;
-                tc_mma_bf16(dS, smem_desc_k_sw128(aQ + off_q), smem_desc_k_sw128(aK + off_k), idesc_s,
-                                k != 0 ? 1u : 0u);
+                const uint32_t off_q = ((k / 4) * (kBM * 128) + (k % 4) * 32) >> 4;
+                const uint32_t off_k = ((k / 4) * (kBN * 128) + (k % 4) * 32) >> 4;
+                tc_mma_bf16(dS, dq + off_q, dk + off_k, idesc_s, k != 0 ? 1u : 0u);
             }
             tc_commit(&bar.s_full[t]);
         };
@@ -247,14 +255,13 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
             if (!mbar_wait(&bar.p_full[t], j & 1)) return false;
             tc_fence_after();
             if (t == 0 && !slot_ready(2 * j + 1)) return false;
-            const uint32_t aV = smem_u32(sKV + ((2 * j + 1) % S) * C::kKBytes);
+            const uint64_t dv = smem_desc_mn_sw128(smem_u32(sKV + ((2 * j + 1) % S) * C::kKBytes), kBN * 128);
             const uint32_t dO = tmem + t * 256 + C::kColO;
             const uint32_t aP = tmem + t * 256;
 #pragma unroll
-            for (int k = 0; k < kBN / 16; ++k) {
-                const uint64_t db = smem_desc_mn_sw128(aV + k * 2048, kBN * 128);
-                tc_mma_bf16_ts(dO, aP + k * 8, db, idesc_o, (j | k) != 0 ? 1u : 0u);
-            }
+            for (int k = 0; k < kBN / 16; ++k)   // 16 tokens = 2048 bytes of V per step
+                tc_mma_bf16_ts(dO, aP + k * 8, dv + static_cast<uint64_t>(k * (2048 >> 4)), idesc_o,
+                               (j | k) != 0 ? 1u : 0u);
             return true;
         };
         if (ok && ntiles > 0) {
@@ -265,7 +272,7 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
                 tc_commit(&bar.slot_empty[0]);
             }
         }
-        for (int j = 0; ok && j < ntiles && !*abort_flag; ++j) {
+        for (int j = 0; ok && j < ntiles; ++j) {
             const bool more = j + 1 < ntiles;
             for (int t = 0; t < 2; ++t) {
                 if (!issue_pv(t, j)) { fail(); ok = false; break; }
@@ -295,7 +302,6 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
         float l = 0.f;
         bool ok = true;
         for (int j = 0; j < ntiles; ++j) {
-            if (*abort_flag) { ok = false; break; }
             // S_t,j ready; O_t += P_t,j-1 V_j-1 has completed as well
             if (!mbar_wait(&bar.s_full[t], j & 1)) { fail(); ok = false; break; }
             tc_fence_after();
