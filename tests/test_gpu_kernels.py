@@ -87,7 +87,10 @@ def test_gemm_gated_residual_parity(cuda, M, N, K, rps):
 
 
 @pytest.mark.parametrize("B,heads,d,n0,n1", [(2, 2, 64, 5, 70), (1, 3, 128, 32, 200), (2, 2, 128, 0, 130),
-                                             (1, 2, 128, 512, 1024)])
+                                             (1, 2, 128, 512, 1024),
+                                             # d = 128 runs on CTA pairs owning 512 query rows: partial
+                                             # blocks, a second pair tile past the segment end, ragged K/V
+                                             (2, 2, 128, 300, 777), (1, 1, 128, 1000, 24), (3, 1, 128, 130, 513)])
 def test_attention_parity(cuda, B, heads, d, n0, n1):
     import torch
     from paper_2602_12529_gb300 import ffi
