@@ -11,7 +11,10 @@ and it shares no code with the CUDA path (only the seeded inputs of
 Modules:
   sde   -- time grids, noise schedules (Table 1), the Flow-SDE update (Eq. 1)
            and its Gaussian transition log-probability.
-  grpo  -- group-normalised advantage and the clipped-ratio policy loss.
+  grpo  -- group-normalised advantage (one or several rewards) and the
+           clipped-ratio policy loss (optionally with per-step weights).
+  awm   -- training-time sampling, the forward process x_t and the
+           advantage-weighted matching loss of Eq. 3.
   dit   -- the flow-matching DiT velocity v_theta(x_t, t): MMDiT double- and
            single-stream blocks (adaLN modulation, QK-RMSNorm, RoPE, joint
            attention, GELU MLP) and the final projection.
@@ -19,7 +22,7 @@ Modules:
 Every array is float64; bf16 weights and inputs are widened exactly.  Nothing
 is rounded between steps.
 
-Parity status: sde and grpo are pinned by closed forms; the DiT pieces are
+Parity status: sde, grpo and awm are pinned by closed forms; the DiT pieces are
 pinned one by one (attention, RoPE, norms, GELU, modulation identity) and the
 whole velocity only through those pieces plus invariants ("parity unpinned" as
 a whole: no printed outputs exist for a random-init network).

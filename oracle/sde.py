@@ -51,6 +51,15 @@ def sigma_ode(t):
     return np.zeros_like(np.asarray(t, dtype=np.float64))
 
 
+def window_sigma(sigma, start: int, length: int) -> np.ndarray:
+    """MixGRPO (Sec. 3.1): SDE noise on steps start .. start + length - 1 only,
+    the deterministic ODE update (sigma = 0) on every other step."""
+    s = np.array(sigma, dtype=np.float64)
+    k = np.arange(s.size)
+    s[(k < start) | (k >= start + length)] = 0.0
+    return s
+
+
 def sde_mean_std(x, v, t: float, t_next: float, sigma: float):
     """Mean and std of the Gaussian transition of Eq. 1 for one sample.
 

@@ -89,3 +89,62 @@ def test_loss_gradient_finite_differences():
         m[b, k] -= h
         fd = (grpo.grpo_loss(p, lp_old, adv)[0] - grpo.grpo_loss(m, lp_old, adv)[0]) / (2 * h)
         assert g[b, k] == pytest.approx(fd, abs=1e-8)
+
+
+def test_multi_reward_single_reward_and_one_hot_weights():
+    rng = np.random.default_rng(7)
+    G, ng, K = 4, 3, 3
+    R = rng.random((G * ng, K))
+    for mode in ("weighted_sum", "per_reward"):
+        # K = 1 with weight 1 is the single-reward advantage
+        np.testing.assert_allclose(grpo.group_advantage_multi(R[:, :1], G, [1.0], mode),
+                                   grpo.group_advantage(R[:, 0], G), rtol=1e-14)
+        # a one-hot weight picks that reward
+        np.testing.assert_allclose(grpo.group_advantage_multi(R, G, [0.0, 1.0, 0.0], mode),
+                                   grpo.group_advantage(R[:, 1], G), rtol=1e-14, atol=1e-15)
+
+
+def test_multi_reward_modes_differ_and_follow_their_definitions():
+    rng = np.random.default_rng(8)
+    G, ng, K = 5, 2, 2
+    R = rng.random((G * ng, K)) * np.array([1.0, 100.0])   # rewards on very different scales
+    w = np.array([0.7, 0.3])
+    ws = grpo.group_advantage_multi(R, G, w, "weighted_sum")
+    pr = grpo.group_advantage_multi(R, G, w, "per_reward")
+    # brute force, one group at a time
+    for g in range(ng):
+        rows = slice(g * G, (g + 1) * G)
+        r = R[rows] @ w
+        np.testing.assert_allclose(ws[rows], (r - r.mean()) / (r.std() + 1e-4), rtol=1e-13)
+        want = sum(w[k] * (R[rows, k] - R[rows, k].mean()) / (R[rows, k].std() + 1e-4) for k in range(K))
+        np.testing.assert_allclose(pr[rows], want, rtol=1e-13)
+    # the weighted sum is dominated by the large-scale reward, per-reward normalisation is not
+    assert np.max(np.abs(ws - pr)) > 0.1
+    np.testing.assert_allclose(pr.reshape(ng, G).mean(axis=1), 0.0, atol=1e-13)
+
+
+def test_step_weights_reduce_to_plain_grpo_and_drop_steps():
+    rng = np.random.default_rng(9)
+    B, T = 3, 4
+    lp_new, lp_old = rng.standard_normal((B, T)) * 0.1, rng.standard_normal((B, T)) * 0.1
+    adv = rng.standard_normal(B)
+    l1, g1 = grpo.grpo_loss(lp_new, lp_old, adv)
+    lw, gw = grpo.grpo_loss(lp_new, lp_old, adv, step_w=np.ones(T))
+    assert lw == l1 and np.array_equal(gw, g1)
+    # weight 0 on steps 1..3 leaves step 0 only, still averaged over B * T
+    w = np.array([1.0, 0.0, 0.0, 0.0])
+    l0, g0 = grpo.grpo_loss(lp_new, lp_old, adv, step_w=w)
+    ls, _ = grpo.grpo_loss(lp_new[:, :1], lp_old[:, :1], adv)
+    assert l0 == pytest.approx(ls / T, rel=1e-14)
+    assert np.all(g0[:, 1:] == 0.0)
+    # linear in the weights, gradient by central differences
+    w2 = rng.random(T)
+    lw2, gw2 = grpo.grpo_loss(lp_new, lp_old, adv, step_w=w2)
+    h = 1e-7
+    for b in range(B):
+        for k in range(T):
+            p, m = lp_new.copy(), lp_new.copy()
+            p[b, k] += h
+            m[b, k] -= h
+            fd = (grpo.grpo_loss(p, lp_old, adv, step_w=w2)[0] - grpo.grpo_loss(m, lp_old, adv, step_w=w2)[0]) / (2 * h)
+            assert gw2[b, k] == pytest.approx(fd, rel=1e-5, abs=1e-10)

@@ -150,3 +150,17 @@ def test_ode_step_logprob_is_zero():
     xn, lp = sde.sde_step_logprob(x, x, [0.5], [0.25], [0.0], eps=np.ones((1, 8)))
     assert lp[0] == 0.0
     np.testing.assert_array_equal(xn, x - x * 0.25)
+
+
+def test_mixgrpo_window_keeps_sigma_inside_and_zeroes_outside():
+    t = sde.time_grid(10, 3.0)
+    s = sde.sigma_flow_sde(t[:-1], 0.7)
+    w = sde.window_sigma(s, 3, 2)
+    np.testing.assert_array_equal(w[3:5], s[3:5])
+    assert np.all(w[:3] == 0.0) and np.all(w[5:] == 0.0)
+    assert np.array_equal(sde.window_sigma(s, 0, 10), s)
+    # an ODE step scores log-prob 0 and moves x by the drift only
+    x, v = np.ones(4), np.full(4, 0.5)
+    mean, std = sde.sde_mean_std(x, v, t[0], t[1], w[0])
+    assert std == 0.0 and sde.gaussian_logprob(mean, mean, std) == 0.0
+    np.testing.assert_allclose(mean, x - v * (t[0] - t[1]))
