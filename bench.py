@@ -312,8 +312,84 @@ def hbm_sweep(ffi, dev, hbm_peak, l2_bytes=129 * 2 ** 20):
                      "frac": per / sec / 1e9 / hbm_peak, "sets": len(sets)})
         del sets
     out["group_advantage"] = rows
+    for name, per_elem in (("forward_process", 12), ("awm_loss", 16)):
+        rows = []
+        for n in (1 << 24, 1 << 26, 1 << 28):
+            B, D = 4, n // 4
+            per = per_elem * n
+            sets = []
+            for _ in range(nsets(per)):
+                x = torch.randn(B, D, device=dev)
+                sets.append((x, torch.randn_like(x), torch.randn_like(x), torch.empty_like(x)))
+            t = torch.full((B,), 0.6, device=dev)
+            adv = torch.randn(B, device=dev)
+            loss = torch.empty(1, device=dev)
+            if name == "forward_process":
+                fns = [lambda s_=s_: ffi.ff_forward_process(s_[0], s_[1], t, s_[3]) for s_ in sets]
+            else:
+                ws = torch.empty(ffi.ff_awm_loss_workspace_size(B, D), dtype=torch.uint8, device=dev)
+                fns = [lambda s_=s_: ffi.ff_awm_loss(s_[0], s_[1], s_[2], adv, ffi.FF_AWM_MEAN, loss, s_[3], ws=ws)
+                       for s_ in sets]
+            sec = timeit(fns)
+            rows.append({"elements": n, "bytes": per, "gbs": per / sec / 1e9, "frac": per / sec / 1e9 / hbm_peak,
+                         "sets": len(sets)})
+            del sets
+        out[name] = rows
     torch.cuda.empty_cache()
     return out
+
+
+def awm_step(args, ffi, model, cfg, dev, x0, txt, eps, rewards, timed, world):
+    """The AWM training step of Eq. 3 on the same workload and batch: training
+    times from the logit-normal sampler, x_t by the forward process, the
+    velocity, and the advantage-weighted loss with its gradient w.r.t. v.
+    Timed like the main step (CUDA events, K steps), and once more with the
+    per-launch events for the two memory-bound kernels' rooflines."""
+    import torch
+    B = x0.shape[0]
+    D = x0.numel() // B
+    z = torch.linspace(-1.5, 1.5, B, device=dev)
+    tt = torch.empty(B, device=dev)
+    xt = torch.empty_like(x0)
+    v = torch.empty_like(x0)
+    gv = torch.empty_like(x0)
+    adv = torch.empty(B, device=dev)
+    ffi.ff_group_advantage(rewards, B, 1e-4, adv)
+    loss = torch.empty(1, device=dev)
+    ws = torch.empty(model.workspace_size(B), dtype=torch.uint8, device=dev)
+    ws_awm = torch.empty(ffi.ff_awm_loss_workspace_size(B, D), dtype=torch.uint8, device=dev)
+
+    def step():
+        ffi.ff_sample_timesteps(ffi.FF_TSAMPLE_LOGIT_NORMAL, z, 0.0, 1.0, tt)
+        ffi.ff_forward_process(x0, eps, tt, xt)
+        model.ff_dit_velocity(xt, txt, tt, v, ws)
+        ffi.ff_awm_loss(v, eps, x0, adv, ffi.FF_AWM_MEAN, loss, gv, ws=ws_awm)
+
+    for _ in range(args.warmup):
+        step()
+    ms = timed(step, args.steps) / args.steps
+    ffi.ff_prof_enable(64 * args.steps + 64)
+    timed(step, args.steps)
+    recs = ffi.ff_prof_records()
+    ffi.ff_prof_disable()
+    _, _, _, peak_src = load_peaks()
+    hbm = load_peaks()[0]
+    roofs = {}
+    for name in ("forward_process", "awm_loss"):
+        r = [(ms_, by) for n_, ms_, fl, by in recs if n_ == name]
+        if r:
+            ach = sum(b for _, b in r) / len(r) / (sum(m for m, _ in r) / len(r) / 1e3) / 1e9
+            roofs[name] = {"bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s", "frac": ach / hbm,
+                           "launches": len(r), "algorithmic_per_launch": r[0][1], "peak_source": f"{peak_src} HBM copy"}
+    n_img = synth_n_img(cfg)
+    return {"ms_per_step": ms, "value": world * B * n_img / (ms / 1e3), "unit": UNIT,
+            "what": "logit-normal t + forward process + velocity + Eq. 3 loss with dL/dv, batch of the main step",
+            "rooflines": roofs}
+
+
+def synth_n_img(cfg):
+    import synth
+    return synth.n_img(cfg)
 
 
 def run_ours(args):
@@ -477,6 +553,7 @@ def run_ours(args):
     e2e_step()
     ms_e2e = timed(e2e_step, args.steps) / args.steps
     e2e_value = world * tokens_per_step / (ms_e2e / 1e3)
+    awm = awm_step(args, ffi, model, cfg, dev, x, txt, eps, rewards, timed, world)
     sweep = hbm_sweep(ffi, dev, hbm) if rank == 0 and not args.no_sweep else None
     clk = clocks.stop() if clocks else None
     status = ffi.ff_check_device_status()
@@ -503,6 +580,7 @@ def run_ours(args):
                 "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                         "ms_per_step": ms_e2e},
                 "hbm_sweep": sweep,
+                "awm_step": awm,
                 "gpu_launches": launches,
                 "clocks": clk,
                 "device_status": status}

@@ -8,6 +8,11 @@
  *   2. x_{t+dt} = Eq. 1 update, log p(x_{t+dt}|x_t) ff_sde_step_logprob
  *   3. A = group-normalised reward                 ff_group_advantage
  *   4. clipped-ratio policy loss over (b, step)    ff_grpo_loss
+ * and its variants: the MixGRPO SDE window (ff_sde_schedule_window), the
+ * GRPO-Guard step weights (ff_grpo_loss_weighted), multi-reward advantage
+ * aggregation (ff_group_advantage_multi), and the AWM training step of
+ * Sec. 3.2, Eq. 3 (ff_sample_timesteps, ff_forward_process, the velocity,
+ * ff_awm_loss).
  *
  * Conventions for every entry point:
  *   - Returns an int status: FF_OK or one of the FF_ERR_* codes below.  On
@@ -51,6 +56,16 @@ extern "C" {
 #define FF_SCHED_DANCE_SDE 1  /* Table 1: sigma_t = eta                     */
 #define FF_SCHED_ODE 2        /* Table 1: sigma_t = 0                       */
 
+#define FF_TSAMPLE_UNIFORM 0       /* Sec. 3.2 training times: t = p0 + (p1 - p0) u          */
+#define FF_TSAMPLE_LOGIT_NORMAL 1  /* t = 1 / (1 + exp(-(p0 + p1 z)))                       */
+#define FF_TSAMPLE_DISCRETE 2      /* t = grid[min(floor(u n), n - 1)]                      */
+
+#define FF_AWM_SUM 0    /* Eq. 3 squared norm: sum over the D elements of a sample */
+#define FF_AWM_MEAN 1   /* ... divided by D (per-element MSE)                     */
+
+#define FF_AGG_WEIGHTED_SUM 0  /* r = sum_k w_k R_k, then group-normalise r          */
+#define FF_AGG_PER_REWARD 1    /* group-normalise each R_k, then sum_k w_k A_k (GDPO) */
+
 #define FF_ARCH_MMDIT 0   /* Flux / Qwen-Image style double + single stream */
 #define FF_ARCH_WAN 1     /* WAN-style video DiT: self-attn + text cross-attn + FFN */
 
@@ -89,6 +104,16 @@ int ff_prof_read(int i, char* name, int name_cap, float* ms, double* flops, doub
  * ------------------------------------------------------------------------ */
 int ff_sde_schedule(int kind, int n_steps, double shift, double eta, double t_clamp,
                     double* t_out, double* sigma_out);
+
+/* ------------------------------------------------------------------------
+ * MixGRPO / Flow-GRPO-Fast (paper Sec. 3.1): SDE noise on the steps
+ * window_start .. window_start + window_len - 1 only and the deterministic
+ * ODE update elsewhere.  Same as ff_sde_schedule, with sigma_out[k] = 0
+ * outside the window (an ODE step's log-prob is 0, see below).  Requires
+ * 0 <= window_start and window_start + window_len <= n_steps.  Host only.
+ * ------------------------------------------------------------------------ */
+int ff_sde_schedule_window(int kind, int n_steps, double shift, double eta, double t_clamp,
+                           int window_start, int window_len, double* t_out, double* sigma_out);
 
 /* ------------------------------------------------------------------------
  * SDE step + Gaussian transition log-probability.  Paper Eq. 1, Table 1.
@@ -169,6 +194,68 @@ int ff_grpo_loss_workspace_size(int B, int T, size_t* bytes);
 int ff_grpo_loss(int B, int T, const float* lp_new, const float* lp_old,
                  const float* adv, float clip_lo, float clip_hi, float* loss,
                  float* grad_lp_new, void* ws, size_t ws_bytes, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
+ * GRPO-Guard (paper Sec. 3.1): the loss above with timestep-dependent
+ * weights.  The term of step k (objective and gradient) is multiplied by
+ * step_w[k]; the paper does not print the weights, so they are an input.
+ *   loss = -1/(B T) sum_{b,k} step_w[k] min(rho A_b, clip(rho) A_b)
+ * step_w: [T] fp32 device, not NULL (all ones gives ff_grpo_loss).  Same
+ * workspace as ff_grpo_loss.
+ * ------------------------------------------------------------------------ */
+int ff_grpo_loss_weighted(int B, int T, const float* lp_new, const float* lp_old,
+                          const float* adv, const float* step_w, float clip_lo, float clip_hi,
+                          float* loss, float* grad_lp_new, void* ws, size_t ws_bytes,
+                          cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Multi-reward advantage (paper Sec. 2.3, configurable advantage
+ * aggregation, "weighted-sum and GDPO-style per-reward normalization").
+ * K rewards per sample, R: [n_groups * G, K] fp32 row-major; w: [K] fp32
+ * device; contiguous groups of G as in ff_group_advantage.
+ *   FF_AGG_WEIGHTED_SUM: r_i = sum_k w_k R[i, k]; A_i = (r_i - mean_g) / (std_g + eps_A)
+ *   FF_AGG_PER_REWARD:   A_i = sum_k w_k (R[i, k] - mean_g,k) / (std_g,k + eps_A)
+ * (population std).  G in [1, 4096], K in [1, 64].  adv: [n_groups * G]
+ * fp32, must not alias rewards.
+ * ------------------------------------------------------------------------ */
+int ff_group_advantage_multi(int n_groups, int G, int K, const float* rewards, const float* w,
+                             int mode, float eps_A, float* adv, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Advantage Weighted Matching (paper Sec. 3.2, Eq. 3).  Time runs from 1
+ * (noise) to 0 (data), as in the sampler above.
+ *
+ * ff_sample_timesteps -- training times t[b] from the caller's random draws
+ * (Sec. 3.2: uniform, logit-normal or discrete timestep sampling):
+ *   FF_TSAMPLE_UNIFORM:      t = p0 + (p1 - p0) draw,   draw = u in [0, 1)
+ *   FF_TSAMPLE_LOGIT_NORMAL: t = 1 / (1 + exp(-(p0 + p1 draw))), draw = z ~ N(0, 1), p1 >= 0
+ *   FF_TSAMPLE_DISCRETE:     t = grid[min(floor(draw n_grid), n_grid - 1)], draw = u
+ *                            (the index is taken in fp32)
+ * draw, t_out: [B] fp32 device; grid: [n_grid] fp32 device (DISCRETE only).
+ *
+ * ff_forward_process -- the noised input of Eq. 3:
+ *   x_t[b, j] = (1 - t[b]) x0[b, j] + t[b] eps[b, j]
+ * x0, eps, x_t: [B, D] fp32 row-major, 16-byte aligned, D % 4 == 0; t: [B]
+ * fp32 device.  x_t may alias x0 or eps.
+ *
+ * ff_awm_loss -- Eq. 3 over a batch (the expectation over t and eps is the
+ * batch mean):
+ *   e_b = sum_j (v[b, j] - (eps[b, j] - x0[b, j]))^2  (/ D for FF_AWM_MEAN)
+ *   loss = (1/B) sum_b A[b] e_b
+ *   grad_v[b, j] = (2/B) A[b] (v[b, j] - (eps[b, j] - x0[b, j]))  (/ D for MEAN)
+ * v, eps, x0: [B, D] fp32 (v = ff_dit_velocity(x_t, t)); adv: [B] fp32;
+ * loss: [1] fp32 written; grad_v: [B, D] fp32 or NULL; err_out: [B] fp32
+ * (e_b) or NULL.  ws: at least ff_awm_loss_workspace_size(B, D) bytes; the
+ * two-pass reduction is deterministic.
+ * ------------------------------------------------------------------------ */
+int ff_sample_timesteps(int mode, int B, const float* draw, float p0, float p1,
+                        const float* grid, int n_grid, float* t_out, cudaStream_t stream);
+int ff_forward_process(int B, int64_t D, const float* x0, const float* eps, const float* t,
+                       float* x_t, cudaStream_t stream);
+int ff_awm_loss_workspace_size(int B, int64_t D, size_t* bytes);
+int ff_awm_loss(int B, int64_t D, const float* v, const float* eps, const float* x0,
+                const float* adv, int reduce, float* loss, float* grad_v, float* err_out,
+                void* ws, size_t ws_bytes, cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
  * DiT velocity v_theta(x_t, t) (the network of Eq. 1 and Eq. 3).

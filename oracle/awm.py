@@ -16,7 +16,10 @@ Readings (the paper leaves these open):
       uniform       t = t_min + (t_max - t_min) u,  u ~ U[0, 1)
       logit-normal  t = 1 / (1 + exp(-(m + s z))),  z ~ N(0, 1)
       discrete      t = grid[min(floor(u n), n - 1)] over a grid of n times
-    The random draws u or z are inputs, not drawn here.
+    The random draws u or z are inputs, not drawn here.  The discrete index
+    is a floating-point decision that picks an integer, so it is taken in
+    float32 (u and n rounded to float32, their product rounded once), the
+    precision the kernel uses; everything else is float64.
 """
 from __future__ import annotations
 
@@ -36,7 +39,8 @@ def sample_timesteps(mode: str, draw, p0: float = 0.0, p1: float = 1.0, grid=Non
     if mode == "discrete":
         g = np.asarray(grid, dtype=np.float64)
         n = g.size
-        idx = np.array([min(int(math.floor(u * n)), n - 1) for u in d.ravel()]).reshape(d.shape)
+        prod = np.float32(d.ravel()).astype(np.float32) * np.float32(n)   # one float32 rounding
+        idx = np.array([max(0, min(int(math.floor(float(x))), n - 1)) for x in prod]).reshape(d.shape)
         return g[idx]
     raise ValueError(mode)
 

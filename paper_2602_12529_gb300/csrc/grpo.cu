@@ -20,6 +20,12 @@ constexpr int kThreads = 256;
 constexpr int kElemsPerBlock = kThreads * 16;
 constexpr int kMaxLossBlocks = 1216;   // 8 blocks of 256 threads on each of 152 SMs
 
+// The group sums run on values shifted by a pivot (the group's first
+// reward): mean = pivot + sum(r - pivot) / G.  A constant group then gets
+// exactly zero advantages (an fp32 mean of G equal values need not equal
+// them), and the shift removes most of the cancellation when the rewards
+// share a large offset.
+//
 // G in {4, 8, 16, 32, 64, 128}: each lane owns 4 consecutive samples (one
 // float4) and a group spans G / 4 lanes; the reductions shuffle within those
 // lanes.  fp32 sums over at most 128 values (the tests bound them against
@@ -30,9 +36,10 @@ __global__ void __launch_bounds__(kThreads) group_advantage_vec_kernel(int64_t n
     const bool live = i < n4;
     const float4 x = live ? r[i] : make_float4(0.f, 0.f, 0.f, 0.f);
     const int lanes = G >> 2;
-    float s = (x.x + x.y) + (x.z + x.w);
+    const float pivot = __shfl_sync(0xffffffffu, x.x, (threadIdx.x & 31) & ~(lanes - 1));
+    float s = ((x.x - pivot) + (x.y - pivot)) + ((x.z - pivot) + (x.w - pivot));
     for (int o = 1; o < lanes; o <<= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-    const float mean = s / G;
+    const float mean = pivot + s / G;
     const float d0 = x.x - mean, d1 = x.y - mean, d2 = x.z - mean, d3 = x.w - mean;
     float q = (d0 * d0 + d1 * d1) + (d2 * d2 + d3 * d3);
     for (int o = 1; o < lanes; o <<= 1) q += __shfl_xor_sync(0xffffffffu, q, o);
@@ -47,11 +54,12 @@ __global__ void __launch_bounds__(kThreads) group_advantage_kernel(int n_groups,
     const int lane = threadIdx.x & 31;
     if (warp >= n_groups) return;
     const float* rg = r + static_cast<int64_t>(warp) * G;
+    const float pivot = rg[0];
     float s = 0.f;
-    for (int i = lane; i < G; i += 32) s += rg[i];
+    for (int i = lane; i < G; i += 32) s += rg[i] - pivot;
 #pragma unroll
     for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-    const float mean = s / G;
+    const float mean = pivot + s / G;
     float q = 0.f;
     for (int i = lane; i < G; i += 32) {
         const float d = rg[i] - mean;
@@ -66,12 +74,69 @@ __global__ void __launch_bounds__(kThreads) group_advantage_kernel(int n_groups,
     for (int i = lane; i < G; i += 32) ag[i] = (rg[i] - mean) / denom;
 }
 
+// Several rewards per sample, R[i, k] row-major [N, K]: one warp per group.
+// WEIGHTED_SUM forms r_i = sum_k w_k R[i, k] on the fly and normalises it;
+// PER_REWARD normalises every column within the group and accumulates
+// w_k A[i, k] into adv (each lane rewrites only its own samples).
+__global__ void __launch_bounds__(kThreads) group_advantage_multi_kernel(int n_groups, int G, int K, const float* R,
+                                                                         const float* w, int mode, float eps,
+                                                                         float* adv) {
+    const int warp = (blockIdx.x * kThreads + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (warp >= n_groups) return;
+    const float* Rg = R + static_cast<int64_t>(warp) * G * K;
+    float* ag = adv + static_cast<int64_t>(warp) * G;
+    auto warp_sum = [](float v) {
+#pragma unroll
+        for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+        return v;
+    };
+    if (mode == FF_AGG_WEIGHTED_SUM) {
+        auto r_of = [&](int i) {
+            float r = 0.f;
+            for (int k = 0; k < K; ++k) r = fmaf(w[k], Rg[static_cast<int64_t>(i) * K + k], r);
+            return r;
+        };
+        const float pivot = r_of(0);
+        float s = 0.f;
+        for (int i = lane; i < G; i += 32) s += r_of(i) - pivot;
+        const float mean = pivot + warp_sum(s) / G;
+        float q = 0.f;
+        for (int i = lane; i < G; i += 32) {
+            const float d = r_of(i) - mean;
+            q = fmaf(d, d, q);
+        }
+        const float denom = sqrtf(warp_sum(q) / G) + eps;
+        for (int i = lane; i < G; i += 32) ag[i] = (r_of(i) - mean) / denom;
+        return;
+    }
+    for (int k = 0; k < K; ++k) {
+        const float pivot = Rg[k];
+        float s = 0.f;
+        for (int i = lane; i < G; i += 32) s += Rg[static_cast<int64_t>(i) * K + k] - pivot;
+        const float mean = pivot + warp_sum(s) / G;
+        float q = 0.f;
+        for (int i = lane; i < G; i += 32) {
+            const float d = Rg[static_cast<int64_t>(i) * K + k] - mean;
+            q = fmaf(d, d, q);
+        }
+        const float c = w[k] / (sqrtf(warp_sum(q) / G) + eps);
+        for (int i = lane; i < G; i += 32) {
+            const float a = c * (Rg[static_cast<int64_t>(i) * K + k] - mean);
+            ag[i] = k == 0 ? a : ag[i] + a;
+        }
+    }
+}
+
 // One fp32 partial per thread over float4 groups (sample index b = i / T in
 // 32-bit arithmetic), fp64 only for the block and cross-block sums.
+// WEIGHTED: GRPO-Guard's per-step weights step_w[k] scale the term of step
+// k (objective and gradient).
+template <bool WEIGHTED>
 __global__ void __launch_bounds__(kThreads) grpo_loss_partial_kernel(int64_t n, int T, const float* lp_new,
                                                                      const float* lp_old, const float* adv,
-                                                                     float lo, float hi, float inv_n,
-                                                                     float* grad, double* partial) {
+                                                                     const float* step_w, float lo, float hi,
+                                                                     float inv_n, float* grad, double* partial) {
     __shared__ double red[kThreads / 32];
     float s = 0.f;
     const int64_t n4 = n >> 2;
@@ -79,13 +144,15 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_partial_kernel(int64_t n, 
     const float4* b4 = reinterpret_cast<const float4*>(lp_old);
     const uint32_t Tu = static_cast<uint32_t>(T);
     auto term = [&](float ln, float lo_, uint32_t idx, float& g) {
-        const float a = adv[idx / Tu];
+        const uint32_t b = idx / Tu;
+        const float a = adv[b];
         const float rho = __expf(ln - lo_);
         const float unclipped = rho * a;
         const float clipped = fminf(fmaxf(rho, 1.0f - lo), 1.0f + hi) * a;
         const bool take = unclipped <= clipped;
-        g = take ? -a * rho * inv_n : 0.0f;
-        return take ? unclipped : clipped;
+        const float w = WEIGHTED ? step_w[idx - b * Tu] : 1.0f;
+        g = take ? -w * a * rho * inv_n : 0.0f;
+        return w * (take ? unclipped : clipped);
     };
     for (int64_t v = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; v < n4;
          v += static_cast<int64_t>(gridDim.x) * kThreads) {
@@ -170,9 +237,14 @@ int ff_grpo_loss_workspace_size(int B, int T, size_t* bytes) {
     return FF_OK;
 }
 
-int ff_grpo_loss(int B, int T, const float* lp_new, const float* lp_old, const float* adv, float clip_lo,
-                 float clip_hi, float* loss, float* grad_lp_new, void* ws, size_t ws_bytes, cudaStream_t stream) {
-    using namespace ff;
+}  // extern "C"
+
+namespace ff {
+namespace {
+
+int grpo_loss_impl(int B, int T, const float* lp_new, const float* lp_old, const float* adv, const float* step_w,
+                   float clip_lo, float clip_hi, float* loss, float* grad_lp_new, void* ws, size_t ws_bytes,
+                   cudaStream_t stream) {
     if (B <= 0 || T <= 0) return set_error(FF_ERR_INVALID_ARG, "loss: B=%d T=%d must be positive", B, T);
     if (!lp_new || !lp_old || !adv || !loss) return set_error(FF_ERR_INVALID_ARG, "loss: null pointer");
     if (!aligned16(lp_new) || !aligned16(lp_old) || (grad_lp_new && !aligned16(grad_lp_new)))
@@ -189,15 +261,56 @@ int ff_grpo_loss(int B, int T, const float* lp_new, const float* lp_old, const f
     double* partial = static_cast<double*>(ws);
     {
     ProfScope prof(stream, "grpo_loss", 0.0, static_cast<double>(n) * (grad_lp_new ? 12.0 : 8.0) + 4.0 * B);
-    grpo_loss_partial_kernel<<<nb, kThreads, 0, stream>>>(n, T, lp_new, lp_old, adv, clip_lo, clip_hi,
-                                                          static_cast<float>(1.0 / static_cast<double>(n)),
-                                                          grad_lp_new, partial);
+    if (step_w)
+        grpo_loss_partial_kernel<true><<<nb, kThreads, 0, stream>>>(
+            n, T, lp_new, lp_old, adv, step_w, clip_lo, clip_hi, static_cast<float>(1.0 / static_cast<double>(n)),
+            grad_lp_new, partial);
+    else
+        grpo_loss_partial_kernel<false><<<nb, kThreads, 0, stream>>>(
+            n, T, lp_new, lp_old, adv, nullptr, clip_lo, clip_hi, static_cast<float>(1.0 / static_cast<double>(n)),
+            grad_lp_new, partial);
     }
     int rc = check_launch("grpo_loss_partial_kernel");
     if (rc) return rc;
     ProfScope prof(stream, "grpo_loss_finalize", 0.0, nb * 8.0 + 4.0);
     grpo_loss_finalize_kernel<<<1, kThreads, 0, stream>>>(nb, partial, 1.0 / static_cast<double>(n), loss);
     return check_launch("grpo_loss_finalize_kernel");
+}
+
+}  // namespace
+}  // namespace ff
+
+extern "C" {
+
+int ff_grpo_loss(int B, int T, const float* lp_new, const float* lp_old, const float* adv, float clip_lo,
+                 float clip_hi, float* loss, float* grad_lp_new, void* ws, size_t ws_bytes, cudaStream_t stream) {
+    return ff::grpo_loss_impl(B, T, lp_new, lp_old, adv, nullptr, clip_lo, clip_hi, loss, grad_lp_new, ws, ws_bytes,
+                              stream);
+}
+
+int ff_grpo_loss_weighted(int B, int T, const float* lp_new, const float* lp_old, const float* adv,
+                          const float* step_w, float clip_lo, float clip_hi, float* loss, float* grad_lp_new,
+                          void* ws, size_t ws_bytes, cudaStream_t stream) {
+    if (!step_w) return ff::set_error(FF_ERR_INVALID_ARG, "loss: step_w is null (use ff_grpo_loss)");
+    return ff::grpo_loss_impl(B, T, lp_new, lp_old, adv, step_w, clip_lo, clip_hi, loss, grad_lp_new, ws, ws_bytes,
+                              stream);
+}
+
+int ff_group_advantage_multi(int n_groups, int G, int K, const float* rewards, const float* weights, int mode,
+                             float eps_A, float* adv, cudaStream_t stream) {
+    using namespace ff;
+    if (n_groups <= 0 || G <= 0 || K <= 0)
+        return set_error(FF_ERR_INVALID_ARG, "advantage (multi): n_groups=%d G=%d K=%d", n_groups, G, K);
+    if (G > 4096 || K > 64) return set_error(FF_ERR_UNSUPPORTED, "advantage (multi): G=%d > 4096 or K=%d > 64", G, K);
+    if (!rewards || !weights || !adv) return set_error(FF_ERR_INVALID_ARG, "advantage (multi): null pointer");
+    if (mode != FF_AGG_WEIGHTED_SUM && mode != FF_AGG_PER_REWARD)
+        return set_error(FF_ERR_INVALID_ARG, "advantage (multi): bad mode %d", mode);
+    if (!(eps_A >= 0.0f)) return set_error(FF_ERR_INVALID_ARG, "advantage (multi): eps_A must be >= 0");
+    ProfScope prof(stream, "group_advantage_multi", 0.0, 4.0 * n_groups * G * (K + 1));
+    const int warps_per_block = kThreads / 32;
+    const int grid = (n_groups + warps_per_block - 1) / warps_per_block;
+    group_advantage_multi_kernel<<<grid, kThreads, 0, stream>>>(n_groups, G, K, rewards, weights, mode, eps_A, adv);
+    return check_launch("group_advantage_multi_kernel");
 }
 
 }  // extern "C"

@@ -220,6 +220,19 @@ extern "C" int ff_sde_schedule(int kind, int n_steps, double shift, double eta, 
     return FF_OK;
 }
 
+extern "C" int ff_sde_schedule_window(int kind, int n_steps, double shift, double eta, double t_clamp,
+                                      int window_start, int window_len, double* t_out, double* sigma_out) {
+    using namespace ff;
+    if (window_start < 0 || window_len < 0 || window_start + window_len > n_steps)
+        return set_error(FF_ERR_INVALID_ARG, "schedule: window [%d, %d) outside the %d steps", window_start,
+                         window_start + window_len, n_steps);
+    const int rc = ff_sde_schedule(kind, n_steps, shift, eta, t_clamp, t_out, sigma_out);
+    if (rc) return rc;
+    for (int k = 0; k < n_steps; ++k)
+        if (k < window_start || k >= window_start + window_len) sigma_out[k] = 0.0;
+    return FF_OK;
+}
+
 // ---------------------------------------------------------------------------
 // ff_sde_step_logprob_noalloc: the same step for callers that cannot hand the
 // library any device memory of their own (see include/ff.h).  The per-chunk

@@ -18,6 +18,9 @@ FF_LP_SUM, FF_LP_MEAN = 0, 1
 FF_SCHED_FLOW_SDE, FF_SCHED_DANCE_SDE, FF_SCHED_ODE = 0, 1, 2
 FF_ARCH_MMDIT, FF_ARCH_WAN = 0, 1
 FF_ACT_NONE, FF_ACT_GELU, FF_ACT_SILU = 0, 1, 2
+FF_TSAMPLE_UNIFORM, FF_TSAMPLE_LOGIT_NORMAL, FF_TSAMPLE_DISCRETE = 0, 1, 2
+FF_AWM_SUM, FF_AWM_MEAN = 0, 1
+FF_AGG_WEIGHTED_SUM, FF_AGG_PER_REWARD = 0, 1
 
 
 class FFError(RuntimeError):
@@ -61,6 +64,13 @@ _SIGS = {
     "ff_group_advantage": ([_I, _I, _P, _F, _P, _P], _I),
     "ff_grpo_loss_workspace_size": ([_I, _I, C.POINTER(_SZ)], _I),
     "ff_grpo_loss": ([_I, _I, _P, _P, _P, _F, _F, _P, _P, _P, _SZ, _P], _I),
+    "ff_grpo_loss_weighted": ([_I, _I, _P, _P, _P, _P, _F, _F, _P, _P, _P, _SZ, _P], _I),
+    "ff_group_advantage_multi": ([_I, _I, _I, _P, _P, _I, _F, _P, _P], _I),
+    "ff_sde_schedule_window": ([_I, _I, _D, _D, _D, _I, _I, C.POINTER(_D), C.POINTER(_D)], _I),
+    "ff_sample_timesteps": ([_I, _I, _P, _F, _F, _P, _I, _P, _P], _I),
+    "ff_forward_process": ([_I, _I64, _P, _P, _P, _P, _P], _I),
+    "ff_awm_loss_workspace_size": ([_I, _I64, C.POINTER(_SZ)], _I),
+    "ff_awm_loss": ([_I, _I64, _P, _P, _P, _P, _I, _P, _P, _P, _P, _SZ, _P], _I),
     "ff_dit_weight_layout": ([C.POINTER(DitConfig), C.POINTER(TensorDesc), _I, C.POINTER(_I), C.POINTER(_I64)], _I),
     "ff_dit_create": ([C.POINTER(DitConfig), _P, C.POINTER(_P)], _I),
     "ff_dit_destroy": ([_P], _I),
@@ -132,6 +142,15 @@ def ff_sde_schedule(kind: int, n_steps: int, shift: float = 1.0, eta: float = 0.
     t = (_D * (n_steps + 1))()
     s = (_D * n_steps)()
     _call("ff_sde_schedule", kind, n_steps, shift, eta, t_clamp, t, s)
+    return list(t), list(s)
+
+
+def ff_sde_schedule_window(kind: int, n_steps: int, shift: float, eta: float, t_clamp: float, start: int,
+                           length: int):
+    """Host-only MixGRPO schedule: sigma zero outside steps [start, start + length)."""
+    t = (_D * (n_steps + 1))()
+    s = (_D * n_steps)()
+    _call("ff_sde_schedule_window", kind, n_steps, shift, eta, t_clamp, start, length, t, s)
     return list(t), list(s)
 
 
@@ -225,6 +244,64 @@ def ff_grpo_loss(lp_new, lp_old, adv, clip_lo: float, clip_hi: float, loss, grad
         ws = torch.empty(ff_grpo_loss_workspace_size(B, T), dtype=torch.uint8, device=lp_new.device)
     _call("ff_grpo_loss", B, T, _ptr(lp_new), _ptr(lp_old), _ptr(adv), clip_lo, clip_hi, _ptr(loss),
           _ptr(grad_lp_new), _ptr(ws), ws.numel(), _stream(stream))
+
+
+def ff_grpo_loss_weighted(lp_new, lp_old, adv, step_w, clip_lo: float, clip_hi: float, loss, grad_lp_new=None,
+                          ws=None, stream=None):
+    import torch
+    B, T = lp_new.shape
+    for n_, a in (("lp_new", lp_new), ("lp_old", lp_old), ("adv", adv), ("step_w", step_w), ("loss", loss)):
+        _check(a, torch.float32, n_)
+    if ws is None:
+        ws = torch.empty(ff_grpo_loss_workspace_size(B, T), dtype=torch.uint8, device=lp_new.device)
+    _call("ff_grpo_loss_weighted", B, T, _ptr(lp_new), _ptr(lp_old), _ptr(adv), _ptr(step_w), clip_lo, clip_hi,
+          _ptr(loss), _ptr(grad_lp_new), _ptr(ws), ws.numel(), _stream(stream))
+
+
+def ff_group_advantage_multi(rewards, G: int, weights, mode: int, eps_A: float, adv, stream=None):
+    """rewards: [N, K] fp32 (N a multiple of G); weights: [K] fp32; adv: [N] fp32."""
+    import torch
+    for n_, a in (("rewards", rewards), ("weights", weights), ("adv", adv)):
+        _check(a, torch.float32, n_)
+    N, K = rewards.shape
+    if N % G:
+        raise ValueError("rewards.shape[0] must be a multiple of G")
+    _call("ff_group_advantage_multi", N // G, G, K, _ptr(rewards), _ptr(weights), mode, eps_A, _ptr(adv),
+          _stream(stream))
+
+
+def ff_sample_timesteps(mode: int, draw, p0: float, p1: float, t_out, grid=None, stream=None):
+    import torch
+    _check(draw, torch.float32, "draw")
+    _check(t_out, torch.float32, "t_out")
+    _call("ff_sample_timesteps", mode, draw.numel(), _ptr(draw), p0, p1, _ptr(grid),
+          0 if grid is None else grid.numel(), _ptr(t_out), _stream(stream))
+
+
+def ff_forward_process(x0, eps, t, x_t, stream=None):
+    import torch
+    for n_, a in (("x0", x0), ("eps", eps), ("t", t), ("x_t", x_t)):
+        _check(a, torch.float32, n_)
+    B = x0.shape[0]
+    _call("ff_forward_process", B, x0.numel() // B, _ptr(x0), _ptr(eps), _ptr(t), _ptr(x_t), _stream(stream))
+
+
+def ff_awm_loss_workspace_size(B: int, D: int) -> int:
+    n = _SZ()
+    _call("ff_awm_loss_workspace_size", B, D, C.byref(n))
+    return n.value
+
+
+def ff_awm_loss(v, eps, x0, adv, reduce: int, loss, grad_v=None, err=None, ws=None, stream=None):
+    import torch
+    for n_, a in (("v", v), ("eps", eps), ("x0", x0), ("adv", adv), ("loss", loss)):
+        _check(a, torch.float32, n_)
+    B = v.shape[0]
+    D = v.numel() // B
+    if ws is None:
+        ws = torch.empty(ff_awm_loss_workspace_size(B, D), dtype=torch.uint8, device=v.device)
+    _call("ff_awm_loss", B, D, _ptr(v), _ptr(eps), _ptr(x0), _ptr(adv), reduce, _ptr(loss), _ptr(grad_v),
+          _ptr(err), _ptr(ws), ws.numel(), _stream(stream))
 
 
 class Dit:

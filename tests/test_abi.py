@@ -121,3 +121,31 @@ def test_dit_handle_and_config_validation(L):
     assert L.ff_dit_create(C.byref(bad), C.c_void_p(256), C.byref(h)) == 1
     bad = ffi.make_config(dict(cfg, head_dim=32, heads=8))
     assert L.ff_dit_create(C.byref(bad), C.c_void_p(256), C.byref(h)) == 2
+
+
+def test_schedule_window_matches_oracle(L):
+    t, s = ffi.ff_sde_schedule(ffi.FF_SCHED_FLOW_SDE, 10, 3.0, 0.7, 0.96)
+    tw, sw = ffi.ff_sde_schedule_window(ffi.FF_SCHED_FLOW_SDE, 10, 3.0, 0.7, 0.96, 2, 3)
+    assert tw == t
+    np.testing.assert_array_equal(sw, osde.window_sigma(s, 2, 3))
+    for bad in ((-1, 2), (9, 2), (0, 11)):
+        with pytest.raises(ffi.FFError):
+            ffi.ff_sde_schedule_window(ffi.FF_SCHED_FLOW_SDE, 10, 3.0, 0.7, 0.96, *bad)
+
+
+def test_awm_and_multi_reward_host_validation(L):
+    assert ffi.ff_awm_loss_workspace_size(4, 262144) == 4 * 65 * 8
+    assert ffi.ff_awm_loss_workspace_size(2, 1 << 26) == 2 * 1025 * 8
+    # rejected before any CUDA call
+    assert L.ff_awm_loss(2, 18, 16, 16, 16, 16, 0, 16, None, None, 16, 1 << 20, None) == 2   # D % 4
+    assert L.ff_awm_loss(2, 16, 16, 16, 16, 16, 3, 16, None, None, 16, 1 << 20, None) == 1   # bad reduce
+    assert L.ff_awm_loss(2, 16, 16, 16, 16, 16, 0, 16, None, None, 16, 8, None) == 3         # workspace
+    assert L.ff_awm_loss(2, 16, None, 16, 16, 16, 0, 16, None, None, 16, 1 << 20, None) == 1
+    assert L.ff_forward_process(2, 18, 16, 16, 16, 16, None) == 2
+    assert L.ff_forward_process(2, 16, 16, 16, None, 16, None) == 1
+    assert L.ff_sample_timesteps(5, 4, 16, 0.0, 1.0, None, 0, 16, None) == 1
+    assert L.ff_sample_timesteps(ffi.FF_TSAMPLE_DISCRETE, 4, 16, 0.0, 1.0, None, 0, 16, None) == 1
+    assert L.ff_sample_timesteps(ffi.FF_TSAMPLE_LOGIT_NORMAL, 4, 16, 0.0, -1.0, None, 0, 16, None) == 1
+    assert L.ff_group_advantage_multi(2, 4, 65, 16, 16, 0, 1e-4, 16, None) == 2
+    assert L.ff_group_advantage_multi(2, 4, 2, 16, 16, 7, 1e-4, 16, None) == 1
+    assert L.ff_grpo_loss_weighted(4, 2, 16, 16, 16, None, 0.2, 0.2, 16, None, 16, 64, None) == 1

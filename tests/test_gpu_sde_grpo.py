@@ -97,6 +97,8 @@ def test_group_advantage_parity(cuda, ng, G):
     r = synth.rewards(ng * G, seed=7 + G)
     if ng > 1:
         r[:G] = 0.25   # a constant group
+    if ng > 2:
+        r[G:2 * G] = 0.3   # one whose fp32 sum is inexact
     rg = _t(r, cuda)
     adv = torch.empty_like(rg)
     ffi.ff_group_advantage(rg, G, 1e-4, adv)
@@ -107,6 +109,8 @@ def test_group_advantage_parity(cuda, ng, G):
     np.testing.assert_array_equal(rg.cpu().numpy(), adv.cpu().numpy())
     if ng > 1:
         assert np.all(adv.cpu().numpy()[:G] == 0.0)
+    if ng > 2:
+        assert np.all(adv.cpu().numpy()[G:2 * G] == 0.0)
 
 
 @pytest.mark.parametrize("B,T,noise", [(32, 10, 0.01), (8, 3, 0.5), (4, 1, 0.3), (4096, 256, 0.4)])
