@@ -54,10 +54,37 @@ def parse_args():
 
 def workload_desc(cfg):
     f, h, w = cfg["grid"]
-    return (f"{cfg['name']}: {cfg['n_double']} double + {cfg['n_single']} single MMDiT blocks, H {cfg['hidden']}, "
-            f"{cfg['heads']}x{cfg['head_dim']} heads, MLP {cfg['mlp']}, {cfg['n_txt']} text + {f * h * w} latent "
-            f"tokens ({h}x{w} grid of 2x2 patches, 64-dim), batch {cfg['batch']} (groups of {cfg['group']}); "
-            f"per step: 1 velocity call + 1 SDE step with log-prob + group advantage + clipped GRPO loss")
+    if cfg.get("arch") == "wan":
+        blocks = f"{cfg['n_double']} WAN blocks (self-attention + text cross-attention + FFN)"
+        grid = f"{f}x{h}x{w} grid of 1x2x2 patches, 64-dim, 3-axis RoPE"
+    else:
+        blocks = f"{cfg['n_double']} double + {cfg['n_single']} single MMDiT blocks"
+        grid = f"{h}x{w} grid of 2x2 patches, 64-dim"
+    return (f"{cfg['name']}: {blocks}, H {cfg['hidden']}, {cfg['heads']}x{cfg['head_dim']} heads, MLP {cfg['mlp']}, "
+            f"{cfg['n_txt']} text + {f * h * w} latent tokens ({grid}), batch {cfg['batch']} (groups of "
+            f"{cfg['group']}); per step: 1 velocity call + 1 SDE step with log-prob + group advantage + clipped "
+            f"GRPO loss")
+
+
+def device_blob(ffi, cfg, dev, seed=0):
+    """Random-init weights drawn on the device (the large workloads hold up to
+    about 20e9 parameters, too many to draw on the host): N(0, 0.02)
+    matrices, zero biases, unit norm scales, as bf16."""
+    import numpy as np
+    import torch
+    import synth
+    specs, total = ffi.ff_dit_weight_layout(cfg)
+    blob = torch.zeros(total, dtype=torch.bfloat16, device=dev)
+    g = torch.Generator(device=dev)
+    g.manual_seed(seed)
+    for name, off, shape in specs:
+        n = int(np.prod(shape))
+        kind = synth.weight_kind(name)
+        if kind == "matrix":
+            blob[off:off + n] = (torch.randn(n, generator=g, device=dev) * 0.02).to(torch.bfloat16)
+        elif kind == "scale":
+            blob[off:off + n] = 1.0
+    return blob
 
 
 def load_peaks():
@@ -158,7 +185,10 @@ class OracleStep:
         import synth
         from oracle import dit as odit
         self.np, self.odit, self.cfg = np, odit, cfg
-        self.P = odit.widen_params(synth.weights(odit.param_specs(cfg), seed=0))
+        wan = cfg.get("arch") == "wan"
+        self.vel = odit.wan_velocity if wan else odit.velocity
+        specs = odit.wan_param_specs(cfg) if wan else odit.param_specs(cfg)
+        self.P = odit.widen_params(synth.weights(specs, seed=0))
         self.x = synth.initial_latent(cfg, batch=1)
         self.txt = odit.widen(synth.text_embeds(cfg, batch=1))
         self.eps = synth.step_noise(cfg, 0, batch=1)
@@ -173,7 +203,7 @@ class OracleStep:
         grid = osde.time_grid(cfg["sde_steps"], cfg["shift"])
         t, tn = grid[0:1], grid[1:2]
         sg = osde.sigma_flow_sde(t, cfg["eta"], cfg["t_clamp"])
-        v = self.odit.velocity(self.P, cfg, self.x, self.txt, t, img_rows=self.rows)
+        v = self.vel(self.P, cfg, self.x, self.txt, t, img_rows=self.rows)
         xn, lp = osde.sde_step_logprob(self.x[:, self.rows], v, t, tn, sg, eps=self.eps[:, self.rows])
         adv = ogrpo.group_advantage(self.rewards, cfg["group"], cfg["eps_adv"])
         lpn = np.full((cfg["group"], 1), lp[0])
@@ -353,8 +383,9 @@ def awm_step(args, ffi, model, cfg, dev, x0, txt, eps, rewards, timed, world):
     xt = torch.empty_like(x0)
     v = torch.empty_like(x0)
     gv = torch.empty_like(x0)
-    adv = torch.empty(B, device=dev)
-    ffi.ff_group_advantage(rewards, B, 1e-4, adv)
+    adv_all = torch.empty(rewards.numel(), device=dev)
+    ffi.ff_group_advantage(rewards, rewards.numel(), 1e-4, adv_all)
+    adv = adv_all[:B]
     loss = torch.empty(1, device=dev)
     ws = torch.empty(model.workspace_size(B), dtype=torch.uint8, device=dev)
     ws_awm = torch.empty(ffi.ff_awm_loss_workspace_size(B, D), dtype=torch.uint8, device=dev)
@@ -368,7 +399,7 @@ def awm_step(args, ffi, model, cfg, dev, x0, txt, eps, rewards, timed, world):
     for _ in range(args.warmup):
         step()
     ms = timed(step, args.steps) / args.steps
-    ffi.ff_prof_enable(64 * args.steps + 64)
+    ffi.ff_prof_enable((16 * (cfg["n_double"] + cfg["n_single"]) + 64) * args.steps + 64)
     timed(step, args.steps)
     recs = ffi.ff_prof_records()
     ffi.ff_prof_disable()
@@ -418,7 +449,11 @@ def run_ours(args):
     D = Ni * P
     steps_per_step = 1
 
-    blob = weights.pack(cfg, lambda n, s: synth.weight(n, s, synth.weight_kind(n), 0), dev)
+    _, n_params = ffi.ff_dit_weight_layout(cfg)
+    if n_params > 2e9:
+        blob = device_blob(ffi, cfg, dev)
+    else:
+        blob = weights.pack(cfg, lambda n, s: synth.weight(n, s, synth.weight_kind(n), 0), dev)
     model = ffi.Dit(cfg, blob)
     tgrid, sig = ffi.ff_sde_schedule(ffi.FF_SCHED_FLOW_SDE, cfg["sde_steps"], cfg["shift"], cfg["eta"],
                                      cfg["t_clamp"])
@@ -429,7 +464,10 @@ def run_ours(args):
     h_t = np.full(B, tgrid[0], np.float32)
     h_tn = np.full(B, tgrid[1], np.float32)
     h_sg = np.full(B, sig[0], np.float32)
-    h_r = synth.rewards(B, seed=7 + seed)
+    # rewards of whole groups (a WAN group of 8 is rolled out one sample at a
+    # time, so it can be larger than the batch); the loss uses the batch's own
+    n_r = -(-B // G) * G
+    h_r = synth.rewards(n_r, seed=7 + seed)
     h_lpold = synth.logprob_jitter((B, 1), seed=9 + seed)   # + lp_new, added on device below
 
     def dev_t(a, dtype=None):
@@ -443,7 +481,8 @@ def run_ours(args):
     x_next = torch.empty_like(x)
     logp = torch.empty((B, 1), dtype=torch.float32, device=dev)
     lp_old = torch.empty((B, 1), dtype=torch.float32, device=dev)
-    adv = torch.empty(B, dtype=torch.float32, device=dev)
+    adv_all = torch.empty(n_r, dtype=torch.float32, device=dev)
+    adv = adv_all[:B]
     loss = torch.zeros(1, dtype=torch.float32, device=dev)
     grad = torch.empty((B, 1), dtype=torch.float32, device=dev)
     ws = torch.empty(model.workspace_size(B), dtype=torch.uint8, device=dev)
@@ -459,7 +498,7 @@ def run_ours(args):
     def step(xi=x, txti=txt, epsi=eps, ti=t, tni=tn, sgi=sg, ri=rewards, lpo=lp_old):
         model.ff_dit_velocity(xi, txti, ti, v, ws)
         ffi.ff_sde_step_logprob(xi, v, epsi, x_next, ti, tni, sgi, logp, ws=ws_sde)
-        ffi.ff_group_advantage(ri, G, cfg["eps_adv"], adv)
+        ffi.ff_group_advantage(ri, G, cfg["eps_adv"], adv_all)
         ffi.ff_grpo_loss(logp, lpo, adv, cfg["clip"], cfg["clip"], loss, grad, ws=ws_loss)
 
     clocks = ClockSampler(local) if rank == 0 else None
@@ -491,7 +530,9 @@ def run_ours(args):
     value = world * tokens_per_step / (ms_step / 1e3)
 
     # ---- per-kernel CUDA-event durations over the same K steps
-    ffi.ff_prof_enable(200 * args.steps + 64)
+    # launches per step: a few per block plus the fixed ones, with headroom
+    per_step = 16 * (cfg["n_double"] + cfg["n_single"]) + 64
+    ffi.ff_prof_enable(per_step * args.steps + 64)
     timed(step, args.steps)
     recs = ffi.ff_prof_records()
     ffi.ff_prof_disable()
@@ -571,7 +612,8 @@ def run_ours(args):
                 "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
                 "config": {"workload": workload_desc(cfg), "batch": B, "group": G, "n_txt": Nt, "n_img": Ni,
                            "hidden": cfg["hidden"], "parallelism": f"dp{world} (independent groups per GPU)",
-                           "l2": "no flush: per-step working set (0.76 GB weights + 1.4 GB activations) > 129 MB L2"},
+                           "l2": f"no flush: per-step working set ({2 * n_params / 1e9:.2f} GB weights + "
+                                 f"{ws.numel() / 1e9:.2f} GB activation workspace) > 129 MB L2"},
                 "roofline": roofline,
                 "dit_tflops": dit_flops / (ms_step / 1e3) / 1e12,
                 "secondary_rooflines": secondary,
