@@ -332,6 +332,34 @@ int ff_dit_velocity(const ff_dit* model, int B, const float* x_t, const void* tx
                     const float* t, float* v_out, void* ws, size_t ws_bytes,
                     cudaStream_t stream);
 
+/* ------------------------------------------------------------------------
+ * Trajectory sampling (paper Sec. 3.1: the SDE rollout that Flow-GRPO's
+ * policy gradient scores, "repeated forward passes for trajectory
+ * sampling").  S denoise steps; at step k = 0 .. S-1, for every sample:
+ *   v = v_theta(x_k, t_k);  x_{k+1} = Eq. 1 step from t_k to t_{k+1} with
+ *   sigma_k and noise eps[k] (ff_sde_step_logprob, SAMPLE mode);
+ *   logp[b * S + k] = log p(x_{k+1} | x_k).
+ * A step with sigma_k == 0 is an ODE step (log-prob 0), so MixGRPO windows
+ * come from ff_sde_schedule_window.
+ *   x:     [B, N_i, P] fp32: x_0 on entry, x_S on return (in place).
+ *   txt:   [B, N_t, D_txt] bf16 text embeddings (as ff_dit_velocity).
+ *   t:     [S + 1] fp32 device, the shared time grid (t_0 > ... > t_S > 0 is
+ *          not checked: device values); sigma: [S] fp32 device.
+ *   eps:   [S, B, N_i, P] fp32 device noise.
+ *   traj:  [S + 1, B, N_i, P] fp32 device (x_0 .. x_S kept, the states the
+ *          training pass re-scores) or NULL.
+ *   logp:  [B, S] fp32 device, per-step log-probs of every sample.
+ *   reduce: FF_LP_SUM or FF_LP_MEAN.
+ *   ws:    at least ff_rollout_workspace_size(model, B, S) bytes, 256-byte
+ *          aligned (holds the velocity workspace, v and the per-step times).
+ * Nothing synchronises, so the call can be captured in a CUDA graph (with
+ * the launch timer off).
+ * ------------------------------------------------------------------------ */
+int ff_rollout_workspace_size(const ff_dit* model, int B, int S, size_t* bytes);
+int ff_rollout(const ff_dit* model, int B, int S, float* x, const void* txt, const float* t,
+               const float* sigma, const float* eps, float* traj, float* logp, int reduce,
+               void* ws, size_t ws_bytes, cudaStream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

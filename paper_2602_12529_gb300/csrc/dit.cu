@@ -199,11 +199,6 @@ void set_qk_norm(GemmEpilogue& e, const ff_dit_config& c, int qk_cols, const __n
     e.axes2 = c.rope_axes[2];
 }
 
-#define FF_TRY(expr)                \
-    do {                            \
-        const int rc_ = (expr);     \
-        if (rc_ != FF_OK) return rc_; \
-    } while (0)
 
 // WAN-style velocity: latent tokens only in the residual stream; the text is
 // embedded once per call and feeds every block's cross-attention keys and
@@ -360,6 +355,9 @@ int wan_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, cons
 }
 
 }  // namespace
+
+const ff_dit_config& model_config(const ff_dit* m) { return m->cfg; }
+
 }  // namespace ff
 
 extern "C" {

@@ -20,6 +20,16 @@ int num_sms();                             // SM count of the current device
 
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+// Return the status of a library call from the enclosing function if it failed.
+#define FF_TRY(expr)                \
+    do {                            \
+        const int rc_ = (expr);     \
+        if (rc_ != FF_OK) return rc_; \
+    } while (0)
+
+// Configuration of a DiT handle (its struct is private to dit.cu).
+const ff_dit_config& model_config(const ff_dit* m);
+
 // ---- optional launch timing (ff_prof_*): RAII scope around one launch ----
 struct ProfScope {
     ProfScope(cudaStream_t s, const char* name, double flops, double bytes);

@@ -76,6 +76,8 @@ _SIGS = {
     "ff_dit_destroy": ([_P], _I),
     "ff_dit_workspace_size": ([_P, _I, C.POINTER(_SZ)], _I),
     "ff_dit_velocity": ([_P, _I, _P, _P, _P, _P, _P, _SZ, _P], _I),
+    "ff_rollout_workspace_size": ([_P, _I, _I, C.POINTER(_SZ)], _I),
+    "ff_rollout": ([_P, _I, _I, _P, _P, _P, _P, _P, _P, _P, _I, _P, _SZ, _P], _I),
     "ff_debug_gemm": ([_I, _I, _I, _P, _I64, _P, _I64, _P, _I, _I, _P, _I64, _P], _I),
     "ff_debug_gemm_gated": ([_I, _I, _I, _P, _I64, _P, _I64, _P, _P, _I64, _P, _I64, _I, _P], _I),
     "ff_debug_attention": ([_I, _I, _I, _I, _P, _I64, _P, _I64, _I, _P, _I64, _P, _I64, _P], _I),
@@ -340,6 +342,24 @@ class Dit:
         B = x_t.shape[0]
         _call("ff_dit_velocity", self._h, B, _ptr(x_t), _ptr(txt), _ptr(t), _ptr(v_out), _ptr(ws), ws.numel(),
               _stream(stream))
+
+    def rollout_workspace_size(self, B: int, S: int) -> int:
+        n = _SZ()
+        _call("ff_rollout_workspace_size", self._h, B, S, C.byref(n))
+        return n.value
+
+    def ff_rollout(self, x, txt, t, sigma, eps, logp, traj=None, reduce: int = FF_LP_SUM, ws=None, stream=None):
+        """x [B, ...] updated in place; t [S+1], sigma [S]; eps [S, B, ...];
+        logp [B, S]; traj [S+1, B, ...] or None."""
+        import torch
+        for n_, a in (("x", x), ("t", t), ("sigma", sigma), ("eps", eps), ("logp", logp)):
+            _check(a, torch.float32, n_)
+        _check(txt, torch.bfloat16, "txt")
+        B, S = x.shape[0], sigma.numel()
+        if ws is None:
+            ws = torch.empty(self.rollout_workspace_size(B, S), dtype=torch.uint8, device=x.device)
+        _call("ff_rollout", self._h, B, S, _ptr(x), _ptr(txt), _ptr(t), _ptr(sigma), _ptr(eps), _ptr(traj),
+              _ptr(logp), reduce, _ptr(ws), ws.numel(), _stream(stream))
 
 
 def ff_check_device_status(stream=None) -> int:
