@@ -423,6 +423,33 @@ def synth_n_img(cfg):
     return synth.n_img(cfg)
 
 
+# ---- multi-rank host logic (one process per GPU; weak scaling) ----------
+# The path shards by whole groups: every rank rolls out its own B samples
+# (B / G prompts) with its own seeds, so no collective touches the data path.
+# Timing is the slowest rank's, and the reported value counts every rank's
+# units.
+
+def rank_seed(rank: int) -> int:
+    """Seed offset of a rank's inputs (distinct prompts, noise and rewards)."""
+    return 1000 * rank
+
+
+def max_over_ranks(ms: float, world: int, device=None) -> float:
+    """Slowest rank's elapsed time (all-reduce MAX); the identity at N = 1."""
+    if world <= 1:
+        return ms
+    import torch
+    import torch.distributed as dist
+    m = torch.tensor([ms], device=device)
+    dist.all_reduce(m, op=dist.ReduceOp.MAX)
+    return float(m.item())
+
+
+def whole_job_rate(world: int, units_per_rank_step: float, ms_step: float) -> float:
+    """Units all ranks processed per second, at the slowest rank's step time."""
+    return world * units_per_rank_step / (ms_step / 1e3)
+
+
 def run_ours(args):
     import numpy as np
     import torch
@@ -457,7 +484,7 @@ def run_ours(args):
     model = ffi.Dit(cfg, blob)
     tgrid, sig = ffi.ff_sde_schedule(ffi.FF_SCHED_FLOW_SDE, cfg["sde_steps"], cfg["shift"], cfg["eta"],
                                      cfg["t_clamp"])
-    seed = 1000 * rank
+    seed = rank_seed(rank)
     h_x = synth.initial_latent(cfg, seed=2 + seed)
     h_txt = synth.text_embeds(cfg, seed=1 + seed).view(np.int16)
     h_eps = synth.step_noise(cfg, 0, seed=100 + seed)
@@ -516,18 +543,15 @@ def run_ours(args):
             fn()
         e1.record(stream)
         torch.cuda.synchronize(dev)
-        ms = e0.elapsed_time(e1)
+        ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
         if world > 1:
-            m = torch.tensor([ms], device=dev)
-            dist.all_reduce(m, op=dist.ReduceOp.MAX)
-            ms = float(m.item())
             dist.barrier()
         return ms
 
     ms_total = timed(step, args.steps)
     ms_step = ms_total / args.steps
     tokens_per_step = B * Ni * steps_per_step
-    value = world * tokens_per_step / (ms_step / 1e3)
+    value = whole_job_rate(world, tokens_per_step, ms_step)
 
     # ---- per-kernel CUDA-event durations over the same K steps
     # launches per step: a few per block plus the fixed ones, with headroom
@@ -593,7 +617,7 @@ def run_ours(args):
 
     e2e_step()
     ms_e2e = timed(e2e_step, args.steps) / args.steps
-    e2e_value = world * tokens_per_step / (ms_e2e / 1e3)
+    e2e_value = whole_job_rate(world, tokens_per_step, ms_e2e)
     awm = awm_step(args, ffi, model, cfg, dev, x, txt, eps, rewards, timed, world)
     sweep = hbm_sweep(ffi, dev, hbm) if rank == 0 and not args.no_sweep else None
     clk = clocks.stop() if clocks else None
