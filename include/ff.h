@@ -66,6 +66,11 @@ extern "C" {
 #define FF_AGG_WEIGHTED_SUM 0  /* r = sum_k w_k R_k, then group-normalise r          */
 #define FF_AGG_PER_REWARD 1    /* group-normalise each R_k, then sum_k w_k A_k (GDPO) */
 
+#define FF_A_MK 0   /* ff_gemm: A stored [M, K] */
+#define FF_A_KM 1   /* ff_gemm: A stored [K, M] */
+#define FF_B_NK 0   /* ff_gemm: B stored [N, K] (D = A B^T, the nn.Linear product) */
+#define FF_B_KN 1   /* ff_gemm: B stored [K, N] (D = A B) */
+
 #define FF_ARCH_MMDIT 0   /* Flux / Qwen-Image style double + single stream */
 #define FF_ARCH_WAN 1     /* WAN-style video DiT: self-attn + text cross-attn + FFN */
 
@@ -331,6 +336,25 @@ int ff_dit_workspace_size(const ff_dit* model, int B, size_t* bytes);
 int ff_dit_velocity(const ff_dit* model, int B, const float* x_t, const void* txt,
                     const float* t, float* v_out, void* ws, size_t ws_bytes,
                     cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
+ * bf16 GEMM with fp32 accumulation on the tcgen05 kernels of the velocity:
+ *   out[M, N] = act(op(A) op(B) + bias),  op(A) [M, K], op(B) [K, N]
+ * a_layout FF_A_MK: A stored [M, K] (lda >= K); FF_A_KM: A stored [K, M]
+ * (lda >= M).  b_layout FF_B_NK: B stored [N, K] (ldb >= K); FF_B_KN: B
+ * stored [K, N] (ldb >= N).  For a Linear y = x W^T (W [N_out, N_in]) on T
+ * tokens, the training backward (the gradient pass that follows the rollout
+ * in Flow-GRPO, Sec. 3.1) needs
+ *   forward      y  = x W^T:   A = x  [T, N_in]  (MK), B = W [N_out, N_in] (NK)
+ *   input grad   dx = dy W:    A = dy [T, N_out] (MK), B = W                (KN)
+ *   weight grad  dW = dy^T x:  A = dy [T, N_out] (KM), B = x [T, N_in]      (KN)
+ * bias: [N] bf16 or NULL; act: FF_ACT_NONE / GELU / SILU; out: bf16
+ * (out_f32 = 0) or fp32 [M, N] with ldo.  K and every leading dimension a
+ * multiple of 8, N a multiple of 32, bases 16-byte aligned.
+ * ------------------------------------------------------------------------ */
+int ff_gemm(int M, int N, int K, const void* A, int64_t lda, int a_layout, const void* B,
+            int64_t ldb, int b_layout, const void* bias, int act, int out_f32, void* out,
+            int64_t ldo, cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
  * Trajectory sampling (paper Sec. 3.1: the SDE rollout that Flow-GRPO's

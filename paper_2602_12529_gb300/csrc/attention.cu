@@ -105,19 +105,6 @@ __device__ __forceinline__ void tc_mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem,
         ::"r"(d_tmem), "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
         : "memory");
 }
-// B operand stored MN-major with 128-byte swizzle (V: rows = K = tokens,
-// 64 contiguous d per 128-byte row): leading byte offset = distance between
-// 64-wide d blocks, stride byte offset = distance between 8-token groups.
-__device__ __forceinline__ uint64_t smem_desc_mn_sw128(uint32_t saddr, uint32_t lbo_bytes) {
-    uint64_t d = 0;
-    d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
-    d |= static_cast<uint64_t>((lbo_bytes >> 4) & 0x3FFFu) << 16;
-    d |= static_cast<uint64_t>(1024 >> 4) << 32;
-    d |= static_cast<uint64_t>(1) << 46;
-    d |= static_cast<uint64_t>(2) << 61;
-    return d;
-}
-
 // Barriers.  Per query tile the chain S -> softmax -> P -> O += P V -> next S
 // is strictly ordered, so no waiter can lag two phases behind a parity wait.
 constexpr int kMaxSlots = 8;

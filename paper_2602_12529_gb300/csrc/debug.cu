@@ -1,6 +1,6 @@
 // debug.cu -- exported per-kernel entry points (include/ff_debug.h) used by
-// the stage-wise parity tests.  They only marshal arguments to the same
-// launchers ff_dit_velocity uses.
+// the stage-wise parity tests, and the general ff_gemm (include/ff.h).  They
+// only marshal arguments to the same launchers ff_dit_velocity uses.
 #include "../../include/ff_debug.h"
 #include "internal.h"
 
@@ -17,6 +17,23 @@ int ff_debug_gemm(int M, int N, int K, const void* A, int64_t lda, const void* B
     e.out0 = out;
     e.ld0 = ldo;
     return gemm_bf16(A, lda, B, ldb, M, N, K, e, stream);
+}
+
+int ff_gemm(int M, int N, int K, const void* A, int64_t lda, int a_layout, const void* B, int64_t ldb, int b_layout,
+            const void* bias, int act, int out_f32, void* out, int64_t ldo, cudaStream_t stream) {
+    using namespace ff;
+    if (act < FF_ACT_NONE || act > FF_ACT_SILU) return set_error(FF_ERR_INVALID_ARG, "gemm: bad act %d", act);
+    if ((a_layout != FF_A_MK && a_layout != FF_A_KM) || (b_layout != FF_B_NK && b_layout != FF_B_KN))
+        return set_error(FF_ERR_INVALID_ARG, "gemm: bad operand layout (%d, %d)", a_layout, b_layout);
+    GemmArgs g{A, lda, B, ldb, M, N, K, GemmEpilogue{}};
+    g.a_mn = a_layout == FF_A_KM;
+    g.b_mn = b_layout == FF_B_KN;
+    g.epi.act = act;
+    g.epi.out_f32 = out_f32 ? 1 : 0;
+    g.epi.bias = static_cast<const __nv_bfloat16*>(bias);
+    g.epi.out0 = out;
+    g.epi.ld0 = ldo;
+    return gemm_bf16_group(&g, 1, stream);
 }
 
 int ff_debug_gemm_gated(int M, int N, int K, const void* A, int64_t lda, const void* B, int64_t ldb, const void* bias,

@@ -387,6 +387,7 @@ __device__ __forceinline__ bool epilogue_tile(const GemmEpilogue& epi, int M, in
 // (the text stream of a double-stream block) fills the tail of a large one.
 struct GemmGroup {
     int M[2], N[2], K[2];
+    int a_mn[2], b_mn[2];   // operand storage per problem (see GemmArgs)
     int num_m[2], num_n[2];
     int tiles0, tiles;
     GemmEpilogue epi[2];
@@ -472,14 +473,26 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_cons
                 uint8_t* sa = smem + stage * C::kStageBytes;
                 uint8_t* sb = sa + C::kABytes;
                 mbar_arrive_expect_tx(&full_bar[stage], C::kStageBytes);
-                tma_load_2d(sa, ta, &full_bar[stage], kb * BK, mb * BM);
-                tma_load_2d(sb, tb, &full_bar[stage], kb * BK, nb * BN);
+                // K-major operands: one box of rows x 64 K; MN-major: boxes
+                // of 64 K rows x 64 MN per 64-wide block (8 KB each)
+                if (g.a_mn[pr]) {
+                    for (int j = 0; j < BM / 64; ++j)
+                        tma_load_2d(sa + j * 8192, ta, &full_bar[stage], mb * BM + 64 * j, kb * BK);
+                } else {
+                    tma_load_2d(sa, ta, &full_bar[stage], kb * BK, mb * BM);
+                }
+                if (g.b_mn[pr]) {
+                    for (int j = 0; j < BN / 64; ++j)
+                        tma_load_2d(sb + j * 8192, tb, &full_bar[stage], nb * BN + 64 * j, kb * BK);
+                } else {
+                    tma_load_2d(sb, tb, &full_bar[stage], kb * BK, nb * BN);
+                }
                 if (++stage == C::kStages) { stage = 0; phase ^= 1; }
             }
         }
     } else if (warp == 1 && lane == 0) {
         // ---------------- MMA issuer
-        constexpr uint32_t idesc = idesc_bf16_f32(BM, BN);
+        constexpr uint32_t idesc0 = idesc_bf16_f32(BM, BN);
         int stage = 0;
         uint32_t phase = 0;
         int acc = 0;
@@ -487,6 +500,9 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_cons
         for (int tile = blockIdx.x; tile < g.tiles && !*abort_flag; tile += gridDim.x) {
             const int pr = tile < g.tiles0 ? 0 : 1;
             const int num_k = (g.K[pr] + BK - 1) / BK;
+            const bool amn = g.a_mn[pr] != 0, bmn = g.b_mn[pr] != 0;
+            const uint32_t idesc = idesc0 | (static_cast<uint32_t>(amn) << 15) | (static_cast<uint32_t>(bmn) << 16);
+            const uint64_t a_step = amn ? 128 : 2, b_step = bmn ? 128 : 2;   // one K16 step, encoded >> 4
             if (!mbar_wait(&tempty_bar[acc], acc_phase ^ 1)) {
                 report_status(status, kStatusWaitTimeout);
                 *abort_flag = 1;
@@ -505,14 +521,11 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_cons
                 tc_fence_after();
                 const uint32_t sa = smem_u32(smem + stage * C::kStageBytes);
                 const uint32_t sb = sa + C::kABytes;
-                const uint64_t da = smem_desc_k_sw128(sa);
-                const uint64_t db = smem_desc_k_sw128(sb);
+                const uint64_t da = amn ? smem_desc_mn_sw128(sa, 8192) : smem_desc_k_sw128(sa);
+                const uint64_t db = bmn ? smem_desc_mn_sw128(sb, 8192) : smem_desc_k_sw128(sb);
 #pragma unroll
-                for (int k = 0; k < BK / 16; ++k) {
-                    // +32 bytes per 16-element K step (encoded >> 4)
-                    tc_mma_bf16(d_tmem, da + static_cast<uint64_t>(2 * k), db + static_cast<uint64_t>(2 * k), idesc,
-                                (kb | k) != 0 ? 1u : 0u);
-                }
+                for (int k = 0; k < BK / 16; ++k)
+                    tc_mma_bf16(d_tmem, da + a_step * k, db + b_step * k, idesc, (kb | k) != 0 ? 1u : 0u);
                 tc_commit(&empty_bar[stage]);
                 if (++stage == C::kStages) { stage = 0; phase ^= 1; }
             }
@@ -684,14 +697,23 @@ gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_constan
                 uint8_t* sb = sa + C::kABytes;
                 const uint32_t fb = mapa_shared(smem_u32(&full_bar[stage]), 0);
                 if (rank == 0) mbar_arrive_expect_tx(&full_bar[stage], 2 * C::kStageBytes);
-                tma_load_2d_pair(sa, ta, fb, kb * BK, mb * PBM + rank * 128);
-                tma_load_2d_pair(sb, tb, fb, kb * BK, nb * PBN + rank * (PBN / 2));
+                const int ma = mb * PBM + rank * 128, nbb = nb * PBN + rank * (PBN / 2);
+                if (g.a_mn[pr]) {
+                    for (int j = 0; j < 2; ++j) tma_load_2d_pair(sa + j * 8192, ta, fb, ma + 64 * j, kb * BK);
+                } else {
+                    tma_load_2d_pair(sa, ta, fb, kb * BK, ma);
+                }
+                if (g.b_mn[pr]) {
+                    for (int j = 0; j < 2; ++j) tma_load_2d_pair(sb + j * 8192, tb, fb, nbb + 64 * j, kb * BK);
+                } else {
+                    tma_load_2d_pair(sb, tb, fb, kb * BK, nbb);
+                }
                 if (++stage == kPairStages) { stage = 0; phase ^= 1; }
             }
         }
     } else if (warp == 1 && lane == 0 && rank == 0) {
         // ---------------- MMA issuer (leader only): 256 x 256 x 16 per instruction
-        constexpr uint32_t idesc = idesc_bf16_f32(PBM, PBN);
+        constexpr uint32_t idesc0 = idesc_bf16_f32(PBM, PBN);
         int stage = 0;
         uint32_t phase = 0;
         int acc = 0;
@@ -699,6 +721,9 @@ gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_constan
         for (int tile = cluster; tile < g.tiles && !*abort_flag; tile += nclusters) {
             const int pr = tile < g.tiles0 ? 0 : 1;
             const int num_k = (g.K[pr] + BK - 1) / BK;
+            const bool amn = g.a_mn[pr] != 0, bmn = g.b_mn[pr] != 0;
+            const uint32_t idesc = idesc0 | (static_cast<uint32_t>(amn) << 15) | (static_cast<uint32_t>(bmn) << 16);
+            const uint64_t a_step = amn ? 128 : 2, b_step = bmn ? 128 : 2;
             if (!mbar_wait(&tempty_bar[acc], acc_phase ^ 1)) {
                 report_status(status, kStatusWaitTimeout);
                 *abort_flag = 1;
@@ -717,12 +742,11 @@ gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_constan
                 tc_fence_after();
                 const uint32_t sa = smem_u32(smem + stage * C::kStageBytes);
                 const uint32_t sb = sa + C::kABytes;
-                const uint64_t da = smem_desc_k_sw128(sa);
-                const uint64_t db = smem_desc_k_sw128(sb);
+                const uint64_t da = amn ? smem_desc_mn_sw128(sa, 8192) : smem_desc_k_sw128(sa);
+                const uint64_t db = bmn ? smem_desc_mn_sw128(sb, 8192) : smem_desc_k_sw128(sb);
 #pragma unroll
                 for (int k = 0; k < BK / 16; ++k)
-                    tc_mma_bf16_pair(d_tmem, da + static_cast<uint64_t>(2 * k), db + static_cast<uint64_t>(2 * k), idesc,
-                                     (kb | k) != 0 ? 1u : 0u);
+                    tc_mma_bf16_pair(d_tmem, da + a_step * k, db + b_step * k, idesc, (kb | k) != 0 ? 1u : 0u);
                 tc_commit_pair_mc(&empty_bar[stage], 0x3);
                 if (++stage == kPairStages) { stage = 0; phase ^= 1; }
             }
@@ -830,9 +854,10 @@ int launch_pair(const GemmArgs* p, int n, cudaStream_t stream) {
         const GemmArgs& a = p[i < n ? i : 0];
         int rc = make_out_maps(a, &om.m[2 * i]);
         if (rc) return rc;
-        rc = make_tmap_bf16(&ta[i], a.A, a.M, a.K, a.lda, 128);
+        rc = a.a_mn ? make_tmap_bf16(&ta[i], a.A, a.K, a.M, a.lda, 64) : make_tmap_bf16(&ta[i], a.A, a.M, a.K, a.lda, 128);
         if (rc) return rc;
-        rc = make_tmap_bf16(&tb[i], a.B, a.N, a.K, a.ldb, PBN / 2);
+        rc = a.b_mn ? make_tmap_bf16(&tb[i], a.B, a.K, a.N, a.ldb, 64)
+                    : make_tmap_bf16(&tb[i], a.B, a.N, a.K, a.ldb, PBN / 2);
         if (rc) return rc;
         if (a.epi.epi == EPI_GATED_RESIDUAL) {
             rc = make_tmap_f32_sw128(&tr[i], a.epi.resid, a.M, a.N, a.epi.ld_resid, 128);
@@ -843,6 +868,8 @@ int launch_pair(const GemmArgs* p, int n, cudaStream_t stream) {
         g.M[i] = a.M;
         g.N[i] = a.N;
         g.K[i] = a.K;
+        g.a_mn[i] = a.a_mn;
+        g.b_mn[i] = a.b_mn;
         g.num_m[i] = (a.M + PBM - 1) / PBM;
         g.num_n[i] = (a.N + PBN - 1) / PBN;
         g.epi[i] = a.epi;
@@ -879,9 +906,9 @@ int launch(const GemmArgs* p, int n, cudaStream_t stream) {
         const GemmArgs& a = p[i < n ? i : 0];
         int rc = make_out_maps(a, &om.m[2 * i]);
         if (rc) return rc;
-        rc = make_tmap_bf16(&ta[i], a.A, a.M, a.K, a.lda, BM);
+        rc = a.a_mn ? make_tmap_bf16(&ta[i], a.A, a.K, a.M, a.lda, 64) : make_tmap_bf16(&ta[i], a.A, a.M, a.K, a.lda, BM);
         if (rc) return rc;
-        rc = make_tmap_bf16(&tb[i], a.B, a.N, a.K, a.ldb, BN);
+        rc = a.b_mn ? make_tmap_bf16(&tb[i], a.B, a.K, a.N, a.ldb, 64) : make_tmap_bf16(&tb[i], a.B, a.N, a.K, a.ldb, BN);
         if (rc) return rc;
         if (a.epi.epi == EPI_GATED_RESIDUAL) {
             rc = make_tmap_f32_sw128(&tr[i], a.epi.resid, a.M, a.N, a.epi.ld_resid, BM);
@@ -892,6 +919,8 @@ int launch(const GemmArgs* p, int n, cudaStream_t stream) {
         g.M[i] = a.M;
         g.N[i] = a.N;
         g.K[i] = a.K;
+        g.a_mn[i] = a.a_mn;
+        g.b_mn[i] = a.b_mn;
         g.num_m[i] = (a.M + BM - 1) / BM;
         g.num_n[i] = (a.N + BN - 1) / BN;
         g.epi[i] = a.epi;
@@ -1052,9 +1081,9 @@ int check_args(const GemmArgs& a) {
     if (!a.A || !a.B) return set_error(FF_ERR_INVALID_ARG, "gemm: null operand");
     if (M <= 0 || N <= 0 || K <= 0) return set_error(FF_ERR_INVALID_ARG, "gemm: bad shape %d x %d x %d", M, N, K);
     if (N % 32 != 0) return set_error(FF_ERR_UNSUPPORTED, "gemm: N=%d not a multiple of 32", N);
-    if (K % 8 != 0 || a.lda % 8 != 0 || a.ldb % 8 != 0 || a.lda < K || a.ldb < K)
-        return set_error(FF_ERR_UNSUPPORTED, "gemm: K/ld must be multiples of 8 (K=%d lda=%lld ldb=%lld)", K,
-                         (long long)a.lda, (long long)a.ldb);
+    if (K % 8 != 0 || a.lda % 8 != 0 || a.ldb % 8 != 0 || a.lda < (a.a_mn ? M : K) || a.ldb < (a.b_mn ? N : K))
+        return set_error(FF_ERR_UNSUPPORTED, "gemm: K/ld must be multiples of 8 and cover the rows (K=%d lda=%lld ldb=%lld)",
+                         K, (long long)a.lda, (long long)a.ldb);
     if (e.bias && !aligned16(e.bias)) return set_error(FF_ERR_INVALID_ARG, "gemm: bias not 16-byte aligned");
     if (e.epi == EPI_GATED_RESIDUAL) {
         if (!e.resid || e.rows_per_sample <= 0 || !aligned16(e.resid) || (e.gate && !aligned16(e.gate)) ||
@@ -1107,7 +1136,8 @@ int gemm_bf16_group(const GemmArgs* p, int n, cudaStream_t stream) {
         return launch<256>(p, n, stream);
     }
     const GemmArgs& a = p[0];
-    const bool gemv_ok = a.K <= kGemvMaxK && a.epi.epi == EPI_STORE && a.epi.split_n >= a.N && a.epi.qk_cols == 0 &&
+    const bool gemv_ok = !a.a_mn && !a.b_mn && a.K <= kGemvMaxK && a.epi.epi == EPI_STORE && a.epi.split_n >= a.N &&
+                         a.epi.qk_cols == 0 &&
                          aligned16(a.A) && aligned16(a.B) && a.lda % 8 == 0 && a.ldb % 8 == 0;
     if (a.epi.rows_gemv && !gemv_ok) return set_error(FF_ERR_UNSUPPORTED, "gemm: rows_gemv needs K <= 8192 and a plain store");
     if (gemv_ok && (a.epi.rows_gemv || a.M <= kGemvMaxRows)) return launch_gemv_rows(a, stream);

@@ -101,11 +101,16 @@ int gemm_bf16(const void* A, int64_t lda, const void* B, int64_t ldb, int M, int
 
 // One or two independent GEMMs in a single persistent launch (tiles of the
 // first problem, then of the second).
+// D[M, N] = op(A) op(B) with A stored [M, K] (a_mn = 0, K contiguous) or
+// [K, M] (a_mn = 1, M contiguous), and B stored [N, K] (b_mn = 0: D = A B^T,
+// the nn.Linear product) or [K, N] (b_mn = 1: D = A B).  Leading dimensions
+// are those of the stored layouts.
 struct GemmArgs {
     const void* A; int64_t lda;
     const void* B; int64_t ldb;
     int M, N, K;
     GemmEpilogue epi;
+    int a_mn = 0, b_mn = 0;
 };
 int gemm_bf16_group(const GemmArgs* problems, int n, cudaStream_t stream);
 

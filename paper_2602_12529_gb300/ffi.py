@@ -21,6 +21,7 @@ FF_ACT_NONE, FF_ACT_GELU, FF_ACT_SILU = 0, 1, 2
 FF_TSAMPLE_UNIFORM, FF_TSAMPLE_LOGIT_NORMAL, FF_TSAMPLE_DISCRETE = 0, 1, 2
 FF_AWM_SUM, FF_AWM_MEAN = 0, 1
 FF_AGG_WEIGHTED_SUM, FF_AGG_PER_REWARD = 0, 1
+FF_A_MK, FF_A_KM, FF_B_NK, FF_B_KN = 0, 1, 0, 1
 
 
 class FFError(RuntimeError):
@@ -77,6 +78,7 @@ _SIGS = {
     "ff_dit_workspace_size": ([_P, _I, C.POINTER(_SZ)], _I),
     "ff_dit_velocity": ([_P, _I, _P, _P, _P, _P, _P, _SZ, _P], _I),
     "ff_rollout_workspace_size": ([_P, _I, _I, C.POINTER(_SZ)], _I),
+    "ff_gemm": ([_I, _I, _I, _P, _I64, _I, _P, _I64, _I, _P, _I, _I, _P, _I64, _P], _I),
     "ff_rollout": ([_P, _I, _I, _P, _P, _P, _P, _P, _P, _P, _I, _P, _SZ, _P], _I),
     "ff_debug_gemm": ([_I, _I, _I, _P, _I64, _P, _I64, _P, _I, _I, _P, _I64, _P], _I),
     "ff_debug_gemm_gated": ([_I, _I, _I, _P, _I64, _P, _I64, _P, _P, _I64, _P, _I64, _I, _P], _I),
@@ -126,6 +128,18 @@ def _stream(stream) -> int:
     import torch
     s = torch.cuda.current_stream() if stream is None else stream
     return s.cuda_stream
+
+
+def _ptr_rows(t) -> int | None:
+    """Device address of a CUDA matrix whose rows are contiguous (any row
+    pitch, passed on as the leading dimension)."""
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("expected a CUDA tensor")
+    if t.dim() != 2 or t.stride(1) != 1:
+        raise ValueError("expected a 2-D tensor with contiguous rows")
+    return t.data_ptr()
 
 
 def _check(t, dtype, name):
@@ -405,6 +419,16 @@ def ff_debug_gemm(A, B, bias, out, act=FF_ACT_NONE, stream=None):
     import torch
     _call("ff_debug_gemm", M, N, K, _ptr(A), A.stride(0), _ptr(B), B.stride(0), _ptr(bias), act,
           1 if out.dtype == torch.float32 else 0, _ptr(out), out.stride(0), _stream(stream))
+
+
+def ff_gemm(A, a_layout: int, B, b_layout: int, out, bias=None, act=FF_ACT_NONE, stream=None):
+    """out[M, N] = act(op(A) op(B) + bias) with the stored layouts of include/ff.h."""
+    import torch
+    M = A.shape[0] if a_layout == FF_A_MK else A.shape[1]
+    K = A.shape[1] if a_layout == FF_A_MK else A.shape[0]
+    N = B.shape[0] if b_layout == FF_B_NK else B.shape[1]
+    _call("ff_gemm", M, N, K, _ptr_rows(A), A.stride(0), a_layout, _ptr_rows(B), B.stride(0), b_layout, _ptr(bias),
+          act, 1 if out.dtype == torch.float32 else 0, _ptr_rows(out), out.stride(0), _stream(stream))
 
 
 def ff_debug_gemm_gated(A, B, bias, resid, gate, rows_per_sample, stream=None):
