@@ -175,6 +175,41 @@ def attention(q, k, v, q_chunk: int = 2048):
     return out
 
 
+def attention_lse(q, k) -> np.ndarray:
+    """Per-row log-sum-exp of the scaled scores, natural log: [Nq, h]."""
+    nq, nh, d = q.shape
+    inv = 1.0 / math.sqrt(d)
+    out = np.empty((nq, nh))
+    for hh in range(nh):
+        s = (q[:, hh, :] @ k[:, hh, :].T) * inv
+        m = s.max(axis=1, keepdims=True)
+        out[:, hh] = (m + np.log(np.exp(s - m).sum(axis=1, keepdims=True)))[:, 0]
+    return out
+
+
+def attention_backward(q, k, v, dout):
+    """Gradients of sum(dout * attention(q, k, v)) w.r.t. q, k and v, written
+    out from the definitions: with P = softmax(S), S = q k^T / sqrt(d),
+      dV = P^T dO,  dP = dO V^T,  dS = P (dP - rowsum(dP P)),
+      dQ = dS K / sqrt(d),  dK = dS^T Q / sqrt(d).
+    q, dout [Nq, h, d]; k, v [Nk, h, d]."""
+    nq, nh, d = q.shape
+    inv = 1.0 / math.sqrt(d)
+    dq, dk, dv = np.zeros_like(q, dtype=np.float64), np.zeros_like(k, dtype=np.float64), np.zeros_like(v, dtype=np.float64)
+    for hh in range(nh):
+        qh, kh, vh, gh = q[:, hh, :], k[:, hh, :], v[:, hh, :], dout[:, hh, :]
+        s = (qh @ kh.T) * inv
+        s = s - s.max(axis=1, keepdims=True)
+        p = np.exp(s)
+        p = p / p.sum(axis=1, keepdims=True)
+        dv[:, hh, :] = p.T @ gh
+        dp = gh @ vh.T
+        ds = p * (dp - (dp * p).sum(axis=1, keepdims=True))
+        dq[:, hh, :] = (ds @ kh) * inv
+        dk[:, hh, :] = (ds.T @ qh) * inv
+    return dq, dk, dv
+
+
 # ---------------------------------------------------------------------------
 # Blocks (one sample at a time: x_* are [N_*, H], mods is [mod_width])
 # ---------------------------------------------------------------------------

@@ -250,3 +250,36 @@ def test_wan_param_count():
     H, F = 5120, 13824
     per_block = 8 * H * H + 2 * H * F
     assert 40 * per_block < n < 40 * per_block * 1.02
+
+
+def test_attention_backward_central_differences():
+    """The attention backward against central differences of the scalar
+    sum(dO * attention(q, k, v)); rowsum(dP P) = rowsum(dO O) is the D of
+    the backward."""
+    rng = np.random.default_rng(21)
+    nq, nk, nh, d = 3, 4, 2, 4
+    q, k, v, g = (rng.standard_normal((nq, nh, d)), rng.standard_normal((nk, nh, d)),
+                  rng.standard_normal((nk, nh, d)), rng.standard_normal((nq, nh, d)))
+    dq, dk, dv = dit.attention_backward(q, k, v, g)
+    loss = lambda q_, k_, v_: float(np.sum(g * dit.attention(q_, k_, v_)))
+    h = 1e-6
+    for arr, grad in ((q, dq), (k, dk), (v, dv)):
+        it = np.nditer(arr, flags=["multi_index"])
+        for _ in it:
+            i = it.multi_index
+            p_, m_ = arr.copy(), arr.copy()
+            p_[i] += h
+            m_[i] -= h
+            pick = lambda a_: [a_ if arr is x else x for x in (q, k, v)]
+            fd = (loss(*pick(p_)) - loss(*pick(m_))) / (2 * h)
+            assert grad[i] == pytest.approx(fd, rel=1e-6, abs=1e-8)
+
+
+def test_attention_lse_matches_logsumexp():
+    from scipy.special import logsumexp
+    rng = np.random.default_rng(22)
+    q, k = rng.standard_normal((5, 2, 8)) * 3, rng.standard_normal((7, 2, 8)) * 3
+    got = dit.attention_lse(q, k)
+    for hh in range(2):
+        want = logsumexp(q[:, hh, :] @ k[:, hh, :].T / math.sqrt(8), axis=1)
+        np.testing.assert_allclose(got[:, hh], want, rtol=1e-13)
