@@ -357,6 +357,33 @@ int ff_gemm(int M, int N, int K, const void* A, int64_t lda, int a_layout, const
             int64_t ldo, cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
+ * Joint attention of the velocity network with its backward (the training
+ * pass after the rollout, Sec. 3.1).  Per sample and head h, over the joint
+ * token sequence [segment 0; segment 1] (text; image):
+ *   O = softmax(Q K^T / sqrt(d)) V,   q, k, v of head h at columns h d,
+ *   H + h d, 2H + h d of the qkv buffers (H = heads * d), O at column h d.
+ * ff_attention_forward also writes lse (fp32, [B, heads, L]) with
+ * L = ff_attention_lse_rows(n0, n1) = pad128(n0) + pad128(n1): the base-2
+ * log-sum-exp of the scaled scores of segment-0 row r at r and of segment-1
+ * row r at pad128(n0) + r (padding rows are not written).
+ * ff_attention_backward (head_dim 128) takes O, its gradient dO (same
+ * layout and pitch ldo) and lse, and writes dq, dk, dv into dqkv buffers laid
+ * out like qkv (columns h d, H + h d, 2H + h d; pitch ldd; other columns are
+ * not touched).  ws: ff_attention_backward_workspace_size bytes (holds
+ * D = rowsum(dO * O)).  A segment with n = 0 may pass NULL buffers.
+ * ------------------------------------------------------------------------ */
+int ff_attention_lse_rows(int n0, int n1);
+int ff_attention_forward(int B, int heads, int head_dim, int n0, const void* qkv0, int64_t ld0,
+                         void* out0, int64_t ldo0, int n1, const void* qkv1, int64_t ld1,
+                         void* out1, int64_t ldo1, float* lse, cudaStream_t stream);
+int ff_attention_backward_workspace_size(int B, int heads, int n0, int n1, size_t* bytes);
+int ff_attention_backward(int B, int heads, int head_dim, int n0, const void* qkv0, int64_t ld0,
+                          const void* out0, const void* dout0, int64_t ldo0, void* dqkv0,
+                          int64_t ldd0, int n1, const void* qkv1, int64_t ld1, const void* out1,
+                          const void* dout1, int64_t ldo1, void* dqkv1, int64_t ldd1,
+                          const float* lse, void* ws, size_t ws_bytes, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
  * Trajectory sampling (paper Sec. 3.1: the SDE rollout that Flow-GRPO's
  * policy gradient scores, "repeated forward passes for trajectory
  * sampling").  S denoise steps; at step k = 0 .. S-1, for every sample:

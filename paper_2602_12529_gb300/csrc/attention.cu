@@ -68,43 +68,11 @@ struct AttnParams {
     float scale_log2;
     __nv_bfloat16* out[2];
     int64_t ldo[2];
+    float* lse;          // optional per-row log-sum-exp (base 2), see AttnSpec
+    int lse_rows;        // its row pitch per (sample, head)
+    int lse_base[2];     // first row of each query segment
 };
 
-__device__ __forceinline__ float ex2(float x) {
-    float y;
-    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-    return y;
-}
-
-__device__ __forceinline__ float max3(float a, float b, float c) {
-    float y;
-    asm("max.f32 %0, %1, %2, %3;" : "=f"(y) : "f"(a), "f"(b), "f"(c));
-    return y;
-}
-
-__device__ __forceinline__ void tmem_st_x32(uint32_t taddr, const uint32_t* r) {
-    asm volatile(
-        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
-        "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, "
-        "%17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr),
-        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]),
-        "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]), "r"(r[17]),
-        "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]),
-        "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
-        : "memory");
-}
-__device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
-
-// D[tmem] (+)= A[tmem] * B[smem]: the P V product with P held in TMEM.
-__device__ __forceinline__ void tc_mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
-                                               uint32_t accumulate) {
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}\n"
-        ::"r"(d_tmem), "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
-        : "memory");
-}
 // Barriers.  Per query tile the chain S -> softmax -> P -> O += P V -> next S
 // is strictly ordered, so no waiter can lag two phases behind a parity wait.
 constexpr int kMaxSlots = 8;
@@ -351,12 +319,15 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
             __syncwarp();
             if (lane == 0) mbar_arrive(&bar.p_full[t]);
         }
-        // ---- epilogue: O / l -> bf16, after the last O += P V
+        // ---- epilogue: O / l -> bf16, after the last O += P V, and the
+        // row's log-sum-exp m + log2(l) (base 2) when it is asked for
         if (ok && ntiles > 0 && mbar_wait(&bar.o_last[t], 0)) {
             tc_fence_after();
             const float inv = 1.f / l;
             const int row = q0 + t * kBM + r;
             const bool live = row < p.nq[seg];
+            if (p.lse && live)
+                p.lse[(static_cast<int64_t>(b) * gridDim.y + h) * p.lse_rows + p.lse_base[seg] + row] = m_used + log2f(l);
             __nv_bfloat16* dst = p.out[seg] + (static_cast<int64_t>(b) * p.nq[seg] + row) * p.ldo[seg] + h * HD;
 #pragma unroll 1
             for (int c = 0; c < HD; c += 32) {
@@ -415,6 +386,10 @@ int launch_attn(const AttnSpec& a, cudaStream_t stream) {
         p.ldo[i] = a.q[i].ldo;
     }
     p.qpairs0 = (a.q[0].n + 2 * kBM - 1) / (2 * kBM);
+    p.lse = a.lse;
+    p.lse_rows = attn_lse_rows(a.q[0].n, a.q[1].n);
+    p.lse_base[0] = 0;
+    p.lse_base[1] = attn_pad128(a.q[0].n);
     p.q_col = a.q_col;
     p.k_col = a.k_col;
     p.v_col = a.v_col;

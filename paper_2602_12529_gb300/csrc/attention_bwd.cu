@@ -1,0 +1,558 @@
+// attention_bwd.cu -- backward of the joint attention O = softmax(Q K^T / sqrt(d)) V
+// (d = 128) on tcgen05, for the training pass that follows the rollout
+// (paper Sec. 3.1: the policy gradient through the velocity network).
+//
+// With P = softmax(S), S = Q K^T a (a = 1/sqrt(d)) per (sample, head) and the
+// forward's per-row log-sum-exp (base 2, lse2 = log2 sum_j 2^(S_ij log2 e)):
+//   P_ij = 2^(S_ij log2(e) - lse2_i),  D_i = sum_c dO_ic O_ic,
+//   dP = dO V^T,  dS = P (dP - D),  dV = P^T dO,  dQ = a dS K,  dK = a dS^T Q.
+// Three kernels:
+//   delta   D_i, one warp per (row, head), into the workspace (lse layout);
+//   dq      one 128-row query tile per CTA, K/V tiles streamed: S = Q K_j^T
+//           and dP = dO V_j^T in TMEM, dS written over S as bf16, then
+//           dQ += dS K_j with dS read from TMEM and K_j taken as an MN-major
+//           operand (the same shared-memory tile feeds S as K-major);
+//   dkdv    one 128-key tile per CTA, query tiles streamed: S^T = K Q_i^T and
+//           dP^T = V dO_i^T in TMEM, P^T and dS^T written over them, then
+//           dV += P^T dO_i and dK += dS^T Q_i (Q_i, dO_i as MN-major
+//           operands); lse and D of the query tile arrive by bulk copies with
+//           the tiles.
+// Query (key) rows past a segment's end read neighbouring or zero-filled
+// rows; their columns are selected to zero (never multiplied, so padding
+// can hold anything) and their rows are not stored.  Every wait is bounded;
+// on a timeout a kernel records the status word, drains its tensor-core
+// work, frees TMEM and returns.
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace ff {
+namespace {
+
+constexpr int HD = 128;
+constexpr int kT = 128;                        // rows of a query / key tile
+constexpr int kTileBytes = kT * HD * 2;         // 32 KB: one bf16 tile (two 64-column boxes)
+constexpr int kSlots = 4;                       // streamed tiles in flight
+constexpr int kThreads = 192;                   // producer, MMA, 4 elementwise warps
+constexpr int kBarBytes = 256;
+
+struct BwdParams {
+    int n[2];              // tokens per sample of each segment (queries = keys)
+    int tiles0;            // 128-row tiles of segment 0 (segment 1's follow)
+    int H;                 // heads * d
+    float scale_log2;      // log2(e) / sqrt(d)
+    float scale;           // 1 / sqrt(d)
+    const float* lse;      // [B, heads, lse_rows] base-2 log-sum-exp of the forward
+    const float* delta;    // D in the same layout
+    int lse_rows, lse_base[2];
+    __nv_bfloat16* dqkv[2];
+    int64_t ldd[2];
+};
+
+struct Bars {
+    uint64_t fixed_full;           // the CTA's own tiles landed
+    uint64_t slot_full[kSlots];
+    uint64_t slot_empty[kSlots];
+    uint64_t s_full;               // MMA -> elementwise: S (S^T) and dP (dP^T) in TMEM
+    uint64_t p_full;               // elementwise -> MMA: dS (P^T, dS^T) in TMEM
+    uint64_t done;                 // MMA -> elementwise: the accumulators are final
+    uint64_t drain;
+    uint32_t tmem_slot;
+    int abort_flag;
+};
+
+__device__ __forceinline__ void bulk_load_1d(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                 ::"r"(smem_u32(dst)), "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar))
+                 : "memory");
+}
+
+// Stores a 128-column fp32 TMEM row of this thread as bf16 (times mul).
+__device__ __forceinline__ void store_row_bf16(uint32_t taddr, float mul, __nv_bfloat16* dst, bool live) {
+#pragma unroll 1
+    for (int c = 0; c < HD; c += 32) {
+        uint32_t o[32];
+        tmem_ld_x32(taddr + c, o);
+        tmem_ld_wait();
+        if (live) {
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const float* f = reinterpret_cast<const float*>(o) + 8 * k;
+                *reinterpret_cast<uint4*>(dst + c + 8 * k) =
+                    make_uint4(pack_bf16x2(f[0] * mul, f[1] * mul), pack_bf16x2(f[2] * mul, f[3] * mul),
+                               pack_bf16x2(f[4] * mul, f[5] * mul), pack_bf16x2(f[6] * mul, f[7] * mul));
+            }
+        }
+    }
+}
+
+// D_i = sum_c dO_ic O_ic: one warp per (token row, head), 4 columns per lane.
+__global__ void __launch_bounds__(256) attn_bwd_delta_kernel(int B, int heads, int n0, int n1,
+                                                             const __nv_bfloat16* o0, const __nv_bfloat16* do0,
+                                                             const __nv_bfloat16* o1, const __nv_bfloat16* do1,
+                                                             int64_t ldo0, int64_t ldo1, int lse_rows, int base1,
+                                                             float* delta) {
+    const int64_t w = (static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    const int64_t rows0 = static_cast<int64_t>(B) * n0;
+    const int64_t total = (rows0 + static_cast<int64_t>(B) * n1) * heads;
+    if (w >= total) return;
+    const int h = static_cast<int>(w % heads);
+    const int64_t r = w / heads;                    // token row over both segments
+    const bool s1 = r >= rows0;
+    const int64_t rr = s1 ? r - rows0 : r;
+    const int n = s1 ? n1 : n0;
+    const int b = static_cast<int>(rr / n);
+    const int row = static_cast<int>(rr - static_cast<int64_t>(b) * n);
+    const int64_t ld = s1 ? ldo1 : ldo0;
+    const __nv_bfloat16* o = (s1 ? o1 : o0) + rr * ld + h * HD + lane * 4;
+    const __nv_bfloat16* g = (s1 ? do1 : do0) + rr * ld + h * HD + lane * 4;
+    const uint2 ov = *reinterpret_cast<const uint2*>(o);
+    const uint2 gv = *reinterpret_cast<const uint2*>(g);
+    const float2 o01 = unpack_bf16x2(ov.x), o23 = unpack_bf16x2(ov.y);
+    const float2 g01 = unpack_bf16x2(gv.x), g23 = unpack_bf16x2(gv.y);
+    float s = o01.x * g01.x + o01.y * g01.y + o23.x * g23.x + o23.y * g23.y;
+#pragma unroll
+    for (int k = 16; k; k >>= 1) s += __shfl_xor_sync(0xffffffffu, s, k);
+    if (lane == 0) delta[(static_cast<int64_t>(b) * heads + h) * lse_rows + (s1 ? base1 : 0) + row] = s;
+}
+
+// ------------------------------------------------------------------ dQ
+// TMEM: S at 0, dP at 128, dQ at 256 (dS as bf16 pairs over S's first 64).
+// Shared memory: Q tile, dO tile, then a ring of K_j / V_j tiles.
+__global__ void __launch_bounds__(kThreads, 1)
+attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_constant__ CUtensorMap tm_qkv1,
+                   const __grid_constant__ CUtensorMap tm_do0, const __grid_constant__ CUtensorMap tm_do1,
+                   const BwdParams p, int* status) {
+    extern __shared__ __align__(1024) uint8_t smem[];
+    uint8_t* sQ = smem;
+    uint8_t* sdO = smem + kTileBytes;
+    uint8_t* sKV = smem + 2 * kTileBytes;                     // [kSlots][tile]
+    Bars& bar = *reinterpret_cast<Bars*>(sKV + kSlots * kTileBytes);
+    volatile int* abort_flag = &bar.abort_flag;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int b = blockIdx.z, h = blockIdx.y;
+    const int seg = blockIdx.x < p.tiles0 ? 0 : 1;
+    const int q0 = (blockIdx.x - (seg ? p.tiles0 : 0)) * kT;
+    const int nt0 = (p.n[0] + kT - 1) / kT;
+    const int ntiles = nt0 + (p.n[1] + kT - 1) / kT;
+    if (threadIdx.x == 0) {
+        *abort_flag = 0;
+        if (smem_u32(smem) & 1023u) {
+            report_status(status, kStatusBadArgument);
+            *abort_flag = 1;
+        }
+        mbar_init(&bar.fixed_full, 1);
+        for (int s = 0; s < kSlots; ++s) {
+            mbar_init(&bar.slot_full[s], 1);
+            mbar_init(&bar.slot_empty[s], 1);
+        }
+        mbar_init(&bar.s_full, 1);
+        mbar_init(&bar.p_full, 4);
+        mbar_init(&bar.done, 1);
+        mbar_init(&bar.drain, 1);
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(&bar.tmem_slot, 512);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = bar.tmem_slot;
+    auto fail = [&]() {
+        report_status(status, kStatusWaitTimeout);
+        *abort_flag = 1;
+    };
+    if (*abort_flag) {
+    } else if (warp == 0 && lane == 0) {
+        // ---- producer: Q and dO of this tile, then K_0, V_0, K_1, ...
+        const CUtensorMap* tq = seg ? &tm_qkv1 : &tm_qkv0;
+        const CUtensorMap* td = seg ? &tm_do1 : &tm_do0;
+        mbar_arrive_expect_tx(&bar.fixed_full, 2 * kTileBytes);
+        for (int c = 0; c < 2; ++c) {
+            tma_load_2d(sQ + c * (kT * 128), tq, &bar.fixed_full, h * HD + c * 64, b * p.n[seg] + q0);
+            tma_load_2d(sdO + c * (kT * 128), td, &bar.fixed_full, h * HD + c * 64, b * p.n[seg] + q0);
+        }
+        for (int n = 0; n < 2 * ntiles; ++n) {
+            const int s = n % kSlots;
+            if (!mbar_wait(&bar.slot_empty[s], ((n / kSlots) & 1) ^ 1)) { fail(); break; }
+            const int j = n >> 1;
+            const int ks = j < nt0 ? 0 : 1;
+            const int row = b * p.n[ks] + (j - (ks ? nt0 : 0)) * kT;
+            const int col = ((n & 1) ? 2 * p.H : p.H) + h * HD;
+            uint8_t* dst = sKV + s * kTileBytes;
+            mbar_arrive_expect_tx(&bar.slot_full[s], kTileBytes);
+            for (int c = 0; c < 2; ++c)
+                tma_load_2d(dst + c * (kT * 128), ks ? &tm_qkv1 : &tm_qkv0, &bar.slot_full[s], col + c * 64, row);
+        }
+    } else if (warp == 1 && lane == 0) {
+        // ---- MMA issuer
+        constexpr uint32_t idesc_s = idesc_bf16_f32(kT, kT);
+        constexpr uint32_t idesc_q = idesc_bf16_f32(kT, HD) | (1u << 16);   // B = K_j, MN-major
+        bool ok = mbar_wait(&bar.fixed_full, 0);
+        if (!ok) fail();
+        const uint64_t dq_ = smem_desc_k_sw128(smem_u32(sQ));
+        const uint64_t ddo = smem_desc_k_sw128(smem_u32(sdO));
+        for (int j = 0; ok && j < ntiles; ++j) {
+            const int nk = 2 * j, nv = 2 * j + 1;
+            if (!mbar_wait(&bar.slot_full[nk % kSlots], (nk / kSlots) & 1) ||
+                !mbar_wait(&bar.slot_full[nv % kSlots], (nv / kSlots) & 1)) { fail(); ok = false; break; }
+            tc_fence_after();
+            const uint32_t aK = smem_u32(sKV + (nk % kSlots) * kTileBytes);
+            const uint32_t aV = smem_u32(sKV + (nv % kSlots) * kTileBytes);
+            const uint64_t dk = smem_desc_k_sw128(aK), dv = smem_desc_k_sw128(aV);
+#pragma unroll
+            for (int k = 0; k < HD / 16; ++k) {
+                const uint32_t off = ((k / 4) * (kT * 128) + (k % 4) * 32) >> 4;
+                tc_mma_bf16(tmem, dq_ + off, dk + off, idesc_s, k != 0 ? 1u : 0u);           // S = Q K^T
+                tc_mma_bf16(tmem + kT, ddo + off, dv + off, idesc_s, k != 0 ? 1u : 0u);      // dP = dO V^T
+            }
+            tc_commit(&bar.s_full);
+            if (!mbar_wait(&bar.p_full, j & 1)) { fail(); ok = false; break; }
+            tc_fence_after();
+            // dQ += dS K_j: dS from TMEM, K_j as [keys (K) x d (N)], MN-major
+            const uint64_t dkm = smem_desc_mn_sw128(aK, kT * 128);
+#pragma unroll
+            for (int k = 0; k < kT / 16; ++k)
+                tc_mma_bf16_ts(tmem + 2 * kT, tmem + k * 8, dkm + static_cast<uint64_t>(k * (2048 >> 4)), idesc_q,
+                               (j | k) != 0 ? 1u : 0u);
+            tc_commit(&bar.slot_empty[nk % kSlots]);
+            tc_commit(&bar.slot_empty[nv % kSlots]);
+        }
+        if (ok) tc_commit(&bar.done);
+        tc_commit(&bar.drain);
+        if (!mbar_wait(&bar.drain, 0)) report_status(status, kStatusWaitTimeout);
+    } else if (warp >= 2) {
+        // ---- elementwise: thread = query row = TMEM lane
+        const int q = warp & 3;
+        const int r = q * 32 + lane;
+        const int row = q0 + r;
+        const uint32_t tS = tmem + (static_cast<uint32_t>(q * 32) << 16);
+        const int64_t li = (static_cast<int64_t>(b) * gridDim.y + h) * p.lse_rows + p.lse_base[seg] + row;
+        const bool live = row < p.n[seg];
+        const float lse = live ? p.lse[li] : 0.f;
+        const float dd = live ? p.delta[li] : 0.f;
+        bool ok = true;
+        for (int j = 0; j < ntiles; ++j) {
+            if (!mbar_wait(&bar.s_full, j & 1)) { fail(); ok = false; break; }
+            tc_fence_after();
+            uint32_t sr[kT], pr_[kT];
+#pragma unroll
+            for (int c = 0; c < kT; c += 32) {
+                tmem_ld_x32(tS + c, *reinterpret_cast<uint32_t(*)[32]>(&sr[c]));
+                tmem_ld_x32(tS + kT + c, *reinterpret_cast<uint32_t(*)[32]>(&pr_[c]));
+            }
+            tmem_ld_wait();
+            const int ks = j < nt0 ? 0 : 1;
+            const int valid = p.n[ks] - (j - (ks ? nt0 : 0)) * kT;   // key columns < valid are real
+#pragma unroll
+            for (int i = 0; i < kT; i += 2) {
+                float ds[2];
+#pragma unroll
+                for (int u = 0; u < 2; ++u) {
+                    const float pv = ex2(fmaf(__uint_as_float(sr[i + u]), p.scale_log2, -lse));
+                    ds[u] = (i + u < valid && live) ? pv * (__uint_as_float(pr_[i + u]) - dd) : 0.f;
+                }
+                sr[i / 2] = pack_bf16x2(ds[0], ds[1]);
+            }
+#pragma unroll
+            for (int c = 0; c < kT / 2; c += 32) tmem_st_x32(tS + c, &sr[c]);
+            tmem_st_wait();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&bar.p_full);
+        }
+        if (ok && mbar_wait(&bar.done, 0)) {
+            tc_fence_after();
+            store_row_bf16(tS + 2 * kT, p.scale,
+                           p.dqkv[seg] + (static_cast<int64_t>(b) * p.n[seg] + row) * p.ldd[seg] + h * HD, live);
+        } else if (ok) {
+            fail();
+        }
+    }
+    if (*abort_flag) {
+        const uint64_t t0 = global_timer_ns();
+        while (global_timer_ns() - t0 < 50000ull) {
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 512);
+    }
+}
+
+// ------------------------------------------------------------------ dK, dV
+// TMEM: S^T at 0, dP^T at 128, dV at 256, dK at 384 (P^T and dS^T as bf16
+// pairs over the first 64 columns of S^T and dP^T).  Shared memory: the K
+// and V tiles of this CTA, then a ring of Q_i / dO_i tiles, then lse / D of
+// each streamed query tile.
+__global__ void __launch_bounds__(kThreads, 1)
+attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_constant__ CUtensorMap tm_qkv1,
+                     const __grid_constant__ CUtensorMap tm_do0, const __grid_constant__ CUtensorMap tm_do1,
+                     const BwdParams p, int* status) {
+    extern __shared__ __align__(1024) uint8_t smem[];
+    uint8_t* sK = smem;
+    uint8_t* sV = smem + kTileBytes;
+    uint8_t* sQD = smem + 2 * kTileBytes;                     // [kSlots][tile]: Q_i, dO_i, Q_i+1, ...
+    float* sLD = reinterpret_cast<float*>(sQD + kSlots * kTileBytes);   // [kSlots / 2][2][kT]: lse, D
+    Bars& bar = *reinterpret_cast<Bars*>(reinterpret_cast<uint8_t*>(sLD) + (kSlots / 2) * 2 * kT * 4);
+    volatile int* abort_flag = &bar.abort_flag;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int b = blockIdx.z, h = blockIdx.y;
+    const int seg = blockIdx.x < p.tiles0 ? 0 : 1;
+    const int k0 = (blockIdx.x - (seg ? p.tiles0 : 0)) * kT;
+    const int nt0 = (p.n[0] + kT - 1) / kT;
+    const int ntiles = nt0 + (p.n[1] + kT - 1) / kT;
+    const int64_t lrow = (static_cast<int64_t>(b) * gridDim.y + h) * p.lse_rows;
+    if (threadIdx.x == 0) {
+        *abort_flag = 0;
+        if (smem_u32(smem) & 1023u) {
+            report_status(status, kStatusBadArgument);
+            *abort_flag = 1;
+        }
+        mbar_init(&bar.fixed_full, 1);
+        for (int s = 0; s < kSlots; ++s) {
+            mbar_init(&bar.slot_full[s], 1);
+            mbar_init(&bar.slot_empty[s], 1);
+        }
+        mbar_init(&bar.s_full, 1);
+        mbar_init(&bar.p_full, 4);
+        mbar_init(&bar.done, 1);
+        mbar_init(&bar.drain, 1);
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(&bar.tmem_slot, 512);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = bar.tmem_slot;
+    auto fail = [&]() {
+        report_status(status, kStatusWaitTimeout);
+        *abort_flag = 1;
+    };
+    if (*abort_flag) {
+    } else if (warp == 0 && lane == 0) {
+        // ---- producer: K and V of this tile, then per query tile i its Q_i
+        // and dO_i (one slot each) with lse_i / D_i riding on dO_i's barrier
+        const CUtensorMap* tk = seg ? &tm_qkv1 : &tm_qkv0;
+        mbar_arrive_expect_tx(&bar.fixed_full, 2 * kTileBytes);
+        for (int c = 0; c < 2; ++c) {
+            tma_load_2d(sK + c * (kT * 128), tk, &bar.fixed_full, p.H + h * HD + c * 64, b * p.n[seg] + k0);
+            tma_load_2d(sV + c * (kT * 128), tk, &bar.fixed_full, 2 * p.H + h * HD + c * 64, b * p.n[seg] + k0);
+        }
+        for (int n = 0; n < 2 * ntiles; ++n) {
+            const int s = n % kSlots;
+            if (!mbar_wait(&bar.slot_empty[s], ((n / kSlots) & 1) ^ 1)) { fail(); break; }
+            const int i = n >> 1;
+            const int qs = i < nt0 ? 0 : 1;
+            const int qi = (i - (qs ? nt0 : 0)) * kT;
+            const int row = b * p.n[qs] + qi;
+            uint8_t* dst = sQD + s * kTileBytes;
+            if (n & 1) {
+                float* ld = sLD + (s >> 1) * 2 * kT;
+                mbar_arrive_expect_tx(&bar.slot_full[s], kTileBytes + 2 * kT * 4);
+                for (int c = 0; c < 2; ++c)
+                    tma_load_2d(dst + c * (kT * 128), qs ? &tm_do1 : &tm_do0, &bar.slot_full[s], h * HD + c * 64, row);
+                bulk_load_1d(ld, p.lse + lrow + p.lse_base[qs] + qi, kT * 4, &bar.slot_full[s]);
+                bulk_load_1d(ld + kT, p.delta + lrow + p.lse_base[qs] + qi, kT * 4, &bar.slot_full[s]);
+            } else {
+                mbar_arrive_expect_tx(&bar.slot_full[s], kTileBytes);
+                for (int c = 0; c < 2; ++c)
+                    tma_load_2d(dst + c * (kT * 128), qs ? &tm_qkv1 : &tm_qkv0, &bar.slot_full[s], h * HD + c * 64,
+                                row);
+            }
+        }
+    } else if (warp == 1 && lane == 0) {
+        // ---- MMA issuer
+        constexpr uint32_t idesc_s = idesc_bf16_f32(kT, kT);
+        constexpr uint32_t idesc_g = idesc_bf16_f32(kT, HD) | (1u << 16);   // B = Q_i / dO_i, MN-major
+        bool ok = mbar_wait(&bar.fixed_full, 0);
+        if (!ok) fail();
+        const uint64_t dk_ = smem_desc_k_sw128(smem_u32(sK));
+        const uint64_t dv_ = smem_desc_k_sw128(smem_u32(sV));
+        for (int i = 0; ok && i < ntiles; ++i) {
+            const int nq = 2 * i, nd = 2 * i + 1;
+            if (!mbar_wait(&bar.slot_full[nq % kSlots], (nq / kSlots) & 1) ||
+                !mbar_wait(&bar.slot_full[nd % kSlots], (nd / kSlots) & 1)) { fail(); ok = false; break; }
+            tc_fence_after();
+            const uint32_t aQ = smem_u32(sQD + (nq % kSlots) * kTileBytes);
+            const uint32_t aD = smem_u32(sQD + (nd % kSlots) * kTileBytes);
+            const uint64_t dq_ = smem_desc_k_sw128(aQ), ddo = smem_desc_k_sw128(aD);
+#pragma unroll
+            for (int k = 0; k < HD / 16; ++k) {
+                const uint32_t off = ((k / 4) * (kT * 128) + (k % 4) * 32) >> 4;
+                tc_mma_bf16(tmem, dk_ + off, dq_ + off, idesc_s, k != 0 ? 1u : 0u);        // S^T = K Q^T
+                tc_mma_bf16(tmem + kT, dv_ + off, ddo + off, idesc_s, k != 0 ? 1u : 0u);   // dP^T = V dO^T
+            }
+            tc_commit(&bar.s_full);
+            if (!mbar_wait(&bar.p_full, i & 1)) { fail(); ok = false; break; }
+            tc_fence_after();
+            const uint64_t ddom = smem_desc_mn_sw128(aD, kT * 128), dqm = smem_desc_mn_sw128(aQ, kT * 128);
+#pragma unroll
+            for (int k = 0; k < kT / 16; ++k) {
+                const uint64_t step = static_cast<uint64_t>(k * (2048 >> 4));
+                tc_mma_bf16_ts(tmem + 2 * kT, tmem + k * 8, ddom + step, idesc_g, (i | k) != 0 ? 1u : 0u);  // dV += P^T dO
+                tc_mma_bf16_ts(tmem + 3 * kT, tmem + kT + k * 8, dqm + step, idesc_g, (i | k) != 0 ? 1u : 0u);  // dK += dS^T Q
+            }
+            tc_commit(&bar.slot_empty[nq % kSlots]);
+            tc_commit(&bar.slot_empty[nd % kSlots]);
+        }
+        if (ok) tc_commit(&bar.done);
+        tc_commit(&bar.drain);
+        if (!mbar_wait(&bar.drain, 0)) report_status(status, kStatusWaitTimeout);
+    } else if (warp >= 2) {
+        // ---- elementwise: thread = key row = TMEM lane
+        const int q = warp & 3;
+        const int r = q * 32 + lane;
+        const int row = k0 + r;
+        const uint32_t tS = tmem + (static_cast<uint32_t>(q * 32) << 16);
+        const bool live = row < p.n[seg];
+        bool ok = true;
+        for (int i = 0; i < ntiles; ++i) {
+            if (!mbar_wait(&bar.s_full, i & 1)) { fail(); ok = false; break; }
+            tc_fence_after();
+            const int nd = 2 * i + 1;
+            const float* lse = sLD + ((nd % kSlots) >> 1) * 2 * kT;
+            const float* dl = lse + kT;
+            const int qs = i < nt0 ? 0 : 1;
+            const int valid = p.n[qs] - (i - (qs ? nt0 : 0)) * kT;   // query columns < valid are real
+            // two halves of 64 query columns; a half's bf16 P^T / dS^T land on
+            // columns whose fp32 values this thread has already read
+#pragma unroll 1
+            for (int hf = 0; hf < 2; ++hf) {
+                uint32_t sr[kT / 2], pr_[kT / 2];
+#pragma unroll
+                for (int c = 0; c < kT / 2; c += 32) {
+                    tmem_ld_x32(tS + hf * (kT / 2) + c, *reinterpret_cast<uint32_t(*)[32]>(&sr[c]));
+                    tmem_ld_x32(tS + kT + hf * (kT / 2) + c, *reinterpret_cast<uint32_t(*)[32]>(&pr_[c]));
+                }
+                tmem_ld_wait();
+#pragma unroll
+                for (int c = 0; c < kT / 2; c += 2) {
+                    float pv[2], ds[2];
+#pragma unroll
+                    for (int u = 0; u < 2; ++u) {
+                        const int col = hf * (kT / 2) + c + u;
+                        const bool real = col < valid;
+                        const float e = ex2(fmaf(__uint_as_float(sr[c + u]), p.scale_log2, -lse[col]));
+                        pv[u] = real ? e : 0.f;
+                        ds[u] = real ? e * (__uint_as_float(pr_[c + u]) - dl[col]) : 0.f;
+                    }
+                    sr[c / 2] = pack_bf16x2(pv[0], pv[1]);
+                    pr_[c / 2] = pack_bf16x2(ds[0], ds[1]);
+                }
+                tmem_st_x32(tS + hf * (kT / 4), sr);
+                tmem_st_x32(tS + kT + hf * (kT / 4), pr_);
+            }
+            tmem_st_wait();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&bar.p_full);
+        }
+        if (ok && mbar_wait(&bar.done, 0)) {
+            tc_fence_after();
+            __nv_bfloat16* dst = p.dqkv[seg] + (static_cast<int64_t>(b) * p.n[seg] + row) * p.ldd[seg];
+            store_row_bf16(tS + 2 * kT, 1.0f, dst + 2 * p.H + h * HD, live);      // dV
+            store_row_bf16(tS + 3 * kT, p.scale, dst + p.H + h * HD, live);       // dK
+        } else if (ok) {
+            fail();
+        }
+    }
+    if (*abort_flag) {
+        const uint64_t t0 = global_timer_ns();
+        while (global_timer_ns() - t0 < 50000ull) {
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 512);
+    }
+}
+
+constexpr int kSmemDq = 2 * kTileBytes + kSlots * kTileBytes + kBarBytes;
+constexpr int kSmemDkdv = 2 * kTileBytes + kSlots * kTileBytes + (kSlots / 2) * 2 * kT * 4 + kBarBytes;
+static_assert(sizeof(Bars) <= kBarBytes, "barrier block too small");
+
+}  // namespace
+
+size_t attention_backward_ws_bytes(int B, int heads, int n0, int n1) {
+    return static_cast<size_t>(B) * heads * attn_lse_rows(n0, n1) * sizeof(float);
+}
+
+int attention_backward(const AttnBwdSeg& s0, const AttnBwdSeg& s1, int B, int heads, int head_dim, const float* lse,
+                       void* ws, size_t ws_bytes, cudaStream_t stream) {
+    if (head_dim != HD) return set_error(FF_ERR_UNSUPPORTED, "attention backward: head_dim %d (128 only)", head_dim);
+    if (B <= 0 || heads <= 0 || B > 65535 || heads > 65535 || s0.n < 0 || s1.n < 0 || s0.n + s1.n <= 0)
+        return set_error(FF_ERR_INVALID_ARG, "attention backward: bad shape");
+    if (!lse || !ws) return set_error(FF_ERR_INVALID_ARG, "attention backward: null lse or workspace");
+    const AttnBwdSeg* sg[2] = {&s0, &s1};
+    const int H = heads * HD;
+    for (int i = 0; i < 2; ++i) {
+        const AttnBwdSeg& s = *sg[i];
+        if (!s.n) continue;
+        if (!s.qkv || !s.o || !s.dout || !s.dqkv || !aligned16(s.o) || !aligned16(s.dout) || !aligned16(s.dqkv) ||
+            s.ld % 8 || s.ldo % 8 || s.ldd % 8 || s.ld < 3 * H || s.ldo < H || s.ldd < 3 * H)
+            return set_error(FF_ERR_INVALID_ARG, "attention backward: bad segment %d", i);
+    }
+    const size_t need = attention_backward_ws_bytes(B, heads, s0.n, s1.n);
+    if (ws_bytes < need || !aligned16(ws))
+        return set_error(FF_ERR_WORKSPACE, "attention backward: workspace %zu B < %zu B", ws_bytes, need);
+    for (auto* f : {(const void*)attn_bwd_dq_kernel, (const void*)attn_bwd_dkdv_kernel}) {
+        const int bytes = f == (const void*)attn_bwd_dq_kernel ? kSmemDq : kSmemDkdv;
+        if (cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) != cudaSuccess)
+            return set_error(FF_ERR_CUDA, "attention backward: cannot set shared memory size");
+    }
+    CUtensorMap tqkv[2], tdo[2];
+    for (int i = 0; i < 2; ++i) {
+        const AttnBwdSeg& s = sg[i]->n > 0 ? *sg[i] : *sg[1 - i];   // an empty segment still needs a valid map
+        FF_TRY(make_tmap_bf16(&tqkv[i], s.qkv, static_cast<int64_t>(B) * s.n, 3 * H, s.ld, kT));
+        FF_TRY(make_tmap_bf16(&tdo[i], s.dout, static_cast<int64_t>(B) * s.n, H, s.ldo, kT));
+    }
+    float* delta = static_cast<float*>(ws);
+    const int rows = attn_lse_rows(s0.n, s1.n);
+    {
+        const int64_t warps = (static_cast<int64_t>(B) * (s0.n + s1.n)) * heads;
+        ProfScope prof(stream, "attn_bwd_delta", 0.0, 4.0 * warps * HD);
+        attn_bwd_delta_kernel<<<static_cast<unsigned>((warps + 7) / 8), 256, 0, stream>>>(
+            B, heads, s0.n, s1.n, s0.o, s0.dout, s1.o, s1.dout, s0.ldo, s1.ldo, rows, attn_pad128(s0.n), delta);
+        FF_TRY(check_launch("attn_bwd_delta_kernel"));
+    }
+    BwdParams p;
+    p.n[0] = s0.n;
+    p.n[1] = s1.n;
+    p.tiles0 = (s0.n + kT - 1) / kT;
+    p.H = H;
+    p.scale_log2 = static_cast<float>(1.4426950408889634 / sqrt(static_cast<double>(HD)));
+    p.scale = static_cast<float>(1.0 / sqrt(static_cast<double>(HD)));
+    p.lse = lse;
+    p.delta = delta;
+    p.lse_rows = rows;
+    p.lse_base[0] = 0;
+    p.lse_base[1] = attn_pad128(s0.n);
+    p.dqkv[0] = s0.dqkv;
+    p.dqkv[1] = s1.dqkv;
+    p.ldd[0] = s0.ldd;
+    p.ldd[1] = s1.ldd;
+    const dim3 grid(p.tiles0 + (s1.n + kT - 1) / kT, heads, B);
+    const double N = static_cast<double>(s0.n + s1.n);
+    {
+        ProfScope prof(stream, "attn_bwd_dq", 6.0 * B * heads * N * N * HD, 0.0);
+        attn_bwd_dq_kernel<<<grid, kThreads, kSmemDq, stream>>>(tqkv[0], tqkv[1], tdo[0], tdo[1], p,
+                                                                 device_status_ptr());
+        FF_TRY(check_launch("attn_bwd_dq_kernel"));
+    }
+    ProfScope prof(stream, "attn_bwd_dkdv", 8.0 * B * heads * N * N * HD, 0.0);
+    attn_bwd_dkdv_kernel<<<grid, kThreads, kSmemDkdv, stream>>>(tqkv[0], tqkv[1], tdo[0], tdo[1], p,
+                                                                 device_status_ptr());
+    return check_launch("attn_bwd_dkdv_kernel");
+}
+
+}  // namespace ff

@@ -36,6 +36,55 @@ int ff_gemm(int M, int N, int K, const void* A, int64_t lda, int a_layout, const
     return gemm_bf16_group(&g, 1, stream);
 }
 
+int ff_attention_lse_rows(int n0, int n1) { return ff::attn_lse_rows(n0 < 0 ? 0 : n0, n1 < 0 ? 0 : n1); }
+
+int ff_attention_forward(int B, int heads, int head_dim, int n0, const void* qkv0, int64_t ld0, void* out0,
+                         int64_t ldo0, int n1, const void* qkv1, int64_t ld1, void* out1, int64_t ldo1, float* lse,
+                         cudaStream_t stream) {
+    using namespace ff;
+    if (lse && !aligned16(lse)) return set_error(FF_ERR_INVALID_ARG, "attention: lse must be 16-byte aligned");
+    AttnSpec a;
+    const int H = heads * head_dim;
+    const void* qkv[2] = {qkv0, qkv1};
+    const int64_t ld[2] = {ld0, ld1}, ldo[2] = {ldo0, ldo1};
+    void* out[2] = {out0, out1};
+    const int n[2] = {n0, n1};
+    for (int i = 0; i < 2; ++i) {
+        a.q[i] = AttnQuerySeg{static_cast<const __nv_bfloat16*>(qkv[i]), ld[i], n[i],
+                              static_cast<__nv_bfloat16*>(out[i]), ldo[i]};
+        a.kv[i] = AttnKvSeg{static_cast<const __nv_bfloat16*>(qkv[i]), ld[i], n[i]};
+    }
+    a.q_col = 0;
+    a.k_col = H;
+    a.v_col = 2 * H;
+    a.B = B;
+    a.heads = heads;
+    a.head_dim = head_dim;
+    a.lse = lse;
+    return attention_general(a, stream);
+}
+
+int ff_attention_backward_workspace_size(int B, int heads, int n0, int n1, size_t* bytes) {
+    using namespace ff;
+    if (!bytes || B <= 0 || heads <= 0 || n0 < 0 || n1 < 0)
+        return set_error(FF_ERR_INVALID_ARG, "attention backward: bad workspace query");
+    *bytes = attention_backward_ws_bytes(B, heads, n0, n1);
+    return FF_OK;
+}
+
+int ff_attention_backward(int B, int heads, int head_dim, int n0, const void* qkv0, int64_t ld0, const void* out0,
+                          const void* dout0, int64_t ldo0, void* dqkv0, int64_t ldd0, int n1, const void* qkv1,
+                          int64_t ld1, const void* out1, const void* dout1, int64_t ldo1, void* dqkv1, int64_t ldd1,
+                          const float* lse, void* ws, size_t ws_bytes, cudaStream_t stream) {
+    using namespace ff;
+    if (lse && !aligned16(lse)) return set_error(FF_ERR_INVALID_ARG, "attention backward: lse must be 16-byte aligned");
+    AttnBwdSeg s0{static_cast<const __nv_bfloat16*>(qkv0), ld0, static_cast<const __nv_bfloat16*>(out0),
+                  static_cast<const __nv_bfloat16*>(dout0), ldo0, static_cast<__nv_bfloat16*>(dqkv0), ldd0, n0};
+    AttnBwdSeg s1{static_cast<const __nv_bfloat16*>(qkv1), ld1, static_cast<const __nv_bfloat16*>(out1),
+                  static_cast<const __nv_bfloat16*>(dout1), ldo1, static_cast<__nv_bfloat16*>(dqkv1), ldd1, n1};
+    return attention_backward(s0, s1, B, heads, head_dim, lse, ws, ws_bytes, stream);
+}
+
 int ff_debug_gemm_gated(int M, int N, int K, const void* A, int64_t lda, const void* B, int64_t ldb, const void* bias,
                         float* resid, int64_t ld_resid, const float* gate, int64_t ld_gate, int rows_per_sample,
                         cudaStream_t stream) {

@@ -168,8 +168,30 @@ struct AttnSpec {
     AttnKvSeg kv[2];
     int q_col, k_col, v_col;
     int B, heads, head_dim;
+    // optional: the per-row log-sum-exp of the scaled scores, in base 2
+    // (lse2 = log2 sum_j 2^(s_j log2(e) / sqrt(d))), kept for the backward:
+    // lse[(b * heads + h) * attn_lse_rows(q0, q1) + (seg ? pad128(q0) : 0) + row]
+    float* lse = nullptr;
 };
+inline int attn_pad128(int n) { return (n + 127) / 128 * 128; }
+inline int attn_lse_rows(int n0, int n1) { return attn_pad128(n0) + attn_pad128(n1); }
 int attention_general(const AttnSpec& a, cudaStream_t stream);
+
+// Backward of joint attention (d = 128): from dO (bf16, the layout of the
+// forward's output) and the forward's lse, the gradients of q, k and v are
+// written into dqkv buffers laid out like the qkv inputs.  ws holds
+// D = rowsum(dO * O) in the lse layout (attention_backward_ws_bytes).
+struct AttnBwdSeg {
+    const __nv_bfloat16* qkv; int64_t ld;   // q, k, v at columns 0, H, 2H
+    const __nv_bfloat16* o;                  // forward output, row pitch ldo
+    const __nv_bfloat16* dout;               // its gradient, row pitch ldo
+    int64_t ldo;
+    __nv_bfloat16* dqkv; int64_t ldd;        // dq, dk, dv at columns 0, H, 2H
+    int n;
+};
+size_t attention_backward_ws_bytes(int B, int heads, int n0, int n1);
+int attention_backward(const AttnBwdSeg& s0, const AttnBwdSeg& s1, int B, int heads, int head_dim,
+                       const float* lse, void* ws, size_t ws_bytes, cudaStream_t stream);
 
 // mods[b, l*6H + j] = e0[b, j] + bias_l[j] (bias_l = bias0 + l*stride), and
 // mods[b, L*6H + j] = e[b, j % H] + fbias[j] for j < 2H (WAN modulation).

@@ -79,6 +79,11 @@ _SIGS = {
     "ff_dit_velocity": ([_P, _I, _P, _P, _P, _P, _P, _SZ, _P], _I),
     "ff_rollout_workspace_size": ([_P, _I, _I, C.POINTER(_SZ)], _I),
     "ff_gemm": ([_I, _I, _I, _P, _I64, _I, _P, _I64, _I, _P, _I, _I, _P, _I64, _P], _I),
+    "ff_attention_lse_rows": ([_I, _I], _I),
+    "ff_attention_forward": ([_I, _I, _I, _I, _P, _I64, _P, _I64, _I, _P, _I64, _P, _I64, _P, _P], _I),
+    "ff_attention_backward_workspace_size": ([_I, _I, _I, _I, C.POINTER(_SZ)], _I),
+    "ff_attention_backward": ([_I, _I, _I, _I, _P, _I64, _P, _P, _I64, _P, _I64, _I, _P, _I64, _P, _P, _I64, _P,
+                               _I64, _P, _P, _SZ, _P], _I),
     "ff_rollout": ([_P, _I, _I, _P, _P, _P, _P, _P, _P, _P, _I, _P, _SZ, _P], _I),
     "ff_debug_gemm": ([_I, _I, _I, _P, _I64, _P, _I64, _P, _I, _I, _P, _I64, _P], _I),
     "ff_debug_gemm_gated": ([_I, _I, _I, _P, _I64, _P, _I64, _P, _P, _I64, _P, _I64, _I, _P], _I),
@@ -429,6 +434,26 @@ def ff_gemm(A, a_layout: int, B, b_layout: int, out, bias=None, act=FF_ACT_NONE,
     N = B.shape[0] if b_layout == FF_B_NK else B.shape[1]
     _call("ff_gemm", M, N, K, _ptr_rows(A), A.stride(0), a_layout, _ptr_rows(B), B.stride(0), b_layout, _ptr(bias),
           act, 1 if out.dtype == torch.float32 else 0, _ptr_rows(out), out.stride(0), _stream(stream))
+
+
+def ff_attention_forward(B, heads, head_dim, qkv0, out0, n0, qkv1, out1, n1, lse=None, stream=None):
+    """Joint attention over [segment 0; segment 1]; lse: [B, heads, ff_attention_lse_rows(n0, n1)] fp32 or None."""
+    _call("ff_attention_forward", B, heads, head_dim, n0, _ptr(qkv0), qkv0.shape[-1], _ptr(out0), out0.shape[-1],
+          n1, _ptr(qkv1), qkv1.shape[-1], _ptr(out1), out1.shape[-1], _ptr(lse), _stream(stream))
+
+
+def ff_attention_backward(B, heads, head_dim, seg0, seg1, lse, ws=None, stream=None):
+    """seg = (n, qkv, out, dout, dqkv) per segment; writes dq, dk, dv into dqkv."""
+    import torch
+    n0, q0, o0, g0, d0 = seg0
+    n1, q1, o1, g1, d1 = seg1
+    if ws is None:
+        sz = _SZ()
+        _call("ff_attention_backward_workspace_size", B, heads, n0, n1, C.byref(sz))
+        ws = torch.empty(sz.value, dtype=torch.uint8, device=lse.device)
+    _call("ff_attention_backward", B, heads, head_dim, n0, _ptr(q0), q0.shape[-1], _ptr(o0), _ptr(g0),
+          o0.shape[-1], _ptr(d0), d0.shape[-1], n1, _ptr(q1), q1.shape[-1], _ptr(o1), _ptr(g1), o1.shape[-1],
+          _ptr(d1), d1.shape[-1], _ptr(lse), _ptr(ws), ws.numel(), _stream(stream))
 
 
 def ff_debug_gemm_gated(A, B, bias, resid, gate, rows_per_sample, stream=None):
