@@ -418,6 +418,64 @@ def awm_step(args, ffi, model, cfg, dev, x0, txt, eps, rewards, timed, world):
             "rooflines": roofs}
 
 
+def backward_kernels(args, ffi, cfg, dev):
+    """The training-backward building blocks at the workload's shapes (one
+    block's attention over the joint sequence, the QKV Linear's three
+    products), CUDA-event timed; algorithmic FLOPs: attention backward
+    10 B h N^2 d (recomputed S, dP, dV, dK, dQ), each GEMM 2 M N K."""
+    import numpy as np
+    import torch
+    B, heads, d = cfg["batch"], cfg["heads"], cfg["head_dim"]
+    if d != 128 or cfg.get("arch") == "wan":
+        return None
+    n0, n1 = cfg["n_txt"], synth_n_img(cfg)
+    H = heads * d
+    g = torch.Generator(device=dev)
+    g.manual_seed(5)
+    rnd = lambda *shape: torch.randn(*shape, generator=g, device=dev).to(torch.bfloat16)
+    q0, q1 = rnd(B * n0, 3 * H), rnd(B * n1, 3 * H)
+    o0, o1 = torch.empty(B * n0, H, device=dev, dtype=torch.bfloat16), torch.empty(B * n1, H, device=dev,
+                                                                                   dtype=torch.bfloat16)
+    g0, g1 = rnd(B * n0, H), rnd(B * n1, H)
+    dq0, dq1 = torch.empty_like(q0), torch.empty_like(q1)
+    lse = torch.empty(B * heads * ffi.lib().ff_attention_lse_rows(n0, n1), device=dev)
+    ffi.ff_attention_forward(B, heads, d, q0, o0, n0, q1, o1, n1, lse=lse)
+    T = B * (n0 + n1)
+    x, W, dy = rnd(T, H), rnd(3 * H, H), rnd(T, 3 * H)
+    y = torch.empty(T, 3 * H, device=dev, dtype=torch.bfloat16)
+    dx = torch.empty(T, H, device=dev, dtype=torch.bfloat16)
+    dW = torch.empty(3 * H, H, device=dev, dtype=torch.float32)
+    N = n0 + n1
+    cases = {
+        "attention_forward_lse": (lambda: ffi.ff_attention_forward(B, heads, d, q0, o0, n0, q1, o1, n1, lse=lse),
+                                  4.0 * B * heads * N * N * d),
+        "attention_backward": (lambda: ffi.ff_attention_backward(B, heads, d, (n0, q0, o0, g0, dq0),
+                                                                 (n1, q1, o1, g1, dq1), lse),
+                               10.0 * B * heads * N * N * d),
+        "qkv_forward": (lambda: ffi.ff_gemm(x, ffi.FF_A_MK, W, ffi.FF_B_NK, y), 2.0 * T * 3 * H * H),
+        "qkv_input_grad": (lambda: ffi.ff_gemm(dy, ffi.FF_A_MK, W, ffi.FF_B_KN, dx), 2.0 * T * 3 * H * H),
+        "qkv_weight_grad": (lambda: ffi.ff_gemm(dy, ffi.FF_A_KM, x, ffi.FF_B_KN, dW), 2.0 * T * 3 * H * H),
+    }
+    _, tc_burst, _, src = load_peaks()
+    out = {}
+    for name, (f, fl) in cases.items():
+        for _ in range(max(3, args.warmup)):
+            f()
+        torch.cuda.synchronize(dev)
+        ts = []
+        for _ in range(max(3, args.steps)):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            f()
+            e1.record()
+            torch.cuda.synchronize(dev)
+            ts.append(e0.elapsed_time(e1))
+        ms = float(np.median(ts))
+        out[name] = {"ms": ms, "tflops": fl / ms / 1e9, "frac": fl / ms / 1e9 / tc_burst}
+    out["peak"] = f"{tc_burst} TFLOP/s ({src} bf16 dense burst)"
+    return out
+
+
 def synth_n_img(cfg):
     import synth
     return synth.n_img(cfg)
@@ -619,6 +677,7 @@ def run_ours(args):
     ms_e2e = timed(e2e_step, args.steps) / args.steps
     e2e_value = whole_job_rate(world, tokens_per_step, ms_e2e)
     awm = awm_step(args, ffi, model, cfg, dev, x, txt, eps, rewards, timed, world)
+    bwd = backward_kernels(args, ffi, cfg, dev) if rank == 0 and not args.no_sweep else None
     sweep = hbm_sweep(ffi, dev, hbm) if rank == 0 and not args.no_sweep else None
     clk = clocks.stop() if clocks else None
     status = ffi.ff_check_device_status()
@@ -647,6 +706,7 @@ def run_ours(args):
                         "ms_per_step": ms_e2e},
                 "hbm_sweep": sweep,
                 "awm_step": awm,
+                "backward_kernels": bwd,
                 "gpu_launches": launches,
                 "clocks": clk,
                 "device_status": status}

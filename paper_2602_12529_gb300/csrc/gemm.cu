@@ -22,6 +22,8 @@
 // Every wait is bounded (ptx.cuh); on a timeout the kernel records
 // kStatusWaitTimeout in the device status word, drains its own tensor-core
 // work, frees TMEM and returns.
+#include <type_traits>
+
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -387,7 +389,6 @@ __device__ __forceinline__ bool epilogue_tile(const GemmEpilogue& epi, int M, in
 // (the text stream of a double-stream block) fills the tail of a large one.
 struct GemmGroup {
     int M[2], N[2], K[2];
-    int a_mn[2], b_mn[2];   // operand storage per problem (see GemmArgs)
     int num_m[2], num_n[2];
     int tiles0, tiles;
     GemmEpilogue epi[2];
@@ -399,7 +400,10 @@ __device__ __forceinline__ void locate(const GemmGroup& g, int tile, int& pr, in
     tile_coords(local, g.num_m[pr], g.num_n[pr], mb, nb);
 }
 
-template <int BN>
+// LAYOUT: bit 0 = A stored MN-major ([K, M]), bit 1 = B stored MN-major
+// ([K, N]); compile-time, so the forward (K-major) kernel issues exactly the
+// instructions it would without the option.
+template <int BN, int LAYOUT>
 __global__ void __launch_bounds__(kThreads, 1)
 gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_constant__ CUtensorMap tm_b0,
                     const __grid_constant__ CUtensorMap tm_a1, const __grid_constant__ CUtensorMap tm_b1,
@@ -475,13 +479,13 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_cons
                 mbar_arrive_expect_tx(&full_bar[stage], C::kStageBytes);
                 // K-major operands: one box of rows x 64 K; MN-major: boxes
                 // of 64 K rows x 64 MN per 64-wide block (8 KB each)
-                if (g.a_mn[pr]) {
+                if (LAYOUT & 1) {
                     for (int j = 0; j < BM / 64; ++j)
                         tma_load_2d(sa + j * 8192, ta, &full_bar[stage], mb * BM + 64 * j, kb * BK);
                 } else {
                     tma_load_2d(sa, ta, &full_bar[stage], kb * BK, mb * BM);
                 }
-                if (g.b_mn[pr]) {
+                if (LAYOUT & 2) {
                     for (int j = 0; j < BN / 64; ++j)
                         tma_load_2d(sb + j * 8192, tb, &full_bar[stage], nb * BN + 64 * j, kb * BK);
                 } else {
@@ -492,7 +496,10 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_cons
         }
     } else if (warp == 1 && lane == 0) {
         // ---------------- MMA issuer
-        constexpr uint32_t idesc0 = idesc_bf16_f32(BM, BN);
+        constexpr bool amn = (LAYOUT & 1) != 0, bmn = (LAYOUT & 2) != 0;
+        constexpr uint32_t idesc = idesc_bf16_f32(BM, BN) | (static_cast<uint32_t>(amn) << 15) |
+                                   (static_cast<uint32_t>(bmn) << 16);
+        constexpr uint64_t a_step = amn ? 128 : 2, b_step = bmn ? 128 : 2;   // one K16 step, encoded >> 4
         int stage = 0;
         uint32_t phase = 0;
         int acc = 0;
@@ -500,9 +507,6 @@ gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_cons
         for (int tile = blockIdx.x; tile < g.tiles && !*abort_flag; tile += gridDim.x) {
             const int pr = tile < g.tiles0 ? 0 : 1;
             const int num_k = (g.K[pr] + BK - 1) / BK;
-            const bool amn = g.a_mn[pr] != 0, bmn = g.b_mn[pr] != 0;
-            const uint32_t idesc = idesc0 | (static_cast<uint32_t>(amn) << 15) | (static_cast<uint32_t>(bmn) << 16);
-            const uint64_t a_step = amn ? 128 : 2, b_step = bmn ? 128 : 2;   // one K16 step, encoded >> 4
             if (!mbar_wait(&tempty_bar[acc], acc_phase ^ 1)) {
                 report_status(status, kStatusWaitTimeout);
                 *abort_flag = 1;
@@ -620,6 +624,7 @@ struct PairCfg {
     static constexpr int kSmemBytes = kPairStages * kStageBytes + kEpiBytes + 1024 + kBarrierBytes;
 };
 
+template <int LAYOUT>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
 gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_constant__ CUtensorMap tm_b0,
                  const __grid_constant__ CUtensorMap tm_a1, const __grid_constant__ CUtensorMap tm_b1,
@@ -698,12 +703,12 @@ gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_constan
                 const uint32_t fb = mapa_shared(smem_u32(&full_bar[stage]), 0);
                 if (rank == 0) mbar_arrive_expect_tx(&full_bar[stage], 2 * C::kStageBytes);
                 const int ma = mb * PBM + rank * 128, nbb = nb * PBN + rank * (PBN / 2);
-                if (g.a_mn[pr]) {
+                if (LAYOUT & 1) {
                     for (int j = 0; j < 2; ++j) tma_load_2d_pair(sa + j * 8192, ta, fb, ma + 64 * j, kb * BK);
                 } else {
                     tma_load_2d_pair(sa, ta, fb, kb * BK, ma);
                 }
-                if (g.b_mn[pr]) {
+                if (LAYOUT & 2) {
                     for (int j = 0; j < 2; ++j) tma_load_2d_pair(sb + j * 8192, tb, fb, nbb + 64 * j, kb * BK);
                 } else {
                     tma_load_2d_pair(sb, tb, fb, kb * BK, nbb);
@@ -713,7 +718,10 @@ gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_constan
         }
     } else if (warp == 1 && lane == 0 && rank == 0) {
         // ---------------- MMA issuer (leader only): 256 x 256 x 16 per instruction
-        constexpr uint32_t idesc0 = idesc_bf16_f32(PBM, PBN);
+        constexpr bool amn = (LAYOUT & 1) != 0, bmn = (LAYOUT & 2) != 0;
+        constexpr uint32_t idesc = idesc_bf16_f32(PBM, PBN) | (static_cast<uint32_t>(amn) << 15) |
+                                   (static_cast<uint32_t>(bmn) << 16);
+        constexpr uint64_t a_step = amn ? 128 : 2, b_step = bmn ? 128 : 2;
         int stage = 0;
         uint32_t phase = 0;
         int acc = 0;
@@ -721,9 +729,6 @@ gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_constan
         for (int tile = cluster; tile < g.tiles && !*abort_flag; tile += nclusters) {
             const int pr = tile < g.tiles0 ? 0 : 1;
             const int num_k = (g.K[pr] + BK - 1) / BK;
-            const bool amn = g.a_mn[pr] != 0, bmn = g.b_mn[pr] != 0;
-            const uint32_t idesc = idesc0 | (static_cast<uint32_t>(amn) << 15) | (static_cast<uint32_t>(bmn) << 16);
-            const uint64_t a_step = amn ? 128 : 2, b_step = bmn ? 128 : 2;
             if (!mbar_wait(&tempty_bar[acc], acc_phase ^ 1)) {
                 report_status(status, kStatusWaitTimeout);
                 *abort_flag = 1;
@@ -841,9 +846,10 @@ int make_out_maps(const GemmArgs& a, CUtensorMap* m) {
     return FF_OK;
 }
 
+template <int LAYOUT>
 int launch_pair(const GemmArgs* p, int n, cudaStream_t stream) {
     using C = PairCfg;
-    if (cudaFuncSetAttribute(gemm_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes) !=
+    if (cudaFuncSetAttribute(gemm_pair_kernel<LAYOUT>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes) !=
         cudaSuccess)
         return set_error(FF_ERR_CUDA, "gemm (pair): cannot set shared memory size (%d B)", C::kSmemBytes);
     CUtensorMap ta[2], tb[2], tr[2];
@@ -868,8 +874,6 @@ int launch_pair(const GemmArgs* p, int n, cudaStream_t stream) {
         g.M[i] = a.M;
         g.N[i] = a.N;
         g.K[i] = a.K;
-        g.a_mn[i] = a.a_mn;
-        g.b_mn[i] = a.b_mn;
         g.num_m[i] = (a.M + PBM - 1) / PBM;
         g.num_n[i] = (a.N + PBN - 1) / PBN;
         g.epi[i] = a.epi;
@@ -887,15 +891,16 @@ int launch_pair(const GemmArgs* p, int n, cudaStream_t stream) {
     g.tiles = g.tiles0 + (n > 1 ? g.num_m[1] * g.num_n[1] : 0);
     const int clusters = g.tiles < num_sms() / 2 ? g.tiles : num_sms() / 2;
     ProfScope prof(stream, "gemm_bf16", flops, bytes);
-    gemm_pair_kernel<<<2 * clusters, kPairThreads, C::kSmemBytes, stream>>>(ta[0], tb[0], ta[1], tb[1], tr[0], tr[1], om,
+    gemm_pair_kernel<LAYOUT><<<2 * clusters, kPairThreads, C::kSmemBytes, stream>>>(ta[0], tb[0], ta[1], tb[1], tr[0], tr[1], om,
                                                                         g, device_status_ptr());
     return check_launch("gemm_pair_kernel");
 }
 
-template <int BN>
+template <int BN, int LAYOUT>
 int launch(const GemmArgs* p, int n, cudaStream_t stream) {
     using C = Cfg<BN>;
-    if (cudaFuncSetAttribute(gemm_tcgen05_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes) !=
+    if (cudaFuncSetAttribute(gemm_tcgen05_kernel<BN, LAYOUT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             C::kSmemBytes) !=
         cudaSuccess)
         return set_error(FF_ERR_CUDA, "gemm: cannot set shared memory size (%d B)", C::kSmemBytes);
     CUtensorMap ta[2], tb[2], tr[2];
@@ -919,8 +924,6 @@ int launch(const GemmArgs* p, int n, cudaStream_t stream) {
         g.M[i] = a.M;
         g.N[i] = a.N;
         g.K[i] = a.K;
-        g.a_mn[i] = a.a_mn;
-        g.b_mn[i] = a.b_mn;
         g.num_m[i] = (a.M + BM - 1) / BM;
         g.num_n[i] = (a.N + BN - 1) / BN;
         g.epi[i] = a.epi;
@@ -938,7 +941,7 @@ int launch(const GemmArgs* p, int n, cudaStream_t stream) {
     for (int i = 0; i < n; ++i)
         if (p[i].epi.epi == EPI_GATED_RESIDUAL && p[i].N % BN)
             return set_error(FF_ERR_UNSUPPORTED, "gemm: gated residual needs N (%d) to be a multiple of %d", p[i].N, BN);
-    gemm_tcgen05_kernel<BN><<<grid, kThreads, C::kSmemBytes, stream>>>(ta[0], tb[0], ta[1], tb[1], tr[0], tr[1], om,
+    gemm_tcgen05_kernel<BN, LAYOUT><<<grid, kThreads, C::kSmemBytes, stream>>>(ta[0], tb[0], ta[1], tb[1], tr[0], tr[1], om,
                                                                        g, device_status_ptr());
     return check_launch("gemm_tcgen05_kernel");
 }
@@ -1111,6 +1114,17 @@ int check_args(const GemmArgs& a) {
 
 }  // namespace
 
+// Calls f with the operand layout as a compile-time constant.
+template <class F>
+int with_layout(int layout, F&& f) {
+    switch (layout) {
+        case 0: return f(std::integral_constant<int, 0>{});
+        case 1: return f(std::integral_constant<int, 1>{});
+        case 2: return f(std::integral_constant<int, 2>{});
+        default: return f(std::integral_constant<int, 3>{});
+    }
+}
+
 int gemm_bf16_group(const GemmArgs* p, int n, cudaStream_t stream) {
     if (!p || n < 1 || n > 2) return set_error(FF_ERR_INVALID_ARG, "gemm: 1 or 2 problems per launch");
     bool qk = false;
@@ -1129,11 +1143,14 @@ int gemm_bf16_group(const GemmArgs* p, int n, cudaStream_t stream) {
         pair = pair && p[i].N % 256 == 0 && p[i].epi.rows_gemv == 0;
         max_m = p[i].M > max_m ? p[i].M : max_m;
     }
-    if (pair && max_m >= 512) return launch_pair(p, n, stream);
+    const int layout = p[0].a_mn | (p[0].b_mn << 1);
+    if (n == 2 && (p[1].a_mn | (p[1].b_mn << 1)) != layout)
+        return set_error(FF_ERR_INVALID_ARG, "gemm: grouped problems must share the operand layout");
+    if (pair && max_m >= 512) return with_layout(layout, [&](auto L) { return launch_pair<L.value>(p, n, stream); });
     if (n == 2 || qk) {
         for (int i = 0; i < n; ++i)
             if (p[i].N <= 128) return set_error(FF_ERR_UNSUPPORTED, "gemm: grouped / fused problems need N > 128");
-        return launch<256>(p, n, stream);
+        return with_layout(layout, [&](auto L) { return launch<256, L.value>(p, n, stream); });
     }
     const GemmArgs& a = p[0];
     const bool gemv_ok = !a.a_mn && !a.b_mn && a.K <= kGemvMaxK && a.epi.epi == EPI_STORE && a.epi.split_n >= a.N &&
@@ -1144,9 +1161,9 @@ int gemm_bf16_group(const GemmArgs* p, int n, cudaStream_t stream) {
     // narrow tiles when wide ones would leave most SMs idle
     const int64_t mblocks = (a.M + BM - 1) / BM;
     const bool few = mblocks * ((a.N + 255) / 256) < num_sms() / 2;
-    if (a.N <= 64 || few) return launch<64>(p, 1, stream);
-    if (a.N <= 128) return launch<128>(p, 1, stream);
-    return launch<256>(p, 1, stream);
+    if (a.N <= 64 || few) return with_layout(layout, [&](auto L) { return launch<64, L.value>(p, 1, stream); });
+    if (a.N <= 128) return with_layout(layout, [&](auto L) { return launch<128, L.value>(p, 1, stream); });
+    return with_layout(layout, [&](auto L) { return launch<256, L.value>(p, 1, stream); });
 }
 
 int gemm_bf16(const void* A, int64_t lda, const void* B, int64_t ldb, int M, int N, int K, const GemmEpilogue& e,
