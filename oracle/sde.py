@@ -104,3 +104,27 @@ def sde_step_logprob(x, v, t, t_next, sigma, eps=None, x_next=None, reduce: str 
             out[b] = np.asarray(x_next[b], dtype=np.float64)
         lp[b] = gaussian_logprob(out[b], mean, std, reduce)
     return out, lp
+
+
+def sde_logprob_grad_v(x, v, x_next, t, t_next, sigma, reduce: str = "sum") -> np.ndarray:
+    """d logp_b / d v_b of the Eq. 1 transition with x_next held fixed (the
+    training pass re-scores the rollout's x_next under the current v).
+
+    logp = -|x_next - mean|^2 / (2 std^2) + const depends on v only through
+    mean, and d mean_j / d v_j = -Delta (1 + sigma^2 (1 - t) / (2 t)), so
+        d logp / d v_j = (x_next_j - mean_j) / std^2 * d mean_j / d v_j
+    (divided by D for the "mean" reduction).  Zero where std = 0 (no density).
+    x, v, x_next: [B, ...]; t, t_next, sigma: [B].
+    """
+    x = np.asarray(x, dtype=np.float64)
+    out = np.zeros_like(x)
+    for b in range(x.shape[0]):
+        tb, sb = float(t[b]), float(sigma[b])
+        mean, std = sde_mean_std(x[b], v[b], tb, float(t_next[b]), sb)
+        if std == 0.0:
+            continue
+        delta = tb - float(t_next[b])
+        dmean_dv = -delta * (1.0 + sb * sb * (1.0 - tb) / (2.0 * tb))
+        g = (np.asarray(x_next[b], dtype=np.float64) - mean) / (std * std) * dmean_dv
+        out[b] = g / x[b].size if reduce == "mean" else g
+    return out
