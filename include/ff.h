@@ -148,6 +148,23 @@ int ff_sde_step_logprob(int B, int64_t D, const float* x_t, const float* v,
                         cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
+ * Gradient of the transition log-probability in v, with x_next held fixed
+ * (the training pass of Flow-GRPO, Sec. 3.1, re-scores the rollout's x_next
+ * under the current velocity).  From Eq. 1, mean depends on v as
+ * d mean_j / d v_j = -Delta (1 + sigma^2 (1 - t) / (2 t)), so
+ *   grad_v[b, j] = grad_logp[b * ld] * (x_next_j - mean_j) / std^2
+ *                  * d mean_j / d v_j   (divided by D for FF_LP_MEAN),
+ * and 0 where std == 0 (no density).  Arrays as ff_sde_step_logprob (EVAL);
+ * grad_logp: fp32 device, read at b * ld (e.g. a column of the
+ * grad_lp_new output of ff_grpo_loss, ld = T); grad_v: [B, D] fp32,
+ * written (may not alias the inputs).  No workspace.
+ * ------------------------------------------------------------------------ */
+int ff_sde_logprob_backward(int B, int64_t D, const float* x_t, const float* v,
+                            const float* x_next, const float* t, const float* t_next,
+                            const float* sigma, int reduce, const float* grad_logp, int ld,
+                            float* grad_v, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
  * ff_sde_step_logprob_noalloc -- the SDE step + log-prob above, for callers
  * that cannot allocate device memory: for example a plug-in running inside a
  * host application that owns every device allocation itself (its own pool,
@@ -336,6 +353,35 @@ int ff_dit_workspace_size(const ff_dit* model, int B, size_t* bytes);
 int ff_dit_velocity(const ff_dit* model, int B, const float* x_t, const void* txt,
                     const float* t, float* v_out, void* ws, size_t ws_bytes,
                     cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Training pass of the velocity network (MMDiT models, head_dim 128): the
+ * forward every GRPO-style trainer runs "again for training" (Sec. 1) and
+ * its gradient, for the policy losses of Sec. 3 (the Flow-GRPO loss through
+ * ff_sde_logprob_backward, AWM's Eq. 3 through ff_awm_loss's dL/dv).
+ *
+ * ff_dit_forward_train: the same computation as ff_dit_velocity (same
+ *   arguments, bit-identical v_out) that also keeps, in ws, every activation
+ *   the backward reads.  ws: ff_dit_train_workspace_size bytes, 256-byte
+ *   aligned; it must stay untouched until the matching ff_dit_backward.
+ * ff_dit_backward: from dv = dL/dv ([B, N_i, P] fp32, device) to
+ *   grad: fp32 device blob of ff_dit_weight_layout's total_elems elements,
+ *     element offsets as in the weight blob; every element of every tensor
+ *     is overwritten with dL/dtheta (the padding between tensors is not
+ *     touched);
+ *   dx_t: [B, N_i, P] fp32 dL/dx_t, or NULL.
+ *   txt must hold the same text embeddings as in the forward.  Every sum
+ *   over tokens runs in a fixed order: the result is deterministic.
+ * Requires B N_t and B N_i multiples of 8.  The workspace holds about
+ * R (30 H + 4 F) bytes per double-stream block and R (22 H + 4 F) per
+ * single-stream block, R = B (N_t + N_i), plus scratch.
+ * ------------------------------------------------------------------------ */
+int ff_dit_train_workspace_size(const ff_dit* model, int B, size_t* bytes);
+int ff_dit_forward_train(const ff_dit* model, int B, const float* x_t, const void* txt,
+                         const float* t, float* v_out, void* ws, size_t ws_bytes,
+                         cudaStream_t stream);
+int ff_dit_backward(const ff_dit* model, int B, const void* txt, const float* dv, float* grad,
+                    float* dx_t, void* ws, size_t ws_bytes, cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
  * bf16 GEMM with fp32 accumulation on the tcgen05 kernels of the velocity:

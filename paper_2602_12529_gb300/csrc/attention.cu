@@ -432,8 +432,9 @@ int attention_general(const AttnSpec& a, cudaStream_t stream) {
 }
 
 int attention(const AttnSegment& s0, const AttnSegment& s1, int B, int heads, int head_dim, int H,
-              cudaStream_t stream) {
+              cudaStream_t stream, float* lse) {
     AttnSpec a;
+    a.lse = lse;
     const AttnSegment* seg[2] = {&s0, &s1};
     for (int i = 0; i < 2; ++i) {
         a.q[i] = AttnQuerySeg{seg[i]->qkv, seg[i]->ld, seg[i]->n, seg[i]->out, seg[i]->ldo};

@@ -89,8 +89,8 @@ __device__ __forceinline__ void store_row_bf16(uint32_t taddr, float mul, __nv_b
 __global__ void __launch_bounds__(256) attn_bwd_delta_kernel(int B, int heads, int n0, int n1,
                                                              const __nv_bfloat16* o0, const __nv_bfloat16* do0,
                                                              const __nv_bfloat16* o1, const __nv_bfloat16* do1,
-                                                             int64_t ldo0, int64_t ldo1, int lse_rows, int base1,
-                                                             float* delta) {
+                                                             int64_t ldo0, int64_t ldo1, int64_t ldg0, int64_t ldg1,
+                                                             int lse_rows, int base1, float* delta) {
     const int64_t w = (static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x) >> 5;
     const int lane = threadIdx.x & 31;
     const int64_t rows0 = static_cast<int64_t>(B) * n0;
@@ -103,9 +103,8 @@ __global__ void __launch_bounds__(256) attn_bwd_delta_kernel(int B, int heads, i
     const int n = s1 ? n1 : n0;
     const int b = static_cast<int>(rr / n);
     const int row = static_cast<int>(rr - static_cast<int64_t>(b) * n);
-    const int64_t ld = s1 ? ldo1 : ldo0;
-    const __nv_bfloat16* o = (s1 ? o1 : o0) + rr * ld + h * HD + lane * 4;
-    const __nv_bfloat16* g = (s1 ? do1 : do0) + rr * ld + h * HD + lane * 4;
+    const __nv_bfloat16* o = (s1 ? o1 : o0) + rr * (s1 ? ldo1 : ldo0) + h * HD + lane * 4;
+    const __nv_bfloat16* g = (s1 ? do1 : do0) + rr * (s1 ? ldg1 : ldg0) + h * HD + lane * 4;
     const uint2 ov = *reinterpret_cast<const uint2*>(o);
     const uint2 gv = *reinterpret_cast<const uint2*>(g);
     const float2 o01 = unpack_bf16x2(ov.x), o23 = unpack_bf16x2(ov.y);
@@ -499,7 +498,8 @@ int attention_backward(const AttnBwdSeg& s0, const AttnBwdSeg& s1, int B, int he
         const AttnBwdSeg& s = *sg[i];
         if (!s.n) continue;
         if (!s.qkv || !s.o || !s.dout || !s.dqkv || !aligned16(s.o) || !aligned16(s.dout) || !aligned16(s.dqkv) ||
-            s.ld % 8 || s.ldo % 8 || s.ldd % 8 || s.ld < 3 * H || s.ldo < H || s.ldd < 3 * H)
+            s.ld % 8 || s.ldo % 8 || s.ldd % 8 || s.ldg % 8 || s.ld < 3 * H || s.ldo < H || s.ldd < 3 * H ||
+            (s.ldg && s.ldg < H))
             return set_error(FF_ERR_INVALID_ARG, "attention backward: bad segment %d", i);
     }
     const size_t need = attention_backward_ws_bytes(B, heads, s0.n, s1.n);
@@ -514,7 +514,7 @@ int attention_backward(const AttnBwdSeg& s0, const AttnBwdSeg& s1, int B, int he
     for (int i = 0; i < 2; ++i) {
         const AttnBwdSeg& s = sg[i]->n > 0 ? *sg[i] : *sg[1 - i];   // an empty segment still needs a valid map
         FF_TRY(make_tmap_bf16(&tqkv[i], s.qkv, static_cast<int64_t>(B) * s.n, 3 * H, s.ld, kT));
-        FF_TRY(make_tmap_bf16(&tdo[i], s.dout, static_cast<int64_t>(B) * s.n, H, s.ldo, kT));
+        FF_TRY(make_tmap_bf16(&tdo[i], s.dout, static_cast<int64_t>(B) * s.n, H, s.ldg ? s.ldg : s.ldo, kT));
     }
     float* delta = static_cast<float*>(ws);
     const int rows = attn_lse_rows(s0.n, s1.n);
@@ -522,7 +522,8 @@ int attention_backward(const AttnBwdSeg& s0, const AttnBwdSeg& s1, int B, int he
         const int64_t warps = (static_cast<int64_t>(B) * (s0.n + s1.n)) * heads;
         ProfScope prof(stream, "attn_bwd_delta", 0.0, 4.0 * warps * HD);
         attn_bwd_delta_kernel<<<static_cast<unsigned>((warps + 7) / 8), 256, 0, stream>>>(
-            B, heads, s0.n, s1.n, s0.o, s0.dout, s1.o, s1.dout, s0.ldo, s1.ldo, rows, attn_pad128(s0.n), delta);
+            B, heads, s0.n, s1.n, s0.o, s0.dout, s1.o, s1.dout, s0.ldo, s1.ldo, s0.ldg ? s0.ldg : s0.ldo,
+            s1.ldg ? s1.ldg : s1.ldo, rows, attn_pad128(s0.n), delta);
         FF_TRY(check_launch("attn_bwd_delta_kernel"));
     }
     BwdParams p;

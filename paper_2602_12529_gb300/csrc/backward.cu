@@ -1,0 +1,486 @@
+// backward.cu -- row and column kernels of the DiT backward (the training
+// pass of the policy update differentiates the loss through v_theta):
+//   * gate_backward: through the gated residual x' = x + gate * y, the
+//     branch gradient dy = g * gate (bf16 GEMM operand) and per-chunk column
+//     sums of g * y (the gate's gradient, per sample) and g * gate (the
+//     branch bias's gradient);
+//   * ln_modulate_backward: through h = LN(x) (1 + scale) + shift, the
+//     residual gradient g += (dn - mean(dn) - n mean(dn n)) / s with
+//     dn = dh (1 + scale), and per-chunk column sums of dh and dh n;
+//   * qk_norm_rope_backward: through q = rope(RMSNorm(q_raw) w), in place on
+//     the q | k gradient columns, with per-CTA partial sums of the scale's
+//     gradient;
+//   * colsum: column sums of a bf16 or fp32 matrix (bias gradients);
+//   * silu_backward: dx = dy SiLU'(pre) for the timestep MLP;
+//   * reduce_chunks: fixed-order fp64 sums of the partials, so every
+//     gradient is deterministic.
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace ff {
+namespace {
+
+constexpr float kLnEps = 1e-6f;
+constexpr float kRmsEps = 1e-6f;
+constexpr int kThreads = 256;
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// Sum over the CTA; red holds one slot per warp and is not reused until
+// every thread has passed a later __syncthreads.
+__device__ __forceinline__ float2 block_sum2(float2 v, float2* red, int lane, int w) {
+    v.x = warp_sum(v.x);
+    v.y = warp_sum(v.y);
+    if (lane == 0) red[w] = v;
+    __syncthreads();
+    float2 t = make_float2(0.f, 0.f);
+#pragma unroll
+    for (int i = 0; i < kThreads / 32; ++i) {
+        t.x += red[i].x;
+        t.y += red[i].y;
+    }
+    return t;
+}
+
+// Chunk c of a segment list -> its segment (copied out with selects, so the
+// parameter struct is never indexed dynamically), sample and row range.
+__device__ __forceinline__ bool chunk_rows(const BwdSegs& s, int c, BwdSeg& sg, int& b, int& r0, int& r1) {
+    const bool second = c >= s.first[1];
+    if (second && s.n < 2) return false;
+    sg.row0 = second ? s.seg[1].row0 : s.seg[0].row0;
+    sg.tokens = second ? s.seg[1].tokens : s.seg[0].tokens;
+    sg.col_a = second ? s.seg[1].col_a : s.seg[0].col_a;
+    sg.col_b = second ? s.seg[1].col_b : s.seg[0].col_b;
+    const int local = c - (second ? s.first[1] : s.first[0]);
+    const int cps = bwd_chunks(sg.tokens);
+    b = local / cps;
+    if (b >= s.B) return false;
+    const int k = local - b * cps;
+    const int start = sg.row0 + b * sg.tokens;
+    r0 = start + k * kBwdChunk;
+    r1 = min(r0 + kBwdChunk, start + sg.tokens);
+    return true;
+}
+
+// ---------------------------------------------------------------- gate
+
+// CTA = (chunk, 1024-column slab); thread t owns columns 4 (slab 256 + t) ..+3.
+__global__ void __launch_bounds__(kThreads) gate_backward_kernel(const float* g, const __nv_bfloat16* y, int64_t ld,
+                                                                  const float* mods, int64_t ld_mods, BwdSegs s, int H,
+                                                                  __nv_bfloat16* dy, float* part) {
+    BwdSeg sg;
+    int b, r0, r1;
+    if (!chunk_rows(s, blockIdx.x, sg, b, r0, r1)) return;
+    const int j = 4 * (blockIdx.y * kThreads + threadIdx.x);
+    if (j >= H) return;
+    const float4 gt = *reinterpret_cast<const float4*>(mods + static_cast<int64_t>(b) * ld_mods + sg.col_a + j);
+    float4 sy = make_float4(0.f, 0.f, 0.f, 0.f), sb = sy;
+    for (int r = r0; r < r1; ++r) {
+        const int64_t o = static_cast<int64_t>(r) * ld + j;
+        const float4 gv = __ldcs(reinterpret_cast<const float4*>(g + o));
+        const uint2 yu = *reinterpret_cast<const uint2*>(y + o);
+        const float2 y01 = unpack_bf16x2(yu.x), y23 = unpack_bf16x2(yu.y);
+        sy.x = fmaf(gv.x, y01.x, sy.x);
+        sy.y = fmaf(gv.y, y01.y, sy.y);
+        sy.z = fmaf(gv.z, y23.x, sy.z);
+        sy.w = fmaf(gv.w, y23.y, sy.w);
+        const float d0 = gv.x * gt.x, d1 = gv.y * gt.y, d2 = gv.z * gt.z, d3 = gv.w * gt.w;
+        sb.x += d0;
+        sb.y += d1;
+        sb.z += d2;
+        sb.w += d3;
+        *reinterpret_cast<uint2*>(dy + o) = make_uint2(pack_bf16x2(d0, d1), pack_bf16x2(d2, d3));
+    }
+    float* p = part + static_cast<int64_t>(blockIdx.x) * 2 * H + j;
+    *reinterpret_cast<float4*>(p) = sy;
+    *reinterpret_cast<float4*>(p + H) = sb;
+}
+
+// ---------------------------------------------------------------- LN-modulate
+
+// CTA = one chunk of rows, all H columns: thread t holds float4s t, t + 256,
+// ... of a row (PER of them).  Per row: mean and centred variance of x (as in
+// the forward), then the two means of the LayerNorm backward; the next row's
+// loads are issued before this row's reductions.
+template <int PER>
+__global__ void __launch_bounds__(kThreads) ln_modulate_backward_kernel(const float* x, const float* dh, float* gx,
+                                                                         int64_t ld, const float* mods,
+                                                                         int64_t ld_mods, BwdSegs s, int H,
+                                                                         float* part) {
+    __shared__ float2 red[3][kThreads / 32];
+    BwdSeg sg;
+    int b, r0, r1;
+    if (!chunk_rows(s, blockIdx.x, sg, b, r0, r1)) return;
+    const int t = threadIdx.x, lane = t & 31, w = t >> 5;
+    const int nv = H >> 2;
+    const float4* scale = reinterpret_cast<const float4*>(mods + static_cast<int64_t>(b) * ld_mods + sg.col_b);
+    float4 sc1[PER];
+#pragma unroll
+    for (int i = 0; i < PER; ++i) {
+        const int k = t + kThreads * i;
+        const float4 c = k < nv ? scale[k] : make_float4(0.f, 0.f, 0.f, 0.f);
+        sc1[i] = make_float4(1.f + c.x, 1.f + c.y, 1.f + c.z, 1.f + c.w);
+    }
+    float4 acc_sh[PER], acc_sc[PER];
+#pragma unroll
+    for (int i = 0; i < PER; ++i) acc_sh[i] = acc_sc[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+    float4 xr[PER], dr[PER];
+    {
+        const float4* xp = reinterpret_cast<const float4*>(x + static_cast<int64_t>(r0) * ld);
+        const float4* dp = reinterpret_cast<const float4*>(dh + static_cast<int64_t>(r0) * ld);
+#pragma unroll
+        for (int i = 0; i < PER; ++i) {
+            const int k = t + kThreads * i;
+            xr[i] = k < nv ? __ldcs(xp + k) : z;
+            dr[i] = k < nv ? __ldcs(dp + k) : z;
+        }
+    }
+    const float invH = 1.f / H;
+    for (int r = r0; r < r1; ++r) {
+        float4 xn[PER], dn[PER];
+        {
+            const bool more = r + 1 < r1;
+            const float4* xp = reinterpret_cast<const float4*>(x + static_cast<int64_t>(r + 1) * ld);
+            const float4* dp = reinterpret_cast<const float4*>(dh + static_cast<int64_t>(r + 1) * ld);
+#pragma unroll
+            for (int i = 0; i < PER; ++i) {
+                const int k = t + kThreads * i;
+                xn[i] = more && k < nv ? __ldcs(xp + k) : z;
+                dn[i] = more && k < nv ? __ldcs(dp + k) : z;
+            }
+        }
+        float sx = 0.f;
+#pragma unroll
+        for (int i = 0; i < PER; ++i) sx += (xr[i].x + xr[i].y) + (xr[i].z + xr[i].w);
+        const float mean = block_sum2(make_float2(sx, 0.f), red[0], lane, w).x * invH;
+        float q = 0.f;
+#pragma unroll
+        for (int i = 0; i < PER; ++i) {
+            if (t + kThreads * i < nv) {
+                const float d0 = xr[i].x - mean, d1 = xr[i].y - mean, d2 = xr[i].z - mean, d3 = xr[i].w - mean;
+                q += (d0 * d0 + d1 * d1) + (d2 * d2 + d3 * d3);
+            }
+        }
+        const float rstd = rsqrtf(block_sum2(make_float2(q, 0.f), red[1], lane, w).x * invH + kLnEps);
+        // n = (x - mean) rstd, dn = dh (1 + scale); overwrite xr with n, dr with dn
+        float s1 = 0.f, s2 = 0.f;
+#pragma unroll
+        for (int i = 0; i < PER; ++i) {
+            float4 n = make_float4((xr[i].x - mean) * rstd, (xr[i].y - mean) * rstd, (xr[i].z - mean) * rstd,
+                                   (xr[i].w - mean) * rstd);
+            if (t + kThreads * i >= nv) n = z;
+            acc_sh[i].x += dr[i].x; acc_sh[i].y += dr[i].y; acc_sh[i].z += dr[i].z; acc_sh[i].w += dr[i].w;
+            acc_sc[i].x = fmaf(dr[i].x, n.x, acc_sc[i].x);
+            acc_sc[i].y = fmaf(dr[i].y, n.y, acc_sc[i].y);
+            acc_sc[i].z = fmaf(dr[i].z, n.z, acc_sc[i].z);
+            acc_sc[i].w = fmaf(dr[i].w, n.w, acc_sc[i].w);
+            const float4 d = make_float4(dr[i].x * sc1[i].x, dr[i].y * sc1[i].y, dr[i].z * sc1[i].z, dr[i].w * sc1[i].w);
+            s1 += (d.x + d.y) + (d.z + d.w);
+            s2 += (d.x * n.x + d.y * n.y) + (d.z * n.z + d.w * n.w);
+            xr[i] = n;
+            dr[i] = d;
+        }
+        const float2 m = block_sum2(make_float2(s1, s2), red[2], lane, w);
+        const float m1 = m.x * invH, m2 = m.y * invH;
+        float4* gp = reinterpret_cast<float4*>(gx + static_cast<int64_t>(r) * ld);
+#pragma unroll
+        for (int i = 0; i < PER; ++i) {
+            const int k = t + kThreads * i;
+            if (k >= nv) continue;
+            float4 o = gp[k];
+            o.x += rstd * (dr[i].x - m1 - xr[i].x * m2);
+            o.y += rstd * (dr[i].y - m1 - xr[i].y * m2);
+            o.z += rstd * (dr[i].z - m1 - xr[i].z * m2);
+            o.w += rstd * (dr[i].w - m1 - xr[i].w * m2);
+            gp[k] = o;
+        }
+#pragma unroll
+        for (int i = 0; i < PER; ++i) {
+            xr[i] = xn[i];
+            dr[i] = dn[i];
+        }
+    }
+    float4* p = reinterpret_cast<float4*>(part + static_cast<int64_t>(blockIdx.x) * 2 * H);
+#pragma unroll
+    for (int i = 0; i < PER; ++i) {
+        const int k = t + kThreads * i;
+        if (k >= nv) continue;
+        p[k] = acc_sh[i];
+        p[nv + k] = acc_sc[i];
+    }
+}
+
+// ---------------------------------------------------------------- QK norm + RoPE
+
+// One warp per (row, head) item, lane owns E = d / 32 consecutive elements
+// (whole rotation pairs).  A CTA covers kQkRows rows of one segment and
+// every head; its warps add their lanes' scale-gradient terms, summed over
+// the CTA at the end into part[cta][q: 0..d | k: d..2d].
+constexpr int kQkRows = kQkBwdRows;
+
+template <int E>
+__global__ void __launch_bounds__(kThreads) qk_norm_rope_backward_kernel(QkBwdArgs a, int ctas_txt) {
+    __shared__ float red[kThreads / 32][2][128];
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    const bool img = static_cast<int>(blockIdx.x) >= ctas_txt;
+    const int r_begin = img ? a.rows_txt + (blockIdx.x - ctas_txt) * kQkRows : blockIdx.x * kQkRows;
+    const int r_end = min(r_begin + kQkRows, img ? a.rows : a.rows_txt);
+    const int c0 = lane * E;
+    const int d = a.head_dim;
+    const __nv_bfloat16* qs = img ? a.q_scale_img : a.q_scale_txt;
+    const __nv_bfloat16* ks = img ? a.k_scale_img : a.k_scale_txt;
+    float wq[E], wk[E], gq[E], gk[E];
+#pragma unroll
+    for (int i = 0; i < E; ++i) {
+        wq[i] = __bfloat162float(qs[c0 + i]);
+        wk[i] = __bfloat162float(ks[c0 + i]);
+        gq[i] = gk[i] = 0.f;
+    }
+    const int h0 = a.axes0 >> 1, h1 = a.axes1 >> 1;
+    const int items = (r_end - r_begin) * a.heads;
+    for (int it = w; it < items; it += kThreads / 32) {
+        const int row = r_begin + it / a.heads;
+        const int head = it - (it / a.heads) * a.heads;
+        // rotation of this lane's pairs (identity for text tokens)
+        float cs[E / 2], sn[E / 2];
+        if (img && a.rope_cs) {
+            const int n = (row - a.rows_txt) % a.n_img;
+            const int hw = a.grid_h * a.grid_w;
+            const int base0 = (n / hw) * h0;
+            const int base1 = a.grid_f * h0 + ((n / a.grid_w) % a.grid_h) * h1 - h0;
+            const int base2 = a.grid_f * h0 + a.grid_h * h1 + (n % a.grid_w) * (a.axes2 >> 1) - h0 - h1;
+#pragma unroll
+            for (int p = 0; p < E / 2; ++p) {
+                const int pair = c0 / 2 + p;
+                const float2 t = a.rope_cs[pair < h0 ? base0 + pair : (pair < h0 + h1 ? base1 + pair : base2 + pair)];
+                cs[p] = t.x;
+                sn[p] = t.y;
+            }
+        } else {
+#pragma unroll
+            for (int p = 0; p < E / 2; ++p) { cs[p] = 1.f; sn[p] = 0.f; }
+        }
+#pragma unroll
+        for (int which = 0; which < 2; ++which) {
+            const int col = which * a.heads * d + head * d + c0;
+            __nv_bfloat16* gp = a.d + static_cast<int64_t>(row) * a.ldd + col;
+            const __nv_bfloat16* xp = a.raw + static_cast<int64_t>(row) * a.ldr + col;
+            float gv[E], xv[E];
+#pragma unroll
+            for (int i = 0; i < E; i += 2) {
+                const float2 g2 = unpack_bf16x2(*reinterpret_cast<const uint32_t*>(gp + i));
+                const float2 x2 = unpack_bf16x2(*reinterpret_cast<const uint32_t*>(xp + i));
+                gv[i] = g2.x; gv[i + 1] = g2.y;
+                xv[i] = x2.x; xv[i + 1] = x2.y;
+            }
+            // transposed rotation: gradient w.r.t. the normalised, scaled values
+            float gy[E];
+#pragma unroll
+            for (int p = 0; p < E / 2; ++p) {
+                gy[2 * p] = gv[2 * p] * cs[p] + gv[2 * p + 1] * sn[p];
+                gy[2 * p + 1] = -gv[2 * p] * sn[p] + gv[2 * p + 1] * cs[p];
+            }
+            float ss = 0.f;
+#pragma unroll
+            for (int i = 0; i < E; ++i) ss = fmaf(xv[i], xv[i], ss);
+            const float r = rsqrtf(warp_sum(ss) / d + kRmsEps);
+            const float* wv = which ? wk : wq;
+            float* acc = which ? gk : gq;
+            float dot = 0.f;
+            float xn[E], gg[E];
+#pragma unroll
+            for (int i = 0; i < E; ++i) {
+                xn[i] = xv[i] * r;
+                gg[i] = gy[i] * wv[i];
+                acc[i] = fmaf(gy[i], xn[i], acc[i]);
+                dot = fmaf(gg[i], xn[i], dot);
+            }
+            const float m = warp_sum(dot) / d;
+#pragma unroll
+            for (int i = 0; i < E; i += 2)
+                *reinterpret_cast<uint32_t*>(gp + i) =
+                    pack_bf16x2(r * (gg[i] - xn[i] * m), r * (gg[i + 1] - xn[i + 1] * m));
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < E; ++i) {
+        red[w][0][c0 + i] = gq[i];
+        red[w][1][c0 + i] = gk[i];
+    }
+    __syncthreads();
+    for (int k = threadIdx.x; k < 2 * d; k += kThreads) {
+        const int which = k / d, j = k - which * d;
+        float s = 0.f;
+#pragma unroll
+        for (int ww = 0; ww < kThreads / 32; ++ww) s += red[ww][which][j];
+        a.part[static_cast<int64_t>(blockIdx.x) * 2 * d + k] = s;
+    }
+}
+
+// ---------------------------------------------------------------- column sums
+
+// CTA = (chunk of kBwdChunk rows, 1024-column slab).
+template <typename T>
+__global__ void __launch_bounds__(kThreads) colsum_partial_kernel(const T* in, int64_t ld, int rows, int ncols,
+                                                                   float* part) {
+    const int j = 4 * (blockIdx.y * kThreads + threadIdx.x);
+    if (j >= ncols) return;
+    const int r0 = blockIdx.x * kBwdChunk, r1 = min(r0 + kBwdChunk, rows);
+    float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int r = r0; r < r1; ++r) {
+        float4 v;
+        if constexpr (sizeof(T) == 4) {
+            v = *reinterpret_cast<const float4*>(in + static_cast<int64_t>(r) * ld + j);
+        } else {
+            const uint2 u = *reinterpret_cast<const uint2*>(in + static_cast<int64_t>(r) * ld + j);
+            const float2 a = unpack_bf16x2(u.x), b = unpack_bf16x2(u.y);
+            v = make_float4(a.x, a.y, b.x, b.y);
+        }
+        s.x += v.x; s.y += v.y; s.z += v.z; s.w += v.w;
+    }
+    *reinterpret_cast<float4*>(part + static_cast<int64_t>(blockIdx.x) * ncols + j) = s;
+}
+
+// ---------------------------------------------------------------- chunk reduction
+
+// out[b * ld_out + j] = sum over sample b's chunks of every span (per_sample),
+// or out[j] = sum over all chunks of every span; fp64 in a fixed order.
+__global__ void reduce_chunks_kernel(const float* part, int64_t ld_part, int ncols, ChunkSpans sp, int per_sample,
+                                     float* out, int64_t ld_out) {
+    const int j = blockIdx.x * blockDim.x + threadIdx.x;
+    if (j >= ncols) return;
+    const int b = blockIdx.y;
+    double s = 0.0;
+    for (int i = 0; i < sp.n; ++i) {
+        const int first = per_sample ? sp.first[i] + b * sp.count[i] : sp.first[i];
+        for (int c = 0; c < sp.count[i]; ++c) s += part[static_cast<int64_t>(first + c) * ld_part + j];
+    }
+    out[static_cast<int64_t>(b) * ld_out + j] = static_cast<float>(s);
+}
+
+// ---------------------------------------------------------------- SiLU
+
+// dx = dy SiLU'(pre) for rows < B, written fp32 [B, n] and bf16 [rows_pad, n]
+// (rows B.. rows_pad - 1 zero: the padded operand of the weight gradient).
+__global__ void silu_backward_kernel(const float* dy, int64_t ld_dy, const __nv_bfloat16* pre, int B, int rows_pad,
+                                     int n, float* dx, __nv_bfloat16* dxb) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= rows_pad * n) return;
+    const int b = i / n, j = i - b * n;
+    float v = 0.f;
+    if (b < B) {
+        const float p = __bfloat162float(pre[i]);
+        const float s = 1.f / (1.f + __expf(-p));
+        v = dy[static_cast<int64_t>(b) * ld_dy + j] * s * (1.f + p * (1.f - s));
+        dx[i] = v;
+    }
+    dxb[i] = __float2bfloat16_rn(v);
+}
+
+int reduce(const float* part, int64_t ld_part, int ncols, const ChunkSpans& sp, int B, float* out, int64_t ld_out,
+           cudaStream_t stream) {
+    dim3 grid((ncols + 255) / 256, B > 0 ? B : 1);
+    reduce_chunks_kernel<<<grid, 256, 0, stream>>>(part, ld_part, ncols, sp, B > 0, out, ld_out);
+    return check_launch("reduce_chunks_kernel");
+}
+
+}  // namespace
+
+BwdSegs bwd_segs(const BwdSeg* segs, int n, int B) {
+    BwdSegs s{};
+    s.n = n;
+    s.B = B;
+    int c = 0;
+    for (int i = 0; i < 2; ++i) {
+        s.first[i] = c;
+        if (i < n) {
+            s.seg[i] = segs[i];
+            c += B * bwd_chunks(segs[i].tokens);
+        }
+    }
+    s.chunks = c;
+    s.rows = 0;
+    for (int i = 0; i < n; ++i) s.rows += static_cast<int64_t>(B) * segs[i].tokens;
+    return s;
+}
+
+int gate_backward(const float* g, const __nv_bfloat16* y, int64_t ld, const float* mods, int64_t ld_mods,
+                  const BwdSegs& s, int H, __nv_bfloat16* dy, float* part, cudaStream_t stream) {
+    if (H % 4 || ld % 4) return set_error(FF_ERR_UNSUPPORTED, "gate_backward: H and ld must be multiples of 4");
+    if (s.chunks == 0) return FF_OK;
+    ProfScope prof(stream, "gate_backward", 0.0, 8.0 * s.rows * H);
+    dim3 grid(s.chunks, (H / 4 + kThreads - 1) / kThreads);
+    gate_backward_kernel<<<grid, kThreads, 0, stream>>>(g, y, ld, mods, ld_mods, s, H, dy, part);
+    return check_launch("gate_backward_kernel");
+}
+
+int ln_modulate_backward(const float* x, const float* dh, float* gx, int64_t ld, const float* mods, int64_t ld_mods,
+                         const BwdSegs& s, int H, float* part, cudaStream_t stream) {
+    if (H % 4 || ld % 4) return set_error(FF_ERR_UNSUPPORTED, "ln_modulate_backward: H and ld must be multiples of 4");
+    const int per = (H / 4 + kThreads - 1) / kThreads;
+    if (per > 8) return set_error(FF_ERR_UNSUPPORTED, "ln_modulate_backward: H=%d > 8192", H);
+    if (s.chunks == 0) return FF_OK;
+    ProfScope prof(stream, "ln_modulate_backward", 0.0, 16.0 * s.rows * H);
+#define FF_LNB(P)                                                                                                   \
+    case P:                                                                                                          \
+        ln_modulate_backward_kernel<P><<<s.chunks, kThreads, 0, stream>>>(x, dh, gx, ld, mods, ld_mods, s, H, part); \
+        break;
+    switch (per) {
+        FF_LNB(1) FF_LNB(2) FF_LNB(3) FF_LNB(4) FF_LNB(5) FF_LNB(6) FF_LNB(7) FF_LNB(8)
+    }
+#undef FF_LNB
+    return check_launch("ln_modulate_backward_kernel");
+}
+
+int qk_norm_rope_backward(const QkBwdArgs& a, int* ctas_txt, int* ctas_img, cudaStream_t stream) {
+    if ((a.head_dim != 64 && a.head_dim != 128) || a.rows_txt < 0 || a.rows < a.rows_txt)
+        return set_error(FF_ERR_UNSUPPORTED, "qk_norm_rope_backward: head_dim %d", a.head_dim);
+    const int ct = (a.rows_txt + kQkRows - 1) / kQkRows;
+    const int ci = (a.rows - a.rows_txt + kQkRows - 1) / kQkRows;
+    *ctas_txt = ct;
+    *ctas_img = ci;
+    if (ct + ci == 0) return FF_OK;
+    ProfScope prof(stream, "qk_norm_rope_backward", 0.0, 12.0 * a.rows * a.heads * a.head_dim);
+    if (a.head_dim == 128) qk_norm_rope_backward_kernel<4><<<ct + ci, kThreads, 0, stream>>>(a, ct);
+    else qk_norm_rope_backward_kernel<2><<<ct + ci, kThreads, 0, stream>>>(a, ct);
+    return check_launch("qk_norm_rope_backward_kernel");
+}
+
+size_t colsum_ws_floats(int rows, int ncols) { return static_cast<size_t>((rows + kBwdChunk - 1) / kBwdChunk) * ncols; }
+
+int colsum(const void* in, bool f32, int64_t ld, int rows, int ncols, float* out, float* ws, cudaStream_t stream) {
+    if (ncols % 4 || ld % 4) return set_error(FF_ERR_UNSUPPORTED, "colsum: ncols and ld must be multiples of 4");
+    if (rows <= 0) return set_error(FF_ERR_INVALID_ARG, "colsum: rows=%d", rows);
+    const int chunks = (rows + kBwdChunk - 1) / kBwdChunk;
+    {
+        ProfScope prof(stream, "colsum", 0.0, static_cast<double>(rows) * ncols * (f32 ? 4 : 2));
+        dim3 grid(chunks, (ncols / 4 + kThreads - 1) / kThreads);
+        if (f32) colsum_partial_kernel<float><<<grid, kThreads, 0, stream>>>(static_cast<const float*>(in), ld, rows, ncols, ws);
+        else colsum_partial_kernel<__nv_bfloat16><<<grid, kThreads, 0, stream>>>(static_cast<const __nv_bfloat16*>(in), ld, rows, ncols, ws);
+        FF_TRY(check_launch("colsum_partial_kernel"));
+    }
+    ChunkSpans sp{};
+    sp.n = 1;
+    sp.first[0] = 0;
+    sp.count[0] = chunks;
+    return reduce(ws, ncols, ncols, sp, 0, out, 0, stream);
+}
+
+int reduce_chunks(const float* part, int64_t ld_part, int ncols, const ChunkSpans& sp, int B, float* out,
+                  int64_t ld_out, cudaStream_t stream) {
+    return reduce(part, ld_part, ncols, sp, B, out, ld_out, stream);
+}
+
+int silu_backward(const float* dy, int64_t ld_dy, const __nv_bfloat16* pre, int B, int rows_pad, int n, float* dx,
+                  __nv_bfloat16* dxb, cudaStream_t stream) {
+    const int total = rows_pad * n;
+    silu_backward_kernel<<<(total + 255) / 256, 256, 0, stream>>>(dy, ld_dy, pre, B, rows_pad, n, dx, dxb);
+    return check_launch("silu_backward_kernel");
+}
+
+}  // namespace ff

@@ -356,7 +356,218 @@ int wan_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, cons
 
 }  // namespace
 
+// The MMDiT velocity: timestep MLP and every adaLN vector, embeddings, the
+// double- and single-stream blocks, the final layer.  Buffers come from f:
+// the inference call passes one shared set (residual updated in place), the
+// training forward one set per block with the pre-activation copies the
+// backward reads.
+int mmdit_forward(const ff_dit* m, int B, const float* x_t, const void* txt, const float* t, float* v_out,
+                  const FwdBufs& f, cudaStream_t stream) {
+    const ff_dit_config& c = m->cfg;
+    const int H = c.hidden, F = c.mlp, P = c.patch_dim;
+    const int Nt = c.n_txt, Ni = c.grid_f * c.grid_h * c.grid_w;
+    const int Rt = B * Nt, Ri = B * Ni, R = Rt + Ri;
+    const int64_t Wm = m->mod_width;
+    auto W = [&](const std::string& n) { return m->w + m->off.at(n); };
+    auto rows = [](auto* p, int64_t r, int64_t ld) { return p ? p + r * ld : p; };
+
+    // ---- rotation table, timestep embedding MLP and every adaLN vector
+    FF_TRY(rope_table(f.rope, c.grid_f, c.grid_h, c.grid_w, c.rope_axes[0], c.rope_axes[1], c.rope_axes[2],
+                      c.rope_theta, stream));
+    FF_TRY(timestep_embed(t, B, c.time_freq_dim, f.temb, stream));
+    {
+        GemmEpilogue e;
+        e.rows_gemv = 1; e.act = ACT_SILU; e.bias = W("t_embed.fc1.b"); e.out0 = f.th; e.ld0 = H;
+        e.aux = f.pre_fc1; e.ld_aux = H;
+        FF_TRY(gemm_bf16(f.temb, c.time_freq_dim, W("t_embed.fc1.w"), c.time_freq_dim, B, H, c.time_freq_dim, e, stream));
+    }
+    {
+        GemmEpilogue e;   // SiLU(c): only the modulation GEMM consumes c
+        e.rows_gemv = 1; e.act = ACT_SILU; e.bias = W("t_embed.fc2.b"); e.out0 = f.tc; e.ld0 = H;
+        e.aux = f.pre_c; e.ld_aux = H;
+        FF_TRY(gemm_bf16(f.th, H, W("t_embed.fc2.w"), H, B, H, H, e, stream));
+    }
+    {
+        GemmEpilogue e;
+        e.rows_gemv = 1; e.out_f32 = 1; e.bias = W("mod.b"); e.out0 = f.mods; e.ld0 = Wm;
+        FF_TRY(gemm_bf16(f.tc, H, W("mod.w"), H, B, static_cast<int>(Wm), H, e, stream));
+    }
+
+    // ---- patch and text embeddings into the residual stream
+    FF_TRY(f32_to_bf16(x_t, f.xb, static_cast<int64_t>(Ri) * P, stream));
+    {
+        // the long-K text product first, so its few expensive tiles start at
+        // once and the short patch-embedding tiles fill in behind them
+        GemmArgs g[2];
+        g[0] = GemmArgs{txt, c.txt_dim, W("txt_in.w"), c.txt_dim, Rt, H, c.txt_dim, GemmEpilogue{}};
+        g[0].epi.out_f32 = 1; g[0].epi.bias = W("txt_in.b"); g[0].epi.out0 = f.x0; g[0].epi.ld0 = H;
+        g[1] = GemmArgs{f.xb, P, W("img_in.w"), P, Ri, H, P, GemmEpilogue{}};
+        g[1].epi.out_f32 = 1; g[1].epi.bias = W("img_in.b"); g[1].epi.out0 = f.x0 + static_cast<int64_t>(Rt) * H;
+        g[1].epi.ld0 = H;
+        FF_TRY(gemm_bf16_group(g, 2, stream));
+    }
+
+    LnModArgs la{};
+    la.ldx = H; la.ldo = H; la.rows = R; la.H = H;
+    la.rows_txt = Rt; la.n_txt = Nt; la.n_img = Ni; la.mods = f.mods; la.ld_mods = Wm;
+
+    struct Stream { const char* name; int row0, rows, tokens; int64_t mod; };
+
+    // ---- double-stream blocks
+    for (int l = 0; l < c.n_double; ++l) {
+        const DitBlockIo io = f.block(l);
+        const int64_t base = static_cast<int64_t>(l) * 12 * H;
+        const Stream st[2] = {{"txt", 0, Rt, Nt, base + 6 * H}, {"img", Rt, Ri, Ni, base}};
+        const std::string pre = "double." + std::to_string(l) + ".";
+        // LN-modulate 1
+        la.x = io.xin; la.out = io.h1;
+        la.shift_txt = static_cast<int>(st[0].mod); la.scale_txt = static_cast<int>(st[0].mod + H);
+        la.shift_img = static_cast<int>(st[1].mod); la.scale_img = static_cast<int>(st[1].mod + H);
+        FF_TRY(ln_modulate(la, stream));
+        // Each GEMM below runs both streams in one launch: image problem
+        // first, the (smaller) text problem filling its tail.
+        const Stream* ord[2] = {&st[1], &st[0]};
+        // QKV, with q / k RMSNorm and RoPE fused into the epilogue
+        {
+            GemmArgs g[2];
+            for (int i = 0; i < 2; ++i) {
+                const Stream& s = *ord[i];
+                const std::string p = pre + s.name + ".";
+                g[i] = GemmArgs{io.h1 + static_cast<int64_t>(s.row0) * H, H, W(p + "qkv.w"), H, s.rows, 3 * H, H,
+                                GemmEpilogue{}};
+                GemmEpilogue& e = g[i].epi;
+                e.bias = W(p + "qkv.b"); e.out0 = io.qkv + static_cast<int64_t>(s.row0) * 3 * H; e.ld0 = 3 * H;
+                e.aux = rows(io.raw, s.row0, 3 * H); e.ld_aux = 3 * H;
+                set_qk_norm(e, c, 2 * H, W(p + "q_norm.scale"), W(p + "k_norm.scale"), s.row0 ? f.rope : nullptr, 0);
+            }
+            FF_TRY(gemm_bf16_group(g, 2, stream));
+        }
+        {
+            AttnSegment a0{io.qkv, 3 * H, io.o, H, Nt};
+            AttnSegment a1{io.qkv + static_cast<int64_t>(Rt) * 3 * H, 3 * H, io.o + static_cast<int64_t>(Rt) * H, H, Ni};
+            FF_TRY(attention(a0, a1, B, c.heads, c.head_dim, H, stream, io.lse));
+        }
+        // projection + gated residual (gate1)
+        {
+            GemmArgs g[2];
+            for (int i = 0; i < 2; ++i) {
+                const Stream& s = *ord[i];
+                const std::string p = pre + s.name + ".";
+                g[i] = GemmArgs{io.o + static_cast<int64_t>(s.row0) * H, H, W(p + "proj.w"), H, s.rows, H, H,
+                                GemmEpilogue{}};
+                GemmEpilogue& e = g[i].epi;
+                e.epi = EPI_GATED_RESIDUAL; e.bias = W(p + "proj.b");
+                e.resid = io.xin + static_cast<int64_t>(s.row0) * H; e.ld_resid = H;
+                if (io.xmid != io.xin) e.resid_out = io.xmid + static_cast<int64_t>(s.row0) * H;
+                e.gate = f.mods + s.mod + 2 * H; e.ld_gate = Wm; e.rows_per_sample = s.tokens;
+                e.aux = rows(io.y1, s.row0, H); e.ld_aux = H;
+            }
+            FF_TRY(gemm_bf16_group(g, 2, stream));
+        }
+        // LN-modulate 2
+        la.x = io.xmid; la.out = io.h2;
+        la.shift_txt = static_cast<int>(st[0].mod + 3 * H); la.scale_txt = static_cast<int>(st[0].mod + 4 * H);
+        la.shift_img = static_cast<int>(st[1].mod + 3 * H); la.scale_img = static_cast<int>(st[1].mod + 4 * H);
+        FF_TRY(ln_modulate(la, stream));
+        // MLP
+        {
+            GemmArgs g[2];
+            for (int i = 0; i < 2; ++i) {
+                const Stream& s = *ord[i];
+                const std::string p = pre + s.name + ".";
+                g[i] = GemmArgs{io.h2 + static_cast<int64_t>(s.row0) * H, H, W(p + "mlp1.w"), H, s.rows, F, H,
+                                GemmEpilogue{}};
+                GemmEpilogue& e = g[i].epi;
+                e.act = ACT_GELU; e.bias = W(p + "mlp1.b"); e.out0 = io.u + static_cast<int64_t>(s.row0) * F; e.ld0 = F;
+                e.aux = rows(io.a1, s.row0, F); e.ld_aux = F;
+            }
+            FF_TRY(gemm_bf16_group(g, 2, stream));
+        }
+        {
+            GemmArgs g[2];
+            for (int i = 0; i < 2; ++i) {
+                const Stream& s = *ord[i];
+                const std::string p = pre + s.name + ".";
+                g[i] = GemmArgs{io.u + static_cast<int64_t>(s.row0) * F, F, W(p + "mlp2.w"), F, s.rows, H, F,
+                                GemmEpilogue{}};
+                GemmEpilogue& e = g[i].epi;
+                e.epi = EPI_GATED_RESIDUAL; e.bias = W(p + "mlp2.b");
+                e.resid = io.xmid + static_cast<int64_t>(s.row0) * H; e.ld_resid = H;
+                if (io.xout != io.xmid) e.resid_out = io.xout + static_cast<int64_t>(s.row0) * H;
+                e.gate = f.mods + s.mod + 5 * H; e.ld_gate = Wm; e.rows_per_sample = s.tokens;
+                e.aux = rows(io.y2, s.row0, H); e.ld_aux = H;
+            }
+            FF_TRY(gemm_bf16_group(g, 2, stream));
+        }
+    }
+
+    // ---- single-stream blocks on the joint sequence
+    for (int l = 0; l < c.n_single; ++l) {
+        const DitBlockIo io = f.block(c.n_double + l);
+        const int64_t off = static_cast<int64_t>(c.n_double) * 12 * H + static_cast<int64_t>(l) * 3 * H;
+        const std::string p = "single." + std::to_string(l) + ".";
+        la.x = io.xin; la.out = io.h1;
+        la.shift_txt = la.shift_img = static_cast<int>(off);
+        la.scale_txt = la.scale_img = static_cast<int>(off + H);
+        FF_TRY(ln_modulate(la, stream));
+        {
+            GemmEpilogue e;   // [q k v] -> qkv ; GELU(mlp) -> u[:, H:]
+            e.bias = W(p + "linear1.b");
+            e.out0 = io.qkv; e.ld0 = 3 * H;
+            e.split_n = 3 * H; e.out1 = io.u; e.ld1 = H + F; e.col1 = H;
+            e.act = ACT_GELU; e.act_from = 3 * H;
+            e.aux = io.raw; e.ld_aux = 3 * H + F;
+            set_qk_norm(e, c, 2 * H, W(p + "q_norm.scale"), W(p + "k_norm.scale"), f.rope, Rt);
+            FF_TRY(gemm_bf16(io.h1, H, W(p + "linear1.w"), H, R, 3 * H + F, H, e, stream));
+        }
+        {
+            AttnSegment a0{io.qkv, 3 * H, io.u, H + F, Nt};
+            AttnSegment a1{io.qkv + static_cast<int64_t>(Rt) * 3 * H, 3 * H, io.u + static_cast<int64_t>(Rt) * (H + F),
+                           H + F, Ni};
+            FF_TRY(attention(a0, a1, B, c.heads, c.head_dim, H, stream, io.lse));
+        }
+        // linear2 + gated residual: one launch, the two segments as two
+        // problems (the sample index of a row differs per segment)
+        {
+            const Stream st[2] = {{"img", Rt, Ri, Ni, off}, {"txt", 0, Rt, Nt, off}};
+            GemmArgs g[2];
+            for (int i = 0; i < 2; ++i) {
+                const Stream& s = st[i];
+                g[i] = GemmArgs{io.u + static_cast<int64_t>(s.row0) * (H + F), H + F, W(p + "linear2.w"), H + F,
+                                s.rows, H, H + F, GemmEpilogue{}};
+                GemmEpilogue& e = g[i].epi;
+                e.epi = EPI_GATED_RESIDUAL; e.bias = W(p + "linear2.b");
+                e.resid = io.xin + static_cast<int64_t>(s.row0) * H; e.ld_resid = H;
+                if (io.xout != io.xin) e.resid_out = io.xout + static_cast<int64_t>(s.row0) * H;
+                e.gate = f.mods + off + 2 * H; e.ld_gate = Wm; e.rows_per_sample = s.tokens;
+                e.aux = rows(io.y2, s.row0, H); e.ld_aux = H;
+            }
+            FF_TRY(gemm_bf16_group(g, 2, stream));
+        }
+    }
+
+    // ---- final layer on image tokens -> v (fp32)
+    {
+        const int64_t off = static_cast<int64_t>(c.n_double) * 12 * H + static_cast<int64_t>(c.n_single) * 3 * H;
+        LnModArgs fl = la;
+        fl.x = f.xfin + static_cast<int64_t>(Rt) * H; fl.rows = Ri; fl.rows_txt = 0; fl.out = f.hf;
+        fl.shift_img = fl.shift_txt = static_cast<int>(off);
+        fl.scale_img = fl.scale_txt = static_cast<int>(off + H);
+        FF_TRY(ln_modulate(fl, stream));
+        GemmEpilogue e;
+        e.out_f32 = 1; e.bias = W("final.b"); e.out0 = v_out; e.ld0 = P;
+        FF_TRY(gemm_bf16(f.hf, H, W("final.w"), H, Ri, P, H, e, stream));
+    }
+    return FF_OK;
+}
+
 const ff_dit_config& model_config(const ff_dit* m) { return m->cfg; }
+const __nv_bfloat16* model_weights(const ff_dit* m) { return m->w; }
+int64_t model_offset(const ff_dit* m, const char* name) {
+    const auto it = m->off.find(name);
+    return it == m->off.end() ? -1 : it->second;
+}
+int64_t model_mod_width(const ff_dit* m) { return m->mod_width; }
 
 }  // namespace ff
 
@@ -432,185 +643,12 @@ int ff_dit_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, c
     if (ws_bytes < w.bytes) return set_error(FF_ERR_WORKSPACE, "workspace %zu B < %zu B needed", ws_bytes, w.bytes);
 
     if (c.arch == FF_ARCH_WAN) return wan_velocity(m, B, x_t, txt, t, v_out, w, stream);
-    const int H = c.hidden, F = c.mlp, P = c.patch_dim, d = c.head_dim;
-    const int Nt = c.n_txt, Ni = c.grid_f * c.grid_h * c.grid_w;
-    const int Rt = B * Nt, Ri = B * Ni, R = Rt + Ri;
-    const int64_t Wm = m->mod_width;
-    auto W = [&](const std::string& n) { return m->w + m->off.at(n); };
-
-    // ---- rotation table, timestep embedding MLP and every adaLN vector
-    FF_TRY(rope_table(w.rope, c.grid_f, c.grid_h, c.grid_w, c.rope_axes[0], c.rope_axes[1], c.rope_axes[2],
-                      c.rope_theta, stream));
-    FF_TRY(timestep_embed(t, B, c.time_freq_dim, w.temb, stream));
-    {
-        GemmEpilogue e;
-        e.rows_gemv = 1; e.act = ACT_SILU; e.bias = W("t_embed.fc1.b"); e.out0 = w.th; e.ld0 = H;
-        FF_TRY(gemm_bf16(w.temb, c.time_freq_dim, W("t_embed.fc1.w"), c.time_freq_dim, B, H, c.time_freq_dim, e, stream));
-    }
-    {
-        GemmEpilogue e;   // SiLU(c): only the modulation GEMM consumes c
-        e.rows_gemv = 1; e.act = ACT_SILU; e.bias = W("t_embed.fc2.b"); e.out0 = w.tc; e.ld0 = H;
-        FF_TRY(gemm_bf16(w.th, H, W("t_embed.fc2.w"), H, B, H, H, e, stream));
-    }
-    {
-        GemmEpilogue e;
-        e.rows_gemv = 1; e.out_f32 = 1; e.bias = W("mod.b"); e.out0 = w.mods; e.ld0 = Wm;
-        FF_TRY(gemm_bf16(w.tc, H, W("mod.w"), H, B, static_cast<int>(Wm), H, e, stream));
-    }
-
-    // ---- patch and text embeddings into the residual stream
-    FF_TRY(f32_to_bf16(x_t, w.xb, static_cast<int64_t>(Ri) * P, stream));
-    {
-        // the long-K text product first, so its few expensive tiles start at
-        // once and the short patch-embedding tiles fill in behind them
-        GemmArgs g[2];
-        g[0] = GemmArgs{txt, c.txt_dim, W("txt_in.w"), c.txt_dim, Rt, H, c.txt_dim, GemmEpilogue{}};
-        g[0].epi.out_f32 = 1; g[0].epi.bias = W("txt_in.b"); g[0].epi.out0 = w.x; g[0].epi.ld0 = H;
-        g[1] = GemmArgs{w.xb, P, W("img_in.w"), P, Ri, H, P, GemmEpilogue{}};
-        g[1].epi.out_f32 = 1; g[1].epi.bias = W("img_in.b"); g[1].epi.out0 = w.x + static_cast<int64_t>(Rt) * H;
-        g[1].epi.ld0 = H;
-        FF_TRY(gemm_bf16_group(g, 2, stream));
-    }
-
-
-    LnModArgs la{};
-    la.x = w.x; la.ldx = H; la.out = w.h; la.ldo = H; la.rows = R; la.H = H;
-    la.rows_txt = Rt; la.n_txt = Nt; la.n_img = Ni; la.mods = w.mods; la.ld_mods = Wm;
-
-    struct Stream { const char* name; int row0, rows, tokens; int64_t mod; };
-
-    // ---- double-stream blocks
-    for (int l = 0; l < c.n_double; ++l) {
-        const int64_t base = static_cast<int64_t>(l) * 12 * H;
-        const Stream st[2] = {{"txt", 0, Rt, Nt, base + 6 * H}, {"img", Rt, Ri, Ni, base}};
-        const std::string pre = "double." + std::to_string(l) + ".";
-        // LN-modulate 1
-        la.shift_txt = static_cast<int>(st[0].mod); la.scale_txt = static_cast<int>(st[0].mod + H);
-        la.shift_img = static_cast<int>(st[1].mod); la.scale_img = static_cast<int>(st[1].mod + H);
-        FF_TRY(ln_modulate(la, stream));
-        // Each GEMM below runs both streams in one launch: image problem
-        // first, the (smaller) text problem filling its tail.
-        const Stream* ord[2] = {&st[1], &st[0]};
-        // QKV, with q / k RMSNorm and RoPE fused into the epilogue
-        {
-            GemmArgs g[2];
-            for (int i = 0; i < 2; ++i) {
-                const Stream& s = *ord[i];
-                const std::string p = pre + s.name + ".";
-                g[i] = GemmArgs{w.h + static_cast<int64_t>(s.row0) * H, H, W(p + "qkv.w"), H, s.rows, 3 * H, H,
-                                GemmEpilogue{}};
-                GemmEpilogue& e = g[i].epi;
-                e.bias = W(p + "qkv.b"); e.out0 = w.qkv + static_cast<int64_t>(s.row0) * 3 * H; e.ld0 = 3 * H;
-                set_qk_norm(e, c, 2 * H, W(p + "q_norm.scale"), W(p + "k_norm.scale"), s.row0 ? w.rope : nullptr, 0);
-            }
-            FF_TRY(gemm_bf16_group(g, 2, stream));
-        }
-        {
-            AttnSegment a0{w.qkv, 3 * H, w.o, H, Nt};
-            AttnSegment a1{w.qkv + static_cast<int64_t>(Rt) * 3 * H, 3 * H, w.o + static_cast<int64_t>(Rt) * H, H, Ni};
-            FF_TRY(attention(a0, a1, B, c.heads, d, H, stream));
-        }
-        // projection + gated residual (gate1)
-        {
-            GemmArgs g[2];
-            for (int i = 0; i < 2; ++i) {
-                const Stream& s = *ord[i];
-                const std::string p = pre + s.name + ".";
-                g[i] = GemmArgs{w.o + static_cast<int64_t>(s.row0) * H, H, W(p + "proj.w"), H, s.rows, H, H,
-                                GemmEpilogue{}};
-                GemmEpilogue& e = g[i].epi;
-                e.epi = EPI_GATED_RESIDUAL; e.bias = W(p + "proj.b");
-                e.resid = w.x + static_cast<int64_t>(s.row0) * H; e.ld_resid = H;
-                e.gate = w.mods + s.mod + 2 * H; e.ld_gate = Wm; e.rows_per_sample = s.tokens;
-            }
-            FF_TRY(gemm_bf16_group(g, 2, stream));
-        }
-        // LN-modulate 2
-        la.shift_txt = static_cast<int>(st[0].mod + 3 * H); la.scale_txt = static_cast<int>(st[0].mod + 4 * H);
-        la.shift_img = static_cast<int>(st[1].mod + 3 * H); la.scale_img = static_cast<int>(st[1].mod + 4 * H);
-        FF_TRY(ln_modulate(la, stream));
-        // MLP
-        {
-            GemmArgs g[2];
-            for (int i = 0; i < 2; ++i) {
-                const Stream& s = *ord[i];
-                const std::string p = pre + s.name + ".";
-                g[i] = GemmArgs{w.h + static_cast<int64_t>(s.row0) * H, H, W(p + "mlp1.w"), H, s.rows, F, H,
-                                GemmEpilogue{}};
-                GemmEpilogue& e = g[i].epi;
-                e.act = ACT_GELU; e.bias = W(p + "mlp1.b"); e.out0 = w.u + static_cast<int64_t>(s.row0) * F; e.ld0 = F;
-            }
-            FF_TRY(gemm_bf16_group(g, 2, stream));
-        }
-        {
-            GemmArgs g[2];
-            for (int i = 0; i < 2; ++i) {
-                const Stream& s = *ord[i];
-                const std::string p = pre + s.name + ".";
-                g[i] = GemmArgs{w.u + static_cast<int64_t>(s.row0) * F, F, W(p + "mlp2.w"), F, s.rows, H, F,
-                                GemmEpilogue{}};
-                GemmEpilogue& e = g[i].epi;
-                e.epi = EPI_GATED_RESIDUAL; e.bias = W(p + "mlp2.b");
-                e.resid = w.x + static_cast<int64_t>(s.row0) * H; e.ld_resid = H;
-                e.gate = w.mods + s.mod + 5 * H; e.ld_gate = Wm; e.rows_per_sample = s.tokens;
-            }
-            FF_TRY(gemm_bf16_group(g, 2, stream));
-        }
-    }
-
-    // ---- single-stream blocks on the joint sequence
-    for (int l = 0; l < c.n_single; ++l) {
-        const int64_t off = static_cast<int64_t>(c.n_double) * 12 * H + static_cast<int64_t>(l) * 3 * H;
-        const std::string p = "single." + std::to_string(l) + ".";
-        la.shift_txt = la.shift_img = static_cast<int>(off);
-        la.scale_txt = la.scale_img = static_cast<int>(off + H);
-        FF_TRY(ln_modulate(la, stream));
-        {
-            GemmEpilogue e;   // [q k v] -> qkv ; GELU(mlp) -> u[:, H:]
-            e.bias = W(p + "linear1.b");
-            e.out0 = w.qkv; e.ld0 = 3 * H;
-            e.split_n = 3 * H; e.out1 = w.u; e.ld1 = H + F; e.col1 = H;
-            e.act = ACT_GELU; e.act_from = 3 * H;
-            set_qk_norm(e, c, 2 * H, W(p + "q_norm.scale"), W(p + "k_norm.scale"), w.rope, Rt);
-            FF_TRY(gemm_bf16(w.h, H, W(p + "linear1.w"), H, R, 3 * H + F, H, e, stream));
-        }
-        {
-            AttnSegment a0{w.qkv, 3 * H, w.u, H + F, Nt};
-            AttnSegment a1{w.qkv + static_cast<int64_t>(Rt) * 3 * H, 3 * H, w.u + static_cast<int64_t>(Rt) * (H + F),
-                           H + F, Ni};
-            FF_TRY(attention(a0, a1, B, c.heads, d, H, stream));
-        }
-        // linear2 + gated residual: one launch, the two segments as two
-        // problems (the sample index of a row differs per segment)
-        {
-            const Stream st[2] = {{"img", Rt, Ri, Ni, off}, {"txt", 0, Rt, Nt, off}};
-            GemmArgs g[2];
-            for (int i = 0; i < 2; ++i) {
-                const Stream& s = st[i];
-                g[i] = GemmArgs{w.u + static_cast<int64_t>(s.row0) * (H + F), H + F, W(p + "linear2.w"), H + F,
-                                s.rows, H, H + F, GemmEpilogue{}};
-                GemmEpilogue& e = g[i].epi;
-                e.epi = EPI_GATED_RESIDUAL; e.bias = W(p + "linear2.b");
-                e.resid = w.x + static_cast<int64_t>(s.row0) * H; e.ld_resid = H;
-                e.gate = w.mods + off + 2 * H; e.ld_gate = Wm; e.rows_per_sample = s.tokens;
-            }
-            FF_TRY(gemm_bf16_group(g, 2, stream));
-        }
-    }
-
-    // ---- final layer on image tokens -> v (fp32)
-    {
-        const int64_t off = static_cast<int64_t>(c.n_double) * 12 * H + static_cast<int64_t>(c.n_single) * 3 * H;
-        LnModArgs f = la;
-        f.x = w.x + static_cast<int64_t>(Rt) * H; f.rows = Ri; f.rows_txt = 0;
-        f.shift_img = f.shift_txt = static_cast<int>(off);
-        f.scale_img = f.scale_txt = static_cast<int>(off + H);
-        FF_TRY(ln_modulate(f, stream));
-        GemmEpilogue e;
-        e.out_f32 = 1; e.bias = W("final.b"); e.out0 = v_out; e.ld0 = P;
-        FF_TRY(gemm_bf16(w.h, H, W("final.w"), H, Ri, P, H, e, stream));
-    }
-    return FF_OK;
+    FwdBufs f{};
+    f.mods = w.mods; f.temb = w.temb; f.th = w.th; f.tc = w.tc; f.xb = w.xb; f.rope = w.rope;
+    f.x0 = f.xfin = w.x;
+    f.hf = w.h;
+    f.shared = DitBlockIo{w.x, w.x, w.x, w.h, w.qkv, nullptr, w.o, nullptr, w.h, nullptr, w.u, nullptr, nullptr};
+    return mmdit_forward(m, B, x_t, txt, t, v_out, f, stream);
 }
 
 }  // extern "C"

@@ -70,6 +70,29 @@ __device__ __forceinline__ void bias_add8(float* v, const __nv_bfloat16* b) {
     }
 }
 
+// 32 consecutive values of one row as bf16 (four 16-byte stores), and back.
+__device__ __forceinline__ void store_bf16x32(__nv_bfloat16* p, const float* v) {
+    uint4* o = reinterpret_cast<uint4*>(p);
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+        o[j] = make_uint4(pack_bf16x2(v[8 * j], v[8 * j + 1]), pack_bf16x2(v[8 * j + 2], v[8 * j + 3]),
+                          pack_bf16x2(v[8 * j + 4], v[8 * j + 5]), pack_bf16x2(v[8 * j + 6], v[8 * j + 7]));
+}
+__device__ __forceinline__ void load_bf16x32(const __nv_bfloat16* p, float* v) {
+    const uint4* s = reinterpret_cast<const uint4*>(p);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        const uint4 u = s[j];
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float2 f = unpack_bf16x2(w[i]);
+            v[8 * j + 2 * i] = f.x;
+            v[8 * j + 2 * i + 1] = f.y;
+        }
+    }
+}
+
 // Gated residual, one 32-column chunk: x[row, n..n+31] += gate[b(row), n..] *
 // (acc + bias).  The residual chunk of the whole 128-row tile sits in shared
 // memory (loaded by TMA with 128-byte swizzle, 16-byte piece j of row r at
@@ -138,6 +161,7 @@ __device__ __forceinline__ void qk_norm_tile(const GemmEpilogue& e, int M, int r
 #pragma unroll
                 for (int j = 0; j < 4; ++j) bias_add8(v + 8 * j, e.bias + col + c + 8 * j);
             }
+            if (e.aux && row < M) store_bf16x32(e.aux + static_cast<int64_t>(row) * e.ld_aux + col + c, v);
 #pragma unroll
             for (int i = 0; i < 32; ++i) ss = fmaf(v[i], v[i], ss);
         }
@@ -196,8 +220,10 @@ __device__ __forceinline__ void load_bias32(const __nv_bfloat16* bias, int n, ui
     for (int j = 0; j < 4; ++j) u[j] = bias ? reinterpret_cast<const uint4*>(bias + n)[j] : make_uint4(0, 0, 0, 0);
 }
 
-// Bias and activation of one 32-column chunk of the row held by this thread.
-__device__ __forceinline__ void epilogue_values(const GemmEpilogue& e, int n, const uint4 (&bu)[4], float (&v)[32]) {
+// Bias and activation of one 32-column chunk of the row held by this thread
+// (plus the optional pre-activation copy and activation-derivative factor).
+__device__ __forceinline__ void epilogue_values(const GemmEpilogue& e, int row, int M, int n, const uint4 (&bu)[4],
+                                                float (&v)[32]) {
     if (e.bias) {
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
@@ -209,6 +235,13 @@ __device__ __forceinline__ void epilogue_values(const GemmEpilogue& e, int n, co
                 v[8 * j + 2 * i + 1] += f.y;
             }
         }
+    }
+    if (e.aux && row < M) store_bf16x32(e.aux + static_cast<int64_t>(row) * e.ld_aux + n, v);
+    if (e.gelu_pre && n >= e.act_from && row < M) {
+        float pre[32];
+        load_bf16x32(e.gelu_pre + static_cast<int64_t>(row) * e.ld_pre + (n - e.act_from), pre);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] *= gelu_tanh_grad(pre[i]);
     }
     if (e.act != ACT_NONE && n >= e.act_from) {
         if (e.act == ACT_GELU) {
@@ -288,6 +321,7 @@ __device__ __forceinline__ bool epilogue_tile(const GemmEpilogue& epi, int M, in
 #pragma unroll
                 for (int j = 0; j < 4; ++j) bias_add8(v + 8 * j, epi.bias + n + 8 * j);
             }
+            if (epi.aux && row < M) store_bf16x32(epi.aux + static_cast<int64_t>(row) * epi.ld_aux + n, v);
             if (!mbar_wait(&rfull_bar[b], ruse[b] & 1)) {
                 report_status(status, kStatusWaitTimeout);
                 *abort_flag = 1;
@@ -306,7 +340,7 @@ __device__ __forceinline__ bool epilogue_tile(const GemmEpilogue& epi, int M, in
             }
             ++ruse[b];
             if (leader && ok) {
-                tma_store_2d(tr, rbuf + b * C::kResidBytes, n, m0);
+                tma_store_2d(&to[0], rbuf + b * C::kResidBytes, n, m0);
                 bulk_commit();
                 if (c + 2 < c_end) {
                     bulk_wait_read<0>();
@@ -358,7 +392,8 @@ __device__ __forceinline__ bool epilogue_tile(const GemmEpilogue& epi, int M, in
 #pragma unroll
             for (int k = 0; k < CW / 32; ++k)
                 if (k < nblk)
-                    epilogue_values(epi, nb * BN + c + 32 * k, *reinterpret_cast<const uint4(*)[4]>(&bcur[4 * k]),
+                    epilogue_values(epi, row, M, nb * BN + c + 32 * k,
+                                    *reinterpret_cast<const uint4(*)[4]>(&bcur[4 * k]),
                                     *reinterpret_cast<float(*)[32]>(&v[32 * k]));
             if (lane == 0) bulk_wait_read<NB - 1>();
             __syncwarp();
@@ -830,7 +865,8 @@ gemm_pair_kernel(const __grid_constant__ CUtensorMap tm_a0, const __grid_constan
 int make_out_maps(const GemmArgs& a, CUtensorMap* m) {
     const GemmEpilogue& e = a.epi;
     if (e.epi == EPI_GATED_RESIDUAL) {
-        const int rc = make_tmap_f32_sw128(&m[0], e.resid, a.M, a.N, e.ld_resid, 128);
+        // the updated residual's store map (the input's when updated in place)
+        const int rc = make_tmap_f32_sw128(&m[0], e.resid_out ? e.resid_out : e.resid, a.M, a.N, e.ld_resid, 128);
         m[1] = m[0];
         return rc;
     }
@@ -1031,6 +1067,7 @@ __global__ void __launch_bounds__(kGemvThreads) gemv_rows_kernel(const __nv_bflo
                     for (int mm = 0; mm < MR; ++mm)
                         if (jj == j && mm == m) v = acc[jj][mm];
                 if (e.bias) v += __bfloat162float(e.bias[n]);
+                if (e.aux) e.aux[static_cast<int64_t>(m) * e.ld_aux + n] = __float2bfloat16_rn(v);
                 if (e.act != ACT_NONE && n >= e.act_from) v = e.act == ACT_GELU ? gelu_tanh(v) : silu(v);
                 if (e.out_f32)
                     static_cast<float*>(e.out0)[static_cast<int64_t>(m) * e.ld0 + n] = v;
@@ -1068,6 +1105,7 @@ int launch_gemv_rows(const GemmArgs& a, cudaStream_t stream) {
         p.A = static_cast<const __nv_bfloat16*>(a.A) + static_cast<int64_t>(m0) * a.lda;
         p.epi.out0 = a.epi.out_f32 ? static_cast<void*>(static_cast<float*>(a.epi.out0) + m0 * a.epi.ld0)
                                    : static_cast<void*>(static_cast<__nv_bfloat16*>(a.epi.out0) + m0 * a.epi.ld0);
+        if (a.epi.aux) p.epi.aux = a.epi.aux + m0 * a.epi.ld_aux;
         int rc;
         if (p.M <= 1) rc = launch_gemv<1>(p, stream);
         else if (p.M <= 2) rc = launch_gemv<2>(p, stream);
@@ -1090,7 +1128,7 @@ int check_args(const GemmArgs& a) {
     if (e.bias && !aligned16(e.bias)) return set_error(FF_ERR_INVALID_ARG, "gemm: bias not 16-byte aligned");
     if (e.epi == EPI_GATED_RESIDUAL) {
         if (!e.resid || e.rows_per_sample <= 0 || !aligned16(e.resid) || (e.gate && !aligned16(e.gate)) ||
-            e.ld_resid % 4 || e.ld_gate % 4)
+            (e.resid_out && !aligned16(e.resid_out)) || e.ld_resid % 4 || e.ld_gate % 4)
             return set_error(FF_ERR_INVALID_ARG, "gemm: bad gated-residual epilogue");
     } else {
         if (!e.out0 || !aligned16(e.out0)) return set_error(FF_ERR_INVALID_ARG, "gemm: bad output");
@@ -1102,6 +1140,11 @@ int check_args(const GemmArgs& a) {
         }
     }
     if (e.act != ACT_NONE && e.act_from % 32) return set_error(FF_ERR_INVALID_ARG, "gemm: act_from % 32 != 0");
+    if (e.aux && (!aligned16(e.aux) || e.ld_aux % 8 || e.ld_aux < N))
+        return set_error(FF_ERR_INVALID_ARG, "gemm: bad pre-activation copy");
+    if (e.gelu_pre && (!aligned16(e.gelu_pre) || e.ld_pre % 8 || e.act_from % 32 || e.act != ACT_NONE ||
+                       e.epi != EPI_STORE || e.qk_cols > 0 || e.ld_pre < N - e.act_from))
+        return set_error(FF_ERR_INVALID_ARG, "gemm: bad activation-backward epilogue");
     if (e.qk_cols > 0) {
         // whole heads per 256-wide tile: head_dim | 256 and qk_cols | 256
         if (e.epi != EPI_STORE || e.out_f32 || (e.head_dim != 64 && e.head_dim != 128) || e.qk_cols % 256 ||
@@ -1154,7 +1197,7 @@ int gemm_bf16_group(const GemmArgs* p, int n, cudaStream_t stream) {
     }
     const GemmArgs& a = p[0];
     const bool gemv_ok = !a.a_mn && !a.b_mn && a.K <= kGemvMaxK && a.epi.epi == EPI_STORE && a.epi.split_n >= a.N &&
-                         a.epi.qk_cols == 0 &&
+                         a.epi.qk_cols == 0 && !a.epi.gelu_pre &&
                          aligned16(a.A) && aligned16(a.B) && a.lda % 8 == 0 && a.ldb % 8 == 0;
     if (a.epi.rows_gemv && !gemv_ok) return set_error(FF_ERR_UNSUPPORTED, "gemm: rows_gemv needs K <= 8192 and a plain store");
     if (gemv_ok && (a.epi.rows_gemv || a.M <= kGemvMaxRows)) return launch_gemv_rows(a, stream);

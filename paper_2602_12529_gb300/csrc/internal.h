@@ -27,8 +27,13 @@ inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 
         if (rc_ != FF_OK) return rc_; \
     } while (0)
 
-// Configuration of a DiT handle (its struct is private to dit.cu).
+// Configuration, weights, parameter offsets (elements into the weight blob,
+// -1 if absent) and modulation width of a DiT handle (its struct is private
+// to dit.cu).
 const ff_dit_config& model_config(const ff_dit* m);
+const __nv_bfloat16* model_weights(const ff_dit* m);
+int64_t model_offset(const ff_dit* m, const char* name);
+int64_t model_mod_width(const ff_dit* m);
 
 // ---- optional launch timing (ff_prof_*): RAII scope around one launch ----
 struct ProfScope {
@@ -68,6 +73,7 @@ struct GemmEpilogue {
     // gate == nullptr means a plain residual update (gate 1)
     float* resid = nullptr;
     int64_t ld_resid = 0;
+    float* resid_out = nullptr;        // updated residual written here (same ld) instead of in place
     const float* gate = nullptr;
     int64_t ld_gate = 0;
     int rows_per_sample = 1;
@@ -88,6 +94,17 @@ struct GemmEpilogue {
     const float2* rope_cs = nullptr;   // null: no rotation at all
     int rope_row0 = 0, n_img = 1, grid_f = 1, grid_h = 1, grid_w = 1;
     int axes0 = 0, axes1 = 0, axes2 = 0;
+    // Pre-activation copy for the training forward: when aux is set, every
+    // column n of acc + bias is also stored as bf16 at aux[row * ld_aux + n]
+    // before the activation, the QK norm or the gate is applied.
+    __nv_bfloat16* aux = nullptr;
+    int64_t ld_aux = 0;
+    // Activation backward for input-gradient products: when gelu_pre is set,
+    // columns n >= act_from of the product are multiplied by
+    // GELU'(gelu_pre[row * ld_pre + n - act_from]), the forward's
+    // pre-activation values (EPI_STORE, no activation).
+    const __nv_bfloat16* gelu_pre = nullptr;
+    int64_t ld_pre = 0;
 };
 
 // cos / sin of every (axis, position, pair) rotation angle pos * theta^(-2j/a):
@@ -154,7 +171,7 @@ struct AttnSegment {
     int n;                                 // tokens per sample in this segment
 };
 int attention(const AttnSegment& s0, const AttnSegment& s1, int B, int heads, int head_dim, int H,
-              cudaStream_t stream);
+              cudaStream_t stream, float* lse = nullptr);
 
 // General form: queries from up to two query segments, keys/values from up
 // to two key/value segments (concatenated per sample), head h of q / k / v
@@ -184,14 +201,71 @@ int attention_general(const AttnSpec& a, cudaStream_t stream);
 struct AttnBwdSeg {
     const __nv_bfloat16* qkv; int64_t ld;   // q, k, v at columns 0, H, 2H
     const __nv_bfloat16* o;                  // forward output, row pitch ldo
-    const __nv_bfloat16* dout;               // its gradient, row pitch ldo
+    const __nv_bfloat16* dout;               // its gradient, row pitch ldg (ldo when ldg = 0)
     int64_t ldo;
     __nv_bfloat16* dqkv; int64_t ldd;        // dq, dk, dv at columns 0, H, 2H
     int n;
+    int64_t ldg = 0;
 };
 size_t attention_backward_ws_bytes(int B, int heads, int n0, int n1);
 int attention_backward(const AttnBwdSeg& s0, const AttnBwdSeg& s1, int B, int heads, int head_dim,
                        const float* lse, void* ws, size_t ws_bytes, cudaStream_t stream);
+
+// ---- DiT backward row / column kernels (backward.cu) ----------------------
+// A segment is one stream's rows [row0, row0 + B * tokens), sample b at
+// row0 + b * tokens; col_a / col_b are the mods columns of the vectors the
+// kernel reads (gate_backward: gate at col_a; ln_modulate_backward: scale at
+// col_b).  Kernels over segments cut each sample's rows into chunks of
+// kBwdChunk rows (a chunk never straddles samples) and write one row of
+// partial column sums per chunk: chunk index = first[seg] + b * chunks(seg) + k.
+constexpr int kBwdChunk = 32;
+__host__ __device__ inline int bwd_chunks(int tokens) { return (tokens + kBwdChunk - 1) / kBwdChunk; }
+struct BwdSeg { int row0, tokens, col_a, col_b; };
+struct BwdSegs {
+    BwdSeg seg[2];
+    int first[2];
+    int n, B, chunks;
+    int64_t rows;
+};
+BwdSegs bwd_segs(const BwdSeg* segs, int n, int B);
+// Spans of chunk partials to add up: span i covers chunks [first, first + count)
+// (all samples), or with a per-sample reduction sample b's chunks
+// [first + b * count, first + (b + 1) * count).
+struct ChunkSpans { int first[2], count[2], n; };
+
+// Through x' = x + gate y: dy = bf16(g gate); part[c * 2H + j] = sum g y,
+// part[c * 2H + H + j] = sum g gate over chunk c's rows.  g, y, dy share ld.
+int gate_backward(const float* g, const __nv_bfloat16* y, int64_t ld, const float* mods, int64_t ld_mods,
+                  const BwdSegs& s, int H, __nv_bfloat16* dy, float* part, cudaStream_t stream);
+// Through h = LN(x) (1 + scale) + shift: gx += dx; part[c * 2H + j] = sum dh,
+// part[c * 2H + H + j] = sum dh n (n = LN(x)).  x, dh, gx share ld.
+int ln_modulate_backward(const float* x, const float* dh, float* gx, int64_t ld, const float* mods, int64_t ld_mods,
+                         const BwdSegs& s, int H, float* part, cudaStream_t stream);
+// Through q = rope(RMSNorm(q_raw) w) for the q (columns [0, H)) and k
+// (columns [H, 2H)) gradients in d, in place; rows >= rows_txt are image
+// tokens (rotated with the cos / sin table, as the forward epilogue does).
+// part[cta * 2d + j] (q scale) and part[cta * 2d + d + j] (k scale): the
+// first ctas_txt CTAs cover text rows, the next ctas_img image rows.
+struct QkBwdArgs {
+    __nv_bfloat16* d; int64_t ldd;
+    const __nv_bfloat16* raw; int64_t ldr;
+    int rows_txt, rows, heads, head_dim;
+    const __nv_bfloat16 *q_scale_txt, *k_scale_txt, *q_scale_img, *k_scale_img;
+    const float2* rope_cs;
+    int n_img, grid_f, grid_h, grid_w, axes0, axes1, axes2;
+    float* part;
+};
+int qk_norm_rope_backward(const QkBwdArgs& a, int* ctas_txt, int* ctas_img, cudaStream_t stream);
+constexpr int kQkBwdRows = 16;   // rows per CTA of qk_norm_rope_backward
+// out[j] = sum over rows of in[r * ld + j] (bf16 or fp32), via ws partials.
+size_t colsum_ws_floats(int rows, int ncols);
+int colsum(const void* in, bool f32, int64_t ld, int rows, int ncols, float* out, float* ws, cudaStream_t stream);
+// B > 0: out[b * ld_out + j] per sample; B == 0: out[j] over every chunk.
+int reduce_chunks(const float* part, int64_t ld_part, int ncols, const ChunkSpans& sp, int B, float* out,
+                  int64_t ld_out, cudaStream_t stream);
+// dx = dy SiLU'(pre) (rows < B; fp32 [B, n]) and its bf16 copy [rows_pad, n], zero-padded.
+int silu_backward(const float* dy, int64_t ld_dy, const __nv_bfloat16* pre, int B, int rows_pad, int n, float* dx,
+                  __nv_bfloat16* dxb, cudaStream_t stream);
 
 // mods[b, l*6H + j] = e0[b, j] + bias_l[j] (bias_l = bias0 + l*stride), and
 // mods[b, L*6H + j] = e[b, j % H] + fbias[j] for j < 2H (WAN modulation).
@@ -199,6 +273,33 @@ int wan_modulation(const float* e, const float* e0, const __nv_bfloat16* bias0, 
                    const __nv_bfloat16* fbias, int B, int H, float* mods, int64_t ld_mods, cudaStream_t stream);
 
 int timestep_embed(const float* t, int B, int dim, __nv_bfloat16* out, cudaStream_t stream);
+
+// ---- the MMDiT forward over caller-chosen buffers (dit.cu) ----------------
+// One block's activations: residual before the block, after its attention
+// half (double-stream blocks) and after it; LN-modulate outputs h1 / h2;
+// normalised and rotated q | k | v; the attention output o (single-stream
+// blocks: u holds [o | GELU(mlp)]); the MLP hidden u.  The pre-activation
+// copies (raw = QKV or linear1 product + bias, y1 / y2 = gated branches
+// before the gate, a1 = MLP1 before GELU) and the attention log-sum-exp are
+// written only when set.
+struct DitBlockIo {
+    float *xin, *xmid, *xout;
+    __nv_bfloat16 *h1, *qkv, *raw, *o, *y1, *h2, *a1, *u, *y2;
+    float* lse;
+};
+struct FwdBufs {
+    float* mods;
+    __nv_bfloat16 *temb, *th, *tc, *pre_fc1, *pre_c, *xb;
+    float2* rope;
+    float* x0;              // residual after the embeddings
+    float* xfin;            // residual after the last block
+    __nv_bfloat16* hf;      // final LN-modulate output
+    DitBlockIo shared;      // every block's buffers when blocks is null
+    const DitBlockIo* blocks;
+    DitBlockIo block(int l) const { return blocks ? blocks[l] : shared; }
+};
+int mmdit_forward(const ff_dit* m, int B, const float* x_t, const void* txt, const float* t, float* v_out,
+                  const FwdBufs& f, cudaStream_t stream);
 int f32_to_bf16(const float* in, __nv_bfloat16* out, int64_t n, cudaStream_t stream);
 
 }  // namespace ff

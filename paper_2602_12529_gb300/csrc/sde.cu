@@ -136,6 +136,51 @@ __global__ void __launch_bounds__(kThreads) sde_logprob_finalize_kernel(int64_t 
     }
 }
 
+// Backward of the log-probability in v with x_next held fixed:
+// d logp / d v_j = (x_next_j - mean_j) / std^2 * cv (divided by D for the
+// mean reduction), times the upstream gradient g[b * ldg].  Zero where
+// std = 0 (no density, logp reported as 0).  Same mean arithmetic as the
+// forward kernel.
+__global__ void __launch_bounds__(kThreads) sde_logprob_backward_kernel(int64_t D, int nblk, const float* x,
+                                                                        const float* v, const float* x_next,
+                                                                        const float* t, const float* t_next,
+                                                                        const float* sigma, const float* g, int ldg,
+                                                                        int reduce, float* dv) {
+    __shared__ float3 coef;
+    const int b = blockIdx.y;
+    if (threadIdx.x == 0) {
+        const StepCoef c = step_coef(t, t_next, sigma, b);
+        const double sd = static_cast<double>(c.std);
+        double k = 0.0;
+        if (sd > 0.0) {
+            const double delta = static_cast<double>(t[b]) - static_cast<double>(t_next[b]);
+            const double sg = sigma[b];
+            const double var = sg * sg * delta;
+            k = static_cast<double>(g[static_cast<int64_t>(b) * ldg]) * static_cast<double>(c.cv) / var;
+            if (reduce == FF_LP_MEAN) k /= static_cast<double>(D);
+        }
+        coef = make_float3(c.cx, c.cv, static_cast<float>(k));
+    }
+    __syncthreads();
+    const float3 c = coef;
+    const int64_t row = static_cast<int64_t>(b) * D;
+    const float4* x4 = reinterpret_cast<const float4*>(x + row);
+    const float4* v4 = reinterpret_cast<const float4*>(v + row);
+    const float4* n4 = reinterpret_cast<const float4*>(x_next + row);
+    float4* d4 = reinterpret_cast<float4*>(dv + row);
+    const int64_t nvec = D >> 2;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; i < nvec;
+         i += static_cast<int64_t>(nblk) * kThreads) {
+        const float4 xv = __ldcs(x4 + i), vv = __ldcs(v4 + i), nv = __ldcs(n4 + i);
+        float4 o;
+        o.x = c.z * (nv.x - fmaf(c.x, xv.x, c.y * vv.x));
+        o.y = c.z * (nv.y - fmaf(c.x, xv.y, c.y * vv.y));
+        o.z = c.z * (nv.z - fmaf(c.x, xv.z, c.y * vv.z));
+        o.w = c.z * (nv.w - fmaf(c.x, xv.w, c.y * vv.w));
+        __stcs(d4 + i, o);
+    }
+}
+
 constexpr int kMaxBlocksPerSample = 1024;
 
 // partial sums (blocks) per sample: one per 4096-element chunk up to 1024,
@@ -194,6 +239,30 @@ int ff_sde_step_logprob(int B, int64_t D, const float* x_t, const float* v, cons
 }
 
 }  // extern "C"
+
+extern "C" int ff_sde_logprob_backward(int B, int64_t D, const float* x_t, const float* v, const float* x_next,
+                                       const float* t, const float* t_next, const float* sigma, int reduce,
+                                       const float* grad_logp, int ld, float* grad_v, cudaStream_t stream) {
+    using namespace ff;
+    if (B <= 0 || D <= 0) return set_error(FF_ERR_INVALID_ARG, "sde backward: B=%d D=%lld must be positive", B, (long long)D);
+    if (D % 4) return set_error(FF_ERR_UNSUPPORTED, "sde backward: D=%lld not a multiple of 4", (long long)D);
+    if (reduce != FF_LP_SUM && reduce != FF_LP_MEAN) return set_error(FF_ERR_INVALID_ARG, "sde backward: bad reduce %d", reduce);
+    if (!x_t || !v || !x_next || !t || !t_next || !sigma || !grad_logp || !grad_v)
+        return set_error(FF_ERR_INVALID_ARG, "sde backward: null pointer");
+    if (!aligned16(x_t) || !aligned16(v) || !aligned16(x_next) || !aligned16(grad_v))
+        return set_error(FF_ERR_INVALID_ARG, "sde backward: arrays must be 16-byte aligned");
+    if (ld < 1) return set_error(FF_ERR_INVALID_ARG, "sde backward: ld=%d < 1", ld);
+    if (B > 65535) return set_error(FF_ERR_UNSUPPORTED, "sde backward: B=%d > 65535", B);
+    const int64_t nvec = D / 4;
+    int64_t nb = (nvec + kThreads * 4 - 1) / (kThreads * 4);   // about four float4 per thread
+    const int64_t cap = (4 * static_cast<int64_t>(num_sms()) + B - 1) / B;
+    if (nb > cap) nb = cap;
+    if (nb < 1) nb = 1;
+    ProfScope prof(stream, "sde_logprob_backward", 0.0, static_cast<double>(B) * D * 16.0);
+    sde_logprob_backward_kernel<<<dim3(static_cast<unsigned>(nb), B), kThreads, 0, stream>>>(
+        D, static_cast<int>(nb), x_t, v, x_next, t, t_next, sigma, grad_logp, ld, reduce, grad_v);
+    return check_launch("sde_logprob_backward_kernel");
+}
 
 extern "C" int ff_sde_schedule(int kind, int n_steps, double shift, double eta, double t_clamp, double* t_out,
                                double* sigma_out) {

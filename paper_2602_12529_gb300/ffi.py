@@ -78,6 +78,10 @@ _SIGS = {
     "ff_dit_workspace_size": ([_P, _I, C.POINTER(_SZ)], _I),
     "ff_dit_velocity": ([_P, _I, _P, _P, _P, _P, _P, _SZ, _P], _I),
     "ff_rollout_workspace_size": ([_P, _I, _I, C.POINTER(_SZ)], _I),
+    "ff_dit_train_workspace_size": ([_P, _I, C.POINTER(_SZ)], _I),
+    "ff_dit_forward_train": ([_P, _I, _P, _P, _P, _P, _P, _SZ, _P], _I),
+    "ff_dit_backward": ([_P, _I, _P, _P, _P, _P, _P, _SZ, _P], _I),
+    "ff_sde_logprob_backward": ([_I, _I64, _P, _P, _P, _P, _P, _P, _I, _P, _I, _P, _P], _I),
     "ff_gemm": ([_I, _I, _I, _P, _I64, _I, _P, _I64, _I, _P, _I, _I, _P, _I64, _P], _I),
     "ff_attention_lse_rows": ([_I, _I], _I),
     "ff_attention_forward": ([_I, _I, _I, _I, _P, _I64, _P, _I64, _I, _P, _I64, _P, _I64, _P, _P], _I),
@@ -245,6 +249,19 @@ def ff_sde_step_logprob_noalloc(x_t, v, eps, x_next, t, t_next, sigma, logp, mod
           _ptr(sigma), mode, reduce, _ptr(logp), ld, _stream(stream))
 
 
+def ff_sde_logprob_backward(x_t, v, x_next, t, t_next, sigma, grad_logp, grad_v, reduce=FF_LP_SUM, ld: int = 1,
+                            stream=None):
+    """grad_v = d logp / d v (x_next fixed) times grad_logp[b * ld]."""
+    import torch
+    for n_, a in (("x_t", x_t), ("v", v), ("x_next", x_next), ("t", t), ("t_next", t_next), ("sigma", sigma),
+                  ("grad_logp", grad_logp), ("grad_v", grad_v)):
+        _check(a, torch.float32, n_)
+    B = x_t.shape[0]
+    D = x_t.numel() // B
+    _call("ff_sde_logprob_backward", B, D, _ptr(x_t), _ptr(v), _ptr(x_next), _ptr(t), _ptr(t_next), _ptr(sigma),
+          reduce, _ptr(grad_logp), ld, _ptr(grad_v), _stream(stream))
+
+
 def ff_group_advantage(rewards, G: int, eps_A: float, adv, stream=None):
     import torch
     _check(rewards, torch.float32, "rewards")
@@ -360,6 +377,33 @@ class Dit:
         _check(v_out, torch.float32, "v_out")
         B = x_t.shape[0]
         _call("ff_dit_velocity", self._h, B, _ptr(x_t), _ptr(txt), _ptr(t), _ptr(v_out), _ptr(ws), ws.numel(),
+              _stream(stream))
+
+    def train_workspace_size(self, B: int) -> int:
+        n = _SZ()
+        _call("ff_dit_train_workspace_size", self._h, B, C.byref(n))
+        return n.value
+
+    def ff_dit_forward_train(self, x_t, txt, t, v_out, ws, stream=None):
+        import torch
+        _check(x_t, torch.float32, "x_t")
+        _check(txt, torch.bfloat16, "txt")
+        _check(t, torch.float32, "t")
+        _check(v_out, torch.float32, "v_out")
+        B = x_t.shape[0]
+        _call("ff_dit_forward_train", self._h, B, _ptr(x_t), _ptr(txt), _ptr(t), _ptr(v_out), _ptr(ws), ws.numel(),
+              _stream(stream))
+
+    def ff_dit_backward(self, txt, dv, grad, ws, dx_t=None, stream=None):
+        """grad: fp32 blob of the weight layout's total_elems elements."""
+        import torch
+        _check(txt, torch.bfloat16, "txt")
+        _check(dv, torch.float32, "dv")
+        _check(grad, torch.float32, "grad")
+        if dx_t is not None:
+            _check(dx_t, torch.float32, "dx_t")
+        B = dv.shape[0]
+        _call("ff_dit_backward", self._h, B, _ptr(txt), _ptr(dv), _ptr(grad), _ptr(dx_t), _ptr(ws), ws.numel(),
               _stream(stream))
 
     def rollout_workspace_size(self, B: int, S: int) -> int:

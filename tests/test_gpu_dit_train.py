@@ -1,0 +1,219 @@
+"""GPU parity of the training pass (ff_dit_forward_train, ff_dit_backward,
+ff_sde_logprob_backward) against the fp64 oracle's vector-Jacobian product
+(oracle/dit_grad.py), tensor by tensor, on small MMDiTs; properties of the
+Flux-shaped block at full size."""
+import numpy as np
+import pytest
+
+import synth
+from conftest import rms_rel
+from oracle import dit as odit
+from oracle import dit_grad, sde
+from oracle import grpo as ogrpo
+
+pytestmark = pytest.mark.gpu
+
+# Per-tensor RMS-relative bound for the gradients: every product runs on
+# bf16 operands (unit roundoff 2^-8) with fp32 accumulation, and a gradient
+# passes through about ten such roundings between dv and a weight, so the
+# relative error grows to about sqrt(10) 2^-8 ~ 1.2e-2; 3e-2 leaves a margin.
+G_TOL = 3e-2
+V_TOL = 2e-2
+
+SMALL = dict(name="train_small", arch="mmdit", hidden=256, heads=2, head_dim=128, mlp=512,
+             n_double=1, n_single=1, patch_dim=64, txt_dim=128, n_txt=16, grid=(1, 4, 8),
+             rope_axes=(16, 56, 56), rope_theta=10000.0, time_freq_dim=256, batch=2)
+
+
+def _cfg(**kw):
+    c = dict(SMALL)
+    c.update(kw)
+    return c
+
+
+class Run:
+    """Model, inputs and one training pass on the GPU."""
+
+    def __init__(self, cfg, dev, seed=0, std=0.05):
+        import torch
+        from paper_2602_12529_gb300 import ffi, weights
+        self.cfg = cfg
+        self.W = {}
+
+        def get(name, shape):
+            a = synth.weight(name, shape, synth.weight_kind(name), seed, std, 0.05, 0.2)
+            self.W[name] = a
+            return a
+
+        self.blob = weights.pack(cfg, get, dev)
+        self.specs, self.total = weights.layout(cfg)
+        self.model = ffi.Dit(cfg, self.blob)
+        B = cfg["batch"]
+        self.B = B
+        self.x = synth.initial_latent(cfg, batch=B)
+        self.txt = synth.text_embeds(cfg, batch=B)
+        self.t = np.linspace(0.9, 0.35, B).astype(np.float32)
+        self.dev = dev
+        self.xg = torch.from_numpy(self.x).to(dev)
+        self.tg = torch.from_numpy(self.txt.view(np.int16)).to(dev).view(torch.bfloat16)
+        self.tt = torch.from_numpy(self.t).to(dev)
+        self.ws = torch.empty(self.model.train_workspace_size(B), dtype=torch.uint8, device=dev)
+        self.v = torch.empty_like(self.xg)
+        self.model.ff_dit_forward_train(self.xg, self.tg, self.tt, self.v, self.ws)
+
+    def backward(self, dv):
+        import torch
+        from paper_2602_12529_gb300 import ffi
+        grad = torch.zeros(self.total, dtype=torch.float32, device=self.dev)
+        dx = torch.empty_like(self.xg)
+        dvg = dv if isinstance(dv, torch.Tensor) else torch.from_numpy(np.ascontiguousarray(dv, np.float32)).to(self.dev)
+        self.model.ff_dit_backward(self.tg, dvg, grad, self.ws, dx_t=dx)
+        torch.cuda.synchronize()
+        assert ffi.ff_check_device_status() == 0
+        return grad.cpu().numpy(), dx.cpu().numpy()
+
+    def tensors(self, grad):
+        return {name: grad[off:off + int(np.prod(shape))].reshape(shape) for name, off, shape in self.specs}
+
+    def oracle(self, dv):
+        P = odit.widen_params(self.W)
+        return dit_grad.velocity_vjp(P, self.cfg, self.x, odit.widen(self.txt), self.t.astype(np.float64), dv)
+
+
+def _compare(run, grad, dx, want_G, want_dx):
+    got = run.tensors(grad)
+    errs = {k: rms_rel(got[k], want_G[k]) for k in want_G}
+    bad = {k: e for k, e in errs.items() if not e <= G_TOL}
+    assert not bad, sorted(bad.items(), key=lambda kv: -kv[1])[:8]
+    assert rms_rel(dx, want_dx) <= G_TOL
+
+
+@pytest.mark.parametrize("over", [{}, {"n_double": 2, "n_single": 0}, {"n_double": 0, "n_single": 2},
+                                  {"grid": (1, 3, 5), "n_txt": 5, "batch": 8},
+                                  {"batch": 3, "n_txt": 8, "grid": (1, 4, 6)}])
+def test_backward_matches_oracle(cuda, over):
+    cfg = _cfg(**over)
+    run = Run(cfg, cuda)
+    dv = np.random.default_rng(5).standard_normal((cfg["batch"], synth.n_img(cfg), cfg["patch_dim"])).astype(np.float32)
+    grad, dx = run.backward(dv)
+    v_ref, G, dx_ref = run.oracle(dv.astype(np.float64))
+    assert rms_rel(run.v.cpu().numpy(), v_ref) <= V_TOL
+    _compare(run, grad, dx, G, dx_ref)
+
+
+def test_forward_train_equals_velocity_and_backward_is_deterministic(cuda):
+    import torch
+    cfg = _cfg()
+    run = Run(cfg, cuda, seed=1)
+    ws = torch.empty(run.model.workspace_size(run.B), dtype=torch.uint8, device=cuda)
+    v = torch.empty_like(run.xg)
+    run.model.ff_dit_velocity(run.xg, run.tg, run.tt, v, ws)
+    torch.cuda.synchronize()
+    assert torch.equal(v, run.v)
+    dv = np.random.default_rng(6).standard_normal(tuple(v.shape)).astype(np.float32)
+    g1, d1 = run.backward(dv)
+    g2, d2 = run.backward(dv)
+    assert np.array_equal(g1, g2) and np.array_equal(d1, d2)
+
+
+def test_sde_logprob_backward_parity(cuda):
+    import torch
+    from paper_2602_12529_gb300 import ffi
+    rng = np.random.default_rng(8)
+    B, D = 5, 4096 * 3 + 64
+    x, v = rng.standard_normal((B, D)).astype(np.float32), rng.standard_normal((B, D)).astype(np.float32)
+    t = np.array([0.95, 0.8, 0.5, 0.3, 0.2], np.float32)
+    tn = (t - np.array([0.1, 0.2, 0.1, 0.05, 0.2], np.float32)).astype(np.float32)
+    sig = np.array([0.7, 0.5, 0.0, 0.9, 0.3], np.float32)
+    xn = (x + 0.3 * rng.standard_normal((B, D))).astype(np.float32)
+    g = rng.standard_normal((B, 3)).astype(np.float32)      # read with ld = 3 (column 1)
+    dev = cuda
+    T = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+    for reduce, name in ((ffi.FF_LP_SUM, "sum"), (ffi.FF_LP_MEAN, "mean")):
+        out = torch.empty(B, D, dtype=torch.float32, device=dev)
+        gcol = T(g.ravel()[1:])           # element b * 3 is g[b, 1]
+        ffi.ff_sde_logprob_backward(T(x), T(v), T(xn), T(t), T(tn), T(sig), gcol, out, reduce=reduce, ld=3)
+        torch.cuda.synchronize()
+        want = sde.sde_logprob_grad_v(x, v, xn, t.astype(np.float64), tn.astype(np.float64),
+                                      sig.astype(np.float64), name) * g[:, 1:2]
+        got = out.cpu().numpy()
+        assert not np.any(got[2])
+        for b in range(B):
+            if sig[b] > 0:
+                assert rms_rel(got[b], want[b]) <= 1e-5, (name, b)
+
+
+def test_grpo_training_step_chain(cuda):
+    """One Flow-GRPO training step for a batch: re-score the rollout's
+    x_next under the current velocity (forward_train, SDE EVAL log-prob),
+    clipped loss and its gradient, then d loss / d theta through
+    ff_sde_logprob_backward and ff_dit_backward.  The oracle takes the same
+    loss gradient and goes through its own log-prob and network backward."""
+    import torch
+    from paper_2602_12529_gb300 import ffi
+    cfg = _cfg(batch=4, n_txt=8)
+    run = Run(cfg, cuda, seed=2)
+    B, Ni, Pd = run.B, synth.n_img(cfg), cfg["patch_dim"]
+    P = odit.widen_params(run.W)
+    t = run.t.astype(np.float64)
+    tn = t - 0.1
+    sig = sde.sigma_flow_sde(t, 0.7)
+    v_o = odit.velocity(P, cfg, run.x, odit.widen(run.txt), t)
+    eps = synth.gaussian((B, Ni, Pd), seed=31)
+    x_next, _ = sde.sde_step_logprob(run.x, v_o, t, tn, sig, eps=eps)
+    x_next = x_next.astype(np.float32)
+    dev = cuda
+    T = lambda a: torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(dev)
+    tg, tng, sg = T(t), T(tn), T(sig)
+    lp = torch.empty(B, 1, dtype=torch.float32, device=dev)
+    ws = torch.empty(ffi.ff_sde_workspace_size(B, Ni * Pd), dtype=torch.uint8, device=dev)
+    xn_g = T(x_next)
+    ffi.ff_sde_step_logprob(run.xg, run.v, None, xn_g, tg, tng, sg, lp, mode=ffi.FF_SDE_EVAL, ws=ws)
+    lp_old = lp + T(synth.logprob_jitter((B, 1), seed=9))
+    adv = T(synth.gaussian((B,), seed=32))
+    loss = torch.empty(1, dtype=torch.float32, device=dev)
+    glp = torch.empty(B, 1, dtype=torch.float32, device=dev)
+    ffi.ff_grpo_loss(lp, lp_old, adv, 0.2, 0.2, loss, grad_lp_new=glp)
+    dv = torch.empty_like(run.xg)
+    ffi.ff_sde_logprob_backward(run.xg, run.v, xn_g, tg, tng, sg, glp, dv, ld=1)
+    grad, dx = run.backward(dv)
+    g = glp.cpu().numpy()[:, 0].astype(np.float64)
+    _, g_want = ogrpo.grpo_loss(lp.cpu().numpy().astype(np.float64), lp_old.cpu().numpy().astype(np.float64),
+                                adv.cpu().numpy())
+    np.testing.assert_allclose(g, g_want[:, 0], rtol=1e-5)
+    dv_o = sde.sde_logprob_grad_v(run.x, v_o, x_next, t, tn, sig) * g[:, None, None]
+    assert rms_rel(dv.cpu().numpy(), dv_o) <= V_TOL
+    _, G, dx_ref = run.oracle(dv_o)
+    _compare(run, grad, dx, G, dx_ref)
+
+
+def test_flux_block_training_pass_properties(cuda):
+    """Flux-shaped double-stream block (H 3072, 24 x 128 heads, MLP 12288,
+    512 text + 4096 image tokens, batch 4) at full size: the training
+    forward equals the velocity call bit for bit; the backward is
+    deterministic, finite, linear in dv, and its final-bias gradient is the
+    token sum of dv."""
+    import torch
+    cfg = synth.config("flux_double_block")
+    run = Run(cfg, cuda, std=0.02)
+    ws = torch.empty(run.model.workspace_size(run.B), dtype=torch.uint8, device=cuda)
+    v = torch.empty_like(run.xg)
+    run.model.ff_dit_velocity(run.xg, run.tg, run.tt, v, ws)
+    torch.cuda.synchronize()
+    assert torch.equal(v, run.v)
+    del ws
+    rng = np.random.default_rng(7)
+    d1 = torch.from_numpy(rng.standard_normal(tuple(v.shape)).astype(np.float32)).to(cuda)
+    d2 = torch.from_numpy(rng.standard_normal(tuple(v.shape)).astype(np.float32)).to(cuda)
+    g1, x1 = run.backward(d1)
+    g1b, _ = run.backward(d1)
+    assert np.array_equal(g1, g1b)
+    assert np.all(np.isfinite(g1)) and np.all(np.isfinite(x1))
+    g2, x2 = run.backward(d2)
+    g12, x12 = run.backward(d1 + d2)
+    got = run.tensors(g12)
+    s1, s2 = run.tensors(g1), run.tensors(g2)
+    for name in got:
+        assert rms_rel(got[name], s1[name] + s2[name]) <= G_TOL, name
+    fb = run.tensors(g1)["final.b"]
+    np.testing.assert_allclose(fb, d1.double().sum(dim=(0, 1)).cpu().numpy(), rtol=1e-4, atol=1e-3)
