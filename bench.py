@@ -476,6 +476,72 @@ def backward_kernels(args, ffi, cfg, dev):
     return out
 
 
+def train_step(args, ffi, model, cfg, dev, x, txt, t, tn, sg, x_next, lp_old, adv, fwd_flops, timed, world):
+    """One Flow-GRPO training step on the batch of the main step: re-score
+    the rollout's x_next under the current velocity (training forward, SDE
+    log-prob in EVAL mode), the clipped loss with dL/dlp, then dL/dv through
+    the log-prob backward and dL/dtheta for every weight through the DiT
+    backward.  Algorithmic FLOPs: the forward's (GEMM 2 M N K, attention
+    4 B h N^2 d), plus twice the GEMM FLOPs (input and weight gradients) and
+    10 B h N^2 d per attention backward (recomputed S, dP, dV, dK, dQ)."""
+    import torch
+    if cfg.get("arch") == "wan" or cfg["head_dim"] != 128:
+        return None
+    B = x.shape[0]
+    D = x.numel() // B
+    need = model.train_workspace_size(B)
+    _, total = ffi.ff_dit_weight_layout(cfg)
+    free, _ = torch.cuda.mem_get_info(dev)
+    if need + 4 * total > 0.9 * free:
+        return {"skipped": f"training workspace {need / 1e9:.1f} GB + fp32 gradients {4 * total / 1e9:.1f} GB "
+                           f"exceed the free device memory ({free / 1e9:.1f} GB)"}
+    ws_t = torch.empty(need, dtype=torch.uint8, device=dev)
+    grad = torch.empty(total, dtype=torch.float32, device=dev)
+    v = torch.empty_like(x)
+    dv = torch.empty_like(x)
+    lp = torch.empty((B, 1), dtype=torch.float32, device=dev)
+    glp = torch.empty((B, 1), dtype=torch.float32, device=dev)
+    loss = torch.empty(1, dtype=torch.float32, device=dev)
+    ws_sde = torch.empty(ffi.ff_sde_workspace_size(B, D), dtype=torch.uint8, device=dev)
+    ws_loss = torch.empty(ffi.ff_grpo_loss_workspace_size(B, 1), dtype=torch.uint8, device=dev)
+
+    def step():
+        model.ff_dit_forward_train(x, txt, t, v, ws_t)
+        ffi.ff_sde_step_logprob(x, v, None, x_next, t, tn, sg, lp, mode=ffi.FF_SDE_EVAL, ws=ws_sde)
+        ffi.ff_grpo_loss(lp, lp_old, adv, cfg["clip"], cfg["clip"], loss, glp, ws=ws_loss)
+        ffi.ff_sde_logprob_backward(x, v, x_next, t, tn, sg, glp, dv)
+        model.ff_dit_backward(txt, dv, grad, ws_t)
+
+    for _ in range(args.warmup):
+        step()
+    ms = timed(step, args.steps) / args.steps
+    ffi.ff_prof_enable((48 * (cfg["n_double"] + cfg["n_single"]) + 128) * args.steps + 64)
+    timed(step, args.steps)
+    recs = ffi.ff_prof_records()
+    ffi.ff_prof_disable()
+    kern = {}
+    for name, ms_, fl, by in recs:
+        k = kern.setdefault(name, [0, 0.0])
+        k[0] += 1
+        k[1] += ms_
+    tot = sum(k[1] for k in kern.values())
+    N = cfg["n_txt"] + synth_n_img(cfg)
+    L = cfg["n_double"] + cfg["n_single"]
+    attn_fwd = 4.0 * B * cfg["heads"] * N * N * cfg["head_dim"] * L
+    gemm_fwd = fwd_flops - attn_fwd
+    flops = 3.0 * gemm_fwd + attn_fwd + 2.5 * attn_fwd
+    _, tc_burst, tc_sust, src = load_peaks()
+    return {"ms_per_step": ms, "value": world * B * synth_n_img(cfg) / (ms / 1e3), "unit": UNIT,
+            "what": "training forward (activations kept) + SDE EVAL log-prob + clipped loss and dL/dlp + "
+                    "log-prob backward + DiT backward to every weight (fp32 gradients), batch of the main step",
+            "tflops": flops / (ms / 1e3) / 1e12, "frac": flops / (ms / 1e3) / 1e12 / tc_burst,
+            "frac_vs_sustained": flops / (ms / 1e3) / 1e12 / tc_sust if tc_sust else None,
+            "algorithmic_flops": flops, "workspace_gb": need / 1e9, "gpu_launches": len(recs) // args.steps,
+            "kernels": {k: {"launches": v_[0] // args.steps, "ms_per_step": v_[1] / args.steps, "share": v_[1] / tot}
+                        for k, v_ in sorted(kern.items(), key=lambda kv: -kv[1][1])},
+            "peak": f"{tc_burst} TFLOP/s ({src} bf16 dense burst)"}
+
+
 def synth_n_img(cfg):
     import synth
     return synth.n_img(cfg)
@@ -677,6 +743,7 @@ def run_ours(args):
     ms_e2e = timed(e2e_step, args.steps) / args.steps
     e2e_value = whole_job_rate(world, tokens_per_step, ms_e2e)
     awm = awm_step(args, ffi, model, cfg, dev, x, txt, eps, rewards, timed, world)
+    train = train_step(args, ffi, model, cfg, dev, x, txt, t, tn, sg, x_next, lp_old, adv, dit_flops, timed, world)
     bwd = backward_kernels(args, ffi, cfg, dev) if rank == 0 and not args.no_sweep else None
     sweep = hbm_sweep(ffi, dev, hbm) if rank == 0 and not args.no_sweep else None
     clk = clocks.stop() if clocks else None
@@ -706,6 +773,7 @@ def run_ours(args):
                         "ms_per_step": ms_e2e},
                 "hbm_sweep": sweep,
                 "awm_step": awm,
+                "train_step": train,
                 "backward_kernels": bwd,
                 "gpu_launches": launches,
                 "clocks": clk,

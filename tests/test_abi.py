@@ -149,3 +149,44 @@ def test_awm_and_multi_reward_host_validation(L):
     assert L.ff_group_advantage_multi(2, 4, 65, 16, 16, 0, 1e-4, 16, None) == 2
     assert L.ff_group_advantage_multi(2, 4, 2, 16, 16, 7, 1e-4, 16, None) == 1
     assert L.ff_grpo_loss_weighted(4, 2, 16, 16, 16, None, 0.2, 0.2, 16, None, 16, 64, None) == 1
+
+
+def test_training_pass_host_validation(L):
+    small = dict(synth.config("tiny_mmdit"), hidden=256, heads=2, head_dim=128, mlp=512, n_double=1, n_single=1,
+                 txt_dim=128, n_txt=16, grid=(1, 4, 8), rope_axes=(16, 56, 56))
+    c = ffi.make_config(small)
+    h = C.c_void_p()
+    assert L.ff_dit_create(C.byref(c), C.c_void_p(256), C.byref(h)) == 0
+    n = C.c_size_t()
+    assert L.ff_dit_train_workspace_size(h, 2, C.byref(n)) == 0
+    H, F, R = 256, 512, 2 * (16 + 32)
+    # at least the stored activations of one double- and one single-stream block
+    assert n.value >= R * (30 * H + 4 * F) + R * (22 * H + 4 * F)
+    # B N_t and B N_i must be multiples of 8 (token counts are the K of the weight gradients)
+    odd = ffi.make_config(dict(small, n_txt=5))
+    h5 = C.c_void_p()
+    assert L.ff_dit_create(C.byref(odd), C.c_void_p(256), C.byref(h5)) == 0
+    assert L.ff_dit_train_workspace_size(h5, 2, C.byref(n)) == 2
+    assert L.ff_dit_train_workspace_size(h5, 8, C.byref(n)) == 0
+    assert L.ff_dit_destroy(h5) == 0
+    # rejected on the host: workspace too small, misaligned workspace, null gradient
+    assert L.ff_dit_forward_train(h, 2, 16, 16, 16, 16, 256, 1024, None) == 3
+    assert L.ff_dit_backward(h, 2, 16, 16, 16, None, 256, 1024, None) == 3
+    assert L.ff_dit_backward(h, 2, 16, 16, None, None, 256, 1 << 40, None) == 1
+    assert L.ff_dit_backward(h, 2, 16, 16, 16, None, 255, 1 << 40, None) == 1
+    assert L.ff_dit_destroy(h) == 0
+    # head_dim 64 models and WAN models have no training pass
+    c64 = ffi.make_config(synth.config("tiny_mmdit"))
+    assert L.ff_dit_create(C.byref(c64), C.c_void_p(256), C.byref(h)) == 0
+    assert L.ff_dit_train_workspace_size(h, 4, C.byref(n)) == 2
+    assert L.ff_dit_destroy(h) == 0
+    wan = ffi.make_config(dict(synth.config("wan_40"), hidden=256, heads=2, mlp=512, n_double=1, grid=(2, 4, 4),
+                               rope_axes=(44, 42, 42)))
+    assert L.ff_dit_create(C.byref(wan), C.c_void_p(256), C.byref(h)) == 0
+    assert L.ff_dit_train_workspace_size(h, 4, C.byref(n)) == 2
+    assert L.ff_dit_destroy(h) == 0
+    # the log-prob backward
+    assert L.ff_sde_logprob_backward(2, 18, 16, 16, 16, 16, 16, 16, 0, 16, 1, 16, None) == 2   # D % 4
+    assert L.ff_sde_logprob_backward(2, 16, 16, 16, 16, 16, 16, 16, 5, 16, 1, 16, None) == 1   # reduce
+    assert L.ff_sde_logprob_backward(2, 16, 16, 16, None, 16, 16, 16, 0, 16, 1, 16, None) == 1
+    assert L.ff_sde_logprob_backward(2, 16, 16, 16, 16, 16, 16, 16, 0, 16, 0, 16, None) == 1   # ld
