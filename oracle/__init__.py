@@ -15,6 +15,8 @@ Modules:
            clipped-ratio policy loss (optionally with per-step weights).
   awm   -- training-time sampling, the forward process x_t and the
            advantage-weighted matching loss of Eq. 3.
+  nft   -- the DiffusionNFT loss of Eq. 2 (implicit positive / negative
+           policies read from the cited method).
   dit   -- the flow-matching DiT velocity v_theta(x_t, t): MMDiT double- and
            single-stream blocks (adaLN modulation, QK-RMSNorm, RoPE, joint
            attention, GELU MLP) and the final projection.
