@@ -365,6 +365,24 @@ def hbm_sweep(ffi, dev, hbm_peak, l2_bytes=129 * 2 ** 20):
                          "sets": len(sets)})
             del sets
         out[name] = rows
+    rows = []
+    for n in (1 << 24, 1 << 26, 1 << 28):
+        B, D = 4, n // 4
+        per = 20 * n
+        sets = []
+        for _ in range(nsets(per)):
+            x = torch.randn(B, D, device=dev)
+            sets.append((x, torch.randn_like(x), torch.randn_like(x), torch.randn_like(x), torch.empty_like(x)))
+        r = torch.rand(B, device=dev)
+        loss = torch.empty(1, device=dev)
+        ws = torch.empty(ffi.ff_nft_loss_workspace_size(B, D), dtype=torch.uint8, device=dev)
+        fns = [lambda s_=s_: ffi.ff_nft_loss(s_[0], s_[1], s_[2], s_[3], r, 0.1, ffi.FF_AWM_MEAN, loss, s_[4], ws=ws)
+               for s_ in sets]
+        sec = timeit(fns)
+        rows.append({"elements": n, "bytes": per, "gbs": per / sec / 1e9, "frac": per / sec / 1e9 / hbm_peak,
+                     "sets": len(sets)})
+        del sets
+    out["nft_loss"] = rows
     torch.cuda.empty_cache()
     return out
 

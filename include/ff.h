@@ -280,6 +280,26 @@ int ff_awm_loss(int B, int64_t D, const float* v, const float* eps, const float*
                 void* ws, size_t ws_bytes, cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
+ * DiffusionNFT loss (paper Sec. 3.2, Eq. 2):
+ *   loss = (1/B) sum_b [ r_b e+_b + (1 - r_b) e-_b ],
+ *   e+-_b = ||v+-_b - (eps_b - x0_b)||^2  (divided by D for FF_AWM_MEAN),
+ * with the implicit positive / negative policies of the cited DiffusionNFT
+ * method (the paper names them without defining them):
+ *   v+ = (1 - beta) v_old + beta v,   v- = (1 + beta) v_old - beta v,
+ * v the trained velocity and v_old the frozen velocity of the sampling
+ * policy at the same (x_t, t).  The target eps - x0 is that of Eq. 3.
+ *   v, v_old, eps, x0: [B, D] fp32 (D % 4 == 0); r: [B] fp32 reward weights
+ *   in [0, 1] (device; not checked); beta > 0.
+ *   loss: [1] fp32; grad_v: [B, D] fp32 dL/dv or NULL; err: [B, 2] fp32
+ *   (e+_b, e-_b) or NULL.  ws: ff_nft_loss_workspace_size bytes, 8-byte
+ *   aligned.  Deterministic (fixed-order fp64 sums).
+ * ------------------------------------------------------------------------ */
+int ff_nft_loss_workspace_size(int B, int64_t D, size_t* bytes);
+int ff_nft_loss(int B, int64_t D, const float* v, const float* v_old, const float* eps,
+                const float* x0, const float* r, float beta, int reduce, float* loss,
+                float* grad_v, float* err, void* ws, size_t ws_bytes, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
  * DiT velocity v_theta(x_t, t) (the network of Eq. 1 and Eq. 3).
  *
  * Architecture (MMDiT, Flux / Qwen-Image style): timestep embedding MLP and

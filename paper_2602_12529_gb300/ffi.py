@@ -72,6 +72,8 @@ _SIGS = {
     "ff_forward_process": ([_I, _I64, _P, _P, _P, _P, _P], _I),
     "ff_awm_loss_workspace_size": ([_I, _I64, C.POINTER(_SZ)], _I),
     "ff_awm_loss": ([_I, _I64, _P, _P, _P, _P, _I, _P, _P, _P, _P, _SZ, _P], _I),
+    "ff_nft_loss_workspace_size": ([_I, _I64, C.POINTER(_SZ)], _I),
+    "ff_nft_loss": ([_I, _I64, _P, _P, _P, _P, _P, _F, _I, _P, _P, _P, _P, _SZ, _P], _I),
     "ff_dit_weight_layout": ([C.POINTER(DitConfig), C.POINTER(TensorDesc), _I, C.POINTER(_I), C.POINTER(_I64)], _I),
     "ff_dit_create": ([C.POINTER(DitConfig), _P, C.POINTER(_P)], _I),
     "ff_dit_destroy": ([_P], _I),
@@ -328,6 +330,25 @@ def ff_awm_loss_workspace_size(B: int, D: int) -> int:
     n = _SZ()
     _call("ff_awm_loss_workspace_size", B, D, C.byref(n))
     return n.value
+
+
+def ff_nft_loss_workspace_size(B: int, D: int) -> int:
+    n = _SZ()
+    _call("ff_nft_loss_workspace_size", B, D, C.byref(n))
+    return n.value
+
+
+def ff_nft_loss(v, v_old, eps, x0, r, beta: float, reduce: int, loss, grad_v=None, err=None, ws=None, stream=None):
+    """DiffusionNFT loss (Eq. 2); err: [B, 2] or None."""
+    import torch
+    for n_, a in (("v", v), ("v_old", v_old), ("eps", eps), ("x0", x0), ("r", r), ("loss", loss)):
+        _check(a, torch.float32, n_)
+    B = v.shape[0]
+    D = v.numel() // B
+    if ws is None:
+        ws = torch.empty(ff_nft_loss_workspace_size(B, D), dtype=torch.uint8, device=v.device)
+    _call("ff_nft_loss", B, D, _ptr(v), _ptr(v_old), _ptr(eps), _ptr(x0), _ptr(r), beta, reduce, _ptr(loss),
+          _ptr(grad_v), _ptr(err), _ptr(ws), ws.numel(), _stream(stream))
 
 
 def ff_awm_loss(v, eps, x0, adv, reduce: int, loss, grad_v=None, err=None, ws=None, stream=None):

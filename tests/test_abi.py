@@ -190,3 +190,12 @@ def test_training_pass_host_validation(L):
     assert L.ff_sde_logprob_backward(2, 16, 16, 16, 16, 16, 16, 16, 5, 16, 1, 16, None) == 1   # reduce
     assert L.ff_sde_logprob_backward(2, 16, 16, 16, None, 16, 16, 16, 0, 16, 1, 16, None) == 1
     assert L.ff_sde_logprob_backward(2, 16, 16, 16, 16, 16, 16, 16, 0, 16, 0, 16, None) == 1   # ld
+
+
+def test_nft_host_validation(L):
+    assert ffi.ff_nft_loss_workspace_size(4, 262144) == 4 * 65 * 2 * 8
+    assert L.ff_nft_loss(2, 18, 16, 16, 16, 16, 16, 0.1, 0, 16, None, None, 16, 1 << 20, None) == 2   # D % 4
+    assert L.ff_nft_loss(2, 16, 16, 16, 16, 16, 16, 0.1, 3, 16, None, None, 16, 1 << 20, None) == 1   # reduce
+    assert L.ff_nft_loss(2, 16, 16, 16, 16, 16, 16, 0.0, 0, 16, None, None, 16, 1 << 20, None) == 1   # beta
+    assert L.ff_nft_loss(2, 16, 16, None, 16, 16, 16, 0.1, 0, 16, None, None, 16, 1 << 20, None) == 1
+    assert L.ff_nft_loss(2, 16, 16, 16, 16, 16, 16, 0.1, 0, 16, None, None, 16, 8, None) == 3        # workspace

@@ -217,3 +217,34 @@ def test_flux_block_training_pass_properties(cuda):
         assert rms_rel(got[name], s1[name] + s2[name]) <= G_TOL, name
     fb = run.tensors(g1)["final.b"]
     np.testing.assert_allclose(fb, d1.double().sum(dim=(0, 1)).cpu().numpy(), rtol=1e-4, atol=1e-3)
+
+
+def test_nft_training_step_chain(cuda):
+    """A DiffusionNFT step (Eq. 2): the trained velocity from the training
+    forward, the frozen old policy's velocity from a second model, the loss
+    with dL/dv, then the DiT backward; against the oracle chain."""
+    import torch
+    from oracle import awm as oawm
+    from oracle import nft as onft
+    from paper_2602_12529_gb300 import ffi
+    cfg = _cfg(batch=4, n_txt=8)
+    run = Run(cfg, cuda, seed=3)
+    old = Run(cfg, cuda, seed=4)
+    B, Ni, Pd = run.B, synth.n_img(cfg), cfg["patch_dim"]
+    eps, x0 = synth.gaussian((B, Ni, Pd), 60, "eps"), synth.gaussian((B, Ni, Pd), 61, "x0")
+    r = synth.uniform((B,), 62, "r")
+    T = lambda a: torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(cuda)
+    loss = torch.empty(1, dtype=torch.float32, device=cuda)
+    dv = torch.empty_like(run.xg)
+    beta = 0.5
+    ffi.ff_nft_loss(run.v, old.v, T(eps), T(x0), T(r), beta, ffi.FF_AWM_MEAN, loss, dv)
+    grad, dx = run.backward(dv)
+    P = odit.widen_params(run.W)
+    t = run.t.astype(np.float64)
+    v_o = odit.velocity(P, cfg, run.x, odit.widen(run.txt), t)
+    vold_o = odit.velocity(odit.widen_params(old.W), cfg, old.x, odit.widen(old.txt), t)
+    L_o, dv_o, _ = onft.nft_loss(v_o, vold_o, eps, x0, r, beta, "mean")
+    assert abs(float(loss.item()) - L_o) <= V_TOL * abs(L_o)
+    assert rms_rel(dv.cpu().numpy(), dv_o) <= V_TOL
+    _, G, dx_ref = run.oracle(dv_o)
+    _compare(run, grad, dx, G, dx_ref)
