@@ -31,8 +31,12 @@ namespace {
 constexpr int HD = 128;
 constexpr int kT = 128;                        // rows of a query / key tile
 constexpr int kTileBytes = kT * HD * 2;         // 32 KB: one bf16 tile (two 64-column boxes)
-constexpr int kSlots = 4;                       // streamed tiles in flight
-constexpr int kThreads = 192;                   // producer, MMA, 4 elementwise warps
+constexpr int kSub = 64;                        // query / key columns of one S (S^T) sub-tile
+constexpr int kSlotsDq = 5;                     // streamed K / V tiles in flight (dQ kernel)
+constexpr int kSlotsDkdv = 4;                   // streamed Q / dO tiles in flight (dK dV kernel)
+constexpr int kMaxSlots = 5;
+constexpr int kThreads = 320;                   // producer, MMA, 8 elementwise warps (two per TMEM lane quarter)
+constexpr int kEw = 8;                          // elementwise warps
 constexpr int kBarBytes = 256;
 
 struct BwdParams {
@@ -50,10 +54,10 @@ struct BwdParams {
 
 struct Bars {
     uint64_t fixed_full;           // the CTA's own tiles landed
-    uint64_t slot_full[kSlots];
-    uint64_t slot_empty[kSlots];
-    uint64_t s_full;               // MMA -> elementwise: S (S^T) and dP (dP^T) in TMEM
-    uint64_t p_full;               // elementwise -> MMA: dS (P^T, dS^T) in TMEM
+    uint64_t slot_full[kMaxSlots];
+    uint64_t slot_empty[kMaxSlots];
+    uint64_t s_full[2];            // MMA -> elementwise: S (S^T) and dP (dP^T) of a sub-tile in TMEM buffer b
+    uint64_t p_full[2];            // elementwise -> MMA: dS (P^T, dS^T) of buffer b in TMEM
     uint64_t done;                 // MMA -> elementwise: the accumulators are final
     uint64_t drain;
     uint32_t tmem_slot;
@@ -66,10 +70,11 @@ __device__ __forceinline__ void bulk_load_1d(void* dst, const void* src, uint32_
                  : "memory");
 }
 
-// Stores a 128-column fp32 TMEM row of this thread as bf16 (times mul).
-__device__ __forceinline__ void store_row_bf16(uint32_t taddr, float mul, __nv_bfloat16* dst, bool live) {
+// Stores `cols` fp32 TMEM columns of this thread's row as bf16 (times mul).
+__device__ __forceinline__ void store_row_bf16(uint32_t taddr, float mul, __nv_bfloat16* dst, bool live,
+                                               int cols = HD) {
 #pragma unroll 1
-    for (int c = 0; c < HD; c += 32) {
+    for (int c = 0; c < cols; c += 32) {
         uint32_t o[32];
         tmem_ld_x32(taddr + c, o);
         tmem_ld_wait();
@@ -116,17 +121,24 @@ __global__ void __launch_bounds__(256) attn_bwd_delta_kernel(int B, int heads, i
 }
 
 // ------------------------------------------------------------------ dQ
-// TMEM: S at 0, dP at 128, dQ at 256 (dS as bf16 pairs over S's first 64).
-// Shared memory: Q tile, dO tile, then a ring of K_j / V_j tiles.
+// TMEM: two sub-tile buffers of 128 columns, buffer b holding S (64 key
+// columns) at 128 b and dP at 128 b + 64; the two elementwise warps of a
+// lane quarter take 32 key columns each and write their dS as bf16 pairs over
+// the first 16 of their own S columns (keys 0-31 at 0, keys 32-63 at 32); dQ
+// at 256.  Key tile j is processed as two 64-key
+// halves, half b in buffer b, so the elementwise warps work on one buffer
+// while the MMAs of the other (dQ += dS K, then the next half's S and dP)
+// run.  Shared memory: Q tile, dO tile, then a ring of K_j / V_j tiles.
 __global__ void __launch_bounds__(kThreads, 1)
 attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_constant__ CUtensorMap tm_qkv1,
                    const __grid_constant__ CUtensorMap tm_do0, const __grid_constant__ CUtensorMap tm_do1,
                    const BwdParams p, int* status) {
+    constexpr int S_ = kSlotsDq;
     extern __shared__ __align__(1024) uint8_t smem[];
     uint8_t* sQ = smem;
     uint8_t* sdO = smem + kTileBytes;
-    uint8_t* sKV = smem + 2 * kTileBytes;                     // [kSlots][tile]
-    Bars& bar = *reinterpret_cast<Bars*>(sKV + kSlots * kTileBytes);
+    uint8_t* sKV = smem + 2 * kTileBytes;                     // [S_][tile]
+    Bars& bar = *reinterpret_cast<Bars*>(sKV + S_ * kTileBytes);
     volatile int* abort_flag = &bar.abort_flag;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int b = blockIdx.z, h = blockIdx.y;
@@ -141,12 +153,14 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_con
             *abort_flag = 1;
         }
         mbar_init(&bar.fixed_full, 1);
-        for (int s = 0; s < kSlots; ++s) {
+        for (int s = 0; s < S_; ++s) {
             mbar_init(&bar.slot_full[s], 1);
             mbar_init(&bar.slot_empty[s], 1);
         }
-        mbar_init(&bar.s_full, 1);
-        mbar_init(&bar.p_full, 4);
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(&bar.s_full[s], 1);
+            mbar_init(&bar.p_full[s], kEw);
+        }
         mbar_init(&bar.done, 1);
         mbar_init(&bar.drain, 1);
         fence_mbar_init();
@@ -174,8 +188,8 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_con
             tma_load_2d(sdO + c * (kT * 128), td, &bar.fixed_full, h * HD + c * 64, b * p.n[seg] + q0);
         }
         for (int n = 0; n < 2 * ntiles; ++n) {
-            const int s = n % kSlots;
-            if (!mbar_wait(&bar.slot_empty[s], ((n / kSlots) & 1) ^ 1)) { fail(); break; }
+            const int s = n % S_;
+            if (!mbar_wait(&bar.slot_empty[s], ((n / S_) & 1) ^ 1)) { fail(); break; }
             const int j = n >> 1;
             const int ks = j < nt0 ? 0 : 1;
             const int row = b * p.n[ks] + (j - (ks ? nt0 : 0)) * kT;
@@ -187,44 +201,65 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_con
         }
     } else if (warp == 1 && lane == 0) {
         // ---- MMA issuer
-        constexpr uint32_t idesc_s = idesc_bf16_f32(kT, kT);
-        constexpr uint32_t idesc_q = idesc_bf16_f32(kT, HD) | (1u << 16);   // B = K_j, MN-major
+        constexpr uint32_t idesc_s = idesc_bf16_f32(kT, kSub);
+        constexpr uint32_t idesc_q = idesc_bf16_f32(kT, HD) | (1u << 16);   // B = K_j half, MN-major
         bool ok = mbar_wait(&bar.fixed_full, 0);
         if (!ok) fail();
         const uint64_t dq_ = smem_desc_k_sw128(smem_u32(sQ));
         const uint64_t ddo = smem_desc_k_sw128(smem_u32(sdO));
-        for (int j = 0; ok && j < ntiles; ++j) {
+        auto wait_kv = [&](int j) {
             const int nk = 2 * j, nv = 2 * j + 1;
-            if (!mbar_wait(&bar.slot_full[nk % kSlots], (nk / kSlots) & 1) ||
-                !mbar_wait(&bar.slot_full[nv % kSlots], (nv / kSlots) & 1)) { fail(); ok = false; break; }
-            tc_fence_after();
-            const uint32_t aK = smem_u32(sKV + (nk % kSlots) * kTileBytes);
-            const uint32_t aV = smem_u32(sKV + (nv % kSlots) * kTileBytes);
+            return mbar_wait(&bar.slot_full[nk % S_], (nk / S_) & 1) && mbar_wait(&bar.slot_full[nv % S_], (nv / S_) & 1);
+        };
+        // S = Q K^T and dP = dO V^T of key half hf of tile j into buffer hf
+        auto issue_sdp = [&](int j, int hf) {
+            const uint32_t aK = smem_u32(sKV + ((2 * j) % S_) * kTileBytes) + hf * (kSub * 128);
+            const uint32_t aV = smem_u32(sKV + ((2 * j + 1) % S_) * kTileBytes) + hf * (kSub * 128);
             const uint64_t dk = smem_desc_k_sw128(aK), dv = smem_desc_k_sw128(aV);
+            const uint32_t tb = tmem + hf * 128;
 #pragma unroll
             for (int k = 0; k < HD / 16; ++k) {
                 const uint32_t off = ((k / 4) * (kT * 128) + (k % 4) * 32) >> 4;
-                tc_mma_bf16(tmem, dq_ + off, dk + off, idesc_s, k != 0 ? 1u : 0u);           // S = Q K^T
-                tc_mma_bf16(tmem + kT, ddo + off, dv + off, idesc_s, k != 0 ? 1u : 0u);      // dP = dO V^T
+                tc_mma_bf16(tb, dq_ + off, dk + off, idesc_s, k != 0 ? 1u : 0u);
+                tc_mma_bf16(tb + kSub, ddo + off, dv + off, idesc_s, k != 0 ? 1u : 0u);
             }
-            tc_commit(&bar.s_full);
-            if (!mbar_wait(&bar.p_full, j & 1)) { fail(); ok = false; break; }
+            tc_commit(&bar.s_full[hf]);
+        };
+        if (ok && !wait_kv(0)) { fail(); ok = false; }
+        if (ok) {
             tc_fence_after();
-            // dQ += dS K_j: dS from TMEM, K_j as [keys (K) x d (N)], MN-major
-            const uint64_t dkm = smem_desc_mn_sw128(aK, kT * 128);
+            issue_sdp(0, 0);
+            issue_sdp(0, 1);
+        }
+        for (int u = 0; ok && u < 2 * ntiles; ++u) {
+            const int hf = u & 1, j = u >> 1;
+            if (!mbar_wait(&bar.p_full[hf], (u >> 1) & 1)) { fail(); ok = false; break; }
+            tc_fence_after();
+            // dQ += dS K_j (this half's 64 keys): dS from TMEM, K rows as [keys (K) x d (N)], MN-major
+            const uint64_t dkm = smem_desc_mn_sw128(smem_u32(sKV + ((2 * j) % S_) * kTileBytes) + hf * (kSub * 128),
+                                                    kT * 128);
 #pragma unroll
-            for (int k = 0; k < kT / 16; ++k)
-                tc_mma_bf16_ts(tmem + 2 * kT, tmem + k * 8, dkm + static_cast<uint64_t>(k * (2048 >> 4)), idesc_q,
-                               (j | k) != 0 ? 1u : 0u);
-            tc_commit(&bar.slot_empty[nk % kSlots]);
-            tc_commit(&bar.slot_empty[nv % kSlots]);
+            for (int k = 0; k < kSub / 16; ++k)   // keys 16k.. of the half: packed at (k / 2) * 32 + (k % 2) * 8
+                tc_mma_bf16_ts(tmem + 256, tmem + hf * 128 + (k >> 1) * 32 + (k & 1) * 8,
+                               dkm + static_cast<uint64_t>(k * (2048 >> 4)), idesc_q, (u | k) != 0 ? 1u : 0u);
+            if (hf == 1) {
+                tc_commit(&bar.slot_empty[(2 * j) % S_]);
+                tc_commit(&bar.slot_empty[(2 * j + 1) % S_]);
+            }
+            if (j + 1 < ntiles) {
+                if (hf == 0 && !wait_kv(j + 1)) { fail(); ok = false; break; }
+                tc_fence_after();
+                issue_sdp(j + 1, hf);
+            }
         }
         if (ok) tc_commit(&bar.done);
         tc_commit(&bar.drain);
         if (!mbar_wait(&bar.drain, 0)) report_status(status, kStatusWaitTimeout);
     } else if (warp >= 2) {
-        // ---- elementwise: thread = query row = TMEM lane
+        // ---- elementwise: thread = query row = TMEM lane; the two warps of a
+        // lane quarter take 32 key columns each of a sub-tile
         const int q = warp & 3;
+        const int cg = (warp - 2) >> 2;
         const int r = q * 32 + lane;
         const int row = q0 + r;
         const uint32_t tS = tmem + (static_cast<uint32_t>(q * 32) << 16);
@@ -233,39 +268,40 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_con
         const float lse = live ? p.lse[li] : 0.f;
         const float dd = live ? p.delta[li] : 0.f;
         bool ok = true;
-        for (int j = 0; j < ntiles; ++j) {
-            if (!mbar_wait(&bar.s_full, j & 1)) { fail(); ok = false; break; }
+        for (int u = 0; u < 2 * ntiles; ++u) {
+            const int hf = u & 1, j = u >> 1;
+            if (!mbar_wait(&bar.s_full[hf], (u >> 1) & 1)) { fail(); ok = false; break; }
             tc_fence_after();
-            uint32_t sr[kT], pr_[kT];
-#pragma unroll
-            for (int c = 0; c < kT; c += 32) {
-                tmem_ld_x32(tS + c, *reinterpret_cast<uint32_t(*)[32]>(&sr[c]));
-                tmem_ld_x32(tS + kT + c, *reinterpret_cast<uint32_t(*)[32]>(&pr_[c]));
-            }
+            const uint32_t tb = tS + hf * 128;
+            uint32_t sr[32], pr_[32];
+            tmem_ld_x32(tb + cg * 32, sr);
+            tmem_ld_x32(tb + kSub + cg * 32, pr_);
             tmem_ld_wait();
             const int ks = j < nt0 ? 0 : 1;
-            const int valid = p.n[ks] - (j - (ks ? nt0 : 0)) * kT;   // key columns < valid are real
+            // key columns < valid of this warp's 32 are real
+            const int valid = p.n[ks] - (j - (ks ? nt0 : 0)) * kT - hf * kSub - cg * 32;
 #pragma unroll
-            for (int i = 0; i < kT; i += 2) {
+            for (int i = 0; i < 32; i += 2) {
                 float ds[2];
 #pragma unroll
-                for (int u = 0; u < 2; ++u) {
-                    const float pv = ex2(fmaf(__uint_as_float(sr[i + u]), p.scale_log2, -lse));
-                    ds[u] = (i + u < valid && live) ? pv * (__uint_as_float(pr_[i + u]) - dd) : 0.f;
+                for (int e = 0; e < 2; ++e) {
+                    const float pv = ex2(fmaf(__uint_as_float(sr[i + e]), p.scale_log2, -lse));
+                    ds[e] = (i + e < valid && live) ? pv * (__uint_as_float(pr_[i + e]) - dd) : 0.f;
                 }
                 sr[i / 2] = pack_bf16x2(ds[0], ds[1]);
             }
-#pragma unroll
-            for (int c = 0; c < kT / 2; c += 32) tmem_st_x32(tS + c, &sr[c]);
+            // packed over this warp's own (already read) S columns
+            tmem_st_x16(tb + cg * 32, sr);
             tmem_st_wait();
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&bar.p_full);
+            if (lane == 0) mbar_arrive(&bar.p_full[hf]);
         }
         if (ok && mbar_wait(&bar.done, 0)) {
             tc_fence_after();
-            store_row_bf16(tS + 2 * kT, p.scale,
-                           p.dqkv[seg] + (static_cast<int64_t>(b) * p.n[seg] + row) * p.ldd[seg] + h * HD, live);
+            store_row_bf16(tS + 256 + cg * 64, p.scale,
+                           p.dqkv[seg] + (static_cast<int64_t>(b) * p.n[seg] + row) * p.ldd[seg] + h * HD + cg * 64,
+                           live, 64);
         } else if (ok) {
             fail();
         }
@@ -284,20 +320,25 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_con
 }
 
 // ------------------------------------------------------------------ dK, dV
-// TMEM: S^T at 0, dP^T at 128, dV at 256, dK at 384 (P^T and dS^T as bf16
-// pairs over the first 64 columns of S^T and dP^T).  Shared memory: the K
-// and V tiles of this CTA, then a ring of Q_i / dO_i tiles, then lse / D of
-// each streamed query tile.
+// TMEM: two sub-tile buffers of 128 columns, buffer b holding S^T (64 query
+// columns) at 128 b and dP^T at 128 b + 64; each elementwise warp writes its
+// 32 columns of P^T and dS^T as bf16 pairs over the first 16 of its own S^T /
+// dP^T columns; dV at 256, dK at 384.  Query tile i is
+// processed as two 64-query halves, half b in buffer b, overlapping the
+// elementwise work of one buffer with the MMAs of the other.  Shared memory:
+// the K and V tiles of this CTA, then a ring of Q_i / dO_i tiles, then lse /
+// D of each streamed query tile.
 __global__ void __launch_bounds__(kThreads, 1)
 attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_constant__ CUtensorMap tm_qkv1,
                      const __grid_constant__ CUtensorMap tm_do0, const __grid_constant__ CUtensorMap tm_do1,
                      const BwdParams p, int* status) {
+    constexpr int S_ = kSlotsDkdv;
     extern __shared__ __align__(1024) uint8_t smem[];
     uint8_t* sK = smem;
     uint8_t* sV = smem + kTileBytes;
-    uint8_t* sQD = smem + 2 * kTileBytes;                     // [kSlots][tile]: Q_i, dO_i, Q_i+1, ...
-    float* sLD = reinterpret_cast<float*>(sQD + kSlots * kTileBytes);   // [kSlots / 2][2][kT]: lse, D
-    Bars& bar = *reinterpret_cast<Bars*>(reinterpret_cast<uint8_t*>(sLD) + (kSlots / 2) * 2 * kT * 4);
+    uint8_t* sQD = smem + 2 * kTileBytes;                     // [S_][tile]: Q_i, dO_i, Q_i+1, ...
+    float* sLD = reinterpret_cast<float*>(sQD + S_ * kTileBytes);   // [S_ / 2][2][kT]: lse, D
+    Bars& bar = *reinterpret_cast<Bars*>(reinterpret_cast<uint8_t*>(sLD) + (S_ / 2) * 2 * kT * 4);
     volatile int* abort_flag = &bar.abort_flag;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int b = blockIdx.z, h = blockIdx.y;
@@ -313,12 +354,14 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_c
             *abort_flag = 1;
         }
         mbar_init(&bar.fixed_full, 1);
-        for (int s = 0; s < kSlots; ++s) {
+        for (int s = 0; s < S_; ++s) {
             mbar_init(&bar.slot_full[s], 1);
             mbar_init(&bar.slot_empty[s], 1);
         }
-        mbar_init(&bar.s_full, 1);
-        mbar_init(&bar.p_full, 4);
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(&bar.s_full[s], 1);
+            mbar_init(&bar.p_full[s], kEw);
+        }
         mbar_init(&bar.done, 1);
         mbar_init(&bar.drain, 1);
         fence_mbar_init();
@@ -346,8 +389,8 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_c
             tma_load_2d(sV + c * (kT * 128), tk, &bar.fixed_full, 2 * p.H + h * HD + c * 64, b * p.n[seg] + k0);
         }
         for (int n = 0; n < 2 * ntiles; ++n) {
-            const int s = n % kSlots;
-            if (!mbar_wait(&bar.slot_empty[s], ((n / kSlots) & 1) ^ 1)) { fail(); break; }
+            const int s = n % S_;
+            if (!mbar_wait(&bar.slot_empty[s], ((n / S_) & 1) ^ 1)) { fail(); break; }
             const int i = n >> 1;
             const int qs = i < nt0 ? 0 : 1;
             const int qi = (i - (qs ? nt0 : 0)) * kT;
@@ -369,96 +412,116 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_c
         }
     } else if (warp == 1 && lane == 0) {
         // ---- MMA issuer
-        constexpr uint32_t idesc_s = idesc_bf16_f32(kT, kT);
-        constexpr uint32_t idesc_g = idesc_bf16_f32(kT, HD) | (1u << 16);   // B = Q_i / dO_i, MN-major
+        constexpr uint32_t idesc_s = idesc_bf16_f32(kT, kSub);
+        constexpr uint32_t idesc_g = idesc_bf16_f32(kT, HD) | (1u << 16);   // B = Q_i / dO_i half, MN-major
         bool ok = mbar_wait(&bar.fixed_full, 0);
         if (!ok) fail();
         const uint64_t dk_ = smem_desc_k_sw128(smem_u32(sK));
         const uint64_t dv_ = smem_desc_k_sw128(smem_u32(sV));
-        for (int i = 0; ok && i < ntiles; ++i) {
+        auto wait_qd = [&](int i) {
             const int nq = 2 * i, nd = 2 * i + 1;
-            if (!mbar_wait(&bar.slot_full[nq % kSlots], (nq / kSlots) & 1) ||
-                !mbar_wait(&bar.slot_full[nd % kSlots], (nd / kSlots) & 1)) { fail(); ok = false; break; }
-            tc_fence_after();
-            const uint32_t aQ = smem_u32(sQD + (nq % kSlots) * kTileBytes);
-            const uint32_t aD = smem_u32(sQD + (nd % kSlots) * kTileBytes);
+            return mbar_wait(&bar.slot_full[nq % S_], (nq / S_) & 1) && mbar_wait(&bar.slot_full[nd % S_], (nd / S_) & 1);
+        };
+        // S^T = K Q^T and dP^T = V dO^T of query half hf of tile i into buffer hf
+        auto issue_sdp = [&](int i, int hf) {
+            const uint32_t aQ = smem_u32(sQD + ((2 * i) % S_) * kTileBytes) + hf * (kSub * 128);
+            const uint32_t aD = smem_u32(sQD + ((2 * i + 1) % S_) * kTileBytes) + hf * (kSub * 128);
             const uint64_t dq_ = smem_desc_k_sw128(aQ), ddo = smem_desc_k_sw128(aD);
+            const uint32_t tb = tmem + hf * 128;
 #pragma unroll
             for (int k = 0; k < HD / 16; ++k) {
                 const uint32_t off = ((k / 4) * (kT * 128) + (k % 4) * 32) >> 4;
-                tc_mma_bf16(tmem, dk_ + off, dq_ + off, idesc_s, k != 0 ? 1u : 0u);        // S^T = K Q^T
-                tc_mma_bf16(tmem + kT, dv_ + off, ddo + off, idesc_s, k != 0 ? 1u : 0u);   // dP^T = V dO^T
+                tc_mma_bf16(tb, dk_ + off, dq_ + off, idesc_s, k != 0 ? 1u : 0u);
+                tc_mma_bf16(tb + kSub, dv_ + off, ddo + off, idesc_s, k != 0 ? 1u : 0u);
             }
-            tc_commit(&bar.s_full);
-            if (!mbar_wait(&bar.p_full, i & 1)) { fail(); ok = false; break; }
+            tc_commit(&bar.s_full[hf]);
+        };
+        if (ok && !wait_qd(0)) { fail(); ok = false; }
+        if (ok) {
             tc_fence_after();
+            issue_sdp(0, 0);
+            issue_sdp(0, 1);
+        }
+        for (int u = 0; ok && u < 2 * ntiles; ++u) {
+            const int hf = u & 1, i = u >> 1;
+            if (!mbar_wait(&bar.p_full[hf], (u >> 1) & 1)) { fail(); ok = false; break; }
+            tc_fence_after();
+            const uint32_t aQ = smem_u32(sQD + ((2 * i) % S_) * kTileBytes) + hf * (kSub * 128);
+            const uint32_t aD = smem_u32(sQD + ((2 * i + 1) % S_) * kTileBytes) + hf * (kSub * 128);
             const uint64_t ddom = smem_desc_mn_sw128(aD, kT * 128), dqm = smem_desc_mn_sw128(aQ, kT * 128);
 #pragma unroll
-            for (int k = 0; k < kT / 16; ++k) {
+            for (int k = 0; k < kSub / 16; ++k) {
                 const uint64_t step = static_cast<uint64_t>(k * (2048 >> 4));
-                tc_mma_bf16_ts(tmem + 2 * kT, tmem + k * 8, ddom + step, idesc_g, (i | k) != 0 ? 1u : 0u);  // dV += P^T dO
-                tc_mma_bf16_ts(tmem + 3 * kT, tmem + kT + k * 8, dqm + step, idesc_g, (i | k) != 0 ? 1u : 0u);  // dK += dS^T Q
+                const uint32_t acc = (u | k) != 0 ? 1u : 0u;
+                // queries 16k.. of the half: packed at (k / 2) * 32 + (k % 2) * 8
+                const uint32_t a = tmem + hf * 128 + (k >> 1) * 32 + (k & 1) * 8;
+                tc_mma_bf16_ts(tmem + 256, a, ddom + step, idesc_g, acc);          // dV += P^T dO
+                tc_mma_bf16_ts(tmem + 384, a + kSub, dqm + step, idesc_g, acc);   // dK += dS^T Q
             }
-            tc_commit(&bar.slot_empty[nq % kSlots]);
-            tc_commit(&bar.slot_empty[nd % kSlots]);
+            if (hf == 1) {
+                tc_commit(&bar.slot_empty[(2 * i) % S_]);
+                tc_commit(&bar.slot_empty[(2 * i + 1) % S_]);
+            }
+            if (i + 1 < ntiles) {
+                if (hf == 0 && !wait_qd(i + 1)) { fail(); ok = false; break; }
+                tc_fence_after();
+                issue_sdp(i + 1, hf);
+            }
         }
         if (ok) tc_commit(&bar.done);
         tc_commit(&bar.drain);
         if (!mbar_wait(&bar.drain, 0)) report_status(status, kStatusWaitTimeout);
     } else if (warp >= 2) {
-        // ---- elementwise: thread = key row = TMEM lane
+        // ---- elementwise: thread = key row = TMEM lane; the two warps of a
+        // lane quarter take 32 query columns each of a sub-tile
         const int q = warp & 3;
+        const int cg = (warp - 2) >> 2;
         const int r = q * 32 + lane;
         const int row = k0 + r;
         const uint32_t tS = tmem + (static_cast<uint32_t>(q * 32) << 16);
         const bool live = row < p.n[seg];
         bool ok = true;
-        for (int i = 0; i < ntiles; ++i) {
-            if (!mbar_wait(&bar.s_full, i & 1)) { fail(); ok = false; break; }
+        for (int u = 0; u < 2 * ntiles; ++u) {
+            const int hf = u & 1, i = u >> 1;
+            if (!mbar_wait(&bar.s_full[hf], (u >> 1) & 1)) { fail(); ok = false; break; }
             tc_fence_after();
             const int nd = 2 * i + 1;
-            const float* lse = sLD + ((nd % kSlots) >> 1) * 2 * kT;
+            const float* lse = sLD + ((nd % S_) >> 1) * 2 * kT + hf * kSub + cg * 32;
             const float* dl = lse + kT;
             const int qs = i < nt0 ? 0 : 1;
-            const int valid = p.n[qs] - (i - (qs ? nt0 : 0)) * kT;   // query columns < valid are real
-            // two halves of 64 query columns; a half's bf16 P^T / dS^T land on
-            // columns whose fp32 values this thread has already read
-#pragma unroll 1
-            for (int hf = 0; hf < 2; ++hf) {
-                uint32_t sr[kT / 2], pr_[kT / 2];
+            // query columns < valid of this warp's 32 are real
+            const int valid = p.n[qs] - (i - (qs ? nt0 : 0)) * kT - hf * kSub - cg * 32;
+            const uint32_t tb = tS + hf * 128;
+            uint32_t sr[32], pr_[32];
+            tmem_ld_x32(tb + cg * 32, sr);
+            tmem_ld_x32(tb + kSub + cg * 32, pr_);
+            tmem_ld_wait();
 #pragma unroll
-                for (int c = 0; c < kT / 2; c += 32) {
-                    tmem_ld_x32(tS + hf * (kT / 2) + c, *reinterpret_cast<uint32_t(*)[32]>(&sr[c]));
-                    tmem_ld_x32(tS + kT + hf * (kT / 2) + c, *reinterpret_cast<uint32_t(*)[32]>(&pr_[c]));
+            for (int c = 0; c < 32; c += 2) {
+                float pv[2], ds[2];
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    const bool real = c + e < valid;
+                    const float x = ex2(fmaf(__uint_as_float(sr[c + e]), p.scale_log2, -lse[c + e]));
+                    pv[e] = real ? x : 0.f;
+                    ds[e] = real ? x * (__uint_as_float(pr_[c + e]) - dl[c + e]) : 0.f;
                 }
-                tmem_ld_wait();
-#pragma unroll
-                for (int c = 0; c < kT / 2; c += 2) {
-                    float pv[2], ds[2];
-#pragma unroll
-                    for (int u = 0; u < 2; ++u) {
-                        const int col = hf * (kT / 2) + c + u;
-                        const bool real = col < valid;
-                        const float e = ex2(fmaf(__uint_as_float(sr[c + u]), p.scale_log2, -lse[col]));
-                        pv[u] = real ? e : 0.f;
-                        ds[u] = real ? e * (__uint_as_float(pr_[c + u]) - dl[col]) : 0.f;
-                    }
-                    sr[c / 2] = pack_bf16x2(pv[0], pv[1]);
-                    pr_[c / 2] = pack_bf16x2(ds[0], ds[1]);
-                }
-                tmem_st_x32(tS + hf * (kT / 4), sr);
-                tmem_st_x32(tS + kT + hf * (kT / 4), pr_);
+                sr[c / 2] = pack_bf16x2(pv[0], pv[1]);
+                pr_[c / 2] = pack_bf16x2(ds[0], ds[1]);
             }
+            // packed over this warp's own (already read) S^T / dP^T columns
+            tmem_st_x16(tb + cg * 32, sr);
+            tmem_st_x16(tb + kSub + cg * 32, pr_);
             tmem_st_wait();
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&bar.p_full);
+            if (lane == 0) mbar_arrive(&bar.p_full[hf]);
         }
         if (ok && mbar_wait(&bar.done, 0)) {
             tc_fence_after();
             __nv_bfloat16* dst = p.dqkv[seg] + (static_cast<int64_t>(b) * p.n[seg] + row) * p.ldd[seg];
-            store_row_bf16(tS + 2 * kT, 1.0f, dst + 2 * p.H + h * HD, live);      // dV
-            store_row_bf16(tS + 3 * kT, p.scale, dst + p.H + h * HD, live);       // dK
+            if (cg == 0) store_row_bf16(tS + 256, 1.0f, dst + 2 * p.H + h * HD, live);   // dV
+            else store_row_bf16(tS + 384, p.scale, dst + p.H + h * HD, live);           // dK
         } else if (ok) {
             fail();
         }
@@ -476,8 +539,8 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_c
     }
 }
 
-constexpr int kSmemDq = 2 * kTileBytes + kSlots * kTileBytes + kBarBytes;
-constexpr int kSmemDkdv = 2 * kTileBytes + kSlots * kTileBytes + (kSlots / 2) * 2 * kT * 4 + kBarBytes;
+constexpr int kSmemDq = 2 * kTileBytes + kSlotsDq * kTileBytes + kBarBytes;
+constexpr int kSmemDkdv = 2 * kTileBytes + kSlotsDkdv * kTileBytes + (kSlotsDkdv / 2) * 2 * kT * 4 + kBarBytes;
 static_assert(sizeof(Bars) <= kBarBytes, "barrier block too small");
 
 }  // namespace
