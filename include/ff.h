@@ -375,7 +375,7 @@ int ff_dit_velocity(const ff_dit* model, int B, const float* x_t, const void* tx
                     cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
- * Training pass of the velocity network (MMDiT models, head_dim 128): the
+ * Training pass of the velocity network (MMDiT models): the
  * forward every GRPO-style trainer runs "again for training" (Sec. 1) and
  * its gradient, for the policy losses of Sec. 3 (the Flow-GRPO loss through
  * ff_sde_logprob_backward, AWM's Eq. 3 through ff_awm_loss's dL/dv).
@@ -432,7 +432,7 @@ int ff_gemm(int M, int N, int K, const void* A, int64_t lda, int a_layout, const
  * L = ff_attention_lse_rows(n0, n1) = pad128(n0) + pad128(n1): the base-2
  * log-sum-exp of the scaled scores of segment-0 row r at r and of segment-1
  * row r at pad128(n0) + r (padding rows are not written).
- * ff_attention_backward (head_dim 128) takes O, its gradient dO (same
+ * ff_attention_backward (head_dim 64 or 128) takes O, its gradient dO (same
  * layout and pitch ldo) and lse, and writes dq, dk, dv into dqkv buffers laid
  * out like qkv (columns h d, H + h d, 2H + h d; pitch ldd; other columns are
  * not touched).  ws: ff_attention_backward_workspace_size bytes (holds

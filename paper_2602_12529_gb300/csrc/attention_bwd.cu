@@ -1,5 +1,5 @@
 // attention_bwd.cu -- backward of the joint attention O = softmax(Q K^T / sqrt(d)) V
-// (d = 128) on tcgen05, for the training pass that follows the rollout
+// (d = 64 or 128) on tcgen05, for the training pass that follows the rollout
 // (paper Sec. 3.1: the policy gradient through the velocity network).
 //
 // With P = softmax(S), S = Q K^T a (a = 1/sqrt(d)) per (sample, head) and the
@@ -28,9 +28,7 @@
 namespace ff {
 namespace {
 
-constexpr int HD = 128;
 constexpr int kT = 128;                        // rows of a query / key tile
-constexpr int kTileBytes = kT * HD * 2;         // 32 KB: one bf16 tile (two 64-column boxes)
 constexpr int kSub = 64;                        // query / key columns of one S (S^T) sub-tile
 constexpr int kSlotsDq = 5;                     // streamed K / V tiles in flight (dQ kernel)
 constexpr int kSlotsDkdv = 4;                   // streamed Q / dO tiles in flight (dK dV kernel)
@@ -72,7 +70,7 @@ __device__ __forceinline__ void bulk_load_1d(void* dst, const void* src, uint32_
 
 // Stores `cols` fp32 TMEM columns of this thread's row as bf16 (times mul).
 __device__ __forceinline__ void store_row_bf16(uint32_t taddr, float mul, __nv_bfloat16* dst, bool live,
-                                               int cols = HD) {
+                                               int cols) {
 #pragma unroll 1
     for (int c = 0; c < cols; c += 32) {
         uint32_t o[32];
@@ -90,7 +88,8 @@ __device__ __forceinline__ void store_row_bf16(uint32_t taddr, float mul, __nv_b
     }
 }
 
-// D_i = sum_c dO_ic O_ic: one warp per (token row, head), 4 columns per lane.
+// D_i = sum_c dO_ic O_ic: one warp per (token row, head), HD / 32 columns per lane.
+template <int HD>
 __global__ void __launch_bounds__(256) attn_bwd_delta_kernel(int B, int heads, int n0, int n1,
                                                              const __nv_bfloat16* o0, const __nv_bfloat16* do0,
                                                              const __nv_bfloat16* o1, const __nv_bfloat16* do1,
@@ -108,13 +107,16 @@ __global__ void __launch_bounds__(256) attn_bwd_delta_kernel(int B, int heads, i
     const int n = s1 ? n1 : n0;
     const int b = static_cast<int>(rr / n);
     const int row = static_cast<int>(rr - static_cast<int64_t>(b) * n);
-    const __nv_bfloat16* o = (s1 ? o1 : o0) + rr * (s1 ? ldo1 : ldo0) + h * HD + lane * 4;
-    const __nv_bfloat16* g = (s1 ? do1 : do0) + rr * (s1 ? ldg1 : ldg0) + h * HD + lane * 4;
-    const uint2 ov = *reinterpret_cast<const uint2*>(o);
-    const uint2 gv = *reinterpret_cast<const uint2*>(g);
-    const float2 o01 = unpack_bf16x2(ov.x), o23 = unpack_bf16x2(ov.y);
-    const float2 g01 = unpack_bf16x2(gv.x), g23 = unpack_bf16x2(gv.y);
-    float s = o01.x * g01.x + o01.y * g01.y + o23.x * g23.x + o23.y * g23.y;
+    constexpr int E = HD / 32;
+    const __nv_bfloat16* o = (s1 ? o1 : o0) + rr * (s1 ? ldo1 : ldo0) + h * HD + lane * E;
+    const __nv_bfloat16* g = (s1 ? do1 : do0) + rr * (s1 ? ldg1 : ldg0) + h * HD + lane * E;
+    float s = 0.f;
+#pragma unroll
+    for (int e = 0; e < E; e += 2) {
+        const float2 of = unpack_bf16x2(*reinterpret_cast<const uint32_t*>(o + e));
+        const float2 gf = unpack_bf16x2(*reinterpret_cast<const uint32_t*>(g + e));
+        s = fmaf(of.x, gf.x, fmaf(of.y, gf.y, s));
+    }
 #pragma unroll
     for (int k = 16; k; k >>= 1) s += __shfl_xor_sync(0xffffffffu, s, k);
     if (lane == 0) delta[(static_cast<int64_t>(b) * heads + h) * lse_rows + (s1 ? base1 : 0) + row] = s;
@@ -125,15 +127,18 @@ __global__ void __launch_bounds__(256) attn_bwd_delta_kernel(int B, int heads, i
 // columns) at 128 b and dP at 128 b + 64; the two elementwise warps of a
 // lane quarter take 32 key columns each and write their dS as bf16 pairs over
 // the first 16 of their own S columns (keys 0-31 at 0, keys 32-63 at 32); dQ
-// at 256.  Key tile j is processed as two 64-key
+// (d columns) at 256.  Key tile j is processed as two 64-key
 // halves, half b in buffer b, so the elementwise warps work on one buffer
 // while the MMAs of the other (dQ += dS K, then the next half's S and dP)
 // run.  Shared memory: Q tile, dO tile, then a ring of K_j / V_j tiles.
+template <int HD>
 __global__ void __launch_bounds__(kThreads, 1)
 attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_constant__ CUtensorMap tm_qkv1,
                    const __grid_constant__ CUtensorMap tm_do0, const __grid_constant__ CUtensorMap tm_do1,
                    const BwdParams p, int* status) {
     constexpr int S_ = kSlotsDq;
+    constexpr int kTileBytes = kT * HD * 2;              // one bf16 tile: HD / 64 boxes of 128 rows x 64 columns
+    constexpr int NB = HD / 64;
     extern __shared__ __align__(1024) uint8_t smem[];
     uint8_t* sQ = smem;
     uint8_t* sdO = smem + kTileBytes;
@@ -183,7 +188,7 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_con
         const CUtensorMap* tq = seg ? &tm_qkv1 : &tm_qkv0;
         const CUtensorMap* td = seg ? &tm_do1 : &tm_do0;
         mbar_arrive_expect_tx(&bar.fixed_full, 2 * kTileBytes);
-        for (int c = 0; c < 2; ++c) {
+        for (int c = 0; c < NB; ++c) {
             tma_load_2d(sQ + c * (kT * 128), tq, &bar.fixed_full, h * HD + c * 64, b * p.n[seg] + q0);
             tma_load_2d(sdO + c * (kT * 128), td, &bar.fixed_full, h * HD + c * 64, b * p.n[seg] + q0);
         }
@@ -196,7 +201,7 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_con
             const int col = ((n & 1) ? 2 * p.H : p.H) + h * HD;
             uint8_t* dst = sKV + s * kTileBytes;
             mbar_arrive_expect_tx(&bar.slot_full[s], kTileBytes);
-            for (int c = 0; c < 2; ++c)
+            for (int c = 0; c < NB; ++c)
                 tma_load_2d(dst + c * (kT * 128), ks ? &tm_qkv1 : &tm_qkv0, &bar.slot_full[s], col + c * 64, row);
         }
     } else if (warp == 1 && lane == 0) {
@@ -299,9 +304,9 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_con
         }
         if (ok && mbar_wait(&bar.done, 0)) {
             tc_fence_after();
-            store_row_bf16(tS + 256 + cg * 64, p.scale,
-                           p.dqkv[seg] + (static_cast<int64_t>(b) * p.n[seg] + row) * p.ldd[seg] + h * HD + cg * 64,
-                           live, 64);
+            store_row_bf16(tS + 256 + cg * (HD / 2), p.scale,
+                           p.dqkv[seg] + (static_cast<int64_t>(b) * p.n[seg] + row) * p.ldd[seg] + h * HD + cg * (HD / 2),
+                           live, HD / 2);
         } else if (ok) {
             fail();
         }
@@ -323,16 +328,19 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_con
 // TMEM: two sub-tile buffers of 128 columns, buffer b holding S^T (64 query
 // columns) at 128 b and dP^T at 128 b + 64; each elementwise warp writes its
 // 32 columns of P^T and dS^T as bf16 pairs over the first 16 of its own S^T /
-// dP^T columns; dV at 256, dK at 384.  Query tile i is
+// dP^T columns; dV at 256, dK at 256 + d.  Query tile i is
 // processed as two 64-query halves, half b in buffer b, overlapping the
 // elementwise work of one buffer with the MMAs of the other.  Shared memory:
 // the K and V tiles of this CTA, then a ring of Q_i / dO_i tiles, then lse /
 // D of each streamed query tile.
+template <int HD>
 __global__ void __launch_bounds__(kThreads, 1)
 attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_constant__ CUtensorMap tm_qkv1,
                      const __grid_constant__ CUtensorMap tm_do0, const __grid_constant__ CUtensorMap tm_do1,
                      const BwdParams p, int* status) {
     constexpr int S_ = kSlotsDkdv;
+    constexpr int kTileBytes = kT * HD * 2;
+    constexpr int NB = HD / 64;
     extern __shared__ __align__(1024) uint8_t smem[];
     uint8_t* sK = smem;
     uint8_t* sV = smem + kTileBytes;
@@ -384,7 +392,7 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_c
         // and dO_i (one slot each) with lse_i / D_i riding on dO_i's barrier
         const CUtensorMap* tk = seg ? &tm_qkv1 : &tm_qkv0;
         mbar_arrive_expect_tx(&bar.fixed_full, 2 * kTileBytes);
-        for (int c = 0; c < 2; ++c) {
+        for (int c = 0; c < NB; ++c) {
             tma_load_2d(sK + c * (kT * 128), tk, &bar.fixed_full, p.H + h * HD + c * 64, b * p.n[seg] + k0);
             tma_load_2d(sV + c * (kT * 128), tk, &bar.fixed_full, 2 * p.H + h * HD + c * 64, b * p.n[seg] + k0);
         }
@@ -399,13 +407,13 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_c
             if (n & 1) {
                 float* ld = sLD + (s >> 1) * 2 * kT;
                 mbar_arrive_expect_tx(&bar.slot_full[s], kTileBytes + 2 * kT * 4);
-                for (int c = 0; c < 2; ++c)
+                for (int c = 0; c < NB; ++c)
                     tma_load_2d(dst + c * (kT * 128), qs ? &tm_do1 : &tm_do0, &bar.slot_full[s], h * HD + c * 64, row);
                 bulk_load_1d(ld, p.lse + lrow + p.lse_base[qs] + qi, kT * 4, &bar.slot_full[s]);
                 bulk_load_1d(ld + kT, p.delta + lrow + p.lse_base[qs] + qi, kT * 4, &bar.slot_full[s]);
             } else {
                 mbar_arrive_expect_tx(&bar.slot_full[s], kTileBytes);
-                for (int c = 0; c < 2; ++c)
+                for (int c = 0; c < NB; ++c)
                     tma_load_2d(dst + c * (kT * 128), qs ? &tm_qkv1 : &tm_qkv0, &bar.slot_full[s], h * HD + c * 64,
                                 row);
             }
@@ -455,8 +463,8 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_c
                 const uint32_t acc = (u | k) != 0 ? 1u : 0u;
                 // queries 16k.. of the half: packed at (k / 2) * 32 + (k % 2) * 8
                 const uint32_t a = tmem + hf * 128 + (k >> 1) * 32 + (k & 1) * 8;
-                tc_mma_bf16_ts(tmem + 256, a, ddom + step, idesc_g, acc);          // dV += P^T dO
-                tc_mma_bf16_ts(tmem + 384, a + kSub, dqm + step, idesc_g, acc);   // dK += dS^T Q
+                tc_mma_bf16_ts(tmem + 256, a, ddom + step, idesc_g, acc);              // dV += P^T dO
+                tc_mma_bf16_ts(tmem + 256 + HD, a + kSub, dqm + step, idesc_g, acc);   // dK += dS^T Q
             }
             if (hf == 1) {
                 tc_commit(&bar.slot_empty[(2 * i) % S_]);
@@ -520,8 +528,8 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_c
         if (ok && mbar_wait(&bar.done, 0)) {
             tc_fence_after();
             __nv_bfloat16* dst = p.dqkv[seg] + (static_cast<int64_t>(b) * p.n[seg] + row) * p.ldd[seg];
-            if (cg == 0) store_row_bf16(tS + 256, 1.0f, dst + 2 * p.H + h * HD, live);   // dV
-            else store_row_bf16(tS + 384, p.scale, dst + p.H + h * HD, live);           // dK
+            if (cg == 0) store_row_bf16(tS + 256, 1.0f, dst + 2 * p.H + h * HD, live, HD);     // dV
+            else store_row_bf16(tS + 256 + HD, p.scale, dst + p.H + h * HD, live, HD);    // dK
         } else if (ok) {
             fail();
         }
@@ -539,8 +547,10 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_c
     }
 }
 
-constexpr int kSmemDq = 2 * kTileBytes + kSlotsDq * kTileBytes + kBarBytes;
-constexpr int kSmemDkdv = 2 * kTileBytes + kSlotsDkdv * kTileBytes + (kSlotsDkdv / 2) * 2 * kT * 4 + kBarBytes;
+template <int HD>
+constexpr int smem_dq() { return 2 * kT * HD * 2 + kSlotsDq * kT * HD * 2 + kBarBytes; }
+template <int HD>
+constexpr int smem_dkdv() { return 2 * kT * HD * 2 + kSlotsDkdv * kT * HD * 2 + (kSlotsDkdv / 2) * 2 * kT * 4 + kBarBytes; }
 static_assert(sizeof(Bars) <= kBarBytes, "barrier block too small");
 
 }  // namespace
@@ -549,9 +559,12 @@ size_t attention_backward_ws_bytes(int B, int heads, int n0, int n1) {
     return static_cast<size_t>(B) * heads * attn_lse_rows(n0, n1) * sizeof(float);
 }
 
-int attention_backward(const AttnBwdSeg& s0, const AttnBwdSeg& s1, int B, int heads, int head_dim, const float* lse,
-                       void* ws, size_t ws_bytes, cudaStream_t stream) {
-    if (head_dim != HD) return set_error(FF_ERR_UNSUPPORTED, "attention backward: head_dim %d (128 only)", head_dim);
+namespace {
+
+template <int HD>
+int attention_backward_hd(const AttnBwdSeg& s0, const AttnBwdSeg& s1, int B, int heads, const float* lse, void* ws,
+                          size_t ws_bytes, cudaStream_t stream) {
+    constexpr int kSmemDq = smem_dq<HD>(), kSmemDkdv = smem_dkdv<HD>();
     if (B <= 0 || heads <= 0 || B > 65535 || heads > 65535 || s0.n < 0 || s1.n < 0 || s0.n + s1.n <= 0)
         return set_error(FF_ERR_INVALID_ARG, "attention backward: bad shape");
     if (!lse || !ws) return set_error(FF_ERR_INVALID_ARG, "attention backward: null lse or workspace");
@@ -568,8 +581,8 @@ int attention_backward(const AttnBwdSeg& s0, const AttnBwdSeg& s1, int B, int he
     const size_t need = attention_backward_ws_bytes(B, heads, s0.n, s1.n);
     if (ws_bytes < need || !aligned16(ws))
         return set_error(FF_ERR_WORKSPACE, "attention backward: workspace %zu B < %zu B", ws_bytes, need);
-    for (auto* f : {(const void*)attn_bwd_dq_kernel, (const void*)attn_bwd_dkdv_kernel}) {
-        const int bytes = f == (const void*)attn_bwd_dq_kernel ? kSmemDq : kSmemDkdv;
+    for (auto* f : {(const void*)attn_bwd_dq_kernel<HD>, (const void*)attn_bwd_dkdv_kernel<HD>}) {
+        const int bytes = f == (const void*)attn_bwd_dq_kernel<HD> ? kSmemDq : kSmemDkdv;
         if (cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) != cudaSuccess)
             return set_error(FF_ERR_CUDA, "attention backward: cannot set shared memory size");
     }
@@ -584,7 +597,7 @@ int attention_backward(const AttnBwdSeg& s0, const AttnBwdSeg& s1, int B, int he
     {
         const int64_t warps = (static_cast<int64_t>(B) * (s0.n + s1.n)) * heads;
         ProfScope prof(stream, "attn_bwd_delta", 0.0, 4.0 * warps * HD);
-        attn_bwd_delta_kernel<<<static_cast<unsigned>((warps + 7) / 8), 256, 0, stream>>>(
+        attn_bwd_delta_kernel<HD><<<static_cast<unsigned>((warps + 7) / 8), 256, 0, stream>>>(
             B, heads, s0.n, s1.n, s0.o, s0.dout, s1.o, s1.dout, s0.ldo, s1.ldo, s0.ldg ? s0.ldg : s0.ldo,
             s1.ldg ? s1.ldg : s1.ldo, rows, attn_pad128(s0.n), delta);
         FF_TRY(check_launch("attn_bwd_delta_kernel"));
@@ -609,14 +622,23 @@ int attention_backward(const AttnBwdSeg& s0, const AttnBwdSeg& s1, int B, int he
     const double N = static_cast<double>(s0.n + s1.n);
     {
         ProfScope prof(stream, "attn_bwd_dq", 6.0 * B * heads * N * N * HD, 0.0);
-        attn_bwd_dq_kernel<<<grid, kThreads, kSmemDq, stream>>>(tqkv[0], tqkv[1], tdo[0], tdo[1], p,
+        attn_bwd_dq_kernel<HD><<<grid, kThreads, kSmemDq, stream>>>(tqkv[0], tqkv[1], tdo[0], tdo[1], p,
                                                                  device_status_ptr());
         FF_TRY(check_launch("attn_bwd_dq_kernel"));
     }
     ProfScope prof(stream, "attn_bwd_dkdv", 8.0 * B * heads * N * N * HD, 0.0);
-    attn_bwd_dkdv_kernel<<<grid, kThreads, kSmemDkdv, stream>>>(tqkv[0], tqkv[1], tdo[0], tdo[1], p,
+    attn_bwd_dkdv_kernel<HD><<<grid, kThreads, kSmemDkdv, stream>>>(tqkv[0], tqkv[1], tdo[0], tdo[1], p,
                                                                  device_status_ptr());
     return check_launch("attn_bwd_dkdv_kernel");
+}
+
+}  // namespace
+
+int attention_backward(const AttnBwdSeg& s0, const AttnBwdSeg& s1, int B, int heads, int head_dim, const float* lse,
+                       void* ws, size_t ws_bytes, cudaStream_t stream) {
+    if (head_dim == 128) return attention_backward_hd<128>(s0, s1, B, heads, lse, ws, ws_bytes, stream);
+    if (head_dim == 64) return attention_backward_hd<64>(s0, s1, B, heads, lse, ws, ws_bytes, stream);
+    return set_error(FF_ERR_UNSUPPORTED, "attention backward: head_dim %d (64 or 128)", head_dim);
 }
 
 }  // namespace ff

@@ -139,7 +139,7 @@ int check_model(const ff_dit* m, int B) {
     if (B <= 0) return set_error(FF_ERR_INVALID_ARG, "B=%d must be positive", B);
     const ff_dit_config& c = model_config(m);
     if (c.arch != FF_ARCH_MMDIT) return set_error(FF_ERR_UNSUPPORTED, "training pass: MMDiT models only");
-    if (c.head_dim != 128) return set_error(FF_ERR_UNSUPPORTED, "training pass: head_dim %d (128 only)", c.head_dim);
+
     const int64_t Ni = static_cast<int64_t>(c.grid_f) * c.grid_h * c.grid_w;
     if ((static_cast<int64_t>(B) * c.n_txt) % 8 || (B * Ni) % 8)
         return set_error(FF_ERR_UNSUPPORTED, "training pass: B N_t and B N_i must be multiples of 8");

@@ -1,6 +1,6 @@
-"""GPU parity of the attention backward (dq, dk, dv) and of the forward's
-per-row log-sum-exp against the fp64 oracle, over joint [segment 0;
-segment 1] sequences with ragged segment lengths."""
+"""GPU parity of the attention backward (dq, dk, dv; head dim 64 and 128) and
+of the forward's per-row log-sum-exp against the fp64 oracle, over joint
+[segment 0; segment 1] sequences with ragged segment lengths."""
 import math
 
 import numpy as np
@@ -27,12 +27,12 @@ def _host(t):
     return odit.widen(t.view(torch.int16).cpu().numpy().view(np.uint16))
 
 
-@pytest.mark.parametrize("B,heads,n0,n1", [(2, 2, 5, 70), (1, 3, 32, 200), (2, 2, 0, 130), (1, 2, 300, 777),
-                                           (1, 2, 512, 4096)])
-def test_attention_backward_parity(cuda, B, heads, n0, n1):
+@pytest.mark.parametrize("d,B,heads,n0,n1", [(128, 2, 2, 5, 70), (128, 1, 3, 32, 200), (128, 2, 2, 0, 130),
+                                             (128, 1, 2, 300, 777), (128, 1, 2, 512, 4096),
+                                             (64, 4, 4, 32, 64), (64, 2, 2, 5, 70), (64, 1, 3, 300, 777)])
+def test_attention_backward_parity(cuda, d, B, heads, n0, n1):
     import torch
     from paper_2602_12529_gb300 import ffi
-    d = 128
     H = heads * d
     q0 = _bits((max(B * n0, 1), 3 * H), 31, "bq0")
     q1 = _bits((B * n1, 3 * H), 32, "bq1")

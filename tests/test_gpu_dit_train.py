@@ -88,9 +88,14 @@ def _compare(run, grad, dx, want_G, want_dx):
     assert rms_rel(dx, want_dx) <= G_TOL
 
 
+TINY64 = {k: v for k, v in synth.config("tiny_mmdit").items() if k in SMALL}
+
+
 @pytest.mark.parametrize("over", [{}, {"n_double": 2, "n_single": 0}, {"n_double": 0, "n_single": 2},
                                   {"grid": (1, 3, 5), "n_txt": 5, "batch": 8},
-                                  {"batch": 3, "n_txt": 8, "grid": (1, 4, 6)}])
+                                  {"batch": 3, "n_txt": 8, "grid": (1, 4, 6)},
+                                  dict(TINY64),
+                                  dict(TINY64, n_double=1, n_single=1, grid=(1, 3, 5), n_txt=5, batch=8)])
 def test_backward_matches_oracle(cuda, over):
     cfg = _cfg(**over)
     run = Run(cfg, cuda)
