@@ -349,18 +349,41 @@ __global__ void __launch_bounds__(kThreads) colsum_partial_kernel(const T* in, i
 // ---------------------------------------------------------------- chunk reduction
 
 // out[b * ld_out + j] = sum over sample b's chunks of every span (per_sample),
-// or out[j] = sum over all chunks of every span; fp64 in a fixed order.
-__global__ void reduce_chunks_kernel(const float* part, int64_t ld_part, int ncols, ChunkSpans sp, int per_sample,
-                                     float* out, int64_t ld_out) {
-    const int j = blockIdx.x * blockDim.x + threadIdx.x;
-    if (j >= ncols) return;
+// or out[j] = sum over all chunks of every span.  A CTA takes 32 columns
+// (lane = column, so a chunk row is one 128-byte load per warp); warp w takes
+// the chunks w, w + 8, ... in four interleaved fp64 chains, and the eight
+// warp sums are added in warp order: a fixed order for a given shape.
+__global__ void __launch_bounds__(256) reduce_chunks_kernel(const float* part, int64_t ld_part, int ncols,
+                                                            ChunkSpans sp, int per_sample, float* out,
+                                                            int64_t ld_out) {
+    __shared__ double red[8][32];
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    const int j = blockIdx.x * 32 + lane;
     const int b = blockIdx.y;
-    double s = 0.0;
-    for (int i = 0; i < sp.n; ++i) {
-        const int first = per_sample ? sp.first[i] + b * sp.count[i] : sp.first[i];
-        for (int c = 0; c < sp.count[i]; ++c) s += part[static_cast<int64_t>(first + c) * ld_part + j];
+    double acc[4] = {0.0, 0.0, 0.0, 0.0};
+    if (j < ncols) {
+        for (int i = 0; i < sp.n; ++i) {
+            const int first = per_sample ? sp.first[i] + b * sp.count[i] : sp.first[i];
+            const int cnt = sp.count[i];
+            const float* base = part + static_cast<int64_t>(first) * ld_part + j;
+            int c = w;
+            for (; c + 24 < cnt; c += 32) {
+                acc[0] += base[static_cast<int64_t>(c) * ld_part];
+                acc[1] += base[static_cast<int64_t>(c + 8) * ld_part];
+                acc[2] += base[static_cast<int64_t>(c + 16) * ld_part];
+                acc[3] += base[static_cast<int64_t>(c + 24) * ld_part];
+            }
+            for (; c < cnt; c += 8) acc[0] += base[static_cast<int64_t>(c) * ld_part];
+        }
     }
-    out[static_cast<int64_t>(b) * ld_out + j] = static_cast<float>(s);
+    red[w][lane] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+    __syncthreads();
+    if (w == 0 && j < ncols) {
+        double s = 0.0;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) s += red[k][lane];
+        out[static_cast<int64_t>(b) * ld_out + j] = static_cast<float>(s);
+    }
 }
 
 // ---------------------------------------------------------------- SiLU
@@ -384,7 +407,10 @@ __global__ void silu_backward_kernel(const float* dy, int64_t ld_dy, const __nv_
 
 int reduce(const float* part, int64_t ld_part, int ncols, const ChunkSpans& sp, int B, float* out, int64_t ld_out,
            cudaStream_t stream) {
-    dim3 grid((ncols + 255) / 256, B > 0 ? B : 1);
+    double chunks = 0.0;
+    for (int i = 0; i < sp.n; ++i) chunks += static_cast<double>(sp.count[i]) * (B > 0 ? B : 1);
+    ProfScope prof(stream, "reduce_chunks", 0.0, chunks * ncols * 4.0);
+    dim3 grid((ncols + 31) / 32, B > 0 ? B : 1);
     reduce_chunks_kernel<<<grid, 256, 0, stream>>>(part, ld_part, ncols, sp, B > 0, out, ld_out);
     return check_launch("reduce_chunks_kernel");
 }
