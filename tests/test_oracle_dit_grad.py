@@ -203,3 +203,75 @@ def test_sde_logprob_grad_zero_at_the_mean():
     t, tn, sig = np.array([0.8, 0.6]), np.array([0.6, 0.3]), np.array([0.5, 0.9])
     x_mean, _ = sde.sde_step_logprob(x, v, t, tn, sig, eps=np.zeros((2, 16)))
     np.testing.assert_allclose(sde.sde_logprob_grad_v(x, v, x_mean, t, tn, sig), 0, atol=1e-12)
+
+
+# ---------------------------------------------------------------- the WAN-style network
+
+WAN_TINY = dict(name="wan_grad", arch="wan", hidden=32, heads=2, head_dim=16, mlp=64,
+                n_double=2, n_single=0, patch_dim=8, txt_dim=24, n_txt=3, grid=(2, 2, 3),
+                rope_axes=(4, 6, 6), rope_theta=100.0, time_freq_dim=16, batch=2)
+
+
+def _wan_params(cfg, seed=0):
+    return dit.widen_params(synth.weights(dit.wan_param_specs(cfg), seed=seed, std=0.2,
+                                          bias_std=0.1, scale_std=0.2))
+
+
+@pytest.mark.parametrize("L", [1, 2])
+def test_wan_velocity_vjp_matches_central_differences(L):
+    cfg = dict(WAN_TINY, n_double=L)
+    P = _wan_params(cfg)
+    x, txt, t = _inputs(cfg)
+    rng = np.random.default_rng(21)
+    dv = rng.standard_normal((cfg["batch"], synth.n_img(cfg), cfg["patch_dim"]))
+    v, G, dx = dit_grad.wan_velocity_vjp(P, cfg, x, txt, t, dv)
+    np.testing.assert_allclose(v, dit.wan_velocity(P, cfg, x, txt, t), rtol=1e-12, atol=1e-12)
+
+    def loss(Pm, xm=x):
+        return float(np.sum(dv * dit.wan_velocity(Pm, cfg, xm, txt, t)))
+
+    h = 1e-5
+    for name in P:
+        d = rng.standard_normal(P[name].shape)
+        Pp, Pm = dict(P), dict(P)
+        Pp[name] = P[name] + h * d
+        Pm[name] = P[name] - h * d
+        num = (loss(Pp) - loss(Pm)) / (2 * h)
+        ana = float(np.sum(G[name] * d))
+        assert abs(num - ana) <= 1e-6 * max(1.0, abs(num)), (name, num, ana)
+    d = rng.standard_normal(x.shape)
+    num = (loss(P, x + h * d) - loss(P, x - h * d)) / (2 * h)
+    assert abs(num - float(np.sum(dx * d))) <= 1e-6 * max(1.0, abs(num))
+
+
+def test_wan_velocity_vjp_is_linear_in_dv():
+    cfg = WAN_TINY
+    P = _wan_params(cfg, seed=1)
+    x, txt, t = _inputs(cfg, seed=4)
+    rng = np.random.default_rng(22)
+    shape = (cfg["batch"], synth.n_img(cfg), cfg["patch_dim"])
+    d1, d2 = rng.standard_normal(shape), rng.standard_normal(shape)
+    _, G1, x1 = dit_grad.wan_velocity_vjp(P, cfg, x, txt, t, d1)
+    _, G2, x2 = dit_grad.wan_velocity_vjp(P, cfg, x, txt, t, d2)
+    _, G3, x3 = dit_grad.wan_velocity_vjp(P, cfg, x, txt, t, 2 * d1 - d2)
+    for k in P:
+        np.testing.assert_allclose(G3[k], 2 * G1[k] - G2[k], atol=1e-10)
+    np.testing.assert_allclose(x3, 2 * x1 - x2, atol=1e-10)
+
+
+def test_wan_bias_gradients_are_token_sums():
+    """final.b sums dv over every token; the final layer's shift bias
+    (final.mod.b[:H]) sums the final LN-modulate input gradient, which is
+    dv W_final; and a block's modulation bias gradient equals the
+    shared-modulation gradient summed over the blocks' own contributions."""
+    cfg = WAN_TINY
+    P = _wan_params(cfg, seed=2)
+    x, txt, t = _inputs(cfg, seed=5)
+    dv = np.random.default_rng(23).standard_normal((cfg["batch"], synth.n_img(cfg), cfg["patch_dim"]))
+    _, G, _ = dit_grad.wan_velocity_vjp(P, cfg, x, txt, t, dv)
+    H = cfg["hidden"]
+    np.testing.assert_allclose(G["final.b"], dv.sum(axis=(0, 1)), rtol=1e-13)
+    np.testing.assert_allclose(G["final.mod.b"][:H], (dv @ P["final.w"]).sum(axis=(0, 1)), rtol=1e-12)
+    # mod.b receives what every block's bias receives (e0 + b_l: same partials)
+    np.testing.assert_allclose(G["mod.b"], sum(G[f"blocks.{l}.mod.b"] for l in range(cfg["n_double"])),
+                               rtol=1e-12, atol=1e-14)
