@@ -450,6 +450,28 @@ int ff_attention_backward(int B, int heads, int head_dim, int n0, const void* qk
                           const float* lse, void* ws, size_t ws_bytes, cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
+ * Cross-attention of the WAN-style block (latent queries, text keys and
+ * values) with its backward.  Per sample and head h:
+ *   O = softmax(Q K^T / sqrt(d)) V,  q of head h at column h d of the query
+ *   rows (nq per sample, pitch ldq), k at column h d and v at H + h d of the
+ *   key / value rows (nk per sample, pitch ldkv), O at column h d (pitch ldo).
+ * ff_cross_attention_forward optionally writes lse (fp32, [B, heads,
+ * ff_attention_lse_rows(nq, 0)], base 2, as ff_attention_forward).
+ * ff_cross_attention_backward (head_dim 64 or 128) takes O, dO (pitch ldo)
+ * and lse and writes dq (head h at column h d, pitch lddq) and dk | dv (head
+ * h at columns h d and H + h d, pitch lddkv); ws:
+ * ff_attention_backward_workspace_size(B, heads, nq, 0) bytes.  nq, nk > 0;
+ * pitches multiples of 8 elements, buffers 16-byte aligned.
+ * ------------------------------------------------------------------------ */
+int ff_cross_attention_forward(int B, int heads, int head_dim, int nq, const void* q, int64_t ldq, int nk,
+                               const void* kv, int64_t ldkv, void* out, int64_t ldo, float* lse,
+                               cudaStream_t stream);
+int ff_cross_attention_backward(int B, int heads, int head_dim, int nq, const void* q, int64_t ldq,
+                                const void* out, const void* dout, int64_t ldo, void* dq, int64_t lddq,
+                                int nk, const void* kv, int64_t ldkv, void* dkv, int64_t lddkv,
+                                const float* lse, void* ws, size_t ws_bytes, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
  * Trajectory sampling (paper Sec. 3.1: the SDE rollout that Flow-GRPO's
  * policy gradient scores, "repeated forward passes for trajectory
  * sampling").  S denoise steps; at step k = 0 .. S-1, for every sample:

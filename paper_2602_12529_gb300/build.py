@@ -19,7 +19,7 @@ BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libff.so")
 
 SOURCES = ["runtime.cu", "gemm.cu", "attention.cu", "attention_bwd.cu", "elementwise.cu", "sde.cu", "grpo.cu", "awm.cu", "dit.cu",
-           "rollout.cu", "debug.cu", "backward.cu", "dit_train.cu"]
+           "rollout.cu", "debug.cu", "backward.cu", "dit_train.cu", "wan_train.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr", "-I", INCLUDE]
 

@@ -1,6 +1,10 @@
-// attention_bwd.cu -- backward of the joint attention O = softmax(Q K^T / sqrt(d)) V
+// attention_bwd.cu -- backward of the attention O = softmax(Q K^T / sqrt(d)) V
 // (d = 64 or 128) on tcgen05, for the training pass that follows the rollout
-// (paper Sec. 3.1: the policy gradient through the velocity network).
+// (paper Sec. 3.1: the policy gradient through the velocity network).  Queries
+// come from up to two query segments and keys / values from up to two key
+// segments, each with its own source buffer and columns: the joint
+// [text; image] self-attention of the MMDiT (the same rows on both sides) and
+// the WAN block's cross-attention (latent queries, text keys and values).
 //
 // With P = softmax(S), S = Q K^T a (a = 1/sqrt(d)) per (sample, head) and the
 // forward's per-row log-sum-exp (base 2, lse2 = log2 sum_j 2^(S_ij log2 e)):
@@ -38,16 +42,18 @@ constexpr int kEw = 8;                          // elementwise warps
 constexpr int kBarBytes = 256;
 
 struct BwdParams {
-    int n[2];              // tokens per sample of each segment (queries = keys)
-    int tiles0;            // 128-row tiles of segment 0 (segment 1's follow)
-    int H;                 // heads * d
+    int nq[2], nk[2];      // tokens per sample of each query / key segment
+    int qtiles0, ktiles0;  // 128-row tiles of query / key segment 0 (segment 1's follow)
+    int q_col, k_col, v_col;   // first column of head 0's q, k, v in the source rows
     float scale_log2;      // log2(e) / sqrt(d)
     float scale;           // 1 / sqrt(d)
     const float* lse;      // [B, heads, lse_rows] base-2 log-sum-exp of the forward
     const float* delta;    // D in the same layout
     int lse_rows, lse_base[2];
-    __nv_bfloat16* dqkv[2];
-    int64_t ldd[2];
+    __nv_bfloat16* dq[2];  // head h at column h d
+    int64_t ldq[2];
+    __nv_bfloat16 *dk[2], *dv[2];
+    int64_t ldkv[2];
 };
 
 struct Bars {
@@ -133,7 +139,8 @@ __global__ void __launch_bounds__(256) attn_bwd_delta_kernel(int B, int heads, i
 // run.  Shared memory: Q tile, dO tile, then a ring of K_j / V_j tiles.
 template <int HD>
 __global__ void __launch_bounds__(kThreads, 1)
-attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_constant__ CUtensorMap tm_qkv1,
+attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_constant__ CUtensorMap tm_q1,
+                   const __grid_constant__ CUtensorMap tm_kv0, const __grid_constant__ CUtensorMap tm_kv1,
                    const __grid_constant__ CUtensorMap tm_do0, const __grid_constant__ CUtensorMap tm_do1,
                    const BwdParams p, int* status) {
     constexpr int S_ = kSlotsDq;
@@ -147,10 +154,10 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_con
     volatile int* abort_flag = &bar.abort_flag;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int b = blockIdx.z, h = blockIdx.y;
-    const int seg = blockIdx.x < p.tiles0 ? 0 : 1;
-    const int q0 = (blockIdx.x - (seg ? p.tiles0 : 0)) * kT;
-    const int nt0 = (p.n[0] + kT - 1) / kT;
-    const int ntiles = nt0 + (p.n[1] + kT - 1) / kT;
+    const int seg = blockIdx.x < p.qtiles0 ? 0 : 1;
+    const int q0 = (blockIdx.x - (seg ? p.qtiles0 : 0)) * kT;
+    const int nt0 = (p.nk[0] + kT - 1) / kT;
+    const int ntiles = nt0 + (p.nk[1] + kT - 1) / kT;
     if (threadIdx.x == 0) {
         *abort_flag = 0;
         if (smem_u32(smem) & 1023u) {
@@ -185,24 +192,24 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_con
     if (*abort_flag) {
     } else if (warp == 0 && lane == 0) {
         // ---- producer: Q and dO of this tile, then K_0, V_0, K_1, ...
-        const CUtensorMap* tq = seg ? &tm_qkv1 : &tm_qkv0;
+        const CUtensorMap* tq = seg ? &tm_q1 : &tm_q0;
         const CUtensorMap* td = seg ? &tm_do1 : &tm_do0;
         mbar_arrive_expect_tx(&bar.fixed_full, 2 * kTileBytes);
         for (int c = 0; c < NB; ++c) {
-            tma_load_2d(sQ + c * (kT * 128), tq, &bar.fixed_full, h * HD + c * 64, b * p.n[seg] + q0);
-            tma_load_2d(sdO + c * (kT * 128), td, &bar.fixed_full, h * HD + c * 64, b * p.n[seg] + q0);
+            tma_load_2d(sQ + c * (kT * 128), tq, &bar.fixed_full, p.q_col + h * HD + c * 64, b * p.nq[seg] + q0);
+            tma_load_2d(sdO + c * (kT * 128), td, &bar.fixed_full, h * HD + c * 64, b * p.nq[seg] + q0);
         }
         for (int n = 0; n < 2 * ntiles; ++n) {
             const int s = n % S_;
             if (!mbar_wait(&bar.slot_empty[s], ((n / S_) & 1) ^ 1)) { fail(); break; }
             const int j = n >> 1;
             const int ks = j < nt0 ? 0 : 1;
-            const int row = b * p.n[ks] + (j - (ks ? nt0 : 0)) * kT;
-            const int col = ((n & 1) ? 2 * p.H : p.H) + h * HD;
+            const int row = b * p.nk[ks] + (j - (ks ? nt0 : 0)) * kT;
+            const int col = ((n & 1) ? p.v_col : p.k_col) + h * HD;
             uint8_t* dst = sKV + s * kTileBytes;
             mbar_arrive_expect_tx(&bar.slot_full[s], kTileBytes);
             for (int c = 0; c < NB; ++c)
-                tma_load_2d(dst + c * (kT * 128), ks ? &tm_qkv1 : &tm_qkv0, &bar.slot_full[s], col + c * 64, row);
+                tma_load_2d(dst + c * (kT * 128), ks ? &tm_kv1 : &tm_kv0, &bar.slot_full[s], col + c * 64, row);
         }
     } else if (warp == 1 && lane == 0) {
         // ---- MMA issuer
@@ -269,7 +276,7 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_con
         const int row = q0 + r;
         const uint32_t tS = tmem + (static_cast<uint32_t>(q * 32) << 16);
         const int64_t li = (static_cast<int64_t>(b) * gridDim.y + h) * p.lse_rows + p.lse_base[seg] + row;
-        const bool live = row < p.n[seg];
+        const bool live = row < p.nq[seg];
         const float lse = live ? p.lse[li] : 0.f;
         const float dd = live ? p.delta[li] : 0.f;
         bool ok = true;
@@ -284,7 +291,7 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_con
             tmem_ld_wait();
             const int ks = j < nt0 ? 0 : 1;
             // key columns < valid of this warp's 32 are real
-            const int valid = p.n[ks] - (j - (ks ? nt0 : 0)) * kT - hf * kSub - cg * 32;
+            const int valid = p.nk[ks] - (j - (ks ? nt0 : 0)) * kT - hf * kSub - cg * 32;
 #pragma unroll
             for (int i = 0; i < 32; i += 2) {
                 float ds[2];
@@ -305,7 +312,7 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_con
         if (ok && mbar_wait(&bar.done, 0)) {
             tc_fence_after();
             store_row_bf16(tS + 256 + cg * (HD / 2), p.scale,
-                           p.dqkv[seg] + (static_cast<int64_t>(b) * p.n[seg] + row) * p.ldd[seg] + h * HD + cg * (HD / 2),
+                           p.dq[seg] + (static_cast<int64_t>(b) * p.nq[seg] + row) * p.ldq[seg] + h * HD + cg * (HD / 2),
                            live, HD / 2);
         } else if (ok) {
             fail();
@@ -335,7 +342,8 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_con
 // D of each streamed query tile.
 template <int HD>
 __global__ void __launch_bounds__(kThreads, 1)
-attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_constant__ CUtensorMap tm_qkv1,
+attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_constant__ CUtensorMap tm_q1,
+                     const __grid_constant__ CUtensorMap tm_kv0, const __grid_constant__ CUtensorMap tm_kv1,
                      const __grid_constant__ CUtensorMap tm_do0, const __grid_constant__ CUtensorMap tm_do1,
                      const BwdParams p, int* status) {
     constexpr int S_ = kSlotsDkdv;
@@ -350,10 +358,10 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_c
     volatile int* abort_flag = &bar.abort_flag;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int b = blockIdx.z, h = blockIdx.y;
-    const int seg = blockIdx.x < p.tiles0 ? 0 : 1;
-    const int k0 = (blockIdx.x - (seg ? p.tiles0 : 0)) * kT;
-    const int nt0 = (p.n[0] + kT - 1) / kT;
-    const int ntiles = nt0 + (p.n[1] + kT - 1) / kT;
+    const int seg = blockIdx.x < p.ktiles0 ? 0 : 1;
+    const int k0 = (blockIdx.x - (seg ? p.ktiles0 : 0)) * kT;
+    const int nt0 = (p.nq[0] + kT - 1) / kT;
+    const int ntiles = nt0 + (p.nq[1] + kT - 1) / kT;
     const int64_t lrow = (static_cast<int64_t>(b) * gridDim.y + h) * p.lse_rows;
     if (threadIdx.x == 0) {
         *abort_flag = 0;
@@ -390,11 +398,11 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_c
     } else if (warp == 0 && lane == 0) {
         // ---- producer: K and V of this tile, then per query tile i its Q_i
         // and dO_i (one slot each) with lse_i / D_i riding on dO_i's barrier
-        const CUtensorMap* tk = seg ? &tm_qkv1 : &tm_qkv0;
+        const CUtensorMap* tk = seg ? &tm_kv1 : &tm_kv0;
         mbar_arrive_expect_tx(&bar.fixed_full, 2 * kTileBytes);
         for (int c = 0; c < NB; ++c) {
-            tma_load_2d(sK + c * (kT * 128), tk, &bar.fixed_full, p.H + h * HD + c * 64, b * p.n[seg] + k0);
-            tma_load_2d(sV + c * (kT * 128), tk, &bar.fixed_full, 2 * p.H + h * HD + c * 64, b * p.n[seg] + k0);
+            tma_load_2d(sK + c * (kT * 128), tk, &bar.fixed_full, p.k_col + h * HD + c * 64, b * p.nk[seg] + k0);
+            tma_load_2d(sV + c * (kT * 128), tk, &bar.fixed_full, p.v_col + h * HD + c * 64, b * p.nk[seg] + k0);
         }
         for (int n = 0; n < 2 * ntiles; ++n) {
             const int s = n % S_;
@@ -402,7 +410,7 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_c
             const int i = n >> 1;
             const int qs = i < nt0 ? 0 : 1;
             const int qi = (i - (qs ? nt0 : 0)) * kT;
-            const int row = b * p.n[qs] + qi;
+            const int row = b * p.nq[qs] + qi;
             uint8_t* dst = sQD + s * kTileBytes;
             if (n & 1) {
                 float* ld = sLD + (s >> 1) * 2 * kT;
@@ -414,8 +422,8 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_c
             } else {
                 mbar_arrive_expect_tx(&bar.slot_full[s], kTileBytes);
                 for (int c = 0; c < NB; ++c)
-                    tma_load_2d(dst + c * (kT * 128), qs ? &tm_qkv1 : &tm_qkv0, &bar.slot_full[s], h * HD + c * 64,
-                                row);
+                    tma_load_2d(dst + c * (kT * 128), qs ? &tm_q1 : &tm_q0, &bar.slot_full[s],
+                                p.q_col + h * HD + c * 64, row);
             }
         }
     } else if (warp == 1 && lane == 0) {
@@ -487,7 +495,7 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_c
         const int r = q * 32 + lane;
         const int row = k0 + r;
         const uint32_t tS = tmem + (static_cast<uint32_t>(q * 32) << 16);
-        const bool live = row < p.n[seg];
+        const bool live = row < p.nk[seg];
         bool ok = true;
         for (int u = 0; u < 2 * ntiles; ++u) {
             const int hf = u & 1, i = u >> 1;
@@ -498,7 +506,7 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_c
             const float* dl = lse + kT;
             const int qs = i < nt0 ? 0 : 1;
             // query columns < valid of this warp's 32 are real
-            const int valid = p.n[qs] - (i - (qs ? nt0 : 0)) * kT - hf * kSub - cg * 32;
+            const int valid = p.nq[qs] - (i - (qs ? nt0 : 0)) * kT - hf * kSub - cg * 32;
             const uint32_t tb = tS + hf * 128;
             uint32_t sr[32], pr_[32];
             tmem_ld_x32(tb + cg * 32, sr);
@@ -527,9 +535,9 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_qkv0, const __grid_c
         }
         if (ok && mbar_wait(&bar.done, 0)) {
             tc_fence_after();
-            __nv_bfloat16* dst = p.dqkv[seg] + (static_cast<int64_t>(b) * p.n[seg] + row) * p.ldd[seg];
-            if (cg == 0) store_row_bf16(tS + 256, 1.0f, dst + 2 * p.H + h * HD, live, HD);     // dV
-            else store_row_bf16(tS + 256 + HD, p.scale, dst + p.H + h * HD, live, HD);    // dK
+            const int64_t r = (static_cast<int64_t>(b) * p.nk[seg] + row) * p.ldkv[seg] + h * HD;
+            if (cg == 0) store_row_bf16(tS + 256, 1.0f, p.dv[seg] + r, live, HD);      // dV
+            else store_row_bf16(tS + 256 + HD, p.scale, p.dk[seg] + r, live, HD);     // dK
         } else if (ok) {
             fail();
         }
@@ -562,23 +570,30 @@ size_t attention_backward_ws_bytes(int B, int heads, int n0, int n1) {
 namespace {
 
 template <int HD>
-int attention_backward_hd(const AttnBwdSeg& s0, const AttnBwdSeg& s1, int B, int heads, const float* lse, void* ws,
-                          size_t ws_bytes, cudaStream_t stream) {
+int attention_backward_hd(const AttnBwdSpec& a, void* ws, size_t ws_bytes, cudaStream_t stream) {
     constexpr int kSmemDq = smem_dq<HD>(), kSmemDkdv = smem_dkdv<HD>();
-    if (B <= 0 || heads <= 0 || B > 65535 || heads > 65535 || s0.n < 0 || s1.n < 0 || s0.n + s1.n <= 0)
+    const int B = a.B, heads = a.heads;
+    const int nq0 = a.q[0].n, nq1 = a.q[1].n, nk0 = a.kv[0].n, nk1 = a.kv[1].n;
+    if (B <= 0 || heads <= 0 || B > 65535 || heads > 65535 || nq0 < 0 || nq1 < 0 || nk0 < 0 || nk1 < 0 ||
+        nq0 + nq1 <= 0 || nk0 + nk1 <= 0)
         return set_error(FF_ERR_INVALID_ARG, "attention backward: bad shape");
-    if (!lse || !ws) return set_error(FF_ERR_INVALID_ARG, "attention backward: null lse or workspace");
-    const AttnBwdSeg* sg[2] = {&s0, &s1};
+    if (!a.lse || !ws) return set_error(FF_ERR_INVALID_ARG, "attention backward: null lse or workspace");
     const int H = heads * HD;
+    if (a.q_col < 0 || a.k_col < 0 || a.v_col < 0 || a.q_col % 8 || a.k_col % 8 || a.v_col % 8)
+        return set_error(FF_ERR_INVALID_ARG, "attention backward: q / k / v columns must be multiples of 8");
+    const int kv_cols = (a.k_col > a.v_col ? a.k_col : a.v_col) + H;
     for (int i = 0; i < 2; ++i) {
-        const AttnBwdSeg& s = *sg[i];
-        if (!s.n) continue;
-        if (!s.qkv || !s.o || !s.dout || !s.dqkv || !aligned16(s.o) || !aligned16(s.dout) || !aligned16(s.dqkv) ||
-            s.ld % 8 || s.ldo % 8 || s.ldd % 8 || s.ldg % 8 || s.ld < 3 * H || s.ldo < H || s.ldd < 3 * H ||
-            (s.ldg && s.ldg < H))
-            return set_error(FF_ERR_INVALID_ARG, "attention backward: bad segment %d", i);
+        const AttnBwdQuerySeg& q = a.q[i];
+        if (q.n && (!q.q || !q.o || !q.dout || !q.dq || !aligned16(q.q) || !aligned16(q.o) || !aligned16(q.dout) ||
+                    !aligned16(q.dq) || q.ld % 8 || q.ldo % 8 || q.ldg % 8 || q.ldq % 8 || q.ld < a.q_col + H ||
+                    q.ldo < H || q.ldg < H || q.ldq < H))
+            return set_error(FF_ERR_INVALID_ARG, "attention backward: bad query segment %d", i);
+        const AttnBwdKvSeg& k = a.kv[i];
+        if (k.n && (!k.kv || !k.dk || !k.dv || !aligned16(k.kv) || !aligned16(k.dk) || !aligned16(k.dv) ||
+                    k.ld % 8 || k.ldd % 8 || k.ld < kv_cols || k.ldd < H))
+            return set_error(FF_ERR_INVALID_ARG, "attention backward: bad key / value segment %d", i);
     }
-    const size_t need = attention_backward_ws_bytes(B, heads, s0.n, s1.n);
+    const size_t need = attention_backward_ws_bytes(B, heads, nq0, nq1);
     if (ws_bytes < need || !aligned16(ws))
         return set_error(FF_ERR_WORKSPACE, "attention backward: workspace %zu B < %zu B", ws_bytes, need);
     for (auto* f : {(const void*)attn_bwd_dq_kernel<HD>, (const void*)attn_bwd_dkdv_kernel<HD>}) {
@@ -586,59 +601,94 @@ int attention_backward_hd(const AttnBwdSeg& s0, const AttnBwdSeg& s1, int B, int
         if (cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) != cudaSuccess)
             return set_error(FF_ERR_CUDA, "attention backward: cannot set shared memory size");
     }
-    CUtensorMap tqkv[2], tdo[2];
+    // an empty segment still needs a valid map: it takes its neighbour's
+    CUtensorMap tq[2], tkv[2], tdo[2];
     for (int i = 0; i < 2; ++i) {
-        const AttnBwdSeg& s = sg[i]->n > 0 ? *sg[i] : *sg[1 - i];   // an empty segment still needs a valid map
-        FF_TRY(make_tmap_bf16(&tqkv[i], s.qkv, static_cast<int64_t>(B) * s.n, 3 * H, s.ld, kT));
-        FF_TRY(make_tmap_bf16(&tdo[i], s.dout, static_cast<int64_t>(B) * s.n, H, s.ldg ? s.ldg : s.ldo, kT));
+        const AttnBwdQuerySeg& q = a.q[i].n > 0 ? a.q[i] : a.q[1 - i];
+        FF_TRY(make_tmap_bf16(&tq[i], q.q, static_cast<int64_t>(B) * q.n, a.q_col + H, q.ld, kT));
+        FF_TRY(make_tmap_bf16(&tdo[i], q.dout, static_cast<int64_t>(B) * q.n, H, q.ldg, kT));
+        const AttnBwdKvSeg& k = a.kv[i].n > 0 ? a.kv[i] : a.kv[1 - i];
+        FF_TRY(make_tmap_bf16(&tkv[i], k.kv, static_cast<int64_t>(B) * k.n, kv_cols, k.ld, kT));
     }
     float* delta = static_cast<float*>(ws);
-    const int rows = attn_lse_rows(s0.n, s1.n);
+    const int rows = attn_lse_rows(nq0, nq1);
     {
-        const int64_t warps = (static_cast<int64_t>(B) * (s0.n + s1.n)) * heads;
+        const int64_t warps = (static_cast<int64_t>(B) * (nq0 + nq1)) * heads;
         ProfScope prof(stream, "attn_bwd_delta", 0.0, 4.0 * warps * HD);
         attn_bwd_delta_kernel<HD><<<static_cast<unsigned>((warps + 7) / 8), 256, 0, stream>>>(
-            B, heads, s0.n, s1.n, s0.o, s0.dout, s1.o, s1.dout, s0.ldo, s1.ldo, s0.ldg ? s0.ldg : s0.ldo,
-            s1.ldg ? s1.ldg : s1.ldo, rows, attn_pad128(s0.n), delta);
+            B, heads, nq0, nq1, a.q[0].o, a.q[0].dout, a.q[1].o, a.q[1].dout, a.q[0].ldo, a.q[1].ldo, a.q[0].ldg,
+            a.q[1].ldg, rows, attn_pad128(nq0), delta);
         FF_TRY(check_launch("attn_bwd_delta_kernel"));
     }
     BwdParams p;
-    p.n[0] = s0.n;
-    p.n[1] = s1.n;
-    p.tiles0 = (s0.n + kT - 1) / kT;
-    p.H = H;
+    p.nq[0] = nq0;
+    p.nq[1] = nq1;
+    p.nk[0] = nk0;
+    p.nk[1] = nk1;
+    p.qtiles0 = (nq0 + kT - 1) / kT;
+    p.ktiles0 = (nk0 + kT - 1) / kT;
+    p.q_col = a.q_col;
+    p.k_col = a.k_col;
+    p.v_col = a.v_col;
     p.scale_log2 = static_cast<float>(1.4426950408889634 / sqrt(static_cast<double>(HD)));
     p.scale = static_cast<float>(1.0 / sqrt(static_cast<double>(HD)));
-    p.lse = lse;
+    p.lse = a.lse;
     p.delta = delta;
     p.lse_rows = rows;
     p.lse_base[0] = 0;
-    p.lse_base[1] = attn_pad128(s0.n);
-    p.dqkv[0] = s0.dqkv;
-    p.dqkv[1] = s1.dqkv;
-    p.ldd[0] = s0.ldd;
-    p.ldd[1] = s1.ldd;
-    const dim3 grid(p.tiles0 + (s1.n + kT - 1) / kT, heads, B);
-    const double N = static_cast<double>(s0.n + s1.n);
+    p.lse_base[1] = attn_pad128(nq0);
+    for (int i = 0; i < 2; ++i) {
+        p.dq[i] = a.q[i].dq;
+        p.ldq[i] = a.q[i].ldq;
+        p.dk[i] = a.kv[i].dk;
+        p.dv[i] = a.kv[i].dv;
+        p.ldkv[i] = a.kv[i].ldd;
+    }
+    const double NN = static_cast<double>(nq0 + nq1) * static_cast<double>(nk0 + nk1);
     {
-        ProfScope prof(stream, "attn_bwd_dq", 6.0 * B * heads * N * N * HD, 0.0);
-        attn_bwd_dq_kernel<HD><<<grid, kThreads, kSmemDq, stream>>>(tqkv[0], tqkv[1], tdo[0], tdo[1], p,
+        ProfScope prof(stream, "attn_bwd_dq", 6.0 * B * heads * NN * HD, 0.0);
+        const dim3 grid(p.qtiles0 + (nq1 + kT - 1) / kT, heads, B);
+        attn_bwd_dq_kernel<HD><<<grid, kThreads, kSmemDq, stream>>>(tq[0], tq[1], tkv[0], tkv[1], tdo[0], tdo[1], p,
                                                                  device_status_ptr());
         FF_TRY(check_launch("attn_bwd_dq_kernel"));
     }
-    ProfScope prof(stream, "attn_bwd_dkdv", 8.0 * B * heads * N * N * HD, 0.0);
-    attn_bwd_dkdv_kernel<HD><<<grid, kThreads, kSmemDkdv, stream>>>(tqkv[0], tqkv[1], tdo[0], tdo[1], p,
+    ProfScope prof(stream, "attn_bwd_dkdv", 8.0 * B * heads * NN * HD, 0.0);
+    const dim3 grid(p.ktiles0 + (nk1 + kT - 1) / kT, heads, B);
+    attn_bwd_dkdv_kernel<HD><<<grid, kThreads, kSmemDkdv, stream>>>(tq[0], tq[1], tkv[0], tkv[1], tdo[0], tdo[1], p,
                                                                  device_status_ptr());
     return check_launch("attn_bwd_dkdv_kernel");
 }
 
 }  // namespace
 
+int attention_backward_general(const AttnBwdSpec& a, void* ws, size_t ws_bytes, cudaStream_t stream) {
+    if (a.head_dim == 128) return attention_backward_hd<128>(a, ws, ws_bytes, stream);
+    if (a.head_dim == 64) return attention_backward_hd<64>(a, ws, ws_bytes, stream);
+    return set_error(FF_ERR_UNSUPPORTED, "attention backward: head_dim %d (64 or 128)", a.head_dim);
+}
+
 int attention_backward(const AttnBwdSeg& s0, const AttnBwdSeg& s1, int B, int heads, int head_dim, const float* lse,
                        void* ws, size_t ws_bytes, cudaStream_t stream) {
-    if (head_dim == 128) return attention_backward_hd<128>(s0, s1, B, heads, lse, ws, ws_bytes, stream);
-    if (head_dim == 64) return attention_backward_hd<64>(s0, s1, B, heads, lse, ws, ws_bytes, stream);
-    return set_error(FF_ERR_UNSUPPORTED, "attention backward: head_dim %d (64 or 128)", head_dim);
+    const int64_t H = static_cast<int64_t>(heads) * head_dim;
+    const AttnBwdSeg* sg[2] = {&s0, &s1};
+    AttnBwdSpec a{};
+    for (int i = 0; i < 2; ++i) {
+        const AttnBwdSeg& s = *sg[i];
+        // the joint layout: q, k, v (and their gradients) side by side in one row
+        if (s.n && (!s.dqkv || s.ld < 3 * H || s.ldd < 3 * H))
+            return set_error(FF_ERR_INVALID_ARG, "attention backward: bad segment %d", i);
+        a.q[i] = AttnBwdQuerySeg{s.qkv, s.ld, s.n, s.o, s.ldo, s.dout, s.ldg ? s.ldg : s.ldo, s.dqkv, s.ldd};
+        a.kv[i] = AttnBwdKvSeg{s.qkv, s.ld, s.n, s.dqkv ? s.dqkv + H : nullptr, s.dqkv ? s.dqkv + 2 * H : nullptr,
+                               s.ldd};
+    }
+    a.q_col = 0;
+    a.k_col = static_cast<int>(H);
+    a.v_col = static_cast<int>(2 * H);
+    a.B = B;
+    a.heads = heads;
+    a.head_dim = head_dim;
+    a.lse = lse;
+    return attention_backward_general(a, ws, ws_bytes, stream);
 }
 
 }  // namespace ff

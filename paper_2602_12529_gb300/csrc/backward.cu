@@ -6,12 +6,16 @@
 //     branch bias's gradient);
 //   * ln_modulate_backward: through h = LN(x) (1 + scale) + shift, the
 //     residual gradient g += (dn - mean(dn) - n mean(dn n)) / s with
-//     dn = dh (1 + scale), and per-chunk column sums of dh and dh n;
+//     dn = dh (1 + scale), and per-chunk column sums of dh and dh n; the
+//     affine form h = LN(x) w + b takes dn = dh w (same sums);
 //   * qk_norm_rope_backward: through q = rope(RMSNorm(q_raw) w), in place on
 //     the q | k gradient columns, with per-CTA partial sums of the scale's
 //     gradient;
 //   * colsum: column sums of a bf16 or fp32 matrix (bias gradients);
-//   * silu_backward: dx = dy SiLU'(pre) for the timestep MLP;
+//   * silu_backward: dx = dy SiLU'(pre) (+ a second gradient) for the
+//     timestep MLP;
+//   * wan_modulation_backward: the WAN model's shared modulation e0 + b_l
+//     and final e + b_final, back to d e0, d e and the bias gradients;
 //   * reduce_chunks: fixed-order fp64 sums of the partials, so every
 //     gradient is deterministic.
 #include "internal.h"
@@ -110,20 +114,27 @@ template <int PER>
 __global__ void __launch_bounds__(kThreads) ln_modulate_backward_kernel(const float* x, const float* dh, float* gx,
                                                                          int64_t ld, const float* mods,
                                                                          int64_t ld_mods, BwdSegs s, int H,
-                                                                         float* part) {
+                                                                         const __nv_bfloat16* aff_w, float* part) {
     __shared__ float2 red[3][kThreads / 32];
     BwdSeg sg;
     int b, r0, r1;
     if (!chunk_rows(s, blockIdx.x, sg, b, r0, r1)) return;
     const int t = threadIdx.x, lane = t & 31, w = t >> 5;
     const int nv = H >> 2;
-    const float4* scale = reinterpret_cast<const float4*>(mods + static_cast<int64_t>(b) * ld_mods + sg.col_b);
+    // the multiplier of n: 1 + scale of this sample, or the affine weight
     float4 sc1[PER];
 #pragma unroll
     for (int i = 0; i < PER; ++i) {
         const int k = t + kThreads * i;
-        const float4 c = k < nv ? scale[k] : make_float4(0.f, 0.f, 0.f, 0.f);
-        sc1[i] = make_float4(1.f + c.x, 1.f + c.y, 1.f + c.z, 1.f + c.w);
+        if (aff_w) {
+            const uint2 u = k < nv ? *reinterpret_cast<const uint2*>(aff_w + 4 * k) : make_uint2(0u, 0u);
+            const float2 lo = unpack_bf16x2(u.x), hi = unpack_bf16x2(u.y);
+            sc1[i] = make_float4(lo.x, lo.y, hi.x, hi.y);
+        } else {
+            const float4* scale = reinterpret_cast<const float4*>(mods + static_cast<int64_t>(b) * ld_mods + sg.col_b);
+            const float4 c = k < nv ? scale[k] : make_float4(0.f, 0.f, 0.f, 0.f);
+            sc1[i] = make_float4(1.f + c.x, 1.f + c.y, 1.f + c.z, 1.f + c.w);
+        }
     }
     float4 acc_sh[PER], acc_sc[PER];
 #pragma unroll
@@ -267,6 +278,7 @@ __global__ void __launch_bounds__(kThreads) qk_norm_rope_backward_kernel(QkBwdAr
         }
 #pragma unroll
         for (int which = 0; which < 2; ++which) {
+            if (which >= a.sets) break;
             const int col = which * a.heads * d + head * d + c0;
             __nv_bfloat16* gp = a.d + static_cast<int64_t>(row) * a.ldd + col;
             const __nv_bfloat16* xp = a.raw + static_cast<int64_t>(row) * a.ldr + col;
@@ -391,7 +403,7 @@ __global__ void __launch_bounds__(256) reduce_chunks_kernel(const float* part, i
 // dx = dy SiLU'(pre) for rows < B, written fp32 [B, n] and bf16 [rows_pad, n]
 // (rows B.. rows_pad - 1 zero: the padded operand of the weight gradient).
 __global__ void silu_backward_kernel(const float* dy, int64_t ld_dy, const __nv_bfloat16* pre, int B, int rows_pad,
-                                     int n, float* dx, __nv_bfloat16* dxb) {
+                                     int n, const float* add, float* dx, __nv_bfloat16* dxb) {
     const int i = blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= rows_pad * n) return;
     const int b = i / n, j = i - b * n;
@@ -400,9 +412,41 @@ __global__ void silu_backward_kernel(const float* dy, int64_t ld_dy, const __nv_
         const float p = __bfloat162float(pre[i]);
         const float s = 1.f / (1.f + __expf(-p));
         v = dy[static_cast<int64_t>(b) * ld_dy + j] * s * (1.f + p * (1.f - s));
+        if (add) v += add[i];
         dx[i] = v;
     }
     dxb[i] = __float2bfloat16_rn(v);
+}
+
+// Items, flat: [0, nb) the bias gradients (column j of dm summed over the
+// batch in order; block l's 6H at gbias0 + l stride, the final 2H at
+// gfinal); then rows_pad x 6H of d e0 = sum over blocks in order (bf16 copy
+// zero past B); then B x H of the final layer's d e = d shift + d scale.
+__global__ void wan_modulation_backward_kernel(const float* dm, int64_t ld, int B, int rows_pad, int H, int L,
+                                               float* gbias0, int64_t stride, float* gfinal, float* de0,
+                                               __nv_bfloat16* de0b, float* de_fin) {
+    const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    const int64_t H6 = 6 * static_cast<int64_t>(H), nb = L * H6 + 2 * H, ne0 = rows_pad * H6;
+    if (i < nb) {
+        float acc = 0.f;
+        for (int b = 0; b < B; ++b) acc += dm[b * ld + i];
+        const int64_t l = i / H6;
+        if (l < L) gbias0[l * stride + (i - l * H6)] = acc;
+        else gfinal[i - L * H6] = acc;
+    } else if (i < nb + ne0) {
+        const int64_t k = i - nb;
+        const int64_t b = k / H6, j = k - b * H6;
+        float acc = 0.f;
+        if (b < B) {
+            for (int l = 0; l < L; ++l) acc += dm[b * ld + l * H6 + j];
+            de0[k] = acc;
+        }
+        de0b[k] = __float2bfloat16_rn(acc);
+    } else if (i < nb + ne0 + static_cast<int64_t>(B) * H) {
+        const int64_t k = i - nb - ne0;
+        const int64_t b = k / H, j = k - b * H;
+        de_fin[k] = dm[b * ld + L * H6 + j] + dm[b * ld + L * H6 + H + j];
+    }
 }
 
 int reduce(const float* part, int64_t ld_part, int ncols, const ChunkSpans& sp, int B, float* out, int64_t ld_out,
@@ -446,7 +490,7 @@ int gate_backward(const float* g, const __nv_bfloat16* y, int64_t ld, const floa
 }
 
 int ln_modulate_backward(const float* x, const float* dh, float* gx, int64_t ld, const float* mods, int64_t ld_mods,
-                         const BwdSegs& s, int H, float* part, cudaStream_t stream) {
+                         const BwdSegs& s, int H, float* part, cudaStream_t stream, const __nv_bfloat16* aff_w) {
     if (H % 4 || ld % 4) return set_error(FF_ERR_UNSUPPORTED, "ln_modulate_backward: H and ld must be multiples of 4");
     const int per = (H / 4 + kThreads - 1) / kThreads;
     if (per > 8) return set_error(FF_ERR_UNSUPPORTED, "ln_modulate_backward: H=%d > 8192", H);
@@ -454,7 +498,8 @@ int ln_modulate_backward(const float* x, const float* dh, float* gx, int64_t ld,
     ProfScope prof(stream, "ln_modulate_backward", 0.0, 16.0 * s.rows * H);
 #define FF_LNB(P)                                                                                                   \
     case P:                                                                                                          \
-        ln_modulate_backward_kernel<P><<<s.chunks, kThreads, 0, stream>>>(x, dh, gx, ld, mods, ld_mods, s, H, part); \
+        ln_modulate_backward_kernel<P><<<s.chunks, kThreads, 0, stream>>>(x, dh, gx, ld, mods, ld_mods, s, H, aff_w, \
+                                                                           part);                                     \
         break;
     switch (per) {
         FF_LNB(1) FF_LNB(2) FF_LNB(3) FF_LNB(4) FF_LNB(5) FF_LNB(6) FF_LNB(7) FF_LNB(8)
@@ -503,10 +548,22 @@ int reduce_chunks(const float* part, int64_t ld_part, int ncols, const ChunkSpan
 }
 
 int silu_backward(const float* dy, int64_t ld_dy, const __nv_bfloat16* pre, int B, int rows_pad, int n, float* dx,
-                  __nv_bfloat16* dxb, cudaStream_t stream) {
+                  __nv_bfloat16* dxb, cudaStream_t stream, const float* add) {
     const int total = rows_pad * n;
-    silu_backward_kernel<<<(total + 255) / 256, 256, 0, stream>>>(dy, ld_dy, pre, B, rows_pad, n, dx, dxb);
+    silu_backward_kernel<<<(total + 255) / 256, 256, 0, stream>>>(dy, ld_dy, pre, B, rows_pad, n, add, dx, dxb);
     return check_launch("silu_backward_kernel");
+}
+
+int wan_modulation_backward(const float* dmods, int64_t ld, int B, int rows_pad, int H, int L, float* gbias0,
+                            int64_t stride, float* gfinal, float* de0, __nv_bfloat16* de0b, float* de_fin,
+                            cudaStream_t stream) {
+    if (B <= 0 || rows_pad < B || H <= 0 || L <= 0) return set_error(FF_ERR_INVALID_ARG, "wan_modulation_backward: bad shape");
+    const int64_t total = static_cast<int64_t>(L) * 6 * H + 2 * H + static_cast<int64_t>(rows_pad) * 6 * H +
+                          static_cast<int64_t>(B) * H;
+    ProfScope prof(stream, "wan_modulation_backward", 0.0, 8.0 * B * (static_cast<double>(L) * 6 * H + 2 * H));
+    wan_modulation_backward_kernel<<<static_cast<unsigned>((total + 255) / 256), 256, 0, stream>>>(
+        dmods, ld, B, rows_pad, H, L, gbias0, stride, gfinal, de0, de0b, de_fin);
+    return check_launch("wan_modulation_backward_kernel");
 }
 
 }  // namespace ff

@@ -85,6 +85,50 @@ int ff_attention_backward(int B, int heads, int head_dim, int n0, const void* qk
     return attention_backward(s0, s1, B, heads, head_dim, lse, ws, ws_bytes, stream);
 }
 
+int ff_cross_attention_forward(int B, int heads, int head_dim, int nq, const void* q, int64_t ldq, int nk,
+                               const void* kv, int64_t ldkv, void* out, int64_t ldo, float* lse, cudaStream_t stream) {
+    using namespace ff;
+    if (nq <= 0 || nk <= 0) return set_error(FF_ERR_INVALID_ARG, "cross-attention: nq and nk must be positive");
+    if (lse && !aligned16(lse)) return set_error(FF_ERR_INVALID_ARG, "cross-attention: lse must be 16-byte aligned");
+    AttnSpec a;
+    a.q[0] = AttnQuerySeg{static_cast<const __nv_bfloat16*>(q), ldq, nq, static_cast<__nv_bfloat16*>(out), ldo};
+    a.q[1] = AttnQuerySeg{nullptr, 0, 0, nullptr, 0};
+    a.kv[0] = AttnKvSeg{static_cast<const __nv_bfloat16*>(kv), ldkv, nk};
+    a.kv[1] = AttnKvSeg{nullptr, 0, 0};
+    a.q_col = 0;
+    a.k_col = 0;
+    a.v_col = heads * head_dim;
+    a.B = B;
+    a.heads = heads;
+    a.head_dim = head_dim;
+    a.lse = lse;
+    return attention_general(a, stream);
+}
+
+int ff_cross_attention_backward(int B, int heads, int head_dim, int nq, const void* q, int64_t ldq, const void* out,
+                                const void* dout, int64_t ldo, void* dq, int64_t lddq, int nk, const void* kv,
+                                int64_t ldkv, void* dkv, int64_t lddkv, const float* lse, void* ws, size_t ws_bytes,
+                                cudaStream_t stream) {
+    using namespace ff;
+    if (nq <= 0 || nk <= 0) return set_error(FF_ERR_INVALID_ARG, "cross-attention: nq and nk must be positive");
+    if (lse && !aligned16(lse)) return set_error(FF_ERR_INVALID_ARG, "cross-attention: lse must be 16-byte aligned");
+    const int64_t H = static_cast<int64_t>(heads) * head_dim;
+    if (lddkv < 2 * H) return set_error(FF_ERR_INVALID_ARG, "cross-attention: lddkv %lld < 2H", (long long)lddkv);
+    auto* g = static_cast<__nv_bfloat16*>(dkv);
+    AttnBwdSpec a{};
+    a.q[0] = AttnBwdQuerySeg{static_cast<const __nv_bfloat16*>(q), ldq, nq, static_cast<const __nv_bfloat16*>(out), ldo,
+                             static_cast<const __nv_bfloat16*>(dout), ldo, static_cast<__nv_bfloat16*>(dq), lddq};
+    a.kv[0] = AttnBwdKvSeg{static_cast<const __nv_bfloat16*>(kv), ldkv, nk, g, g ? g + H : nullptr, lddkv};
+    a.q_col = 0;
+    a.k_col = 0;
+    a.v_col = static_cast<int>(H);
+    a.B = B;
+    a.heads = heads;
+    a.head_dim = head_dim;
+    a.lse = lse;
+    return attention_backward_general(a, ws, ws_bytes, stream);
+}
+
 int ff_debug_gemm_gated(int M, int N, int K, const void* A, int64_t lda, const void* B, int64_t ldb, const void* bias,
                         float* resid, int64_t ld_resid, const float* gate, int64_t ld_gate, int rows_per_sample,
                         cudaStream_t stream) {

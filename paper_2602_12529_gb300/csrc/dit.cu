@@ -200,11 +200,14 @@ void set_qk_norm(GemmEpilogue& e, const ff_dit_config& c, int qk_cols, const __n
 }
 
 
+}  // namespace
+
 // WAN-style velocity: latent tokens only in the residual stream; the text is
 // embedded once per call and feeds every block's cross-attention keys and
-// values.
-int wan_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, const float* t, float* v_out,
-                 const Workspace& w, cudaStream_t stream) {
+// values.  Buffers come from f as for mmdit_forward (one shared set for the
+// inference call, one set per block with the raw copies for training).
+int wan_forward(const ff_dit* m, int B, const float* x_t, const void* txt, const float* t, float* v_out,
+                const FwdBufs& f, cudaStream_t stream) {
     const ff_dit_config& c = m->cfg;
     const int H = c.hidden, F = c.mlp, P = c.patch_dim, d = c.head_dim, L = c.n_double;
     const int Nt = c.n_txt, Ni = c.grid_f * c.grid_h * c.grid_w;
@@ -213,148 +216,163 @@ int wan_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, cons
     auto W = [&](const std::string& n) { return m->w + m->off.at(n); };
 
     // rotation table; timestep embedding e (fp32), SiLU(e) (bf16), e0 = SiLU(e) W_mod^T + b; per-block modulation
-    FF_TRY(rope_table(w.rope, c.grid_f, c.grid_h, c.grid_w, c.rope_axes[0], c.rope_axes[1], c.rope_axes[2],
+    FF_TRY(rope_table(f.rope, c.grid_f, c.grid_h, c.grid_w, c.rope_axes[0], c.rope_axes[1], c.rope_axes[2],
                       c.rope_theta, stream));
-    FF_TRY(timestep_embed(t, B, c.time_freq_dim, w.temb, stream));
+    FF_TRY(timestep_embed(t, B, c.time_freq_dim, f.temb, stream));
     {
         GemmEpilogue e;
-        e.rows_gemv = 1; e.act = ACT_SILU; e.bias = W("t_embed.fc1.b"); e.out0 = w.th; e.ld0 = H;
-        FF_TRY(gemm_bf16(w.temb, c.time_freq_dim, W("t_embed.fc1.w"), c.time_freq_dim, B, H, c.time_freq_dim, e, stream));
+        e.rows_gemv = 1; e.act = ACT_SILU; e.bias = W("t_embed.fc1.b"); e.out0 = f.th; e.ld0 = H;
+        e.aux = f.pre_fc1; e.ld_aux = H;
+        FF_TRY(gemm_bf16(f.temb, c.time_freq_dim, W("t_embed.fc1.w"), c.time_freq_dim, B, H, c.time_freq_dim, e, stream));
     }
     {
         GemmEpilogue e;
-        e.rows_gemv = 1; e.out_f32 = 1; e.bias = W("t_embed.fc2.b"); e.out0 = w.e; e.ld0 = H;
-        FF_TRY(gemm_bf16(w.th, H, W("t_embed.fc2.w"), H, B, H, H, e, stream));
+        e.rows_gemv = 1; e.out_f32 = 1; e.bias = W("t_embed.fc2.b"); e.out0 = f.e; e.ld0 = H;
+        FF_TRY(gemm_bf16(f.th, H, W("t_embed.fc2.w"), H, B, H, H, e, stream));
     }
     {
         GemmEpilogue e;
-        e.rows_gemv = 1; e.act = ACT_SILU; e.bias = W("t_embed.fc2.b"); e.out0 = w.tc; e.ld0 = H;
-        FF_TRY(gemm_bf16(w.th, H, W("t_embed.fc2.w"), H, B, H, H, e, stream));
+        e.rows_gemv = 1; e.act = ACT_SILU; e.bias = W("t_embed.fc2.b"); e.out0 = f.tc; e.ld0 = H;
+        e.aux = f.pre_c; e.ld_aux = H;
+        FF_TRY(gemm_bf16(f.th, H, W("t_embed.fc2.w"), H, B, H, H, e, stream));
     }
     {
         GemmEpilogue e;
-        e.rows_gemv = 1; e.out_f32 = 1; e.bias = W("mod.b"); e.out0 = w.e0; e.ld0 = 6 * H;
-        FF_TRY(gemm_bf16(w.tc, H, W("mod.w"), H, B, 6 * H, H, e, stream));
+        e.rows_gemv = 1; e.out_f32 = 1; e.bias = W("mod.b"); e.out0 = f.e0; e.ld0 = 6 * H;
+        FF_TRY(gemm_bf16(f.tc, H, W("mod.w"), H, B, 6 * H, H, e, stream));
     }
     const int64_t stride = L > 1 ? m->off.at("blocks.1.mod.b") - m->off.at("blocks.0.mod.b") : 0;
-    FF_TRY(wan_modulation(w.e, w.e0, W("blocks.0.mod.b"), stride, L, W("final.mod.b"), B, H, w.mods, Wm, stream));
+    FF_TRY(wan_modulation(f.e, f.e0, W("blocks.0.mod.b"), stride, L, W("final.mod.b"), B, H, f.mods, Wm, stream));
 
     // latent tokens and text embeddings
-    FF_TRY(f32_to_bf16(x_t, w.xb, static_cast<int64_t>(Ri) * P, stream));
+    FF_TRY(f32_to_bf16(x_t, f.xb, static_cast<int64_t>(Ri) * P, stream));
     {
         GemmEpilogue e;
-        e.out_f32 = 1; e.bias = W("img_in.b"); e.out0 = w.x; e.ld0 = H;
-        FF_TRY(gemm_bf16(w.xb, P, W("img_in.w"), P, Ri, H, P, e, stream));
+        e.out_f32 = 1; e.bias = W("img_in.b"); e.out0 = f.x0; e.ld0 = H;
+        FF_TRY(gemm_bf16(f.xb, P, W("img_in.w"), P, Ri, H, P, e, stream));
     }
     {
         GemmEpilogue e;
-        e.act = ACT_GELU; e.bias = W("txt_in.b"); e.out0 = w.txt1; e.ld0 = H;
+        e.act = ACT_GELU; e.bias = W("txt_in.b"); e.out0 = f.txt1; e.ld0 = H;
+        e.aux = f.txt_pre; e.ld_aux = H;
         FF_TRY(gemm_bf16(txt, c.txt_dim, W("txt_in.w"), c.txt_dim, Rt, H, c.txt_dim, e, stream));
     }
     {
         GemmEpilogue e;
-        e.bias = W("txt_in2.b"); e.out0 = w.txth; e.ld0 = H;
-        FF_TRY(gemm_bf16(w.txt1, H, W("txt_in2.w"), H, Rt, H, H, e, stream));
+        e.bias = W("txt_in2.b"); e.out0 = f.txth; e.ld0 = H;
+        FF_TRY(gemm_bf16(f.txt1, H, W("txt_in2.w"), H, Rt, H, H, e, stream));
     }
 
     LnModArgs la{};
-    la.x = w.x; la.ldx = H; la.out = w.h; la.ldo = H; la.rows = Ri; la.H = H;
-    la.rows_txt = 0; la.n_txt = 1; la.n_img = Ni; la.mods = w.mods; la.ld_mods = Wm;
+    la.ldx = H; la.ldo = H; la.rows = Ri; la.H = H;
+    la.rows_txt = 0; la.n_txt = 1; la.n_img = Ni; la.mods = f.mods; la.ld_mods = Wm;
 
-
-    __nv_bfloat16* qc = w.qkv;   // cross-attention queries reuse the QKV buffer ([Ri, H])
     for (int l = 0; l < L; ++l) {
+        const DitBlockIo io = f.block(l);
         const std::string p = "blocks." + std::to_string(l) + ".";
         const int base = l * 6 * H;
         // self-attention
+        la.x = io.xin; la.out = io.h1;
         la.aff_w = la.aff_b = nullptr;
         la.shift_txt = la.shift_img = base;
         la.scale_txt = la.scale_img = base + H;
         FF_TRY(ln_modulate(la, stream));
         {
             GemmEpilogue e;
-            e.bias = W(p + "qkv.b"); e.out0 = w.qkv; e.ld0 = 3 * H;
-            set_qk_norm(e, c, 2 * H, W(p + "q_norm.scale"), W(p + "k_norm.scale"), w.rope, 0);
-            FF_TRY(gemm_bf16(w.h, H, W(p + "qkv.w"), H, Ri, 3 * H, H, e, stream));
+            e.bias = W(p + "qkv.b"); e.out0 = io.qkv; e.ld0 = 3 * H;
+            e.aux = io.raw; e.ld_aux = 3 * H;
+            set_qk_norm(e, c, 2 * H, W(p + "q_norm.scale"), W(p + "k_norm.scale"), f.rope, 0);
+            FF_TRY(gemm_bf16(io.h1, H, W(p + "qkv.w"), H, Ri, 3 * H, H, e, stream));
         }
         {
             AttnSpec a{};
             a.q[0] = AttnQuerySeg{nullptr, 0, 0, nullptr, 0};
-            a.q[1] = AttnQuerySeg{w.qkv, 3 * H, Ni, w.o, H};
+            a.q[1] = AttnQuerySeg{io.qkv, 3 * H, Ni, io.o, H};
             a.kv[0] = AttnKvSeg{nullptr, 0, 0};
-            a.kv[1] = AttnKvSeg{w.qkv, 3 * H, Ni};
+            a.kv[1] = AttnKvSeg{io.qkv, 3 * H, Ni};
             a.q_col = 0; a.k_col = H; a.v_col = 2 * H;
             a.B = B; a.heads = c.heads; a.head_dim = d;
+            a.lse = io.lse;
             FF_TRY(attention_general(a, stream));
         }
         {
             GemmEpilogue e;
             e.epi = EPI_GATED_RESIDUAL; e.bias = W(p + "proj.b");
-            e.resid = w.x; e.ld_resid = H;
-            e.gate = w.mods + base + 2 * H; e.ld_gate = Wm; e.rows_per_sample = Ni;
-            FF_TRY(gemm_bf16(w.o, H, W(p + "proj.w"), H, Ri, H, H, e, stream));
+            e.resid = io.xin; e.ld_resid = H;
+            if (io.xmid != io.xin) e.resid_out = io.xmid;
+            e.gate = f.mods + base + 2 * H; e.ld_gate = Wm; e.rows_per_sample = Ni;
+            e.aux = io.y1; e.ld_aux = H;
+            FF_TRY(gemm_bf16(io.o, H, W(p + "proj.w"), H, Ri, H, H, e, stream));
         }
         // cross-attention to the text
+        la.x = io.xmid; la.out = io.hc;
         la.aff_w = W(p + "cross_norm.scale");
         la.aff_b = W(p + "cross_norm.b");
         FF_TRY(ln_modulate(la, stream));
         {
             GemmEpilogue e;   // cross q with its RMSNorm fused (no rotation)
-            e.bias = W(p + "cross_q.b"); e.out0 = qc; e.ld0 = H;
+            e.bias = W(p + "cross_q.b"); e.out0 = io.qc; e.ld0 = H;
+            e.aux = io.qc_raw; e.ld_aux = H;
             set_qk_norm(e, c, H, W(p + "cross_q_norm.scale"), W(p + "cross_q_norm.scale"), nullptr, 0);
-            FF_TRY(gemm_bf16(w.h, H, W(p + "cross_q.w"), H, Ri, H, H, e, stream));
+            FF_TRY(gemm_bf16(io.hc, H, W(p + "cross_q.w"), H, Ri, H, H, e, stream));
         }
         {
             GemmEpilogue e;   // cross k | v of the text, RMSNorm on k fused
-            e.bias = W(p + "cross_kv.b"); e.out0 = w.kvc; e.ld0 = 2 * H;
+            e.bias = W(p + "cross_kv.b"); e.out0 = io.kv; e.ld0 = 2 * H;
+            e.aux = io.kv_raw; e.ld_aux = 2 * H;
             set_qk_norm(e, c, H, W(p + "cross_k_norm.scale"), W(p + "cross_k_norm.scale"), nullptr, 0);
-            FF_TRY(gemm_bf16(w.txth, H, W(p + "cross_kv.w"), H, Rt, 2 * H, H, e, stream));
+            FF_TRY(gemm_bf16(f.txth, H, W(p + "cross_kv.w"), H, Rt, 2 * H, H, e, stream));
         }
         {
             AttnSpec a{};
             a.q[0] = AttnQuerySeg{nullptr, 0, 0, nullptr, 0};
-            a.q[1] = AttnQuerySeg{qc, H, Ni, w.o, H};
-            a.kv[0] = AttnKvSeg{w.kvc, 2 * H, Nt};
+            a.q[1] = AttnQuerySeg{io.qc, H, Ni, io.oc, H};
+            a.kv[0] = AttnKvSeg{io.kv, 2 * H, Nt};
             a.kv[1] = AttnKvSeg{nullptr, 0, 0};
             a.q_col = 0; a.k_col = 0; a.v_col = H;
             a.B = B; a.heads = c.heads; a.head_dim = d;
+            a.lse = io.lse_c;
             FF_TRY(attention_general(a, stream));
         }
         {
             GemmEpilogue e;   // plain residual: no gate on the cross-attention branch
             e.epi = EPI_GATED_RESIDUAL; e.bias = W(p + "cross_proj.b");
-            e.resid = w.x; e.ld_resid = H; e.gate = nullptr; e.rows_per_sample = Ni;
-            FF_TRY(gemm_bf16(w.o, H, W(p + "cross_proj.w"), H, Ri, H, H, e, stream));
+            e.resid = io.xmid; e.ld_resid = H; e.gate = nullptr; e.rows_per_sample = Ni;
+            if (io.x3 != io.xmid) e.resid_out = io.x3;
+            FF_TRY(gemm_bf16(io.oc, H, W(p + "cross_proj.w"), H, Ri, H, H, e, stream));
         }
         // FFN
+        la.x = io.x3; la.out = io.h2;
         la.aff_w = la.aff_b = nullptr;
         la.shift_txt = la.shift_img = base + 3 * H;
         la.scale_txt = la.scale_img = base + 4 * H;
         FF_TRY(ln_modulate(la, stream));
         {
             GemmEpilogue e;
-            e.act = ACT_GELU; e.bias = W(p + "mlp1.b"); e.out0 = w.u; e.ld0 = F;
-            FF_TRY(gemm_bf16(w.h, H, W(p + "mlp1.w"), H, Ri, F, H, e, stream));
+            e.act = ACT_GELU; e.bias = W(p + "mlp1.b"); e.out0 = io.u; e.ld0 = F;
+            e.aux = io.a1; e.ld_aux = F;
+            FF_TRY(gemm_bf16(io.h2, H, W(p + "mlp1.w"), H, Ri, F, H, e, stream));
         }
         {
             GemmEpilogue e;
             e.epi = EPI_GATED_RESIDUAL; e.bias = W(p + "mlp2.b");
-            e.resid = w.x; e.ld_resid = H;
-            e.gate = w.mods + base + 5 * H; e.ld_gate = Wm; e.rows_per_sample = Ni;
-            FF_TRY(gemm_bf16(w.u, F, W(p + "mlp2.w"), F, Ri, H, F, e, stream));
+            e.resid = io.x3; e.ld_resid = H;
+            if (io.xout != io.x3) e.resid_out = io.xout;
+            e.gate = f.mods + base + 5 * H; e.ld_gate = Wm; e.rows_per_sample = Ni;
+            e.aux = io.y2; e.ld_aux = H;
+            FF_TRY(gemm_bf16(io.u, F, W(p + "mlp2.w"), F, Ri, H, F, e, stream));
         }
     }
     // final layer
+    la.x = f.xfin; la.out = f.hf;
     la.aff_w = la.aff_b = nullptr;
     la.shift_txt = la.shift_img = L * 6 * H;
     la.scale_txt = la.scale_img = L * 6 * H + H;
     FF_TRY(ln_modulate(la, stream));
     GemmEpilogue e;
     e.out_f32 = 1; e.bias = W("final.b"); e.out0 = v_out; e.ld0 = P;
-    return gemm_bf16(w.h, H, W("final.w"), H, Ri, P, H, e, stream);
+    return gemm_bf16(f.hf, H, W("final.w"), H, Ri, P, H, e, stream);
 }
-
-}  // namespace
 
 // The MMDiT velocity: timestep MLP and every adaLN vector, embeddings, the
 // double- and single-stream blocks, the final layer.  Buffers come from f:
@@ -642,12 +660,22 @@ int ff_dit_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, c
     const Workspace w = plan(c, B, static_cast<uint8_t*>(ws));
     if (ws_bytes < w.bytes) return set_error(FF_ERR_WORKSPACE, "workspace %zu B < %zu B needed", ws_bytes, w.bytes);
 
-    if (c.arch == FF_ARCH_WAN) return wan_velocity(m, B, x_t, txt, t, v_out, w, stream);
     FwdBufs f{};
     f.mods = w.mods; f.temb = w.temb; f.th = w.th; f.tc = w.tc; f.xb = w.xb; f.rope = w.rope;
     f.x0 = f.xfin = w.x;
     f.hf = w.h;
     f.shared = DitBlockIo{w.x, w.x, w.x, w.h, w.qkv, nullptr, w.o, nullptr, w.h, nullptr, w.u, nullptr, nullptr};
+    if (c.arch == FF_ARCH_WAN) {
+        // one buffer per role, reused by every block: the residual in place,
+        // cross q in the QKV buffer, the cross-attention output in o
+        f.shared.x3 = w.x;
+        f.shared.hc = w.h;
+        f.shared.qc = w.qkv;
+        f.shared.kv = w.kvc;
+        f.shared.oc = w.o;
+        f.e = w.e; f.e0 = w.e0; f.txt1 = w.txt1; f.txth = w.txth;
+        return wan_forward(m, B, x_t, txt, t, v_out, f, stream);
+    }
     return mmdit_forward(m, B, x_t, txt, t, v_out, f, stream);
 }
 

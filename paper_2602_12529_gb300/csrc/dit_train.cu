@@ -138,7 +138,6 @@ int check_model(const ff_dit* m, int B) {
     if (!m) return set_error(FF_ERR_INVALID_ARG, "model is null");
     if (B <= 0) return set_error(FF_ERR_INVALID_ARG, "B=%d must be positive", B);
     const ff_dit_config& c = model_config(m);
-    if (c.arch != FF_ARCH_MMDIT) return set_error(FF_ERR_UNSUPPORTED, "training pass: MMDiT models only");
 
     const int64_t Ni = static_cast<int64_t>(c.grid_f) * c.grid_h * c.grid_w;
     if ((static_cast<int64_t>(B) * c.n_txt) % 8 || (B * Ni) % 8)
@@ -146,24 +145,11 @@ int check_model(const ff_dit* m, int B) {
     return FF_OK;
 }
 
-// A weight-gradient product dW[M, N] = dy^T x over K token rows (dy [K, M],
-// x [K, N], both row-major) into the fp32 gradient blob.
 GemmArgs wgrad(const void* dy, int64_t lddy, const void* x, int64_t ldx, int M, int N, int K, float* out) {
-    GemmArgs g{dy, lddy, x, ldx, M, N, K, GemmEpilogue{}};
-    g.a_mn = 1;
-    g.b_mn = 1;
-    g.epi.out_f32 = 1;
-    g.epi.out0 = out;
-    g.epi.ld0 = N;
-    return g;
+    return gemm_wgrad(dy, lddy, x, ldx, M, N, K, out);
 }
-
-// An input-gradient product dx[M, N] = dy[M, K] W[K, N] (W the forward's
-// [out, in] weight read as an MN-major B operand).
 GemmArgs dgrad(const void* dy, int64_t lddy, const void* w, int M, int N, int K) {
-    GemmArgs g{dy, lddy, w, N, M, N, K, GemmEpilogue{}};
-    g.b_mn = 1;
-    return g;
+    return gemm_dgrad(dy, lddy, w, M, N, K);
 }
 
 }  // namespace
@@ -175,7 +161,8 @@ int ff_dit_train_workspace_size(const ff_dit* m, int B, size_t* bytes) {
     using namespace ff;
     FF_TRY(check_model(m, B));
     if (!bytes) return set_error(FF_ERR_INVALID_ARG, "bytes is null");
-    *bytes = plan(model_config(m), model_mod_width(m), B, nullptr).bytes;
+    *bytes = model_config(m).arch == FF_ARCH_WAN ? wan_train_workspace_bytes(m, B)
+                                                 : plan(model_config(m), model_mod_width(m), B, nullptr).bytes;
     return FF_OK;
 }
 
@@ -187,6 +174,7 @@ int ff_dit_forward_train(const ff_dit* m, int B, const float* x_t, const void* t
     if (!aligned16(x_t) || !aligned16(txt) || !aligned16(v_out) || (reinterpret_cast<uintptr_t>(ws) % kAlign))
         return set_error(FF_ERR_INVALID_ARG, "misaligned pointer (arrays 16 B, workspace 256 B)");
     const ff_dit_config& c = model_config(m);
+    if (c.arch == FF_ARCH_WAN) return wan_forward_train(m, B, x_t, txt, t, v_out, ws, ws_bytes, stream);
     TrainPlan p = plan(c, model_mod_width(m), B, static_cast<uint8_t*>(ws));
     if (ws_bytes < p.bytes) return set_error(FF_ERR_WORKSPACE, "workspace %zu B < %zu B needed", ws_bytes, p.bytes);
     p.f.blocks = p.blk.data();
@@ -210,6 +198,7 @@ int ff_dit_backward(const ff_dit* m, int B, const void* txt, const float* dv, fl
         (reinterpret_cast<uintptr_t>(ws) % kAlign))
         return set_error(FF_ERR_INVALID_ARG, "misaligned pointer (arrays 16 B, workspace 256 B)");
     const ff_dit_config& c = model_config(m);
+    if (c.arch == FF_ARCH_WAN) return wan_backward(m, B, txt, dv, grad, dx_t, ws, ws_bytes, stream);
     const int64_t Wm = model_mod_width(m);
     TrainPlan p = plan(c, Wm, B, static_cast<uint8_t*>(ws));
     if (ws_bytes < p.bytes) return set_error(FF_ERR_WORKSPACE, "workspace %zu B < %zu B needed", ws_bytes, p.bytes);

@@ -130,6 +130,24 @@ struct GemmArgs {
     int a_mn = 0, b_mn = 0;
 };
 int gemm_bf16_group(const GemmArgs* problems, int n, cudaStream_t stream);
+// A weight-gradient product dW[M, N] = dy^T x over K token rows (dy [K, M],
+// x [K, N], both row-major) into fp32 out (pitch N).
+inline GemmArgs gemm_wgrad(const void* dy, int64_t lddy, const void* x, int64_t ldx, int M, int N, int K, float* out) {
+    GemmArgs g{dy, lddy, x, ldx, M, N, K, GemmEpilogue{}};
+    g.a_mn = 1;
+    g.b_mn = 1;
+    g.epi.out_f32 = 1;
+    g.epi.out0 = out;
+    g.epi.ld0 = N;
+    return g;
+}
+// An input-gradient product dx[M, N] = dy[M, K] W[K, N] (W the forward's
+// [out, in] weight read as an MN-major B operand); the caller sets the output.
+inline GemmArgs gemm_dgrad(const void* dy, int64_t lddy, const void* w, int M, int N, int K) {
+    GemmArgs g{dy, lddy, w, N, M, N, K, GemmEpilogue{}};
+    g.b_mn = 1;
+    return g;
+}
 
 // ---- elementwise / row kernels -------------------------------------------
 // Row r of x (fp32 [rows, H]) belongs to segment txt if r < rows_txt, else img;
@@ -194,7 +212,7 @@ inline int attn_pad128(int n) { return (n + 127) / 128 * 128; }
 inline int attn_lse_rows(int n0, int n1) { return attn_pad128(n0) + attn_pad128(n1); }
 int attention_general(const AttnSpec& a, cudaStream_t stream);
 
-// Backward of joint attention (d = 128): from dO (bf16, the layout of the
+// Backward of joint attention (d = 64 or 128): from dO (bf16, the layout of the
 // forward's output) and the forward's lse, the gradients of q, k and v are
 // written into dqkv buffers laid out like the qkv inputs.  ws holds
 // D = rowsum(dO * O) in the lse layout (attention_backward_ws_bytes).
@@ -207,6 +225,32 @@ struct AttnBwdSeg {
     int n;
     int64_t ldg = 0;
 };
+// The same for attention_general's form: query segments (q at column q_col
+// of their rows, O, dO, and where dq goes) and key / value segments (k, v at
+// columns k_col, v_col, and where dk, dv go); head h of dq / dk / dv at
+// column h d of its destination.  lse: the forward's (AttnSpec layout over
+// the query segments).
+struct AttnBwdQuerySeg {
+    const __nv_bfloat16* q; int64_t ld;
+    int n;
+    const __nv_bfloat16* o; int64_t ldo;
+    const __nv_bfloat16* dout; int64_t ldg;
+    __nv_bfloat16* dq; int64_t ldq;
+};
+struct AttnBwdKvSeg {
+    const __nv_bfloat16* kv; int64_t ld;
+    int n;
+    __nv_bfloat16 *dk, *dv; int64_t ldd;
+};
+struct AttnBwdSpec {
+    AttnBwdQuerySeg q[2];
+    AttnBwdKvSeg kv[2];
+    int q_col, k_col, v_col;
+    int B, heads, head_dim;
+    const float* lse;
+};
+int attention_backward_general(const AttnBwdSpec& a, void* ws, size_t ws_bytes, cudaStream_t stream);
+// D lives in the lse layout of the query segments (n0, n1 = query counts).
 size_t attention_backward_ws_bytes(int B, int heads, int n0, int n1);
 int attention_backward(const AttnBwdSeg& s0, const AttnBwdSeg& s1, int B, int heads, int head_dim,
                        const float* lse, void* ws, size_t ws_bytes, cudaStream_t stream);
@@ -238,9 +282,11 @@ struct ChunkSpans { int first[2], count[2], n; };
 int gate_backward(const float* g, const __nv_bfloat16* y, int64_t ld, const float* mods, int64_t ld_mods,
                   const BwdSegs& s, int H, __nv_bfloat16* dy, float* part, cudaStream_t stream);
 // Through h = LN(x) (1 + scale) + shift: gx += dx; part[c * 2H + j] = sum dh,
-// part[c * 2H + H + j] = sum dh n (n = LN(x)).  x, dh, gx share ld.
+// part[c * 2H + H + j] = sum dh n (n = LN(x)).  x, dh, gx share ld.  With
+// aff_w set, through the affine h = LN(x) w + b instead (mods unused; the
+// same sums are then the bias and weight gradients' partials).
 int ln_modulate_backward(const float* x, const float* dh, float* gx, int64_t ld, const float* mods, int64_t ld_mods,
-                         const BwdSegs& s, int H, float* part, cudaStream_t stream);
+                         const BwdSegs& s, int H, float* part, cudaStream_t stream, const __nv_bfloat16* aff_w = nullptr);
 // Through q = rope(RMSNorm(q_raw) w) for the q (columns [0, H)) and k
 // (columns [H, 2H)) gradients in d, in place; rows >= rows_txt are image
 // tokens (rotated with the cos / sin table, as the forward epilogue does).
@@ -254,6 +300,7 @@ struct QkBwdArgs {
     const float2* rope_cs;
     int n_img, grid_f, grid_h, grid_w, axes0, axes1, axes2;
     float* part;
+    int sets = 2;   // 1: q columns only (a lone query or key block at column 0)
 };
 int qk_norm_rope_backward(const QkBwdArgs& a, int* ctas_txt, int* ctas_img, cudaStream_t stream);
 constexpr int kQkBwdRows = 16;   // rows per CTA of qk_norm_rope_backward
@@ -263,9 +310,18 @@ int colsum(const void* in, bool f32, int64_t ld, int rows, int ncols, float* out
 // B > 0: out[b * ld_out + j] per sample; B == 0: out[j] over every chunk.
 int reduce_chunks(const float* part, int64_t ld_part, int ncols, const ChunkSpans& sp, int B, float* out,
                   int64_t ld_out, cudaStream_t stream);
-// dx = dy SiLU'(pre) (rows < B; fp32 [B, n]) and its bf16 copy [rows_pad, n], zero-padded.
+// dx = dy SiLU'(pre) (+ add, fp32 [B, n], when set) (rows < B; fp32 [B, n]) and
+// its bf16 copy [rows_pad, n], zero-padded.
 int silu_backward(const float* dy, int64_t ld_dy, const __nv_bfloat16* pre, int B, int rows_pad, int n, float* dx,
-                  __nv_bfloat16* dxb, cudaStream_t stream);
+                  __nv_bfloat16* dxb, cudaStream_t stream, const float* add = nullptr);
+// Backward of wan_modulation: from dmods [B, ld] (block l's 6H at l 6H, the
+// final layer's shift | scale at L 6H) the bias gradients (blocks.l.mod.b at
+// gbias0 + l stride, final.mod.b at gfinal; sums over the batch), d e0 =
+// sum over blocks (fp32 [B, 6H] and bf16 [rows_pad, 6H], zero-padded) and
+// the final layer's part of d e (fp32 [B, H]).  Fixed summation order.
+int wan_modulation_backward(const float* dmods, int64_t ld, int B, int rows_pad, int H, int L, float* gbias0,
+                            int64_t stride, float* gfinal, float* de0, __nv_bfloat16* de0b, float* de_fin,
+                            cudaStream_t stream);
 
 // mods[b, l*6H + j] = e0[b, j] + bias_l[j] (bias_l = bias0 + l*stride), and
 // mods[b, L*6H + j] = e[b, j % H] + fbias[j] for j < 2H (WAN modulation).
@@ -286,6 +342,13 @@ struct DitBlockIo {
     float *xin, *xmid, *xout;
     __nv_bfloat16 *h1, *qkv, *raw, *o, *y1, *h2, *a1, *u, *y2;
     float* lse;
+    // WAN blocks (xmid: after the self-attention): the residual after the
+    // cross-attention, the affine-LN output, the normalised cross q and text
+    // k | v with their raw copies (written only when set), the
+    // cross-attention output and its log-sum-exp
+    float* x3;
+    __nv_bfloat16 *hc, *qc, *qc_raw, *kv, *kv_raw, *oc;
+    float* lse_c;
 };
 struct FwdBufs {
     float* mods;
@@ -297,9 +360,24 @@ struct FwdBufs {
     DitBlockIo shared;      // every block's buffers when blocks is null
     const DitBlockIo* blocks;
     DitBlockIo block(int l) const { return blocks ? blocks[l] : shared; }
+    // WAN: the timestep embedding e (fp32 [B, H]), the shared modulation e0
+    // (fp32 [B, 6H]); the text MLP's pre-GELU copy (when set), its GELU
+    // output and the embedded text (bf16 [B N_t, H])
+    float *e, *e0;
+    __nv_bfloat16 *txt_pre, *txt1, *txth;
 };
 int mmdit_forward(const ff_dit* m, int B, const float* x_t, const void* txt, const float* t, float* v_out,
                   const FwdBufs& f, cudaStream_t stream);
+int wan_forward(const ff_dit* m, int B, const float* x_t, const void* txt, const float* t, float* v_out,
+                const FwdBufs& f, cudaStream_t stream);
+// The WAN model's training pass (wan_train.cu): workspace bytes, the forward
+// that keeps what the backward reads, and the backward (arguments as
+// ff_dit_forward_train / ff_dit_backward, already validated).
+size_t wan_train_workspace_bytes(const ff_dit* m, int B);
+int wan_forward_train(const ff_dit* m, int B, const float* x_t, const void* txt, const float* t, float* v_out,
+                      void* ws, size_t ws_bytes, cudaStream_t stream);
+int wan_backward(const ff_dit* m, int B, const void* txt, const float* dv, float* grad, float* dx_t, void* ws,
+                 size_t ws_bytes, cudaStream_t stream);
 int f32_to_bf16(const float* in, __nv_bfloat16* out, int64_t n, cudaStream_t stream);
 
 }  // namespace ff

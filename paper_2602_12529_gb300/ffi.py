@@ -90,6 +90,9 @@ _SIGS = {
     "ff_attention_backward_workspace_size": ([_I, _I, _I, _I, C.POINTER(_SZ)], _I),
     "ff_attention_backward": ([_I, _I, _I, _I, _P, _I64, _P, _P, _I64, _P, _I64, _I, _P, _I64, _P, _P, _I64, _P,
                                _I64, _P, _P, _SZ, _P], _I),
+    "ff_cross_attention_forward": ([_I, _I, _I, _I, _P, _I64, _I, _P, _I64, _P, _I64, _P, _P], _I),
+    "ff_cross_attention_backward": ([_I, _I, _I, _I, _P, _I64, _P, _P, _I64, _P, _I64, _I, _P, _I64, _P, _I64, _P,
+                                     _P, _SZ, _P], _I),
     "ff_rollout": ([_P, _I, _I, _P, _P, _P, _P, _P, _P, _P, _I, _P, _SZ, _P], _I),
     "ff_debug_gemm": ([_I, _I, _I, _P, _I64, _P, _I64, _P, _I, _I, _P, _I64, _P], _I),
     "ff_debug_gemm_gated": ([_I, _I, _I, _P, _I64, _P, _I64, _P, _P, _I64, _P, _I64, _I, _P], _I),
@@ -519,6 +522,25 @@ def ff_attention_backward(B, heads, head_dim, seg0, seg1, lse, ws=None, stream=N
     _call("ff_attention_backward", B, heads, head_dim, n0, _ptr(q0), q0.shape[-1], _ptr(o0), _ptr(g0),
           o0.shape[-1], _ptr(d0), d0.shape[-1], n1, _ptr(q1), q1.shape[-1], _ptr(o1), _ptr(g1), o1.shape[-1],
           _ptr(d1), d1.shape[-1], _ptr(lse), _ptr(ws), ws.numel(), _stream(stream))
+
+
+def ff_cross_attention_forward(B, heads, head_dim, q, nq, kv, nk, out, lse=None, stream=None):
+    """Cross-attention: q [B nq, >= H] (q at columns h d), kv [B nk, >= 2H] (k at
+    h d, v at H + h d), out [B nq, >= H]; lse [B, heads, ff_attention_lse_rows(nq, 0)] or None."""
+    _call("ff_cross_attention_forward", B, heads, head_dim, nq, _ptr(q), q.shape[-1], nk, _ptr(kv), kv.shape[-1],
+          _ptr(out), out.shape[-1], _ptr(lse), _stream(stream))
+
+
+def ff_cross_attention_backward(B, heads, head_dim, q, nq, out, dout, dq, kv, nk, dkv, lse, ws=None, stream=None):
+    """Writes dq (like q) and dk | dv (like kv) from dO (like out) and the forward's lse."""
+    import torch
+    if ws is None:
+        sz = _SZ()
+        _call("ff_attention_backward_workspace_size", B, heads, nq, 0, C.byref(sz))
+        ws = torch.empty(sz.value, dtype=torch.uint8, device=lse.device)
+    _call("ff_cross_attention_backward", B, heads, head_dim, nq, _ptr(q), q.shape[-1], _ptr(out), _ptr(dout),
+          out.shape[-1], _ptr(dq), dq.shape[-1], nk, _ptr(kv), kv.shape[-1], _ptr(dkv), dkv.shape[-1], _ptr(lse),
+          _ptr(ws), ws.numel(), _stream(stream))
 
 
 def ff_debug_gemm_gated(A, B, bias, resid, gate, rows_per_sample, stream=None):

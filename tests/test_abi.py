@@ -175,15 +175,26 @@ def test_training_pass_host_validation(L):
     assert L.ff_dit_backward(h, 2, 16, 16, None, None, 256, 1 << 40, None) == 1
     assert L.ff_dit_backward(h, 2, 16, 16, 16, None, 255, 1 << 40, None) == 1
     assert L.ff_dit_destroy(h) == 0
-    # head_dim 64 models have a training pass; WAN models do not
+    # head_dim 64 models and WAN models have a training pass too
     c64 = ffi.make_config(synth.config("tiny_mmdit"))
     assert L.ff_dit_create(C.byref(c64), C.c_void_p(256), C.byref(h)) == 0
     assert L.ff_dit_train_workspace_size(h, 4, C.byref(n)) == 0
     assert L.ff_dit_destroy(h) == 0
-    wan = ffi.make_config(dict(synth.config("wan_40"), hidden=256, heads=2, mlp=512, n_double=1, grid=(2, 4, 4),
-                               rope_axes=(44, 42, 42)))
+    wcfg = dict(synth.config("wan_40"), hidden=256, heads=2, mlp=512, n_double=2, grid=(2, 4, 4),
+                rope_axes=(44, 42, 42))
+    wan = ffi.make_config(wcfg)
     assert L.ff_dit_create(C.byref(wan), C.c_void_p(256), C.byref(h)) == 0
+    assert L.ff_dit_train_workspace_size(h, 4, C.byref(n)) == 0
+    # per block: three fp32 residuals, nine bf16 [R_i, H] values, raw and
+    # normalised qkv, the MLP's two [R_i, F] values, the text's raw and
+    # normalised k | v
+    Ri, Rt = 4 * 32, 4 * wcfg["n_txt"]
+    assert n.value >= 2 * (Ri * (42 * 256 + 4 * 512) + Rt * 8 * 256)
+    assert L.ff_dit_destroy(h) == 0
+    wodd = ffi.make_config(dict(wcfg, n_txt=5))      # B N_t = 20: not a multiple of 8
+    assert L.ff_dit_create(C.byref(wodd), C.c_void_p(256), C.byref(h)) == 0
     assert L.ff_dit_train_workspace_size(h, 4, C.byref(n)) == 2
+    assert L.ff_dit_train_workspace_size(h, 8, C.byref(n)) == 0
     assert L.ff_dit_destroy(h) == 0
     # the log-prob backward
     assert L.ff_sde_logprob_backward(2, 18, 16, 16, 16, 16, 16, 16, 0, 16, 1, 16, None) == 2   # D % 4

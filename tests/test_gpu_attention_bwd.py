@@ -70,3 +70,43 @@ def test_attention_backward_parity(cuda, d, B, heads, n0, n1):
             assert err <= 2e-2, (b, name, err)
     # columns past 3H are not written
     assert float(dq1[:, 3 * H:].float().abs().max()) == 0.0
+
+
+@pytest.mark.parametrize("d,B,heads,nq,nk", [(128, 2, 2, 130, 77), (128, 1, 3, 300, 512), (64, 2, 4, 5, 200),
+                                             (64, 1, 2, 777, 33), (128, 1, 2, 64, 3)])
+def test_cross_attention_backward_parity(cuda, d, B, heads, nq, nk):
+    """Latent queries against text keys / values (the WAN block's
+    cross-attention): lse and dq, dk, dv against the fp64 definitions."""
+    import torch
+    from paper_2602_12529_gb300 import ffi
+    H = heads * d
+    qb = _bits((B * nq, H), 41, "cq")
+    kvb = _bits((B * nk, 2 * H), 42, "ckv")
+    gb = _bits((B * nq, H), 43, "cg")
+    L = ffi.lib().ff_attention_lse_rows(nq, 0)
+    lse = torch.zeros(B * heads * L, dtype=torch.float32, device=cuda)
+    q, kv = _dev(qb, cuda), _dev(kvb, cuda)
+    o = torch.zeros((B * nq, H), dtype=torch.bfloat16, device=cuda)
+    ffi.ff_cross_attention_forward(B, heads, d, q, nq, kv, nk, o, lse=lse)
+    dq = torch.zeros((B * nq, H), dtype=torch.bfloat16, device=cuda)
+    dkv = torch.zeros((B * nk, 2 * H + 64), dtype=torch.bfloat16, device=cuda)
+    ffi.ff_cross_attention_backward(B, heads, d, q, nq, o, _dev(gb, cuda), dq, kv, nk, dkv, lse)
+    torch.cuda.synchronize()
+    assert ffi.ff_check_device_status() == 0
+    wq, wkv, wg = odit.widen(qb), odit.widen(kvb), odit.widen(gb)
+    lse_h = lse.cpu().numpy().reshape(B, heads, L)
+    gq, gkv = _host(dq), _host(dkv)
+    for b in range(B):
+        qh = wq[b * nq:(b + 1) * nq].reshape(nq, heads, d)
+        kh = wkv[b * nk:(b + 1) * nk, :H].reshape(nk, heads, d)
+        vh = wkv[b * nk:(b + 1) * nk, H:].reshape(nk, heads, d)
+        gh = wg[b * nq:(b + 1) * nq].reshape(nq, heads, d)
+        np.testing.assert_allclose(lse_h[b, :, :nq].T, odit.attention_lse(qh, kh) / math.log(2.0),
+                                   rtol=2e-4, atol=2e-4)
+        want_dq, want_dk, want_dv = odit.attention_backward(qh, kh, vh, gh)
+        for name, got, want in (("dq", gq[b * nq:(b + 1) * nq], want_dq),
+                                ("dk", gkv[b * nk:(b + 1) * nk, :H], want_dk),
+                                ("dv", gkv[b * nk:(b + 1) * nk, H:2 * H], want_dv)):
+            err = rms_rel(got, want.reshape(-1, H))
+            assert err <= 2e-2, (b, name, err)
+    assert float(dkv[:, 2 * H:].float().abs().max()) == 0.0

@@ -1,7 +1,7 @@
 """GPU parity of the training pass (ff_dit_forward_train, ff_dit_backward,
 ff_sde_logprob_backward) against the fp64 oracle's vector-Jacobian product
-(oracle/dit_grad.py), tensor by tensor, on small MMDiTs; properties of the
-Flux-shaped block at full size."""
+(oracle/dit_grad.py), tensor by tensor, on small MMDiTs and WAN-style models;
+properties of the Flux-shaped block at full size."""
 import numpy as np
 import pytest
 
@@ -77,7 +77,8 @@ class Run:
 
     def oracle(self, dv):
         P = odit.widen_params(self.W)
-        return dit_grad.velocity_vjp(P, self.cfg, self.x, odit.widen(self.txt), self.t.astype(np.float64), dv)
+        vjp = dit_grad.wan_velocity_vjp if self.cfg["arch"] == "wan" else dit_grad.velocity_vjp
+        return vjp(P, self.cfg, self.x, odit.widen(self.txt), self.t.astype(np.float64), dv)
 
 
 def _compare(run, grad, dx, want_G, want_dx):
@@ -116,6 +117,42 @@ def test_forward_train_equals_velocity_and_backward_is_deterministic(cuda):
     torch.cuda.synchronize()
     assert torch.equal(v, run.v)
     dv = np.random.default_rng(6).standard_normal(tuple(v.shape)).astype(np.float32)
+    g1, d1 = run.backward(dv)
+    g2, d2 = run.backward(dv)
+    assert np.array_equal(g1, g2) and np.array_equal(d1, d2)
+
+
+WAN_TRAIN = dict(name="wan_train", arch="wan", hidden=256, heads=2, head_dim=128, mlp=512, n_double=1,
+                 n_single=0, patch_dim=64, txt_dim=128, n_txt=16, grid=(2, 4, 4), rope_axes=(44, 42, 42),
+                 rope_theta=10000.0, time_freq_dim=256, batch=2)
+
+
+@pytest.mark.parametrize("over", [{}, {"n_double": 2},
+                                  {"heads": 4, "head_dim": 64, "rope_axes": (20, 22, 22)},
+                                  {"grid": (1, 3, 5), "n_txt": 5, "batch": 8},
+                                  {"batch": 3, "n_txt": 8, "grid": (2, 2, 6), "n_double": 2}])
+def test_wan_backward_matches_oracle(cuda, over):
+    """The WAN-style block's backward (affine LN, ungated cross-attention with
+    text keys / values, shared modulation) against wan_velocity_vjp."""
+    cfg = dict(WAN_TRAIN, **over)
+    run = Run(cfg, cuda)
+    dv = np.random.default_rng(7).standard_normal((cfg["batch"], synth.n_img(cfg), cfg["patch_dim"])).astype(np.float32)
+    grad, dx = run.backward(dv)
+    v_ref, G, dx_ref = run.oracle(dv.astype(np.float64))
+    assert rms_rel(run.v.cpu().numpy(), v_ref) <= V_TOL
+    _compare(run, grad, dx, G, dx_ref)
+
+
+def test_wan_forward_train_equals_velocity_and_backward_is_deterministic(cuda):
+    import torch
+    cfg = dict(WAN_TRAIN, n_double=2)
+    run = Run(cfg, cuda, seed=2)
+    ws = torch.empty(run.model.workspace_size(run.B), dtype=torch.uint8, device=cuda)
+    v = torch.empty_like(run.xg)
+    run.model.ff_dit_velocity(run.xg, run.tg, run.tt, v, ws)
+    torch.cuda.synchronize()
+    assert torch.equal(v, run.v)
+    dv = np.random.default_rng(9).standard_normal(tuple(v.shape)).astype(np.float32)
     g1, d1 = run.backward(dv)
     g2, d2 = run.backward(dv)
     assert np.array_equal(g1, g2) and np.array_equal(d1, d2)
