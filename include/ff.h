@@ -375,7 +375,7 @@ int ff_dit_velocity(const ff_dit* model, int B, const float* x_t, const void* tx
                     cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
- * Training pass of the velocity network (MMDiT models): the
+ * Training pass of the velocity network (MMDiT and WAN-style models): the
  * forward every GRPO-style trainer runs "again for training" (Sec. 1) and
  * its gradient, for the policy losses of Sec. 3 (the Flow-GRPO loss through
  * ff_sde_logprob_backward, AWM's Eq. 3 through ff_awm_loss's dL/dv).
@@ -394,7 +394,8 @@ int ff_dit_velocity(const ff_dit* model, int B, const float* x_t, const void* tx
  *   over tokens runs in a fixed order: the result is deterministic.
  * Requires B N_t and B N_i multiples of 8.  The workspace holds about
  * R (30 H + 4 F) bytes per double-stream block and R (22 H + 4 F) per
- * single-stream block, R = B (N_t + N_i), plus scratch.
+ * single-stream block, R = B (N_t + N_i), plus scratch; per WAN block
+ * R_i (42 H + 4 F) + 8 R_t H bytes (R_i = B N_i, R_t = B N_t).
  * ------------------------------------------------------------------------ */
 int ff_dit_train_workspace_size(const ff_dit* model, int B, size_t* bytes);
 int ff_dit_forward_train(const ff_dit* model, int B, const float* x_t, const void* txt,

@@ -275,3 +275,76 @@ def test_wan_bias_gradients_are_token_sums():
     # mod.b receives what every block's bias receives (e0 + b_l: same partials)
     np.testing.assert_allclose(G["mod.b"], sum(G[f"blocks.{l}.mod.b"] for l in range(cfg["n_double"])),
                                rtol=1e-12, atol=1e-14)
+
+
+# ---------------------------------------------------------------- the pins catch planted mistakes
+
+def _worst_mismatch(vjp, vel, cfg, P):
+    """Largest |numeric - analytic| / max(1, |numeric|) over one random
+    direction per parameter tensor and one for x_t."""
+    x, txt, t = _inputs(cfg)
+    rng = np.random.default_rng(31)
+    dv = rng.standard_normal((cfg["batch"], synth.n_img(cfg), cfg["patch_dim"]))
+    _, G, dx = vjp(P, cfg, x, txt, t, dv)
+
+    def loss(Pm, xm=x):
+        return float(np.sum(dv * vel(Pm, cfg, xm, txt, t)))
+
+    h, worst = 1e-5, 0.0
+    for name in P:
+        d = rng.standard_normal(P[name].shape)
+        Pp, Pm = dict(P), dict(P)
+        Pp[name] = P[name] + h * d
+        Pm[name] = P[name] - h * d
+        num = (loss(Pp) - loss(Pm)) / (2 * h)
+        worst = max(worst, abs(num - float(np.sum(G[name] * d))) / max(1.0, abs(num)))
+    d = rng.standard_normal(x.shape)
+    num = (loss(P, x + h * d) - loss(P, x - h * d)) / (2 * h)
+    return max(worst, abs(num - float(np.sum(dx * d))) / max(1.0, abs(num)))
+
+
+def _ln_no_projection(x, dn, eps=dit.LN_EPS):
+    mu = x.mean(axis=-1, keepdims=True)
+    s = np.sqrt(((x - mu) ** 2).mean(axis=-1, keepdims=True) + eps)
+    return (dn - dn.mean(axis=-1, keepdims=True)) / s          # drops - n mean(dn n)
+
+
+_RMS_BWD = dit_grad.rms_norm_bwd
+
+
+def _rms_sign(x, w, dy, eps=dit.RMS_EPS):
+    dx, dw = _RMS_BWD(x, w, dy, eps)
+    return dx, -dw                                              # wrong sign of the scale gradient
+
+
+def _rope_untransposed(dy, angles):
+    return dit.apply_rope(dy, angles)                          # rotation not transposed
+
+
+def _silu_half(x):
+    return 1.0 / (1.0 + np.exp(-x))                            # drops the x sigma (1 - sigma) term
+
+
+def _gelu_no_cubic(x):
+    th = np.tanh(np.sqrt(2.0 / np.pi) * (x + 0.044715 * x ** 3))
+    return 0.5 * (1.0 + th) + 0.5 * x * (1.0 - th * th) * np.sqrt(2.0 / np.pi)   # drops 3 c x^2
+
+
+def _modulate_no_scale(n, scale, dy):
+    return dy, dy.sum(axis=0), (dy * n).sum(axis=0)             # drops the (1 + scale) factor
+
+
+@pytest.mark.parametrize("arch", ["mmdit", "wan"])
+@pytest.mark.parametrize("target,wrong", [("layer_norm_bwd", _ln_no_projection), ("rms_norm_bwd", _rms_sign),
+                                          ("rope_bwd", _rope_untransposed), ("silu_grad", _silu_half),
+                                          ("gelu_tanh_grad", _gelu_no_cubic), ("modulate_bwd", _modulate_no_scale)])
+def test_planted_mistakes_fail_the_central_difference_pin(monkeypatch, arch, target, wrong):
+    if arch == "wan":
+        cfg, P = dict(WAN_TINY, n_double=1), _wan_params(dict(WAN_TINY, n_double=1))
+        vjp, vel = dit_grad.wan_velocity_vjp, dit.wan_velocity
+    else:
+        cfg = _cfg()
+        P, vjp, vel = _params(cfg), dit_grad.velocity_vjp, dit.velocity
+    assert _worst_mismatch(vjp, vel, cfg, P) <= 1e-6
+    monkeypatch.setattr(dit_grad, target, wrong)
+    assert _worst_mismatch(vjp, vel, cfg, P) > 1e-4
