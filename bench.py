@@ -720,11 +720,11 @@ def run_ours(args):
     ffi.ff_sde_step_logprob(x, v, eps, x_next, t, tn, sg, logp, ws=ws_sde)
     torch.add(logp, jitter, out=lp_old)
 
-    def step(xi=x, txti=txt, epsi=eps, ti=t, tni=tn, sgi=sg, ri=rewards, lpo=lp_old):
+    def step(xi=x, txti=txt, epsi=eps, ti=t, tni=tn, sgi=sg, ri=rewards, lpo=lp_old, xo=x_next, lpn=logp, lo=loss):
         model.ff_dit_velocity(xi, txti, ti, v, ws)
-        ffi.ff_sde_step_logprob(xi, v, epsi, x_next, ti, tni, sgi, logp, ws=ws_sde)
+        ffi.ff_sde_step_logprob(xi, v, epsi, xo, ti, tni, sgi, lpn, ws=ws_sde)
         ffi.ff_group_advantage(ri, G, cfg["eps_adv"], adv_all)
-        ffi.ff_grpo_loss(logp, lpo, adv, cfg["clip"], cfg["clip"], loss, grad, ws=ws_loss)
+        ffi.ff_grpo_loss(lpn, lpo, adv, cfg["clip"], cfg["clip"], lo, grad, ws=ws_loss)
 
     clocks = ClockSampler(local) if rank == 0 else None
     for _ in range(args.warmup):
@@ -791,31 +791,44 @@ def run_ours(args):
     dit_flops = sum(v[2] for v in kern.values()) / args.steps
     secondary = {k: roof(k) for k in ("attention", "sde_step") if k in kern}
 
-    # ---- end to end through the public API with host inputs
+    # ---- end to end through the public API with host inputs: every step
+    # copies its inputs in from pinned host memory and its results (x_next,
+    # log-probs, loss) out; HostFedPipeline overlaps step k + 1's copies in
+    # and step k's copies out with step k's kernels (two device buffer sets,
+    # a copy stream, events).  The serial form (copies on the compute stream)
+    # is reported beside it.
+    from paper_2602_12529_gb300.pipeline import HostFedPipeline
     pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
-    hx, htxt, heps = pin(h_x), pin(h_txt), pin(h_eps)
-    ht, htn, hsg, hr, hlpo = pin(h_t), pin(h_tn), pin(h_sg), pin(h_r), lp_old.cpu().pin_memory()
-    o_x = torch.empty(x.shape, dtype=torch.float32).pin_memory()
-    o_lp = torch.empty((B, 1), dtype=torch.float32).pin_memory()
-    o_loss = torch.empty(1, dtype=torch.float32).pin_memory()
-    dx, dtxt, deps = torch.empty_like(x), torch.empty_like(txt.view(torch.int16)), torch.empty_like(eps)
-    dt_, dtn, dsg, dr, dlpo = (torch.empty_like(t), torch.empty_like(tn), torch.empty_like(sg),
-                               torch.empty_like(rewards), torch.empty_like(lp_old))
-    h2d = sum(a.numel() * a.element_size() for a in (hx, htxt, heps, ht, htn, hsg, hr, hlpo))
-    d2h = sum(a.numel() * a.element_size() for a in (o_x, o_lp, o_loss))
+    h_in = {"x": pin(h_x), "txt": pin(h_txt), "eps": pin(h_eps), "t": pin(h_t), "tn": pin(h_tn), "sg": pin(h_sg),
+            "r": pin(h_r), "lpo": lp_old.cpu().pin_memory()}
+    h_out = [{"x_next": torch.empty(x.shape, dtype=torch.float32).pin_memory(),
+              "logp": torch.empty((B, 1), dtype=torch.float32).pin_memory(),
+              "loss": torch.empty(1, dtype=torch.float32).pin_memory()} for _ in range(2)]
+    h2d = sum(a.numel() * a.element_size() for a in h_in.values())
+    d2h = sum(a.numel() * a.element_size() for a in h_out[0].values())
 
-    def e2e_step():
-        for d_, h_ in ((dx, hx), (dtxt, htxt), (deps, heps), (dt_, ht), (dtn, htn), (dsg, hsg), (dr, hr),
-                       (dlpo, hlpo)):
-            d_.copy_(h_, non_blocking=True)
-        step(dx, dtxt.view(torch.bfloat16), deps, dt_, dtn, dsg, dr, dlpo)
-        o_x.copy_(x_next, non_blocking=True)
-        o_lp.copy_(logp, non_blocking=True)
-        o_loss.copy_(loss, non_blocking=True)
+    def e2e_body(i, o):
+        step(i["x"], i["txt"].view(torch.bfloat16), i["eps"], i["t"], i["tn"], i["sg"], i["r"], i["lpo"],
+             o["x_next"], o["logp"], o["loss"])
 
-    e2e_step()
-    ms_e2e = timed(e2e_step, args.steps) / args.steps
+    like_in = {"x": x, "txt": txt.view(torch.int16), "eps": eps, "t": t, "tn": tn, "sg": sg, "r": rewards,
+               "lpo": lp_old}
+    pipe = HostFedPipeline(dev, like_in, {"x_next": x_next, "logp": logp, "loss": loss}, e2e_body)
+    K = args.steps
+    pipe.run([h_in] * 2, h_out)
+    ms_e2e = timed(lambda: pipe.run([h_in] * K, [h_out[k % 2] for k in range(K)]), 1) / K
     e2e_value = whole_job_rate(world, tokens_per_step, ms_e2e)
+
+    def e2e_serial():
+        i = pipe.ins[0]
+        for name, h_ in h_in.items():
+            i[name].copy_(h_, non_blocking=True)
+        e2e_body(i, pipe.outs[0])
+        for name, h_ in h_out[0].items():
+            h_.copy_(pipe.outs[0][name], non_blocking=True)
+
+    e2e_serial()
+    ms_e2e_serial = timed(e2e_serial, K) / K
     awm = awm_step(args, ffi, model, cfg, dev, x, txt, eps, rewards, timed, world)
     train = train_step(args, ffi, model, cfg, dev, x, txt, t, tn, sg, x_next, lp_old, adv, dit_flops, timed, world)
     bwd = backward_kernels(args, ffi, cfg, dev) if rank == 0 and not args.no_sweep else None
@@ -845,7 +858,9 @@ def run_ours(args):
                 "kernel_breakdown": breakdown,
                 "cpu_baseline": cpu,
                 "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                        "ms_per_step": ms_e2e},
+                        "ms_per_step": ms_e2e, "copies": "overlapped with the previous / next step's kernels "
+                        "(HostFedPipeline: copy stream, two device buffer sets)",
+                        "serial_ms_per_step": ms_e2e_serial},
                 "hbm_sweep": sweep,
                 "awm_step": awm,
                 "train_step": train,
