@@ -106,16 +106,35 @@ __global__ void __launch_bounds__(kThreads) gate_backward_kernel(const float* g,
 
 // ---------------------------------------------------------------- LN-modulate
 
+// Sum of three values over the CTA (same slot discipline as block_sum2).
+__device__ __forceinline__ float3 block_sum3(float3 v, float3* red, int lane, int w) {
+    v.x = warp_sum(v.x);
+    v.y = warp_sum(v.y);
+    v.z = warp_sum(v.z);
+    if (lane == 0) red[w] = v;
+    __syncthreads();
+    float3 t = make_float3(0.f, 0.f, 0.f);
+#pragma unroll
+    for (int i = 0; i < kThreads / 32; ++i) {
+        t.x += red[i].x;
+        t.y += red[i].y;
+        t.z += red[i].z;
+    }
+    return t;
+}
+
 // CTA = one chunk of rows, all H columns: thread t holds float4s t, t + 256,
-// ... of a row (PER of them).  Per row: mean and centred variance of x (as in
-// the forward), then the two means of the LayerNorm backward; the next row's
-// loads are issued before this row's reductions.
+// ... of a row (PER of them).  Per row, with d = dh (1 + scale) (or dh w):
+// one reduction of (sum x, sum d, sum d x), one of the centred variance (as
+// in the forward); mean(d n) = (sum d x - mean sum d) rstd / H.  The next
+// row's x, dh and g are loaded before this row's reductions.
 template <int PER>
 __global__ void __launch_bounds__(kThreads) ln_modulate_backward_kernel(const float* x, const float* dh, float* gx,
                                                                          int64_t ld, const float* mods,
                                                                          int64_t ld_mods, BwdSegs s, int H,
                                                                          const __nv_bfloat16* aff_w, float* part) {
-    __shared__ float2 red[3][kThreads / 32];
+    __shared__ float3 red3[2][kThreads / 32];
+    __shared__ float2 red2[2][kThreads / 32];
     BwdSeg sg;
     int b, r0, r1;
     if (!chunk_rows(s, blockIdx.x, sg, b, r0, r1)) return;
@@ -140,35 +159,48 @@ __global__ void __launch_bounds__(kThreads) ln_modulate_backward_kernel(const fl
 #pragma unroll
     for (int i = 0; i < PER; ++i) acc_sh[i] = acc_sc[i] = make_float4(0.f, 0.f, 0.f, 0.f);
     const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
-    float4 xr[PER], dr[PER];
+    float4 xr[PER], dr[PER], gr[PER];
     {
         const float4* xp = reinterpret_cast<const float4*>(x + static_cast<int64_t>(r0) * ld);
         const float4* dp = reinterpret_cast<const float4*>(dh + static_cast<int64_t>(r0) * ld);
+        const float4* gp = reinterpret_cast<const float4*>(gx + static_cast<int64_t>(r0) * ld);
 #pragma unroll
         for (int i = 0; i < PER; ++i) {
             const int k = t + kThreads * i;
             xr[i] = k < nv ? __ldcs(xp + k) : z;
             dr[i] = k < nv ? __ldcs(dp + k) : z;
+            gr[i] = k < nv ? gp[k] : z;
         }
     }
     const float invH = 1.f / H;
-    for (int r = r0; r < r1; ++r) {
-        float4 xn[PER], dn[PER];
+    int par = 0;
+    for (int r = r0; r < r1; ++r, par ^= 1) {
+        float4 xn[PER], dn[PER], gn[PER];
         {
             const bool more = r + 1 < r1;
             const float4* xp = reinterpret_cast<const float4*>(x + static_cast<int64_t>(r + 1) * ld);
             const float4* dp = reinterpret_cast<const float4*>(dh + static_cast<int64_t>(r + 1) * ld);
+            const float4* gp = reinterpret_cast<const float4*>(gx + static_cast<int64_t>(r + 1) * ld);
 #pragma unroll
             for (int i = 0; i < PER; ++i) {
                 const int k = t + kThreads * i;
                 xn[i] = more && k < nv ? __ldcs(xp + k) : z;
                 dn[i] = more && k < nv ? __ldcs(dp + k) : z;
+                gn[i] = more && k < nv ? gp[k] : z;
             }
         }
-        float sx = 0.f;
+        // d = dh (1 + scale); sums of x, d and d x
+        float sx = 0.f, sd = 0.f, sdx = 0.f;
 #pragma unroll
-        for (int i = 0; i < PER; ++i) sx += (xr[i].x + xr[i].y) + (xr[i].z + xr[i].w);
-        const float mean = block_sum2(make_float2(sx, 0.f), red[0], lane, w).x * invH;
+        for (int i = 0; i < PER; ++i) {
+            const float4 d = make_float4(dr[i].x * sc1[i].x, dr[i].y * sc1[i].y, dr[i].z * sc1[i].z,
+                                         dr[i].w * sc1[i].w);
+            sx += (xr[i].x + xr[i].y) + (xr[i].z + xr[i].w);
+            sd += (d.x + d.y) + (d.z + d.w);
+            sdx += (d.x * xr[i].x + d.y * xr[i].y) + (d.z * xr[i].z + d.w * xr[i].w);
+        }
+        const float3 s3 = block_sum3(make_float3(sx, sd, sdx), red3[par], lane, w);
+        const float mean = s3.x * invH;
         float q = 0.f;
 #pragma unroll
         for (int i = 0; i < PER; ++i) {
@@ -177,43 +209,32 @@ __global__ void __launch_bounds__(kThreads) ln_modulate_backward_kernel(const fl
                 q += (d0 * d0 + d1 * d1) + (d2 * d2 + d3 * d3);
             }
         }
-        const float rstd = rsqrtf(block_sum2(make_float2(q, 0.f), red[1], lane, w).x * invH + kLnEps);
-        // n = (x - mean) rstd, dn = dh (1 + scale); overwrite xr with n, dr with dn
-        float s1 = 0.f, s2 = 0.f;
-#pragma unroll
-        for (int i = 0; i < PER; ++i) {
-            float4 n = make_float4((xr[i].x - mean) * rstd, (xr[i].y - mean) * rstd, (xr[i].z - mean) * rstd,
-                                   (xr[i].w - mean) * rstd);
-            if (t + kThreads * i >= nv) n = z;
-            acc_sh[i].x += dr[i].x; acc_sh[i].y += dr[i].y; acc_sh[i].z += dr[i].z; acc_sh[i].w += dr[i].w;
-            acc_sc[i].x = fmaf(dr[i].x, n.x, acc_sc[i].x);
-            acc_sc[i].y = fmaf(dr[i].y, n.y, acc_sc[i].y);
-            acc_sc[i].z = fmaf(dr[i].z, n.z, acc_sc[i].z);
-            acc_sc[i].w = fmaf(dr[i].w, n.w, acc_sc[i].w);
-            const float4 d = make_float4(dr[i].x * sc1[i].x, dr[i].y * sc1[i].y, dr[i].z * sc1[i].z, dr[i].w * sc1[i].w);
-            s1 += (d.x + d.y) + (d.z + d.w);
-            s2 += (d.x * n.x + d.y * n.y) + (d.z * n.z + d.w * n.w);
-            xr[i] = n;
-            dr[i] = d;
-        }
-        const float2 m = block_sum2(make_float2(s1, s2), red[2], lane, w);
-        const float m1 = m.x * invH, m2 = m.y * invH;
+        const float rstd = rsqrtf(block_sum2(make_float2(q, 0.f), red2[par], lane, w).x * invH + kLnEps);
+        const float m1 = s3.y * invH, m2 = (s3.z - mean * s3.y) * rstd * invH;
         float4* gp = reinterpret_cast<float4*>(gx + static_cast<int64_t>(r) * ld);
 #pragma unroll
         for (int i = 0; i < PER; ++i) {
             const int k = t + kThreads * i;
             if (k >= nv) continue;
-            float4 o = gp[k];
-            o.x += rstd * (dr[i].x - m1 - xr[i].x * m2);
-            o.y += rstd * (dr[i].y - m1 - xr[i].y * m2);
-            o.z += rstd * (dr[i].z - m1 - xr[i].z * m2);
-            o.w += rstd * (dr[i].w - m1 - xr[i].w * m2);
+            const float4 n = make_float4((xr[i].x - mean) * rstd, (xr[i].y - mean) * rstd, (xr[i].z - mean) * rstd,
+                                         (xr[i].w - mean) * rstd);
+            acc_sh[i].x += dr[i].x; acc_sh[i].y += dr[i].y; acc_sh[i].z += dr[i].z; acc_sh[i].w += dr[i].w;
+            acc_sc[i].x = fmaf(dr[i].x, n.x, acc_sc[i].x);
+            acc_sc[i].y = fmaf(dr[i].y, n.y, acc_sc[i].y);
+            acc_sc[i].z = fmaf(dr[i].z, n.z, acc_sc[i].z);
+            acc_sc[i].w = fmaf(dr[i].w, n.w, acc_sc[i].w);
+            float4 o = gr[i];
+            o.x += rstd * (dr[i].x * sc1[i].x - m1 - n.x * m2);
+            o.y += rstd * (dr[i].y * sc1[i].y - m1 - n.y * m2);
+            o.z += rstd * (dr[i].z * sc1[i].z - m1 - n.z * m2);
+            o.w += rstd * (dr[i].w * sc1[i].w - m1 - n.w * m2);
             gp[k] = o;
         }
 #pragma unroll
         for (int i = 0; i < PER; ++i) {
             xr[i] = xn[i];
             dr[i] = dn[i];
+            gr[i] = gn[i];
         }
     }
     float4* p = reinterpret_cast<float4*>(part + static_cast<int64_t>(blockIdx.x) * 2 * H);
