@@ -1021,14 +1021,21 @@ __global__ void __launch_bounds__(kGemvThreads) gemv_rows_kernel(const __nv_bflo
         for (int j = 0; j < kGemvCols; ++j)
             w[j] = reinterpret_cast<const uint4*>(W + static_cast<int64_t>(min(n0 + j, N - 1)) * ldw);
         // per lane: K chunks lane, lane + 32, ...; two chunks of every column
-        // in flight (8 independent 16-byte loads) before they are used
+        // (8 independent 16-byte loads) per step, and the next step's loads
+        // are issued before this step's arithmetic
+        uint4 wv[2][kGemvCols];
+#pragma unroll
+        for (int j = 0; j < kGemvCols; ++j) {
+            wv[0][j] = lane < k8 ? __ldcs(w[j] + lane) : make_uint4(0u, 0u, 0u, 0u);
+            wv[1][j] = lane + 32 < k8 ? __ldcs(w[j] + lane + 32) : make_uint4(0u, 0u, 0u, 0u);
+        }
         for (int c = lane; c < k8; c += 64) {
-            uint4 wv[2][kGemvCols];
             const bool two = c + 32 < k8;
+            uint4 wn[2][kGemvCols];
 #pragma unroll
             for (int j = 0; j < kGemvCols; ++j) {
-                wv[0][j] = __ldcs(w[j] + c);
-                wv[1][j] = two ? __ldcs(w[j] + c + 32) : make_uint4(0u, 0u, 0u, 0u);
+                wn[0][j] = c + 64 < k8 ? __ldcs(w[j] + c + 64) : make_uint4(0u, 0u, 0u, 0u);
+                wn[1][j] = c + 96 < k8 ? __ldcs(w[j] + c + 96) : make_uint4(0u, 0u, 0u, 0u);
             }
 #pragma unroll
             for (int u = 0; u < 2; ++u) {
@@ -1048,6 +1055,11 @@ __global__ void __launch_bounds__(kGemvThreads) gemv_rows_kernel(const __nv_bflo
                         }
                     }
                 }
+            }
+#pragma unroll
+            for (int j = 0; j < kGemvCols; ++j) {
+                wv[0][j] = wn[0][j];
+                wv[1][j] = wn[1][j];
             }
         }
 #pragma unroll
