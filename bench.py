@@ -276,6 +276,42 @@ def run_reference(args):
 # the CUDA path
 # ---------------------------------------------------------------------------
 
+def at_config_small_kernels(ffi, dev, hbm_peak, cases, reps=100):
+    """Per-launch time of each case at the workload's sizes: `reps`
+    back-to-back calls captured in one CUDA graph, replayed three times
+    (median).  The inputs fit in L2, so these are launch- and L2-bound; the
+    HBM sweep gives the bandwidth at sizes beyond L2."""
+    import torch
+    out = {}
+    for name, (fn, nbytes) in cases.items():
+        fn()
+        side = torch.cuda.Stream(dev)
+        side.wait_stream(torch.cuda.current_stream(dev))
+        with torch.cuda.stream(side):
+            fn()
+        torch.cuda.current_stream(dev).wait_stream(side)
+        torch.cuda.synchronize(dev)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            for _ in range(reps):
+                fn()
+        g.replay()
+        torch.cuda.synchronize(dev)
+        ts = []
+        for _ in range(3):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            g.replay()
+            e1.record()
+            torch.cuda.synchronize(dev)
+            ts.append(e0.elapsed_time(e1))
+        us = sorted(ts)[1] * 1e3 / reps
+        out[name] = {"us_per_call": us, "bytes": nbytes, "gbs": nbytes / us / 1e3,
+                     "frac_of_hbm": nbytes / us / 1e3 / hbm_peak, "calls_per_graph": reps}
+        del g
+    return out
+
+
 def hbm_sweep(ffi, dev, hbm_peak, l2_bytes=129 * 2 ** 20):
     """Bandwidth of the memory-bound kernels at sizes well beyond L2, with
     enough rotating buffer sets that every launch reads from HBM."""
@@ -831,6 +867,19 @@ def run_ours(args):
     ms_e2e_serial = timed(e2e_serial, K) / K
     awm = awm_step(args, ffi, model, cfg, dev, x, txt, eps, rewards, timed, world)
     train = train_step(args, ffi, model, cfg, dev, x, txt, t, tn, sg, x_next, lp_old, adv, dit_flops, timed, world)
+    at_cfg = None
+    if rank == 0 and not args.no_sweep:
+        # the memory-bound kernels at the workload's own sizes (inputs L2-resident):
+        # 100 back-to-back launches captured in one CUDA graph, per-launch time
+        sde_bytes = 16.0 * x.numel()
+        at_cfg = at_config_small_kernels(ffi, dev, hbm, {
+            "sde_step (SAMPLE, log-prob)": (lambda: ffi.ff_sde_step_logprob(x, v, eps, x_next, t, tn, sg, logp,
+                                                                             ws=ws_sde), sde_bytes),
+            "group_advantage": (lambda: ffi.ff_group_advantage(rewards, G, cfg["eps_adv"], adv_all),
+                                8.0 * rewards.numel()),
+            "grpo_loss (+ dL/dlp)": (lambda: ffi.ff_grpo_loss(logp, lp_old, adv, cfg["clip"], cfg["clip"], loss, grad,
+                                                              ws=ws_loss), 16.0 * logp.numel() + 4.0 * B),
+        })
     bwd = backward_kernels(args, ffi, cfg, dev) if rank == 0 and not args.no_sweep else None
     wan_train = wan_block_train(args, ffi, dev, timed) if rank == 0 and world == 1 and not args.no_sweep else None
     sweep = hbm_sweep(ffi, dev, hbm) if rank == 0 and not args.no_sweep else None
@@ -862,6 +911,7 @@ def run_ours(args):
                         "(HostFedPipeline: copy stream, two device buffer sets)",
                         "serial_ms_per_step": ms_e2e_serial},
                 "hbm_sweep": sweep,
+                "small_kernels_at_config": at_cfg,
                 "awm_step": awm,
                 "train_step": train,
                 "backward_kernels": bwd,
