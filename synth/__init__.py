@@ -137,7 +137,8 @@ def weights(specs, seed: int = 0, std: float = 0.02, bias_std: float = 0.0,
 
 
 # ---------------------------------------------------------------------------
-# Activations and rollout randomness (seeds as stated in the design doc).
+# Activations and rollout randomness: text embeddings seed 1, initial latent
+# seed 2, step-k noise seed 100 + k, rewards seed 7, old-log-prob jitter seed 9.
 # ---------------------------------------------------------------------------
 
 def text_embeds(cfg: dict, seed: int = 1, batch: int | None = None) -> np.ndarray:
