@@ -277,6 +277,7 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_const
         const uint32_t tS = tmem + (static_cast<uint32_t>(q * 32) << 16);
         const int64_t li = (static_cast<int64_t>(b) * gridDim.y + h) * p.lse_rows + p.lse_base[seg] + row;
         const bool live = row < p.nq[seg];
+        const bool full_rows = q0 + kT <= p.nq[seg];   // every row of the tile is real (warp-uniform)
         const float lse = live ? p.lse[li] : 0.f;
         const float dd = live ? p.delta[li] : 0.f;
         bool ok = true;
@@ -292,15 +293,28 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_const
             const int ks = j < nt0 ? 0 : 1;
             // key columns < valid of this warp's 32 are real
             const int valid = p.nk[ks] - (j - (ks ? nt0 : 0)) * kT - hf * kSub - cg * 32;
+            if (valid >= 32 && full_rows) {
+                // every column and row real: paired fp32 arithmetic, no selects
+                const float2 c2 = make_float2(p.scale_log2, p.scale_log2), nl2 = make_float2(-lse, -lse);
+                const float2 nd2 = make_float2(-dd, -dd);
 #pragma unroll
-            for (int i = 0; i < 32; i += 2) {
-                float ds[2];
-#pragma unroll
-                for (int e = 0; e < 2; ++e) {
-                    const float pv = ex2(fmaf(__uint_as_float(sr[i + e]), p.scale_log2, -lse));
-                    ds[e] = (i + e < valid && live) ? pv * (__uint_as_float(pr_[i + e]) - dd) : 0.f;
+                for (int i = 0; i < 32; i += 2) {
+                    const float2 x = __ffma2_rn(make_float2(__uint_as_float(sr[i]), __uint_as_float(sr[i + 1])), c2, nl2);
+                    const float2 dp = __fadd2_rn(make_float2(__uint_as_float(pr_[i]), __uint_as_float(pr_[i + 1])), nd2);
+                    const float2 ds = __fmul2_rn(make_float2(ex2(x.x), ex2(x.y)), dp);
+                    sr[i / 2] = pack_bf16x2(ds.x, ds.y);
                 }
-                sr[i / 2] = pack_bf16x2(ds[0], ds[1]);
+            } else {
+#pragma unroll
+                for (int i = 0; i < 32; i += 2) {
+                    float ds[2];
+#pragma unroll
+                    for (int e = 0; e < 2; ++e) {
+                        const float pv = ex2(fmaf(__uint_as_float(sr[i + e]), p.scale_log2, -lse));
+                        ds[e] = (i + e < valid && live) ? pv * (__uint_as_float(pr_[i + e]) - dd) : 0.f;
+                    }
+                    sr[i / 2] = pack_bf16x2(ds[0], ds[1]);
+                }
             }
             // packed over this warp's own (already read) S columns
             tmem_st_x16(tb + cg * 32, sr);
@@ -512,18 +526,36 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_con
             tmem_ld_x32(tb + cg * 32, sr);
             tmem_ld_x32(tb + kSub + cg * 32, pr_);
             tmem_ld_wait();
+            if (valid >= 32) {
+                // every query column real: paired fp32 arithmetic, no selects
+                const float2 c2 = make_float2(p.scale_log2, p.scale_log2);
 #pragma unroll
-            for (int c = 0; c < 32; c += 2) {
-                float pv[2], ds[2];
-#pragma unroll
-                for (int e = 0; e < 2; ++e) {
-                    const bool real = c + e < valid;
-                    const float x = ex2(fmaf(__uint_as_float(sr[c + e]), p.scale_log2, -lse[c + e]));
-                    pv[e] = real ? x : 0.f;
-                    ds[e] = real ? x * (__uint_as_float(pr_[c + e]) - dl[c + e]) : 0.f;
+                for (int c = 0; c < 32; c += 2) {
+                    const float2 l2 = *reinterpret_cast<const float2*>(lse + c);
+                    const float2 d2 = *reinterpret_cast<const float2*>(dl + c);
+                    const float2 x = __ffma2_rn(make_float2(__uint_as_float(sr[c]), __uint_as_float(sr[c + 1])), c2,
+                                                make_float2(-l2.x, -l2.y));
+                    const float2 pv = make_float2(ex2(x.x), ex2(x.y));
+                    const float2 dp = __fadd2_rn(make_float2(__uint_as_float(pr_[c]), __uint_as_float(pr_[c + 1])),
+                                                 make_float2(-d2.x, -d2.y));
+                    const float2 ds = __fmul2_rn(pv, dp);
+                    sr[c / 2] = pack_bf16x2(pv.x, pv.y);
+                    pr_[c / 2] = pack_bf16x2(ds.x, ds.y);
                 }
-                sr[c / 2] = pack_bf16x2(pv[0], pv[1]);
-                pr_[c / 2] = pack_bf16x2(ds[0], ds[1]);
+            } else {
+#pragma unroll
+                for (int c = 0; c < 32; c += 2) {
+                    float pv[2], ds[2];
+#pragma unroll
+                    for (int e = 0; e < 2; ++e) {
+                        const bool real = c + e < valid;
+                        const float x = ex2(fmaf(__uint_as_float(sr[c + e]), p.scale_log2, -lse[c + e]));
+                        pv[e] = real ? x : 0.f;
+                        ds[e] = real ? x * (__uint_as_float(pr_[c + e]) - dl[c + e]) : 0.f;
+                    }
+                    sr[c / 2] = pack_bf16x2(pv[0], pv[1]);
+                    pr_[c / 2] = pack_bf16x2(ds[0], ds[1]);
+                }
             }
             // packed over this warp's own (already read) S^T / dP^T columns
             tmem_st_x16(tb + cg * 32, sr);
