@@ -19,11 +19,14 @@ Modules:
            policies read from the cited method).
   dit   -- the flow-matching DiT velocity v_theta(x_t, t): MMDiT double- and
            single-stream blocks (adaLN modulation, QK-RMSNorm, RoPE, joint
-           attention, GELU MLP) and the final projection.
+           attention, GELU MLP) and the final projection, and the WAN-style
+           network (self-attention, text cross-attention, FFN).
   dit_grad -- the gradient of <dv, v_theta> with respect to every weight and
            x_t: the training pass's vector-Jacobian product, one elementary
            backward per forward step.
   linalg -- the three dense products of a Linear's backward.
+  philox -- counter-based Gaussian noise for SAMPLE steps: Philox4x32-10 and
+           the Box-Muller transform.
 
 Every array is float64; bf16 weights and inputs are widened exactly.  Nothing
 is rounded between steps.
@@ -32,5 +35,7 @@ Parity status: sde, grpo and awm are pinned by closed forms; the DiT pieces are
 pinned one by one (attention, RoPE, norms, GELU, modulation identity) and the
 whole velocity only through those pieces plus invariants ("parity unpinned" as
 a whole: no printed outputs exist for a random-init network).  dit_grad is
-pinned by central differences of that velocity, per tensor.
+pinned by central differences of that velocity, per tensor.  philox is pinned
+by an independent library implementation of the generator and by the
+Gaussian statistics of its output.
 """
