@@ -148,6 +148,34 @@ int ff_sde_step_logprob(int B, int64_t D, const float* x_t, const float* v,
                         cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
+ * Counter-based noise for SAMPLE steps (the eps of Eq. 1 drawn on the device;
+ * the paper does not say where the noise comes from).  Philox4x32 with 10
+ * rounds (Salmon, Moraes, Dror, Shaw, SC 2011) and the Box-Muller transform:
+ * elements 4g .. 4g + 3 of sample b in stream `rng_stream` (the step index)
+ * come from one call with counter (g, b, rng_stream, 0) and key (seed mod
+ * 2^32, seed div 2^32).  Each output word w gives u = (floor(w / 512) + 1/2)
+ * 2^-23, and the pairs (u0, u1), (u2, u3) give sqrt(-2 ln u0) (cos 2 pi u1,
+ * sin 2 pi u1), sqrt(-2 ln u2) (cos 2 pi u3, sin 2 pi u3).  Any element of
+ * any step is reproducible from (seed, rng_stream, b, index) alone.
+ *
+ * ff_philox_normal: out [B, D] fp32 (device, 16-byte aligned) = those noises.
+ * ff_sde_step_logprob_philox: ff_sde_step_logprob in FF_SDE_SAMPLE mode with
+ *   eps drawn inside the kernel instead of read (12 bytes per element of
+ *   HBM traffic instead of 16); x_next and logp equal those of
+ *   ff_sde_step_logprob given eps = ff_philox_normal(B, D, seed, rng_stream)
+ *   up to the order of floating-point operations.
+ * D a multiple of 4 and D / 4 < 2^32; other arguments and errors as
+ * ff_sde_step_logprob.
+ * ------------------------------------------------------------------------ */
+int ff_philox_normal(int B, int64_t D, uint64_t seed, uint32_t rng_stream, float* out,
+                     cudaStream_t stream);
+int ff_sde_step_logprob_philox(int B, int64_t D, const float* x_t, const float* v,
+                               float* x_next, const float* t, const float* t_next,
+                               const float* sigma, uint64_t seed, uint32_t rng_stream,
+                               int reduce, float* logp, int ld, void* ws, size_t ws_bytes,
+                               cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
  * Gradient of the transition log-probability in v, with x_next held fixed
  * (the training pass of Flow-GRPO, Sec. 3.1, re-scores the rollout's x_next
  * under the current velocity).  From Eq. 1, mean depends on v as

@@ -5,7 +5,8 @@
 //   mean = x - Delta (v + a (x + (1 - t) v)) = cx x + cv v,
 //          cx = 1 - Delta a,  cv = -Delta (1 + a (1 - t))
 //   std  = sigma sqrt(Delta)
-//   SAMPLE: x_next = mean + std eps;  EVAL: x_next given
+//   SAMPLE: x_next = mean + std eps;  EVAL: x_next given; SAMPLE with eps
+//   drawn in the kernel from the counter-based generator of rng.cuh
 //   logp = -sum (x_next - mean)^2 / (2 std^2) - D ln std - D/2 ln 2 pi
 // The per-sample coefficients are formed in fp64 once per thread; the
 // elementwise work is fp32 FMAs over 128-bit streaming loads.  Pass 1 writes
@@ -14,11 +15,13 @@
 // does not depend on scheduling.
 #include "internal.h"
 #include "ptx.cuh"
+#include "rng.cuh"
 
 namespace ff {
 namespace {
 
 constexpr int kThreads = 256;
+constexpr int kModePhilox = 2;                                // SAMPLE, eps from rng.cuh (internal mode)
 constexpr int kVecPerThread = 4;                              // float4 per thread per chunk
 constexpr int kChunk = kThreads * kVecPerThread * 4;          // 4096 elements
 
@@ -60,7 +63,8 @@ template <int MODE>
 __global__ void __launch_bounds__(kThreads) sde_step_partial_kernel(int64_t D, int nblk, const float* x,
                                                                     const float* v, const float* eps, float* x_next,
                                                                     const float* t, const float* t_next,
-                                                                    const float* sigma, double* partial) {
+                                                                    const float* sigma, double* partial,
+                                                                    PhiloxKey key, uint32_t rng_stream) {
     __shared__ double red[kThreads / 32];
     __shared__ StepCoef coef;
     const int b = blockIdx.y;
@@ -83,7 +87,9 @@ __global__ void __launch_bounds__(kThreads) sde_step_partial_kernel(int64_t D, i
             if (i < nvec) {
                 xv[j] = __ldcs(x4 + i);
                 vv[j] = __ldcs(v4 + i);
-                ev[j] = MODE == FF_SDE_SAMPLE ? __ldcs(e4 + i) : __ldcs(reinterpret_cast<const float4*>(n4) + i);
+                if (MODE == FF_SDE_SAMPLE) ev[j] = __ldcs(e4 + i);
+                else if (MODE == kModePhilox) ev[j] = philox_normal4(static_cast<uint32_t>(i), b, rng_stream, key);
+                else ev[j] = __ldcs(reinterpret_cast<const float4*>(n4) + i);
             }
         }
 #pragma unroll
@@ -93,7 +99,7 @@ __global__ void __launch_bounds__(kThreads) sde_step_partial_kernel(int64_t D, i
                 float m[4] = {fmaf(c.cx, xv[j].x, c.cv * vv[j].x), fmaf(c.cx, xv[j].y, c.cv * vv[j].y),
                               fmaf(c.cx, xv[j].z, c.cv * vv[j].z), fmaf(c.cx, xv[j].w, c.cv * vv[j].w)};
                 float o[4];
-                if (MODE == FF_SDE_SAMPLE) {
+                if (MODE != FF_SDE_EVAL) {
                     o[0] = fmaf(c.std, ev[j].x, m[0]);
                     o[1] = fmaf(c.std, ev[j].y, m[1]);
                     o[2] = fmaf(c.std, ev[j].z, m[2]);
@@ -112,6 +118,17 @@ __global__ void __launch_bounds__(kThreads) sde_step_partial_kernel(int64_t D, i
     }
     const double s = block_sum(static_cast<double>(ss), red);
     if (threadIdx.x == 0) partial[static_cast<int64_t>(b) * nblk + blockIdx.x] = s;
+}
+
+// out[b, 4g .. 4g + 3] = the normals of element group g of sample b (rng.cuh).
+__global__ void __launch_bounds__(kThreads) philox_normal_kernel(int B, int64_t nvec, PhiloxKey key,
+                                                                 uint32_t rng_stream, float4* out) {
+    const int64_t total = static_cast<int64_t>(B) * nvec;
+    for (int64_t k = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; k < total;
+         k += static_cast<int64_t>(gridDim.x) * kThreads) {
+        const int64_t b = k / nvec, g = k - b * nvec;
+        __stcs(out + k, philox_normal4(static_cast<uint32_t>(g), static_cast<uint32_t>(b), rng_stream, key));
+    }
 }
 
 __global__ void __launch_bounds__(kThreads) sde_logprob_finalize_kernel(int64_t D, int nchunk, const double* partial,
@@ -202,13 +219,18 @@ int ff_sde_workspace_size(int B, int64_t D, size_t* bytes) {
     return FF_OK;
 }
 
-int ff_sde_step_logprob(int B, int64_t D, const float* x_t, const float* v, const float* eps, float* x_next,
-                        const float* t, const float* t_next, const float* sigma, int mode, int reduce, float* logp,
-                        int ld, void* ws, size_t ws_bytes, cudaStream_t stream) {
-    using namespace ff;
+}  // extern "C"
+
+namespace ff {
+namespace {
+
+// Argument checks and the two launches of one SDE step (mode FF_SDE_SAMPLE,
+// FF_SDE_EVAL or kModePhilox).
+int sde_step(int B, int64_t D, const float* x_t, const float* v, const float* eps, float* x_next, const float* t,
+             const float* t_next, const float* sigma, int mode, int reduce, float* logp, int ld, void* ws,
+             size_t ws_bytes, PhiloxKey key, uint32_t rng_stream, cudaStream_t stream) {
     if (B <= 0 || D <= 0) return set_error(FF_ERR_INVALID_ARG, "sde: B=%d D=%lld must be positive", B, (long long)D);
     if (D % 4) return set_error(FF_ERR_UNSUPPORTED, "sde: D=%lld not a multiple of 4", (long long)D);
-    if (mode != FF_SDE_SAMPLE && mode != FF_SDE_EVAL) return set_error(FF_ERR_INVALID_ARG, "sde: bad mode %d", mode);
     if (reduce != FF_LP_SUM && reduce != FF_LP_MEAN) return set_error(FF_ERR_INVALID_ARG, "sde: bad reduce %d", reduce);
     if (!x_t || !v || !x_next || !t || !t_next || !sigma || !logp || (mode == FF_SDE_SAMPLE && !eps))
         return set_error(FF_ERR_INVALID_ARG, "sde: null pointer");
@@ -216,6 +238,8 @@ int ff_sde_step_logprob(int B, int64_t D, const float* x_t, const float* v, cons
         return set_error(FF_ERR_INVALID_ARG, "sde: arrays must be 16-byte aligned");
     if (ld < 1) return set_error(FF_ERR_INVALID_ARG, "sde: ld=%d < 1", ld);
     if (B > 65535) return set_error(FF_ERR_UNSUPPORTED, "sde: B=%d > 65535", B);
+    if (mode == kModePhilox && D / 4 > 0xFFFFFFFFll)
+        return set_error(FF_ERR_UNSUPPORTED, "sde: D=%lld too large for the generator's counter", (long long)D);
     const int nc = nchunks(D);
     const size_t need = static_cast<size_t>(B) * nc * sizeof(double);
     if (!ws || ws_bytes < need || (reinterpret_cast<uintptr_t>(ws) & 7))
@@ -223,19 +247,60 @@ int ff_sde_step_logprob(int B, int64_t D, const float* x_t, const float* v, cons
     double* partial = static_cast<double*>(ws);
     const dim3 grid(nc, B);
     {
-    ProfScope prof(stream, "sde_step", 0.0, static_cast<double>(B) * D * (mode == FF_SDE_SAMPLE ? 16.0 : 12.0));
-    if (mode == FF_SDE_SAMPLE)
-        sde_step_partial_kernel<FF_SDE_SAMPLE><<<grid, kThreads, 0, stream>>>(D, nc, x_t, v, eps, x_next, t, t_next,
-                                                                              sigma, partial);
-    else
-        sde_step_partial_kernel<FF_SDE_EVAL><<<grid, kThreads, 0, stream>>>(D, nc, x_t, v, eps, x_next, t, t_next,
-                                                                            sigma, partial);
+        ProfScope prof(stream, "sde_step", 0.0, static_cast<double>(B) * D * (mode == FF_SDE_SAMPLE ? 16.0 : 12.0));
+        if (mode == FF_SDE_SAMPLE)
+            sde_step_partial_kernel<FF_SDE_SAMPLE><<<grid, kThreads, 0, stream>>>(D, nc, x_t, v, eps, x_next, t, t_next,
+                                                                                  sigma, partial, key, rng_stream);
+        else if (mode == kModePhilox)
+            sde_step_partial_kernel<kModePhilox><<<grid, kThreads, 0, stream>>>(D, nc, x_t, v, eps, x_next, t, t_next,
+                                                                                sigma, partial, key, rng_stream);
+        else
+            sde_step_partial_kernel<FF_SDE_EVAL><<<grid, kThreads, 0, stream>>>(D, nc, x_t, v, eps, x_next, t, t_next,
+                                                                                sigma, partial, key, rng_stream);
     }
     int rc = check_launch("sde_step_partial_kernel");
     if (rc) return rc;
     ProfScope prof(stream, "sde_finalize", 0.0, static_cast<double>(B) * nc * 8.0 + B * 16.0);
     sde_logprob_finalize_kernel<<<B, kThreads, 0, stream>>>(D, nc, partial, t, t_next, sigma, reduce, logp, ld);
     return check_launch("sde_logprob_finalize_kernel");
+}
+
+}  // namespace
+}  // namespace ff
+
+extern "C" {
+
+int ff_sde_step_logprob(int B, int64_t D, const float* x_t, const float* v, const float* eps, float* x_next,
+                        const float* t, const float* t_next, const float* sigma, int mode, int reduce, float* logp,
+                        int ld, void* ws, size_t ws_bytes, cudaStream_t stream) {
+    using namespace ff;
+    if (mode != FF_SDE_SAMPLE && mode != FF_SDE_EVAL) return set_error(FF_ERR_INVALID_ARG, "sde: bad mode %d", mode);
+    return sde_step(B, D, x_t, v, eps, x_next, t, t_next, sigma, mode, reduce, logp, ld, ws, ws_bytes, PhiloxKey{0, 0},
+                    0u, stream);
+}
+
+int ff_sde_step_logprob_philox(int B, int64_t D, const float* x_t, const float* v, float* x_next, const float* t,
+                               const float* t_next, const float* sigma, uint64_t seed, uint32_t rng_stream, int reduce,
+                               float* logp, int ld, void* ws, size_t ws_bytes, cudaStream_t stream) {
+    using namespace ff;
+    return sde_step(B, D, x_t, v, nullptr, x_next, t, t_next, sigma, kModePhilox, reduce, logp, ld, ws, ws_bytes,
+                    philox_key(seed), rng_stream, stream);
+}
+
+int ff_philox_normal(int B, int64_t D, uint64_t seed, uint32_t rng_stream, float* out, cudaStream_t stream) {
+    using namespace ff;
+    if (B <= 0 || D <= 0 || !out) return set_error(FF_ERR_INVALID_ARG, "philox: B=%d D=%lld out=%p", B, (long long)D, out);
+    if (D % 4) return set_error(FF_ERR_UNSUPPORTED, "philox: D=%lld not a multiple of 4", (long long)D);
+    if (D / 4 > 0xFFFFFFFFll) return set_error(FF_ERR_UNSUPPORTED, "philox: D=%lld too large", (long long)D);
+    if (!aligned16(out)) return set_error(FF_ERR_INVALID_ARG, "philox: out must be 16-byte aligned");
+    const int64_t nvec = D / 4, total = static_cast<int64_t>(B) * nvec;
+    int64_t blocks = (total + kThreads - 1) / kThreads;
+    const int64_t cap = 8 * static_cast<int64_t>(num_sms());
+    if (blocks > cap) blocks = cap;
+    ProfScope prof(stream, "philox_normal", 0.0, static_cast<double>(B) * D * 4.0);
+    philox_normal_kernel<<<static_cast<unsigned>(blocks), kThreads, 0, stream>>>(B, nvec, philox_key(seed), rng_stream,
+                                                                                 reinterpret_cast<float4*>(out));
+    return check_launch("philox_normal_kernel");
 }
 
 }  // extern "C"
@@ -371,10 +436,10 @@ extern "C" int ff_sde_step_logprob_noalloc(int B, int64_t D, const float* x_t, c
     const dim3 grid(nc, B);
     if (mode == FF_SDE_SAMPLE)
         sde_step_partial_kernel<FF_SDE_SAMPLE><<<grid, kThreads, 0, stream>>>(D, nc, x_t, v, eps, x_next, t, t_next,
-                                                                              sigma, partial);
+                                                                              sigma, partial, PhiloxKey{0, 0}, 0u);
     else
         sde_step_partial_kernel<FF_SDE_EVAL><<<grid, kThreads, 0, stream>>>(D, nc, x_t, v, eps, x_next, t, t_next,
-                                                                            sigma, partial);
+                                                                            sigma, partial, PhiloxKey{0, 0}, 0u);
     int rc = check_launch("sde_step_partial_kernel (no-alloc)");
     if (rc) return rc;
     sde_logprob_finalize_kernel<<<B, kThreads, 0, stream>>>(D, nc, partial, t, t_next, sigma, reduce, logp, ld);

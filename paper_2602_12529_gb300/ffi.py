@@ -61,6 +61,9 @@ _SIGS = {
     "ff_sde_schedule": ([_I, _I, _D, _D, _D, C.POINTER(_D), C.POINTER(_D)], _I),
     "ff_sde_workspace_size": ([_I, _I64, C.POINTER(_SZ)], _I),
     "ff_sde_step_logprob": ([_I, _I64, _P, _P, _P, _P, _P, _P, _P, _I, _I, _P, _I, _P, _SZ, _P], _I),
+    "ff_philox_normal": ([_I, _I64, C.c_uint64, C.c_uint32, _P, _P], _I),
+    "ff_sde_step_logprob_philox": ([_I, _I64, _P, _P, _P, _P, _P, _P, C.c_uint64, C.c_uint32, _I, _P, _I, _P, _SZ,
+                                    _P], _I),
     "ff_sde_step_logprob_noalloc": ([_I, _I64, _P, _P, _P, _P, _P, _P, _P, _I, _I, _P, _I, _P], _I),
     "ff_group_advantage": ([_I, _I, _P, _F, _P, _P], _I),
     "ff_grpo_loss_workspace_size": ([_I, _I, C.POINTER(_SZ)], _I),
@@ -238,6 +241,30 @@ def ff_sde_step_logprob(x_t, v, eps, x_next, t, t_next, sigma, logp, mode=FF_SDE
         ws = torch.empty(ff_sde_workspace_size(B, D), dtype=torch.uint8, device=x_t.device)
     _call("ff_sde_step_logprob", B, D, _ptr(x_t), _ptr(v), _ptr(eps), _ptr(x_next), _ptr(t), _ptr(t_next),
           _ptr(sigma), mode, reduce, _ptr(logp), ld, _ptr(ws), ws.numel(), _stream(stream))
+
+
+def ff_philox_normal(out, seed: int, rng_stream: int, stream=None):
+    """out [B, ...] fp32 (device) = the counter-based standard normals of
+    (seed, rng_stream), sample b = row b (include/ff.h)."""
+    import torch
+    _check(out, torch.float32, "out")
+    B = out.shape[0]
+    _call("ff_philox_normal", B, out.numel() // B, int(seed), int(rng_stream), _ptr(out), _stream(stream))
+
+
+def ff_sde_step_logprob_philox(x_t, v, x_next, t, t_next, sigma, logp, seed: int, rng_stream: int,
+                               reduce=FF_LP_SUM, ld=1, ws=None, stream=None):
+    """The SAMPLE step with eps drawn in the kernel (ff_philox_normal's values)."""
+    import torch
+    B = x_t.shape[0]
+    D = x_t.numel() // B
+    for n_, a in (("x_t", x_t), ("v", v), ("x_next", x_next), ("t", t), ("t_next", t_next), ("sigma", sigma),
+                  ("logp", logp)):
+        _check(a, torch.float32, n_)
+    if ws is None:
+        ws = torch.empty(ff_sde_workspace_size(B, D), dtype=torch.uint8, device=x_t.device)
+    _call("ff_sde_step_logprob_philox", B, D, _ptr(x_t), _ptr(v), _ptr(x_next), _ptr(t), _ptr(t_next), _ptr(sigma),
+          int(seed), int(rng_stream), reduce, _ptr(logp), ld, _ptr(ws), ws.numel(), _stream(stream))
 
 
 def ff_sde_step_logprob_noalloc(x_t, v, eps, x_next, t, t_next, sigma, logp, mode=FF_SDE_SAMPLE,

@@ -196,6 +196,12 @@ def test_training_pass_host_validation(L):
     assert L.ff_dit_train_workspace_size(h, 4, C.byref(n)) == 2
     assert L.ff_dit_train_workspace_size(h, 8, C.byref(n)) == 0
     assert L.ff_dit_destroy(h) == 0
+    # the counter-based noise and the SDE step that draws it
+    assert L.ff_philox_normal(2, 18, 1, 0, 16, None) == 2                  # D % 4
+    assert L.ff_philox_normal(2, 16, 1, 0, None, None) == 1                # null out
+    assert L.ff_philox_normal(2, 16, 1, 0, 8, None) == 1                   # misaligned
+    assert L.ff_sde_step_logprob_philox(2, 18, 16, 16, 16, 16, 16, 16, 1, 0, 0, 16, 1, 16, 1 << 20, None) == 2
+    assert L.ff_sde_step_logprob_philox(2, 16, 16, 16, 16, 16, 16, 16, 1, 0, 0, 16, 1, 16, 8, None) == 3
     # the log-prob backward
     assert L.ff_sde_logprob_backward(2, 18, 16, 16, 16, 16, 16, 16, 0, 16, 1, 16, None) == 2   # D % 4
     assert L.ff_sde_logprob_backward(2, 16, 16, 16, 16, 16, 16, 16, 5, 16, 1, 16, None) == 1   # reduce
