@@ -353,6 +353,26 @@ def hbm_sweep(ffi, dev, hbm_peak, l2_bytes=129 * 2 ** 20):
         del sets
     out["sde_step"] = rows
     rows = []
+    for n in (1 << 24, 1 << 26, 1 << 28):
+        B, D = 4, n // 4
+        per = 12 * n
+        sets = []
+        for _ in range(nsets(per)):
+            x = torch.randn(B, D, device=dev)
+            sets.append((x, torch.randn_like(x), torch.empty_like(x)))
+        t = torch.full((B,), 0.75, device=dev)
+        tn = torch.full((B,), 0.5, device=dev)
+        sg = torch.full((B,), 0.7, device=dev)
+        lp = torch.empty(B, device=dev)
+        ws = torch.empty(ffi.ff_sde_workspace_size(B, D), dtype=torch.uint8, device=dev)
+        fns = [lambda s_=s_: ffi.ff_sde_step_logprob_philox(s_[0], s_[1], s_[2], t, tn, sg, lp, 7, 0, ws=ws)
+               for s_ in sets]
+        sec = timeit(fns)
+        rows.append({"elements": n, "bytes": per, "gbs": per / sec / 1e9, "frac": per / sec / 1e9 / hbm_peak,
+                     "sets": len(sets)})
+        del sets
+    out["sde_step_device_noise"] = rows
+    rows = []
     for n in (1 << 22, 1 << 24, 1 << 26):
         Bq, T = n // 16, 16
         per = 12 * n + 4 * Bq
@@ -753,12 +773,13 @@ def run_ours(args):
 
     # old log-probs of the (synthetic) rollout policy: new + N(0, 0.01^2)
     model.ff_dit_velocity(x, txt, t, v, ws)
-    ffi.ff_sde_step_logprob(x, v, eps, x_next, t, tn, sg, logp, ws=ws_sde)
+    noise_seed = 100 + seed          # the step's noise: drawn in the SDE kernel from (seed, step 0)
+    ffi.ff_sde_step_logprob_philox(x, v, x_next, t, tn, sg, logp, noise_seed, 0, ws=ws_sde)
     torch.add(logp, jitter, out=lp_old)
 
-    def step(xi=x, txti=txt, epsi=eps, ti=t, tni=tn, sgi=sg, ri=rewards, lpo=lp_old, xo=x_next, lpn=logp, lo=loss):
+    def step(xi=x, txti=txt, ti=t, tni=tn, sgi=sg, ri=rewards, lpo=lp_old, xo=x_next, lpn=logp, lo=loss):
         model.ff_dit_velocity(xi, txti, ti, v, ws)
-        ffi.ff_sde_step_logprob(xi, v, epsi, xo, ti, tni, sgi, lpn, ws=ws_sde)
+        ffi.ff_sde_step_logprob_philox(xi, v, xo, ti, tni, sgi, lpn, noise_seed, 0, ws=ws_sde)
         ffi.ff_group_advantage(ri, G, cfg["eps_adv"], adv_all)
         ffi.ff_grpo_loss(lpn, lpo, adv, cfg["clip"], cfg["clip"], lo, grad, ws=ws_loss)
 
@@ -835,7 +856,7 @@ def run_ours(args):
     # is reported beside it.
     from paper_2602_12529_gb300.pipeline import HostFedPipeline
     pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
-    h_in = {"x": pin(h_x), "txt": pin(h_txt), "eps": pin(h_eps), "t": pin(h_t), "tn": pin(h_tn), "sg": pin(h_sg),
+    h_in = {"x": pin(h_x), "txt": pin(h_txt), "t": pin(h_t), "tn": pin(h_tn), "sg": pin(h_sg),
             "r": pin(h_r), "lpo": lp_old.cpu().pin_memory()}
     h_out = [{"x_next": torch.empty(x.shape, dtype=torch.float32).pin_memory(),
               "logp": torch.empty((B, 1), dtype=torch.float32).pin_memory(),
@@ -844,10 +865,10 @@ def run_ours(args):
     d2h = sum(a.numel() * a.element_size() for a in h_out[0].values())
 
     def e2e_body(i, o):
-        step(i["x"], i["txt"].view(torch.bfloat16), i["eps"], i["t"], i["tn"], i["sg"], i["r"], i["lpo"],
+        step(i["x"], i["txt"].view(torch.bfloat16), i["t"], i["tn"], i["sg"], i["r"], i["lpo"],
              o["x_next"], o["logp"], o["loss"])
 
-    like_in = {"x": x, "txt": txt.view(torch.int16), "eps": eps, "t": t, "tn": tn, "sg": sg, "r": rewards,
+    like_in = {"x": x, "txt": txt.view(torch.int16), "t": t, "tn": tn, "sg": sg, "r": rewards,
                "lpo": lp_old}
     pipe = HostFedPipeline(dev, like_in, {"x_next": x_next, "logp": logp, "loss": loss}, e2e_body)
     K = args.steps
@@ -873,8 +894,11 @@ def run_ours(args):
         # 100 back-to-back launches captured in one CUDA graph, per-launch time
         sde_bytes = 16.0 * x.numel()
         at_cfg = at_config_small_kernels(ffi, dev, hbm, {
-            "sde_step (SAMPLE, log-prob)": (lambda: ffi.ff_sde_step_logprob(x, v, eps, x_next, t, tn, sg, logp,
-                                                                             ws=ws_sde), sde_bytes),
+            "sde_step (SAMPLE, eps drawn in the kernel, log-prob)": (
+                lambda: ffi.ff_sde_step_logprob_philox(x, v, x_next, t, tn, sg, logp, noise_seed, 0, ws=ws_sde),
+                12.0 * x.numel()),
+            "sde_step (SAMPLE, eps read from memory, log-prob)": (
+                lambda: ffi.ff_sde_step_logprob(x, v, eps, x_next, t, tn, sg, logp, ws=ws_sde), sde_bytes),
             "group_advantage": (lambda: ffi.ff_group_advantage(rewards, G, cfg["eps_adv"], adv_all),
                                 8.0 * rewards.numel()),
             "grpo_loss (+ dL/dlp)": (lambda: ffi.ff_grpo_loss(logp, lp_old, adv, cfg["clip"], cfg["clip"], loss, grad,

@@ -527,6 +527,13 @@ int ff_rollout_workspace_size(const ff_dit* model, int B, int S, size_t* bytes);
 int ff_rollout(const ff_dit* model, int B, int S, float* x, const void* txt, const float* t,
                const float* sigma, const float* eps, float* traj, float* logp, int reduce,
                void* ws, size_t ws_bytes, cudaStream_t stream);
+/* ff_rollout with the noise drawn on the device: step k uses
+ * ff_philox_normal's noise of (seed, rng_stream = k), inside the SDE kernel
+ * (no eps buffer; the trajectory is reproducible from the seed alone).
+ * Equal to ff_rollout given eps[k] = ff_philox_normal(B, D, seed, k). */
+int ff_rollout_philox(const ff_dit* model, int B, int S, float* x, const void* txt, const float* t,
+                      const float* sigma, uint64_t seed, float* traj, float* logp, int reduce,
+                      void* ws, size_t ws_bytes, cudaStream_t stream);
 
 #ifdef __cplusplus
 }

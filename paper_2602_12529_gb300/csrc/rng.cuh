@@ -48,14 +48,19 @@ __device__ __forceinline__ float philox_uniform(uint32_t w) {
 }
 
 // The four standard normals of element group g of sample b in stream s.
+// The angle is taken as 2 pi (u - 1/2) in (-pi, pi), where the hardware sine
+// and cosine are accurate to a few 1e-7 absolute (cos 2 pi u = -cos 2 pi
+// (u - 1/2), likewise sin); the logarithm stays the accurate one (ln u near
+// u = 1 needs relative accuracy).
 __device__ __forceinline__ float4 philox_normal4(uint32_t g, uint32_t b, uint32_t s, PhiloxKey k) {
+    constexpr float kTwoPi = 6.28318530717958647692f;
     const uint4 w = philox4x32_10(make_uint4(g, b, s, 0u), k);
     const float r0 = sqrtf(-2.f * logf(philox_uniform(w.x)));
     const float r1 = sqrtf(-2.f * logf(philox_uniform(w.z)));
     float s0, c0, s1, c1;
-    sincospif(2.f * philox_uniform(w.y), &s0, &c0);
-    sincospif(2.f * philox_uniform(w.w), &s1, &c1);
-    return make_float4(r0 * c0, r0 * s0, r1 * c1, r1 * s1);
+    __sincosf(kTwoPi * (philox_uniform(w.y) - 0.5f), &s0, &c0);
+    __sincosf(kTwoPi * (philox_uniform(w.w) - 0.5f), &s1, &c1);
+    return make_float4(-r0 * c0, -r0 * s0, -r1 * c1, -r1 * s1);
 }
 
 }  // namespace ff

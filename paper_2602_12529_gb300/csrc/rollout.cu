@@ -59,14 +59,21 @@ int ff_rollout_workspace_size(const ff_dit* model, int B, int S, size_t* bytes) 
     return FF_OK;
 }
 
-int ff_rollout(const ff_dit* model, int B, int S, float* x, const void* txt, const float* t, const float* sigma,
-               const float* eps, float* traj, float* logp, int reduce, void* ws, size_t ws_bytes,
-               cudaStream_t stream) {
-    using namespace ff;
+}  // extern "C"
+
+namespace ff {
+namespace {
+
+// The rollout loop; step k's noise is eps[k] (eps set) or the counter-based
+// noise of (seed, stream k) drawn inside the SDE kernel.
+int rollout(const ff_dit* model, int B, int S, float* x, const void* txt, const float* t, const float* sigma,
+            const float* eps, uint64_t seed, float* traj, float* logp, int reduce, void* ws, size_t ws_bytes,
+            cudaStream_t stream) {
     if (!model) return set_error(FF_ERR_INVALID_ARG, "rollout: model is null");
     if (B <= 0 || S <= 0) return set_error(FF_ERR_INVALID_ARG, "rollout: B=%d S=%d must be positive", B, S);
-    if (!x || !txt || !t || !sigma || !eps || !logp || !ws) return set_error(FF_ERR_INVALID_ARG, "rollout: null pointer");
-    if (!aligned16(x) || !aligned16(eps) || (traj && !aligned16(traj)) || (reinterpret_cast<uintptr_t>(ws) % kAlign))
+    if (!x || !txt || !t || !sigma || !logp || !ws) return set_error(FF_ERR_INVALID_ARG, "rollout: null pointer");
+    if (!aligned16(x) || (eps && !aligned16(eps)) || (traj && !aligned16(traj)) ||
+        (reinterpret_cast<uintptr_t>(ws) % kAlign))
         return set_error(FF_ERR_INVALID_ARG, "rollout: misaligned pointer (arrays 16 B, workspace 256 B)");
     if (reduce != FF_LP_SUM && reduce != FF_LP_MEAN) return set_error(FF_ERR_INVALID_ARG, "rollout: bad reduce %d", reduce);
     const int64_t D = latent_elems(model);
@@ -89,14 +96,37 @@ int ff_rollout(const ff_dit* model, int B, int S, float* x, const void* txt, con
         float* xk = traj ? traj + static_cast<int64_t>(k) * B * D : x;
         float* xn = traj ? traj + static_cast<int64_t>(k + 1) * B * D : x;
         FF_TRY(ff_dit_velocity(model, B, xk, txt, tb + k * B, v, base + p.vel, p.v - p.vel, stream));
-        FF_TRY(ff_sde_step_logprob(B, D, xk, v, eps + static_cast<int64_t>(k) * B * D, xn, tb + k * B,
-                                   tb + (k + 1) * B, sb + k * B, FF_SDE_SAMPLE, reduce, logp + k, S, base + p.sde,
-                                   p.total - p.sde, stream));
+        if (eps)
+            FF_TRY(ff_sde_step_logprob(B, D, xk, v, eps + static_cast<int64_t>(k) * B * D, xn, tb + k * B,
+                                       tb + (k + 1) * B, sb + k * B, FF_SDE_SAMPLE, reduce, logp + k, S, base + p.sde,
+                                       p.total - p.sde, stream));
+        else
+            FF_TRY(ff_sde_step_logprob_philox(B, D, xk, v, xn, tb + k * B, tb + (k + 1) * B, sb + k * B, seed,
+                                              static_cast<uint32_t>(k), reduce, logp + k, S, base + p.sde,
+                                              p.total - p.sde, stream));
     }
     if (traj && cudaMemcpyAsync(x, traj + static_cast<int64_t>(S) * B * D, xbytes, cudaMemcpyDeviceToDevice,
                                 stream) != cudaSuccess)
         return set_error(FF_ERR_CUDA, "rollout: final copy failed");
     return FF_OK;
+}
+
+}  // namespace
+}  // namespace ff
+
+extern "C" {
+
+int ff_rollout(const ff_dit* model, int B, int S, float* x, const void* txt, const float* t, const float* sigma,
+               const float* eps, float* traj, float* logp, int reduce, void* ws, size_t ws_bytes,
+               cudaStream_t stream) {
+    if (!eps) return ff::set_error(FF_ERR_INVALID_ARG, "rollout: null eps (ff_rollout_philox draws it)");
+    return ff::rollout(model, B, S, x, txt, t, sigma, eps, 0, traj, logp, reduce, ws, ws_bytes, stream);
+}
+
+int ff_rollout_philox(const ff_dit* model, int B, int S, float* x, const void* txt, const float* t,
+                      const float* sigma, uint64_t seed, float* traj, float* logp, int reduce, void* ws,
+                      size_t ws_bytes, cudaStream_t stream) {
+    return ff::rollout(model, B, S, x, txt, t, sigma, nullptr, seed, traj, logp, reduce, ws, ws_bytes, stream);
 }
 
 }  // extern "C"

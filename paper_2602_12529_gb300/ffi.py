@@ -97,6 +97,7 @@ _SIGS = {
     "ff_cross_attention_backward": ([_I, _I, _I, _I, _P, _I64, _P, _P, _I64, _P, _I64, _I, _P, _I64, _P, _I64, _P,
                                      _P, _SZ, _P], _I),
     "ff_rollout": ([_P, _I, _I, _P, _P, _P, _P, _P, _P, _P, _I, _P, _SZ, _P], _I),
+    "ff_rollout_philox": ([_P, _I, _I, _P, _P, _P, _P, C.c_uint64, _P, _P, _I, _P, _SZ, _P], _I),
     "ff_debug_gemm": ([_I, _I, _I, _P, _I64, _P, _I64, _P, _I, _I, _P, _I64, _P], _I),
     "ff_debug_gemm_gated": ([_I, _I, _I, _P, _I64, _P, _I64, _P, _P, _I64, _P, _I64, _I, _P], _I),
     "ff_debug_attention": ([_I, _I, _I, _I, _P, _I64, _P, _I64, _I, _P, _I64, _P, _I64, _P], _I),
@@ -473,6 +474,19 @@ class Dit:
         if ws is None:
             ws = torch.empty(self.rollout_workspace_size(B, S), dtype=torch.uint8, device=x.device)
         _call("ff_rollout", self._h, B, S, _ptr(x), _ptr(txt), _ptr(t), _ptr(sigma), _ptr(eps), _ptr(traj),
+              _ptr(logp), reduce, _ptr(ws), ws.numel(), _stream(stream))
+
+    def ff_rollout_philox(self, x, txt, t, sigma, seed: int, logp, traj=None, reduce: int = FF_LP_SUM, ws=None,
+                          stream=None):
+        """ff_rollout with step k's noise drawn on the device from (seed, k)."""
+        import torch
+        for n_, a in (("x", x), ("t", t), ("sigma", sigma), ("logp", logp)):
+            _check(a, torch.float32, n_)
+        _check(txt, torch.bfloat16, "txt")
+        B, S = x.shape[0], sigma.numel()
+        if ws is None:
+            ws = torch.empty(self.rollout_workspace_size(B, S), dtype=torch.uint8, device=x.device)
+        _call("ff_rollout_philox", self._h, B, S, _ptr(x), _ptr(txt), _ptr(t), _ptr(sigma), int(seed), _ptr(traj),
               _ptr(logp), reduce, _ptr(ws), ws.numel(), _stream(stream))
 
 

@@ -53,3 +53,35 @@ def test_sde_step_with_in_kernel_noise_equals_the_step_fed_that_noise(cuda, redu
     got = h(xn_b)
     for b in range(B):
         assert np.sqrt(np.mean((got[b] - xn_ref[b]) ** 2)) <= 1e-5 * np.sqrt(np.mean(xn_ref[b] ** 2))
+
+
+def test_rollout_with_device_noise_equals_the_rollout_fed_that_noise(cuda):
+    import torch
+    import synth
+    from paper_2602_12529_gb300 import ffi, weights
+    cfg = synth.config("tiny_mmdit")
+    B, S = cfg["batch"], 4
+    model = ffi.Dit(cfg, weights.pack(cfg, lambda n, s: synth.weight(n, s, synth.weight_kind(n), 0), cuda))
+    x0 = torch.from_numpy(synth.initial_latent(cfg)).to(cuda)
+    txt = torch.from_numpy(synth.text_embeds(cfg).view(np.int16)).to(cuda).view(torch.bfloat16)
+    tg, sg = ffi.ff_sde_schedule(ffi.FF_SCHED_FLOW_SDE, S, 1.0, 0.7, 0.96)
+    t = torch.tensor(tg, dtype=torch.float32, device=cuda)
+    sigma = torch.tensor(sg, dtype=torch.float32, device=cuda)
+    seed = 5150
+    eps = torch.empty((S,) + tuple(x0.shape), dtype=torch.float32, device=cuda)
+    for k in range(S):
+        ffi.ff_philox_normal(eps[k], seed, k)
+    xa, xb = x0.clone(), x0.clone()
+    la, lb = torch.empty((B, S), device=cuda), torch.empty((B, S), device=cuda)
+    ta = torch.empty((S + 1,) + tuple(x0.shape), device=cuda)
+    tb = torch.empty_like(ta)
+    model.ff_rollout(xa, txt, t, sigma, eps, la, traj=ta)
+    model.ff_rollout_philox(xb, txt, t, sigma, seed, lb, traj=tb)
+    torch.cuda.synchronize()
+    assert ffi.ff_check_device_status() == 0
+    assert torch.equal(ta, tb) and torch.equal(la, lb) and torch.equal(xa, xb)
+    # another seed gives another trajectory
+    xc = x0.clone()
+    model.ff_rollout_philox(xc, txt, t, sigma, seed + 1, lb)
+    torch.cuda.synchronize()
+    assert not torch.equal(xc, xa)
