@@ -11,7 +11,8 @@ pytestmark = pytest.mark.gpu
 
 
 @pytest.mark.parametrize("B,D,seed,stream", [(3, 4096 + 64, 0, 0), (2, 1 << 16, 12345, 7),
-                                             (1, 8, (1 << 40) + 3, 4000000000), (5, 262144, 2024, 1)])
+                                             (1, 8, (1 << 40) + 3, 4000000000), (5, 262144, 2024, 1),
+                                             (32, 65536, 3, 9), (1, 2096640, 77, 1)])
 def test_philox_normal_matches_oracle(cuda, B, D, seed, stream):
     import torch
     from paper_2602_12529_gb300 import ffi

@@ -46,7 +46,7 @@ def _check_sample(ffi, dev, x, v, e, t, tn, sg, reduce=0, inplace=False, ld=1):
     return got_x, got_lp
 
 
-@pytest.mark.parametrize("B,D", [(4, 4096), (3, 12340), (1, 4), (4, 262144)])
+@pytest.mark.parametrize("B,D", [(4, 4096), (3, 12340), (1, 4), (4, 262144), (32, 65536), (1, 2096640)])
 def test_sde_sample_parity(cuda, B, D):
     from paper_2602_12529_gb300 import ffi
     grid = osde.time_grid(10, 3.0)
