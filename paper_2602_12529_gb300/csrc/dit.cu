@@ -29,6 +29,7 @@ struct ff_dit {
     const __nv_bfloat16* w;
     std::unordered_map<std::string, int64_t> off;
     int64_t mod_width;
+    int train_recompute = 0;   // training pass: keep block inputs only, re-run each block before its backward
 };
 
 namespace ff {
@@ -205,9 +206,14 @@ void set_qk_norm(GemmEpilogue& e, const ff_dit_config& c, int qk_cols, const __n
 // WAN-style velocity: latent tokens only in the residual stream; the text is
 // embedded once per call and feeds every block's cross-attention keys and
 // values.  Buffers come from f as for mmdit_forward (one shared set for the
-// inference call, one set per block with the raw copies for training).
-int wan_forward(const ff_dit* m, int B, const float* x_t, const void* txt, const float* t, float* v_out,
-                const FwdBufs& f, cudaStream_t stream) {
+// inference call, one set per block with the raw copies for training).  In
+// three parts, so a training pass can re-run one block alone:
+//   wan_forward_prologue  rotation table, timestep embedding, modulation,
+//                         patch and text embeddings (into f.x0, f.txth);
+//   wan_forward_block     block l from io.xin to io.xout;
+//   wan_forward_final     the final layer from f.xfin to v.
+int wan_forward_prologue(const ff_dit* m, int B, const float* x_t, const void* txt, const float* t,
+                         const FwdBufs& f, cudaStream_t stream) {
     const ff_dit_config& c = m->cfg;
     const int H = c.hidden, F = c.mlp, P = c.patch_dim, d = c.head_dim, L = c.n_double;
     const int Nt = c.n_txt, Ni = c.grid_f * c.grid_h * c.grid_w;
@@ -262,13 +268,29 @@ int wan_forward(const ff_dit* m, int B, const float* x_t, const void* txt, const
         e.bias = W("txt_in2.b"); e.out0 = f.txth; e.ld0 = H;
         FF_TRY(gemm_bf16(f.txt1, H, W("txt_in2.w"), H, Rt, H, H, e, stream));
     }
+    return FF_OK;
+}
 
+namespace {
+LnModArgs wan_ln_args(const ff_dit* m, int B, const FwdBufs& f) {
+    const ff_dit_config& c = m->cfg;
+    const int H = c.hidden, Ni = c.grid_f * c.grid_h * c.grid_w;
     LnModArgs la{};
-    la.ldx = H; la.ldo = H; la.rows = Ri; la.H = H;
-    la.rows_txt = 0; la.n_txt = 1; la.n_img = Ni; la.mods = f.mods; la.ld_mods = Wm;
+    la.ldx = H; la.ldo = H; la.rows = B * Ni; la.H = H;
+    la.rows_txt = 0; la.n_txt = 1; la.n_img = Ni; la.mods = f.mods; la.ld_mods = m->mod_width;
+    return la;
+}
+}  // namespace
 
-    for (int l = 0; l < L; ++l) {
-        const DitBlockIo io = f.block(l);
+int wan_forward_block(const ff_dit* m, int B, int l, const DitBlockIo& io, const FwdBufs& f, cudaStream_t stream) {
+    const ff_dit_config& c = m->cfg;
+    const int H = c.hidden, F = c.mlp, d = c.head_dim;
+    const int Nt = c.n_txt, Ni = c.grid_f * c.grid_h * c.grid_w;
+    const int Rt = B * Nt, Ri = B * Ni;
+    const int64_t Wm = m->mod_width;
+    auto W = [&](const std::string& n) { return m->w + m->off.at(n); };
+    LnModArgs la = wan_ln_args(m, B, f);
+    {
         const std::string p = "blocks." + std::to_string(l) + ".";
         const int base = l * 6 * H;
         // self-attention
@@ -363,7 +385,16 @@ int wan_forward(const ff_dit* m, int B, const float* x_t, const void* txt, const
             FF_TRY(gemm_bf16(io.u, F, W(p + "mlp2.w"), F, Ri, H, F, e, stream));
         }
     }
-    // final layer
+    return FF_OK;
+}
+
+int wan_forward_final(const ff_dit* m, int B, const FwdBufs& f, float* v_out, cudaStream_t stream) {
+    const ff_dit_config& c = m->cfg;
+    const int H = c.hidden, P = c.patch_dim, L = c.n_double;
+    const int Ni = c.grid_f * c.grid_h * c.grid_w;
+    const int Ri = B * Ni;
+    auto W = [&](const std::string& n) { return m->w + m->off.at(n); };
+    LnModArgs la = wan_ln_args(m, B, f);
     la.x = f.xfin; la.out = f.hf;
     la.aff_w = la.aff_b = nullptr;
     la.shift_txt = la.shift_img = L * 6 * H;
@@ -372,6 +403,13 @@ int wan_forward(const ff_dit* m, int B, const float* x_t, const void* txt, const
     GemmEpilogue e;
     e.out_f32 = 1; e.bias = W("final.b"); e.out0 = v_out; e.ld0 = P;
     return gemm_bf16(f.hf, H, W("final.w"), H, Ri, P, H, e, stream);
+}
+
+int wan_forward(const ff_dit* m, int B, const float* x_t, const void* txt, const float* t, float* v_out,
+                const FwdBufs& f, cudaStream_t stream) {
+    FF_TRY(wan_forward_prologue(m, B, x_t, txt, t, f, stream));
+    for (int l = 0; l < m->cfg.n_double; ++l) FF_TRY(wan_forward_block(m, B, l, f.block(l), f, stream));
+    return wan_forward_final(m, B, f, v_out, stream);
 }
 
 // The MMDiT velocity: timestep MLP and every adaLN vector, embeddings, the
@@ -586,6 +624,7 @@ int64_t model_offset(const ff_dit* m, const char* name) {
     return it == m->off.end() ? -1 : it->second;
 }
 int64_t model_mod_width(const ff_dit* m) { return m->mod_width; }
+int model_train_recompute(const ff_dit* m) { return m->train_recompute; }
 
 }  // namespace ff
 
@@ -637,6 +676,15 @@ int ff_dit_create(const ff_dit_config* cfg, const void* weights_dev, ff_dit** ou
 
 int ff_dit_destroy(ff_dit* m) {
     delete m;
+    return FF_OK;
+}
+
+int ff_dit_set_train_recompute(ff_dit* m, int on) {
+    using namespace ff;
+    if (!m) return set_error(FF_ERR_INVALID_ARG, "model is null");
+    if (on && m->cfg.arch != FF_ARCH_WAN)
+        return set_error(FF_ERR_UNSUPPORTED, "training recompute: WAN-style models only");
+    m->train_recompute = on ? 1 : 0;
     return FF_OK;
 }
 

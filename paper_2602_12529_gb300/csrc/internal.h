@@ -34,6 +34,7 @@ const ff_dit_config& model_config(const ff_dit* m);
 const __nv_bfloat16* model_weights(const ff_dit* m);
 int64_t model_offset(const ff_dit* m, const char* name);
 int64_t model_mod_width(const ff_dit* m);
+int model_train_recompute(const ff_dit* m);
 
 // ---- optional launch timing (ff_prof_*): RAII scope around one launch ----
 struct ProfScope {
@@ -370,6 +371,12 @@ int mmdit_forward(const ff_dit* m, int B, const float* x_t, const void* txt, con
                   const FwdBufs& f, cudaStream_t stream);
 int wan_forward(const ff_dit* m, int B, const float* x_t, const void* txt, const float* t, float* v_out,
                 const FwdBufs& f, cudaStream_t stream);
+// Its three parts: embeddings and modulation; block l from io.xin to
+// io.xout; the final layer from f.xfin.
+int wan_forward_prologue(const ff_dit* m, int B, const float* x_t, const void* txt, const float* t,
+                         const FwdBufs& f, cudaStream_t stream);
+int wan_forward_block(const ff_dit* m, int B, int l, const DitBlockIo& io, const FwdBufs& f, cudaStream_t stream);
+int wan_forward_final(const ff_dit* m, int B, const FwdBufs& f, float* v_out, cudaStream_t stream);
 // The WAN model's training pass (wan_train.cu): workspace bytes, the forward
 // that keeps what the backward reads, and the backward (arguments as
 // ff_dit_forward_train / ff_dit_backward, already validated).

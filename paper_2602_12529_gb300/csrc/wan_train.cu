@@ -23,6 +23,10 @@
 //   oc, h2, y2 bf16 [R_i, H]; raw and normalised qkv [R_i, 3H]; k | v of the
 //   text (+ raw) [R_t, 2H]; a1, u [R_i, F]; both attentions' log-sum-exp;
 //   the final residual and LN-modulate output; then the backward's scratch.
+// In recompute mode (ff_dit_set_train_recompute) the blocks share one set of
+// those activations and only their input residuals are kept; the backward
+// re-runs block l's forward (bit-identical, every kernel is deterministic)
+// just before its backward.
 #include <string>
 #include <vector>
 
@@ -48,7 +52,7 @@ struct WanPlan {
     size_t bytes;
 };
 
-WanPlan plan(const ff_dit_config& c, int64_t Wm, int B, uint8_t* base) {
+WanPlan plan(const ff_dit_config& c, int64_t Wm, int B, uint8_t* base, bool recompute) {
     const size_t H = c.hidden, F = c.mlp, P = c.patch_dim, tf = c.time_freq_dim, d = c.head_dim;
     const size_t Nt = c.n_txt, Ni = static_cast<size_t>(c.grid_f) * c.grid_h * c.grid_w;
     const size_t Rt = B * Nt, Ri = B * Ni;
@@ -79,8 +83,18 @@ WanPlan plan(const ff_dit_config& c, int64_t Wm, int B, uint8_t* base) {
     p.blk.resize(L);
     float* x = f32(Ri * H);
     f.x0 = x;
+    // recompute: one activation set shared by every block (re-filled by the
+    // backward), only the block inputs kept
+    DitBlockIo shared{};
     for (int l = 0; l < L; ++l) {
         DitBlockIo& io = p.blk[l];
+        if (recompute && l > 0) {
+            io = shared;
+            io.xin = x;
+            x = f32(Ri * H);
+            io.xout = x;
+            continue;
+        }
         io = DitBlockIo{};
         io.xin = x;
         io.h1 = b16(Ri * H);
@@ -104,6 +118,7 @@ WanPlan plan(const ff_dit_config& c, int64_t Wm, int B, uint8_t* base) {
         io.y2 = b16(Ri * H);
         x = f32(Ri * H);
         io.xout = x;
+        shared = io;
     }
     f.xfin = x;
     f.hf = b16(Ri * H);
@@ -145,13 +160,13 @@ WanPlan plan(const ff_dit_config& c, int64_t Wm, int B, uint8_t* base) {
 }  // namespace
 
 size_t wan_train_workspace_bytes(const ff_dit* m, int B) {
-    return plan(model_config(m), model_mod_width(m), B, nullptr).bytes;
+    return plan(model_config(m), model_mod_width(m), B, nullptr, model_train_recompute(m) != 0).bytes;
 }
 
 int wan_forward_train(const ff_dit* m, int B, const float* x_t, const void* txt, const float* t, float* v_out,
                       void* ws, size_t ws_bytes, cudaStream_t stream) {
     const ff_dit_config& c = model_config(m);
-    WanPlan p = plan(c, model_mod_width(m), B, static_cast<uint8_t*>(ws));
+    WanPlan p = plan(c, model_mod_width(m), B, static_cast<uint8_t*>(ws), model_train_recompute(m) != 0);
     if (ws_bytes < p.bytes) return set_error(FF_ERR_WORKSPACE, "workspace %zu B < %zu B needed", ws_bytes, p.bytes);
     p.f.blocks = p.blk.data();
     // the time-MLP operands' padding rows (the weight-gradient products read them)
@@ -169,7 +184,8 @@ int wan_backward(const ff_dit* m, int B, const void* txt, const float* dv, float
                  size_t ws_bytes, cudaStream_t stream) {
     const ff_dit_config& c = model_config(m);
     const int64_t Wm = model_mod_width(m);
-    WanPlan p = plan(c, Wm, B, static_cast<uint8_t*>(ws));
+    const bool recompute = model_train_recompute(m) != 0;
+    WanPlan p = plan(c, Wm, B, static_cast<uint8_t*>(ws), recompute);
     if (ws_bytes < p.bytes) return set_error(FF_ERR_WORKSPACE, "workspace %zu B < %zu B needed", ws_bytes, p.bytes);
     const FwdBufs& f = p.f;
     const int H = c.hidden, F = c.mlp, P = c.patch_dim, d = c.head_dim, heads = c.heads, tf = c.time_freq_dim;
@@ -231,6 +247,8 @@ int wan_backward(const ff_dit* m, int B, const void* txt, const float* dv, float
     // ---- blocks, last first
     for (int l = L - 1; l >= 0; --l) {
         const DitBlockIo& io = p.blk[l];
+        // recompute: this block's activations again, from its kept input
+        if (recompute) FF_TRY(wan_forward_block(m, B, l, io, f, stream));
         const int base = l * 6 * H;
         const std::string pre = "blocks." + std::to_string(l) + ".";
         // FFN half: x_out = x3 + g2 (GELU(LNmod2(x3) W1^T + b1) W2^T + b2)

@@ -83,6 +83,7 @@ _SIGS = {
     "ff_dit_workspace_size": ([_P, _I, C.POINTER(_SZ)], _I),
     "ff_dit_velocity": ([_P, _I, _P, _P, _P, _P, _P, _SZ, _P], _I),
     "ff_rollout_workspace_size": ([_P, _I, _I, C.POINTER(_SZ)], _I),
+    "ff_dit_set_train_recompute": ([_P, _I], _I),
     "ff_dit_train_workspace_size": ([_P, _I, C.POINTER(_SZ)], _I),
     "ff_dit_forward_train": ([_P, _I, _P, _P, _P, _P, _P, _SZ, _P], _I),
     "ff_dit_backward": ([_P, _I, _P, _P, _P, _P, _P, _SZ, _P], _I),
@@ -457,6 +458,10 @@ class Dit:
         B = dv.shape[0]
         _call("ff_dit_backward", self._h, B, _ptr(txt), _ptr(dv), _ptr(grad), _ptr(dx_t), _ptr(ws), ws.numel(),
               _stream(stream))
+
+    def set_train_recompute(self, on: bool):
+        """Training pass keeps only block inputs and re-runs each block in the backward (WAN-style models)."""
+        _call("ff_dit_set_train_recompute", self._h, 1 if on else 0)
 
     def rollout_workspace_size(self, B: int, S: int) -> int:
         n = _SZ()

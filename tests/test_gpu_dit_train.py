@@ -158,6 +158,31 @@ def test_wan_forward_train_equals_velocity_and_backward_is_deterministic(cuda):
     assert np.array_equal(g1, g2) and np.array_equal(d1, d2)
 
 
+@pytest.mark.parametrize("L", [1, 3])
+def test_wan_recompute_gives_the_same_gradient(cuda, L):
+    """Recompute mode (block inputs kept, each block re-run before its
+    backward) gives bit for bit the stored-activation pass's v and gradients."""
+    import torch
+    from paper_2602_12529_gb300 import ffi
+    cfg = dict(WAN_TRAIN, n_double=L)
+    run = Run(cfg, cuda, seed=3)
+    dv = np.random.default_rng(10).standard_normal(tuple(run.v.shape)).astype(np.float32)
+    g1, d1 = run.backward(dv)
+    run.model.set_train_recompute(True)
+    ws = torch.empty(run.model.train_workspace_size(run.B), dtype=torch.uint8, device=cuda)
+    assert ws.numel() < run.ws.numel() or L == 1
+    v2 = torch.empty_like(run.v)
+    run.model.ff_dit_forward_train(run.xg, run.tg, run.tt, v2, ws)
+    grad = torch.zeros(run.total, dtype=torch.float32, device=cuda)
+    dx = torch.empty_like(run.xg)
+    run.model.ff_dit_backward(run.tg, torch.from_numpy(dv).to(cuda), grad, ws, dx_t=dx)
+    torch.cuda.synchronize()
+    assert ffi.ff_check_device_status() == 0
+    assert torch.equal(v2, run.v)
+    assert np.array_equal(grad.cpu().numpy(), g1) and np.array_equal(dx.cpu().numpy(), d1)
+    run.model.set_train_recompute(False)
+
+
 def test_sde_logprob_backward_parity(cuda):
     import torch
     from paper_2602_12529_gb300 import ffi
