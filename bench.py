@@ -616,31 +616,43 @@ def train_step(args, ffi, model, cfg, dev, x, txt, t, tn, sg, x_next, lp_old, ad
             "peak": f"{tc_burst} TFLOP/s ({src} bf16 dense burst)"}
 
 
-def wan_block_train(args, ffi, dev, timed):
-    """The WAN-style model's training pass on one full-width block (H 5120,
-    40 x 128 heads, MLP 13824; batch 1 of 32760 latent + 512 text tokens):
-    the training forward (activations kept) and the DiT backward from a
-    random dL/dv to every weight.  Weights N(0, 0.02), norm scales 1.
-    Algorithmic FLOPs: 3x the forward's GEMM FLOPs (forward, input and weight
-    gradients) + 3.5x its attention FLOPs (forward 4 B h N_q N_k d, backward
-    10 B h N_q N_k d), for the self-attention and the cross-attention."""
+def wan_train(args, ffi, dev, timed, blocks=1, recompute=False):
+    """The WAN-style model's training pass at full width (H 5120, 40 x 128
+    heads, MLP 13824; batch 1 of 32760 latent + 512 text tokens): the
+    training forward and the DiT backward from a random dL/dv to every
+    weight, on `blocks` blocks (the whole model is 40).  With `recompute`
+    the forward keeps only the block inputs and the backward re-runs every
+    block (one more forward of the blocks, not counted as work).  Weights
+    N(0, 0.02), norm scales 1, drawn on the device.  Algorithmic FLOPs: 3x
+    the forward's GEMM FLOPs (forward, input and weight gradients) + 3.5x
+    its attention FLOPs (forward 4 B h N_q N_k d, backward 10 B h N_q N_k
+    d), for the self-attention and the cross-attention."""
     import numpy as np
     import torch
     import synth
-    cfg = dict(synth.config("wan_40"), n_double=1, batch=1)
+    cfg = dict(synth.config("wan_40"), n_double=blocks, batch=1)
     B, H, F, P = 1, cfg["hidden"], cfg["mlp"], cfg["patch_dim"]
     Nt, Ni = cfg["n_txt"], synth_n_img(cfg)
     specs, total = ffi.ff_dit_weight_layout(cfg)
+    free, _ = torch.cuda.mem_get_info(dev)
+    if 6 * total > 0.8 * free:
+        return {"skipped": f"{total / 1e9:.1f} G parameters: weights and fp32 gradients exceed the free memory"}
     g = torch.Generator(device=dev)
     g.manual_seed(11)
-    blob = (torch.randn(total, generator=g, device=dev) * 0.02).to(torch.bfloat16)
+    blob = torch.empty(total, dtype=torch.bfloat16, device=dev)
+    for i in range(0, total, 1 << 28):          # drawn in pieces (no fp32 copy of the whole blob)
+        n = min(1 << 28, total - i)
+        blob[i:i + n] = (torch.randn(n, generator=g, device=dev) * 0.02).to(torch.bfloat16)
     for name, off, shape in specs:
         if name.endswith("scale"):
             blob[off:off + int(np.prod(shape))] = 1.0
     model = ffi.Dit(cfg, blob)
+    if recompute:
+        model.set_train_recompute(True)
     need = model.train_workspace_size(B)
     free, _ = torch.cuda.mem_get_info(dev)
     if need + 4 * total > 0.9 * free:
+        model.close()
         return {"skipped": f"training workspace {need / 1e9:.1f} GB exceeds the free device memory"}
     ws = torch.empty(need, dtype=torch.uint8, device=dev)
     grad = torch.empty(total, dtype=torch.float32, device=dev)
@@ -653,22 +665,24 @@ def wan_block_train(args, ffi, dev, timed):
         model.ff_dit_forward_train(x, txt, t, v, ws)
         model.ff_dit_backward(txt, dv, grad, ws)
 
-    for _ in range(max(2, args.warmup)):
+    warm = 1 if blocks > 1 else max(2, args.warmup)
+    for _ in range(warm):
         step()
-    k = max(2, min(args.steps, 5))
+    k = 2 if blocks > 1 else max(2, min(args.steps, 5))
     ms = timed(step, k) / k
-    gemm = 2.0 * B * Ni * (6 * H * H + 2 * H * F) + 2.0 * B * Nt * 2 * H * H + 2.0 * B * Ni * 2 * P * H \
-        + 2.0 * B * Nt * (cfg["txt_dim"] * H + H * H)
-    attn = 4.0 * B * H * Ni * (Ni + Nt)
+    per_block = 2.0 * B * Ni * (6 * H * H + 2 * H * F) + 2.0 * B * Nt * 2 * H * H
+    gemm = blocks * per_block + 2.0 * B * Ni * 2 * P * H + 2.0 * B * Nt * (cfg["txt_dim"] * H + H * H)
+    attn = blocks * 4.0 * B * H * Ni * (Ni + Nt)
     flops = 3.0 * gemm + 3.5 * attn
     _, tc_burst, tc_sust, src = load_peaks()
     model.close()
     return {"ms_per_step": ms, "value": B * Ni / (ms / 1e3), "unit": UNIT,
-            "what": "WAN-style block at full width (1 of 40 blocks of the 14B-class video DiT): training forward + "
-                    "DiT backward from dL/dv to every weight, batch 1, 32760 latent + 512 text tokens",
+            "what": f"WAN-style model at full width, {blocks} of its 40 blocks "
+                    f"({total / 1e9:.2f} G parameters): training forward + DiT backward from dL/dv to every weight, "
+                    f"batch 1, 32760 latent + 512 text tokens" + (", block activations recomputed" if recompute else ""),
             "tflops": flops / (ms / 1e3) / 1e12, "frac": flops / (ms / 1e3) / 1e12 / tc_burst,
             "frac_vs_sustained": flops / (ms / 1e3) / 1e12 / tc_sust if tc_sust else None,
-            "algorithmic_flops": flops, "workspace_gb": need / 1e9,
+            "algorithmic_flops": flops, "workspace_gb": need / 1e9, "parameters": total,
             "peak": f"{tc_burst} TFLOP/s ({src} bf16 dense burst)"}
 
 
@@ -905,7 +919,12 @@ def run_ours(args):
                                                               ws=ws_loss), 16.0 * logp.numel() + 4.0 * B),
         })
     bwd = backward_kernels(args, ffi, cfg, dev) if rank == 0 and not args.no_sweep else None
-    wan_train = wan_block_train(args, ffi, dev, timed) if rank == 0 and world == 1 and not args.no_sweep else None
+    wan_train1 = wan_full = None
+    if rank == 0 and world == 1 and not args.no_sweep:
+        wan_train1 = wan_train(args, ffi, dev, timed)
+        torch.cuda.empty_cache()
+        wan_full = wan_train(args, ffi, dev, timed, blocks=40, recompute=True)
+        torch.cuda.empty_cache()
     sweep = hbm_sweep(ffi, dev, hbm) if rank == 0 and not args.no_sweep else None
     clk = clocks.stop() if clocks else None
     status = ffi.ff_check_device_status()
@@ -939,7 +958,8 @@ def run_ours(args):
                 "awm_step": awm,
                 "train_step": train,
                 "backward_kernels": bwd,
-                "wan_block_train_step": wan_train,
+                "wan_block_train_step": wan_train1,
+                "wan_full_train_step": wan_full,
                 "gpu_launches": launches,
                 "clocks": clk,
                 "device_status": status}
