@@ -425,15 +425,14 @@ int ff_dit_velocity(const ff_dit* model, int B, const float* x_t, const void* tx
  * single-stream block, R = B (N_t + N_i), plus scratch; per WAN block
  * R_i (42 H + 4 F) + 8 R_t H bytes (R_i = B N_i, R_t = B N_t).
  * ------------------------------------------------------------------------ */
-/* Recompute mode of the training pass (WAN-style models; FF_ERR_UNSUPPORTED
- * for others): ff_dit_forward_train keeps only every block's input residual
- * (fp32 [B N_i, H] per block) and the backward re-runs block l's forward
- * into one shared activation set just before that block's backward.  One
- * more forward of the blocks; about R_i (4 H) bytes per block instead of
- * R_i (42 H + 4 F) + 8 R_t H.  The gradient is bit-identical to the
- * stored-activation pass (every kernel is deterministic).  Set it before
- * ff_dit_train_workspace_size and keep it unchanged until the matching
- * ff_dit_backward. */
+/* Recompute mode of the training pass: ff_dit_forward_train keeps only every
+ * block's input residual (fp32, 4 H bytes per residual row) and the backward
+ * re-runs block l's forward into one shared activation set (one per block
+ * kind) just before that block's backward.  One more forward of the blocks;
+ * 4 H bytes per row and block instead of the stored activations.  The
+ * gradient is bit-identical to the stored-activation pass (every kernel is
+ * deterministic).  Set it before ff_dit_train_workspace_size and keep it
+ * unchanged until the matching ff_dit_backward. */
 int ff_dit_set_train_recompute(ff_dit* model, int on);
 int ff_dit_train_workspace_size(const ff_dit* model, int B, size_t* bytes);
 int ff_dit_forward_train(const ff_dit* model, int B, const float* x_t, const void* txt,

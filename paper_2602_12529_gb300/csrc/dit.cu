@@ -416,9 +416,11 @@ int wan_forward(const ff_dit* m, int B, const float* x_t, const void* txt, const
 // double- and single-stream blocks, the final layer.  Buffers come from f:
 // the inference call passes one shared set (residual updated in place), the
 // training forward one set per block with the pre-activation copies the
-// backward reads.
-int mmdit_forward(const ff_dit* m, int B, const float* x_t, const void* txt, const float* t, float* v_out,
-                  const FwdBufs& f, cudaStream_t stream) {
+// backward reads.  In four parts, so a training pass can re-run one block:
+// prologue (rotation table, time MLP, modulation, embeddings into f.x0),
+// double-stream block l, single-stream block l (io.xin -> io.xout), final.
+int mmdit_forward_prologue(const ff_dit* m, int B, const float* x_t, const void* txt, const float* t,
+                           const FwdBufs& f, cudaStream_t stream) {
     const ff_dit_config& c = m->cfg;
     const int H = c.hidden, F = c.mlp, P = c.patch_dim;
     const int Nt = c.n_txt, Ni = c.grid_f * c.grid_h * c.grid_w;
@@ -462,16 +464,32 @@ int mmdit_forward(const ff_dit* m, int B, const float* x_t, const void* txt, con
         g[1].epi.ld0 = H;
         FF_TRY(gemm_bf16_group(g, 2, stream));
     }
+    return FF_OK;
+}
 
+namespace {
+LnModArgs mmdit_ln_args(const ff_dit* m, int B, const FwdBufs& f) {
+    const ff_dit_config& c = m->cfg;
+    const int Nt = c.n_txt, Ni = c.grid_f * c.grid_h * c.grid_w;
     LnModArgs la{};
-    la.ldx = H; la.ldo = H; la.rows = R; la.H = H;
-    la.rows_txt = Rt; la.n_txt = Nt; la.n_img = Ni; la.mods = f.mods; la.ld_mods = Wm;
+    la.ldx = c.hidden; la.ldo = c.hidden; la.rows = B * (Nt + Ni); la.H = c.hidden;
+    la.rows_txt = B * Nt; la.n_txt = Nt; la.n_img = Ni; la.mods = f.mods; la.ld_mods = m->mod_width;
+    return la;
+}
+struct Stream { const char* name; int row0, rows, tokens; int64_t mod; };
+}  // namespace
 
-    struct Stream { const char* name; int row0, rows, tokens; int64_t mod; };
-
-    // ---- double-stream blocks
-    for (int l = 0; l < c.n_double; ++l) {
-        const DitBlockIo io = f.block(l);
+int mmdit_forward_double(const ff_dit* m, int B, int l, const DitBlockIo& io, const FwdBufs& f,
+                         cudaStream_t stream) {
+    const ff_dit_config& c = m->cfg;
+    const int H = c.hidden, F = c.mlp, P = c.patch_dim;
+    const int Nt = c.n_txt, Ni = c.grid_f * c.grid_h * c.grid_w;
+    const int Rt = B * Nt, Ri = B * Ni, R = Rt + Ri;
+    const int64_t Wm = m->mod_width;
+    auto W = [&](const std::string& n) { return m->w + m->off.at(n); };
+    auto rows = [](auto* p, int64_t r, int64_t ld) { return p ? p + r * ld : p; };
+    LnModArgs la = mmdit_ln_args(m, B, f);
+    {
         const int64_t base = static_cast<int64_t>(l) * 12 * H;
         const Stream st[2] = {{"txt", 0, Rt, Nt, base + 6 * H}, {"img", Rt, Ri, Ni, base}};
         const std::string pre = "double." + std::to_string(l) + ".";
@@ -556,10 +574,20 @@ int mmdit_forward(const ff_dit* m, int B, const float* x_t, const void* txt, con
             FF_TRY(gemm_bf16_group(g, 2, stream));
         }
     }
+    return FF_OK;
+}
 
-    // ---- single-stream blocks on the joint sequence
-    for (int l = 0; l < c.n_single; ++l) {
-        const DitBlockIo io = f.block(c.n_double + l);
+int mmdit_forward_single(const ff_dit* m, int B, int l, const DitBlockIo& io, const FwdBufs& f,
+                         cudaStream_t stream) {
+    const ff_dit_config& c = m->cfg;
+    const int H = c.hidden, F = c.mlp, P = c.patch_dim;
+    const int Nt = c.n_txt, Ni = c.grid_f * c.grid_h * c.grid_w;
+    const int Rt = B * Nt, Ri = B * Ni, R = Rt + Ri;
+    const int64_t Wm = m->mod_width;
+    auto W = [&](const std::string& n) { return m->w + m->off.at(n); };
+    auto rows = [](auto* p, int64_t r, int64_t ld) { return p ? p + r * ld : p; };
+    LnModArgs la = mmdit_ln_args(m, B, f);
+    {
         const int64_t off = static_cast<int64_t>(c.n_double) * 12 * H + static_cast<int64_t>(l) * 3 * H;
         const std::string p = "single." + std::to_string(l) + ".";
         la.x = io.xin; la.out = io.h1;
@@ -601,7 +629,18 @@ int mmdit_forward(const ff_dit* m, int B, const float* x_t, const void* txt, con
             FF_TRY(gemm_bf16_group(g, 2, stream));
         }
     }
+    return FF_OK;
+}
 
+int mmdit_forward_final(const ff_dit* m, int B, const FwdBufs& f, float* v_out, cudaStream_t stream) {
+    const ff_dit_config& c = m->cfg;
+    const int H = c.hidden, F = c.mlp, P = c.patch_dim;
+    const int Nt = c.n_txt, Ni = c.grid_f * c.grid_h * c.grid_w;
+    const int Rt = B * Nt, Ri = B * Ni, R = Rt + Ri;
+    const int64_t Wm = m->mod_width;
+    auto W = [&](const std::string& n) { return m->w + m->off.at(n); };
+    auto rows = [](auto* p, int64_t r, int64_t ld) { return p ? p + r * ld : p; };
+    LnModArgs la = mmdit_ln_args(m, B, f);
     // ---- final layer on image tokens -> v (fp32)
     {
         const int64_t off = static_cast<int64_t>(c.n_double) * 12 * H + static_cast<int64_t>(c.n_single) * 3 * H;
@@ -615,6 +654,15 @@ int mmdit_forward(const ff_dit* m, int B, const float* x_t, const void* txt, con
         FF_TRY(gemm_bf16(f.hf, H, W("final.w"), H, Ri, P, H, e, stream));
     }
     return FF_OK;
+}
+
+int mmdit_forward(const ff_dit* m, int B, const float* x_t, const void* txt, const float* t, float* v_out,
+                  const FwdBufs& f, cudaStream_t stream) {
+    FF_TRY(mmdit_forward_prologue(m, B, x_t, txt, t, f, stream));
+    for (int l = 0; l < m->cfg.n_double; ++l) FF_TRY(mmdit_forward_double(m, B, l, f.block(l), f, stream));
+    for (int l = 0; l < m->cfg.n_single; ++l)
+        FF_TRY(mmdit_forward_single(m, B, l, f.block(m->cfg.n_double + l), f, stream));
+    return mmdit_forward_final(m, B, f, v_out, stream);
 }
 
 const ff_dit_config& model_config(const ff_dit* m) { return m->cfg; }
@@ -682,8 +730,6 @@ int ff_dit_destroy(ff_dit* m) {
 int ff_dit_set_train_recompute(ff_dit* m, int on) {
     using namespace ff;
     if (!m) return set_error(FF_ERR_INVALID_ARG, "model is null");
-    if (on && m->cfg.arch != FF_ARCH_WAN)
-        return set_error(FF_ERR_UNSUPPORTED, "training recompute: WAN-style models only");
     m->train_recompute = on ? 1 : 0;
     return FF_OK;
 }

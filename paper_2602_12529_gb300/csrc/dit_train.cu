@@ -26,6 +26,10 @@
 //   per single-stream block: x_in fp32; h, y2 bf16 [R, H]; raw linear1 bf16
 //   [R, 3H + F]; qkv bf16 [R, 3H]; u = [o | GELU(mlp)] bf16 [R, H + F]; lse;
 //   the final residual and LN-modulate output; then the backward's scratch.
+// In recompute mode (ff_dit_set_train_recompute) the blocks of each kind
+// share one set of those activations and only the block inputs are kept;
+// the backward re-runs each block's forward (bit-identical: every kernel is
+// deterministic) just before its backward.
 #include <string>
 #include <vector>
 
@@ -51,7 +55,7 @@ struct TrainPlan {
     size_t bytes;
 };
 
-TrainPlan plan(const ff_dit_config& c, int64_t Wm, int B, uint8_t* base) {
+TrainPlan plan(const ff_dit_config& c, int64_t Wm, int B, uint8_t* base, bool recompute) {
     const size_t H = c.hidden, F = c.mlp, P = c.patch_dim, tf = c.time_freq_dim, d = c.head_dim;
     const size_t Nt = c.n_txt, Ni = static_cast<size_t>(c.grid_f) * c.grid_h * c.grid_w;
     const size_t Rt = B * Nt, Ri = B * Ni, R = Rt + Ri;
@@ -77,9 +81,21 @@ TrainPlan plan(const ff_dit_config& c, int64_t Wm, int B, uint8_t* base) {
     p.blk.resize(L);
     float* x = f32(R * H);
     f.x0 = x;
+    // recompute: one activation set per block kind, shared by the blocks of
+    // that kind (re-filled by the backward); only the block inputs kept
+    DitBlockIo shared_dbl{}, shared_sgl{};
+    bool have_dbl = false, have_sgl = false;
     for (int l = 0; l < L; ++l) {
         DitBlockIo& io = p.blk[l];
         const bool dbl = l < c.n_double;
+        if (recompute && (dbl ? have_dbl : have_sgl)) {
+            io = dbl ? shared_dbl : shared_sgl;
+            io.xin = x;
+            if (!dbl) io.xmid = x;
+            x = f32(R * H);
+            io.xout = x;
+            continue;
+        }
         io = DitBlockIo{};
         io.xin = x;
         io.h1 = b16(R * H);
@@ -100,6 +116,8 @@ TrainPlan plan(const ff_dit_config& c, int64_t Wm, int B, uint8_t* base) {
         io.y2 = b16(R * H);
         x = f32(R * H);
         io.xout = x;
+        if (dbl) { shared_dbl = io; have_dbl = true; }
+        else { shared_sgl = io; have_sgl = true; }
     }
     f.xfin = x;
     f.hf = b16(Ri * H);
@@ -161,8 +179,9 @@ int ff_dit_train_workspace_size(const ff_dit* m, int B, size_t* bytes) {
     using namespace ff;
     FF_TRY(check_model(m, B));
     if (!bytes) return set_error(FF_ERR_INVALID_ARG, "bytes is null");
-    *bytes = model_config(m).arch == FF_ARCH_WAN ? wan_train_workspace_bytes(m, B)
-                                                 : plan(model_config(m), model_mod_width(m), B, nullptr).bytes;
+    *bytes = model_config(m).arch == FF_ARCH_WAN
+                 ? wan_train_workspace_bytes(m, B)
+                 : plan(model_config(m), model_mod_width(m), B, nullptr, model_train_recompute(m) != 0).bytes;
     return FF_OK;
 }
 
@@ -175,7 +194,7 @@ int ff_dit_forward_train(const ff_dit* m, int B, const float* x_t, const void* t
         return set_error(FF_ERR_INVALID_ARG, "misaligned pointer (arrays 16 B, workspace 256 B)");
     const ff_dit_config& c = model_config(m);
     if (c.arch == FF_ARCH_WAN) return wan_forward_train(m, B, x_t, txt, t, v_out, ws, ws_bytes, stream);
-    TrainPlan p = plan(c, model_mod_width(m), B, static_cast<uint8_t*>(ws));
+    TrainPlan p = plan(c, model_mod_width(m), B, static_cast<uint8_t*>(ws), model_train_recompute(m) != 0);
     if (ws_bytes < p.bytes) return set_error(FF_ERR_WORKSPACE, "workspace %zu B < %zu B needed", ws_bytes, p.bytes);
     p.f.blocks = p.blk.data();
     // the time-MLP operands' padding rows (the weight-gradient products read them)
@@ -200,7 +219,8 @@ int ff_dit_backward(const ff_dit* m, int B, const void* txt, const float* dv, fl
     const ff_dit_config& c = model_config(m);
     if (c.arch == FF_ARCH_WAN) return wan_backward(m, B, txt, dv, grad, dx_t, ws, ws_bytes, stream);
     const int64_t Wm = model_mod_width(m);
-    TrainPlan p = plan(c, Wm, B, static_cast<uint8_t*>(ws));
+    const bool recompute = model_train_recompute(m) != 0;
+    TrainPlan p = plan(c, Wm, B, static_cast<uint8_t*>(ws), recompute);
     if (ws_bytes < p.bytes) return set_error(FF_ERR_WORKSPACE, "workspace %zu B < %zu B needed", ws_bytes, p.bytes);
     const FwdBufs& f = p.f;
     const int H = c.hidden, F = c.mlp, P = c.patch_dim, d = c.head_dim, heads = c.heads, tf = c.time_freq_dim;
@@ -250,6 +270,7 @@ int ff_dit_backward(const ff_dit* m, int B, const void* txt, const float* dv, fl
     // ---- single-stream blocks, last first
     for (int l = c.n_single - 1; l >= 0; --l) {
         const DitBlockIo& io = p.blk[c.n_double + l];
+        if (recompute) FF_TRY(mmdit_forward_single(m, B, l, io, f, stream));
         const int off = static_cast<int>(static_cast<int64_t>(c.n_double) * 12 * H + static_cast<int64_t>(l) * 3 * H);
         const std::string pre = "single." + std::to_string(l) + ".";
         const int W1 = 3 * H + F;
@@ -323,6 +344,7 @@ int ff_dit_backward(const ff_dit* m, int B, const void* txt, const float* dv, fl
     struct Stream { const char* name; int row0, rows, tokens, mod, first, cps; };
     for (int l = c.n_double - 1; l >= 0; --l) {
         const DitBlockIo& io = p.blk[l];
+        if (recompute) FF_TRY(mmdit_forward_double(m, B, l, io, f, stream));
         const int base = l * 12 * H;
         const int first_img = B * cps_t;
         const Stream st[2] = {{"img", Rt, Ri, Ni, base, first_img, cps_i}, {"txt", 0, Rt, Nt, base + 6 * H, 0, cps_t}};

@@ -369,6 +369,13 @@ struct FwdBufs {
 };
 int mmdit_forward(const ff_dit* m, int B, const float* x_t, const void* txt, const float* t, float* v_out,
                   const FwdBufs& f, cudaStream_t stream);
+// Its four parts: embeddings and modulation; double-stream block l and
+// single-stream block l, each from io.xin to io.xout; the final layer.
+int mmdit_forward_prologue(const ff_dit* m, int B, const float* x_t, const void* txt, const float* t,
+                           const FwdBufs& f, cudaStream_t stream);
+int mmdit_forward_double(const ff_dit* m, int B, int l, const DitBlockIo& io, const FwdBufs& f, cudaStream_t stream);
+int mmdit_forward_single(const ff_dit* m, int B, int l, const DitBlockIo& io, const FwdBufs& f, cudaStream_t stream);
+int mmdit_forward_final(const ff_dit* m, int B, const FwdBufs& f, float* v_out, cudaStream_t stream);
 int wan_forward(const ff_dit* m, int B, const float* x_t, const void* txt, const float* t, float* v_out,
                 const FwdBufs& f, cudaStream_t stream);
 // Its three parts: embeddings and modulation; block l from io.xin to

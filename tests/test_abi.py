@@ -200,10 +200,14 @@ def test_training_pass_host_validation(L):
     assert L.ff_dit_train_workspace_size(hr, 4, C.byref(n)) == 0
     assert n.value < full - Ri * (38 * 256 + 4 * 512)
     assert L.ff_dit_destroy(hr) == 0
-    c64b = ffi.make_config(synth.config("tiny_mmdit"))
+    c64b = ffi.make_config(synth.config("tiny_mmdit"))                 # 2 double blocks
     assert L.ff_dit_create(C.byref(c64b), C.c_void_p(256), C.byref(hr)) == 0
-    assert L.ff_dit_set_train_recompute(hr, 1) == 2                    # WAN-style models only
-    assert L.ff_dit_set_train_recompute(hr, 0) == 0
+    assert L.ff_dit_train_workspace_size(hr, 4, C.byref(n)) == 0
+    stored = n.value
+    assert L.ff_dit_set_train_recompute(hr, 1) == 0
+    assert L.ff_dit_train_workspace_size(hr, 4, C.byref(n)) == 0
+    assert n.value < stored
+    assert L.ff_dit_set_train_recompute(None, 1) == 1
     assert L.ff_dit_destroy(hr) == 0
     wodd = ffi.make_config(dict(wcfg, n_txt=5))      # B N_t = 20: not a multiple of 8
     assert L.ff_dit_create(C.byref(wodd), C.c_void_p(256), C.byref(h)) == 0

@@ -158,13 +158,16 @@ def test_wan_forward_train_equals_velocity_and_backward_is_deterministic(cuda):
     assert np.array_equal(g1, g2) and np.array_equal(d1, d2)
 
 
-@pytest.mark.parametrize("L", [1, 3])
-def test_wan_recompute_gives_the_same_gradient(cuda, L):
+@pytest.mark.parametrize("cfg", [dict(WAN_TRAIN, n_double=1), dict(WAN_TRAIN, n_double=3),
+                                 _cfg(n_double=2, n_single=0), _cfg(n_double=0, n_single=3),
+                                 _cfg(n_double=2, n_single=2, grid=(1, 3, 5), n_txt=5, batch=8)])
+def test_recompute_gives_the_same_gradient(cuda, cfg):
     """Recompute mode (block inputs kept, each block re-run before its
-    backward) gives bit for bit the stored-activation pass's v and gradients."""
+    backward) gives bit for bit the stored-activation pass's v and gradients,
+    for WAN-style and MMDiT models."""
     import torch
     from paper_2602_12529_gb300 import ffi
-    cfg = dict(WAN_TRAIN, n_double=L)
+    L = cfg["n_double"] + cfg["n_single"]
     run = Run(cfg, cuda, seed=3)
     dv = np.random.default_rng(10).standard_normal(tuple(run.v.shape)).astype(np.float32)
     g1, d1 = run.backward(dv)
