@@ -559,16 +559,21 @@ def train_step(args, ffi, model, cfg, dev, x, txt, t, tn, sg, x_next, lp_old, ad
     4 B h N^2 d), plus twice the GEMM FLOPs (input and weight gradients) and
     10 B h N^2 d per attention backward (recomputed S, dP, dV, dK, dQ)."""
     import torch
-    if cfg.get("arch") == "wan" or cfg["head_dim"] != 128:
-        return None
     B = x.shape[0]
     D = x.numel() // B
     need = model.train_workspace_size(B)
     _, total = ffi.ff_dit_weight_layout(cfg)
     free, _ = torch.cuda.mem_get_info(dev)
+    recompute = False
     if need + 4 * total > 0.9 * free:
-        return {"skipped": f"training workspace {need / 1e9:.1f} GB + fp32 gradients {4 * total / 1e9:.1f} GB "
-                           f"exceed the free device memory ({free / 1e9:.1f} GB)"}
+        # keep only the block inputs and re-run each block in the backward
+        model.set_train_recompute(True)
+        recompute = True
+        need = model.train_workspace_size(B)
+        if need + 4 * total > 0.9 * free:
+            model.set_train_recompute(False)
+            return {"skipped": f"training workspace {need / 1e9:.1f} GB (recompute mode) + fp32 gradients "
+                               f"{4 * total / 1e9:.1f} GB exceed the free device memory ({free / 1e9:.1f} GB)"}
     ws_t = torch.empty(need, dtype=torch.uint8, device=dev)
     grad = torch.empty(total, dtype=torch.float32, device=dev)
     v = torch.empty_like(x)
@@ -593,15 +598,21 @@ def train_step(args, ffi, model, cfg, dev, x, txt, t, tn, sg, x_next, lp_old, ad
     timed(step, args.steps)
     recs = ffi.ff_prof_records()
     ffi.ff_prof_disable()
+    if recompute:
+        model.set_train_recompute(False)
     kern = {}
     for name, ms_, fl, by in recs:
         k = kern.setdefault(name, [0, 0.0])
         k[0] += 1
         k[1] += ms_
     tot = sum(k[1] for k in kern.values())
-    N = cfg["n_txt"] + synth_n_img(cfg)
+    Ni = synth_n_img(cfg)
     L = cfg["n_double"] + cfg["n_single"]
-    attn_fwd = 4.0 * B * cfg["heads"] * N * N * cfg["head_dim"] * L
+    if cfg.get("arch") == "wan":   # self-attention over the latents + cross-attention to the text
+        attn_fwd = 4.0 * B * cfg["hidden"] * Ni * (Ni + cfg["n_txt"]) * L
+    else:                          # joint attention over text + latents
+        N = cfg["n_txt"] + Ni
+        attn_fwd = 4.0 * B * cfg["heads"] * N * N * cfg["head_dim"] * L
     gemm_fwd = fwd_flops - attn_fwd
     flops = 3.0 * gemm_fwd + attn_fwd + 2.5 * attn_fwd
     _, tc_burst, tc_sust, src = load_peaks()
@@ -610,7 +621,8 @@ def train_step(args, ffi, model, cfg, dev, x, txt, t, tn, sg, x_next, lp_old, ad
                     "log-prob backward + DiT backward to every weight (fp32 gradients), batch of the main step",
             "tflops": flops / (ms / 1e3) / 1e12, "frac": flops / (ms / 1e3) / 1e12 / tc_burst,
             "frac_vs_sustained": flops / (ms / 1e3) / 1e12 / tc_sust if tc_sust else None,
-            "algorithmic_flops": flops, "workspace_gb": need / 1e9, "gpu_launches": len(recs) // args.steps,
+            "algorithmic_flops": flops, "workspace_gb": need / 1e9, "recompute": recompute,
+            "gpu_launches": len(recs) // args.steps,
             "kernels": {k: {"launches": v_[0] // args.steps, "ms_per_step": v_[1] / args.steps, "share": v_[1] / tot}
                         for k, v_ in sorted(kern.items(), key=lambda kv: -kv[1][1])},
             "peak": f"{tc_burst} TFLOP/s ({src} bf16 dense burst)"}
