@@ -432,7 +432,9 @@ int ff_dit_velocity(const ff_dit* model, int B, const float* x_t, const void* tx
  * 4 H bytes per row and block instead of the stored activations.  The
  * gradient is bit-identical to the stored-activation pass (every kernel is
  * deterministic).  Set it before ff_dit_train_workspace_size and keep it
- * unchanged until the matching ff_dit_backward. */
+ * unchanged until the matching ff_dit_backward: ff_dit_backward returns
+ * FF_ERR_INVALID_ARG when the mode differs from that of the model's latest
+ * ff_dit_forward_train (or when there was none). */
 int ff_dit_set_train_recompute(ff_dit* model, int on);
 int ff_dit_train_workspace_size(const ff_dit* model, int B, size_t* bytes);
 int ff_dit_forward_train(const ff_dit* model, int B, const float* x_t, const void* txt,

@@ -30,6 +30,7 @@ struct ff_dit {
     std::unordered_map<std::string, int64_t> off;
     int64_t mod_width;
     int train_recompute = 0;   // training pass: keep block inputs only, re-run each block before its backward
+    mutable int fwd_recompute = -1;   // the mode of the latest ff_dit_forward_train (-1: none yet)
 };
 
 namespace ff {
@@ -673,6 +674,8 @@ int64_t model_offset(const ff_dit* m, const char* name) {
 }
 int64_t model_mod_width(const ff_dit* m) { return m->mod_width; }
 int model_train_recompute(const ff_dit* m) { return m->train_recompute; }
+void model_note_forward_train(const ff_dit* m) { m->fwd_recompute = m->train_recompute; }
+int model_forward_train_mode(const ff_dit* m) { return m->fwd_recompute; }
 
 }  // namespace ff
 

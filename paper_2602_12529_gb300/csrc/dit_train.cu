@@ -193,6 +193,7 @@ int ff_dit_forward_train(const ff_dit* m, int B, const float* x_t, const void* t
     if (!aligned16(x_t) || !aligned16(txt) || !aligned16(v_out) || (reinterpret_cast<uintptr_t>(ws) % kAlign))
         return set_error(FF_ERR_INVALID_ARG, "misaligned pointer (arrays 16 B, workspace 256 B)");
     const ff_dit_config& c = model_config(m);
+    model_note_forward_train(m);
     if (c.arch == FF_ARCH_WAN) return wan_forward_train(m, B, x_t, txt, t, v_out, ws, ws_bytes, stream);
     TrainPlan p = plan(c, model_mod_width(m), B, static_cast<uint8_t*>(ws), model_train_recompute(m) != 0);
     if (ws_bytes < p.bytes) return set_error(FF_ERR_WORKSPACE, "workspace %zu B < %zu B needed", ws_bytes, p.bytes);
@@ -217,6 +218,10 @@ int ff_dit_backward(const ff_dit* m, int B, const void* txt, const float* dv, fl
         (reinterpret_cast<uintptr_t>(ws) % kAlign))
         return set_error(FF_ERR_INVALID_ARG, "misaligned pointer (arrays 16 B, workspace 256 B)");
     const ff_dit_config& c = model_config(m);
+    if (model_forward_train_mode(m) != model_train_recompute(m))
+        return set_error(FF_ERR_INVALID_ARG, model_forward_train_mode(m) < 0
+                                                 ? "backward: no ff_dit_forward_train on this model yet"
+                                                 : "backward: recompute mode changed since ff_dit_forward_train");
     if (c.arch == FF_ARCH_WAN) return wan_backward(m, B, txt, dv, grad, dx_t, ws, ws_bytes, stream);
     const int64_t Wm = model_mod_width(m);
     const bool recompute = model_train_recompute(m) != 0;

@@ -35,6 +35,10 @@ const __nv_bfloat16* model_weights(const ff_dit* m);
 int64_t model_offset(const ff_dit* m, const char* name);
 int64_t model_mod_width(const ff_dit* m);
 int model_train_recompute(const ff_dit* m);
+// The training forward records its recompute mode on the handle; the
+// backward refuses to run in another mode (the workspace layouts differ).
+void model_note_forward_train(const ff_dit* m);
+int model_forward_train_mode(const ff_dit* m);
 
 // ---- optional launch timing (ff_prof_*): RAII scope around one launch ----
 struct ProfScope {

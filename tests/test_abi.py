@@ -208,6 +208,17 @@ def test_training_pass_host_validation(L):
     assert L.ff_dit_train_workspace_size(hr, 4, C.byref(n)) == 0
     assert n.value < stored
     assert L.ff_dit_set_train_recompute(None, 1) == 1
+    # the backward runs only in the mode of the model's latest training forward
+    assert L.ff_dit_destroy(hr) == 0
+    assert L.ff_dit_create(C.byref(c64b), C.c_void_p(256), C.byref(hr)) == 0
+    assert L.ff_dit_backward(hr, 4, 16, 16, 16, None, 256, 1 << 40, None) == 1       # no forward yet
+    assert b"no ff_dit_forward_train" in L.ff_last_error()
+    assert L.ff_dit_forward_train(hr, 4, 16, 16, 16, 16, 256, 1024, None) == 3        # workspace too small
+    assert L.ff_dit_set_train_recompute(hr, 1) == 0
+    assert L.ff_dit_backward(hr, 4, 16, 16, 16, None, 256, 1 << 40, None) == 1       # mode changed since
+    assert b"recompute mode changed" in L.ff_last_error()
+    assert L.ff_dit_set_train_recompute(hr, 0) == 0
+    assert L.ff_dit_backward(hr, 4, 16, 16, 16, None, 256, 1024, None) == 3          # same mode: on to the workspace check
     assert L.ff_dit_destroy(hr) == 0
     wodd = ffi.make_config(dict(wcfg, n_txt=5))      # B N_t = 20: not a multiple of 8
     assert L.ff_dit_create(C.byref(wodd), C.c_void_p(256), C.byref(h)) == 0
