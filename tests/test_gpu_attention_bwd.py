@@ -28,7 +28,7 @@ def _host(t):
 
 
 @pytest.mark.parametrize("d,B,heads,n0,n1", [(128, 2, 2, 5, 70), (128, 1, 3, 32, 200), (128, 2, 2, 0, 130),
-                                             (128, 1, 2, 300, 777), (128, 1, 2, 512, 4096),
+                                             (128, 1, 2, 300, 777), (128, 1, 2, 512, 4096), (128, 1, 8, 512, 4096),
                                              (64, 4, 4, 32, 64), (64, 2, 2, 5, 70), (64, 1, 3, 300, 777)])
 def test_attention_backward_parity(cuda, d, B, heads, n0, n1):
     import torch
