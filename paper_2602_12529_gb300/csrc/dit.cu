@@ -216,7 +216,7 @@ void set_qk_norm(GemmEpilogue& e, const ff_dit_config& c, int qk_cols, const __n
 int wan_forward_prologue(const ff_dit* m, int B, const float* x_t, const void* txt, const float* t,
                          const FwdBufs& f, cudaStream_t stream) {
     const ff_dit_config& c = m->cfg;
-    const int H = c.hidden, F = c.mlp, P = c.patch_dim, d = c.head_dim, L = c.n_double;
+    const int H = c.hidden, P = c.patch_dim, L = c.n_double;
     const int Nt = c.n_txt, Ni = c.grid_f * c.grid_h * c.grid_w;
     const int Rt = B * Nt, Ri = B * Ni;
     const int64_t Wm = m->mod_width;
@@ -423,12 +423,11 @@ int wan_forward(const ff_dit* m, int B, const float* x_t, const void* txt, const
 int mmdit_forward_prologue(const ff_dit* m, int B, const float* x_t, const void* txt, const float* t,
                            const FwdBufs& f, cudaStream_t stream) {
     const ff_dit_config& c = m->cfg;
-    const int H = c.hidden, F = c.mlp, P = c.patch_dim;
+    const int H = c.hidden, P = c.patch_dim;
     const int Nt = c.n_txt, Ni = c.grid_f * c.grid_h * c.grid_w;
-    const int Rt = B * Nt, Ri = B * Ni, R = Rt + Ri;
+    const int Rt = B * Nt, Ri = B * Ni;
     const int64_t Wm = m->mod_width;
     auto W = [&](const std::string& n) { return m->w + m->off.at(n); };
-    auto rows = [](auto* p, int64_t r, int64_t ld) { return p ? p + r * ld : p; };
 
     // ---- rotation table, timestep embedding MLP and every adaLN vector
     FF_TRY(rope_table(f.rope, c.grid_f, c.grid_h, c.grid_w, c.rope_axes[0], c.rope_axes[1], c.rope_axes[2],
@@ -483,9 +482,9 @@ struct Stream { const char* name; int row0, rows, tokens; int64_t mod; };
 int mmdit_forward_double(const ff_dit* m, int B, int l, const DitBlockIo& io, const FwdBufs& f,
                          cudaStream_t stream) {
     const ff_dit_config& c = m->cfg;
-    const int H = c.hidden, F = c.mlp, P = c.patch_dim;
+    const int H = c.hidden, F = c.mlp;
     const int Nt = c.n_txt, Ni = c.grid_f * c.grid_h * c.grid_w;
-    const int Rt = B * Nt, Ri = B * Ni, R = Rt + Ri;
+    const int Rt = B * Nt, Ri = B * Ni;
     const int64_t Wm = m->mod_width;
     auto W = [&](const std::string& n) { return m->w + m->off.at(n); };
     auto rows = [](auto* p, int64_t r, int64_t ld) { return p ? p + r * ld : p; };
@@ -581,7 +580,7 @@ int mmdit_forward_double(const ff_dit* m, int B, int l, const DitBlockIo& io, co
 int mmdit_forward_single(const ff_dit* m, int B, int l, const DitBlockIo& io, const FwdBufs& f,
                          cudaStream_t stream) {
     const ff_dit_config& c = m->cfg;
-    const int H = c.hidden, F = c.mlp, P = c.patch_dim;
+    const int H = c.hidden, F = c.mlp;
     const int Nt = c.n_txt, Ni = c.grid_f * c.grid_h * c.grid_w;
     const int Rt = B * Nt, Ri = B * Ni, R = Rt + Ri;
     const int64_t Wm = m->mod_width;
@@ -635,12 +634,10 @@ int mmdit_forward_single(const ff_dit* m, int B, int l, const DitBlockIo& io, co
 
 int mmdit_forward_final(const ff_dit* m, int B, const FwdBufs& f, float* v_out, cudaStream_t stream) {
     const ff_dit_config& c = m->cfg;
-    const int H = c.hidden, F = c.mlp, P = c.patch_dim;
+    const int H = c.hidden, P = c.patch_dim;
     const int Nt = c.n_txt, Ni = c.grid_f * c.grid_h * c.grid_w;
-    const int Rt = B * Nt, Ri = B * Ni, R = Rt + Ri;
-    const int64_t Wm = m->mod_width;
+    const int Rt = B * Nt, Ri = B * Ni;
     auto W = [&](const std::string& n) { return m->w + m->off.at(n); };
-    auto rows = [](auto* p, int64_t r, int64_t ld) { return p ? p + r * ld : p; };
     LnModArgs la = mmdit_ln_args(m, B, f);
     // ---- final layer on image tokens -> v (fp32)
     {
