@@ -225,6 +225,14 @@ def test_training_pass_host_validation(L):
     assert L.ff_dit_train_workspace_size(h, 4, C.byref(n)) == 2
     assert L.ff_dit_train_workspace_size(h, 8, C.byref(n)) == 0
     assert L.ff_dit_destroy(h) == 0
+    # cross-attention (latent queries, text keys / values): rejected on the host
+    assert L.ff_cross_attention_forward(1, 2, 128, 0, 16, 256, 8, 16, 512, 16, 256, None, None) == 1   # nq = 0
+    assert L.ff_cross_attention_forward(1, 2, 128, 8, 16, 256, 0, 16, 512, 16, 256, None, None) == 1   # nk = 0
+    assert L.ff_cross_attention_forward(1, 2, 128, 8, 16, 256, 8, 16, 512, 16, 256, 8, None) == 1      # lse misaligned
+    assert L.ff_cross_attention_backward(1, 2, 128, 8, 16, 256, 16, 16, 256, 16, 256, 8, 16, 512, 16, 256,
+                                         16, 16, 1 << 20, None) == 1                                     # lddkv < 2H
+    assert L.ff_cross_attention_backward(1, 2, 96, 8, 16, 192, 16, 16, 192, 16, 192, 8, 16, 384, 16, 384,
+                                         16, 16, 1 << 20, None) == 2                                     # head_dim 96
     # the counter-based noise and the SDE step that draws it
     assert L.ff_philox_normal(2, 18, 1, 0, 16, None) == 2                  # D % 4
     assert L.ff_philox_normal(2, 16, 1, 0, None, None) == 1                # null out
