@@ -20,6 +20,7 @@
 //     gradient is deterministic.
 #include "internal.h"
 #include "ptx.cuh"
+#include "reduce_jobs.h"
 
 namespace ff {
 namespace {
@@ -381,41 +382,61 @@ __global__ void __launch_bounds__(kThreads) colsum_partial_kernel(const T* in, i
 
 // ---------------------------------------------------------------- chunk reduction
 
-// out[b * ld_out + j] = sum over sample b's chunks of every span (per_sample),
-// or out[j] = sum over all chunks of every span.  A CTA takes 32 columns
-// (lane = column, so a chunk row is one 128-byte load per warp); warp w takes
-// the chunks w, w + 8, ... in four interleaved fp64 chains, and the eight
-// warp sums are added in warp order: a fixed order for a given shape.
-__global__ void __launch_bounds__(256) reduce_chunks_kernel(const float* part, int64_t ld_part, int ncols,
-                                                            ChunkSpans sp, int per_sample, float* out,
-                                                            int64_t ld_out) {
+// A batch of fixed-order sums: column block x of the grid belongs to job k
+// (blk0[k] <= x < blk0[k + 1]), blockIdx.y is the sample of a per-sample job.
+// out[b * ld_out + j] = sum over sample b's chunks of every span
+// (per_sample), or out[j] = sum over all chunks of every span.  A CTA takes 32
+// columns (lane = column, so a chunk row is one 128-byte load per warp); warp
+// w takes the chunks w, w + 8, ... in four interleaved fp64 chains, and the
+// eight warp sums are added in warp order: a fixed order for a given shape,
+// the same whichever jobs share the launch.
+struct ReduceBatch {
+    ReduceJob job[kMaxReduceJobs];
+    int blk0[kMaxReduceJobs + 1];
+    int n;
+};
+
+__global__ void __launch_bounds__(256) reduce_chunks_kernel(ReduceBatch rb) {
     __shared__ double red[8][32];
-    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-    const int j = blockIdx.x * 32 + lane;
+    // the job of this column block, picked by selects (no dynamic indexing
+    // of the parameter struct)
+    const int x = blockIdx.x;
+    ReduceJob jb = rb.job[0];
+    int blk0 = 0;
+#pragma unroll
+    for (int k = 1; k < kMaxReduceJobs; ++k)
+        if (k < rb.n && x >= rb.blk0[k]) {
+            jb = rb.job[k];
+            blk0 = rb.blk0[k];
+        }
     const int b = blockIdx.y;
+    if (!jb.per_sample && b > 0) return;   // uniform over the CTA
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    const int j = (x - blk0) * 32 + lane;
     double acc[4] = {0.0, 0.0, 0.0, 0.0};
-    if (j < ncols) {
-        for (int i = 0; i < sp.n; ++i) {
-            const int first = per_sample ? sp.first[i] + b * sp.count[i] : sp.first[i];
-            const int cnt = sp.count[i];
-            const float* base = part + static_cast<int64_t>(first) * ld_part + j;
+    if (j < jb.ncols) {
+        for (int i = 0; i < jb.sp.n; ++i) {
+            const int cnt = i ? jb.sp.count[1] : jb.sp.count[0];
+            const int first = (i ? jb.sp.first[1] : jb.sp.first[0]) + (jb.per_sample ? b * cnt : 0);
+            const float* base = jb.part + static_cast<int64_t>(first) * jb.ld_part + j;
+            const int64_t ld = jb.ld_part;
             int c = w;
             for (; c + 24 < cnt; c += 32) {
-                acc[0] += base[static_cast<int64_t>(c) * ld_part];
-                acc[1] += base[static_cast<int64_t>(c + 8) * ld_part];
-                acc[2] += base[static_cast<int64_t>(c + 16) * ld_part];
-                acc[3] += base[static_cast<int64_t>(c + 24) * ld_part];
+                acc[0] += base[static_cast<int64_t>(c) * ld];
+                acc[1] += base[static_cast<int64_t>(c + 8) * ld];
+                acc[2] += base[static_cast<int64_t>(c + 16) * ld];
+                acc[3] += base[static_cast<int64_t>(c + 24) * ld];
             }
-            for (; c < cnt; c += 8) acc[0] += base[static_cast<int64_t>(c) * ld_part];
+            for (; c < cnt; c += 8) acc[0] += base[static_cast<int64_t>(c) * ld];
         }
     }
     red[w][lane] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
     __syncthreads();
-    if (w == 0 && j < ncols) {
+    if (w == 0 && j < jb.ncols) {
         double s = 0.0;
 #pragma unroll
         for (int k = 0; k < 8; ++k) s += red[k][lane];
-        out[static_cast<int64_t>(b) * ld_out + j] = static_cast<float>(s);
+        jb.out[static_cast<int64_t>(b) * jb.ld_out + j] = static_cast<float>(s);
     }
 }
 
@@ -472,12 +493,8 @@ __global__ void wan_modulation_backward_kernel(const float* dm, int64_t ld, int 
 
 int reduce(const float* part, int64_t ld_part, int ncols, const ChunkSpans& sp, int B, float* out, int64_t ld_out,
            cudaStream_t stream) {
-    double chunks = 0.0;
-    for (int i = 0; i < sp.n; ++i) chunks += static_cast<double>(sp.count[i]) * (B > 0 ? B : 1);
-    ProfScope prof(stream, "reduce_chunks", 0.0, chunks * ncols * 4.0);
-    dim3 grid((ncols + 31) / 32, B > 0 ? B : 1);
-    reduce_chunks_kernel<<<grid, 256, 0, stream>>>(part, ld_part, ncols, sp, B > 0, out, ld_out);
-    return check_launch("reduce_chunks_kernel");
+    const ReduceJob j{part, ld_part, ncols, sp, B > 0 ? 1 : 0, out, ld_out};
+    return reduce_chunks_batch(&j, 1, B, stream);
 }
 
 }  // namespace
@@ -566,6 +583,34 @@ int colsum(const void* in, bool f32, int64_t ld, int rows, int ncols, float* out
 int reduce_chunks(const float* part, int64_t ld_part, int ncols, const ChunkSpans& sp, int B, float* out,
                   int64_t ld_out, cudaStream_t stream) {
     return reduce(part, ld_part, ncols, sp, B, out, ld_out, stream);
+}
+
+int reduce_chunks_batch(const ReduceJob* jobs, int n, int B, cudaStream_t stream) {
+    for (int at = 0; at < n; at += kMaxReduceJobs) {
+        ReduceBatch rb{};
+        rb.n = n - at < kMaxReduceJobs ? n - at : kMaxReduceJobs;
+        bool any_per_sample = false;
+        double bytes = 0.0;
+        int blocks = 0;
+        for (int k = 0; k < rb.n; ++k) {
+            const ReduceJob& j = jobs[at + k];
+            if (j.ncols <= 0 || j.sp.n < 1 || j.sp.n > 2 || (j.per_sample && B <= 0))
+                return set_error(FF_ERR_INVALID_ARG, "reduce_chunks: job %d: ncols=%d spans=%d B=%d", at + k, j.ncols,
+                                 j.sp.n, B);
+            rb.job[k] = j;
+            rb.blk0[k] = blocks;
+            blocks += (j.ncols + 31) / 32;
+            any_per_sample = any_per_sample || j.per_sample;
+            double chunks = 0.0;
+            for (int i = 0; i < j.sp.n; ++i) chunks += static_cast<double>(j.sp.count[i]) * (j.per_sample ? B : 1);
+            bytes += chunks * j.ncols * 4.0;
+        }
+        rb.blk0[rb.n] = blocks;
+        ProfScope prof(stream, "reduce_chunks", 0.0, bytes);
+        reduce_chunks_kernel<<<dim3(blocks, any_per_sample ? B : 1), 256, 0, stream>>>(rb);
+        FF_TRY(check_launch("reduce_chunks_kernel"));
+    }
+    return FF_OK;
 }
 
 int silu_backward(const float* dy, int64_t ld_dy, const __nv_bfloat16* pre, int B, int rows_pad, int n, float* dx,

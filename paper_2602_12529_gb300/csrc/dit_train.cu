@@ -30,10 +30,12 @@
 // share one set of those activations and only the block inputs are kept;
 // the backward re-runs each block's forward (bit-identical: every kernel is
 // deterministic) just before its backward.
+#include <initializer_list>
 #include <string>
 #include <vector>
 
 #include "internal.h"
+#include "reduce_jobs.h"
 
 namespace ff {
 namespace {
@@ -237,16 +239,16 @@ int ff_dit_backward(const ff_dit* m, int B, const void* txt, const float* dv, fl
     auto W = [&](const std::string& n) { return w0 + model_offset(m, n.c_str()); };
     auto G = [&](const std::string& n) { return grad + model_offset(m, n.c_str()); };
     auto group = [&](GemmArgs* g, int n) { return gemm_bf16_group(g, n, stream); };
-    // reductions of chunk partials (columns ncols of part at offset col)
+    // reductions of chunk partials (columns ncols of part at offset col),
+    // the ones that follow one backward kernel batched into one launch
     auto per_sample = [&](int first, int count, int col, float* out) {
-        ChunkSpans sp{};
-        sp.n = 1; sp.first[0] = first; sp.count[0] = count;
-        return reduce_chunks(p.part + col, 2 * H, H, sp, B, out, Wm, stream);
+        return ReduceJob{p.part + col, 2 * H, H, chunk_span(first, count), 1, out, Wm};
     };
     auto total = [&](int first, int count, int col, int64_t ld, int ncols, float* out) {
-        ChunkSpans sp{};
-        sp.n = 1; sp.first[0] = first; sp.count[0] = count;
-        return reduce_chunks(p.part + col, ld, ncols, sp, 0, out, 0, stream);
+        return ReduceJob{p.part + col, ld, ncols, chunk_span(first, count), 0, out, 0};
+    };
+    auto reduce = [&](std::initializer_list<ReduceJob> jobs) {
+        return reduce_chunks_batch(jobs.begin(), static_cast<int>(jobs.size()), B, stream);
     };
 
     // ---- final layer: v = LNmod(x_img) W_f^T + b_f
@@ -268,8 +270,7 @@ int ff_dit_backward(const ff_dit* m, int B, const void* txt, const float* dv, fl
         const BwdSeg sg{Rt, Ni, 0, static_cast<int>(off_f + H)};
         const BwdSegs s = bwd_segs(&sg, 1, B);
         FF_TRY(ln_modulate_backward(f.xfin, p.dh, p.gx, H, f.mods, Wm, s, H, p.part, stream));
-        FF_TRY(per_sample(0, cps_i, 0, p.dmods + off_f));
-        FF_TRY(per_sample(0, cps_i, H, p.dmods + off_f + H));
+        FF_TRY(reduce({per_sample(0, cps_i, 0, p.dmods + off_f), per_sample(0, cps_i, H, p.dmods + off_f + H)}));
     }
 
     // ---- single-stream blocks, last first
@@ -286,9 +287,10 @@ int ff_dit_backward(const ff_dit* m, int B, const void* txt, const float* dv, fl
             FF_TRY(gate_backward(p.gx, io.y2, H, f.mods, Wm, s, H, p.dy, p.part, stream));
             ChunkSpans sp{};
             sp.n = 2; sp.first[0] = 0; sp.count[0] = cps_t; sp.first[1] = s.first[1]; sp.count[1] = cps_i;
-            FF_TRY(reduce_chunks(p.part, 2 * H, H, sp, B, p.dmods + off + 2 * H, Wm, stream));
-            sp.count[0] = B * cps_t; sp.count[1] = B * cps_i;
-            FF_TRY(reduce_chunks(p.part + H, 2 * H, H, sp, 0, G(pre + "linear2.b"), 0, stream));
+            ChunkSpans all = sp;
+            all.count[0] = B * cps_t; all.count[1] = B * cps_i;
+            FF_TRY(reduce({ReduceJob{p.part, 2 * H, H, sp, 1, p.dmods + off + 2 * H, Wm},
+                           ReduceJob{p.part + H, 2 * H, H, all, 0, G(pre + "linear2.b"), 0}}));
         }
         {
             GemmArgs g = wgrad(p.dy, H, io.u, H + F, H, H + F, R, G(pre + "linear2.w"));
@@ -321,8 +323,8 @@ int ff_dit_backward(const ff_dit* m, int B, const void* txt, const float* dv, fl
             a.part = p.part;
             int ct = 0, ci = 0;
             FF_TRY(qk_norm_rope_backward(a, &ct, &ci, stream));
-            FF_TRY(total(0, ct + ci, 0, 2 * d, d, G(pre + "q_norm.scale")));
-            FF_TRY(total(0, ct + ci, d, 2 * d, d, G(pre + "k_norm.scale")));
+            FF_TRY(reduce({total(0, ct + ci, 0, 2 * d, d, G(pre + "q_norm.scale")),
+                           total(0, ct + ci, d, 2 * d, d, G(pre + "k_norm.scale"))}));
         }
         FF_TRY(colsum(p.dbig, false, W1, R, W1, G(pre + "linear1.b"), p.cs_ws, stream));
         {
@@ -340,8 +342,8 @@ int ff_dit_backward(const ff_dit* m, int B, const void* txt, const float* dv, fl
             FF_TRY(ln_modulate_backward(io.xin, p.dh, p.gx, H, f.mods, Wm, s, H, p.part, stream));
             ChunkSpans sp{};
             sp.n = 2; sp.first[0] = 0; sp.count[0] = cps_t; sp.first[1] = s.first[1]; sp.count[1] = cps_i;
-            FF_TRY(reduce_chunks(p.part, 2 * H, H, sp, B, p.dmods + off, Wm, stream));
-            FF_TRY(reduce_chunks(p.part + H, 2 * H, H, sp, B, p.dmods + off + H, Wm, stream));
+            FF_TRY(reduce({ReduceJob{p.part, 2 * H, H, sp, 1, p.dmods + off, Wm},
+                           ReduceJob{p.part + H, 2 * H, H, sp, 1, p.dmods + off + H, Wm}}));
         }
     }
 
@@ -363,11 +365,10 @@ int ff_dit_backward(const ff_dit* m, int B, const void* txt, const float* dv, fl
             sg[1].col_a = st[0].mod + k * H;
             const BwdSegs s = bwd_segs(sg, 2, B);
             FF_TRY(gate_backward(p.gx, y, H, f.mods, Wm, s, H, p.dy, p.part, stream));
-            for (const Stream& x : st) {
-                FF_TRY(per_sample(x.first, x.cps, 0, p.dmods + x.mod + k * H));
-                FF_TRY(total(x.first, B * x.cps, H, 2 * H, H, G(P_(x, bias))));
-            }
-            return FF_OK;
+            return reduce({per_sample(st[0].first, st[0].cps, 0, p.dmods + st[0].mod + k * H),
+                           total(st[0].first, B * st[0].cps, H, 2 * H, H, G(P_(st[0], bias))),
+                           per_sample(st[1].first, st[1].cps, 0, p.dmods + st[1].mod + k * H),
+                           total(st[1].first, B * st[1].cps, H, 2 * H, H, G(P_(st[1], bias)))});
         };
         auto lnmod = [&](const float* x, int k_shift) {
             BwdSeg sg[2] = {seg_txt, seg_img};
@@ -375,11 +376,10 @@ int ff_dit_backward(const ff_dit* m, int B, const void* txt, const float* dv, fl
             sg[1].col_b = st[0].mod + (k_shift + 1) * H;
             const BwdSegs s = bwd_segs(sg, 2, B);
             FF_TRY(ln_modulate_backward(x, p.dh, p.gx, H, f.mods, Wm, s, H, p.part, stream));
-            for (const Stream& x_ : st) {
-                FF_TRY(per_sample(x_.first, x_.cps, 0, p.dmods + x_.mod + k_shift * H));
-                FF_TRY(per_sample(x_.first, x_.cps, H, p.dmods + x_.mod + (k_shift + 1) * H));
-            }
-            return FF_OK;
+            return reduce({per_sample(st[0].first, st[0].cps, 0, p.dmods + st[0].mod + k_shift * H),
+                           per_sample(st[0].first, st[0].cps, H, p.dmods + st[0].mod + (k_shift + 1) * H),
+                           per_sample(st[1].first, st[1].cps, 0, p.dmods + st[1].mod + k_shift * H),
+                           per_sample(st[1].first, st[1].cps, H, p.dmods + st[1].mod + (k_shift + 1) * H)});
         };
         // MLP half: x_out = x_mid + gate2 (GELU(LNmod2(x_mid) W1^T + b1) W2^T + b2)
         FF_TRY(gate(io.y2, 5, "mlp2.b"));
@@ -452,10 +452,10 @@ int ff_dit_backward(const ff_dit* m, int B, const void* txt, const float* dv, fl
             a.part = p.part;
             int ct = 0, ci = 0;
             FF_TRY(qk_norm_rope_backward(a, &ct, &ci, stream));
-            FF_TRY(total(0, ct, 0, 2 * d, d, G(pre + "txt.q_norm.scale")));
-            FF_TRY(total(0, ct, d, 2 * d, d, G(pre + "txt.k_norm.scale")));
-            FF_TRY(total(ct, ci, 0, 2 * d, d, G(pre + "img.q_norm.scale")));
-            FF_TRY(total(ct, ci, d, 2 * d, d, G(pre + "img.k_norm.scale")));
+            FF_TRY(reduce({total(0, ct, 0, 2 * d, d, G(pre + "txt.q_norm.scale")),
+                           total(0, ct, d, 2 * d, d, G(pre + "txt.k_norm.scale")),
+                           total(ct, ci, 0, 2 * d, d, G(pre + "img.q_norm.scale")),
+                           total(ct, ci, d, 2 * d, d, G(pre + "img.k_norm.scale"))}));
         }
         for (const Stream& s : st)
             FF_TRY(colsum(p.dqkv + static_cast<int64_t>(s.row0) * 3 * H, false, 3 * H, s.rows, 3 * H, G(P_(s, "qkv.b")),

@@ -27,10 +27,12 @@
 // those activations and only their input residuals are kept; the backward
 // re-runs block l's forward (bit-identical, every kernel is deterministic)
 // just before its backward.
+#include <initializer_list>
 #include <string>
 #include <vector>
 
 #include "internal.h"
+#include "reduce_jobs.h"
 
 namespace ff {
 namespace {
@@ -202,31 +204,29 @@ int wan_backward(const ff_dit* m, int B, const void* txt, const float* dv, float
     const BwdSeg img{0, Ni, 0, 0};
     // per-sample sums of the chunk partials (columns [col, col + H) of part) into dmods
     auto per_sample = [&](int col, float* out) {
-        ChunkSpans sp{};
-        sp.n = 1; sp.first[0] = 0; sp.count[0] = cps;
-        return reduce_chunks(p.part + col, 2 * H, H, sp, B, out, Wm, stream);
+        return ReduceJob{p.part + col, 2 * H, H, chunk_span(0, cps), 1, out, Wm};
     };
     // sums over every chunk (ncols columns of part at col, pitch ld)
     auto total = [&](int count, int col, int64_t ld, int ncols, float* out) {
-        ChunkSpans sp{};
-        sp.n = 1; sp.first[0] = 0; sp.count[0] = count;
-        return reduce_chunks(p.part + col, ld, ncols, sp, 0, out, 0, stream);
+        return ReduceJob{p.part + col, ld, ncols, chunk_span(0, count), 0, out, 0};
+    };
+    // the sums that follow one backward kernel, in one launch
+    auto reduce = [&](std::initializer_list<ReduceJob> jobs) {
+        return reduce_chunks_batch(jobs.begin(), static_cast<int>(jobs.size()), B, stream);
     };
     auto gate = [&](const __nv_bfloat16* y, int col_gate, float* dgate, float* dbias) {
         BwdSeg sg = img;
         sg.col_a = col_gate;
         const BwdSegs s = bwd_segs(&sg, 1, B);
         FF_TRY(gate_backward(p.gx, y, H, f.mods, Wm, s, H, p.dy, p.part, stream));
-        FF_TRY(per_sample(0, dgate));
-        return total(B * cps, H, 2 * H, H, dbias);
+        return reduce({per_sample(0, dgate), total(B * cps, H, 2 * H, H, dbias)});
     };
     auto lnmod = [&](const float* x, int col_shift) {
         BwdSeg sg = img;
         sg.col_b = col_shift + H;
         const BwdSegs s = bwd_segs(&sg, 1, B);
         FF_TRY(ln_modulate_backward(x, p.dh, p.gx, H, f.mods, Wm, s, H, p.part, stream));
-        FF_TRY(per_sample(0, p.dmods + col_shift));
-        return per_sample(H, p.dmods + col_shift + H);
+        return reduce({per_sample(0, p.dmods + col_shift), per_sample(H, p.dmods + col_shift + H)});
     };
 
     // ---- final layer: v = LNmod(x) W_f^T + b_f (shift | scale at L 6H)
@@ -301,11 +301,11 @@ int wan_backward(const ff_dit* m, int B, const void* txt, const float* dv, float
             a.d = p.dy; a.ldd = H; a.raw = io.qc_raw; a.ldr = H; a.rows = Ri;
             a.q_scale_txt = a.q_scale_img = a.k_scale_txt = a.k_scale_img = W(pre + "cross_q_norm.scale");
             FF_TRY(qk_norm_rope_backward(a, &ct, &ci, stream));
-            FF_TRY(total(ct + ci, 0, 2 * d, d, G(pre + "cross_q_norm.scale")));
+            FF_TRY(reduce({total(ct + ci, 0, 2 * d, d, G(pre + "cross_q_norm.scale"))}));
             a.d = p.dkv; a.ldd = 2 * H; a.raw = io.kv_raw; a.ldr = 2 * H; a.rows = Rt;
             a.q_scale_txt = a.q_scale_img = a.k_scale_txt = a.k_scale_img = W(pre + "cross_k_norm.scale");
             FF_TRY(qk_norm_rope_backward(a, &ct, &ci, stream));
-            FF_TRY(total(ct + ci, 0, 2 * d, d, G(pre + "cross_k_norm.scale")));
+            FF_TRY(reduce({total(ct + ci, 0, 2 * d, d, G(pre + "cross_k_norm.scale"))}));
         }
         FF_TRY(colsum(p.dy, false, H, Ri, H, G(pre + "cross_q.b"), p.cs_ws, stream));
         FF_TRY(gemm1(gemm_wgrad(p.dy, H, io.hc, H, H, H, Ri, G(pre + "cross_q.w"))));
@@ -327,8 +327,8 @@ int wan_backward(const ff_dit* m, int B, const void* txt, const float* dv, float
             const BwdSegs s = bwd_segs(&img, 1, B);
             FF_TRY(ln_modulate_backward(io.xmid, p.dh, p.gx, H, nullptr, 0, s, H, p.part, stream,
                                         W(pre + "cross_norm.scale")));
-            FF_TRY(total(B * cps, 0, 2 * H, H, G(pre + "cross_norm.b")));
-            FF_TRY(total(B * cps, H, 2 * H, H, G(pre + "cross_norm.scale")));
+            FF_TRY(reduce({total(B * cps, 0, 2 * H, H, G(pre + "cross_norm.b")),
+                           total(B * cps, H, 2 * H, H, G(pre + "cross_norm.scale"))}));
         }
 
         // self-attention half: x_mid = x_in + g1 (Attn(...) W_p^T + b_p)
@@ -355,8 +355,8 @@ int wan_backward(const ff_dit* m, int B, const void* txt, const float* dv, float
             a.part = p.part;
             int ct = 0, ci = 0;
             FF_TRY(qk_norm_rope_backward(a, &ct, &ci, stream));
-            FF_TRY(total(ct + ci, 0, 2 * d, d, G(pre + "q_norm.scale")));
-            FF_TRY(total(ct + ci, d, 2 * d, d, G(pre + "k_norm.scale")));
+            FF_TRY(reduce({total(ct + ci, 0, 2 * d, d, G(pre + "q_norm.scale")),
+                           total(ct + ci, d, 2 * d, d, G(pre + "k_norm.scale"))}));
         }
         FF_TRY(colsum(p.dbig, false, W3, Ri, W3, G(pre + "qkv.b"), p.cs_ws, stream));
         FF_TRY(gemm1(gemm_wgrad(p.dbig, W3, io.h1, H, W3, H, Ri, G(pre + "qkv.w"))));
