@@ -250,15 +250,20 @@ __global__ void __launch_bounds__(kThreads) ln_modulate_backward_kernel(const fl
 
 // ---------------------------------------------------------------- QK norm + RoPE
 
-// One warp per (row, head) item, lane owns E = d / 32 consecutive elements
-// (whole rotation pairs).  A CTA covers kQkRows rows of one segment and
-// every head; its warps add their lanes' scale-gradient terms, summed over
-// the CTA at the end into part[cta][q: 0..d | k: d..2d].
+// A warp takes whole rows (rows r_begin + w, r_begin + w + 8, ...) and, per
+// row, every head in order; lane owns E = d / 32 consecutive elements of a
+// head (whole rotation pairs).  The rotation of a lane's pairs depends on
+// the row only, so it is looked up once per row and serves every head of q
+// and k.  The q and k gradient and raw loads of the next head are issued
+// before the current head's arithmetic (the loop is bound by load latency).  A CTA covers kQkRows rows of one segment; its warps add
+// their lanes' scale-gradient terms, summed over the CTA at the end into
+// part[cta][q: 0..d | k: d..2d].
 constexpr int kQkRows = kQkBwdRows;
+constexpr int kQkWarps = kThreads / 32;
 
 template <int E>
 __global__ void __launch_bounds__(kThreads) qk_norm_rope_backward_kernel(QkBwdArgs a, int ctas_txt) {
-    __shared__ float red[kThreads / 32][2][128];
+    __shared__ float red[kQkWarps][2][128];
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
     const bool img = static_cast<int>(blockIdx.x) >= ctas_txt;
     const int r_begin = img ? a.rows_txt + (blockIdx.x - ctas_txt) * kQkRows : blockIdx.x * kQkRows;
@@ -275,10 +280,7 @@ __global__ void __launch_bounds__(kThreads) qk_norm_rope_backward_kernel(QkBwdAr
         gq[i] = gk[i] = 0.f;
     }
     const int h0 = a.axes0 >> 1, h1 = a.axes1 >> 1;
-    const int items = (r_end - r_begin) * a.heads;
-    for (int it = w; it < items; it += kThreads / 32) {
-        const int row = r_begin + it / a.heads;
-        const int head = it - (it / a.heads) * a.heads;
+    for (int row = r_begin + w; row < r_end; row += kQkWarps) {
         // rotation of this lane's pairs (identity for text tokens)
         float cs[E / 2], sn[E / 2];
         if (img && a.rope_cs) {
@@ -298,47 +300,76 @@ __global__ void __launch_bounds__(kThreads) qk_norm_rope_backward_kernel(QkBwdAr
 #pragma unroll
             for (int p = 0; p < E / 2; ++p) { cs[p] = 1.f; sn[p] = 0.f; }
         }
+        __nv_bfloat16* grow = a.d + static_cast<int64_t>(row) * a.ldd + c0;
+        const __nv_bfloat16* xrow = a.raw + static_cast<int64_t>(row) * a.ldr + c0;
+        // packed bf16 pairs of head h (cur) and of head h + 1 (nxt, loaded
+        // before head h's arithmetic and stores)
+        uint32_t cur_g[2][E / 2], cur_x[2][E / 2], nxt_g[2][E / 2], nxt_x[2][E / 2];
+        auto load_head = [&](int head, uint32_t (&g)[2][E / 2], uint32_t (&x)[2][E / 2]) {
 #pragma unroll
-        for (int which = 0; which < 2; ++which) {
-            if (which >= a.sets) break;
-            const int col = which * a.heads * d + head * d + c0;
-            __nv_bfloat16* gp = a.d + static_cast<int64_t>(row) * a.ldd + col;
-            const __nv_bfloat16* xp = a.raw + static_cast<int64_t>(row) * a.ldr + col;
-            float gv[E], xv[E];
+            for (int which = 0; which < 2; ++which) {
+                if (which >= a.sets) break;
+                const int col = (which * a.heads + head) * d;
 #pragma unroll
-            for (int i = 0; i < E; i += 2) {
-                const float2 g2 = unpack_bf16x2(*reinterpret_cast<const uint32_t*>(gp + i));
-                const float2 x2 = unpack_bf16x2(*reinterpret_cast<const uint32_t*>(xp + i));
-                gv[i] = g2.x; gv[i + 1] = g2.y;
-                xv[i] = x2.x; xv[i + 1] = x2.y;
+                for (int i = 0; i < E / 2; ++i) {
+                    g[which][i] = *reinterpret_cast<const uint32_t*>(grow + col + 2 * i);
+                    x[which][i] = *reinterpret_cast<const uint32_t*>(xrow + col + 2 * i);
+                }
             }
-            // transposed rotation: gradient w.r.t. the normalised, scaled values
-            float gy[E];
+        };
+        load_head(0, cur_g, cur_x);
+        for (int head = 0; head < a.heads; ++head) {
+            if (head + 1 < a.heads) load_head(head + 1, nxt_g, nxt_x);
+            float gv[2][E], xv[2][E];
 #pragma unroll
-            for (int p = 0; p < E / 2; ++p) {
-                gy[2 * p] = gv[2 * p] * cs[p] + gv[2 * p + 1] * sn[p];
-                gy[2 * p + 1] = -gv[2 * p] * sn[p] + gv[2 * p + 1] * cs[p];
+            for (int which = 0; which < 2; ++which) {
+#pragma unroll
+                for (int i = 0; i < E / 2; ++i) {
+                    const float2 g2 = unpack_bf16x2(cur_g[which][i]);
+                    const float2 x2 = unpack_bf16x2(cur_x[which][i]);
+                    gv[which][2 * i] = g2.x; gv[which][2 * i + 1] = g2.y;
+                    xv[which][2 * i] = x2.x; xv[which][2 * i + 1] = x2.y;
+                }
             }
-            float ss = 0.f;
 #pragma unroll
-            for (int i = 0; i < E; ++i) ss = fmaf(xv[i], xv[i], ss);
-            const float r = rsqrtf(warp_sum(ss) / d + kRmsEps);
-            const float* wv = which ? wk : wq;
-            float* acc = which ? gk : gq;
-            float dot = 0.f;
-            float xn[E], gg[E];
+            for (int which = 0; which < 2; ++which) {
+                if (which >= a.sets) break;
+                // transposed rotation: gradient w.r.t. the normalised, scaled values
+                float gy[E];
 #pragma unroll
-            for (int i = 0; i < E; ++i) {
-                xn[i] = xv[i] * r;
-                gg[i] = gy[i] * wv[i];
-                acc[i] = fmaf(gy[i], xn[i], acc[i]);
-                dot = fmaf(gg[i], xn[i], dot);
+                for (int p = 0; p < E / 2; ++p) {
+                    gy[2 * p] = gv[which][2 * p] * cs[p] + gv[which][2 * p + 1] * sn[p];
+                    gy[2 * p + 1] = -gv[which][2 * p] * sn[p] + gv[which][2 * p + 1] * cs[p];
+                }
+                float ss = 0.f;
+#pragma unroll
+                for (int i = 0; i < E; ++i) ss = fmaf(xv[which][i], xv[which][i], ss);
+                const float r = rsqrtf(warp_sum(ss) / d + kRmsEps);
+                const float* wv = which ? wk : wq;
+                float* acc = which ? gk : gq;
+                float dot = 0.f;
+                float xn[E], gg[E];
+#pragma unroll
+                for (int i = 0; i < E; ++i) {
+                    xn[i] = xv[which][i] * r;
+                    gg[i] = gy[i] * wv[i];
+                    acc[i] = fmaf(gy[i], xn[i], acc[i]);
+                    dot = fmaf(gg[i], xn[i], dot);
+                }
+                const float m = warp_sum(dot) / d;
+                __nv_bfloat16* gp = grow + (which * a.heads + head) * d;
+#pragma unroll
+                for (int i = 0; i < E; i += 2)
+                    *reinterpret_cast<uint32_t*>(gp + i) =
+                        pack_bf16x2(r * (gg[i] - xn[i] * m), r * (gg[i + 1] - xn[i + 1] * m));
             }
-            const float m = warp_sum(dot) / d;
 #pragma unroll
-            for (int i = 0; i < E; i += 2)
-                *reinterpret_cast<uint32_t*>(gp + i) =
-                    pack_bf16x2(r * (gg[i] - xn[i] * m), r * (gg[i + 1] - xn[i + 1] * m));
+            for (int which = 0; which < 2; ++which)
+#pragma unroll
+                for (int i = 0; i < E / 2; ++i) {
+                    cur_g[which][i] = nxt_g[which][i];
+                    cur_x[which][i] = nxt_x[which][i];
+                }
         }
     }
 #pragma unroll
@@ -351,7 +382,7 @@ __global__ void __launch_bounds__(kThreads) qk_norm_rope_backward_kernel(QkBwdAr
         const int which = k / d, j = k - which * d;
         float s = 0.f;
 #pragma unroll
-        for (int ww = 0; ww < kThreads / 32; ++ww) s += red[ww][which][j];
+        for (int ww = 0; ww < kQkWarps; ++ww) s += red[ww][which][j];
         a.part[static_cast<int64_t>(blockIdx.x) * 2 * d + k] = s;
     }
 }
