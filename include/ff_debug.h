@@ -52,6 +52,20 @@ int ff_debug_qk_norm_rope(int rows, int rows_txt, int heads, int head_dim, void*
                           const void* q_scale, const void* k_scale, int grid_f, int grid_h, int grid_w,
                           const int* rope_axes, float rope_theta, cudaStream_t stream);
 
+/* Fixed-order column sums of per-chunk partials (the gradient reductions of
+ * the training pass), n jobs run as launches of up to 8.  Job i sums columns
+ * [0, ncols[i]) of the fp32 chunk rows at part + part_off[i] (row pitch
+ * ld_part[i] floats) over one or two spans of rows: span s starts at row
+ * first[2i + s] and has count[2i + s] rows (count[2i + 1] == 0: one span).
+ * per_sample[i] != 0: sample b < B sums rows first + b count .. of each span
+ * into out + out_off[i] + b ld_out[i]; else all count rows of each span into
+ * out + out_off[i].  Each sum is taken in fp64 in a fixed order that does not
+ * depend on the other jobs of the launch.  The job arrays are host memory,
+ * read before the call returns; part and out are device memory. */
+int ff_debug_reduce_chunks(int n, int B, const float* part, float* out, const int64_t* part_off,
+                           const int64_t* ld_part, const int* ncols, const int* first, const int* count,
+                           const int* per_sample, const int64_t* out_off, const int64_t* ld_out, cudaStream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

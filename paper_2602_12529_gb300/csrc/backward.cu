@@ -617,6 +617,11 @@ int reduce_chunks(const float* part, int64_t ld_part, int ncols, const ChunkSpan
 }
 
 int reduce_chunks_batch(const ReduceJob* jobs, int n, int B, cudaStream_t stream) {
+    for (int i = 0; i < n; ++i) {   // every job checked before the first launch
+        const ReduceJob& j = jobs[i];
+        if (j.ncols <= 0 || j.sp.n < 1 || j.sp.n > 2 || (j.per_sample && B <= 0))
+            return set_error(FF_ERR_INVALID_ARG, "reduce_chunks: job %d: ncols=%d spans=%d B=%d", i, j.ncols, j.sp.n, B);
+    }
     for (int at = 0; at < n; at += kMaxReduceJobs) {
         ReduceBatch rb{};
         rb.n = n - at < kMaxReduceJobs ? n - at : kMaxReduceJobs;
@@ -625,9 +630,6 @@ int reduce_chunks_batch(const ReduceJob* jobs, int n, int B, cudaStream_t stream
         int blocks = 0;
         for (int k = 0; k < rb.n; ++k) {
             const ReduceJob& j = jobs[at + k];
-            if (j.ncols <= 0 || j.sp.n < 1 || j.sp.n > 2 || (j.per_sample && B <= 0))
-                return set_error(FF_ERR_INVALID_ARG, "reduce_chunks: job %d: ncols=%d spans=%d B=%d", at + k, j.ncols,
-                                 j.sp.n, B);
             rb.job[k] = j;
             rb.blk0[k] = blocks;
             blocks += (j.ncols + 31) / 32;

@@ -3,6 +3,9 @@
 // only marshal arguments to the same launchers ff_dit_velocity uses.
 #include "../../include/ff_debug.h"
 #include "internal.h"
+#include "reduce_jobs.h"
+
+#include <vector>
 
 extern "C" {
 
@@ -184,6 +187,31 @@ int ff_debug_qk_norm_rope(int rows, int rows_txt, int heads, int head_dim, void*
     a.col[1] = heads * head_dim;
     a.rope = 1;
     return qk_norm_rope(a, stream);
+}
+
+int ff_debug_reduce_chunks(int n, int B, const float* part, float* out, const int64_t* part_off,
+                           const int64_t* ld_part, const int* ncols, const int* first, const int* count,
+                           const int* per_sample, const int64_t* out_off, const int64_t* ld_out, cudaStream_t stream) {
+    using namespace ff;
+    if (n < 0 || B < 0) return set_error(FF_ERR_INVALID_ARG, "reduce_chunks: n=%d B=%d", n, B);
+    if (n == 0) return FF_OK;
+    if (!part || !out || !part_off || !ld_part || !ncols || !first || !count || !per_sample || !out_off || !ld_out)
+        return set_error(FF_ERR_INVALID_ARG, "reduce_chunks: null argument");
+    std::vector<ReduceJob> jobs(n);
+    for (int i = 0; i < n; ++i) {
+        if (first[2 * i] < 0 || count[2 * i] <= 0 || count[2 * i + 1] < 0 || (count[2 * i + 1] > 0 && first[2 * i + 1] < 0) ||
+            part_off[i] < 0 || out_off[i] < 0 || ld_part[i] < ncols[i] || (per_sample[i] && ld_out[i] < ncols[i]))
+            return set_error(FF_ERR_INVALID_ARG, "reduce_chunks: job %d has a bad span or pitch", i);
+        ChunkSpans sp{};
+        sp.n = count[2 * i + 1] > 0 ? 2 : 1;
+        for (int k = 0; k < sp.n; ++k) {
+            sp.first[k] = first[2 * i + k];
+            sp.count[k] = count[2 * i + k];
+        }
+        jobs[i] = ReduceJob{part + part_off[i], ld_part[i], ncols[i], sp, per_sample[i] ? 1 : 0, out + out_off[i],
+                            ld_out[i]};
+    }
+    return reduce_chunks_batch(jobs.data(), n, B, stream);
 }
 
 }  // extern "C"

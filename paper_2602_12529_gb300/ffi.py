@@ -104,6 +104,8 @@ _SIGS = {
     "ff_debug_attention": ([_I, _I, _I, _I, _P, _I64, _P, _I64, _I, _P, _I64, _P, _I64, _P], _I),
     "ff_debug_ln_modulate": ([_I, _I, _P, _P, _I64, _I, _I, _I, _P, _P], _I),
     "ff_debug_qk_norm_rope": ([_I, _I, _I, _I, _P, _I64, _P, _P, _I, _I, _I, C.POINTER(_I), _F, _P], _I),
+    "ff_debug_reduce_chunks": ([_I, _I, _P, _P, C.POINTER(_I64), C.POINTER(_I64), C.POINTER(_I), C.POINTER(_I),
+                                C.POINTER(_I), C.POINTER(_I), C.POINTER(_I64), C.POINTER(_I64), _P], _I),
 }
 
 _lib = None
@@ -605,6 +607,21 @@ def ff_debug_ln_modulate(x, mods, shift_off, scale_off, tokens_per_sample, out, 
     rows, H = x.shape
     _call("ff_debug_ln_modulate", rows, H, _ptr(x), _ptr(mods), mods.shape[-1], shift_off, scale_off,
           tokens_per_sample, _ptr(out), _stream(stream))
+
+
+def ff_debug_reduce_chunks(part, out, jobs, B, stream=None):
+    """jobs: dicts with part_off, ld_part, ncols, spans [(first, count), ...
+    up to 2], per_sample, out_off, ld_out (offsets in floats from part and
+    out, both fp32 device tensors)."""
+    n = len(jobs)
+    arr = lambda t, vals: (t * max(n, 1))(*vals)
+    spans = [list(j["spans"]) + [(0, 0)] * (2 - len(j["spans"])) for j in jobs]
+    first = (_I * max(2 * n, 2))(*[f for sp in spans for f, _ in sp])
+    count = (_I * max(2 * n, 2))(*[c for sp in spans for _, c in sp])
+    _call("ff_debug_reduce_chunks", n, B, _ptr(part), _ptr(out), arr(_I64, [j["part_off"] for j in jobs]),
+          arr(_I64, [j["ld_part"] for j in jobs]), arr(_I, [j["ncols"] for j in jobs]), first, count,
+          arr(_I, [int(bool(j["per_sample"])) for j in jobs]), arr(_I64, [j["out_off"] for j in jobs]),
+          arr(_I64, [j["ld_out"] for j in jobs]), _stream(stream))
 
 
 def ff_debug_qk_norm_rope(qkv, rows_txt, heads, head_dim, q_scale, k_scale, grid, rope_axes, theta, stream=None):

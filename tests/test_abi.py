@@ -246,6 +246,29 @@ def test_training_pass_host_validation(L):
     assert L.ff_sde_logprob_backward(2, 16, 16, 16, 16, 16, 16, 16, 0, 16, 0, 16, None) == 1   # ld
 
 
+def test_reduce_chunks_host_validation(L):
+    I2 = C.c_int * 2
+    I64 = C.c_int64 * 1
+    I1 = C.c_int * 1
+    # no jobs: nothing to do, no device needed
+    assert L.ff_debug_reduce_chunks(0, 1, None, None, None, None, None, None, None, None, None, None, None) == 0
+    assert L.ff_debug_reduce_chunks(-1, 1, None, None, None, None, None, None, None, None, None, None, None) == 1
+    args = dict(part_off=I64(0), ld_part=I64(64), ncols=I1(64), first=I2(0, 0), count=I2(4, 0),
+                per_sample=I1(1), out_off=I64(0), ld_out=I64(64))
+
+    def call(B=2, part=16, out=16, **over):
+        a = dict(args, **over)
+        return L.ff_debug_reduce_chunks(1, B, part, out, a["part_off"], a["ld_part"], a["ncols"], a["first"],
+                                        a["count"], a["per_sample"], a["out_off"], a["ld_out"], None)
+    assert call(part=None) == 1
+    assert call(count=I2(0, 0)) == 1          # empty span
+    assert call(first=I2(-1, 0)) == 1         # negative first row
+    assert call(ld_part=I64(32)) == 1         # pitch below ncols
+    assert call(ld_out=I64(32)) == 1          # per-sample output pitch below ncols
+    assert call(B=0) == 1                     # per-sample job without samples
+    assert call(ncols=I1(0), ld_part=I64(0)) == 1
+
+
 def test_nft_host_validation(L):
     assert ffi.ff_nft_loss_workspace_size(4, 262144) == 4 * 65 * 2 * 8
     assert L.ff_nft_loss(2, 18, 16, 16, 16, 16, 16, 0.1, 0, 16, None, None, 16, 1 << 20, None) == 2   # D % 4
