@@ -74,7 +74,11 @@ __device__ __forceinline__ bool chunk_rows(const BwdSegs& s, int c, BwdSeg& sg, 
 // ---------------------------------------------------------------- gate
 
 // CTA = (chunk, 1024-column slab); thread t owns columns 4 (slab 256 + t) ..+3.
-__global__ void __launch_bounds__(kThreads) gate_backward_kernel(const float* g, const __nv_bfloat16* y, int64_t ld,
+// Rows go in groups of four whose g and y loads are all issued before the
+// group's arithmetic and dy stores (the loop is bound by load latency); the
+// sums still add the rows in order.
+constexpr int kGateRows = 4;
+__global__ void __launch_bounds__(kThreads, 5) gate_backward_kernel(const float* g, const __nv_bfloat16* y, int64_t ld,
                                                                   const float* mods, int64_t ld_mods, BwdSegs s, int H,
                                                                   __nv_bfloat16* dy, float* part) {
     BwdSeg sg;
@@ -84,21 +88,32 @@ __global__ void __launch_bounds__(kThreads) gate_backward_kernel(const float* g,
     if (j >= H) return;
     const float4 gt = *reinterpret_cast<const float4*>(mods + static_cast<int64_t>(b) * ld_mods + sg.col_a + j);
     float4 sy = make_float4(0.f, 0.f, 0.f, 0.f), sb = sy;
-    for (int r = r0; r < r1; ++r) {
-        const int64_t o = static_cast<int64_t>(r) * ld + j;
-        const float4 gv = __ldcs(reinterpret_cast<const float4*>(g + o));
-        const uint2 yu = *reinterpret_cast<const uint2*>(y + o);
-        const float2 y01 = unpack_bf16x2(yu.x), y23 = unpack_bf16x2(yu.y);
-        sy.x = fmaf(gv.x, y01.x, sy.x);
-        sy.y = fmaf(gv.y, y01.y, sy.y);
-        sy.z = fmaf(gv.z, y23.x, sy.z);
-        sy.w = fmaf(gv.w, y23.y, sy.w);
-        const float d0 = gv.x * gt.x, d1 = gv.y * gt.y, d2 = gv.z * gt.z, d3 = gv.w * gt.w;
-        sb.x += d0;
-        sb.y += d1;
-        sb.z += d2;
-        sb.w += d3;
-        *reinterpret_cast<uint2*>(dy + o) = make_uint2(pack_bf16x2(d0, d1), pack_bf16x2(d2, d3));
+    for (int r = r0; r < r1; r += kGateRows) {
+        float4 gv[kGateRows];
+        uint2 yu[kGateRows];
+#pragma unroll
+        for (int k = 0; k < kGateRows; ++k) {
+            if (r + k >= r1) break;
+            const int64_t o = static_cast<int64_t>(r + k) * ld + j;
+            gv[k] = __ldcs(reinterpret_cast<const float4*>(g + o));
+            yu[k] = *reinterpret_cast<const uint2*>(y + o);
+        }
+#pragma unroll
+        for (int k = 0; k < kGateRows; ++k) {
+            if (r + k >= r1) break;
+            const int64_t o = static_cast<int64_t>(r + k) * ld + j;
+            const float2 y01 = unpack_bf16x2(yu[k].x), y23 = unpack_bf16x2(yu[k].y);
+            sy.x = fmaf(gv[k].x, y01.x, sy.x);
+            sy.y = fmaf(gv[k].y, y01.y, sy.y);
+            sy.z = fmaf(gv[k].z, y23.x, sy.z);
+            sy.w = fmaf(gv[k].w, y23.y, sy.w);
+            const float d0 = gv[k].x * gt.x, d1 = gv[k].y * gt.y, d2 = gv[k].z * gt.z, d3 = gv[k].w * gt.w;
+            sb.x += d0;
+            sb.y += d1;
+            sb.z += d2;
+            sb.w += d3;
+            *reinterpret_cast<uint2*>(dy + o) = make_uint2(pack_bf16x2(d0, d1), pack_bf16x2(d2, d3));
+        }
     }
     float* p = part + static_cast<int64_t>(blockIdx.x) * 2 * H + j;
     *reinterpret_cast<float4*>(p) = sy;
