@@ -145,7 +145,7 @@ __device__ __forceinline__ float3 block_sum3(float3 v, float3* red, int lane, in
 // in the forward); mean(d n) = (sum d x - mean sum d) rstd / H.  The next
 // row's x, dh and g are loaded before this row's reductions.
 template <int PER>
-__global__ void __launch_bounds__(kThreads) ln_modulate_backward_kernel(const float* x, const float* dh, float* gx,
+__global__ void __launch_bounds__(kThreads, (PER <= 3 ? 2 : 1)) ln_modulate_backward_kernel(const float* x, const float* dh, float* gx,
                                                                          int64_t ld, const float* mods,
                                                                          int64_t ld_mods, BwdSegs s, int H,
                                                                          const __nv_bfloat16* aff_w, float* part) {
