@@ -39,7 +39,7 @@ __device__ __forceinline__ float block_sum(float v, float* red, int lane, int w)
 }
 
 template <int PER>
-__global__ void __launch_bounds__(kLnThreads) ln_modulate_kernel(LnModArgs a) {
+__global__ void __launch_bounds__(kLnThreads, (PER <= 3 ? 8 : 1)) ln_modulate_kernel(LnModArgs a) {
     __shared__ float red[2][kLnThreads / 32];
     const int row = blockIdx.x;
     const int t = threadIdx.x, lane = t & 31, w = t >> 5;
