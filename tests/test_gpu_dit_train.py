@@ -143,6 +143,20 @@ def test_wan_backward_matches_oracle(cuda, over):
     _compare(run, grad, dx, G, dx_ref)
 
 
+@pytest.mark.parametrize("hidden", [5120])
+def test_wan_backward_matches_oracle_wide_rows(cuda, hidden):
+    """Rows of 5120 columns (the WAN model's width): the LN backward runs
+    512-thread CTAs there.  Few tokens keep the fp64 oracle quick; the
+    weight scale shrinks with the width so activations stay O(1)."""
+    cfg = dict(WAN_TRAIN, hidden=hidden, heads=hidden // 128, grid=(1, 2, 4), n_txt=8, batch=2)
+    run = Run(cfg, cuda, std=0.01)
+    dv = np.random.default_rng(7).standard_normal((cfg["batch"], synth.n_img(cfg), cfg["patch_dim"])).astype(np.float32)
+    grad, dx = run.backward(dv)
+    v_ref, G, dx_ref = run.oracle(dv.astype(np.float64))
+    assert rms_rel(run.v.cpu().numpy(), v_ref) <= V_TOL
+    _compare(run, grad, dx, G, dx_ref)
+
+
 def test_wan_forward_train_equals_velocity_and_backward_is_deterministic(cuda):
     import torch
     cfg = dict(WAN_TRAIN, n_double=2)
