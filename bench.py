@@ -1,10 +1,12 @@
 #!/usr/bin/env python
 """Throughput of the rollout denoising step on GB300.
 
-One step = one DiT velocity call + one Flow-SDE step with its log-prob
-(sample mode) + the group advantage + the clipped GRPO loss, over one batch
-of the Flux-shaped double-stream block workload (H 3072, 24 x 128 heads,
-MLP 12288, 512 text + 4096 image tokens, batch 4 = one group of 4).
+Headline workload (default): the WAN-shaped video model -- 40 blocks, H 5120,
+40 x 128 heads, MLP 13824, self-attention over 32760 latent tokens (21 x 30
+x 52 grid, 3-axis RoPE) plus cross-attention to 512 text tokens, batch 1 per
+sample, groups of 8 rolled out one sample at a time.  One step = one
+velocity call + one Flow-SDE step with its log-prob (noise drawn in the
+kernel) + the group advantage over the 8 rewards + the clipped GRPO loss.
 
 Prints ONE JSON line (rank 0).  Metric: latent tokens x denoise steps / s.
   value   -- inputs resident in HBM, K steps timed with CUDA events
@@ -13,6 +15,9 @@ Prints ONE JSON line (rank 0).  Metric: latent tokens x denoise steps / s.
   roofline -- dominant kernel by device time: algorithmic work per launch
              divided by its CUDA-event launch duration in the timed region
   cpu_baseline -- the fp64 oracle on a bounded sample of the same workload
+  other_workloads -- the Flux-shaped block (batch 4), the Flux-shaped
+             rollout model (a full 10-step rollout of batch 32 per step) and
+             the Qwen-Image-shaped 60-block model, each timed on its own
 
 --impl reference times the oracle itself (the CPU reference of this path).
 Multi-GPU (torchrun): every rank runs its own independent groups; no
@@ -36,7 +41,7 @@ sys.path.insert(0, ROOT)
 
 METRIC = "latent tokens x denoise steps/sec at 1 GB300; % bf16 TC peak (DiT), % HBM BW (SDE/loss)"
 UNIT = "latent_tokens*steps/s"
-WORKLOAD = "flux_double_block"
+WORKLOAD = "wan_40"
 PROFILE_DIR = os.path.join(ROOT, "profiles")
 
 
@@ -52,7 +57,7 @@ def parse_args():
     return p.parse_args()
 
 
-def workload_desc(cfg):
+def workload_desc(cfg, rollout=False):
     f, h, w = cfg["grid"]
     if cfg.get("arch") == "wan":
         blocks = f"{cfg['n_double']} WAN blocks (self-attention + text cross-attention + FFN)"
@@ -60,10 +65,15 @@ def workload_desc(cfg):
     else:
         blocks = f"{cfg['n_double']} double + {cfg['n_single']} single MMDiT blocks"
         grid = f"{h}x{w} grid of 2x2 patches, 64-dim"
+    if rollout:
+        per = (f"per step: a {cfg['steps_run']}-step SDE rollout of the whole batch (velocity + SDE step with "
+               f"in-kernel noise + log-prob each step, every log-prob kept) + group advantage + clipped GRPO loss "
+               f"over [batch, steps]")
+    else:
+        per = ("per step: 1 velocity call + 1 SDE step with log-prob + group advantage + clipped GRPO loss")
     return (f"{cfg['name']}: {blocks}, H {cfg['hidden']}, {cfg['heads']}x{cfg['head_dim']} heads, MLP {cfg['mlp']}, "
             f"{cfg['n_txt']} text + {f * h * w} latent tokens ({grid}), batch {cfg['batch']} (groups of "
-            f"{cfg['group']}); per step: 1 velocity call + 1 SDE step with log-prob + group advantage + clipped "
-            f"GRPO loss")
+            f"{cfg['group']}); {per}")
 
 
 def device_blob(ffi, cfg, dev, seed=0):
@@ -174,12 +184,47 @@ class ClockSampler:
 # the oracle on a bounded sample (CPU baseline and the reference arm)
 # ---------------------------------------------------------------------------
 
-class OracleStep:
-    """fp64 oracle of one rollout step for ONE sample of the batch, restricted
-    to `rows` latent tokens in the last block / final layer (all tokens still
-    feed keys and values).  Rate = rows latent-token-steps per call."""
+def velocity_flops(cfg, B=1):
+    """Algorithmic FLOPs of one velocity call: 2 M N K per Linear, 4 N_q N_k d
+    per head of attention (the accounting of the measurement section)."""
+    H, F, P, L = cfg["hidden"], cfg["mlp"], cfg["patch_dim"], cfg["n_double"]
+    Nt, Ni = cfg["n_txt"], synth_n_img(cfg)
+    tf = cfg["time_freq_dim"]
+    if cfg.get("arch") == "wan":
+        per_block = 2.0 * Ni * (6 * H * H + 2 * H * F) + 2.0 * Nt * 2 * H * H \
+            + 4.0 * H * Ni * Ni + 4.0 * H * Ni * Nt
+        fixed = 2.0 * Ni * P * H * 2 + 2.0 * Nt * (cfg["txt_dim"] * H + H * H) + 2.0 * (tf * H + H * H + 6 * H * H)
+        return B * (L * per_block + fixed)
+    N = Nt + Ni
+    Ls = cfg["n_single"]
+    per_block = 2.0 * N * (4 * H * H + 2 * H * F) + 4.0 * H * N * N
+    mod_w = L * 12 * H + Ls * 3 * H + 2 * H
+    fixed = 2.0 * Ni * P * H * 2 + 2.0 * Nt * cfg["txt_dim"] * H + 2.0 * (tf * H + H * H + mod_w * H)
+    return B * ((L + Ls) * per_block + fixed)
 
-    def __init__(self, cfg, rows=None):
+
+def oracle_sample(cfg):
+    """(sample config, exact, description) of the oracle's bounded sample of a
+    workload: the whole call for one sample where that takes seconds, else
+    one block (one of each kind) of the same width, and for the video model a
+    3 x 16 x 16 latent grid; the rate is then scaled to the whole call by
+    the ratio of algorithmic FLOPs (an estimate)."""
+    if cfg.get("arch") == "wan":
+        s = dict(cfg, n_double=1, grid=(3, 16, 16), batch=1)
+        return s, False, (f"1 of {cfg['n_double']} blocks on a 3x16x16 latent grid (768 of {synth_n_img(cfg)} "
+                          f"tokens), 1 sample")
+    if cfg["n_double"] + cfg["n_single"] <= 2 and synth_n_img(cfg) * cfg["hidden"] <= 4096 * 3072:
+        return dict(cfg, batch=1), True, f"1 of {cfg['batch']} samples, whole velocity call"
+    s = dict(cfg, n_double=min(cfg["n_double"], 1), n_single=min(cfg["n_single"], 1), batch=1)
+    return s, False, (f"{s['n_double']} double + {s['n_single']} single of the {cfg['n_double']} + "
+                      f"{cfg['n_single']} blocks at full width and sequence length, 1 sample")
+
+
+class OracleStep:
+    """fp64 oracle of one rollout step (velocity + SDE step + log-prob +
+    advantage + loss) for one sample of a (sample) configuration."""
+
+    def __init__(self, cfg):
         import numpy as np
 
         import synth
@@ -192,8 +237,6 @@ class OracleStep:
         self.x = synth.initial_latent(cfg, batch=1)
         self.txt = odit.widen(synth.text_embeds(cfg, batch=1))
         self.eps = synth.step_noise(cfg, 0, batch=1)
-        n = synth.n_img(cfg)
-        self.rows = np.arange(n) if rows is None else np.arange(rows)
         self.rewards = synth.rewards(cfg["group"])
 
     def __call__(self):
@@ -203,12 +246,11 @@ class OracleStep:
         grid = osde.time_grid(cfg["sde_steps"], cfg["shift"])
         t, tn = grid[0:1], grid[1:2]
         sg = osde.sigma_flow_sde(t, cfg["eta"], cfg["t_clamp"])
-        v = self.vel(self.P, cfg, self.x, self.txt, t, img_rows=self.rows)
-        xn, lp = osde.sde_step_logprob(self.x[:, self.rows], v, t, tn, sg, eps=self.eps[:, self.rows])
+        v = self.vel(self.P, cfg, self.x, self.txt, t)
+        xn, lp = osde.sde_step_logprob(self.x, v, t, tn, sg, eps=self.eps)
         adv = ogrpo.group_advantage(self.rewards, cfg["group"], cfg["eps_adv"])
         lpn = np.full((cfg["group"], 1), lp[0])
         ogrpo.grpo_loss(lpn, lpn + 0.01, adv, cfg["clip"], cfg["clip"])
-        return len(self.rows)
 
 
 def cpu_cores():
@@ -218,13 +260,24 @@ def cpu_cores():
         return os.cpu_count()
 
 
-def oracle_rate(cfg, budget_s, rows=None):
-    """(rate in latent-token-steps/s, seconds, rows) of the oracle step."""
-    step = OracleStep(cfg, rows)
+def oracle_scale(cfg, scfg):
+    """Seconds of the whole call per second of the sample (FLOP ratio)."""
+    return velocity_flops(cfg) / velocity_flops(scfg)
+
+
+def oracle_rate(cfg):
+    """(rate in latent-token-steps/s, seconds of the sample, description)."""
+    scfg, exact, what = oracle_sample(cfg)
+    step = OracleStep(scfg)
     t0 = time.perf_counter()
-    n = step()
+    step()
     dt = time.perf_counter() - t0
-    return n / dt, dt, n
+    scale = 1.0 if exact else oracle_scale(cfg, scfg)
+    rate = synth_n_img(cfg) / (dt * scale)
+    desc = (f"{what} + SDE step + log-prob + advantage + loss, fp64 numpy, {dt:.1f} s"
+            + ("" if exact else f"; whole-call time estimated as {scale:.1f} x the sample's (algorithmic FLOP "
+                                f"ratio)"))
+    return rate, dt, desc
 
 
 def run_reference(args):
@@ -234,21 +287,9 @@ def run_reference(args):
     import synth
     cfg = synth.config(args.workload)
     n_img = synth.n_img(cfg)
-    # size the per-step sample so the whole run stays within a few minutes
-    probe_rows = min(256, n_img)
-    step = OracleStep(cfg, probe_rows)
-    t0 = time.perf_counter()
-    step()
-    t_probe = time.perf_counter() - t0
-    total = args.steps + args.warmup
-    rows = probe_rows
-    if t_probe * total < 150.0:
-        full = OracleStep(cfg, None)
-        t0 = time.perf_counter()
-        full()
-        t_full = time.perf_counter() - t0
-        if t_full * total < 200.0:
-            step, rows = full, n_img
+    scfg, exact, what = oracle_sample(cfg)
+    scale = 1.0 if exact else oracle_scale(cfg, scfg)
+    step = OracleStep(scfg)
     for _ in range(args.warmup):
         step()
     times = []
@@ -256,10 +297,11 @@ def run_reference(args):
         t0 = time.perf_counter()
         step()
         times.append(time.perf_counter() - t0)
-    dt = sum(times) / len(times)
-    value = rows / dt
-    sample = (f"1 sample of {cfg['batch']}, velocity of {rows} of {n_img} latent tokens (all tokens feed K/V) + "
-              f"SDE step + log-prob + advantage + loss, fp64 numpy")
+    dt = sum(times) / len(times) * scale
+    value = n_img / dt
+    sample = (f"{what} + SDE step + log-prob + advantage + loss, fp64 numpy, {dt / scale:.2f} s per step"
+              + ("" if exact else f"; whole-call time estimated as {scale:.1f} x the sample's (algorithmic FLOP "
+                                  f"ratio)"))
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
@@ -276,100 +318,123 @@ def run_reference(args):
 # the CUDA path
 # ---------------------------------------------------------------------------
 
-def at_config_small_kernels(ffi, dev, hbm_peak, cases, reps=100):
-    """Per-launch time of each case at the workload's sizes: `reps`
-    back-to-back calls captured in one CUDA graph, replayed three times
-    (median).  The inputs fit in L2, so these are launch- and L2-bound; the
-    HBM sweep gives the bandwidth at sizes beyond L2."""
+def graph_time_us(dev, fns, reps):
+    """Per-call microseconds of fns[0..] called round-robin `reps` times,
+    captured in one CUDA graph (no host dispatch in the timed region) and
+    replayed three times (median replay)."""
     import torch
+    for f in fns[:2]:
+        f()
+    side = torch.cuda.Stream(dev)
+    side.wait_stream(torch.cuda.current_stream(dev))
+    with torch.cuda.stream(side):
+        for f in fns[:2]:
+            f()
+    torch.cuda.current_stream(dev).wait_stream(side)
+    torch.cuda.synchronize(dev)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        for i in range(reps):
+            fns[i % len(fns)]()
+    g.replay()
+    torch.cuda.synchronize(dev)
+    ts = []
+    for _ in range(3):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        g.replay()
+        e1.record()
+        torch.cuda.synchronize(dev)
+        ts.append(e0.elapsed_time(e1))
+    del g
+    return sorted(ts)[1] * 1e3 / reps
+
+
+def at_config_small_kernels(ffi, dev, hbm_peak, cfg, rank, reps=100):
+    """Per-launch time of the memory-bound kernels at the workload's own sizes
+    (inputs L2-resident): `reps` back-to-back calls captured in one CUDA
+    graph.  These are launch- and L2-bound; the HBM sweep gives bandwidth."""
+    import torch
+    si = StepInputs(ffi, cfg, dev, rank)
+    B, G = si.B, si.G
+    D = si.x.numel() // B
+    v = torch.randn_like(si.x)
+    eps = torch.randn_like(si.x)
+    x_next = torch.empty_like(si.x)
+    logp = torch.empty((B, 1), dtype=torch.float32, device=dev)
+    lp_old = logp + 0.01
+    adv_all = torch.empty(si.n_r, dtype=torch.float32, device=dev)
+    loss = torch.zeros(1, dtype=torch.float32, device=dev)
+    grad = torch.empty((B, 1), dtype=torch.float32, device=dev)
+    ws_sde = torch.zeros(ffi.ff_sde_workspace_size(B, D), dtype=torch.uint8, device=dev)
+    ws_loss = torch.zeros(ffi.ff_grpo_loss_workspace_size(B, 1), dtype=torch.uint8, device=dev)
+    cases = {
+        "sde_step (SAMPLE, eps drawn in the kernel, log-prob)": (
+            lambda: ffi.ff_sde_step_logprob_philox(si.x, v, x_next, si.t, si.tn, si.sg, logp, 7, 0, ws=ws_sde),
+            12.0 * si.x.numel()),
+        "sde_step (SAMPLE, eps read from memory, log-prob)": (
+            lambda: ffi.ff_sde_step_logprob(si.x, v, eps, x_next, si.t, si.tn, si.sg, logp, ws=ws_sde),
+            16.0 * si.x.numel()),
+        "group_advantage": (lambda: ffi.ff_group_advantage(si.r, G, cfg["eps_adv"], adv_all), 8.0 * si.n_r),
+        "grpo_loss (+ dL/dlp)": (lambda: ffi.ff_grpo_loss(logp, lp_old, adv_all[:B], cfg["clip"], cfg["clip"], loss,
+                                                          grad, ws=ws_loss), 16.0 * logp.numel() + 4.0 * B),
+    }
     out = {}
     for name, (fn, nbytes) in cases.items():
-        fn()
-        side = torch.cuda.Stream(dev)
-        side.wait_stream(torch.cuda.current_stream(dev))
-        with torch.cuda.stream(side):
-            fn()
-        torch.cuda.current_stream(dev).wait_stream(side)
-        torch.cuda.synchronize(dev)
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g):
-            for _ in range(reps):
-                fn()
-        g.replay()
-        torch.cuda.synchronize(dev)
-        ts = []
-        for _ in range(3):
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            e0.record()
-            g.replay()
-            e1.record()
-            torch.cuda.synchronize(dev)
-            ts.append(e0.elapsed_time(e1))
-        us = sorted(ts)[1] * 1e3 / reps
+        us = graph_time_us(dev, [fn], reps)
         out[name] = {"us_per_call": us, "bytes": nbytes, "gbs": nbytes / us / 1e3,
                      "frac_of_hbm": nbytes / us / 1e3 / hbm_peak, "calls_per_graph": reps}
-        del g
     return out
 
 
 def hbm_sweep(ffi, dev, hbm_peak, l2_bytes=129 * 2 ** 20):
     """Bandwidth of the memory-bound kernels at sizes well beyond L2, with
-    enough rotating buffer sets that every launch reads from HBM."""
+    enough rotating buffer sets that every launch reads from HBM; each point
+    is a CUDA graph of back-to-back calls over the sets (no host dispatch
+    inside the timed region)."""
     import torch
 
-    def timeit(fns, reps=10):
-        for f in fns[:3]:
-            f()
-        torch.cuda.synchronize(dev)
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record()
-        for i in range(reps):
-            fns[i % len(fns)]()
-        e1.record()
-        torch.cuda.synchronize(dev)
-        return e0.elapsed_time(e1) / reps / 1e3
+    def timeit(fns, reps=12):
+        return graph_time_us(dev, fns, reps) / 1e6
 
     def nsets(nbytes):
-        return max(1, -(-4 * l2_bytes // nbytes))
+        return max(2, -(-4 * l2_bytes // nbytes))
+
+    def row(n, per, sets, sec, **kw):
+        return dict({"elements": n, "bytes": per, "gbs": per / sec / 1e9, "frac": per / sec / 1e9 / hbm_peak,
+                     "sets": sets}, **kw)
 
     out = {}
+    B = 4
+    t = torch.full((B,), 0.75, device=dev)
+    tn = torch.full((B,), 0.5, device=dev)
+    sg = torch.full((B,), 0.7, device=dev)
+    lp = torch.empty(B, device=dev)
     rows = []
     for n in (1 << 24, 1 << 26, 1 << 28):
-        B, D = 4, n // 4
+        D = n // B
         per = 16 * n
         sets = []
         for _ in range(nsets(per)):
             x = torch.randn(B, D, device=dev)
             sets.append((x, torch.randn_like(x), torch.randn_like(x), torch.empty_like(x)))
-        t = torch.full((B,), 0.75, device=dev)
-        tn = torch.full((B,), 0.5, device=dev)
-        sg = torch.full((B,), 0.7, device=dev)
-        lp = torch.empty(B, device=dev)
-        ws = torch.empty(ffi.ff_sde_workspace_size(B, D), dtype=torch.uint8, device=dev)
+        ws = torch.zeros(ffi.ff_sde_workspace_size(B, D), dtype=torch.uint8, device=dev)
         fns = [lambda s_=s_: ffi.ff_sde_step_logprob(s_[0], s_[1], s_[2], s_[3], t, tn, sg, lp, ws=ws) for s_ in sets]
-        sec = timeit(fns)
-        rows.append({"elements": n, "bytes": per, "gbs": per / sec / 1e9, "frac": per / sec / 1e9 / hbm_peak,
-                     "sets": len(sets)})
+        rows.append(row(n, per, len(sets), timeit(fns)))
         del sets
     out["sde_step"] = rows
     rows = []
     for n in (1 << 24, 1 << 26, 1 << 28):
-        B, D = 4, n // 4
+        D = n // B
         per = 12 * n
         sets = []
         for _ in range(nsets(per)):
             x = torch.randn(B, D, device=dev)
             sets.append((x, torch.randn_like(x), torch.empty_like(x)))
-        t = torch.full((B,), 0.75, device=dev)
-        tn = torch.full((B,), 0.5, device=dev)
-        sg = torch.full((B,), 0.7, device=dev)
-        lp = torch.empty(B, device=dev)
-        ws = torch.empty(ffi.ff_sde_workspace_size(B, D), dtype=torch.uint8, device=dev)
+        ws = torch.zeros(ffi.ff_sde_workspace_size(B, D), dtype=torch.uint8, device=dev)
         fns = [lambda s_=s_: ffi.ff_sde_step_logprob_philox(s_[0], s_[1], s_[2], t, tn, sg, lp, 7, 0, ws=ws)
                for s_ in sets]
-        sec = timeit(fns)
-        rows.append({"elements": n, "bytes": per, "gbs": per / sec / 1e9, "frac": per / sec / 1e9 / hbm_peak,
-                     "sets": len(sets)})
+        rows.append(row(n, per, len(sets), timeit(fns)))
         del sets
     out["sde_step_device_noise"] = rows
     rows = []
@@ -381,11 +446,9 @@ def hbm_sweep(ffi, dev, hbm_peak, l2_bytes=129 * 2 ** 20):
             a = torch.randn(Bq, T, device=dev)
             sets.append((a, a + 0.01 * torch.randn_like(a), torch.randn(Bq, device=dev), torch.empty_like(a)))
         loss = torch.empty(1, device=dev)
-        ws = torch.empty(ffi.ff_grpo_loss_workspace_size(Bq, T), dtype=torch.uint8, device=dev)
+        ws = torch.zeros(ffi.ff_grpo_loss_workspace_size(Bq, T), dtype=torch.uint8, device=dev)
         fns = [lambda s_=s_: ffi.ff_grpo_loss(s_[0], s_[1], s_[2], 0.2, 0.2, loss, s_[3], ws=ws) for s_ in sets]
-        sec = timeit(fns)
-        rows.append({"elements": n, "bytes": per, "gbs": per / sec / 1e9, "frac": per / sec / 1e9 / hbm_peak,
-                     "sets": len(sets)})
+        rows.append(row(n, per, len(sets), timeit(fns)))
         del sets
     out["grpo_loss"] = rows
     rows = []
@@ -393,37 +456,33 @@ def hbm_sweep(ffi, dev, hbm_peak, l2_bytes=129 * 2 ** 20):
         per = 8 * n
         sets = [(torch.rand(n, device=dev), torch.empty(n, device=dev)) for _ in range(nsets(per))]
         fns = [lambda s_=s_: ffi.ff_group_advantage(s_[0], 16, 1e-4, s_[1]) for s_ in sets]
-        sec = timeit(fns)
-        rows.append({"elements": n, "group": 16, "bytes": per, "gbs": per / sec / 1e9,
-                     "frac": per / sec / 1e9 / hbm_peak, "sets": len(sets)})
+        rows.append(row(n, per, len(sets), timeit(fns), group=16))
         del sets
     out["group_advantage"] = rows
     for name, per_elem in (("forward_process", 12), ("awm_loss", 16)):
         rows = []
         for n in (1 << 24, 1 << 26, 1 << 28):
-            B, D = 4, n // 4
+            D = n // B
             per = per_elem * n
             sets = []
             for _ in range(nsets(per)):
                 x = torch.randn(B, D, device=dev)
                 sets.append((x, torch.randn_like(x), torch.randn_like(x), torch.empty_like(x)))
-            t = torch.full((B,), 0.6, device=dev)
+            tt = torch.full((B,), 0.6, device=dev)
             adv = torch.randn(B, device=dev)
             loss = torch.empty(1, device=dev)
             if name == "forward_process":
-                fns = [lambda s_=s_: ffi.ff_forward_process(s_[0], s_[1], t, s_[3]) for s_ in sets]
+                fns = [lambda s_=s_: ffi.ff_forward_process(s_[0], s_[1], tt, s_[3]) for s_ in sets]
             else:
                 ws = torch.empty(ffi.ff_awm_loss_workspace_size(B, D), dtype=torch.uint8, device=dev)
                 fns = [lambda s_=s_: ffi.ff_awm_loss(s_[0], s_[1], s_[2], adv, ffi.FF_AWM_MEAN, loss, s_[3], ws=ws)
                        for s_ in sets]
-            sec = timeit(fns)
-            rows.append({"elements": n, "bytes": per, "gbs": per / sec / 1e9, "frac": per / sec / 1e9 / hbm_peak,
-                         "sets": len(sets)})
+            rows.append(row(n, per, len(sets), timeit(fns)))
             del sets
         out[name] = rows
     rows = []
     for n in (1 << 24, 1 << 26, 1 << 28):
-        B, D = 4, n // 4
+        D = n // B
         per = 20 * n
         sets = []
         for _ in range(nsets(per)):
@@ -434,9 +493,7 @@ def hbm_sweep(ffi, dev, hbm_peak, l2_bytes=129 * 2 ** 20):
         ws = torch.empty(ffi.ff_nft_loss_workspace_size(B, D), dtype=torch.uint8, device=dev)
         fns = [lambda s_=s_: ffi.ff_nft_loss(s_[0], s_[1], s_[2], s_[3], r, 0.1, ffi.FF_AWM_MEAN, loss, s_[4], ws=ws)
                for s_ in sets]
-        sec = timeit(fns)
-        rows.append({"elements": n, "bytes": per, "gbs": per / sec / 1e9, "frac": per / sec / 1e9 / hbm_peak,
-                     "sets": len(sets)})
+        rows.append(row(n, per, len(sets), timeit(fns)))
         del sets
     out["nft_loss"] = rows
     torch.cuda.empty_cache()
@@ -581,8 +638,8 @@ def train_step(args, ffi, model, cfg, dev, x, txt, t, tn, sg, x_next, lp_old, ad
     lp = torch.empty((B, 1), dtype=torch.float32, device=dev)
     glp = torch.empty((B, 1), dtype=torch.float32, device=dev)
     loss = torch.empty(1, dtype=torch.float32, device=dev)
-    ws_sde = torch.empty(ffi.ff_sde_workspace_size(B, D), dtype=torch.uint8, device=dev)
-    ws_loss = torch.empty(ffi.ff_grpo_loss_workspace_size(B, 1), dtype=torch.uint8, device=dev)
+    ws_sde = torch.zeros(ffi.ff_sde_workspace_size(B, D), dtype=torch.uint8, device=dev)
+    ws_loss = torch.zeros(ffi.ff_grpo_loss_workspace_size(B, 1), dtype=torch.uint8, device=dev)
 
     def step():
         model.ff_dit_forward_train(x, txt, t, v, ws_t)
@@ -628,76 +685,6 @@ def train_step(args, ffi, model, cfg, dev, x, txt, t, tn, sg, x_next, lp_old, ad
             "peak": f"{tc_burst} TFLOP/s ({src} bf16 dense burst)"}
 
 
-def wan_train(args, ffi, dev, timed, blocks=1, recompute=False):
-    """The WAN-style model's training pass at full width (H 5120, 40 x 128
-    heads, MLP 13824; batch 1 of 32760 latent + 512 text tokens): the
-    training forward and the DiT backward from a random dL/dv to every
-    weight, on `blocks` blocks (the whole model is 40).  With `recompute`
-    the forward keeps only the block inputs and the backward re-runs every
-    block (one more forward of the blocks, not counted as work).  Weights
-    N(0, 0.02), norm scales 1, drawn on the device.  Algorithmic FLOPs: 3x
-    the forward's GEMM FLOPs (forward, input and weight gradients) + 3.5x
-    its attention FLOPs (forward 4 B h N_q N_k d, backward 10 B h N_q N_k
-    d), for the self-attention and the cross-attention."""
-    import numpy as np
-    import torch
-    import synth
-    cfg = dict(synth.config("wan_40"), n_double=blocks, batch=1)
-    B, H, F, P = 1, cfg["hidden"], cfg["mlp"], cfg["patch_dim"]
-    Nt, Ni = cfg["n_txt"], synth_n_img(cfg)
-    specs, total = ffi.ff_dit_weight_layout(cfg)
-    free, _ = torch.cuda.mem_get_info(dev)
-    if 6 * total > 0.8 * free:
-        return {"skipped": f"{total / 1e9:.1f} G parameters: weights and fp32 gradients exceed the free memory"}
-    g = torch.Generator(device=dev)
-    g.manual_seed(11)
-    blob = torch.empty(total, dtype=torch.bfloat16, device=dev)
-    for i in range(0, total, 1 << 28):          # drawn in pieces (no fp32 copy of the whole blob)
-        n = min(1 << 28, total - i)
-        blob[i:i + n] = (torch.randn(n, generator=g, device=dev) * 0.02).to(torch.bfloat16)
-    for name, off, shape in specs:
-        if name.endswith("scale"):
-            blob[off:off + int(np.prod(shape))] = 1.0
-    model = ffi.Dit(cfg, blob)
-    if recompute:
-        model.set_train_recompute(True)
-    need = model.train_workspace_size(B)
-    free, _ = torch.cuda.mem_get_info(dev)
-    if need + 4 * total > 0.9 * free:
-        model.close()
-        return {"skipped": f"training workspace {need / 1e9:.1f} GB exceeds the free device memory"}
-    ws = torch.empty(need, dtype=torch.uint8, device=dev)
-    grad = torch.empty(total, dtype=torch.float32, device=dev)
-    x = torch.randn(B, Ni, P, generator=g, device=dev)
-    txt = torch.randn(B * Nt, cfg["txt_dim"], generator=g, device=dev).to(torch.bfloat16)
-    t = torch.full((B,), 0.9, device=dev)
-    v, dv = torch.empty_like(x), torch.randn(B, Ni, P, generator=g, device=dev)
-
-    def step():
-        model.ff_dit_forward_train(x, txt, t, v, ws)
-        model.ff_dit_backward(txt, dv, grad, ws)
-
-    warm = 1 if blocks > 1 else max(2, args.warmup)
-    for _ in range(warm):
-        step()
-    k = 2 if blocks > 1 else max(2, min(args.steps, 5))
-    ms = timed(step, k) / k
-    per_block = 2.0 * B * Ni * (6 * H * H + 2 * H * F) + 2.0 * B * Nt * 2 * H * H
-    gemm = blocks * per_block + 2.0 * B * Ni * 2 * P * H + 2.0 * B * Nt * (cfg["txt_dim"] * H + H * H)
-    attn = blocks * 4.0 * B * H * Ni * (Ni + Nt)
-    flops = 3.0 * gemm + 3.5 * attn
-    _, tc_burst, tc_sust, src = load_peaks()
-    model.close()
-    return {"ms_per_step": ms, "value": B * Ni / (ms / 1e3), "unit": UNIT,
-            "what": f"WAN-style model at full width, {blocks} of its 40 blocks "
-                    f"({total / 1e9:.2f} G parameters): training forward + DiT backward from dL/dv to every weight, "
-                    f"batch 1, 32760 latent + 512 text tokens" + (", block activations recomputed" if recompute else ""),
-            "tflops": flops / (ms / 1e3) / 1e12, "frac": flops / (ms / 1e3) / 1e12 / tc_burst,
-            "frac_vs_sustained": flops / (ms / 1e3) / 1e12 / tc_sust if tc_sust else None,
-            "algorithmic_flops": flops, "workspace_gb": need / 1e9, "parameters": total,
-            "peak": f"{tc_burst} TFLOP/s ({src} bf16 dense burst)"}
-
-
 def synth_n_img(cfg):
     import synth
     return synth.n_img(cfg)
@@ -730,13 +717,225 @@ def whole_job_rate(world: int, units_per_rank_step: float, ms_step: float) -> fl
     return world * units_per_rank_step / (ms_step / 1e3)
 
 
+def make_model(ffi, cfg, dev):
+    """(handle, weight blob, parameter count) of a random-init model."""
+    import synth
+    from paper_2602_12529_gb300 import weights
+    _, n_params = ffi.ff_dit_weight_layout(cfg)
+    if n_params > 2e9:
+        blob = device_blob(ffi, cfg, dev)
+    else:
+        blob = weights.pack(cfg, lambda n, s: synth.weight(n, s, synth.weight_kind(n), 0), dev)
+    return ffi.Dit(cfg, blob), blob, n_params
+
+
+def kernel_table(ffi, step, steps, timed, cfg):
+    """Per-kernel CUDA-event durations of `steps` calls of step():
+    {name: [launches, ms, flops, bytes]} and the launch count."""
+    per_step = 16 * (cfg["n_double"] + cfg["n_single"]) * max(1, cfg.get("steps_run", 1)) + 64
+    ffi.ff_prof_enable(per_step * steps + 64)
+    timed(step, steps)
+    recs = ffi.ff_prof_records()
+    ffi.ff_prof_disable()
+    kern = {}
+    for name, ms, fl, by in recs:
+        k = kern.setdefault(name, [0, 0.0, 0.0, 0.0])
+        k[0] += 1
+        k[1] += ms
+        k[2] += fl
+        k[3] += by
+    return kern, len(recs)
+
+
+def roofline_of(kern, name, workload):
+    """Roofline object of one kernel from its per-launch algorithmic work and
+    CUDA-event durations (tensor-bound if it counts FLOPs, else HBM)."""
+    n, ms, fl, by = kern[name]
+    total = sum(k[1] for k in kern.values())
+    hbm, tc_burst, tc_sust, peak_src = load_peaks()
+    if fl > 0:
+        ach = fl / n / (ms / n / 1e3) / 1e12
+        return {"bound": "tensor", "achieved": ach, "peak": tc_burst, "unit": "TFLOP/s",
+                "frac": ach / tc_burst, "frac_vs_sustained": ach / tc_sust if tc_sust else None,
+                "traffic": profile_traffic(name, workload), "kernel": name, "launches": n,
+                "share_of_device_time": ms / total, "algorithmic_per_launch": fl / n,
+                "peak_source": f"{peak_src} bf16 dense (burst)"}
+    ach = by / n / (ms / n / 1e3) / 1e9
+    return {"bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s", "frac": ach / hbm,
+            "traffic": profile_traffic(name, workload), "kernel": name, "launches": n,
+            "share_of_device_time": ms / total, "algorithmic_per_launch": by / n,
+            "peak_source": f"{peak_src} HBM copy"}
+
+
+def breakdown_of(kern, steps):
+    total = sum(k[1] for k in kern.values())
+    return {k: {"launches": v[0] // steps, "ms_per_step": v[1] / steps, "share": v[1] / total}
+            for k, v in sorted(kern.items(), key=lambda kv: -kv[1][1])}
+
+
+class StepInputs:
+    """Device inputs of one rollout step of a workload (seeded, synthetic) and
+    the host copies they came from."""
+
+    def __init__(self, ffi, cfg, dev, rank):
+        import numpy as np
+        import torch
+
+        import synth
+        B, G = cfg["batch"], cfg["group"]
+        self.B, self.G = B, G
+        tgrid, sig = ffi.ff_sde_schedule(ffi.FF_SCHED_FLOW_SDE, cfg["sde_steps"], cfg["shift"], cfg["eta"],
+                                         cfg["t_clamp"])
+        self.tgrid, self.sig = tgrid, sig
+        seed = rank_seed(rank)
+        self.noise_seed = 100 + seed
+        self.h = {
+            "x": synth.initial_latent(cfg, seed=2 + seed),
+            "txt": synth.text_embeds(cfg, seed=1 + seed).view(np.int16),
+            "t": np.full(B, tgrid[0], np.float32),
+            "tn": np.full(B, tgrid[1], np.float32),
+            "sg": np.full(B, sig[0], np.float32),
+        }
+        # rewards of whole groups (a WAN group of 8 is rolled out one sample
+        # at a time, so it can be larger than the batch)
+        self.n_r = -(-B // G) * G
+        self.h["r"] = synth.rewards(self.n_r, seed=7 + seed)
+        self.h_jitter = synth.logprob_jitter((B, 1), seed=9 + seed)
+
+        def dev_t(a):
+            return torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+        self.x, self.t, self.tn, self.sg, self.r = (dev_t(self.h[k]) for k in ("x", "t", "tn", "sg", "r"))
+        self.txt = dev_t(self.h["txt"]).view(torch.bfloat16)
+        self.jitter = dev_t(self.h_jitter)
+
+
+def measure_step_workload(args, ffi, cfg, dev, rank, world, timed, steps, warmup, keep_model=False):
+    """One rollout step of `cfg` (velocity + SDE step with in-kernel noise and
+    its log-prob + group advantage + clipped GRPO loss with dL/dlp): time per
+    step, kernel breakdown and the dominant kernel's roofline."""
+    import torch
+    import synth
+    model, blob, n_params = make_model(ffi, cfg, dev)
+    si = StepInputs(ffi, cfg, dev, rank)
+    B, G = si.B, si.G
+    D = si.x.numel() // B
+    v = torch.empty_like(si.x)
+    x_next = torch.empty_like(si.x)
+    logp = torch.empty((B, 1), dtype=torch.float32, device=dev)
+    lp_old = torch.empty((B, 1), dtype=torch.float32, device=dev)
+    adv_all = torch.empty(si.n_r, dtype=torch.float32, device=dev)
+    adv = adv_all[:B]
+    loss = torch.zeros(1, dtype=torch.float32, device=dev)
+    grad = torch.empty((B, 1), dtype=torch.float32, device=dev)
+    ws = torch.empty(model.workspace_size(B), dtype=torch.uint8, device=dev)
+    ws_sde = torch.zeros(ffi.ff_sde_workspace_size(B, D), dtype=torch.uint8, device=dev)
+    ws_loss = torch.zeros(ffi.ff_grpo_loss_workspace_size(B, 1), dtype=torch.uint8, device=dev)
+    # old log-probs of the (synthetic) rollout policy: new + N(0, 0.01^2)
+    model.ff_dit_velocity(si.x, si.txt, si.t, v, ws)
+    ffi.ff_sde_step_logprob_philox(si.x, v, x_next, si.t, si.tn, si.sg, logp, si.noise_seed, 0, ws=ws_sde)
+    torch.add(logp, si.jitter, out=lp_old)
+
+    def step(xi=si.x, txti=si.txt, ti=si.t, tni=si.tn, sgi=si.sg, ri=si.r, lpo=lp_old, xo=x_next, lpn=logp,
+             lo=loss):
+        model.ff_dit_velocity(xi, txti, ti, v, ws)
+        ffi.ff_sde_step_logprob_philox(xi, v, xo, ti, tni, sgi, lpn, si.noise_seed, 0, ws=ws_sde)
+        ffi.ff_group_advantage(ri, G, cfg["eps_adv"], adv_all)
+        ffi.ff_grpo_loss(lpn, lpo, adv, cfg["clip"], cfg["clip"], lo, grad, ws=ws_loss)
+
+    for _ in range(warmup):
+        step()
+    torch.cuda.synchronize(dev)
+    ms_step = timed(step, steps) / steps
+    n_img = synth.n_img(cfg)
+    prof_steps = max(1, min(steps, 5))
+    kern, launches = kernel_table(ffi, step, prof_steps, timed, cfg)
+    dominant = max(kern, key=lambda k: kern[k][1])
+    dit_flops = sum(k[2] for k in kern.values()) / prof_steps
+    _, tc_burst, _, _ = load_peaks()
+    out = {"workload": workload_desc(cfg), "ms_per_step": ms_step,
+           "value": whole_job_rate(world, B * n_img, ms_step), "unit": UNIT, "steps": steps, "warmup": warmup,
+           "dit_tflops": dit_flops / (ms_step / 1e3) / 1e12,
+           "dit_frac_of_burst": dit_flops / (ms_step / 1e3) / 1e12 / tc_burst,
+           "roofline": roofline_of(kern, dominant, cfg["name"]),
+           "secondary_rooflines": {k: roofline_of(kern, k, cfg["name"]) for k in ("gemm_bf16", "attention",
+                                                                                   "sde_step", "grpo_loss")
+                                   if k in kern and k != dominant},
+           "kernel_breakdown": breakdown_of(kern, prof_steps),
+           "gpu_launches_per_step": launches // prof_steps,
+           "weights_gb": 2 * n_params / 1e9, "workspace_gb": ws.numel() / 1e9}
+    ctx = {"model": model, "blob": blob, "si": si, "step": step, "v": v, "x_next": x_next, "logp": logp,
+           "lp_old": lp_old, "loss": loss, "adv": adv, "adv_all": adv_all, "grad": grad, "ws": ws,
+           "ws_sde": ws_sde, "ws_loss": ws_loss, "launches_per_step": launches // prof_steps,
+           "dit_flops": dit_flops, "n_params": n_params}
+    if not keep_model:
+        model.close()
+        del ctx, blob
+        torch.cuda.empty_cache()
+        return out, None
+    return out, ctx
+
+
+def measure_rollout_workload(ffi, cfg, dev, rank, world, timed, steps=3, warmup=1):
+    """The configured trajectory sampling of a workload: S denoise steps
+    (velocity + SDE step with in-kernel noise + log-prob, all S log-probs
+    kept) from x_T for the whole batch (ff_rollout_philox), then the group
+    advantage and the clipped GRPO loss over [B, S] with dL/dlp."""
+    import torch
+    import synth
+    model, blob, n_params = make_model(ffi, cfg, dev)
+    si = StepInputs(ffi, cfg, dev, rank)
+    B, G, S = si.B, si.G, cfg["steps_run"]
+    t = torch.tensor(si.tgrid[:S + 1], dtype=torch.float32, device=dev)
+    sg = torch.tensor(si.sig[:S], dtype=torch.float32, device=dev)
+    x = torch.empty_like(si.x)
+    logp = torch.empty((B, S), dtype=torch.float32, device=dev)
+    lp_old = torch.empty_like(logp)
+    adv = torch.empty(si.n_r, dtype=torch.float32, device=dev)
+    loss = torch.zeros(1, dtype=torch.float32, device=dev)
+    grad = torch.empty_like(logp)
+    ws = torch.empty(model.rollout_workspace_size(B, S), dtype=torch.uint8, device=dev)
+    ws_loss = torch.zeros(ffi.ff_grpo_loss_workspace_size(B, S), dtype=torch.uint8, device=dev)
+    g = torch.Generator(device=dev)
+    g.manual_seed(9 + rank_seed(rank))
+    x.copy_(si.x)
+    model.ff_rollout_philox(x, si.txt, t, sg, si.noise_seed, logp, ws=ws)
+    torch.add(logp, 0.01 * torch.randn(logp.shape, generator=g, device=dev), out=lp_old)
+
+    def step():
+        x.copy_(si.x)                       # every rollout starts from x_T
+        model.ff_rollout_philox(x, si.txt, t, sg, si.noise_seed, logp, ws=ws)
+        ffi.ff_group_advantage(si.r, G, cfg["eps_adv"], adv)
+        ffi.ff_grpo_loss(logp, lp_old, adv[:B], cfg["clip"], cfg["clip"], loss, grad, ws=ws_loss)
+
+    for _ in range(warmup):
+        step()
+    torch.cuda.synchronize(dev)
+    ms = timed(step, steps) / steps
+    kern, launches = kernel_table(ffi, step, 1, timed, cfg)
+    dominant = max(kern, key=lambda k: kern[k][1])
+    dit_flops = sum(k[2] for k in kern.values())
+    _, tc_burst, _, _ = load_peaks()
+    n_img = synth.n_img(cfg)
+    out = {"workload": workload_desc(cfg, rollout=True), "ms_per_step": ms,
+           "value": whole_job_rate(world, B * n_img * S, ms), "unit": UNIT, "steps": steps, "warmup": warmup,
+           "denoise_steps_per_rollout": S,
+           "dit_tflops": dit_flops / (ms / 1e3) / 1e12, "dit_frac_of_burst": dit_flops / (ms / 1e3) / 1e12 / tc_burst,
+           "roofline": roofline_of(kern, dominant, cfg["name"]),
+           "kernel_breakdown": breakdown_of(kern, 1), "gpu_launches_per_step": launches,
+           "weights_gb": 2 * n_params / 1e9}
+    model.close()
+    del blob, ws
+    torch.cuda.empty_cache()
+    return out
+
+
 def run_ours(args):
     import numpy as np
     import torch
     import torch.distributed as dist
 
     import synth
-    from paper_2602_12529_gb300 import build, ffi, weights
+    from paper_2602_12529_gb300 import build, ffi
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -750,69 +949,7 @@ def run_ours(args):
     if world > 1:
         dist.barrier()
     ffi.lib()
-
-    cfg = synth.config(args.workload)
-    B, G, Nt, Ni, P = cfg["batch"], cfg["group"], cfg["n_txt"], synth.n_img(cfg), cfg["patch_dim"]
-    D = Ni * P
-    steps_per_step = 1
-
-    _, n_params = ffi.ff_dit_weight_layout(cfg)
-    if n_params > 2e9:
-        blob = device_blob(ffi, cfg, dev)
-    else:
-        blob = weights.pack(cfg, lambda n, s: synth.weight(n, s, synth.weight_kind(n), 0), dev)
-    model = ffi.Dit(cfg, blob)
-    tgrid, sig = ffi.ff_sde_schedule(ffi.FF_SCHED_FLOW_SDE, cfg["sde_steps"], cfg["shift"], cfg["eta"],
-                                     cfg["t_clamp"])
-    seed = rank_seed(rank)
-    h_x = synth.initial_latent(cfg, seed=2 + seed)
-    h_txt = synth.text_embeds(cfg, seed=1 + seed).view(np.int16)
-    h_eps = synth.step_noise(cfg, 0, seed=100 + seed)
-    h_t = np.full(B, tgrid[0], np.float32)
-    h_tn = np.full(B, tgrid[1], np.float32)
-    h_sg = np.full(B, sig[0], np.float32)
-    # rewards of whole groups (a WAN group of 8 is rolled out one sample at a
-    # time, so it can be larger than the batch); the loss uses the batch's own
-    n_r = -(-B // G) * G
-    h_r = synth.rewards(n_r, seed=7 + seed)
-    h_lpold = synth.logprob_jitter((B, 1), seed=9 + seed)   # + lp_new, added on device below
-
-    def dev_t(a, dtype=None):
-        t = torch.from_numpy(np.ascontiguousarray(a)).to(dev)
-        return t.view(dtype) if dtype is not None else t
-
-    x, txt, eps = dev_t(h_x), dev_t(h_txt, torch.bfloat16), dev_t(h_eps)
-    t, tn, sg = dev_t(h_t), dev_t(h_tn), dev_t(h_sg)
-    rewards, jitter = dev_t(h_r), dev_t(h_lpold)
-    v = torch.empty_like(x)
-    x_next = torch.empty_like(x)
-    logp = torch.empty((B, 1), dtype=torch.float32, device=dev)
-    lp_old = torch.empty((B, 1), dtype=torch.float32, device=dev)
-    adv_all = torch.empty(n_r, dtype=torch.float32, device=dev)
-    adv = adv_all[:B]
-    loss = torch.zeros(1, dtype=torch.float32, device=dev)
-    grad = torch.empty((B, 1), dtype=torch.float32, device=dev)
-    ws = torch.empty(model.workspace_size(B), dtype=torch.uint8, device=dev)
-    ws_sde = torch.empty(ffi.ff_sde_workspace_size(B, D), dtype=torch.uint8, device=dev)
-    ws_loss = torch.empty(ffi.ff_grpo_loss_workspace_size(B, 1), dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
-
-    # old log-probs of the (synthetic) rollout policy: new + N(0, 0.01^2)
-    model.ff_dit_velocity(x, txt, t, v, ws)
-    noise_seed = 100 + seed          # the step's noise: drawn in the SDE kernel from (seed, step 0)
-    ffi.ff_sde_step_logprob_philox(x, v, x_next, t, tn, sg, logp, noise_seed, 0, ws=ws_sde)
-    torch.add(logp, jitter, out=lp_old)
-
-    def step(xi=x, txti=txt, ti=t, tni=tn, sgi=sg, ri=rewards, lpo=lp_old, xo=x_next, lpn=logp, lo=loss):
-        model.ff_dit_velocity(xi, txti, ti, v, ws)
-        ffi.ff_sde_step_logprob_philox(xi, v, xo, ti, tni, sgi, lpn, noise_seed, 0, ws=ws_sde)
-        ffi.ff_group_advantage(ri, G, cfg["eps_adv"], adv_all)
-        ffi.ff_grpo_loss(lpn, lpo, adv, cfg["clip"], cfg["clip"], lo, grad, ws=ws_loss)
-
-    clocks = ClockSampler(local) if rank == 0 else None
-    for _ in range(args.warmup):
-        step()
-    torch.cuda.synchronize(dev)
 
     def timed(fn, k):
         if world > 1:
@@ -829,50 +966,13 @@ def run_ours(args):
             dist.barrier()
         return ms
 
-    ms_total = timed(step, args.steps)
-    ms_step = ms_total / args.steps
-    tokens_per_step = B * Ni * steps_per_step
-    value = whole_job_rate(world, tokens_per_step, ms_step)
-
-    # ---- per-kernel CUDA-event durations over the same K steps
-    # launches per step: a few per block plus the fixed ones, with headroom
-    per_step = 16 * (cfg["n_double"] + cfg["n_single"]) + 64
-    ffi.ff_prof_enable(per_step * args.steps + 64)
-    timed(step, args.steps)
-    recs = ffi.ff_prof_records()
-    ffi.ff_prof_disable()
-    kern = {}
-    for name, ms, fl, by in recs:
-        k = kern.setdefault(name, [0, 0.0, 0.0, 0.0])
-        k[0] += 1
-        k[1] += ms
-        k[2] += fl
-        k[3] += by
-    launches = len(recs)
-    prof_total = sum(k[1] for k in kern.values())
-    hbm, tc_burst, tc_sust, peak_src = load_peaks()
-
-    def roof(name):
-        n, ms, fl, by = kern[name]
-        if fl > 0:
-            ach = fl / n / (ms / n / 1e3) / 1e12
-            return {"bound": "tensor", "achieved": ach, "peak": tc_burst, "unit": "TFLOP/s",
-                    "frac": ach / tc_burst, "frac_vs_sustained": ach / tc_sust if tc_sust else None,
-                    "traffic": profile_traffic(name, args.workload), "kernel": name, "launches": n,
-                    "share_of_device_time": ms / prof_total, "algorithmic_per_launch": fl / n,
-                    "peak_source": f"{peak_src} bf16 dense (burst)"}
-        ach = by / n / (ms / n / 1e3) / 1e9
-        return {"bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s", "frac": ach / hbm,
-                "traffic": profile_traffic(name, args.workload), "kernel": name, "launches": n,
-                "share_of_device_time": ms / prof_total, "algorithmic_per_launch": by / n,
-                "peak_source": f"{peak_src} HBM copy"}
-
-    dominant = max(kern, key=lambda k: kern[k][1])
-    roofline = roof(dominant)
-    breakdown = {k: {"launches": v[0], "ms_per_step": v[1] / args.steps, "share": v[1] / prof_total}
-                 for k, v in sorted(kern.items(), key=lambda kv: -kv[1][1])}
-    dit_flops = sum(v[2] for v in kern.values()) / args.steps
-    secondary = {k: roof(k) for k in ("attention", "sde_step") if k in kern}
+    cfg = synth.config(args.workload)
+    B, G, Nt, Ni = cfg["batch"], cfg["group"], cfg["n_txt"], synth.n_img(cfg)
+    clocks = ClockSampler(local) if rank == 0 else None
+    head, ctx = measure_step_workload(args, ffi, cfg, dev, rank, world, timed, args.steps, args.warmup,
+                                      keep_model=True)
+    model, si, step = ctx["model"], ctx["si"], ctx["step"]
+    ms_step = head["ms_per_step"]
 
     # ---- end to end through the public API with host inputs: every step
     # copies its inputs in from pinned host memory and its results (x_next,
@@ -882,9 +982,9 @@ def run_ours(args):
     # is reported beside it.
     from paper_2602_12529_gb300.pipeline import HostFedPipeline
     pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
-    h_in = {"x": pin(h_x), "txt": pin(h_txt), "t": pin(h_t), "tn": pin(h_tn), "sg": pin(h_sg),
-            "r": pin(h_r), "lpo": lp_old.cpu().pin_memory()}
-    h_out = [{"x_next": torch.empty(x.shape, dtype=torch.float32).pin_memory(),
+    h_in = {k: pin(si.h[k]) for k in ("x", "txt", "t", "tn", "sg", "r")}
+    h_in["lpo"] = ctx["lp_old"].cpu().pin_memory()
+    h_out = [{"x_next": torch.empty(si.x.shape, dtype=torch.float32).pin_memory(),
               "logp": torch.empty((B, 1), dtype=torch.float32).pin_memory(),
               "loss": torch.empty(1, dtype=torch.float32).pin_memory()} for _ in range(2)]
     h2d = sum(a.numel() * a.element_size() for a in h_in.values())
@@ -894,13 +994,14 @@ def run_ours(args):
         step(i["x"], i["txt"].view(torch.bfloat16), i["t"], i["tn"], i["sg"], i["r"], i["lpo"],
              o["x_next"], o["logp"], o["loss"])
 
-    like_in = {"x": x, "txt": txt.view(torch.int16), "t": t, "tn": tn, "sg": sg, "r": rewards,
-               "lpo": lp_old}
-    pipe = HostFedPipeline(dev, like_in, {"x_next": x_next, "logp": logp, "loss": loss}, e2e_body)
-    K = args.steps
+    like_in = {"x": si.x, "txt": si.txt.view(torch.int16), "t": si.t, "tn": si.tn, "sg": si.sg, "r": si.r,
+               "lpo": ctx["lp_old"]}
+    pipe = HostFedPipeline(dev, like_in, {"x_next": ctx["x_next"], "logp": ctx["logp"], "loss": ctx["loss"]},
+                           e2e_body)
+    K_e2e = args.steps if ms_step < 200 else max(3, min(args.steps, 8))
     pipe.run([h_in] * 2, h_out)
-    ms_e2e = timed(lambda: pipe.run([h_in] * K, [h_out[k % 2] for k in range(K)]), 1) / K
-    e2e_value = whole_job_rate(world, tokens_per_step, ms_e2e)
+    ms_e2e = timed(lambda: pipe.run([h_in] * K_e2e, [h_out[k % 2] for k in range(K_e2e)]), 1) / K_e2e
+    e2e_value = whole_job_rate(world, B * Ni, ms_e2e)
 
     def e2e_serial():
         i = pipe.ins[0]
@@ -911,68 +1012,73 @@ def run_ours(args):
             h_.copy_(pipe.outs[0][name], non_blocking=True)
 
     e2e_serial()
-    ms_e2e_serial = timed(e2e_serial, K) / K
-    awm = awm_step(args, ffi, model, cfg, dev, x, txt, eps, rewards, timed, world)
-    train = train_step(args, ffi, model, cfg, dev, x, txt, t, tn, sg, x_next, lp_old, adv, dit_flops, timed, world)
-    at_cfg = None
-    if rank == 0 and not args.no_sweep:
-        # the memory-bound kernels at the workload's own sizes (inputs L2-resident):
-        # 100 back-to-back launches captured in one CUDA graph, per-launch time
-        sde_bytes = 16.0 * x.numel()
-        at_cfg = at_config_small_kernels(ffi, dev, hbm, {
-            "sde_step (SAMPLE, eps drawn in the kernel, log-prob)": (
-                lambda: ffi.ff_sde_step_logprob_philox(x, v, x_next, t, tn, sg, logp, noise_seed, 0, ws=ws_sde),
-                12.0 * x.numel()),
-            "sde_step (SAMPLE, eps read from memory, log-prob)": (
-                lambda: ffi.ff_sde_step_logprob(x, v, eps, x_next, t, tn, sg, logp, ws=ws_sde), sde_bytes),
-            "group_advantage": (lambda: ffi.ff_group_advantage(rewards, G, cfg["eps_adv"], adv_all),
-                                8.0 * rewards.numel()),
-            "grpo_loss (+ dL/dlp)": (lambda: ffi.ff_grpo_loss(logp, lp_old, adv, cfg["clip"], cfg["clip"], loss, grad,
-                                                              ws=ws_loss), 16.0 * logp.numel() + 4.0 * B),
-        })
-    bwd = backward_kernels(args, ffi, cfg, dev) if rank == 0 and not args.no_sweep else None
-    wan_train1 = wan_full = None
-    if rank == 0 and world == 1 and not args.no_sweep:
-        wan_train1 = wan_train(args, ffi, dev, timed)
-        torch.cuda.empty_cache()
-        wan_full = wan_train(args, ffi, dev, timed, blocks=40, recompute=True)
-        torch.cuda.empty_cache()
-    sweep = hbm_sweep(ffi, dev, hbm) if rank == 0 and not args.no_sweep else None
+    K_ser = min(K_e2e, 3)
+    ms_e2e_serial = timed(e2e_serial, K_ser) / K_ser
+    del pipe
+
+    extras = not args.no_sweep and rank == 0 and world == 1
+    light = argparse.Namespace(steps=min(args.steps, 3), warmup=min(args.warmup, 2))
+    awm = awm_step(light, ffi, model, cfg, dev, si.x, si.txt, torch.randn_like(si.x), si.r, timed, world) \
+        if extras else None
+    train = train_step(argparse.Namespace(steps=2, warmup=1) if ms_step > 200 else light, ffi, model, cfg, dev,
+                       si.x, si.txt, si.t, si.tn, si.sg, ctx["x_next"], ctx["lp_old"], ctx["adv"], ctx["dit_flops"],
+                       timed, world) if extras else None
+    model.close()
+    del ctx, model, step
+    torch.cuda.empty_cache()
+
+    # ---- the other workloads, each timed on its own (rank 0, one GPU)
+    others = {}
+    if extras:
+        for name in ("flux_double_block", "flux_8d16s", "qwen_image_60d", "wan_40"):
+            if name == args.workload:
+                continue
+            ocfg = synth.config(name)
+            if name == "flux_8d16s":
+                others[name] = measure_rollout_workload(ffi, ocfg, dev, rank, world, timed)
+            elif name == "wan_40":
+                others[name], _ = measure_step_workload(args, ffi, ocfg, dev, rank, world, timed, 3, 2)
+            else:
+                others[name], _ = measure_step_workload(args, ffi, ocfg, dev, rank, world, timed,
+                                                        10 if name == "flux_double_block" else 5, 3)
+            torch.cuda.empty_cache()
+    bwd = backward_kernels(args, ffi, synth.config("flux_double_block"), dev) if extras else None
+    at_cfg = at_config_small_kernels(ffi, dev, load_peaks()[0], cfg, rank) if extras else None
+    sweep = hbm_sweep(ffi, dev, load_peaks()[0]) if extras else None
     clk = clocks.stop() if clocks else None
     status = ffi.ff_check_device_status()
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        rate, secs, rows = oracle_rate(cfg, 30.0)
-        cpu = {"value": rate, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
-               "sample": f"1 of {B} samples, full velocity ({rows} latent tokens) + SDE step + log-prob + "
-                         f"advantage + loss, fp64 numpy, {secs:.1f} s"}
+        rate, secs, sample = oracle_rate(cfg)
+        cpu = {"value": rate, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle", "sample": sample}
 
     if rank == 0:
-        line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        line = {"metric": METRIC, "value": head["value"], "unit": UNIT, "n_gpus": world, "steps": args.steps,
                 "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
                 "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-                "config": {"workload": workload_desc(cfg), "batch": B, "group": G, "n_txt": Nt, "n_img": Ni,
+                "config": {"workload": head["workload"], "batch": B, "group": G, "n_txt": Nt, "n_img": Ni,
                            "hidden": cfg["hidden"], "parallelism": f"dp{world} (independent groups per GPU)",
-                           "l2": f"no flush: per-step working set ({2 * n_params / 1e9:.2f} GB weights + "
-                                 f"{ws.numel() / 1e9:.2f} GB activation workspace) > 129 MB L2"},
-                "roofline": roofline,
-                "dit_tflops": dit_flops / (ms_step / 1e3) / 1e12,
-                "secondary_rooflines": secondary,
-                "kernel_breakdown": breakdown,
+                           "l2": f"no flush: per-step working set ({head['weights_gb']:.2f} GB weights + "
+                                 f"{head['workspace_gb']:.2f} GB activation workspace) > 129 MB L2"},
+                "roofline": head["roofline"],
+                "dit_tflops": head["dit_tflops"],
+                "dit_frac_of_burst": head["dit_frac_of_burst"],
+                "secondary_rooflines": head["secondary_rooflines"],
+                "kernel_breakdown": head["kernel_breakdown"],
                 "cpu_baseline": cpu,
                 "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                        "ms_per_step": ms_e2e, "copies": "overlapped with the previous / next step's kernels "
-                        "(HostFedPipeline: copy stream, two device buffer sets)",
+                        "ms_per_step": ms_e2e, "steps": K_e2e,
+                        "copies": "overlapped with the previous / next step's kernels "
+                                  "(HostFedPipeline: copy stream, two device buffer sets)",
                         "serial_ms_per_step": ms_e2e_serial},
+                "other_workloads": others,
                 "hbm_sweep": sweep,
                 "small_kernels_at_config": at_cfg,
                 "awm_step": awm,
                 "train_step": train,
                 "backward_kernels": bwd,
-                "wan_block_train_step": wan_train1,
-                "wan_full_train_step": wan_full,
-                "gpu_launches": launches,
+                "gpu_launches": head["gpu_launches_per_step"] * args.steps,
                 "clocks": clk,
                 "device_status": status}
         print(json.dumps(line), flush=True)

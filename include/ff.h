@@ -138,7 +138,16 @@ int ff_sde_schedule_window(int kind, int n_steps, double shift, double eta, doub
  *                require 0 < t, t_next < t, sigma >= 0 (not checked on the
  *                host: device values).
  *   logp:        fp32, logp[b * ld] written for b < B; ld >= 1.
- *   ws:          workspace of at least ff_sde_workspace_size(B, D) bytes.
+ *   ws:          workspace of at least ff_sde_workspace_size(B, D) bytes,
+ *                16-byte aligned.  Its first 256 KiB hold ticket counters
+ *                that must be ZERO before the first call that uses the
+ *                workspace (cudaMemsetAsync it once after allocating); every
+ *                call leaves them zero again, so a workspace zeroed once
+ *                serves any number of calls of any B and D in stream order.
+ *                Calls that share a workspace must not overlap on the GPU.
+ * B <= 65535.  One kernel launch: every block stores a partial sum of its
+ * squared residuals and the last block of each sample adds that sample's
+ * partials in a fixed order, so logp is deterministic.
  * ------------------------------------------------------------------------ */
 int ff_sde_workspace_size(int B, int64_t D, size_t* bytes);
 int ff_sde_step_logprob(int B, int64_t D, const float* x_t, const float* v,
@@ -202,19 +211,24 @@ int ff_sde_logprob_backward(int B, int64_t D, const float* x_t, const float* v,
  *
  * Same arguments and results as ff_sde_step_logprob, minus the workspace.
  * The caller still passes every input and output.  The scratch is a fixed
- * 512 KiB array of fp64 partial sums built into the library, held on every
- * GPU that loads the library until the process exits.  Limit:
- * B * min(ceil(D / 4096), 1024) <= 65536 partial sums, which holds for any
- * D when B <= 64; larger calls are rejected with FF_ERR_UNSUPPORTED and a
- * message naming the limit.  Nothing here calls cudaMalloc, cudaFree or any other
- * allocating routine.
+ * 528 KiB array built into the library (4096 ticket counters, then 65536
+ * fp64 partial sums), held on every GPU that loads the library until the
+ * process exits.  Limits: B <= 4096 and B * min(ceil(D / 2048), 1024) <=
+ * 65536 partial sums, which holds for any D when B <= 64; larger calls are
+ * rejected with FF_ERR_UNSUPPORTED and a message naming the limit, before any
+ * pointer is looked at.  Nothing here calls cudaMalloc, cudaFree or any
+ * other allocating routine.
  *
  * The first call on each device looks up the array's device address
- * (cudaGetSymbolAddress, with that device current) and caches it; make that
- * first call before any stream capture begins.  Every call on a device uses
- * the same array, and each call rewrites every slot it reads, so no clearing
- * is needed; but calls whose kernels overlap on the GPU (different streams,
- * no ordering between them) race on the array and must not be issued.
+ * (cudaGetSymbolAddress, with that device current) and caches it per device
+ * ordinal; make that first call before any stream capture begins.  The
+ * cached address belongs to the device's primary context: it is not valid
+ * for a caller that drives the device through another context, and it goes
+ * stale after cudaDeviceReset.  Every call on a device uses the same array.
+ * The ticket counters start at zero when the library loads and every call
+ * leaves them zero; the partial slots are rewritten before they are read.
+ * Calls whose kernels overlap on the GPU (different streams, no ordering
+ * between them) race on the array and must not be issued.
  * ------------------------------------------------------------------------ */
 int ff_sde_step_logprob_noalloc(int B, int64_t D, const float* x_t, const float* v,
                                 const float* eps, float* x_next, const float* t,
@@ -238,7 +252,12 @@ int ff_group_advantage(int n_groups, int G, const float* rewards, float eps_A,
  *   minimum (ties: unclipped), else 0.
  * lp_new, lp_old: [B, T] fp32 row-major; adv: [B] fp32; loss: [1] fp32
  * (written); grad_lp_new: [B, T] fp32 or NULL.
- * ws: workspace of at least ff_grpo_loss_workspace_size(B, T) bytes.
+ * ws: workspace of at least ff_grpo_loss_workspace_size(B, T) bytes,
+ *   16-byte aligned.  Its first 16 bytes hold a ticket counter that must be
+ *   ZERO before the first call that uses the workspace (clear it once after
+ *   allocating); every call leaves it zero.  Calls sharing a workspace must
+ *   not overlap on the GPU.  One kernel launch; the last block to finish
+ *   adds the per-block partial sums in a fixed order (deterministic loss).
  * ------------------------------------------------------------------------ */
 int ff_grpo_loss_workspace_size(int B, int T, size_t* bytes);
 int ff_grpo_loss(int B, int T, const float* lp_new, const float* lp_old,

@@ -273,11 +273,22 @@ def single_block(P, l, cfg, x, mods, ang, rows=None):
 
 
 def modulation(P, cfg, t):
-    """[B, mod_width]: SiLU(c) W_mod^T + b_mod with c the timestep embedding MLP."""
+    """[B, mod_width]: SiLU(c) W_mod^T + b_mod with c the timestep embedding MLP.
+
+    W_mod is read 12H rows (one double block's share) at a time, so a model
+    with many blocks never holds the whole matrix in fp64 at once; every
+    output is the same dot product as in one product."""
     emb = timestep_embedding(t, cfg["time_freq_dim"])
     c = linear(silu(linear(emb, P["t_embed.fc1.w"], P["t_embed.fc1.b"])),
                P["t_embed.fc2.w"], P["t_embed.fc2.b"])
-    return linear(silu(c), P["mod.w"], P["mod.b"])
+    a = silu(c)
+    w, b = P["mod.w"], P["mod.b"]
+    n = b.shape[0]
+    out = np.empty((a.shape[0], n))
+    step = 12 * cfg["hidden"]
+    for r0 in range(0, n, step):
+        out[:, r0:r0 + step] = linear(a, w[r0:r0 + step], b[r0:r0 + step])
+    return out
 
 
 def velocity(P, cfg, x_t, txt, t, img_rows=None):

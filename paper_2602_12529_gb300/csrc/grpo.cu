@@ -1,15 +1,18 @@
 // grpo.cu -- group-relative advantage and the clipped-ratio policy loss of
 // Flow-GRPO (paper Sec. 2.3 "advantage computation", Sec. 3.1).
 //
-// Advantage: one warp per group of G contiguous samples; mean and population
-// std in fp64 (two passes over the group held in L1), then
-// A = (r - mean) / (std + eps_A).
+// Advantage: G / 4 lanes per group (G a power of two in [4, 128]), else one
+// warp per group.  Mean and population std are fp32 sums of the rewards
+// shifted by a pivot (the group's first reward), then
+// A = (r - mean) / (std + eps_A).  The tests bound the result against the
+// fp64 oracle at 1e-5 relative to the group's spread.
 //
 // Loss: rho = exp(lp_new - lp_old) per (sample, step);
 //   obj = min(rho A, clip(rho, 1 - lo, 1 + hi) A), loss = -sum(obj) / (B T),
 //   grad_lp_new = -A rho / (B T) where the unclipped term is the minimum.
-// Pass 1 writes one fp64 partial per block (grid size depends only on B T, so
-// the summation order is fixed); pass 2 adds the partials in order.
+// One launch: every block writes one fp64 partial (the grid size depends only
+// on B T), takes a ticket, and the block with the last ticket adds the
+// partials in index order, writes the loss and resets the ticket to zero.
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -19,6 +22,9 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kElemsPerBlock = kThreads * 16;
 constexpr int kMaxLossBlocks = 1216;   // 8 blocks of 256 threads on each of 152 SMs
+// Workspace: the ticket word at offset 0 (its own 16 bytes), then the fp64
+// partials.
+constexpr size_t kLossTicketBytes = 16;
 
 // The group sums run on values shifted by a pivot (the group's first
 // reward): mean = pivot + sum(r - pivot) / G.  A constant group then gets
@@ -132,11 +138,14 @@ __global__ void __launch_bounds__(kThreads) group_advantage_multi_kernel(int n_g
 // 32-bit arithmetic), fp64 only for the block and cross-block sums.
 // WEIGHTED: GRPO-Guard's per-step weights step_w[k] scale the term of step
 // k (objective and gradient).
+// ticket: zero on entry; the last block to store its partial sets it back
+// to zero.
 template <bool WEIGHTED>
 __global__ void __launch_bounds__(kThreads) grpo_loss_partial_kernel(int64_t n, int T, const float* lp_new,
                                                                      const float* lp_old, const float* adv,
                                                                      const float* step_w, float lo, float hi,
-                                                                     float inv_n, float* grad, double* partial) {
+                                                                     float inv_n, float* grad, double* partial,
+                                                                     unsigned* ticket, double inv_nd, float* loss) {
     __shared__ double red[kThreads / 32];
     float s = 0.f;
     const int64_t n4 = n >> 2;
@@ -177,25 +186,29 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_partial_kernel(int64_t n, 
     for (int o = 16; o; o >>= 1) d += __shfl_xor_sync(0xffffffffu, d, o);
     if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = d;
     __syncthreads();
+    __shared__ bool last;
     if (threadIdx.x == 0) {
         double t = 0.0;
         for (int w = 0; w < kThreads / 32; ++w) t += red[w];
         partial[blockIdx.x] = t;
+        __threadfence();                                   // partial visible before the ticket
+        last = atomicAdd(ticket, 1u) == gridDim.x - 1;
     }
-}
-
-__global__ void grpo_loss_finalize_kernel(int nblocks, const double* partial, double inv_n, float* loss) {
-    __shared__ double red[kThreads / 32];
-    double s = 0.0;
-    for (int i = threadIdx.x; i < nblocks; i += blockDim.x) s += partial[i];
+    __syncthreads();
+    if (!last) return;
+    // every partial is stored: add them in index order
+    __threadfence();
+    double acc = 0.0;
+    for (int i = threadIdx.x; i < static_cast<int>(gridDim.x); i += kThreads) acc += __ldcg(partial + i);
 #pragma unroll
-    for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
+    for (int o = 16; o; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
     __syncthreads();
     if (threadIdx.x == 0) {
         double t = 0.0;
-        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += red[w];
-        *loss = static_cast<float>(-t * inv_n);
+        for (int w = 0; w < kThreads / 32; ++w) t += red[w];
+        *ticket = 0u;
+        *loss = static_cast<float>(-t * inv_nd);
     }
 }
 
@@ -233,7 +246,7 @@ int ff_group_advantage(int n_groups, int G, const float* rewards, float eps_A, f
 int ff_grpo_loss_workspace_size(int B, int T, size_t* bytes) {
     if (!bytes) return ff::set_error(FF_ERR_INVALID_ARG, "bytes is null");
     if (B <= 0 || T <= 0) return ff::set_error(FF_ERR_INVALID_ARG, "B=%d T=%d must be positive", B, T);
-    *bytes = static_cast<size_t>(ff::loss_blocks(static_cast<int64_t>(B) * T)) * sizeof(double);
+    *bytes = ff::kLossTicketBytes + static_cast<size_t>(ff::loss_blocks(static_cast<int64_t>(B) * T)) * sizeof(double);
     return FF_OK;
 }
 
@@ -255,26 +268,24 @@ int grpo_loss_impl(int B, int T, const float* lp_new, const float* lp_old, const
         return set_error(FF_ERR_INVALID_ARG, "loss: clip range must satisfy 0 <= lo < 1, hi >= 0");
     const int64_t n = static_cast<int64_t>(B) * T;
     const int nb = loss_blocks(n);
-    const size_t need = static_cast<size_t>(nb) * sizeof(double);
-    if (!ws || ws_bytes < need || (reinterpret_cast<uintptr_t>(ws) & 7))
-        return set_error(FF_ERR_WORKSPACE, "loss: workspace %zu B < %zu B needed (or misaligned)", ws_bytes, need);
-    double* partial = static_cast<double*>(ws);
-    {
+    const size_t need = kLossTicketBytes + static_cast<size_t>(nb) * sizeof(double);
+    if (!ws || ws_bytes < need || (reinterpret_cast<uintptr_t>(ws) & 15))
+        return set_error(FF_ERR_WORKSPACE, "loss: workspace %zu B < %zu B needed (or not 16-byte aligned)", ws_bytes,
+                         need);
+    unsigned* ticket = static_cast<unsigned*>(ws);
+    double* partial = reinterpret_cast<double*>(static_cast<uint8_t*>(ws) + kLossTicketBytes);
+    const float inv_f = static_cast<float>(1.0 / static_cast<double>(n));
+    const double inv_d = 1.0 / static_cast<double>(n);
     ProfScope prof(stream, "grpo_loss", 0.0, static_cast<double>(n) * (grad_lp_new ? 12.0 : 8.0) + 4.0 * B);
     if (step_w)
-        grpo_loss_partial_kernel<true><<<nb, kThreads, 0, stream>>>(
-            n, T, lp_new, lp_old, adv, step_w, clip_lo, clip_hi, static_cast<float>(1.0 / static_cast<double>(n)),
-            grad_lp_new, partial);
+        grpo_loss_partial_kernel<true><<<nb, kThreads, 0, stream>>>(n, T, lp_new, lp_old, adv, step_w, clip_lo,
+                                                                    clip_hi, inv_f, grad_lp_new, partial, ticket,
+                                                                    inv_d, loss);
     else
-        grpo_loss_partial_kernel<false><<<nb, kThreads, 0, stream>>>(
-            n, T, lp_new, lp_old, adv, nullptr, clip_lo, clip_hi, static_cast<float>(1.0 / static_cast<double>(n)),
-            grad_lp_new, partial);
-    }
-    int rc = check_launch("grpo_loss_partial_kernel");
-    if (rc) return rc;
-    ProfScope prof(stream, "grpo_loss_finalize", 0.0, nb * 8.0 + 4.0);
-    grpo_loss_finalize_kernel<<<1, kThreads, 0, stream>>>(nb, partial, 1.0 / static_cast<double>(n), loss);
-    return check_launch("grpo_loss_finalize_kernel");
+        grpo_loss_partial_kernel<false><<<nb, kThreads, 0, stream>>>(n, T, lp_new, lp_old, adv, nullptr, clip_lo,
+                                                                     clip_hi, inv_f, grad_lp_new, partial, ticket,
+                                                                     inv_d, loss);
+    return check_launch("grpo_loss_kernel");
 }
 
 }  // namespace

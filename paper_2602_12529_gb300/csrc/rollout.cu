@@ -84,6 +84,10 @@ int rollout(const ff_dit* model, int B, int S, float* x, const void* txt, const 
     float* v = reinterpret_cast<float*>(base + p.v);
     float* tb = reinterpret_cast<float*>(base + p.tb);
     float* sb = reinterpret_cast<float*>(base + p.sb);
+    // the SDE step's ticket words must be zero before its first launch (each
+    // launch leaves them zero); the rest of the workspace needs no clearing
+    if (cudaMemsetAsync(base + p.sde, 0, p.total - p.sde, stream) != cudaSuccess)
+        return set_error(FF_ERR_CUDA, "rollout: clearing the SDE step's scratch failed");
     const int n = (S + 1) * B;
     broadcast_steps_kernel<<<(n + 255) / 256, 256, 0, stream>>>(S, B, t, sigma, tb, sb);
     FF_TRY(check_launch("broadcast_steps_kernel"));

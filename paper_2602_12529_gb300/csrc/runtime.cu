@@ -3,6 +3,7 @@
 #include <stdarg.h>
 #include <stdio.h>
 
+#include <atomic>
 #include <mutex>
 
 #include "internal.h"
@@ -16,8 +17,10 @@ thread_local char g_err[512] = "";
 __device__ int g_device_status;
 
 constexpr int kMaxDevices = 64;
-int* g_status_ptr[kMaxDevices] = {};
-int g_num_sms[kMaxDevices] = {};
+// Per-device caches, keyed by device ordinal: they hold the primary
+// context's values and go stale after cudaDeviceReset.
+std::atomic<int*> g_status_ptr[kMaxDevices] = {};
+std::atomic<int> g_num_sms[kMaxDevices] = {};
 std::mutex g_mu;
 
 using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -51,26 +54,30 @@ int check_launch(const char* what) {
 int* device_status_ptr() {
     const int d = current_device();
     if (d < 0) return nullptr;
-    if (!g_status_ptr[d]) {
+    int* p = g_status_ptr[d].load(std::memory_order_acquire);
+    if (!p) {
         std::lock_guard<std::mutex> lk(g_mu);
-        if (!g_status_ptr[d]) {
-            void* p = nullptr;
-            if (cudaGetSymbolAddress(&p, g_device_status) != cudaSuccess) return nullptr;
-            g_status_ptr[d] = static_cast<int*>(p);
+        p = g_status_ptr[d].load(std::memory_order_relaxed);
+        if (!p) {
+            void* q = nullptr;
+            if (cudaGetSymbolAddress(&q, g_device_status) != cudaSuccess) return nullptr;
+            p = static_cast<int*>(q);
+            g_status_ptr[d].store(p, std::memory_order_release);
         }
     }
-    return g_status_ptr[d];
+    return p;
 }
 
 int num_sms() {
     const int d = current_device();
     if (d < 0) return 1;
-    if (!g_num_sms[d]) {
-        int n = 0;
+    int n = g_num_sms[d].load(std::memory_order_relaxed);
+    if (!n) {
         cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, d);
-        g_num_sms[d] = n > 0 ? n : 1;
+        if (n <= 0) n = 1;
+        g_num_sms[d].store(n, std::memory_order_relaxed);
     }
-    return g_num_sms[d];
+    return n;
 }
 
 int make_tmap_f32_sw128(CUtensorMap* tm, const void* base, int64_t rows, int64_t cols, int64_t ld, int box_rows) {

@@ -8,11 +8,12 @@
 //   SAMPLE: x_next = mean + std eps;  EVAL: x_next given; SAMPLE with eps
 //   drawn in the kernel from the counter-based generator of rng.cuh
 //   logp = -sum (x_next - mean)^2 / (2 std^2) - D ln std - D/2 ln 2 pi
-// The per-sample coefficients are formed in fp64 once per thread; the
-// elementwise work is fp32 FMAs over 128-bit streaming loads.  Pass 1 writes
-// one fp64 partial sum of squared residuals per 4096-element chunk; pass 2
-// (one block per sample) adds the partials in a fixed order, so the result
-// does not depend on scheduling.
+// The per-sample coefficients are formed in fp64 once per block; the
+// elementwise work is fp32 FMAs over 128-bit streaming loads.  One launch:
+// every block writes one fp64 partial sum of squared residuals, then takes a
+// ticket; the block that draws the sample's last ticket adds that sample's
+// partials in index order (so the result does not depend on which block
+// finished last), writes logp and puts the ticket word back to zero.
 #include "internal.h"
 #include "ptx.cuh"
 #include "rng.cuh"
@@ -22,8 +23,8 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kModePhilox = 2;                                // SAMPLE, eps from rng.cuh (internal mode)
-constexpr int kVecPerThread = 4;                              // float4 per thread per chunk
-constexpr int kChunk = kThreads * kVecPerThread * 4;          // 4096 elements
+constexpr int kVecPerThread = 2;                              // float4 per thread per chunk
+constexpr int kChunk = kThreads * kVecPerThread * 4;          // 2048 elements
 
 struct StepCoef {
     float cx, cv, std;
@@ -55,15 +56,34 @@ __device__ __forceinline__ double block_sum(double v, double* red) {
     return s;   // valid in thread 0
 }
 
+// The log-probability of sample b from its summed squared residual ss:
+// -ss / (2 std^2) - D ln std - D/2 ln 2 pi (divided by D for FF_LP_MEAN), in
+// fp64; 0 when std == 0 (no density).
+__device__ __forceinline__ float logprob_of(double ss, int64_t D, const float* t, const float* t_next,
+                                            const float* sigma, int b, int reduce) {
+    const double delta = static_cast<double>(t[b]) - static_cast<double>(t_next[b]);
+    const double sd = static_cast<double>(sigma[b]) * sqrt(delta);
+    double lp = 0.0;
+    if (sd > 0.0) {
+        const double dd = static_cast<double>(D);
+        lp = -0.5 * ss / (sd * sd) - dd * log(sd) - 0.5 * dd * log(2.0 * 3.14159265358979323846);
+        if (reduce == FF_LP_MEAN) lp /= dd;
+    }
+    return static_cast<float>(lp);
+}
+
 // Grid (blocks_per_sample, B); block k of sample b handles chunks
 // k, k + blocks_per_sample, ... and writes one fp64 partial.  The number of
-// blocks per sample depends only on D (see nblocks), so the summation order
+// blocks per sample depends only on D (see nchunks), so the summation order
 // is fixed.  The per-sample coefficients are formed once per block in fp64.
+// ticket[b] counts the blocks of sample b that have stored their partial; it
+// is zero on entry and the last block of the sample sets it back to zero.
 template <int MODE>
 __global__ void __launch_bounds__(kThreads) sde_step_partial_kernel(int64_t D, int nblk, const float* x,
                                                                     const float* v, const float* eps, float* x_next,
                                                                     const float* t, const float* t_next,
                                                                     const float* sigma, double* partial,
+                                                                    unsigned* ticket, int reduce, float* logp, int ld,
                                                                     PhiloxKey key, uint32_t rng_stream) {
     __shared__ double red[kThreads / 32];
     __shared__ StepCoef coef;
@@ -117,7 +137,24 @@ __global__ void __launch_bounds__(kThreads) sde_step_partial_kernel(int64_t D, i
         }
     }
     const double s = block_sum(static_cast<double>(ss), red);
-    if (threadIdx.x == 0) partial[static_cast<int64_t>(b) * nblk + blockIdx.x] = s;
+    __shared__ bool last;
+    if (threadIdx.x == 0) {
+        partial[static_cast<int64_t>(b) * nblk + blockIdx.x] = s;
+        __threadfence();                                   // partial visible before the ticket
+        last = atomicAdd(ticket + b, 1u) == static_cast<unsigned>(nblk - 1);
+    }
+    __syncthreads();
+    if (!last) return;
+    // every partial of sample b is stored; add them in index order
+    __threadfence();
+    const double* pb = partial + static_cast<int64_t>(b) * nblk;
+    double acc = 0.0;
+    for (int i = threadIdx.x; i < nblk; i += kThreads) acc += __ldcg(pb + i);
+    acc = block_sum(acc, red);
+    if (threadIdx.x == 0) {
+        ticket[b] = 0u;
+        logp[static_cast<int64_t>(b) * ld] = logprob_of(acc, D, t, t_next, sigma, b, reduce);
+    }
 }
 
 // out[b, 4g .. 4g + 3] = the normals of element group g of sample b (rng.cuh).
@@ -128,28 +165,6 @@ __global__ void __launch_bounds__(kThreads) philox_normal_kernel(int B, int64_t 
          k += static_cast<int64_t>(gridDim.x) * kThreads) {
         const int64_t b = k / nvec, g = k - b * nvec;
         __stcs(out + k, philox_normal4(static_cast<uint32_t>(g), static_cast<uint32_t>(b), rng_stream, key));
-    }
-}
-
-__global__ void __launch_bounds__(kThreads) sde_logprob_finalize_kernel(int64_t D, int nchunk, const double* partial,
-                                                                        const float* t, const float* t_next,
-                                                                        const float* sigma, int reduce, float* logp,
-                                                                        int ld) {
-    __shared__ double red[kThreads / 32];
-    const int b = blockIdx.x;
-    double s = 0.0;
-    for (int i = threadIdx.x; i < nchunk; i += kThreads) s += partial[static_cast<int64_t>(b) * nchunk + i];
-    s = block_sum(s, red);
-    if (threadIdx.x == 0) {
-        const double delta = static_cast<double>(t[b]) - static_cast<double>(t_next[b]);
-        const double sd = static_cast<double>(sigma[b]) * sqrt(delta);
-        double lp = 0.0;
-        if (sd > 0.0) {
-            const double dd = static_cast<double>(D);
-            lp = -0.5 * s / (sd * sd) - dd * log(sd) - 0.5 * dd * log(2.0 * 3.14159265358979323846);
-            if (reduce == FF_LP_MEAN) lp /= dd;
-        }
-        logp[static_cast<int64_t>(b) * ld] = static_cast<float>(lp);
     }
 }
 
@@ -199,8 +214,16 @@ __global__ void __launch_bounds__(kThreads) sde_logprob_backward_kernel(int64_t 
 }
 
 constexpr int kMaxBlocksPerSample = 1024;
+constexpr int kMaxSamples = 65535;
 
-// partial sums (blocks) per sample: one per 4096-element chunk up to 1024,
+// Workspace layout: the ticket words of up to kMaxSamples samples at a fixed
+// place (offset 0), then the fp64 partials.  Keeping the tickets at the same
+// offset whatever B and D are means a workspace zeroed once stays valid for
+// calls of any shape: no call ever stores a partial over a ticket word.
+constexpr size_t kTicketBytes = 256 * 1024;
+static_assert(kTicketBytes >= sizeof(unsigned) * kMaxSamples, "ticket region too small");
+
+// partial sums (blocks) per sample: one per 2048-element chunk up to 1024,
 // then every block loops over several chunks
 int nchunks(int64_t D) {
     const int64_t c = (D + kChunk - 1) / kChunk;
@@ -215,7 +238,7 @@ extern "C" {
 int ff_sde_workspace_size(int B, int64_t D, size_t* bytes) {
     if (!bytes) return ff::set_error(FF_ERR_INVALID_ARG, "bytes is null");
     if (B <= 0 || D <= 0) return ff::set_error(FF_ERR_INVALID_ARG, "B and D must be positive");
-    *bytes = static_cast<size_t>(B) * static_cast<size_t>(ff::nchunks(D)) * sizeof(double);
+    *bytes = ff::kTicketBytes + static_cast<size_t>(B) * static_cast<size_t>(ff::nchunks(D)) * sizeof(double);
     return FF_OK;
 }
 
@@ -224,8 +247,28 @@ int ff_sde_workspace_size(int B, int64_t D, size_t* bytes) {
 namespace ff {
 namespace {
 
-// Argument checks and the two launches of one SDE step (mode FF_SDE_SAMPLE,
-// FF_SDE_EVAL or kModePhilox).
+// One launch of the SDE step (mode FF_SDE_SAMPLE, FF_SDE_EVAL or
+// kModePhilox) over caller scratch: tickets (zero on entry, zero again on
+// exit) and B * nchunks(D) fp64 partials.
+int launch_sde_step(int B, int64_t D, int nc, const float* x_t, const float* v, const float* eps, float* x_next,
+                    const float* t, const float* t_next, const float* sigma, int mode, int reduce, float* logp,
+                    int ld, unsigned* ticket, double* partial, PhiloxKey key, uint32_t rng_stream,
+                    cudaStream_t stream) {
+    const dim3 grid(nc, B);
+    ProfScope prof(stream, "sde_step", 0.0, static_cast<double>(B) * D * (mode == FF_SDE_SAMPLE ? 16.0 : 12.0));
+    if (mode == FF_SDE_SAMPLE)
+        sde_step_partial_kernel<FF_SDE_SAMPLE><<<grid, kThreads, 0, stream>>>(
+            D, nc, x_t, v, eps, x_next, t, t_next, sigma, partial, ticket, reduce, logp, ld, key, rng_stream);
+    else if (mode == kModePhilox)
+        sde_step_partial_kernel<kModePhilox><<<grid, kThreads, 0, stream>>>(
+            D, nc, x_t, v, eps, x_next, t, t_next, sigma, partial, ticket, reduce, logp, ld, key, rng_stream);
+    else
+        sde_step_partial_kernel<FF_SDE_EVAL><<<grid, kThreads, 0, stream>>>(
+            D, nc, x_t, v, eps, x_next, t, t_next, sigma, partial, ticket, reduce, logp, ld, key, rng_stream);
+    return check_launch("sde_step_kernel");
+}
+
+// Argument checks of one SDE step, then its launch.
 int sde_step(int B, int64_t D, const float* x_t, const float* v, const float* eps, float* x_next, const float* t,
              const float* t_next, const float* sigma, int mode, int reduce, float* logp, int ld, void* ws,
              size_t ws_bytes, PhiloxKey key, uint32_t rng_stream, cudaStream_t stream) {
@@ -237,32 +280,18 @@ int sde_step(int B, int64_t D, const float* x_t, const float* v, const float* ep
     if (!aligned16(x_t) || !aligned16(v) || !aligned16(x_next) || (mode == FF_SDE_SAMPLE && !aligned16(eps)))
         return set_error(FF_ERR_INVALID_ARG, "sde: arrays must be 16-byte aligned");
     if (ld < 1) return set_error(FF_ERR_INVALID_ARG, "sde: ld=%d < 1", ld);
-    if (B > 65535) return set_error(FF_ERR_UNSUPPORTED, "sde: B=%d > 65535", B);
+    if (B > kMaxSamples) return set_error(FF_ERR_UNSUPPORTED, "sde: B=%d > %d", B, kMaxSamples);
     if (mode == kModePhilox && D / 4 > 0xFFFFFFFFll)
         return set_error(FF_ERR_UNSUPPORTED, "sde: D=%lld too large for the generator's counter", (long long)D);
     const int nc = nchunks(D);
-    const size_t need = static_cast<size_t>(B) * nc * sizeof(double);
-    if (!ws || ws_bytes < need || (reinterpret_cast<uintptr_t>(ws) & 7))
-        return set_error(FF_ERR_WORKSPACE, "sde: workspace %zu B < %zu B needed (or misaligned)", ws_bytes, need);
-    double* partial = static_cast<double*>(ws);
-    const dim3 grid(nc, B);
-    {
-        ProfScope prof(stream, "sde_step", 0.0, static_cast<double>(B) * D * (mode == FF_SDE_SAMPLE ? 16.0 : 12.0));
-        if (mode == FF_SDE_SAMPLE)
-            sde_step_partial_kernel<FF_SDE_SAMPLE><<<grid, kThreads, 0, stream>>>(D, nc, x_t, v, eps, x_next, t, t_next,
-                                                                                  sigma, partial, key, rng_stream);
-        else if (mode == kModePhilox)
-            sde_step_partial_kernel<kModePhilox><<<grid, kThreads, 0, stream>>>(D, nc, x_t, v, eps, x_next, t, t_next,
-                                                                                sigma, partial, key, rng_stream);
-        else
-            sde_step_partial_kernel<FF_SDE_EVAL><<<grid, kThreads, 0, stream>>>(D, nc, x_t, v, eps, x_next, t, t_next,
-                                                                                sigma, partial, key, rng_stream);
-    }
-    int rc = check_launch("sde_step_partial_kernel");
-    if (rc) return rc;
-    ProfScope prof(stream, "sde_finalize", 0.0, static_cast<double>(B) * nc * 8.0 + B * 16.0);
-    sde_logprob_finalize_kernel<<<B, kThreads, 0, stream>>>(D, nc, partial, t, t_next, sigma, reduce, logp, ld);
-    return check_launch("sde_logprob_finalize_kernel");
+    const size_t need = kTicketBytes + static_cast<size_t>(B) * nc * sizeof(double);
+    if (!ws || ws_bytes < need || (reinterpret_cast<uintptr_t>(ws) & 15))
+        return set_error(FF_ERR_WORKSPACE, "sde: workspace %zu B < %zu B needed (or not 16-byte aligned)", ws_bytes,
+                         need);
+    unsigned* ticket = static_cast<unsigned*>(ws);
+    double* partial = reinterpret_cast<double*>(static_cast<uint8_t*>(ws) + kTicketBytes);
+    return launch_sde_step(B, D, nc, x_t, v, eps, x_next, t, t_next, sigma, mode, reduce, logp, ld, ticket, partial,
+                           key, rng_stream, stream);
 }
 
 }  // namespace
@@ -369,40 +398,53 @@ extern "C" int ff_sde_schedule_window(int kind, int n_steps, double shift, doubl
 
 // ---------------------------------------------------------------------------
 // ff_sde_step_logprob_noalloc: the same step for callers that cannot hand the
-// library any device memory of their own (see include/ff.h).  The per-chunk
-// partial sums live in a fixed array in the library's device image instead
-// of a caller workspace.
+// library any device memory of their own (see include/ff.h).  The tickets and
+// the per-chunk partial sums live in a fixed array in the library's device
+// image instead of a caller workspace.
 // ---------------------------------------------------------------------------
+#include <atomic>
 #include <mutex>
 
 namespace ff {
 namespace {
 
-constexpr int kNoAllocMaxPartials = 65536;   // 512 KiB of fp64 partial sums on every device
+constexpr int kNoAllocMaxSamples = 4096;      // ticket words, at the front of the array
+constexpr int kNoAllocMaxPartials = 65536;    // fp64 partial sums after them
+constexpr int kNoAllocTicketSlots = kNoAllocMaxSamples / 2;   // two 32-bit tickets per fp64 slot
 
-// Shared by every call on a device; each call overwrites every slot it later
-// reads, so nothing has to start at zero.
-static __device__ __align__(256) double g_sde_scratch[kNoAllocMaxPartials];
+// Shared by every call on a device (528 KiB).  The ticket words start at
+// zero (device globals are zero-initialised when the module loads) and every
+// call leaves them at zero; the partial slots are rewritten before they are
+// read, so nothing else has to be cleared.
+static __device__ __align__(256) double g_sde_scratch[kNoAllocTicketSlots + kNoAllocMaxPartials];
 
 constexpr int kNoAllocMaxDevices = 64;
-double* g_sde_scratch_addr[kNoAllocMaxDevices] = {};
+std::atomic<double*> g_sde_scratch_addr[kNoAllocMaxDevices] = {};
 std::mutex g_sde_scratch_mu;
 
 // Device address of g_sde_scratch on the current device, looked up once per
 // device with that device current (host code cannot use the symbol itself).
+// The cache is keyed by device ordinal and holds the primary context's
+// address: it is wrong for a caller that runs the library in another context
+// on that device, and stale after cudaDeviceReset.
 int sde_scratch_address(double** out) {
     int dev = -1;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kNoAllocMaxDevices)
         return set_error(FF_ERR_CUDA, "sde (no-alloc): no usable current device");
-    std::lock_guard<std::mutex> lk(g_sde_scratch_mu);
-    if (!g_sde_scratch_addr[dev]) {
-        void* p = nullptr;
-        const cudaError_t e = cudaGetSymbolAddress(&p, g_sde_scratch);
-        if (e != cudaSuccess || !p)
-            return set_error(FF_ERR_CUDA, "sde (no-alloc): cudaGetSymbolAddress failed: %s", cudaGetErrorString(e));
-        g_sde_scratch_addr[dev] = static_cast<double*>(p);
+    double* p = g_sde_scratch_addr[dev].load(std::memory_order_acquire);
+    if (!p) {
+        std::lock_guard<std::mutex> lk(g_sde_scratch_mu);
+        p = g_sde_scratch_addr[dev].load(std::memory_order_relaxed);
+        if (!p) {
+            void* q = nullptr;
+            const cudaError_t e = cudaGetSymbolAddress(&q, g_sde_scratch);
+            if (e != cudaSuccess || !q)
+                return set_error(FF_ERR_CUDA, "sde (no-alloc): cudaGetSymbolAddress failed: %s", cudaGetErrorString(e));
+            p = static_cast<double*>(q);
+            g_sde_scratch_addr[dev].store(p, std::memory_order_release);
+        }
     }
-    *out = g_sde_scratch_addr[dev];
+    *out = p;
     return FF_OK;
 }
 
@@ -415,6 +457,17 @@ extern "C" int ff_sde_step_logprob_noalloc(int B, int64_t D, const float* x_t, c
     using namespace ff;
     if (B <= 0 || D <= 0) return set_error(FF_ERR_INVALID_ARG, "sde (no-alloc): B=%d D=%lld must be positive", B, (long long)D);
     if (D % 4) return set_error(FF_ERR_UNSUPPORTED, "sde (no-alloc): D=%lld not a multiple of 4", (long long)D);
+    // the scratch limits come first, so an oversized call is rejected
+    // whatever its pointers are
+    if (B > kNoAllocMaxSamples)
+        return set_error(FF_ERR_UNSUPPORTED, "sde (no-alloc): B=%d exceeds the built-in scratch's %d samples; use "
+                         "ff_sde_step_logprob with a workspace", B, kNoAllocMaxSamples);
+    const int nc = nchunks(D);
+    if (static_cast<int64_t>(B) * nc > kNoAllocMaxPartials)
+        return set_error(FF_ERR_UNSUPPORTED,
+                         "sde (no-alloc): B * min(ceil(D / %d), %d) = %lld partial sums exceed the built-in scratch "
+                         "of %d; use ff_sde_step_logprob with a workspace",
+                         kChunk, kMaxBlocksPerSample, (long long)B * nc, kNoAllocMaxPartials);
     if (mode != FF_SDE_SAMPLE && mode != FF_SDE_EVAL) return set_error(FF_ERR_INVALID_ARG, "sde (no-alloc): bad mode %d", mode);
     if (reduce != FF_LP_SUM && reduce != FF_LP_MEAN)
         return set_error(FF_ERR_INVALID_ARG, "sde (no-alloc): bad reduce %d", reduce);
@@ -423,25 +476,11 @@ extern "C" int ff_sde_step_logprob_noalloc(int B, int64_t D, const float* x_t, c
     if (!aligned16(x_t) || !aligned16(v) || !aligned16(x_next) || (mode == FF_SDE_SAMPLE && !aligned16(eps)))
         return set_error(FF_ERR_INVALID_ARG, "sde (no-alloc): arrays must be 16-byte aligned");
     if (ld < 1) return set_error(FF_ERR_INVALID_ARG, "sde (no-alloc): ld=%d < 1", ld);
-    if (B > 65535) return set_error(FF_ERR_UNSUPPORTED, "sde (no-alloc): B=%d > 65535", B);
-    const int nc = nchunks(D);
-    if (static_cast<int64_t>(B) * nc > kNoAllocMaxPartials)
-        return set_error(FF_ERR_UNSUPPORTED,
-                         "sde (no-alloc): B * min(ceil(D / %d), %d) = %lld partial sums exceed the built-in scratch "
-                         "of %d; use ff_sde_step_logprob with a workspace",
-                         kChunk, kMaxBlocksPerSample, (long long)B * nc, kNoAllocMaxPartials);
-    double* partial = nullptr;
-    const int rc0 = sde_scratch_address(&partial);
+    double* scratch = nullptr;
+    const int rc0 = sde_scratch_address(&scratch);
     if (rc0) return rc0;
-    const dim3 grid(nc, B);
-    if (mode == FF_SDE_SAMPLE)
-        sde_step_partial_kernel<FF_SDE_SAMPLE><<<grid, kThreads, 0, stream>>>(D, nc, x_t, v, eps, x_next, t, t_next,
-                                                                              sigma, partial, PhiloxKey{0, 0}, 0u);
-    else
-        sde_step_partial_kernel<FF_SDE_EVAL><<<grid, kThreads, 0, stream>>>(D, nc, x_t, v, eps, x_next, t, t_next,
-                                                                            sigma, partial, PhiloxKey{0, 0}, 0u);
-    int rc = check_launch("sde_step_partial_kernel (no-alloc)");
-    if (rc) return rc;
-    sde_logprob_finalize_kernel<<<B, kThreads, 0, stream>>>(D, nc, partial, t, t_next, sigma, reduce, logp, ld);
-    return check_launch("sde_logprob_finalize_kernel (no-alloc)");
+    unsigned* ticket = reinterpret_cast<unsigned*>(scratch);
+    double* partial = scratch + kNoAllocTicketSlots;
+    return launch_sde_step(B, D, nc, x_t, v, eps, x_next, t, t_next, sigma, mode, reduce, logp, ld, ticket, partial,
+                           PhiloxKey{0, 0}, 0u, stream);
 }

@@ -168,6 +168,33 @@ def _check(t, dtype, name):
         raise TypeError(f"{name}: expected {dtype}, got {t.dtype}")
 
 
+def _need(t, n: int, name: str):
+    """Raise unless tensor t holds at least n elements (the kernels index
+    that far; a shorter buffer would be read or written past its end)."""
+    if t.numel() < n:
+        raise ValueError(f"{name}: {t.numel()} elements, the call touches {n}")
+
+
+def _sde_args(x_t, v, eps, x_next, t, t_next, sigma, logp, ld, need_eps):
+    """dtype and size checks shared by the SDE step wrappers: [B, D] arrays,
+    [B] times and sigmas, logp read at b * ld."""
+    import torch
+    B = x_t.shape[0]
+    D = x_t.numel() // B
+    arrays = [("x_t", x_t), ("v", v), ("x_next", x_next)] + ([("eps", eps)] if need_eps else [])
+    for n_, a in arrays:
+        _check(a, torch.float32, n_)
+        _need(a, B * D, n_)
+    for n_, a in (("t", t), ("t_next", t_next), ("sigma", sigma)):
+        _check(a, torch.float32, n_)
+        _need(a, B, n_)
+    _check(logp, torch.float32, "logp")
+    if ld < 1:
+        raise ValueError("ld must be >= 1")
+    _need(logp, (B - 1) * ld + 1, "logp")
+    return B, D
+
+
 # ------------------------------------------------------------ host queries
 
 def ff_version() -> int:
@@ -236,13 +263,9 @@ def ff_dit_weight_layout(cfg: dict):
 def ff_sde_step_logprob(x_t, v, eps, x_next, t, t_next, sigma, logp, mode=FF_SDE_SAMPLE, reduce=FF_LP_SUM,
                         ld=1, ws=None, stream=None):
     import torch
-    B = x_t.shape[0]
-    D = x_t.numel() // B
-    for n_, a in (("x_t", x_t), ("v", v), ("x_next", x_next), ("t", t), ("t_next", t_next), ("sigma", sigma),
-                  ("logp", logp)):
-        _check(a, torch.float32, n_)
+    B, D = _sde_args(x_t, v, eps, x_next, t, t_next, sigma, logp, ld, mode == FF_SDE_SAMPLE)
     if ws is None:
-        ws = torch.empty(ff_sde_workspace_size(B, D), dtype=torch.uint8, device=x_t.device)
+        ws = torch.zeros(ff_sde_workspace_size(B, D), dtype=torch.uint8, device=x_t.device)
     _call("ff_sde_step_logprob", B, D, _ptr(x_t), _ptr(v), _ptr(eps), _ptr(x_next), _ptr(t), _ptr(t_next),
           _ptr(sigma), mode, reduce, _ptr(logp), ld, _ptr(ws), ws.numel(), _stream(stream))
 
@@ -260,13 +283,9 @@ def ff_sde_step_logprob_philox(x_t, v, x_next, t, t_next, sigma, logp, seed: int
                                reduce=FF_LP_SUM, ld=1, ws=None, stream=None):
     """The SAMPLE step with eps drawn in the kernel (ff_philox_normal's values)."""
     import torch
-    B = x_t.shape[0]
-    D = x_t.numel() // B
-    for n_, a in (("x_t", x_t), ("v", v), ("x_next", x_next), ("t", t), ("t_next", t_next), ("sigma", sigma),
-                  ("logp", logp)):
-        _check(a, torch.float32, n_)
+    B, D = _sde_args(x_t, v, None, x_next, t, t_next, sigma, logp, ld, False)
     if ws is None:
-        ws = torch.empty(ff_sde_workspace_size(B, D), dtype=torch.uint8, device=x_t.device)
+        ws = torch.zeros(ff_sde_workspace_size(B, D), dtype=torch.uint8, device=x_t.device)
     _call("ff_sde_step_logprob_philox", B, D, _ptr(x_t), _ptr(v), _ptr(x_next), _ptr(t), _ptr(t_next), _ptr(sigma),
           int(seed), int(rng_stream), reduce, _ptr(logp), ld, _ptr(ws), ws.numel(), _stream(stream))
 
@@ -275,12 +294,7 @@ def ff_sde_step_logprob_noalloc(x_t, v, eps, x_next, t, t_next, sigma, logp, mod
                                 reduce=FF_LP_SUM, ld=1, stream=None):
     """ff_sde_step_logprob without a workspace: scratch is the library's own
     fixed device array (for callers that cannot allocate device memory)."""
-    import torch
-    B = x_t.shape[0]
-    D = x_t.numel() // B
-    for n_, a in (("x_t", x_t), ("v", v), ("x_next", x_next), ("t", t), ("t_next", t_next), ("sigma", sigma),
-                  ("logp", logp)):
-        _check(a, torch.float32, n_)
+    B, D = _sde_args(x_t, v, eps, x_next, t, t_next, sigma, logp, ld, mode == FF_SDE_SAMPLE)
     _call("ff_sde_step_logprob_noalloc", B, D, _ptr(x_t), _ptr(v), _ptr(eps), _ptr(x_next), _ptr(t), _ptr(t_next),
           _ptr(sigma), mode, reduce, _ptr(logp), ld, _stream(stream))
 
@@ -289,11 +303,9 @@ def ff_sde_logprob_backward(x_t, v, x_next, t, t_next, sigma, grad_logp, grad_v,
                             stream=None):
     """grad_v = d logp / d v (x_next fixed) times grad_logp[b * ld]."""
     import torch
-    for n_, a in (("x_t", x_t), ("v", v), ("x_next", x_next), ("t", t), ("t_next", t_next), ("sigma", sigma),
-                  ("grad_logp", grad_logp), ("grad_v", grad_v)):
-        _check(a, torch.float32, n_)
-    B = x_t.shape[0]
-    D = x_t.numel() // B
+    B, D = _sde_args(x_t, v, None, x_next, t, t_next, sigma, grad_logp, ld, False)
+    _check(grad_v, torch.float32, "grad_v")
+    _need(grad_v, B * D, "grad_v")
     _call("ff_sde_logprob_backward", B, D, _ptr(x_t), _ptr(v), _ptr(x_next), _ptr(t), _ptr(t_next), _ptr(sigma),
           reduce, _ptr(grad_logp), ld, _ptr(grad_v), _stream(stream))
 
@@ -305,7 +317,18 @@ def ff_group_advantage(rewards, G: int, eps_A: float, adv, stream=None):
     n = rewards.numel()
     if n % G:
         raise ValueError("rewards.numel() must be a multiple of G")
+    _need(adv, n, "adv")
     _call("ff_group_advantage", n // G, G, _ptr(rewards), eps_A, _ptr(adv), _stream(stream))
+
+
+def _loss_sizes(B, T, lp_old, adv, loss, grad):
+    import torch
+    _need(lp_old, B * T, "lp_old")
+    _need(adv, B, "adv")
+    _need(loss, 1, "loss")
+    if grad is not None:
+        _check(grad, torch.float32, "grad_lp_new")
+        _need(grad, B * T, "grad_lp_new")
 
 
 def ff_grpo_loss(lp_new, lp_old, adv, clip_lo: float, clip_hi: float, loss, grad_lp_new=None, ws=None,
@@ -314,8 +337,9 @@ def ff_grpo_loss(lp_new, lp_old, adv, clip_lo: float, clip_hi: float, loss, grad
     B, T = lp_new.shape
     for n_, a in (("lp_new", lp_new), ("lp_old", lp_old), ("adv", adv), ("loss", loss)):
         _check(a, torch.float32, n_)
+    _loss_sizes(B, T, lp_old, adv, loss, grad_lp_new)
     if ws is None:
-        ws = torch.empty(ff_grpo_loss_workspace_size(B, T), dtype=torch.uint8, device=lp_new.device)
+        ws = torch.zeros(ff_grpo_loss_workspace_size(B, T), dtype=torch.uint8, device=lp_new.device)
     _call("ff_grpo_loss", B, T, _ptr(lp_new), _ptr(lp_old), _ptr(adv), clip_lo, clip_hi, _ptr(loss),
           _ptr(grad_lp_new), _ptr(ws), ws.numel(), _stream(stream))
 
@@ -326,8 +350,10 @@ def ff_grpo_loss_weighted(lp_new, lp_old, adv, step_w, clip_lo: float, clip_hi: 
     B, T = lp_new.shape
     for n_, a in (("lp_new", lp_new), ("lp_old", lp_old), ("adv", adv), ("step_w", step_w), ("loss", loss)):
         _check(a, torch.float32, n_)
+    _loss_sizes(B, T, lp_old, adv, loss, grad_lp_new)
+    _need(step_w, T, "step_w")
     if ws is None:
-        ws = torch.empty(ff_grpo_loss_workspace_size(B, T), dtype=torch.uint8, device=lp_new.device)
+        ws = torch.zeros(ff_grpo_loss_workspace_size(B, T), dtype=torch.uint8, device=lp_new.device)
     _call("ff_grpo_loss_weighted", B, T, _ptr(lp_new), _ptr(lp_old), _ptr(adv), _ptr(step_w), clip_lo, clip_hi,
           _ptr(loss), _ptr(grad_lp_new), _ptr(ws), ws.numel(), _stream(stream))
 
@@ -357,6 +383,9 @@ def ff_forward_process(x0, eps, t, x_t, stream=None):
     for n_, a in (("x0", x0), ("eps", eps), ("t", t), ("x_t", x_t)):
         _check(a, torch.float32, n_)
     B = x0.shape[0]
+    for n_, a in (("eps", eps), ("x_t", x_t)):
+        _need(a, x0.numel(), n_)
+    _need(t, B, "t")
     _call("ff_forward_process", B, x0.numel() // B, _ptr(x0), _ptr(eps), _ptr(t), _ptr(x_t), _stream(stream))
 
 
@@ -379,6 +408,11 @@ def ff_nft_loss(v, v_old, eps, x0, r, beta: float, reduce: int, loss, grad_v=Non
         _check(a, torch.float32, n_)
     B = v.shape[0]
     D = v.numel() // B
+    for n_, a in (("v_old", v_old), ("eps", eps), ("x0", x0)) + ((("grad_v", grad_v),) if grad_v is not None else ()):
+        _need(a, B * D, n_)
+    _need(r, B, "r")
+    if err is not None:
+        _need(err, 2 * B, "err")
     if ws is None:
         ws = torch.empty(ff_nft_loss_workspace_size(B, D), dtype=torch.uint8, device=v.device)
     _call("ff_nft_loss", B, D, _ptr(v), _ptr(v_old), _ptr(eps), _ptr(x0), _ptr(r), beta, reduce, _ptr(loss),
@@ -391,6 +425,11 @@ def ff_awm_loss(v, eps, x0, adv, reduce: int, loss, grad_v=None, err=None, ws=No
         _check(a, torch.float32, n_)
     B = v.shape[0]
     D = v.numel() // B
+    for n_, a in (("eps", eps), ("x0", x0)) + ((("grad_v", grad_v),) if grad_v is not None else ()):
+        _need(a, B * D, n_)
+    _need(adv, B, "adv")
+    if err is not None:
+        _need(err, B, "err")
     if ws is None:
         ws = torch.empty(ff_awm_loss_workspace_size(B, D), dtype=torch.uint8, device=v.device)
     _call("ff_awm_loss", B, D, _ptr(v), _ptr(eps), _ptr(x0), _ptr(adv), reduce, _ptr(loss), _ptr(grad_v),

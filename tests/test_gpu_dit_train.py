@@ -250,7 +250,7 @@ def test_grpo_training_step_chain(cuda):
     T = lambda a: torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(dev)
     tg, tng, sg = T(t), T(tn), T(sig)
     lp = torch.empty(B, 1, dtype=torch.float32, device=dev)
-    ws = torch.empty(ffi.ff_sde_workspace_size(B, Ni * Pd), dtype=torch.uint8, device=dev)
+    ws = torch.zeros(ffi.ff_sde_workspace_size(B, Ni * Pd), dtype=torch.uint8, device=dev)
     xn_g = T(x_next)
     ffi.ff_sde_step_logprob(run.xg, run.v, None, xn_g, tg, tng, sg, lp, mode=ffi.FF_SDE_EVAL, ws=ws)
     lp_old = lp + T(synth.logprob_jitter((B, 1), seed=9))

@@ -19,8 +19,8 @@ def test_host_fed_pipeline_matches_serial_steps(cuda):
     D = synth.n_img(cfg) * cfg["patch_dim"]
     v = torch.empty((B, synth.n_img(cfg), cfg["patch_dim"]), dtype=torch.float32, device=cuda)
     ws = torch.empty(model.workspace_size(B), dtype=torch.uint8, device=cuda)
-    ws_sde = torch.empty(ffi.ff_sde_workspace_size(B, D), dtype=torch.uint8, device=cuda)
-    ws_loss = torch.empty(ffi.ff_grpo_loss_workspace_size(B, 1), dtype=torch.uint8, device=cuda)
+    ws_sde = torch.zeros(ffi.ff_sde_workspace_size(B, D), dtype=torch.uint8, device=cuda)
+    ws_loss = torch.zeros(ffi.ff_grpo_loss_workspace_size(B, 1), dtype=torch.uint8, device=cuda)
     adv = torch.empty(B, dtype=torch.float32, device=cuda)
     grad = torch.empty((B, 1), dtype=torch.float32, device=cuda)
 

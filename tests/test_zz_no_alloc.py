@@ -57,9 +57,14 @@ def test_noalloc_matches_workspace_entry_point_on_consecutive_calls(cuda):
 def test_noalloc_rejects_sizes_beyond_its_scratch(cuda):
     from paper_2602_12529_gb300 import ffi
     lib = ffi.lib()
-    # 65536 partial sums at most, 1024 per sample once D >= 2^22: B = 128
-    # samples of 2^23 elements need 131072 -> rejected on the host, before
-    # any launch (the pointers here are placeholders and are never used)
-    rc = lib.ff_sde_step_logprob_noalloc(128, 1 << 23, 16, 16, 16, 16, 16, 16, 16, 0, 0, 16, 1, None)
+    # the scratch limits are checked before the pointers, so these calls pass
+    # no pointers at all and can never reach a launch
+    # 65536 partial sums at most, 1024 per sample once D >= 2^21: 128
+    # samples of 2^23 elements need 131072
+    rc = lib.ff_sde_step_logprob_noalloc(128, 1 << 23, None, None, None, None, None, None, None, 0, 0, None, 1, None)
+    assert rc == 2
+    assert b"scratch" in lib.ff_last_error()
+    # 4096 ticket counters at most
+    rc = lib.ff_sde_step_logprob_noalloc(4097, 4, None, None, None, None, None, None, None, 0, 0, None, 1, None)
     assert rc == 2
     assert b"scratch" in lib.ff_last_error()
