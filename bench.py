@@ -53,7 +53,13 @@ def parse_args():
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default=WORKLOAD)
     p.add_argument("--no-cpu-baseline", action="store_true")
-    p.add_argument("--no-sweep", action="store_true", help="skip the HBM bandwidth sweep of the memory-bound kernels")
+    p.add_argument("--no-sweep", action="store_true",
+                   help="skip the extra measurements (other workloads, training, sweeps)")
+    p.add_argument("--profile-kernel", default=None,
+                   choices=["sde_step", "sde_step_philox", "grpo_loss", "group_advantage", "ln_modulate",
+                            "attention", "velocity"],
+                   help="launch only this kernel (a few times, no timing) for an ncu capture")
+    p.add_argument("--elements", type=int, default=1 << 24, help="problem size of --profile-kernel's HBM kernels")
     return p.parse_args()
 
 
@@ -1087,10 +1093,99 @@ def run_ours(args):
     return 0
 
 
+def profile_kernel(args):
+    """Launch one kernel `reps` times on rotating inputs, for an ncu capture
+    (`-k regex:<kernel> -s <skip> -c <count>`); prints what it launched.
+    HBM kernels run at --elements elements (two input sets, each larger
+    than L2 at the default 2^24); attention and LN-modulate at the
+    workload's own shapes; velocity is one whole velocity call."""
+    import torch
+
+    import synth
+    from paper_2602_12529_gb300 import build, ffi
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    build.build()
+    ffi.lib()
+    n, k, reps = args.elements, args.profile_kernel, 4
+    cfg = synth.config(args.workload)
+    g = torch.Generator(device=dev)
+    g.manual_seed(3)
+    rnd = lambda *shape: torch.randn(*shape, generator=g, device=dev)
+    if k in ("sde_step", "sde_step_philox"):
+        B, D = 4, n // 4
+        sets = [tuple(rnd(B, D) for _ in range(4)) for _ in range(2)]
+        t, tn, sg = torch.full((B,), 0.75, device=dev), torch.full((B,), 0.5, device=dev), torch.full((B,), 0.7,
+                                                                                                      device=dev)
+        lp = torch.empty(B, device=dev)
+        ws = torch.zeros(ffi.ff_sde_workspace_size(B, D), dtype=torch.uint8, device=dev)
+        for i in range(reps):
+            x, v, e, o = sets[i % 2]
+            if k == "sde_step":
+                ffi.ff_sde_step_logprob(x, v, e, o, t, tn, sg, lp, ws=ws)
+            else:
+                ffi.ff_sde_step_logprob_philox(x, v, o, t, tn, sg, lp, 7, 0, ws=ws)
+        what = f"{k}: B 4 x D {D} fp32 ({(16 if k == 'sde_step' else 12) * n / 1e6:.0f} MB per launch)"
+    elif k == "grpo_loss":
+        Bq, T = n // 16, 16
+        sets = []
+        for _ in range(2):
+            a = rnd(Bq, T)
+            sets.append((a, a + 0.01 * rnd(Bq, T), rnd(Bq), torch.empty_like(a)))
+        loss = torch.empty(1, device=dev)
+        ws = torch.zeros(ffi.ff_grpo_loss_workspace_size(Bq, T), dtype=torch.uint8, device=dev)
+        for i in range(reps):
+            a, b, adv, gr = sets[i % 2]
+            ffi.ff_grpo_loss(a, b, adv, 0.2, 0.2, loss, gr, ws=ws)
+        what = f"grpo_loss with dL/dlp: B {Bq} x T {T} ({(12 * n + 4 * Bq) / 1e6:.0f} MB per launch)"
+    elif k == "group_advantage":
+        sets = [(torch.rand(n, generator=g, device=dev), torch.empty(n, device=dev)) for _ in range(2)]
+        for i in range(reps):
+            ffi.ff_group_advantage(sets[i % 2][0], 16, 1e-4, sets[i % 2][1])
+        what = f"group_advantage: {n} rewards in groups of 16 ({8 * n / 1e6:.0f} MB per launch)"
+    elif k == "ln_modulate":
+        rows, H = cfg["batch"] * (synth.n_img(cfg) + cfg["n_txt"]), cfg["hidden"]
+        x = rnd(rows, H)
+        mods = rnd(cfg["batch"], 2 * H)
+        out = torch.empty(rows, H, dtype=torch.bfloat16, device=dev)
+        for _ in range(reps):
+            ffi.ff_debug_ln_modulate(x, mods, 0, H, rows // cfg["batch"], out)
+        what = f"ln_modulate: {rows} rows x {H} fp32 -> bf16 ({6 * rows * H / 1e6:.0f} MB per launch)"
+    elif k == "attention":
+        B, heads, d = cfg["batch"], cfg["heads"], cfg["head_dim"]
+        H = heads * d
+        if cfg.get("arch") == "wan":
+            n0, n1 = 0, synth.n_img(cfg)
+        else:
+            n0, n1 = cfg["n_txt"], synth.n_img(cfg)
+        q0 = rnd(max(B * n0, 1), 3 * H).to(torch.bfloat16)
+        q1 = rnd(B * n1, 3 * H).to(torch.bfloat16)
+        o0 = torch.empty(max(B * n0, 1), H, dtype=torch.bfloat16, device=dev)
+        o1 = torch.empty(B * n1, H, dtype=torch.bfloat16, device=dev)
+        for _ in range(reps):
+            ffi.ff_attention_forward(B, heads, d, q0, o0, n0, q1, o1, n1)
+        what = f"attention: B {B}, {heads} x {d} heads, {n0} + {n1} tokens"
+    else:
+        model, blob, _ = make_model(ffi, cfg, dev)
+        si = StepInputs(ffi, cfg, dev, 0)
+        v = torch.empty_like(si.x)
+        ws = torch.empty(model.workspace_size(si.B), dtype=torch.uint8, device=dev)
+        for _ in range(2):
+            model.ff_dit_velocity(si.x, si.txt, si.t, v, ws)
+        what = f"velocity: {workload_desc(cfg)} (2 calls)"
+        reps = 2
+    torch.cuda.synchronize(dev)
+    print(json.dumps({"profile_kernel": k, "launches": reps, "what": what,
+                      "device_status": ffi.ff_check_device_status()}), flush=True)
+    return 0
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
         return run_reference(args)
+    if args.profile_kernel:
+        return profile_kernel(args)
     return run_ours(args)
 
 

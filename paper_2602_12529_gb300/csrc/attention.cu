@@ -20,31 +20,44 @@
 //               (M 128, N d, A = P from TMEM, B = V from shared memory) ->
 //               S_t,j+1; the two tiles alternate, so the tensor core works on
 //               one tile while the other tile's softmax runs.  Keeping P in
-//               TMEM halves the shared-memory operand traffic of P V, which
-//               is what bounds narrow MMAs.
+//               TMEM halves the shared-memory operand traffic of P V.
 //   warps 2..9  two softmax warpgroups, one per query tile: thread = query
-//               row = TMEM lane.  Reads its S row, keeps the running max /
-//               sum in base 2 (log2 e folded into the scale), writes
-//               P = exp2(S - m) as bf16 pairs over the S columns, and
-//               rescales its O row in TMEM only when the running max grows by
-//               more than 8 (2^8 headroom), which makes corrections rare.
-//               Finally O / l goes out as bf16.
+//               row = TMEM lane.  Reads its S row (one 128-column TMEM load),
+//               writes P = exp2(S scale - m) as bf16 pairs over the S
+//               columns and keeps the row sum l; O / l goes out as bf16.
+//
+// The MMA thread's instruction stream is what bounds this kernel: the tensor
+// pipe's queue is short, so every barrier wait or commit the thread executes
+// between MMA batches leaves the pipe idle unless it is short.  Hence:
+//   * the K/V ring is signalled in groups: group 0 = K_0, group j + 1 =
+//     (V_j, K_j+1), the operands of step j's MMAs, one barrier arrival pair
+//     per group (ring of four barriers), so the MMA thread waits once per
+//     step for its operands;
+//   * slots are released by the commit that already publishes S_1,j+1 to
+//     tile 1's softmax (a ring of four barriers, one per step): when S_1,j+1
+//     is done, every MMA of step j is done, so V_j and K_j+1 may be
+//     overwritten.  Step j's MMA thread work is two waits for P, one wait
+//     for the operand group and two commits;
+//   * the softmax keeps its first tile's row maximum m as the reference for
+//     every later tile (softmax does not depend on the reference, and P in
+//     bf16 / l in fp32 lose nothing when later scores exceed m), so only
+//     the first tile pays for a max pass.  A tile whose row sum passes 2^40
+//     (or overflows) is redone against its true maximum, rescaling l and O,
+//     which keeps every P at or below 2^40.
 // Every wait is bounded; on a timeout the kernel records the status word,
 // drains its tensor-core work, frees TMEM and returns.  The MMA and softmax
 // loops do not poll the abort flag: a role that gave up stops signalling, so
-// the others run into their own bounded waits, and a shared-memory load per
-// step would queue behind the S = Q K^T operand reads, which take nearly all
-// of the shared-memory bandwidth while they run.
+// the others run into their own bounded waits.
 #include "internal.h"
 #include "ptx.cuh"
 
 namespace ff {
 namespace {
 
+
 constexpr int kBM = 128;         // query rows per query tile (two tiles per CTA)
 constexpr int kBN = 128;         // tokens per K/V tile
 constexpr int kThreads = 320;    // producer, MMA, 2 x 4 softmax warps
-constexpr float kRescaleThreshold = 8.0f;   // log2 units
 
 template <int HD>
 struct ACfg {
@@ -74,15 +87,20 @@ struct AttnParams {
 };
 
 // Barriers.  Per query tile the chain S -> softmax -> P -> O += P V -> next S
-// is strictly ordered, so no waiter can lag two phases behind a parity wait.
+// is strictly ordered.  A parity wait is unambiguous as long as its barrier
+// cannot complete two phases past the one waited for: the two-phase
+// barriers below are waited in lockstep with their producer, and the rings
+// of four are waited at most one step behind (ring item n = 2 j (K_j) or
+// 2 j + 1 (V_j) lives in slot n % kSlots and belongs to group (n + 1) / 2).
 constexpr int kMaxSlots = 8;
 struct Bars {
     uint64_t q_full;
-    uint64_t slot_full[kMaxSlots];    // ring item n = 2 j (K_j) or 2 j + 1 (V_j) lives in slot n % kSlots
-    uint64_t slot_empty[kMaxSlots];
-    uint64_t s_full[2];       // [query tile] MMA -> softmax: S_t,j is in TMEM (and O += P V_{j-1} done)
-    uint64_t p_full[2];       //              softmax -> MMA: P_t,j is in TMEM, O rescaled
-    uint64_t o_last[2];       //              MMA -> softmax: the last O += P V has landed
+    uint64_t grp_full[4];     // producer -> MMA: K/V group g landed (ring entry g % 4; two arrivals)
+    uint64_t s0_full;         // MMA -> softmax 0: S_0,j is in TMEM (and O_0 += P V_{j-1} done)
+    uint64_t s1_ring[4];      // MMA -> softmax 1 and producer: S_1,j done (ring entry j % 4), so
+                              // every MMA up to step j - 1 is done and its K/V slots are free
+    uint64_t p_full[2];       // softmax -> MMA: P_t,j is in TMEM, O_t rescaled if needed
+    uint64_t o_last[2];       // MMA -> softmax: the last O += P V has landed
     uint64_t drain;
     uint32_t tmem_slot;
     int abort_flag;
@@ -119,12 +137,12 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
             *abort_flag = 1;
         }
         mbar_init(&bar.q_full, 1);
-        for (int s = 0; s < S; ++s) {
-            mbar_init(&bar.slot_full[s], 1);
-            mbar_init(&bar.slot_empty[s], 1);
+        for (int g = 0; g < 4; ++g) {
+            mbar_init(&bar.grp_full[g], 2);
+            mbar_init(&bar.s1_ring[g], 1);
         }
+        mbar_init(&bar.s0_full, 1);
         for (int t = 0; t < 2; ++t) {
-            mbar_init(&bar.s_full[t], 1);
             mbar_init(&bar.p_full[t], 4);
             mbar_init(&bar.o_last[t], 1);
         }
@@ -161,16 +179,25 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
                             b * p.nq[seg] + q0 + t * kBM);
         for (int n = 0; n < 2 * ntiles && !*abort_flag; ++n) {
             const int s = n % S;
-            if (!mbar_wait(&bar.slot_empty[s], ((n / S) & 1) ^ 1)) { fail(); break; }
+            // item n - S (group c = (n - S + 1) / 2) leaves slot s once the
+            // MMAs of group c are done, i.e. once S_1,c is done (S_1,c is the
+            // last MMA of step c - 1, and K_0's only readers are S_0,0 and
+            // S_1,0)
+            if (n >= S) {
+                const int c = (n - S + 1) >> 1;
+                if (!mbar_wait(&bar.s1_ring[c & 3], (c >> 2) & 1)) { fail(); break; }
+            }
+            uint64_t* fb = &bar.grp_full[((n + 1) >> 1) & 3];
             const int j = n >> 1;
             const int ks = j < nt0 ? 0 : 1;
             const int row = b * p.nkv[ks] + (j - (ks ? nt0 : 0)) * kBN;
             const CUtensorMap* tkv = ks ? &tm_kv1 : &tm_kv0;
             const int col = ((n & 1) ? p.v_col : p.k_col) + h * HD;
             uint8_t* dst = sKV + s * C::kKBytes;
-            mbar_arrive_expect_tx(&bar.slot_full[s], C::kKBytes);
+            mbar_arrive_expect_tx(fb, C::kKBytes);
             for (int c = 0; c < HD / 64; ++c)
-                tma_load_2d(dst + c * (kBN * 128), tkv, &bar.slot_full[s], col + c * 64, row);
+                tma_load_2d(dst + c * (kBN * 128), tkv, fb, col + c * 64, row);
+            if (n == 0 || n == 2 * ntiles - 1) mbar_arrive(fb);   // one-item groups: the second arrival
         }
     } else if (warp == 1 && lane == 0) {
         // ------------------------------------------------------------ MMA issuer
@@ -178,14 +205,14 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
         // S_t,j+1.  The two tiles interleave so one tile's MMAs run while the
         // other tile's softmax works.  tcgen05.mma from one thread executes in
         // issue order, so S_t,j+1 overwrites the columns of P_t,j only after
-        // O_t += P_t,j V_j has read them.  K_0 is released once both S_t,0 are
-        // done, V_j and K_j+1 together after step j.
+        // O_t += P_t,j V_j has read them.  Operand group j + 1 (V_j, K_j+1)
+        // is awaited once per step, before O_0 += P_0,j V_j.
         constexpr uint32_t idesc_s = idesc_bf16_f32(kBM, kBN);
         constexpr uint32_t idesc_o = idesc_bf16_f32(kBM, HD) | (1u << 16);   // B (V) is MN-major
         bool ok = mbar_wait(&bar.q_full, 0);
         if (!ok) fail();
-        auto slot_ready = [&](int n) {
-            if (!mbar_wait(&bar.slot_full[n % S], (n / S) & 1)) return false;
+        auto group_ready = [&](int g) {
+            if (!mbar_wait(&bar.grp_full[g & 3], (g >> 2) & 1)) return false;
             tc_fence_after();
             return true;
         };
@@ -204,12 +231,12 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
                 const uint32_t off_k = ((k / 4) * (kBN * 128) + (k % 4) * 32) >> 4;
                 tc_mma_bf16(dS, dq + off_q, dk + off_k, idesc_s, k != 0 ? 1u : 0u);
             }
-            tc_commit(&bar.s_full[t]);
+            tc_commit(t == 0 ? &bar.s0_full : &bar.s1_ring[j & 3]);
         };
         auto issue_pv = [&](int t, int j) -> bool {
+            if (t == 0 && !group_ready(j + 1)) return false;   // V_j and K_j+1
             if (!mbar_wait(&bar.p_full[t], j & 1)) return false;
             tc_fence_after();
-            if (t == 0 && !slot_ready(2 * j + 1)) return false;
             const uint64_t dv = smem_desc_mn_sw128(smem_u32(sKV + ((2 * j + 1) % S) * C::kKBytes), kBN * 128);
             const uint32_t dO = tmem + t * 256 + C::kColO;
             const uint32_t aP = tmem + t * 256;
@@ -220,25 +247,19 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
             return true;
         };
         if (ok && ntiles > 0) {
-            if (!slot_ready(0)) { fail(); ok = false; }
+            if (!group_ready(0)) { fail(); ok = false; }
             else {
                 issue_s(0, 0);
                 issue_s(1, 0);
-                tc_commit(&bar.slot_empty[0]);
             }
         }
         for (int j = 0; ok && j < ntiles; ++j) {
             const bool more = j + 1 < ntiles;
             for (int t = 0; t < 2; ++t) {
                 if (!issue_pv(t, j)) { fail(); ok = false; break; }
-                if (more) {
-                    if (t == 0 && !slot_ready(2 * j + 2)) { fail(); ok = false; break; }
-                    issue_s(t, j + 1);
-                }
+                if (more) issue_s(t, j + 1);
             }
             if (!ok) break;
-            tc_commit(&bar.slot_empty[(2 * j + 1) % S]);
-            if (more) tc_commit(&bar.slot_empty[(2 * j + 2) % S]);
         }
         if (ok) {
             tc_commit(&bar.o_last[0]);
@@ -258,11 +279,14 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
         bool ok = true;
         for (int j = 0; j < ntiles; ++j) {
             // S_t,j ready; O_t += P_t,j-1 V_j-1 has completed as well
-            if (!mbar_wait(&bar.s_full[t], j & 1)) { fail(); ok = false; break; }
+            if (!(t == 0 ? mbar_wait(&bar.s0_full, j & 1) : mbar_wait(&bar.s1_ring[j & 3], (j >> 2) & 1))) {
+                fail();
+                ok = false;
+                break;
+            }
             tc_fence_after();
             uint32_t sr[kBN];
-#pragma unroll
-            for (int c = 0; c < kBN; c += 32) tmem_ld_x32(tS + c, *reinterpret_cast<uint32_t(*)[32]>(&sr[c]));
+            tmem_ld_x128(tS, sr);
             tmem_ld_wait();
 
             const int ks = j < nt0 ? 0 : 1;
@@ -272,35 +296,54 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
                 for (int i = 0; i < kBN; ++i)
                     if (i >= valid) sr[i] = __float_as_uint(-INFINITY);
             }
-            float mc[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+            auto row_max = [&]() {
+                float mc[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-            for (int i = 0; i < kBN; i += 8) {
+                for (int i = 0; i < kBN; i += 8) {
 #pragma unroll
-                for (int k = 0; k < 4; ++k)
-                    mc[k] = max3(mc[k], __uint_as_float(sr[i + 2 * k]), __uint_as_float(sr[i + 2 * k + 1]));
-            }
-            const float mx = max3(mc[0], mc[1], fmaxf(mc[2], mc[3])) * p.scale_log2;
-            const bool grow = mx > m_used + kRescaleThreshold;
-            const float m_new = grow ? mx : m_used;
-            const float alpha = ex2(m_used - m_new);   // 0 on the first tile, 1 without growth
-            const float2 c2 = make_float2(p.scale_log2, p.scale_log2);
-            const float2 nm2 = make_float2(-m_new, -m_new);
-            float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
-                             make_float2(0.f, 0.f)};
+                    for (int k = 0; k < 4; ++k)
+                        mc[k] = max3(mc[k], __uint_as_float(sr[i + 2 * k]), __uint_as_float(sr[i + 2 * k + 1]));
+                }
+                return max3(mc[0], mc[1], fmaxf(mc[2], mc[3])) * p.scale_log2;
+            };
+            // P = exp2(S scale - m) packed over the front of sr; returns the row sum
+            auto exps = [&](float m) {
+                const float2 c2 = make_float2(p.scale_log2, p.scale_log2);
+                const float2 nm2 = make_float2(-m, -m);
+                float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                                 make_float2(0.f, 0.f)};
 #pragma unroll
-            for (int i = 0; i < kBN; i += 2) {
-                const float2 x = __ffma2_rn(make_float2(__uint_as_float(sr[i]), __uint_as_float(sr[i + 1])), c2, nm2);
-                const float2 e = make_float2(ex2(x.x), ex2(x.y));
-                acc[(i >> 1) & 3] = __fadd2_rn(acc[(i >> 1) & 3], e);
-                sr[i / 2] = pack_bf16x2(e.x, e.y);   // P packed over the front of the S registers
-            }
-            const float2 a01 = __fadd2_rn(acc[0], acc[1]);
-            const float2 a23 = __fadd2_rn(acc[2], acc[3]);
-            l = l * alpha + ((a01.x + a01.y) + (a23.x + a23.y));
-            m_used = m_new;
-            // a grown max rescales this warp's O rows (O is stable: its last
-            // update completed before S_t,j was published)
-            if (j >= 1 && __any_sync(0xffffffffu, grow)) {
+                for (int i = 0; i < kBN; i += 2) {
+                    const float2 x = __ffma2_rn(make_float2(__uint_as_float(sr[i]), __uint_as_float(sr[i + 1])), c2, nm2);
+                    const float2 e = make_float2(ex2(x.x), ex2(x.y));
+                    acc[(i >> 1) & 3] = __fadd2_rn(acc[(i >> 1) & 3], e);
+                    sr[i / 2] = pack_bf16x2(e.x, e.y);
+                }
+                const float2 a01 = __fadd2_rn(acc[0], acc[1]);
+                const float2 a23 = __fadd2_rn(acc[2], acc[3]);
+                return (a01.x + a01.y) + (a23.x + a23.y);
+            };
+            // Softmax is unchanged by the reference m subtracted before the
+            // exponentials, so after the first tile the row keeps its first
+            // maximum as the reference and skips the max pass.  Later scores
+            // may exceed it: P up to 2^40 is exact enough in bf16 / fp32, and
+            // a tile whose row sum passes 2^40 (or overflows) is redone with
+            // the true maximum, rescaling l and O.
+            if (j == 0) m_used = row_max();
+            float lt = exps(m_used);
+            if (j > 0 && __any_sync(0xffffffffu, !(lt <= 0x1p40f))) {
+                tmem_ld_x128(tS, sr);
+                tmem_ld_wait();
+                if (valid < kBN) {
+#pragma unroll
+                    for (int i = 0; i < kBN; ++i)
+                        if (i >= valid) sr[i] = __float_as_uint(-INFINITY);
+                }
+                const float m_new = fmaxf(m_used, row_max());
+                const float alpha = ex2(m_used - m_new);
+                lt = exps(m_new);
+                l *= alpha;
+                m_used = m_new;
 #pragma unroll 1
                 for (int c = 0; c < HD; c += 32) {
                     uint32_t o[32];
@@ -311,6 +354,7 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
                     tmem_st_x32(tO + c, o);
                 }
             }
+            l += lt;
             // P_t,j (bf16 pairs) over the first kBN/2 columns of S_t
 #pragma unroll
             for (int c = 0; c < kBN / 2; c += 32) tmem_st_x32(tS + c, &sr[c]);

@@ -181,23 +181,24 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_partial_kernel(int64_t n, 
         s += term(lp_new[i], lp_old[i], static_cast<uint32_t>(i), g);
         if (grad) grad[i] = g;
     }
-    double d = s;
+    // fp32 within the block (fp64 arithmetic is slow on this part), fp64
+    // across blocks
 #pragma unroll
-    for (int o = 16; o; o >>= 1) d += __shfl_xor_sync(0xffffffffu, d, o);
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = d;
+    for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    __shared__ float redf[kThreads / 32];
+    if ((threadIdx.x & 31) == 0) redf[threadIdx.x >> 5] = s;
     __syncthreads();
     __shared__ bool last;
     if (threadIdx.x == 0) {
-        double t = 0.0;
-        for (int w = 0; w < kThreads / 32; ++w) t += red[w];
-        partial[blockIdx.x] = t;
-        __threadfence();                                   // partial visible before the ticket
-        last = atomicAdd(ticket, 1u) == gridDim.x - 1;
+        float t = 0.f;
+        for (int w = 0; w < kThreads / 32; ++w) t += redf[w];
+        partial[blockIdx.x] = static_cast<double>(t);
+        last = ticket_add_acq_rel(ticket, 1u) == gridDim.x - 1;
     }
     __syncthreads();
     if (!last) return;
-    // every partial is stored: add them in index order
-    __threadfence();
+    // every partial is stored (the last ticket acquired them): add them in
+    // index order
     double acc = 0.0;
     for (int i = threadIdx.x; i < static_cast<int>(gridDim.x); i += kThreads) acc += __ldcg(partial + i);
 #pragma unroll

@@ -23,24 +23,40 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kModePhilox = 2;                                // SAMPLE, eps from rng.cuh (internal mode)
-constexpr int kVecPerThread = 2;                              // float4 per thread per chunk
-constexpr int kChunk = kThreads * kVecPerThread * 4;          // 2048 elements
+constexpr int kVecPerThread = 4;                              // float4 per thread per chunk
+constexpr int kChunk = kThreads * kVecPerThread * 4;          // 4096 elements
 
 struct StepCoef {
     float cx, cv, std;
 };
 
+// Per-sample coefficients in fp32 (every thread forms its own: no barrier,
+// and fp64 arithmetic is slow on this part).  Relative error a few ulp.
 __device__ __forceinline__ StepCoef step_coef(const float* t, const float* t_next, const float* sigma, int b) {
-    const double tt = t[b];
-    const double tn = t_next[b];
-    const double sg = sigma[b];
-    const double delta = tt - tn;
-    const double a = sg * sg / (2.0 * tt);
+    const float tt = __ldg(t + b);
+    const float tn = __ldg(t_next + b);
+    const float sg = __ldg(sigma + b);
+    const float delta = tt - tn;
+    const float a = sg * sg / (2.0f * tt);
     StepCoef c;
-    c.cx = static_cast<float>(1.0 - delta * a);
-    c.cv = static_cast<float>(-delta * (1.0 + a * (1.0 - tt)));
-    c.std = static_cast<float>(sg * sqrt(delta));
+    c.cx = fmaf(-delta, a, 1.0f);
+    c.cv = -delta * fmaf(a, 1.0f - tt, 1.0f);
+    c.std = sg * sqrtf(delta);
     return c;
+}
+
+// Sum over the block in fp32 (shuffles, then the warps' sums in order by
+// thread 0); valid in thread 0.
+__device__ __forceinline__ float block_sum_f32(float v, float* red) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+    __syncthreads();
+    float s = 0.f;
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < (int)(blockDim.x >> 5); ++i) s += red[i];
+    }
+    return s;
 }
 
 __device__ __forceinline__ double block_sum(double v, double* red) {
@@ -73,9 +89,9 @@ __device__ __forceinline__ float logprob_of(double ss, int64_t D, const float* t
 }
 
 // Grid (blocks_per_sample, B); block k of sample b handles chunks
-// k, k + blocks_per_sample, ... and writes one fp64 partial.  The number of
-// blocks per sample depends only on D (see nchunks), so the summation order
-// is fixed.  The per-sample coefficients are formed once per block in fp64.
+// k, k + blocks_per_sample, ... and writes one partial (fp32 within the
+// block, stored as fp64).  The number of blocks per sample depends only on D
+// (see nchunks), so the summation order is fixed.
 // ticket[b] counts the blocks of sample b that have stored their partial; it
 // is zero on entry and the last block of the sample sets it back to zero.
 template <int MODE>
@@ -85,12 +101,10 @@ __global__ void __launch_bounds__(kThreads) sde_step_partial_kernel(int64_t D, i
                                                                     const float* sigma, double* partial,
                                                                     unsigned* ticket, int reduce, float* logp, int ld,
                                                                     PhiloxKey key, uint32_t rng_stream) {
+    __shared__ float redf[kThreads / 32];
     __shared__ double red[kThreads / 32];
-    __shared__ StepCoef coef;
     const int b = blockIdx.y;
-    if (threadIdx.x == 0) coef = step_coef(t, t_next, sigma, b);
-    __syncthreads();
-    const StepCoef c = coef;
+    const StepCoef c = step_coef(t, t_next, sigma, b);
     const int64_t row = static_cast<int64_t>(b) * D;
     const float4* x4 = reinterpret_cast<const float4*>(x + row);
     const float4* v4 = reinterpret_cast<const float4*>(v + row);
@@ -100,16 +114,25 @@ __global__ void __launch_bounds__(kThreads) sde_step_partial_kernel(int64_t D, i
     float ss = 0.f;
     for (int64_t base = static_cast<int64_t>(blockIdx.x) * (kChunk / 4); base < nvec;
          base += static_cast<int64_t>(nblk) * (kChunk / 4)) {
+        // every load of the chunk is issued before any arithmetic; the
+        // inputs keep the default cache policy (a rollout's v and x_t are
+        // often still in L2) and so does x_next (the next step reads it)
         float4 xv[kVecPerThread], vv[kVecPerThread], ev[kVecPerThread];
 #pragma unroll
         for (int j = 0; j < kVecPerThread; ++j) {
             const int64_t i = base + threadIdx.x + j * kThreads;
             if (i < nvec) {
-                xv[j] = __ldcs(x4 + i);
-                vv[j] = __ldcs(v4 + i);
-                if (MODE == FF_SDE_SAMPLE) ev[j] = __ldcs(e4 + i);
-                else if (MODE == kModePhilox) ev[j] = philox_normal4(static_cast<uint32_t>(i), b, rng_stream, key);
-                else ev[j] = __ldcs(reinterpret_cast<const float4*>(n4) + i);
+                xv[j] = __ldg(x4 + i);
+                vv[j] = __ldg(v4 + i);
+                if (MODE == FF_SDE_SAMPLE) ev[j] = __ldg(e4 + i);
+                else if (MODE == FF_SDE_EVAL) ev[j] = *(reinterpret_cast<const float4*>(n4) + i);
+            }
+        }
+        if (MODE == kModePhilox) {
+#pragma unroll
+            for (int j = 0; j < kVecPerThread; ++j) {
+                const int64_t i = base + threadIdx.x + j * kThreads;
+                if (i < nvec) ev[j] = philox_normal4(static_cast<uint32_t>(i), b, rng_stream, key);
             }
         }
 #pragma unroll
@@ -124,7 +147,7 @@ __global__ void __launch_bounds__(kThreads) sde_step_partial_kernel(int64_t D, i
                     o[1] = fmaf(c.std, ev[j].y, m[1]);
                     o[2] = fmaf(c.std, ev[j].z, m[2]);
                     o[3] = fmaf(c.std, ev[j].w, m[3]);
-                    __stcs(n4 + i, make_float4(o[0], o[1], o[2], o[3]));
+                    n4[i] = make_float4(o[0], o[1], o[2], o[3]);
                 } else {
                     o[0] = ev[j].x; o[1] = ev[j].y; o[2] = ev[j].z; o[3] = ev[j].w;
                 }
@@ -136,17 +159,16 @@ __global__ void __launch_bounds__(kThreads) sde_step_partial_kernel(int64_t D, i
             }
         }
     }
-    const double s = block_sum(static_cast<double>(ss), red);
+    const float s = block_sum_f32(ss, redf);
     __shared__ bool last;
     if (threadIdx.x == 0) {
-        partial[static_cast<int64_t>(b) * nblk + blockIdx.x] = s;
-        __threadfence();                                   // partial visible before the ticket
-        last = atomicAdd(ticket + b, 1u) == static_cast<unsigned>(nblk - 1);
+        partial[static_cast<int64_t>(b) * nblk + blockIdx.x] = static_cast<double>(s);
+        last = ticket_add_acq_rel(ticket + b, 1u) == static_cast<unsigned>(nblk - 1);
     }
     __syncthreads();
     if (!last) return;
-    // every partial of sample b is stored; add them in index order
-    __threadfence();
+    // every partial of sample b is stored (the last ticket acquired them);
+    // add them in index order
     const double* pb = partial + static_cast<int64_t>(b) * nblk;
     double acc = 0.0;
     for (int i = threadIdx.x; i < nblk; i += kThreads) acc += __ldcg(pb + i);
@@ -223,7 +245,7 @@ constexpr int kMaxSamples = 65535;
 constexpr size_t kTicketBytes = 256 * 1024;
 static_assert(kTicketBytes >= sizeof(unsigned) * kMaxSamples, "ticket region too small");
 
-// partial sums (blocks) per sample: one per 2048-element chunk up to 1024,
+// partial sums (blocks) per sample: one per 4096-element chunk up to 1024,
 // then every block loops over several chunks
 int nchunks(int64_t D) {
     const int64_t c = (D + kChunk - 1) / kChunk;

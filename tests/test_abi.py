@@ -78,9 +78,9 @@ def test_weight_layout_matches_oracle_parameters(L, name):
 
 def test_workspace_queries(L):
     # SDE: a fixed 256 KiB ticket region, then one fp64 partial per
-    # 2048-element chunk (at most 1024 per sample)
+    # 4096-element chunk (at most 1024 per sample)
     n1 = ffi.ff_sde_workspace_size(4, 262144)
-    assert n1 == 256 * 1024 + 4 * 128 * 8
+    assert n1 == 256 * 1024 + 4 * 64 * 8
     # loss: a 16-byte ticket, then one fp64 partial per block (at most 1216)
     assert ffi.ff_grpo_loss_workspace_size(32, 10) == 16 + 8
     assert ffi.ff_grpo_loss_workspace_size(1 << 20, 64) == 16 + 1216 * 8

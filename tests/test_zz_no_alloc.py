@@ -59,7 +59,7 @@ def test_noalloc_rejects_sizes_beyond_its_scratch(cuda):
     lib = ffi.lib()
     # the scratch limits are checked before the pointers, so these calls pass
     # no pointers at all and can never reach a launch
-    # 65536 partial sums at most, 1024 per sample once D >= 2^21: 128
+    # 65536 partial sums at most, 1024 per sample once D >= 2^22: 128
     # samples of 2^23 elements need 131072
     rc = lib.ff_sde_step_logprob_noalloc(128, 1 << 23, None, None, None, None, None, None, None, 0, 0, None, 1, None)
     assert rc == 2
