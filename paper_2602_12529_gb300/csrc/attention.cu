@@ -81,6 +81,8 @@ struct AttnParams {
     float scale_log2;
     __nv_bfloat16* out[2];
     int64_t ldo[2];
+    __nv_bfloat16* out_lo[2];   // optional: O - bf16(O), rounded to bf16 (training)
+    int64_t ldo_lo[2];
     float* lse;          // optional per-row log-sum-exp (base 2), see AttnSpec
     int lse_rows;        // its row pitch per (sample, head)
     int lse_base[2];     // first row of each query segment
@@ -372,7 +374,9 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
             const bool live = row < p.nq[seg];
             if (p.lse && live)
                 p.lse[(static_cast<int64_t>(b) * gridDim.y + h) * p.lse_rows + p.lse_base[seg] + row] = m_used + log2f(l);
-            __nv_bfloat16* dst = p.out[seg] + (static_cast<int64_t>(b) * p.nq[seg] + row) * p.ldo[seg] + h * HD;
+            const int64_t grow = static_cast<int64_t>(b) * p.nq[seg] + row;
+            __nv_bfloat16* dst = p.out[seg] + grow * p.ldo[seg] + h * HD;
+            __nv_bfloat16* dst_lo = p.out_lo[seg] ? p.out_lo[seg] + grow * p.ldo_lo[seg] + h * HD : nullptr;
 #pragma unroll 1
             for (int c = 0; c < HD; c += 32) {
                 uint32_t o[32];
@@ -381,10 +385,23 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
                 if (live) {
 #pragma unroll
                     for (int k = 0; k < 4; ++k) {
-                        const float* f = reinterpret_cast<const float*>(o) + 8 * k;
-                        *reinterpret_cast<uint4*>(dst + c + 8 * k) =
-                            make_uint4(pack_bf16x2(f[0] * inv, f[1] * inv), pack_bf16x2(f[2] * inv, f[3] * inv),
-                                       pack_bf16x2(f[4] * inv, f[5] * inv), pack_bf16x2(f[6] * inv, f[7] * inv));
+                        float f[8];
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) f[i] = __uint_as_float(o[8 * k + i]) * inv;
+                        const uint4 hi = make_uint4(pack_bf16x2(f[0], f[1]), pack_bf16x2(f[2], f[3]),
+                                                    pack_bf16x2(f[4], f[5]), pack_bf16x2(f[6], f[7]));
+                        *reinterpret_cast<uint4*>(dst + c + 8 * k) = hi;
+                        if (dst_lo) {
+                            // what bf16 dropped, itself in bf16
+                            const uint32_t hw[4] = {hi.x, hi.y, hi.z, hi.w};
+                            uint32_t lw[4];
+#pragma unroll
+                            for (int i = 0; i < 4; ++i) {
+                                const float2 r = unpack_bf16x2(hw[i]);
+                                lw[i] = pack_bf16x2(f[2 * i] - r.x, f[2 * i + 1] - r.y);
+                            }
+                            *reinterpret_cast<uint4*>(dst_lo + c + 8 * k) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+                        }
                     }
                 }
             }
@@ -428,6 +445,8 @@ int launch_attn(const AttnSpec& a, cudaStream_t stream) {
         p.nkv[i] = a.kv[i].n;
         p.out[i] = a.q[i].out;
         p.ldo[i] = a.q[i].ldo;
+        p.out_lo[i] = a.q[i].out_lo;
+        p.ldo_lo[i] = a.q[i].ldo_lo;
     }
     p.qpairs0 = (a.q[0].n + 2 * kBM - 1) / (2 * kBM);
     p.lse = a.lse;
@@ -457,6 +476,8 @@ int attention_general(const AttnSpec& a, cudaStream_t stream) {
         if (a.q[i].n < 0 || a.kv[i].n < 0) return set_error(FF_ERR_INVALID_ARG, "attention: negative token count");
         if (a.q[i].n && (!a.q[i].buf || !a.q[i].out || !aligned16(a.q[i].out) || a.q[i].ld % 8 || a.q[i].ldo % 8))
             return set_error(FF_ERR_INVALID_ARG, "attention: bad query segment %d", i);
+        if (a.q[i].n && a.q[i].out_lo && (!aligned16(a.q[i].out_lo) || a.q[i].ldo_lo % 8))
+            return set_error(FF_ERR_INVALID_ARG, "attention: bad low-part output of query segment %d", i);
         if (a.kv[i].n && (!a.kv[i].buf || a.kv[i].ld % 8))
             return set_error(FF_ERR_INVALID_ARG, "attention: bad key/value segment %d", i);
     }
@@ -481,7 +502,8 @@ int attention(const AttnSegment& s0, const AttnSegment& s1, int B, int heads, in
     a.lse = lse;
     const AttnSegment* seg[2] = {&s0, &s1};
     for (int i = 0; i < 2; ++i) {
-        a.q[i] = AttnQuerySeg{seg[i]->qkv, seg[i]->ld, seg[i]->n, seg[i]->out, seg[i]->ldo};
+        a.q[i] = AttnQuerySeg{seg[i]->qkv, seg[i]->ld, seg[i]->n, seg[i]->out, seg[i]->ldo, seg[i]->out_lo,
+                              seg[i]->ldo_lo};
         a.kv[i] = AttnKvSeg{seg[i]->qkv, seg[i]->ld, seg[i]->n};
     }
     a.q_col = 0;

@@ -94,13 +94,18 @@ __device__ __forceinline__ void store_row_bf16(uint32_t taddr, float mul, __nv_b
     }
 }
 
-// D_i = sum_c dO_ic O_ic: one warp per (token row, head), HD / 32 columns per lane.
+// D_i = sum_c dO_ic O_ic: one warp per (token row, head), HD / 32 columns per
+// lane.  With the forward's low parts (o_lo), O = o + o_lo: D = rowsum(P dP)
+// subtracts nearly equal terms when the rows of V are close to each other,
+// and bf16 O alone would leave a relative error of 2^-9 |dO| |O| in D.
 template <int HD>
 __global__ void __launch_bounds__(256) attn_bwd_delta_kernel(int B, int heads, int n0, int n1,
                                                              const __nv_bfloat16* o0, const __nv_bfloat16* do0,
                                                              const __nv_bfloat16* o1, const __nv_bfloat16* do1,
                                                              int64_t ldo0, int64_t ldo1, int64_t ldg0, int64_t ldg1,
-                                                             int lse_rows, int base1, float* delta) {
+                                                             const __nv_bfloat16* ol0, const __nv_bfloat16* ol1,
+                                                             int64_t ldl0, int64_t ldl1, int lse_rows, int base1,
+                                                             float* delta) {
     const int64_t w = (static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x) >> 5;
     const int lane = threadIdx.x & 31;
     const int64_t rows0 = static_cast<int64_t>(B) * n0;
@@ -116,10 +121,17 @@ __global__ void __launch_bounds__(256) attn_bwd_delta_kernel(int B, int heads, i
     constexpr int E = HD / 32;
     const __nv_bfloat16* o = (s1 ? o1 : o0) + rr * (s1 ? ldo1 : ldo0) + h * HD + lane * E;
     const __nv_bfloat16* g = (s1 ? do1 : do0) + rr * (s1 ? ldg1 : ldg0) + h * HD + lane * E;
+    const __nv_bfloat16* olb = s1 ? ol1 : ol0;
+    const __nv_bfloat16* ol = olb ? olb + rr * (s1 ? ldl1 : ldl0) + h * HD + lane * E : nullptr;
     float s = 0.f;
 #pragma unroll
     for (int e = 0; e < E; e += 2) {
-        const float2 of = unpack_bf16x2(*reinterpret_cast<const uint32_t*>(o + e));
+        float2 of = unpack_bf16x2(*reinterpret_cast<const uint32_t*>(o + e));
+        if (ol) {
+            const float2 lf = unpack_bf16x2(*reinterpret_cast<const uint32_t*>(ol + e));
+            of.x += lf.x;
+            of.y += lf.y;
+        }
         const float2 gf = unpack_bf16x2(*reinterpret_cast<const uint32_t*>(g + e));
         s = fmaf(of.x, gf.x, fmaf(of.y, gf.y, s));
     }
@@ -646,10 +658,11 @@ int attention_backward_hd(const AttnBwdSpec& a, void* ws, size_t ws_bytes, cudaS
     const int rows = attn_lse_rows(nq0, nq1);
     {
         const int64_t warps = (static_cast<int64_t>(B) * (nq0 + nq1)) * heads;
-        ProfScope prof(stream, "attn_bwd_delta", 0.0, 4.0 * warps * HD);
+        const bool lo = a.q[0].o_lo || a.q[1].o_lo;
+        ProfScope prof(stream, "attn_bwd_delta", 0.0, (lo ? 6.0 : 4.0) * warps * HD);
         attn_bwd_delta_kernel<HD><<<static_cast<unsigned>((warps + 7) / 8), 256, 0, stream>>>(
             B, heads, nq0, nq1, a.q[0].o, a.q[0].dout, a.q[1].o, a.q[1].dout, a.q[0].ldo, a.q[1].ldo, a.q[0].ldg,
-            a.q[1].ldg, rows, attn_pad128(nq0), delta);
+            a.q[1].ldg, a.q[0].o_lo, a.q[1].o_lo, a.q[0].ldo_lo, a.q[1].ldo_lo, rows, attn_pad128(nq0), delta);
         FF_TRY(check_launch("attn_bwd_delta_kernel"));
     }
     BwdParams p;
@@ -709,7 +722,8 @@ int attention_backward(const AttnBwdSeg& s0, const AttnBwdSeg& s1, int B, int he
         // the joint layout: q, k, v (and their gradients) side by side in one row
         if (s.n && (!s.dqkv || s.ld < 3 * H || s.ldd < 3 * H))
             return set_error(FF_ERR_INVALID_ARG, "attention backward: bad segment %d", i);
-        a.q[i] = AttnBwdQuerySeg{s.qkv, s.ld, s.n, s.o, s.ldo, s.dout, s.ldg ? s.ldg : s.ldo, s.dqkv, s.ldd};
+        a.q[i] = AttnBwdQuerySeg{s.qkv, s.ld, s.n, s.o, s.ldo, s.dout, s.ldg ? s.ldg : s.ldo, s.dqkv, s.ldd, s.o_lo,
+                                 s.ldo_lo};
         a.kv[i] = AttnBwdKvSeg{s.qkv, s.ld, s.n, s.dqkv ? s.dqkv + H : nullptr, s.dqkv ? s.dqkv + 2 * H : nullptr,
                                s.ldd};
     }

@@ -310,7 +310,7 @@ int wan_forward_block(const ff_dit* m, int B, int l, const DitBlockIo& io, const
         {
             AttnSpec a{};
             a.q[0] = AttnQuerySeg{nullptr, 0, 0, nullptr, 0};
-            a.q[1] = AttnQuerySeg{io.qkv, 3 * H, Ni, io.o, H};
+            a.q[1] = AttnQuerySeg{io.qkv, 3 * H, Ni, io.o, H, io.o_lo, H};
             a.kv[0] = AttnKvSeg{nullptr, 0, 0};
             a.kv[1] = AttnKvSeg{io.qkv, 3 * H, Ni};
             a.q_col = 0; a.k_col = H; a.v_col = 2 * H;
@@ -349,7 +349,7 @@ int wan_forward_block(const ff_dit* m, int B, int l, const DitBlockIo& io, const
         {
             AttnSpec a{};
             a.q[0] = AttnQuerySeg{nullptr, 0, 0, nullptr, 0};
-            a.q[1] = AttnQuerySeg{io.qc, H, Ni, io.oc, H};
+            a.q[1] = AttnQuerySeg{io.qc, H, Ni, io.oc, H, io.oc_lo, H};
             a.kv[0] = AttnKvSeg{io.kv, 2 * H, Nt};
             a.kv[1] = AttnKvSeg{nullptr, 0, 0};
             a.q_col = 0; a.k_col = 0; a.v_col = H;
@@ -517,8 +517,9 @@ int mmdit_forward_double(const ff_dit* m, int B, int l, const DitBlockIo& io, co
             FF_TRY(gemm_bf16_group(g, 2, stream));
         }
         {
-            AttnSegment a0{io.qkv, 3 * H, io.o, H, Nt};
-            AttnSegment a1{io.qkv + static_cast<int64_t>(Rt) * 3 * H, 3 * H, io.o + static_cast<int64_t>(Rt) * H, H, Ni};
+            AttnSegment a0{io.qkv, 3 * H, io.o, H, Nt, io.o_lo, H};
+            AttnSegment a1{io.qkv + static_cast<int64_t>(Rt) * 3 * H, 3 * H, io.o + static_cast<int64_t>(Rt) * H, H, Ni,
+                           io.o_lo ? io.o_lo + static_cast<int64_t>(Rt) * H : nullptr, H};
             FF_TRY(attention(a0, a1, B, c.heads, c.head_dim, H, stream, io.lse));
         }
         // projection + gated residual (gate1)
@@ -605,9 +606,9 @@ int mmdit_forward_single(const ff_dit* m, int B, int l, const DitBlockIo& io, co
             FF_TRY(gemm_bf16(io.h1, H, W(p + "linear1.w"), H, R, 3 * H + F, H, e, stream));
         }
         {
-            AttnSegment a0{io.qkv, 3 * H, io.u, H + F, Nt};
+            AttnSegment a0{io.qkv, 3 * H, io.u, H + F, Nt, io.o_lo, H};
             AttnSegment a1{io.qkv + static_cast<int64_t>(Rt) * 3 * H, 3 * H, io.u + static_cast<int64_t>(Rt) * (H + F),
-                           H + F, Ni};
+                           H + F, Ni, io.o_lo ? io.o_lo + static_cast<int64_t>(Rt) * H : nullptr, H};
             FF_TRY(attention(a0, a1, B, c.heads, c.head_dim, H, stream, io.lse));
         }
         // linear2 + gated residual: one launch, the two segments as two

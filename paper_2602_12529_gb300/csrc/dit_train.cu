@@ -22,9 +22,12 @@
 //   zero-padded to a multiple of 8 rows, and their pre-activation copies;
 //   per double-stream block: x_in, x_mid fp32 [R, H]; h1, h2, o, y1, y2 bf16
 //   [R, H]; raw and normalised qkv bf16 [R, 3H]; a1 = MLP1 + bias and
-//   u = GELU(a1) bf16 [R, F]; the attention log-sum-exp;
+//   u = GELU(a1) bf16 [R, F]; the attention log-sum-exp and the bf16
+//   rounding residual of its output (bf16 [R, H]: the backward's
+//   D = rowsum(dO O) is formed from O to about 16 bits);
 //   per single-stream block: x_in fp32; h, y2 bf16 [R, H]; raw linear1 bf16
-//   [R, 3H + F]; qkv bf16 [R, 3H]; u = [o | GELU(mlp)] bf16 [R, H + F]; lse;
+//   [R, 3H + F]; qkv bf16 [R, 3H]; u = [o | GELU(mlp)] bf16 [R, H + F]; o's
+//   residual; lse;
 //   the final residual and LN-modulate output; then the backward's scratch.
 // In recompute mode (ff_dit_set_train_recompute) the blocks of each kind
 // share one set of those activations and only the block inputs are kept;
@@ -104,6 +107,7 @@ TrainPlan plan(const ff_dit_config& c, int64_t Wm, int B, uint8_t* base, bool re
         io.raw = b16(R * (dbl ? 3 * H : 3 * H + F));
         io.qkv = b16(R * 3 * H);
         io.lse = f32(lse_n);
+        io.o_lo = b16(R * H);
         if (dbl) {
             io.o = b16(R * H);
             io.y1 = b16(R * H);
@@ -307,9 +311,10 @@ int ff_dit_backward(const ff_dit* m, int B, const void* txt, const float* dv, fl
             FF_TRY(group(&g, 1));
         }
         {
-            AttnBwdSeg s0{io.qkv, 3 * H, io.u, p.dob, H + F, p.dbig, W1, Nt, H};
+            AttnBwdSeg s0{io.qkv, 3 * H, io.u, p.dob, H + F, p.dbig, W1, Nt, H, io.o_lo, H};
             AttnBwdSeg s1{io.qkv + static_cast<int64_t>(Rt) * 3 * H, 3 * H, io.u + static_cast<int64_t>(Rt) * (H + F),
-                          p.dob + static_cast<int64_t>(Rt) * H, H + F, p.dbig + static_cast<int64_t>(Rt) * W1, W1, Ni, H};
+                          p.dob + static_cast<int64_t>(Rt) * H, H + F, p.dbig + static_cast<int64_t>(Rt) * W1, W1, Ni, H,
+                          io.o_lo + static_cast<int64_t>(Rt) * H, H};
             FF_TRY(attention_backward(s0, s1, B, heads, d, io.lse, p.attn_ws, p.attn_ws_bytes, stream));
         }
         {
@@ -436,9 +441,10 @@ int ff_dit_backward(const ff_dit* m, int B, const void* txt, const float* dv, fl
             FF_TRY(group(g, 2));
         }
         {
-            AttnBwdSeg s0{io.qkv, 3 * H, io.o, p.dob, H, p.dqkv, 3 * H, Nt, 0};
+            AttnBwdSeg s0{io.qkv, 3 * H, io.o, p.dob, H, p.dqkv, 3 * H, Nt, 0, io.o_lo, H};
             AttnBwdSeg s1{io.qkv + static_cast<int64_t>(Rt) * 3 * H, 3 * H, io.o + static_cast<int64_t>(Rt) * H,
-                          p.dob + static_cast<int64_t>(Rt) * H, H, p.dqkv + static_cast<int64_t>(Rt) * 3 * H, 3 * H, Ni, 0};
+                          p.dob + static_cast<int64_t>(Rt) * H, H, p.dqkv + static_cast<int64_t>(Rt) * 3 * H, 3 * H, Ni, 0,
+                          io.o_lo + static_cast<int64_t>(Rt) * H, H};
             FF_TRY(attention_backward(s0, s1, B, heads, d, io.lse, p.attn_ws, p.attn_ws_bytes, stream));
         }
         {

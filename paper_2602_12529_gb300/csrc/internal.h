@@ -192,6 +192,9 @@ struct AttnSegment {
     const __nv_bfloat16* qkv; int64_t ld;  // q at col 0, k at col H, v at col 2H (row = token)
     __nv_bfloat16* out; int64_t ldo;       // output row = token, head h at col h*d
     int n;                                 // tokens per sample in this segment
+    // optional (training): O - bf16(O) rounded to bf16, laid out like out
+    // with row pitch ldo_lo; out + out_lo carries O to about 16 bits
+    __nv_bfloat16* out_lo = nullptr; int64_t ldo_lo = 0;
 };
 int attention(const AttnSegment& s0, const AttnSegment& s1, int B, int heads, int head_dim, int H,
               cudaStream_t stream, float* lse = nullptr);
@@ -201,7 +204,10 @@ int attention(const AttnSegment& s0, const AttnSegment& s1, int B, int heads, in
 // at columns q_col / k_col / v_col + h * d of its buffer.  Joint attention
 // uses the same buffers for both; cross-attention uses image queries and
 // text keys/values.
-struct AttnQuerySeg { const __nv_bfloat16* buf; int64_t ld; int n; __nv_bfloat16* out; int64_t ldo; };
+struct AttnQuerySeg {
+    const __nv_bfloat16* buf; int64_t ld; int n; __nv_bfloat16* out; int64_t ldo;
+    __nv_bfloat16* out_lo = nullptr; int64_t ldo_lo = 0;   // optional low part of O (see AttnSegment)
+};
 struct AttnKvSeg { const __nv_bfloat16* buf; int64_t ld; int n; };
 struct AttnSpec {
     AttnQuerySeg q[2];
@@ -229,6 +235,9 @@ struct AttnBwdSeg {
     __nv_bfloat16* dqkv; int64_t ldd;        // dq, dk, dv at columns 0, H, 2H
     int n;
     int64_t ldg = 0;
+    // optional: the forward's low part of O (AttnSegment::out_lo); D then
+    // comes from O to about 16 bits instead of bf16 O
+    const __nv_bfloat16* o_lo = nullptr; int64_t ldo_lo = 0;
 };
 // The same for attention_general's form: query segments (q at column q_col
 // of their rows, O, dO, and where dq goes) and key / value segments (k, v at
@@ -241,6 +250,7 @@ struct AttnBwdQuerySeg {
     const __nv_bfloat16* o; int64_t ldo;
     const __nv_bfloat16* dout; int64_t ldg;
     __nv_bfloat16* dq; int64_t ldq;
+    const __nv_bfloat16* o_lo = nullptr; int64_t ldo_lo = 0;   // optional low part of O
 };
 struct AttnBwdKvSeg {
     const __nv_bfloat16* kv; int64_t ld;
@@ -347,6 +357,11 @@ struct DitBlockIo {
     float *xin, *xmid, *xout;
     __nv_bfloat16 *h1, *qkv, *raw, *o, *y1, *h2, *a1, *u, *y2;
     float* lse;
+    // training only: the attention outputs' low parts (O - bf16(O) in bf16,
+    // [R, H] with pitch H; o_lo for the self / joint attention, oc_lo for
+    // the WAN cross-attention), so the backward's D = rowsum(dO O) sees O to
+    // about 16 bits
+    __nv_bfloat16 *o_lo, *oc_lo;
     // WAN blocks (xmid: after the self-attention): the residual after the
     // cross-attention, the affine-LN output, the normalised cross q and text
     // k | v with their raw copies (written only when set), the

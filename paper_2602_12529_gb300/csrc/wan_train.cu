@@ -104,6 +104,7 @@ WanPlan plan(const ff_dit_config& c, int64_t Wm, int B, uint8_t* base, bool reco
         io.qkv = b16(Ri * 3 * H);
         io.lse = f32(lse_n);
         io.o = b16(Ri * H);
+        io.o_lo = b16(Ri * H);
         io.y1 = b16(Ri * H);
         io.xmid = f32(Ri * H);
         io.hc = b16(Ri * H);
@@ -112,6 +113,7 @@ WanPlan plan(const ff_dit_config& c, int64_t Wm, int B, uint8_t* base, bool reco
         io.kv_raw = b16(Rt * 2 * H);
         io.kv = b16(Rt * 2 * H);
         io.oc = b16(Ri * H);
+        io.oc_lo = b16(Ri * H);
         io.lse_c = f32(lse_n);
         io.x3 = f32(Ri * H);
         io.h2 = b16(Ri * H);
@@ -282,7 +284,7 @@ int wan_backward(const ff_dit* m, int B, const void* txt, const float* dv, float
             // dq of the latent queries into dy (free again), dk | dv of the text into dkv
             AttnBwdSpec a{};
             a.q[0] = AttnBwdQuerySeg{nullptr, 0, 0, nullptr, 0, nullptr, 0, nullptr, 0};
-            a.q[1] = AttnBwdQuerySeg{io.qc, H, Ni, io.oc, H, p.dob, H, p.dy, H};
+            a.q[1] = AttnBwdQuerySeg{io.qc, H, Ni, io.oc, H, p.dob, H, p.dy, H, io.oc_lo, H};
             a.kv[0] = AttnBwdKvSeg{io.kv, 2 * H, Nt, p.dkv, p.dkv + H, 2 * H};
             a.kv[1] = AttnBwdKvSeg{nullptr, 0, 0, nullptr, nullptr, 0};
             a.q_col = 0; a.k_col = 0; a.v_col = H;
@@ -341,7 +343,7 @@ int wan_backward(const ff_dit* m, int B, const void* txt, const float* dv, float
         }
         {
             const AttnBwdSeg s0{nullptr, 0, nullptr, nullptr, 0, nullptr, 0, 0, 0};
-            const AttnBwdSeg s1{io.qkv, W3, io.o, p.dob, H, p.dbig, W3, Ni, H};
+            const AttnBwdSeg s1{io.qkv, W3, io.o, p.dob, H, p.dbig, W3, Ni, H, io.o_lo, H};
             FF_TRY(attention_backward(s0, s1, B, heads, d, io.lse, p.attn_ws, p.attn_ws_bytes, stream));
         }
         {
