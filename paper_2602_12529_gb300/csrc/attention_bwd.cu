@@ -36,7 +36,6 @@ constexpr int kT = 128;                        // rows of a query / key tile
 constexpr int kSub = 64;                        // query / key columns of one S (S^T) sub-tile
 constexpr int kSlotsDq = 5;                     // streamed K / V tiles in flight (dQ kernel)
 constexpr int kSlotsDkdv = 4;                   // streamed Q / dO tiles in flight (dK dV kernel)
-constexpr int kMaxSlots = 5;
 constexpr int kThreads = 320;                   // producer, MMA, 8 elementwise warps (two per TMEM lane quarter)
 constexpr int kEw = 8;                          // elementwise warps
 constexpr int kBarBytes = 256;
@@ -56,11 +55,20 @@ struct BwdParams {
     int64_t ldkv[2];
 };
 
+// The streamed tiles of step i (K_i and V_i in the dQ kernel, Q_i and dO_i
+// in the dK dV kernel; item 2 i and 2 i + 1 of the ring, in slots n % S)
+// arrive on one barrier, and one commit after the step's last MMA that reads
+// them releases both slots.  The MMA thread waits once per step for its
+// operands and commits three times (buffer 0, buffer 1, release) instead of
+// twice for each.  A parity wait on a ring of four barriers is unambiguous
+// while its waiter is at most three phases behind, which the ring's slot
+// count guarantees.
 struct Bars {
     uint64_t fixed_full;           // the CTA's own tiles landed
-    uint64_t slot_full[kMaxSlots];
-    uint64_t slot_empty[kMaxSlots];
-    uint64_t s_full[2];            // MMA -> elementwise: S (S^T) and dP (dP^T) of a sub-tile in TMEM buffer b
+    uint64_t grp_full[4];          // producer -> MMA: both streamed tiles of step i landed (entry i % 4)
+    uint64_t rel[4];               // MMA -> producer: step i's tiles are read (entry i % 4)
+    uint64_t s0_full;              // MMA -> elementwise: S (S^T) and dP (dP^T) of buffer 0 in TMEM
+    uint64_t s1_ring[4];           // MMA -> elementwise: buffer 1's S and dP of step i (entry i % 4)
     uint64_t p_full[2];            // elementwise -> MMA: dS (P^T, dS^T) of buffer b in TMEM
     uint64_t done;                 // MMA -> elementwise: the accumulators are final
     uint64_t drain;
@@ -177,14 +185,13 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_const
             *abort_flag = 1;
         }
         mbar_init(&bar.fixed_full, 1);
-        for (int s = 0; s < S_; ++s) {
-            mbar_init(&bar.slot_full[s], 1);
-            mbar_init(&bar.slot_empty[s], 1);
+        for (int g = 0; g < 4; ++g) {
+            mbar_init(&bar.grp_full[g], 2);
+            mbar_init(&bar.rel[g], 1);
+            mbar_init(&bar.s1_ring[g], 1);
         }
-        for (int s = 0; s < 2; ++s) {
-            mbar_init(&bar.s_full[s], 1);
-            mbar_init(&bar.p_full[s], kEw);
-        }
+        mbar_init(&bar.s0_full, 1);
+        for (int s = 0; s < 2; ++s) mbar_init(&bar.p_full[s], kEw);
         mbar_init(&bar.done, 1);
         mbar_init(&bar.drain, 1);
         fence_mbar_init();
@@ -213,15 +220,19 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_const
         }
         for (int n = 0; n < 2 * ntiles; ++n) {
             const int s = n % S_;
-            if (!mbar_wait(&bar.slot_empty[s], ((n / S_) & 1) ^ 1)) { fail(); break; }
+            if (n >= S_) {   // slot s held a tile of step (n - S_) / 2
+                const int r = (n - S_) >> 1;
+                if (!mbar_wait(&bar.rel[r & 3], (r >> 2) & 1)) { fail(); break; }
+            }
+            uint64_t* fb = &bar.grp_full[(n >> 1) & 3];
             const int j = n >> 1;
             const int ks = j < nt0 ? 0 : 1;
             const int row = b * p.nk[ks] + (j - (ks ? nt0 : 0)) * kT;
             const int col = ((n & 1) ? p.v_col : p.k_col) + h * HD;
             uint8_t* dst = sKV + s * kTileBytes;
-            mbar_arrive_expect_tx(&bar.slot_full[s], kTileBytes);
+            mbar_arrive_expect_tx(fb, kTileBytes);
             for (int c = 0; c < NB; ++c)
-                tma_load_2d(dst + c * (kT * 128), ks ? &tm_kv1 : &tm_kv0, &bar.slot_full[s], col + c * 64, row);
+                tma_load_2d(dst + c * (kT * 128), ks ? &tm_kv1 : &tm_kv0, fb, col + c * 64, row);
         }
     } else if (warp == 1 && lane == 0) {
         // ---- MMA issuer
@@ -231,10 +242,7 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_const
         if (!ok) fail();
         const uint64_t dq_ = smem_desc_k_sw128(smem_u32(sQ));
         const uint64_t ddo = smem_desc_k_sw128(smem_u32(sdO));
-        auto wait_kv = [&](int j) {
-            const int nk = 2 * j, nv = 2 * j + 1;
-            return mbar_wait(&bar.slot_full[nk % S_], (nk / S_) & 1) && mbar_wait(&bar.slot_full[nv % S_], (nv / S_) & 1);
-        };
+        auto wait_kv = [&](int j) { return mbar_wait(&bar.grp_full[j & 3], (j >> 2) & 1); };
         // S = Q K^T and dP = dO V^T of key half hf of tile j into buffer hf
         auto issue_sdp = [&](int j, int hf) {
             const uint32_t aK = smem_u32(sKV + ((2 * j) % S_) * kTileBytes) + hf * (kSub * 128);
@@ -247,7 +255,7 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_const
                 tc_mma_bf16(tb, dq_ + off, dk + off, idesc_s, k != 0 ? 1u : 0u);
                 tc_mma_bf16(tb + kSub, ddo + off, dv + off, idesc_s, k != 0 ? 1u : 0u);
             }
-            tc_commit(&bar.s_full[hf]);
+            tc_commit(hf == 0 ? &bar.s0_full : &bar.s1_ring[j & 3]);
         };
         if (ok && !wait_kv(0)) { fail(); ok = false; }
         if (ok) {
@@ -266,10 +274,7 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_const
             for (int k = 0; k < kSub / 16; ++k)   // keys 16k.. of the half: packed at (k / 2) * 32 + (k % 2) * 8
                 tc_mma_bf16_ts(tmem + 256, tmem + hf * 128 + (k >> 1) * 32 + (k & 1) * 8,
                                dkm + static_cast<uint64_t>(k * (2048 >> 4)), idesc_q, (u | k) != 0 ? 1u : 0u);
-            if (hf == 1) {
-                tc_commit(&bar.slot_empty[(2 * j) % S_]);
-                tc_commit(&bar.slot_empty[(2 * j + 1) % S_]);
-            }
+            if (hf == 1) tc_commit(&bar.rel[j & 3]);   // K_j, V_j read for the last time
             if (j + 1 < ntiles) {
                 if (hf == 0 && !wait_kv(j + 1)) { fail(); ok = false; break; }
                 tc_fence_after();
@@ -295,7 +300,12 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_const
         bool ok = true;
         for (int u = 0; u < 2 * ntiles; ++u) {
             const int hf = u & 1, j = u >> 1;
-            if (!mbar_wait(&bar.s_full[hf], (u >> 1) & 1)) { fail(); ok = false; break; }
+            if (!(hf == 0 ? mbar_wait(&bar.s0_full, (u >> 1) & 1)
+                          : mbar_wait(&bar.s1_ring[(u >> 1) & 3], (u >> 3) & 1))) {
+                fail();
+                ok = false;
+                break;
+            }
             tc_fence_after();
             const uint32_t tb = tS + hf * 128;
             uint32_t sr[32], pr_[32];
@@ -396,14 +406,13 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_con
             *abort_flag = 1;
         }
         mbar_init(&bar.fixed_full, 1);
-        for (int s = 0; s < S_; ++s) {
-            mbar_init(&bar.slot_full[s], 1);
-            mbar_init(&bar.slot_empty[s], 1);
+        for (int g = 0; g < 4; ++g) {
+            mbar_init(&bar.grp_full[g], 2);
+            mbar_init(&bar.rel[g], 1);
+            mbar_init(&bar.s1_ring[g], 1);
         }
-        for (int s = 0; s < 2; ++s) {
-            mbar_init(&bar.s_full[s], 1);
-            mbar_init(&bar.p_full[s], kEw);
-        }
+        mbar_init(&bar.s0_full, 1);
+        for (int s = 0; s < 2; ++s) mbar_init(&bar.p_full[s], kEw);
         mbar_init(&bar.done, 1);
         mbar_init(&bar.drain, 1);
         fence_mbar_init();
@@ -432,7 +441,11 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_con
         }
         for (int n = 0; n < 2 * ntiles; ++n) {
             const int s = n % S_;
-            if (!mbar_wait(&bar.slot_empty[s], ((n / S_) & 1) ^ 1)) { fail(); break; }
+            if (n >= S_) {   // slot s held a tile of step (n - S_) / 2
+                const int r = (n - S_) >> 1;
+                if (!mbar_wait(&bar.rel[r & 3], (r >> 2) & 1)) { fail(); break; }
+            }
+            uint64_t* fb = &bar.grp_full[(n >> 1) & 3];
             const int i = n >> 1;
             const int qs = i < nt0 ? 0 : 1;
             const int qi = (i - (qs ? nt0 : 0)) * kT;
@@ -440,16 +453,15 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_con
             uint8_t* dst = sQD + s * kTileBytes;
             if (n & 1) {
                 float* ld = sLD + (s >> 1) * 2 * kT;
-                mbar_arrive_expect_tx(&bar.slot_full[s], kTileBytes + 2 * kT * 4);
+                mbar_arrive_expect_tx(fb, kTileBytes + 2 * kT * 4);
                 for (int c = 0; c < NB; ++c)
-                    tma_load_2d(dst + c * (kT * 128), qs ? &tm_do1 : &tm_do0, &bar.slot_full[s], h * HD + c * 64, row);
-                bulk_load_1d(ld, p.lse + lrow + p.lse_base[qs] + qi, kT * 4, &bar.slot_full[s]);
-                bulk_load_1d(ld + kT, p.delta + lrow + p.lse_base[qs] + qi, kT * 4, &bar.slot_full[s]);
+                    tma_load_2d(dst + c * (kT * 128), qs ? &tm_do1 : &tm_do0, fb, h * HD + c * 64, row);
+                bulk_load_1d(ld, p.lse + lrow + p.lse_base[qs] + qi, kT * 4, fb);
+                bulk_load_1d(ld + kT, p.delta + lrow + p.lse_base[qs] + qi, kT * 4, fb);
             } else {
-                mbar_arrive_expect_tx(&bar.slot_full[s], kTileBytes);
+                mbar_arrive_expect_tx(fb, kTileBytes);
                 for (int c = 0; c < NB; ++c)
-                    tma_load_2d(dst + c * (kT * 128), qs ? &tm_q1 : &tm_q0, &bar.slot_full[s],
-                                p.q_col + h * HD + c * 64, row);
+                    tma_load_2d(dst + c * (kT * 128), qs ? &tm_q1 : &tm_q0, fb, p.q_col + h * HD + c * 64, row);
             }
         }
     } else if (warp == 1 && lane == 0) {
@@ -460,10 +472,7 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_con
         if (!ok) fail();
         const uint64_t dk_ = smem_desc_k_sw128(smem_u32(sK));
         const uint64_t dv_ = smem_desc_k_sw128(smem_u32(sV));
-        auto wait_qd = [&](int i) {
-            const int nq = 2 * i, nd = 2 * i + 1;
-            return mbar_wait(&bar.slot_full[nq % S_], (nq / S_) & 1) && mbar_wait(&bar.slot_full[nd % S_], (nd / S_) & 1);
-        };
+        auto wait_qd = [&](int i) { return mbar_wait(&bar.grp_full[i & 3], (i >> 2) & 1); };
         // S^T = K Q^T and dP^T = V dO^T of query half hf of tile i into buffer hf
         auto issue_sdp = [&](int i, int hf) {
             const uint32_t aQ = smem_u32(sQD + ((2 * i) % S_) * kTileBytes) + hf * (kSub * 128);
@@ -476,7 +485,7 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_con
                 tc_mma_bf16(tb, dk_ + off, dq_ + off, idesc_s, k != 0 ? 1u : 0u);
                 tc_mma_bf16(tb + kSub, dv_ + off, ddo + off, idesc_s, k != 0 ? 1u : 0u);
             }
-            tc_commit(&bar.s_full[hf]);
+            tc_commit(hf == 0 ? &bar.s0_full : &bar.s1_ring[i & 3]);
         };
         if (ok && !wait_qd(0)) { fail(); ok = false; }
         if (ok) {
@@ -500,10 +509,7 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_con
                 tc_mma_bf16_ts(tmem + 256, a, ddom + step, idesc_g, acc);              // dV += P^T dO
                 tc_mma_bf16_ts(tmem + 256 + HD, a + kSub, dqm + step, idesc_g, acc);   // dK += dS^T Q
             }
-            if (hf == 1) {
-                tc_commit(&bar.slot_empty[(2 * i) % S_]);
-                tc_commit(&bar.slot_empty[(2 * i + 1) % S_]);
-            }
+            if (hf == 1) tc_commit(&bar.rel[i & 3]);   // Q_i, dO_i read for the last time
             if (i + 1 < ntiles) {
                 if (hf == 0 && !wait_qd(i + 1)) { fail(); ok = false; break; }
                 tc_fence_after();
@@ -525,7 +531,12 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_con
         bool ok = true;
         for (int u = 0; u < 2 * ntiles; ++u) {
             const int hf = u & 1, i = u >> 1;
-            if (!mbar_wait(&bar.s_full[hf], (u >> 1) & 1)) { fail(); ok = false; break; }
+            if (!(hf == 0 ? mbar_wait(&bar.s0_full, (u >> 1) & 1)
+                          : mbar_wait(&bar.s1_ring[(u >> 1) & 3], (u >> 3) & 1))) {
+                fail();
+                ok = false;
+                break;
+            }
             tc_fence_after();
             const int nd = 2 * i + 1;
             const float* lse = sLD + ((nd % S_) >> 1) * 2 * kT + hf * kSub + cg * 32;
