@@ -211,8 +211,8 @@ int ff_sde_logprob_backward(int B, int64_t D, const float* x_t, const float* v,
  *
  * Same arguments and results as ff_sde_step_logprob, minus the workspace.
  * The caller still passes every input and output.  The scratch is a fixed
- * 528 KiB array built into the library (4096 ticket counters, then 65536
- * fp64 partial sums), held on every GPU that loads the library until the
+ * 272 KiB array built into the library (4096 ticket counters, then 65536
+ * fp32 partial sums), held on every GPU that loads the library until the
  * process exits.  Limits: B <= 4096 and B * min(ceil(D / 4096), 1024) <=
  * 65536 partial sums, which holds for any D when B <= 64; larger calls are
  * rejected with FF_ERR_UNSUPPORTED and a message naming the limit, before any

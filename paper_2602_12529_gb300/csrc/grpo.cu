@@ -10,9 +10,11 @@
 // Loss: rho = exp(lp_new - lp_old) per (sample, step);
 //   obj = min(rho A, clip(rho, 1 - lo, 1 + hi) A), loss = -sum(obj) / (B T),
 //   grad_lp_new = -A rho / (B T) where the unclipped term is the minimum.
-// One launch: every block writes one fp64 partial (the grid size depends only
+// One launch: every block writes one fp32 partial (the grid size depends only
 // on B T), takes a ticket, and the block with the last ticket adds the
-// partials in index order, writes the loss and resets the ticket to zero.
+// partials in a fixed order, writes the loss and resets the ticket to zero.
+// All fp32 (fp64 arithmetic is slow on this part): per-thread sums of a few
+// terms, shuffles, then at most 1216 partials, about 1e-6 relative error.
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -22,7 +24,7 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kElemsPerBlock = kThreads * 16;
 constexpr int kMaxLossBlocks = 1216;   // 8 blocks of 256 threads on each of 152 SMs
-// Workspace: the ticket word at offset 0 (its own 16 bytes), then the fp64
+// Workspace: the ticket word at offset 0 (its own 16 bytes), then the fp32
 // partials.
 constexpr size_t kLossTicketBytes = 16;
 
@@ -144,9 +146,8 @@ template <bool WEIGHTED>
 __global__ void __launch_bounds__(kThreads) grpo_loss_partial_kernel(int64_t n, int T, const float* lp_new,
                                                                      const float* lp_old, const float* adv,
                                                                      const float* step_w, float lo, float hi,
-                                                                     float inv_n, float* grad, double* partial,
-                                                                     unsigned* ticket, double inv_nd, float* loss) {
-    __shared__ double red[kThreads / 32];
+                                                                     float inv_n, float* grad, float* partial,
+                                                                     unsigned* ticket, float* loss) {
     float s = 0.f;
     const int64_t n4 = n >> 2;
     const float4* a4 = reinterpret_cast<const float4*>(lp_new);
@@ -181,8 +182,6 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_partial_kernel(int64_t n, 
         s += term(lp_new[i], lp_old[i], static_cast<uint32_t>(i), g);
         if (grad) grad[i] = g;
     }
-    // fp32 within the block (fp64 arithmetic is slow on this part), fp64
-    // across blocks
 #pragma unroll
     for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
     __shared__ float redf[kThreads / 32];
@@ -192,24 +191,24 @@ __global__ void __launch_bounds__(kThreads) grpo_loss_partial_kernel(int64_t n, 
     if (threadIdx.x == 0) {
         float t = 0.f;
         for (int w = 0; w < kThreads / 32; ++w) t += redf[w];
-        partial[blockIdx.x] = static_cast<double>(t);
+        partial[blockIdx.x] = t;
         last = ticket_add_acq_rel(ticket, 1u) == gridDim.x - 1;
     }
     __syncthreads();
     if (!last) return;
     // every partial is stored (the last ticket acquired them): add them in
     // index order
-    double acc = 0.0;
+    float acc = 0.f;
     for (int i = threadIdx.x; i < static_cast<int>(gridDim.x); i += kThreads) acc += __ldcg(partial + i);
 #pragma unroll
     for (int o = 16; o; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
+    if ((threadIdx.x & 31) == 0) redf[threadIdx.x >> 5] = acc;
     __syncthreads();
     if (threadIdx.x == 0) {
-        double t = 0.0;
-        for (int w = 0; w < kThreads / 32; ++w) t += red[w];
+        float t = 0.f;
+        for (int w = 0; w < kThreads / 32; ++w) t += redf[w];
         *ticket = 0u;
-        *loss = static_cast<float>(-t * inv_nd);
+        *loss = -t * inv_n;
     }
 }
 
@@ -247,7 +246,7 @@ int ff_group_advantage(int n_groups, int G, const float* rewards, float eps_A, f
 int ff_grpo_loss_workspace_size(int B, int T, size_t* bytes) {
     if (!bytes) return ff::set_error(FF_ERR_INVALID_ARG, "bytes is null");
     if (B <= 0 || T <= 0) return ff::set_error(FF_ERR_INVALID_ARG, "B=%d T=%d must be positive", B, T);
-    *bytes = ff::kLossTicketBytes + static_cast<size_t>(ff::loss_blocks(static_cast<int64_t>(B) * T)) * sizeof(double);
+    *bytes = ff::kLossTicketBytes + static_cast<size_t>(ff::loss_blocks(static_cast<int64_t>(B) * T)) * sizeof(float);
     return FF_OK;
 }
 
@@ -269,23 +268,22 @@ int grpo_loss_impl(int B, int T, const float* lp_new, const float* lp_old, const
         return set_error(FF_ERR_INVALID_ARG, "loss: clip range must satisfy 0 <= lo < 1, hi >= 0");
     const int64_t n = static_cast<int64_t>(B) * T;
     const int nb = loss_blocks(n);
-    const size_t need = kLossTicketBytes + static_cast<size_t>(nb) * sizeof(double);
+    const size_t need = kLossTicketBytes + static_cast<size_t>(nb) * sizeof(float);
     if (!ws || ws_bytes < need || (reinterpret_cast<uintptr_t>(ws) & 15))
         return set_error(FF_ERR_WORKSPACE, "loss: workspace %zu B < %zu B needed (or not 16-byte aligned)", ws_bytes,
                          need);
     unsigned* ticket = static_cast<unsigned*>(ws);
-    double* partial = reinterpret_cast<double*>(static_cast<uint8_t*>(ws) + kLossTicketBytes);
+    float* partial = reinterpret_cast<float*>(static_cast<uint8_t*>(ws) + kLossTicketBytes);
     const float inv_f = static_cast<float>(1.0 / static_cast<double>(n));
-    const double inv_d = 1.0 / static_cast<double>(n);
     ProfScope prof(stream, "grpo_loss", 0.0, static_cast<double>(n) * (grad_lp_new ? 12.0 : 8.0) + 4.0 * B);
     if (step_w)
         grpo_loss_partial_kernel<true><<<nb, kThreads, 0, stream>>>(n, T, lp_new, lp_old, adv, step_w, clip_lo,
                                                                     clip_hi, inv_f, grad_lp_new, partial, ticket,
-                                                                    inv_d, loss);
+                                                                    loss);
     else
         grpo_loss_partial_kernel<false><<<nb, kThreads, 0, stream>>>(n, T, lp_new, lp_old, adv, nullptr, clip_lo,
                                                                      clip_hi, inv_f, grad_lp_new, partial, ticket,
-                                                                     inv_d, loss);
+                                                                     loss);
     return check_launch("grpo_loss_kernel");
 }
 

@@ -8,12 +8,16 @@
 //   SAMPLE: x_next = mean + std eps;  EVAL: x_next given; SAMPLE with eps
 //   drawn in the kernel from the counter-based generator of rng.cuh
 //   logp = -sum (x_next - mean)^2 / (2 std^2) - D ln std - D/2 ln 2 pi
-// The per-sample coefficients are formed in fp64 once per block; the
-// elementwise work is fp32 FMAs over 128-bit streaming loads.  One launch:
-// every block writes one fp64 partial sum of squared residuals, then takes a
-// ticket; the block that draws the sample's last ticket adds that sample's
-// partials in index order (so the result does not depend on which block
-// finished last), writes logp and puts the ticket word back to zero.
+// Everything is fp32: fp64 arithmetic runs on very few units of this part,
+// and a handful of dependent fp64 operations (a log, a square root, a
+// shuffle reduction) cost microseconds.  The per-sample coefficients are
+// formed by every thread; the elementwise work is FMAs over 128-bit loads.
+// One launch: every block writes one partial sum of squared residuals, then
+// takes a ticket; the block that draws the sample's last ticket adds that
+// sample's partials in a fixed order (so the result does not depend on which
+// block finished last), writes logp and puts the ticket word back to zero.
+// The partials of up to 1024 blocks are added pairwise-ish (four per thread,
+// then shuffles, then eight warps in order): relative error about 1e-6.
 #include "internal.h"
 #include "ptx.cuh"
 #include "rng.cuh"
@@ -59,50 +63,36 @@ __device__ __forceinline__ float block_sum_f32(float v, float* red) {
     return s;
 }
 
-__device__ __forceinline__ double block_sum(double v, double* red) {
-#pragma unroll
-    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    const int w = threadIdx.x >> 5;
-    if ((threadIdx.x & 31) == 0) red[w] = v;
-    __syncthreads();
-    double s = 0.0;
-    if (threadIdx.x == 0) {
-        for (int i = 0; i < (int)(blockDim.x >> 5); ++i) s += red[i];
-    }
-    return s;   // valid in thread 0
-}
-
 // The log-probability of sample b from its summed squared residual ss:
-// -ss / (2 std^2) - D ln std - D/2 ln 2 pi (divided by D for FF_LP_MEAN), in
-// fp64; 0 when std == 0 (no density).
-__device__ __forceinline__ float logprob_of(double ss, int64_t D, const float* t, const float* t_next,
+// -ss / (2 std^2) - D ln std - D/2 ln 2 pi (divided by D for FF_LP_MEAN);
+// 0 when std == 0 (no density).  The three terms are each about D in size
+// and do not cancel, so fp32 keeps about 1e-6 of relative accuracy.
+__device__ __forceinline__ float logprob_of(float ss, int64_t D, const float* t, const float* t_next,
                                             const float* sigma, int b, int reduce) {
-    const double delta = static_cast<double>(t[b]) - static_cast<double>(t_next[b]);
-    const double sd = static_cast<double>(sigma[b]) * sqrt(delta);
-    double lp = 0.0;
-    if (sd > 0.0) {
-        const double dd = static_cast<double>(D);
-        lp = -0.5 * ss / (sd * sd) - dd * log(sd) - 0.5 * dd * log(2.0 * 3.14159265358979323846);
-        if (reduce == FF_LP_MEAN) lp /= dd;
-    }
-    return static_cast<float>(lp);
+    const float delta = t[b] - t_next[b];
+    const float sd = sigma[b] * sqrtf(delta);
+    if (!(sd > 0.f)) return 0.f;
+    const float dd = static_cast<float>(D);
+    const float kHalfLog2Pi = 0.91893853320467274f;   // ln(2 pi) / 2
+    float lp = -(0.5f * ss / (sd * sd) + dd * (logf(sd) + kHalfLog2Pi));
+    if (reduce == FF_LP_MEAN) lp /= dd;
+    return lp;
 }
 
 // Grid (blocks_per_sample, B); block k of sample b handles chunks
-// k, k + blocks_per_sample, ... and writes one partial (fp32 within the
-// block, stored as fp64).  The number of blocks per sample depends only on D
-// (see nchunks), so the summation order is fixed.
+// k, k + blocks_per_sample, ... and writes one fp32 partial.  The number of
+// blocks per sample depends only on D (see nchunks), so the summation order
+// is fixed.
 // ticket[b] counts the blocks of sample b that have stored their partial; it
 // is zero on entry and the last block of the sample sets it back to zero.
 template <int MODE>
 __global__ void __launch_bounds__(kThreads) sde_step_partial_kernel(int64_t D, int nblk, const float* x,
                                                                     const float* v, const float* eps, float* x_next,
                                                                     const float* t, const float* t_next,
-                                                                    const float* sigma, double* partial,
+                                                                    const float* sigma, float* partial,
                                                                     unsigned* ticket, int reduce, float* logp, int ld,
                                                                     PhiloxKey key, uint32_t rng_stream) {
     __shared__ float redf[kThreads / 32];
-    __shared__ double red[kThreads / 32];
     const int b = blockIdx.y;
     const StepCoef c = step_coef(t, t_next, sigma, b);
     const int64_t row = static_cast<int64_t>(b) * D;
@@ -162,17 +152,17 @@ __global__ void __launch_bounds__(kThreads) sde_step_partial_kernel(int64_t D, i
     const float s = block_sum_f32(ss, redf);
     __shared__ bool last;
     if (threadIdx.x == 0) {
-        partial[static_cast<int64_t>(b) * nblk + blockIdx.x] = static_cast<double>(s);
+        partial[static_cast<int64_t>(b) * nblk + blockIdx.x] = s;
         last = ticket_add_acq_rel(ticket + b, 1u) == static_cast<unsigned>(nblk - 1);
     }
     __syncthreads();
     if (!last) return;
     // every partial of sample b is stored (the last ticket acquired them);
     // add them in index order
-    const double* pb = partial + static_cast<int64_t>(b) * nblk;
-    double acc = 0.0;
+    const float* pb = partial + static_cast<int64_t>(b) * nblk;
+    float acc = 0.f;
     for (int i = threadIdx.x; i < nblk; i += kThreads) acc += __ldcg(pb + i);
-    acc = block_sum(acc, red);
+    acc = block_sum_f32(acc, redf);
     if (threadIdx.x == 0) {
         ticket[b] = 0u;
         logp[static_cast<int64_t>(b) * ld] = logprob_of(acc, D, t, t_next, sigma, b, reduce);
@@ -200,23 +190,16 @@ __global__ void __launch_bounds__(kThreads) sde_logprob_backward_kernel(int64_t 
                                                                         const float* t, const float* t_next,
                                                                         const float* sigma, const float* g, int ldg,
                                                                         int reduce, float* dv) {
-    __shared__ float3 coef;
     const int b = blockIdx.y;
-    if (threadIdx.x == 0) {
-        const StepCoef c = step_coef(t, t_next, sigma, b);
-        const double sd = static_cast<double>(c.std);
-        double k = 0.0;
-        if (sd > 0.0) {
-            const double delta = static_cast<double>(t[b]) - static_cast<double>(t_next[b]);
-            const double sg = sigma[b];
-            const double var = sg * sg * delta;
-            k = static_cast<double>(g[static_cast<int64_t>(b) * ldg]) * static_cast<double>(c.cv) / var;
-            if (reduce == FF_LP_MEAN) k /= static_cast<double>(D);
-        }
-        coef = make_float3(c.cx, c.cv, static_cast<float>(k));
+    const StepCoef sc = step_coef(t, t_next, sigma, b);
+    float k = 0.f;
+    if (sc.std > 0.f) {
+        const float delta = t[b] - t_next[b];
+        const float sg = sigma[b];
+        k = g[static_cast<int64_t>(b) * ldg] * sc.cv / (sg * sg * delta);
+        if (reduce == FF_LP_MEAN) k /= static_cast<float>(D);
     }
-    __syncthreads();
-    const float3 c = coef;
+    const float3 c = make_float3(sc.cx, sc.cv, k);
     const int64_t row = static_cast<int64_t>(b) * D;
     const float4* x4 = reinterpret_cast<const float4*>(x + row);
     const float4* v4 = reinterpret_cast<const float4*>(v + row);
@@ -260,7 +243,7 @@ extern "C" {
 int ff_sde_workspace_size(int B, int64_t D, size_t* bytes) {
     if (!bytes) return ff::set_error(FF_ERR_INVALID_ARG, "bytes is null");
     if (B <= 0 || D <= 0) return ff::set_error(FF_ERR_INVALID_ARG, "B and D must be positive");
-    *bytes = ff::kTicketBytes + static_cast<size_t>(B) * static_cast<size_t>(ff::nchunks(D)) * sizeof(double);
+    *bytes = ff::kTicketBytes + static_cast<size_t>(B) * static_cast<size_t>(ff::nchunks(D)) * sizeof(float);
     return FF_OK;
 }
 
@@ -274,7 +257,7 @@ namespace {
 // exit) and B * nchunks(D) fp64 partials.
 int launch_sde_step(int B, int64_t D, int nc, const float* x_t, const float* v, const float* eps, float* x_next,
                     const float* t, const float* t_next, const float* sigma, int mode, int reduce, float* logp,
-                    int ld, unsigned* ticket, double* partial, PhiloxKey key, uint32_t rng_stream,
+                    int ld, unsigned* ticket, float* partial, PhiloxKey key, uint32_t rng_stream,
                     cudaStream_t stream) {
     const dim3 grid(nc, B);
     ProfScope prof(stream, "sde_step", 0.0, static_cast<double>(B) * D * (mode == FF_SDE_SAMPLE ? 16.0 : 12.0));
@@ -306,12 +289,12 @@ int sde_step(int B, int64_t D, const float* x_t, const float* v, const float* ep
     if (mode == kModePhilox && D / 4 > 0xFFFFFFFFll)
         return set_error(FF_ERR_UNSUPPORTED, "sde: D=%lld too large for the generator's counter", (long long)D);
     const int nc = nchunks(D);
-    const size_t need = kTicketBytes + static_cast<size_t>(B) * nc * sizeof(double);
+    const size_t need = kTicketBytes + static_cast<size_t>(B) * nc * sizeof(float);
     if (!ws || ws_bytes < need || (reinterpret_cast<uintptr_t>(ws) & 15))
         return set_error(FF_ERR_WORKSPACE, "sde: workspace %zu B < %zu B needed (or not 16-byte aligned)", ws_bytes,
                          need);
     unsigned* ticket = static_cast<unsigned*>(ws);
-    double* partial = reinterpret_cast<double*>(static_cast<uint8_t*>(ws) + kTicketBytes);
+    float* partial = reinterpret_cast<float*>(static_cast<uint8_t*>(ws) + kTicketBytes);
     return launch_sde_step(B, D, nc, x_t, v, eps, x_next, t, t_next, sigma, mode, reduce, logp, ld, ticket, partial,
                            key, rng_stream, stream);
 }
@@ -431,17 +414,16 @@ namespace ff {
 namespace {
 
 constexpr int kNoAllocMaxSamples = 4096;      // ticket words, at the front of the array
-constexpr int kNoAllocMaxPartials = 65536;    // fp64 partial sums after them
-constexpr int kNoAllocTicketSlots = kNoAllocMaxSamples / 2;   // two 32-bit tickets per fp64 slot
+constexpr int kNoAllocMaxPartials = 65536;    // fp32 partial sums after them
 
-// Shared by every call on a device (528 KiB).  The ticket words start at
+// Shared by every call on a device (272 KiB).  The ticket words start at
 // zero (device globals are zero-initialised when the module loads) and every
 // call leaves them at zero; the partial slots are rewritten before they are
 // read, so nothing else has to be cleared.
-static __device__ __align__(256) double g_sde_scratch[kNoAllocTicketSlots + kNoAllocMaxPartials];
+static __device__ __align__(256) float g_sde_scratch[kNoAllocMaxSamples + kNoAllocMaxPartials];
 
 constexpr int kNoAllocMaxDevices = 64;
-std::atomic<double*> g_sde_scratch_addr[kNoAllocMaxDevices] = {};
+std::atomic<float*> g_sde_scratch_addr[kNoAllocMaxDevices] = {};
 std::mutex g_sde_scratch_mu;
 
 // Device address of g_sde_scratch on the current device, looked up once per
@@ -449,11 +431,11 @@ std::mutex g_sde_scratch_mu;
 // The cache is keyed by device ordinal and holds the primary context's
 // address: it is wrong for a caller that runs the library in another context
 // on that device, and stale after cudaDeviceReset.
-int sde_scratch_address(double** out) {
+int sde_scratch_address(float** out) {
     int dev = -1;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kNoAllocMaxDevices)
         return set_error(FF_ERR_CUDA, "sde (no-alloc): no usable current device");
-    double* p = g_sde_scratch_addr[dev].load(std::memory_order_acquire);
+    float* p = g_sde_scratch_addr[dev].load(std::memory_order_acquire);
     if (!p) {
         std::lock_guard<std::mutex> lk(g_sde_scratch_mu);
         p = g_sde_scratch_addr[dev].load(std::memory_order_relaxed);
@@ -462,7 +444,7 @@ int sde_scratch_address(double** out) {
             const cudaError_t e = cudaGetSymbolAddress(&q, g_sde_scratch);
             if (e != cudaSuccess || !q)
                 return set_error(FF_ERR_CUDA, "sde (no-alloc): cudaGetSymbolAddress failed: %s", cudaGetErrorString(e));
-            p = static_cast<double*>(q);
+            p = static_cast<float*>(q);
             g_sde_scratch_addr[dev].store(p, std::memory_order_release);
         }
     }
@@ -498,11 +480,11 @@ extern "C" int ff_sde_step_logprob_noalloc(int B, int64_t D, const float* x_t, c
     if (!aligned16(x_t) || !aligned16(v) || !aligned16(x_next) || (mode == FF_SDE_SAMPLE && !aligned16(eps)))
         return set_error(FF_ERR_INVALID_ARG, "sde (no-alloc): arrays must be 16-byte aligned");
     if (ld < 1) return set_error(FF_ERR_INVALID_ARG, "sde (no-alloc): ld=%d < 1", ld);
-    double* scratch = nullptr;
+    float* scratch = nullptr;
     const int rc0 = sde_scratch_address(&scratch);
     if (rc0) return rc0;
     unsigned* ticket = reinterpret_cast<unsigned*>(scratch);
-    double* partial = scratch + kNoAllocTicketSlots;
+    float* partial = scratch + kNoAllocMaxSamples;
     return launch_sde_step(B, D, nc, x_t, v, eps, x_next, t, t_next, sigma, mode, reduce, logp, ld, ticket, partial,
                            PhiloxKey{0, 0}, 0u, stream);
 }

@@ -77,14 +77,14 @@ def test_weight_layout_matches_oracle_parameters(L, name):
 
 
 def test_workspace_queries(L):
-    # SDE: a fixed 256 KiB ticket region, then one fp64 partial per
+    # SDE: a fixed 256 KiB ticket region, then one fp32 partial per
     # 4096-element chunk (at most 1024 per sample)
     n1 = ffi.ff_sde_workspace_size(4, 262144)
-    assert n1 == 256 * 1024 + 4 * 64 * 8
-    # loss: a 16-byte ticket, then one fp64 partial per block (at most 1216)
-    assert ffi.ff_grpo_loss_workspace_size(32, 10) == 16 + 8
-    assert ffi.ff_grpo_loss_workspace_size(1 << 20, 64) == 16 + 1216 * 8
-    assert ffi.ff_sde_workspace_size(4, 1 << 26) == 256 * 1024 + 4 * 1024 * 8
+    assert n1 == 256 * 1024 + 4 * 64 * 4
+    # loss: a 16-byte ticket, then one fp32 partial per block (at most 1216)
+    assert ffi.ff_grpo_loss_workspace_size(32, 10) == 16 + 4
+    assert ffi.ff_grpo_loss_workspace_size(1 << 20, 64) == 16 + 1216 * 4
+    assert ffi.ff_sde_workspace_size(4, 1 << 26) == 256 * 1024 + 4 * 1024 * 4
     with pytest.raises(ffi.FFError):
         ffi.ff_sde_workspace_size(0, 16)
 
