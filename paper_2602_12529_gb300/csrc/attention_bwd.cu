@@ -13,14 +13,15 @@
 // Three kernels:
 //   delta   D_i, one warp per (row, head), into the workspace (lse layout);
 //   dq      one 128-row query tile per CTA, K/V tiles streamed: S = Q K_j^T
-//           and dP = dO V_j^T in TMEM, dS written over S as bf16, then
-//           dQ += dS K_j with dS read from TMEM and K_j taken as an MN-major
-//           operand (the same shared-memory tile feeds S as K-major);
+//           and dP = dO V_j^T in TMEM (whole 128-key tiles), dS to its own
+//           TMEM columns as bf16, then dQ += dS K_j with dS read from TMEM
+//           and K_j taken as an MN-major operand (the same shared-memory tile
+//           feeds S as K-major);
 //   dkdv    one 128-key tile per CTA, query tiles streamed: S^T = K Q_i^T and
-//           dP^T = V dO_i^T in TMEM, P^T and dS^T written over them, then
-//           dV += P^T dO_i and dK += dS^T Q_i (Q_i, dO_i as MN-major
-//           operands); lse and D of the query tile arrive by bulk copies with
-//           the tiles.
+//           dP^T = V dO_i^T in TMEM (whole 128-query tiles), P^T and dS^T
+//           written over them, then dV += P^T dO_i and dK += dS^T Q_i (Q_i,
+//           dO_i as MN-major operands); lse and D of the query tile arrive by
+//           bulk copies with the tiles.
 // Query (key) rows past a segment's end read neighbouring or zero-filled
 // rows; their columns are selected to zero (never multiplied, so padding
 // can hold anything) and their rows are not stored.  Every wait is bounded;
@@ -33,7 +34,6 @@ namespace ff {
 namespace {
 
 constexpr int kT = 128;                        // rows of a query / key tile
-constexpr int kSub = 64;                        // query / key columns of one S (S^T) sub-tile
 constexpr int kSlotsDq = 5;                     // streamed K / V tiles in flight (dQ kernel)
 constexpr int kSlotsDkdv = 4;                   // streamed Q / dO tiles in flight (dK dV kernel)
 constexpr int kThreads = 320;                   // producer, MMA, 8 elementwise warps (two per TMEM lane quarter)
@@ -58,18 +58,17 @@ struct BwdParams {
 // The streamed tiles of step i (K_i and V_i in the dQ kernel, Q_i and dO_i
 // in the dK dV kernel; item 2 i and 2 i + 1 of the ring, in slots n % S)
 // arrive on one barrier, and one commit after the step's last MMA that reads
-// them releases both slots.  The MMA thread waits once per step for its
-// operands and commits three times (buffer 0, buffer 1, release) instead of
-// twice for each.  A parity wait on a ring of four barriers is unambiguous
-// while its waiter is at most three phases behind, which the ring's slot
-// count guarantees.
+// them releases both slots.  A parity wait on a ring of four barriers is
+// unambiguous while its waiter is at most three phases behind, which the
+// ring's slot count guarantees; the two-phase barriers are waited in
+// lockstep with their producers.
 struct Bars {
     uint64_t fixed_full;           // the CTA's own tiles landed
     uint64_t grp_full[4];          // producer -> MMA: both streamed tiles of step i landed (entry i % 4)
-    uint64_t rel[4];               // MMA -> producer: step i's tiles are read (entry i % 4)
-    uint64_t s0_full;              // MMA -> elementwise: S (S^T) and dP (dP^T) of buffer 0 in TMEM
-    uint64_t s1_ring[4];           // MMA -> elementwise: buffer 1's S and dP of step i (entry i % 4)
-    uint64_t p_full[2];            // elementwise -> MMA: dS (P^T, dS^T) of buffer b in TMEM
+    uint64_t rel[4];               // MMA -> producer (and dQ's elementwise warps): step i's MMAs are done
+    uint64_t s0_full;              // MMA -> elementwise: S (S^T) and dP (dP^T) of the step in TMEM
+    uint64_t p_full[2];            // elementwise -> MMA: dQ kernel: [0] S / dP read, [1] dS written;
+                                   // dK dV kernel: [0] P^T and dS^T written
     uint64_t done;                 // MMA -> elementwise: the accumulators are final
     uint64_t drain;
     uint32_t tmem_slot;
@@ -149,14 +148,16 @@ __global__ void __launch_bounds__(256) attn_bwd_delta_kernel(int B, int heads, i
 }
 
 // ------------------------------------------------------------------ dQ
-// TMEM: two sub-tile buffers of 128 columns, buffer b holding S (64 key
-// columns) at 128 b and dP at 128 b + 64; the two elementwise warps of a
-// lane quarter take 32 key columns each and write their dS as bf16 pairs over
-// the first 16 of their own S columns (keys 0-31 at 0, keys 32-63 at 32); dQ
-// (d columns) at 256.  Key tile j is processed as two 64-key
-// halves, half b in buffer b, so the elementwise warps work on one buffer
-// while the MMAs of the other (dQ += dS K, then the next half's S and dP)
-// run.  Shared memory: Q tile, dO tile, then a ring of K_j / V_j tiles.
+// One 128-row query tile per CTA; K / V tiles streamed through the ring.
+// TMEM: S = Q K_j^T at columns 0..127 and dP = dO V_j^T at 128..255 (fp32,
+// the whole 128-key tile: N = 128 MMAs), dS as bf16 pairs at 256..319, dQ
+// (d columns) at 384.  Per key tile j the elementwise warps load their S and
+// dP columns into registers and hand the buffer back at once, so the MMAs of
+// tile j + 1 (S, dP) run while they form dS_j; dS_j goes to its own columns,
+// and dQ += dS_j K_j follows.  The MMA thread's work per tile: three waits
+// (S / dP consumed, operands of j + 1, dS_j written) and two commits (S / dP
+// of j + 1 ready; dQ_j done, which also frees K_j / V_j and the dS columns).
+// Shared memory: Q tile, dO tile, then the ring of K_j / V_j tiles.
 template <int HD>
 __global__ void __launch_bounds__(kThreads, 1)
 attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_constant__ CUtensorMap tm_q1,
@@ -166,6 +167,7 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_const
     constexpr int S_ = kSlotsDq;
     constexpr int kTileBytes = kT * HD * 2;              // one bf16 tile: HD / 64 boxes of 128 rows x 64 columns
     constexpr int NB = HD / 64;
+    constexpr uint32_t kColS = 0, kColP = kT, kColDs = 2 * kT, kColDq = 384;
     extern __shared__ __align__(1024) uint8_t smem[];
     uint8_t* sQ = smem;
     uint8_t* sdO = smem + kTileBytes;
@@ -188,10 +190,10 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_const
         for (int g = 0; g < 4; ++g) {
             mbar_init(&bar.grp_full[g], 2);
             mbar_init(&bar.rel[g], 1);
-            mbar_init(&bar.s1_ring[g], 1);
         }
-        mbar_init(&bar.s0_full, 1);
-        for (int s = 0; s < 2; ++s) mbar_init(&bar.p_full[s], kEw);
+        mbar_init(&bar.s0_full, 1);        // S and dP of tile j in TMEM
+        mbar_init(&bar.p_full[0], kEw);    // every elementwise warp has read S / dP of tile j
+        mbar_init(&bar.p_full[1], kEw);    // every elementwise warp has written its dS_j
         mbar_init(&bar.done, 1);
         mbar_init(&bar.drain, 1);
         fence_mbar_init();
@@ -210,7 +212,8 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_const
     };
     if (*abort_flag) {
     } else if (warp == 0 && lane == 0) {
-        // ---- producer: Q and dO of this tile, then K_0, V_0, K_1, ...
+        // ---- producer: Q and dO of this tile, then K_0, V_0, K_1, ...; the
+        // slot of a tile's K / V is free again once dQ of that tile is done
         const CUtensorMap* tq = seg ? &tm_q1 : &tm_q0;
         const CUtensorMap* td = seg ? &tm_do1 : &tm_do0;
         mbar_arrive_expect_tx(&bar.fixed_full, 2 * kTileBytes);
@@ -236,57 +239,54 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_const
         }
     } else if (warp == 1 && lane == 0) {
         // ---- MMA issuer
-        constexpr uint32_t idesc_s = idesc_bf16_f32(kT, kSub);
-        constexpr uint32_t idesc_q = idesc_bf16_f32(kT, HD) | (1u << 16);   // B = K_j half, MN-major
+        constexpr uint32_t idesc_s = idesc_bf16_f32(kT, kT);
+        constexpr uint32_t idesc_q = idesc_bf16_f32(kT, HD) | (1u << 16);   // B = K_j, MN-major
         bool ok = mbar_wait(&bar.fixed_full, 0);
         if (!ok) fail();
         const uint64_t dq_ = smem_desc_k_sw128(smem_u32(sQ));
         const uint64_t ddo = smem_desc_k_sw128(smem_u32(sdO));
         auto wait_kv = [&](int j) { return mbar_wait(&bar.grp_full[j & 3], (j >> 2) & 1); };
-        // S = Q K^T and dP = dO V^T of key half hf of tile j into buffer hf
-        auto issue_sdp = [&](int j, int hf) {
-            const uint32_t aK = smem_u32(sKV + ((2 * j) % S_) * kTileBytes) + hf * (kSub * 128);
-            const uint32_t aV = smem_u32(sKV + ((2 * j + 1) % S_) * kTileBytes) + hf * (kSub * 128);
-            const uint64_t dk = smem_desc_k_sw128(aK), dv = smem_desc_k_sw128(aV);
-            const uint32_t tb = tmem + hf * 128;
+        // S = Q K_j^T and dP = dO V_j^T of the whole key tile
+        auto issue_sdp = [&](int j) {
+            const uint64_t dk = smem_desc_k_sw128(smem_u32(sKV + ((2 * j) % S_) * kTileBytes));
+            const uint64_t dv = smem_desc_k_sw128(smem_u32(sKV + ((2 * j + 1) % S_) * kTileBytes));
 #pragma unroll
             for (int k = 0; k < HD / 16; ++k) {
                 const uint32_t off = ((k / 4) * (kT * 128) + (k % 4) * 32) >> 4;
-                tc_mma_bf16(tb, dq_ + off, dk + off, idesc_s, k != 0 ? 1u : 0u);
-                tc_mma_bf16(tb + kSub, ddo + off, dv + off, idesc_s, k != 0 ? 1u : 0u);
+                tc_mma_bf16(tmem + kColS, dq_ + off, dk + off, idesc_s, k != 0 ? 1u : 0u);
+                tc_mma_bf16(tmem + kColP, ddo + off, dv + off, idesc_s, k != 0 ? 1u : 0u);
             }
-            tc_commit(hf == 0 ? &bar.s0_full : &bar.s1_ring[j & 3]);
+            tc_commit(&bar.s0_full);
         };
         if (ok && !wait_kv(0)) { fail(); ok = false; }
         if (ok) {
             tc_fence_after();
-            issue_sdp(0, 0);
-            issue_sdp(0, 1);
+            issue_sdp(0);
         }
-        for (int u = 0; ok && u < 2 * ntiles; ++u) {
-            const int hf = u & 1, j = u >> 1;
-            if (!mbar_wait(&bar.p_full[hf], (u >> 1) & 1)) { fail(); ok = false; break; }
-            tc_fence_after();
-            // dQ += dS K_j (this half's 64 keys): dS from TMEM, K rows as [keys (K) x d (N)], MN-major
-            const uint64_t dkm = smem_desc_mn_sw128(smem_u32(sKV + ((2 * j) % S_) * kTileBytes) + hf * (kSub * 128),
-                                                    kT * 128);
-#pragma unroll
-            for (int k = 0; k < kSub / 16; ++k)   // keys 16k.. of the half: packed at (k / 2) * 32 + (k % 2) * 8
-                tc_mma_bf16_ts(tmem + 256, tmem + hf * 128 + (k >> 1) * 32 + (k & 1) * 8,
-                               dkm + static_cast<uint64_t>(k * (2048 >> 4)), idesc_q, (u | k) != 0 ? 1u : 0u);
-            if (hf == 1) tc_commit(&bar.rel[j & 3]);   // K_j, V_j read for the last time
+        for (int j = 0; ok && j < ntiles; ++j) {
+            // the elementwise warps hold S_j / dP_j in registers: the next tile's may go in
+            if (!mbar_wait(&bar.p_full[0], j & 1)) { fail(); ok = false; break; }
             if (j + 1 < ntiles) {
-                if (hf == 0 && !wait_kv(j + 1)) { fail(); ok = false; break; }
+                if (!wait_kv(j + 1)) { fail(); ok = false; break; }
                 tc_fence_after();
-                issue_sdp(j + 1, hf);
+                issue_sdp(j + 1);
             }
+            if (!mbar_wait(&bar.p_full[1], j & 1)) { fail(); ok = false; break; }
+            tc_fence_after();
+            // dQ += dS_j K_j: dS (keys 16 k.. at columns 8 k..) from TMEM, K_j rows as [keys (K) x d (N)]
+            const uint64_t dkm = smem_desc_mn_sw128(smem_u32(sKV + ((2 * j) % S_) * kTileBytes), kT * 128);
+#pragma unroll
+            for (int k = 0; k < kT / 16; ++k)
+                tc_mma_bf16_ts(tmem + kColDq, tmem + kColDs + k * 8, dkm + static_cast<uint64_t>(k * (2048 >> 4)),
+                               idesc_q, (j | k) != 0 ? 1u : 0u);
+            tc_commit(&bar.rel[j & 3]);   // K_j, V_j and the dS columns are free again
         }
         if (ok) tc_commit(&bar.done);
         tc_commit(&bar.drain);
         if (!mbar_wait(&bar.drain, 0)) report_status(status, kStatusWaitTimeout);
     } else if (warp >= 2) {
         // ---- elementwise: thread = query row = TMEM lane; the two warps of a
-        // lane quarter take 32 key columns each of a sub-tile
+        // lane quarter take 64 key columns each of a tile
         const int q = warp & 3;
         const int cg = (warp - 2) >> 2;
         const int r = q * 32 + lane;
@@ -298,29 +298,27 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_const
         const float lse = live ? p.lse[li] : 0.f;
         const float dd = live ? p.delta[li] : 0.f;
         bool ok = true;
-        for (int u = 0; u < 2 * ntiles; ++u) {
-            const int hf = u & 1, j = u >> 1;
-            if (!(hf == 0 ? mbar_wait(&bar.s0_full, (u >> 1) & 1)
-                          : mbar_wait(&bar.s1_ring[(u >> 1) & 3], (u >> 3) & 1))) {
-                fail();
-                ok = false;
-                break;
-            }
+        for (int j = 0; j < ntiles; ++j) {
+            if (!mbar_wait(&bar.s0_full, j & 1)) { fail(); ok = false; break; }
             tc_fence_after();
-            const uint32_t tb = tS + hf * 128;
-            uint32_t sr[32], pr_[32];
-            tmem_ld_x32(tb + cg * 32, sr);
-            tmem_ld_x32(tb + kSub + cg * 32, pr_);
+            uint32_t sr[64], pr_[64];
+            tmem_ld_x32(tS + kColS + cg * 64, *reinterpret_cast<uint32_t(*)[32]>(&sr[0]));
+            tmem_ld_x32(tS + kColS + cg * 64 + 32, *reinterpret_cast<uint32_t(*)[32]>(&sr[32]));
+            tmem_ld_x32(tS + kColP + cg * 64, *reinterpret_cast<uint32_t(*)[32]>(&pr_[0]));
+            tmem_ld_x32(tS + kColP + cg * 64 + 32, *reinterpret_cast<uint32_t(*)[32]>(&pr_[32]));
             tmem_ld_wait();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&bar.p_full[0]);   // S_j / dP_j consumed: the buffer may be refilled
             const int ks = j < nt0 ? 0 : 1;
-            // key columns < valid of this warp's 32 are real
-            const int valid = p.nk[ks] - (j - (ks ? nt0 : 0)) * kT - hf * kSub - cg * 32;
-            if (valid >= 32 && full_rows) {
+            // key columns < valid of this warp's 64 are real
+            const int valid = p.nk[ks] - (j - (ks ? nt0 : 0)) * kT - cg * 64;
+            if (valid >= 64 && full_rows) {
                 // every column and row real: paired fp32 arithmetic, no selects
                 const float2 c2 = make_float2(p.scale_log2, p.scale_log2), nl2 = make_float2(-lse, -lse);
                 const float2 nd2 = make_float2(-dd, -dd);
 #pragma unroll
-                for (int i = 0; i < 32; i += 2) {
+                for (int i = 0; i < 64; i += 2) {
                     const float2 x = __ffma2_rn(make_float2(__uint_as_float(sr[i]), __uint_as_float(sr[i + 1])), c2, nl2);
                     const float2 dp = __fadd2_rn(make_float2(__uint_as_float(pr_[i]), __uint_as_float(pr_[i + 1])), nd2);
                     const float2 ds = __fmul2_rn(make_float2(ex2(x.x), ex2(x.y)), dp);
@@ -328,7 +326,7 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_const
                 }
             } else {
 #pragma unroll
-                for (int i = 0; i < 32; i += 2) {
+                for (int i = 0; i < 64; i += 2) {
                     float ds[2];
 #pragma unroll
                     for (int e = 0; e < 2; ++e) {
@@ -338,16 +336,18 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_const
                     sr[i / 2] = pack_bf16x2(ds[0], ds[1]);
                 }
             }
-            // packed over this warp's own (already read) S columns
-            tmem_st_x16(tb + cg * 32, sr);
+            // dS_j over the dS columns once dQ_j-1 has read them
+            if (j > 0 && !mbar_wait(&bar.rel[(j - 1) & 3], ((j - 1) >> 2) & 1)) { fail(); ok = false; break; }
+            tc_fence_after();
+            tmem_st_x32(tS + kColDs + cg * 32, sr);
             tmem_st_wait();
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&bar.p_full[hf]);
+            if (lane == 0) mbar_arrive(&bar.p_full[1]);
         }
         if (ok && mbar_wait(&bar.done, 0)) {
             tc_fence_after();
-            store_row_bf16(tS + 256 + cg * (HD / 2), p.scale,
+            store_row_bf16(tS + kColDq + cg * (HD / 2), p.scale,
                            p.dq[seg] + (static_cast<int64_t>(b) * p.nq[seg] + row) * p.ldq[seg] + h * HD + cg * (HD / 2),
                            live, HD / 2);
         } else if (ok) {
@@ -368,12 +368,15 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_const
 }
 
 // ------------------------------------------------------------------ dK, dV
-// TMEM: two sub-tile buffers of 128 columns, buffer b holding S^T (64 query
-// columns) at 128 b and dP^T at 128 b + 64; each elementwise warp writes its
-// 32 columns of P^T and dS^T as bf16 pairs over the first 16 of its own S^T /
-// dP^T columns; dV at 256, dK at 256 + d.  Query tile i is
-// processed as two 64-query halves, half b in buffer b, overlapping the
-// elementwise work of one buffer with the MMAs of the other.  Shared memory:
+// TMEM: S^T = K Q_i^T at columns 0..127 and dP^T = V dO_i^T at 128..255
+// (fp32, the whole 128-query tile: N = 128 MMAs); each elementwise warp
+// writes its 64 columns of P^T and dS^T as bf16 pairs over the first 32 of
+// its own S^T / dP^T columns; dV at 256, dK at 256 + d.  Per query tile i
+// the MMA thread issues dV += P^T dO_i and dK += dS^T Q_i, then at once
+// S^T / dP^T of tile i + 1: the tensor pipe runs one thread's MMAs in issue
+// order, so they overwrite P^T / dS^T only after dV / dK have read them.  Its
+// work per tile: two waits (P^T / dS^T written, operands of i + 1) and two
+// commits (tile i's slots free; S^T / dP^T of i + 1 ready).  Shared memory:
 // the K and V tiles of this CTA, then a ring of Q_i / dO_i tiles, then lse /
 // D of each streamed query tile.
 template <int HD>
@@ -409,7 +412,6 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_con
         for (int g = 0; g < 4; ++g) {
             mbar_init(&bar.grp_full[g], 2);
             mbar_init(&bar.rel[g], 1);
-            mbar_init(&bar.s1_ring[g], 1);
         }
         mbar_init(&bar.s0_full, 1);
         for (int s = 0; s < 2; ++s) mbar_init(&bar.p_full[s], kEw);
@@ -466,54 +468,49 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_con
         }
     } else if (warp == 1 && lane == 0) {
         // ---- MMA issuer
-        constexpr uint32_t idesc_s = idesc_bf16_f32(kT, kSub);
-        constexpr uint32_t idesc_g = idesc_bf16_f32(kT, HD) | (1u << 16);   // B = Q_i / dO_i half, MN-major
+        constexpr uint32_t idesc_s = idesc_bf16_f32(kT, kT);
+        constexpr uint32_t idesc_g = idesc_bf16_f32(kT, HD) | (1u << 16);   // B = Q_i / dO_i, MN-major
         bool ok = mbar_wait(&bar.fixed_full, 0);
         if (!ok) fail();
         const uint64_t dk_ = smem_desc_k_sw128(smem_u32(sK));
         const uint64_t dv_ = smem_desc_k_sw128(smem_u32(sV));
         auto wait_qd = [&](int i) { return mbar_wait(&bar.grp_full[i & 3], (i >> 2) & 1); };
-        // S^T = K Q^T and dP^T = V dO^T of query half hf of tile i into buffer hf
-        auto issue_sdp = [&](int i, int hf) {
-            const uint32_t aQ = smem_u32(sQD + ((2 * i) % S_) * kTileBytes) + hf * (kSub * 128);
-            const uint32_t aD = smem_u32(sQD + ((2 * i + 1) % S_) * kTileBytes) + hf * (kSub * 128);
-            const uint64_t dq_ = smem_desc_k_sw128(aQ), ddo = smem_desc_k_sw128(aD);
-            const uint32_t tb = tmem + hf * 128;
+        // S^T = K Q_i^T and dP^T = V dO_i^T of the whole query tile
+        auto issue_sdp = [&](int i) {
+            const uint64_t dq_ = smem_desc_k_sw128(smem_u32(sQD + ((2 * i) % S_) * kTileBytes));
+            const uint64_t ddo = smem_desc_k_sw128(smem_u32(sQD + ((2 * i + 1) % S_) * kTileBytes));
 #pragma unroll
             for (int k = 0; k < HD / 16; ++k) {
                 const uint32_t off = ((k / 4) * (kT * 128) + (k % 4) * 32) >> 4;
-                tc_mma_bf16(tb, dk_ + off, dq_ + off, idesc_s, k != 0 ? 1u : 0u);
-                tc_mma_bf16(tb + kSub, dv_ + off, ddo + off, idesc_s, k != 0 ? 1u : 0u);
+                tc_mma_bf16(tmem, dk_ + off, dq_ + off, idesc_s, k != 0 ? 1u : 0u);
+                tc_mma_bf16(tmem + kT, dv_ + off, ddo + off, idesc_s, k != 0 ? 1u : 0u);
             }
-            tc_commit(hf == 0 ? &bar.s0_full : &bar.s1_ring[i & 3]);
+            tc_commit(&bar.s0_full);
         };
         if (ok && !wait_qd(0)) { fail(); ok = false; }
         if (ok) {
             tc_fence_after();
-            issue_sdp(0, 0);
-            issue_sdp(0, 1);
+            issue_sdp(0);
         }
-        for (int u = 0; ok && u < 2 * ntiles; ++u) {
-            const int hf = u & 1, i = u >> 1;
-            if (!mbar_wait(&bar.p_full[hf], (u >> 1) & 1)) { fail(); ok = false; break; }
+        for (int i = 0; ok && i < ntiles; ++i) {
+            if (!mbar_wait(&bar.p_full[0], i & 1)) { fail(); ok = false; break; }
             tc_fence_after();
-            const uint32_t aQ = smem_u32(sQD + ((2 * i) % S_) * kTileBytes) + hf * (kSub * 128);
-            const uint32_t aD = smem_u32(sQD + ((2 * i + 1) % S_) * kTileBytes) + hf * (kSub * 128);
-            const uint64_t ddom = smem_desc_mn_sw128(aD, kT * 128), dqm = smem_desc_mn_sw128(aQ, kT * 128);
+            const uint64_t dqm = smem_desc_mn_sw128(smem_u32(sQD + ((2 * i) % S_) * kTileBytes), kT * 128);
+            const uint64_t ddom = smem_desc_mn_sw128(smem_u32(sQD + ((2 * i + 1) % S_) * kTileBytes), kT * 128);
 #pragma unroll
-            for (int k = 0; k < kSub / 16; ++k) {
+            for (int k = 0; k < kT / 16; ++k) {
                 const uint64_t step = static_cast<uint64_t>(k * (2048 >> 4));
-                const uint32_t acc = (u | k) != 0 ? 1u : 0u;
-                // queries 16k.. of the half: packed at (k / 2) * 32 + (k % 2) * 8
-                const uint32_t a = tmem + hf * 128 + (k >> 1) * 32 + (k & 1) * 8;
-                tc_mma_bf16_ts(tmem + 256, a, ddom + step, idesc_g, acc);              // dV += P^T dO
-                tc_mma_bf16_ts(tmem + 256 + HD, a + kSub, dqm + step, idesc_g, acc);   // dK += dS^T Q
+                const uint32_t acc = (i | k) != 0 ? 1u : 0u;
+                // queries 16 k.. : each warp's 64 queries packed over the first 32 of its columns
+                const uint32_t a = tmem + (k >> 2) * 64 + (k & 3) * 8;
+                tc_mma_bf16_ts(tmem + 256, a, ddom + step, idesc_g, acc);             // dV += P^T dO
+                tc_mma_bf16_ts(tmem + 256 + HD, a + kT, dqm + step, idesc_g, acc);    // dK += dS^T Q
             }
-            if (hf == 1) tc_commit(&bar.rel[i & 3]);   // Q_i, dO_i read for the last time
+            tc_commit(&bar.rel[i & 3]);   // Q_i, dO_i, lse_i and D_i read for the last time
             if (i + 1 < ntiles) {
-                if (hf == 0 && !wait_qd(i + 1)) { fail(); ok = false; break; }
+                if (!wait_qd(i + 1)) { fail(); ok = false; break; }
                 tc_fence_after();
-                issue_sdp(i + 1, hf);
+                issue_sdp(i + 1);
             }
         }
         if (ok) tc_commit(&bar.done);
@@ -521,7 +518,7 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_con
         if (!mbar_wait(&bar.drain, 0)) report_status(status, kStatusWaitTimeout);
     } else if (warp >= 2) {
         // ---- elementwise: thread = key row = TMEM lane; the two warps of a
-        // lane quarter take 32 query columns each of a sub-tile
+        // lane quarter take 64 query columns each of a tile
         const int q = warp & 3;
         const int cg = (warp - 2) >> 2;
         const int r = q * 32 + lane;
@@ -529,31 +526,27 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_con
         const uint32_t tS = tmem + (static_cast<uint32_t>(q * 32) << 16);
         const bool live = row < p.nk[seg];
         bool ok = true;
-        for (int u = 0; u < 2 * ntiles; ++u) {
-            const int hf = u & 1, i = u >> 1;
-            if (!(hf == 0 ? mbar_wait(&bar.s0_full, (u >> 1) & 1)
-                          : mbar_wait(&bar.s1_ring[(u >> 1) & 3], (u >> 3) & 1))) {
-                fail();
-                ok = false;
-                break;
-            }
+        for (int i = 0; i < ntiles; ++i) {
+            if (!mbar_wait(&bar.s0_full, i & 1)) { fail(); ok = false; break; }
             tc_fence_after();
             const int nd = 2 * i + 1;
-            const float* lse = sLD + ((nd % S_) >> 1) * 2 * kT + hf * kSub + cg * 32;
+            const float* lse = sLD + ((nd % S_) >> 1) * 2 * kT + cg * 64;
             const float* dl = lse + kT;
             const int qs = i < nt0 ? 0 : 1;
-            // query columns < valid of this warp's 32 are real
-            const int valid = p.nq[qs] - (i - (qs ? nt0 : 0)) * kT - hf * kSub - cg * 32;
-            const uint32_t tb = tS + hf * 128;
-            uint32_t sr[32], pr_[32];
-            tmem_ld_x32(tb + cg * 32, sr);
-            tmem_ld_x32(tb + kSub + cg * 32, pr_);
+            // query columns < valid of this warp's 64 are real
+            const int valid = p.nq[qs] - (i - (qs ? nt0 : 0)) * kT - cg * 64;
+            const uint32_t tb = tS + cg * 64;
+            uint32_t sr[64], pr_[64];
+            tmem_ld_x32(tb, *reinterpret_cast<uint32_t(*)[32]>(&sr[0]));
+            tmem_ld_x32(tb + 32, *reinterpret_cast<uint32_t(*)[32]>(&sr[32]));
+            tmem_ld_x32(tb + kT, *reinterpret_cast<uint32_t(*)[32]>(&pr_[0]));
+            tmem_ld_x32(tb + kT + 32, *reinterpret_cast<uint32_t(*)[32]>(&pr_[32]));
             tmem_ld_wait();
-            if (valid >= 32) {
+            if (valid >= 64) {
                 // every query column real: paired fp32 arithmetic, no selects
                 const float2 c2 = make_float2(p.scale_log2, p.scale_log2);
 #pragma unroll
-                for (int c = 0; c < 32; c += 2) {
+                for (int c = 0; c < 64; c += 2) {
                     const float2 l2 = *reinterpret_cast<const float2*>(lse + c);
                     const float2 d2 = *reinterpret_cast<const float2*>(dl + c);
                     const float2 x = __ffma2_rn(make_float2(__uint_as_float(sr[c]), __uint_as_float(sr[c + 1])), c2,
@@ -567,7 +560,7 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_con
                 }
             } else {
 #pragma unroll
-                for (int c = 0; c < 32; c += 2) {
+                for (int c = 0; c < 64; c += 2) {
                     float pv[2], ds[2];
 #pragma unroll
                     for (int e = 0; e < 2; ++e) {
@@ -581,12 +574,12 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_con
                 }
             }
             // packed over this warp's own (already read) S^T / dP^T columns
-            tmem_st_x16(tb + cg * 32, sr);
-            tmem_st_x16(tb + kSub + cg * 32, pr_);
+            tmem_st_x32(tb, sr);
+            tmem_st_x32(tb + kT, pr_);
             tmem_st_wait();
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&bar.p_full[hf]);
+            if (lane == 0) mbar_arrive(&bar.p_full[0]);
         }
         if (ok && mbar_wait(&bar.done, 0)) {
             tc_fence_after();
