@@ -495,7 +495,8 @@ int ff_gemm(int M, int N, int K, const void* A, int64_t lda, int a_layout, const
  * layout and pitch ldo) and lse, and writes dq, dk, dv into dqkv buffers laid
  * out like qkv (columns h d, H + h d, 2H + h d; pitch ldd; other columns are
  * not touched).  ws: ff_attention_backward_workspace_size bytes (holds
- * D = rowsum(dO * O)).  A segment with n = 0 may pass NULL buffers.
+ * -D = -rowsum(dO * O) and a copy of -lse, each [B, heads, L]).  A segment
+ * with n = 0 may pass NULL buffers.
  * ------------------------------------------------------------------------ */
 int ff_attention_lse_rows(int n0, int n1);
 int ff_attention_forward(int B, int heads, int head_dim, int n0, const void* qkv0, int64_t ld0,

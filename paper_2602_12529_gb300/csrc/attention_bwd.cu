@@ -37,7 +37,7 @@ constexpr int kT = 128;                        // rows of a query / key tile
 constexpr int kSlotsDq = 5;                     // streamed K / V tiles in flight (dQ kernel):
 constexpr int kKSlots = 3, kVSlots = 2;         //   three K slots, then two V slots
 static_assert(kKSlots + kVSlots == kSlotsDq, "dQ slots");
-constexpr int kSlotsDkdv = 4;                   // streamed Q / dO tiles in flight (dK dV kernel)
+constexpr int kQSlots = 3, kDoSlots = 2;       // streamed Q_i / dO_i tiles in flight (dK dV kernel)
 constexpr int kThreads = 320;                   // producer, MMA, 8 elementwise warps (two per TMEM lane quarter)
 constexpr int kEw = 8;                          // elementwise warps
 constexpr int kBarBytes = 256;
@@ -49,7 +49,8 @@ struct BwdParams {
     float scale_log2;      // log2(e) / sqrt(d)
     float scale;           // 1 / sqrt(d)
     const float* lse;      // [B, heads, lse_rows] base-2 log-sum-exp of the forward
-    const float* delta;    // D in the same layout
+    const float* nlse;     // -lse in the same layout (workspace copy, read by the dK dV kernel)
+    const float* ndelta;   // -D in the same layout
     int lse_rows, lse_base[2];
     __nv_bfloat16* dq[2];  // head h at column h d
     int64_t ldq[2];
@@ -66,13 +67,16 @@ struct BwdParams {
 // lockstep with their producers.
 struct Bars {
     uint64_t fixed_full;           // the CTA's own tiles landed
-    uint64_t grp_full[4];          // producer -> MMA: both streamed tiles of step i landed (entry i % 4)
+    uint64_t grp_full[4];          // producer -> MMA: both streamed tiles of step i landed (entry i % 4);
+                                   // dK dV kernel: Q_i and lse_i landed
+    uint64_t do_full[4];           // producer -> MMA: dO_i and D_i landed (dK dV kernel, entry i % 4)
     uint64_t rel[4];               // MMA -> producer (and dQ's elementwise warps): step i's MMAs are done
-    uint64_t s0_full;              // MMA -> elementwise: S^T and dP^T of the step in TMEM (dK dV kernel)
+    uint64_t s0_full;              // MMA -> elementwise: S^T of the step in TMEM (dK dV kernel)
+    uint64_t s1_full;              // MMA -> elementwise: dP^T of the step in TMEM (dK dV kernel)
     uint64_t s0_ring[4];           // MMA -> elementwise and producer: S and dP of step j in TMEM (entry
                                    // j % 4), so V_j is read (dQ kernel)
     uint64_t p_full[2];            // elementwise -> MMA: dQ kernel: [0] S / dP read, [1] dS written;
-                                   // dK dV kernel: [0] P^T and dS^T written
+                                   // dK dV kernel: [0] P^T written, [1] dS^T written
     uint64_t done;                 // MMA -> elementwise: the accumulators are final
     uint64_t drain;
     uint32_t tmem_slot;
@@ -105,10 +109,17 @@ __device__ __forceinline__ void store_row_bf16(uint32_t taddr, float mul, __nv_b
     }
 }
 
-// D_i = sum_c dO_ic O_ic: one warp per (token row, head), HD / 32 columns per
-// lane.  With the forward's low parts (o_lo), O = o + o_lo: D = rowsum(P dP)
+// D_i = sum_c dO_ic O_ic, stored negated, with a negated copy of lse_i
+// beside it (the dK dV kernel adds both per score).  A block takes kDeltaRows
+// consecutive token rows of one head, sample and segment (so its lse / D
+// reads and writes are contiguous); the d / 8 threads of a row each load 16
+// bytes of O and of dO (a head's row is 2 d contiguous bytes) and are summed
+// by shuffles; each thread takes four rows, their loads issued together.
+// With the forward's low parts (o_lo), O = o + o_lo: D = rowsum(P dP)
 // subtracts nearly equal terms when the rows of V are close to each other,
 // and bf16 O alone would leave a relative error of 2^-9 |dO| |O| in D.
+template <int HD>
+constexpr int delta_rows() { return 4 * 8 * (32 / (HD / 8)); }   // four rows per thread, 256 threads
 template <int HD>
 __global__ void __launch_bounds__(256) attn_bwd_delta_kernel(int B, int heads, int n0, int n1,
                                                              const __nv_bfloat16* o0, const __nv_bfloat16* do0,
@@ -116,39 +127,62 @@ __global__ void __launch_bounds__(256) attn_bwd_delta_kernel(int B, int heads, i
                                                              int64_t ldo0, int64_t ldo1, int64_t ldg0, int64_t ldg1,
                                                              const __nv_bfloat16* ol0, const __nv_bfloat16* ol1,
                                                              int64_t ldl0, int64_t ldl1, int lse_rows, int base1,
-                                                             float* delta) {
-    const int64_t w = (static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x) >> 5;
-    const int lane = threadIdx.x & 31;
-    const int64_t rows0 = static_cast<int64_t>(B) * n0;
-    const int64_t total = (rows0 + static_cast<int64_t>(B) * n1) * heads;
-    if (w >= total) return;
-    const int h = static_cast<int>(w % heads);
-    const int64_t r = w / heads;                    // token row over both segments
-    const bool s1 = r >= rows0;
-    const int64_t rr = s1 ? r - rows0 : r;
+                                                             const float* lse, float* ndelta, float* nlse) {
+    constexpr int kLanes = HD / 8;                  // threads per row
+    constexpr int kRowsPerPass = 256 / kLanes;      // rows one pass of the block covers
+    constexpr int R = delta_rows<HD>();
+    constexpr int kPer = R / kRowsPerPass;          // rows per thread
+    const int t0 = (n0 + R - 1) / R, t1 = (n1 + R - 1) / R;
+    const int b = blockIdx.x / (t0 + t1);
+    const int t = blockIdx.x - b * (t0 + t1);
+    const bool s1 = t >= t0;
     const int n = s1 ? n1 : n0;
-    const int b = static_cast<int>(rr / n);
-    const int row = static_cast<int>(rr - static_cast<int64_t>(b) * n);
-    constexpr int E = HD / 32;
-    const __nv_bfloat16* o = (s1 ? o1 : o0) + rr * (s1 ? ldo1 : ldo0) + h * HD + lane * E;
-    const __nv_bfloat16* g = (s1 ? do1 : do0) + rr * (s1 ? ldg1 : ldg0) + h * HD + lane * E;
-    const __nv_bfloat16* olb = s1 ? ol1 : ol0;
-    const __nv_bfloat16* ol = olb ? olb + rr * (s1 ? ldl1 : ldl0) + h * HD + lane * E : nullptr;
-    float s = 0.f;
+    const int h = blockIdx.y;
+    const int c = threadIdx.x & (kLanes - 1);
+    const int first = (s1 ? t - t0 : t) * R + threadIdx.x / kLanes;
+    const int64_t ld_o = s1 ? ldo1 : ldo0, ld_g = s1 ? ldg1 : ldg0, ld_l = s1 ? ldl1 : ldl0;
+    const int64_t rowbase = static_cast<int64_t>(b) * n;
+    const __nv_bfloat16* o = (s1 ? o1 : o0) + h * HD + c * 8;
+    const __nv_bfloat16* g = (s1 ? do1 : do0) + h * HD + c * 8;
+    const __nv_bfloat16* ol = s1 ? ol1 : ol0;
+    const int64_t lbase = (static_cast<int64_t>(b) * heads + h) * lse_rows + (s1 ? base1 : 0);
+    uint4 ov[kPer], gv[kPer], lv[kPer];
+    float lse_v[kPer];
 #pragma unroll
-    for (int e = 0; e < E; e += 2) {
-        float2 of = unpack_bf16x2(*reinterpret_cast<const uint32_t*>(o + e));
-        if (ol) {
-            const float2 lf = unpack_bf16x2(*reinterpret_cast<const uint32_t*>(ol + e));
-            of.x += lf.x;
-            of.y += lf.y;
-        }
-        const float2 gf = unpack_bf16x2(*reinterpret_cast<const uint32_t*>(g + e));
-        s = fmaf(of.x, gf.x, fmaf(of.y, gf.y, s));
+    for (int k = 0; k < kPer; ++k) {
+        const int row = first + k * kRowsPerPass;
+        ov[k] = gv[k] = lv[k] = make_uint4(0u, 0u, 0u, 0u);
+        lse_v[k] = 0.f;
+        if (row >= n) continue;
+        const int64_t r = rowbase + row;
+        ov[k] = *reinterpret_cast<const uint4*>(o + r * ld_o);
+        gv[k] = *reinterpret_cast<const uint4*>(g + r * ld_g);
+        if (ol) lv[k] = *reinterpret_cast<const uint4*>(ol + h * HD + c * 8 + r * ld_l);
+        if (c == 0) lse_v[k] = lse[lbase + row];
     }
 #pragma unroll
-    for (int k = 16; k; k >>= 1) s += __shfl_xor_sync(0xffffffffu, s, k);
-    if (lane == 0) delta[(static_cast<int64_t>(b) * heads + h) * lse_rows + (s1 ? base1 : 0) + row] = s;
+    for (int k = 0; k < kPer; ++k) {
+        const int row = first + k * kRowsPerPass;
+        const uint32_t ow[4] = {ov[k].x, ov[k].y, ov[k].z, ov[k].w}, gw[4] = {gv[k].x, gv[k].y, gv[k].z, gv[k].w},
+                       lw[4] = {lv[k].x, lv[k].y, lv[k].z, lv[k].w};
+        float s = 0.f;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            float2 of = unpack_bf16x2(ow[e]);
+            const float2 lf = unpack_bf16x2(lw[e]);
+            of.x += lf.x;
+            of.y += lf.y;
+            const float2 gf = unpack_bf16x2(gw[e]);
+            s = fmaf(of.x, gf.x, fmaf(of.y, gf.y, s));
+        }
+        // rows past n summed zeros; every lane takes part in the shuffles
+#pragma unroll
+        for (int m = kLanes / 2; m; m >>= 1) s += __shfl_xor_sync(0xffffffffu, s, m);
+        if (c == 0 && row < n) {
+            ndelta[lbase + row] = -s;
+            nlse[lbase + row] = -lse_v[k];
+        }
+    }
 }
 
 // ------------------------------------------------------------------ dQ
@@ -254,10 +288,16 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_const
         const uint64_t dq_ = smem_desc_k_sw128(smem_u32(sQ));
         const uint64_t ddo = smem_desc_k_sw128(smem_u32(sdO));
         auto wait_kv = [&](int j) { return mbar_wait(&bar.grp_full[j & 3], (j >> 2) & 1); };
-        // S = Q K_j^T and dP = dO V_j^T of the whole key tile
-        auto issue_sdp = [&](int j) {
-            const uint64_t dk = smem_desc_k_sw128(smem_u32(sKV + (j % kKSlots) * kTileBytes));
-            const uint64_t dv = smem_desc_k_sw128(smem_u32(sKV + (kKSlots + j % kVSlots) * kTileBytes));
+        // slot descriptors: slot s starts s * kTileBytes further on, s * kTileBytes / 16
+        // in the descriptor's start-address field
+        constexpr uint32_t kSlotStep = kTileBytes >> 4;
+        const uint64_t k_k0 = smem_desc_k_sw128(smem_u32(sKV));
+        const uint64_t k_m0 = smem_desc_mn_sw128(smem_u32(sKV), kT * 128);
+        const uint64_t v_k0 = smem_desc_k_sw128(smem_u32(sKV + kKSlots * kTileBytes));
+        // S = Q K_j^T and dP = dO V_j^T of the whole key tile (K_j in K slot ks, V_j in V slot vs)
+        auto issue_sdp = [&](int j, int ks, int vs) {
+            const uint64_t dk = k_k0 + ks * kSlotStep;
+            const uint64_t dv = v_k0 + vs * kSlotStep;
 #pragma unroll
             for (int k = 0; k < HD / 16; ++k) {
                 const uint32_t off = ((k / 4) * (kT * 128) + (k % 4) * 32) >> 4;
@@ -269,20 +309,23 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_const
         if (ok && !wait_kv(0)) { fail(); ok = false; }
         if (ok) {
             tc_fence_after();
-            issue_sdp(0);
+            issue_sdp(0, 0, 0);
         }
+        int ks = 0, vs = 0;   // slots of K_j and V_j
         for (int j = 0; ok && j < ntiles; ++j) {
+            const uint64_t dkm = k_m0 + ks * kSlotStep;
+            ks = ks + 1 == kKSlots ? 0 : ks + 1;
+            vs = vs + 1 == kVSlots ? 0 : vs + 1;
             // the elementwise warps hold S_j / dP_j in registers: the next tile's may go in
             if (!mbar_wait(&bar.p_full[0], j & 1)) { fail(); ok = false; break; }
             if (j + 1 < ntiles) {
                 if (!wait_kv(j + 1)) { fail(); ok = false; break; }
                 tc_fence_after();
-                issue_sdp(j + 1);
+                issue_sdp(j + 1, ks, vs);
             }
             if (!mbar_wait(&bar.p_full[1], j & 1)) { fail(); ok = false; break; }
             tc_fence_after();
             // dQ += dS_j K_j: dS (keys 16 k.. at columns 8 k..) from TMEM, K_j rows as [keys (K) x d (N)]
-            const uint64_t dkm = smem_desc_mn_sw128(smem_u32(sKV + (j % kKSlots) * kTileBytes), kT * 128);
 #pragma unroll
             for (int k = 0; k < kT / 16; ++k)
                 tc_mma_bf16_ts(tmem + kColDq, tmem + kColDs + k * 8, dkm + static_cast<uint64_t>(k * (2048 >> 4)),
@@ -304,7 +347,7 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_const
         const bool live = row < p.nq[seg];
         const bool full_rows = q0 + kT <= p.nq[seg];   // every row of the tile is real (warp-uniform)
         const float lse = live ? p.lse[li] : 0.f;
-        const float dd = live ? p.delta[li] : 0.f;
+        const float ndd = live ? p.ndelta[li] : 0.f;   // -D
         bool ok = true;
         for (int j = 0; j < ntiles; ++j) {
             if (!mbar_wait(&bar.s0_ring[j & 3], (j >> 2) & 1)) { fail(); ok = false; break; }
@@ -324,7 +367,7 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_const
             if (valid >= 64 && full_rows) {
                 // every column and row real: paired fp32 arithmetic, no selects
                 const float2 c2 = make_float2(p.scale_log2, p.scale_log2), nl2 = make_float2(-lse, -lse);
-                const float2 nd2 = make_float2(-dd, -dd);
+                const float2 nd2 = make_float2(ndd, ndd);
 #pragma unroll
                 for (int i = 0; i < 64; i += 2) {
                     const float2 x = __ffma2_rn(make_float2(__uint_as_float(sr[i]), __uint_as_float(sr[i + 1])), c2, nl2);
@@ -339,7 +382,7 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_const
 #pragma unroll
                     for (int e = 0; e < 2; ++e) {
                         const float pv = ex2(fmaf(__uint_as_float(sr[i + e]), p.scale_log2, -lse));
-                        ds[e] = (i + e < valid && live) ? pv * (__uint_as_float(pr_[i + e]) - dd) : 0.f;
+                        ds[e] = (i + e < valid && live) ? pv * (__uint_as_float(pr_[i + e]) + ndd) : 0.f;
                     }
                     sr[i / 2] = pack_bf16x2(ds[0], ds[1]);
                 }
@@ -380,28 +423,31 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_const
 // (fp32, the whole 128-query tile: N = 128 MMAs); each elementwise warp
 // writes its 64 columns of P^T and dS^T as bf16 pairs over the first 32 of
 // its own S^T / dP^T columns; dV at 256, dK at 256 + d.  Per query tile i
-// the MMA thread issues dV += P^T dO_i and dK += dS^T Q_i, then at once
-// S^T / dP^T of tile i + 1: the tensor pipe runs one thread's MMAs in issue
-// order, so they overwrite P^T / dS^T only after dV / dK have read them.  Its
-// work per tile: two waits (P^T / dS^T written, operands of i + 1) and two
-// commits (tile i's slots free; S^T / dP^T of i + 1 ready).  Shared memory:
-// the K and V tiles of this CTA, then a ring of Q_i / dO_i tiles, then lse /
-// D of each streamed query tile.
+// the MMA thread issues dV += P^T dO_i once P^T is written, S^T of tile
+// i + 1 behind it, dK += dS^T Q_i once dS^T is written, then dP^T of i + 1:
+// the tensor pipe runs one thread's MMAs in issue order, so S^T_{i+1}
+// overwrites P^T_i only after dV_i has read it (dP^T_{i+1} and dS^T_i
+// likewise), and the elementwise work of a tile runs under the MMAs of its
+// neighbours.  Shared memory: the K and V tiles of this CTA, three Q_i slots,
+// two dO_i slots, lse_i per Q slot and D_i per dO slot.  Q_i and dO_i are
+// both read for the last time by dK_i / dV_i, but Q_i + 1 is needed a whole
+// step before dO_i + 1 (S^T comes first), so it gets the deeper ring.
 template <int HD>
 __global__ void __launch_bounds__(kThreads, 1)
 attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_constant__ CUtensorMap tm_q1,
                      const __grid_constant__ CUtensorMap tm_kv0, const __grid_constant__ CUtensorMap tm_kv1,
                      const __grid_constant__ CUtensorMap tm_do0, const __grid_constant__ CUtensorMap tm_do1,
                      const BwdParams p, int* status) {
-    constexpr int S_ = kSlotsDkdv;
     constexpr int kTileBytes = kT * HD * 2;
     constexpr int NB = HD / 64;
     extern __shared__ __align__(1024) uint8_t smem[];
     uint8_t* sK = smem;
     uint8_t* sV = smem + kTileBytes;
-    uint8_t* sQD = smem + 2 * kTileBytes;                     // [S_][tile]: Q_i, dO_i, Q_i+1, ...
-    float* sLD = reinterpret_cast<float*>(sQD + S_ * kTileBytes);   // [S_ / 2][2][kT]: lse, D
-    Bars& bar = *reinterpret_cast<Bars*>(reinterpret_cast<uint8_t*>(sLD) + (S_ / 2) * 2 * kT * 4);
+    uint8_t* sQ = smem + 2 * kTileBytes;                      // [kQSlots][tile]: Q_i in slot i % 3
+    uint8_t* sDo = sQ + kQSlots * kTileBytes;                 // [kDoSlots][tile]: dO_i in slot i % 2
+    float* sL = reinterpret_cast<float*>(sDo + kDoSlots * kTileBytes);   // [kQSlots][kT]: -lse_i
+    float* sD = sL + kQSlots * kT;                                         // [kDoSlots][kT]: -D_i
+    Bars& bar = *reinterpret_cast<Bars*>(sD + kDoSlots * kT);
     volatile int* abort_flag = &bar.abort_flag;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int b = blockIdx.z, h = blockIdx.y;
@@ -418,10 +464,12 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_con
         }
         mbar_init(&bar.fixed_full, 1);
         for (int g = 0; g < 4; ++g) {
-            mbar_init(&bar.grp_full[g], 2);
+            mbar_init(&bar.grp_full[g], 1);
+            mbar_init(&bar.do_full[g], 1);
             mbar_init(&bar.rel[g], 1);
         }
         mbar_init(&bar.s0_full, 1);
+        mbar_init(&bar.s1_full, 1);
         for (int s = 0; s < 2; ++s) mbar_init(&bar.p_full[s], kEw);
         mbar_init(&bar.done, 1);
         mbar_init(&bar.drain, 1);
@@ -441,38 +489,49 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_con
     };
     if (*abort_flag) {
     } else if (warp == 0 && lane == 0) {
-        // ---- producer: K and V of this tile, then per query tile i its Q_i
-        // and dO_i (one slot each) with lse_i / D_i riding on dO_i's barrier
+        // ---- producer: K and V of this tile, then Q_0, then per step n
+        // Q_n+1 and dO_n: both wait for step n - 2's MMAs (Q_n+1 goes into
+        // the slot of Q_n-2, dO_n into that of dO_n-2); lse_i rides on Q_i's
+        // barrier, D_i on dO_i's
         const CUtensorMap* tk = seg ? &tm_kv1 : &tm_kv0;
         mbar_arrive_expect_tx(&bar.fixed_full, 2 * kTileBytes);
         for (int c = 0; c < NB; ++c) {
             tma_load_2d(sK + c * (kT * 128), tk, &bar.fixed_full, p.k_col + h * HD + c * 64, b * p.nk[seg] + k0);
             tma_load_2d(sV + c * (kT * 128), tk, &bar.fixed_full, p.v_col + h * HD + c * 64, b * p.nk[seg] + k0);
         }
-        for (int n = 0; n < 2 * ntiles; ++n) {
-            const int s = n % S_;
-            if (n >= S_) {   // slot s held a tile of step (n - S_) / 2
-                const int r = (n - S_) >> 1;
+        auto tile_row = [&](int i, int& qs, int& qi) {
+            qs = i < nt0 ? 0 : 1;
+            qi = (i - (qs ? nt0 : 0)) * kT;
+        };
+        auto load_q = [&](int i) {
+            int qs, qi;
+            tile_row(i, qs, qi);
+            uint64_t* fb = &bar.grp_full[i & 3];
+            mbar_arrive_expect_tx(fb, kTileBytes + kT * 4);
+            uint8_t* dst = sQ + (i % kQSlots) * kTileBytes;
+            for (int c = 0; c < NB; ++c)
+                tma_load_2d(dst + c * (kT * 128), qs ? &tm_q1 : &tm_q0, fb, p.q_col + h * HD + c * 64, b * p.nq[qs] + qi);
+            bulk_load_1d(sL + (i % kQSlots) * kT, p.nlse + lrow + p.lse_base[qs] + qi, kT * 4, fb);
+        };
+        auto load_do = [&](int i) {
+            int qs, qi;
+            tile_row(i, qs, qi);
+            uint64_t* fb = &bar.do_full[i & 3];
+            mbar_arrive_expect_tx(fb, kTileBytes + kT * 4);
+            uint8_t* dst = sDo + (i % kDoSlots) * kTileBytes;
+            for (int c = 0; c < NB; ++c)
+                tma_load_2d(dst + c * (kT * 128), qs ? &tm_do1 : &tm_do0, fb, h * HD + c * 64, b * p.nq[qs] + qi);
+            bulk_load_1d(sD + (i % kDoSlots) * kT, p.ndelta + lrow + p.lse_base[qs] + qi, kT * 4, fb);
+        };
+        static_assert(kQSlots == kDoSlots + 1, "Q_n+1 and dO_n share their release");
+        load_q(0);
+        for (int n = 0; n < ntiles; ++n) {
+            if (n >= kDoSlots) {   // step n - 2's slots
+                const int r = n - kDoSlots;
                 if (!mbar_wait(&bar.rel[r & 3], (r >> 2) & 1)) { fail(); break; }
             }
-            uint64_t* fb = &bar.grp_full[(n >> 1) & 3];
-            const int i = n >> 1;
-            const int qs = i < nt0 ? 0 : 1;
-            const int qi = (i - (qs ? nt0 : 0)) * kT;
-            const int row = b * p.nq[qs] + qi;
-            uint8_t* dst = sQD + s * kTileBytes;
-            if (n & 1) {
-                float* ld = sLD + (s >> 1) * 2 * kT;
-                mbar_arrive_expect_tx(fb, kTileBytes + 2 * kT * 4);
-                for (int c = 0; c < NB; ++c)
-                    tma_load_2d(dst + c * (kT * 128), qs ? &tm_do1 : &tm_do0, fb, h * HD + c * 64, row);
-                bulk_load_1d(ld, p.lse + lrow + p.lse_base[qs] + qi, kT * 4, fb);
-                bulk_load_1d(ld + kT, p.delta + lrow + p.lse_base[qs] + qi, kT * 4, fb);
-            } else {
-                mbar_arrive_expect_tx(fb, kTileBytes);
-                for (int c = 0; c < NB; ++c)
-                    tma_load_2d(dst + c * (kT * 128), qs ? &tm_q1 : &tm_q0, fb, p.q_col + h * HD + c * 64, row);
-            }
+            if (n + 1 < ntiles) load_q(n + 1);
+            load_do(n);
         }
     } else if (warp == 1 && lane == 0) {
         // ---- MMA issuer
@@ -482,43 +541,81 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_con
         if (!ok) fail();
         const uint64_t dk_ = smem_desc_k_sw128(smem_u32(sK));
         const uint64_t dv_ = smem_desc_k_sw128(smem_u32(sV));
-        auto wait_qd = [&](int i) { return mbar_wait(&bar.grp_full[i & 3], (i >> 2) & 1); };
-        // S^T = K Q_i^T and dP^T = V dO_i^T of the whole query tile
-        auto issue_sdp = [&](int i) {
-            const uint64_t dq_ = smem_desc_k_sw128(smem_u32(sQD + ((2 * i) % S_) * kTileBytes));
-            const uint64_t ddo = smem_desc_k_sw128(smem_u32(sQD + ((2 * i + 1) % S_) * kTileBytes));
+        auto wait_q = [&](int i) { return mbar_wait(&bar.grp_full[i & 3], (i >> 2) & 1); };
+        auto wait_do = [&](int i) { return mbar_wait(&bar.do_full[i & 3], (i >> 2) & 1); };
+        // slot descriptors: slot s of a ring starts s * kTileBytes further on,
+        // s * kTileBytes / 16 in the descriptor's start-address field
+        constexpr uint32_t kSlotStep = kTileBytes >> 4;
+        const uint64_t q_k0 = smem_desc_k_sw128(smem_u32(sQ)), q_m0 = smem_desc_mn_sw128(smem_u32(sQ), kT * 128);
+        const uint64_t do_k0 = smem_desc_k_sw128(smem_u32(sDo)), do_m0 = smem_desc_mn_sw128(smem_u32(sDo), kT * 128);
+        // S^T = K Q_i^T and dP^T = V dO_i^T of the whole query tile, each
+        // published on its own barrier
+        auto issue_st = [&](int slot) {
+            const uint64_t dq_ = q_k0 + slot * kSlotStep;
 #pragma unroll
             for (int k = 0; k < HD / 16; ++k) {
                 const uint32_t off = ((k / 4) * (kT * 128) + (k % 4) * 32) >> 4;
                 tc_mma_bf16(tmem, dk_ + off, dq_ + off, idesc_s, k != 0 ? 1u : 0u);
-                tc_mma_bf16(tmem + kT, dv_ + off, ddo + off, idesc_s, k != 0 ? 1u : 0u);
             }
             tc_commit(&bar.s0_full);
         };
-        if (ok && !wait_qd(0)) { fail(); ok = false; }
+        auto issue_dpt = [&](int slot) {
+            const uint64_t ddo = do_k0 + slot * kSlotStep;
+#pragma unroll
+            for (int k = 0; k < HD / 16; ++k) {
+                const uint32_t off = ((k / 4) * (kT * 128) + (k % 4) * 32) >> 4;
+                tc_mma_bf16(tmem + kT, dv_ + off, ddo + off, idesc_s, k != 0 ? 1u : 0u);
+            }
+            tc_commit(&bar.s1_full);
+        };
+        if (ok && !wait_q(0)) { fail(); ok = false; }
         if (ok) {
             tc_fence_after();
-            issue_sdp(0);
+            issue_st(0);
         }
+        if (ok && !wait_do(0)) { fail(); ok = false; }
+        if (ok) {
+            tc_fence_after();
+            issue_dpt(0);
+        }
+        int qs = 0, ds = 0;   // slots of Q_i and dO_i
+        // Per query tile i: dV_i as soon as P^T_i is written, S^T_{i+1} behind
+        // it (it overwrites P^T_i, which dV_i has read: the tensor pipe runs
+        // one thread's MMAs in order), dK_i once dS^T_i is written, then
+        // dP^T_{i+1} over dS^T_i.  The elementwise warps form P^T_{i+1} while
+        // dK_i and dP^T_{i+1} run and dS^T_{i+1} while dV_{i+1} and
+        // S^T_{i+2} run, so the tensor pipe does not wait for them.
         for (int i = 0; ok && i < ntiles; ++i) {
+            const uint64_t dqm = q_m0 + qs * kSlotStep;
+            const uint64_t ddom = do_m0 + ds * kSlotStep;
+            qs = qs + 1 == kQSlots ? 0 : qs + 1;
+            ds = ds + 1 == kDoSlots ? 0 : ds + 1;
             if (!mbar_wait(&bar.p_full[0], i & 1)) { fail(); ok = false; break; }
             tc_fence_after();
-            const uint64_t dqm = smem_desc_mn_sw128(smem_u32(sQD + ((2 * i) % S_) * kTileBytes), kT * 128);
-            const uint64_t ddom = smem_desc_mn_sw128(smem_u32(sQD + ((2 * i + 1) % S_) * kTileBytes), kT * 128);
 #pragma unroll
             for (int k = 0; k < kT / 16; ++k) {
-                const uint64_t step = static_cast<uint64_t>(k * (2048 >> 4));
-                const uint32_t acc = (i | k) != 0 ? 1u : 0u;
                 // queries 16 k.. : each warp's 64 queries packed over the first 32 of its columns
                 const uint32_t a = tmem + (k >> 2) * 64 + (k & 3) * 8;
-                tc_mma_bf16_ts(tmem + 256, a, ddom + step, idesc_g, acc);             // dV += P^T dO
-                tc_mma_bf16_ts(tmem + 256 + HD, a + kT, dqm + step, idesc_g, acc);    // dK += dS^T Q
+                tc_mma_bf16_ts(tmem + 256, a, ddom + k * (2048 >> 4), idesc_g, (i | k) != 0 ? 1u : 0u);   // dV += P^T dO
+            }
+            const bool more = i + 1 < ntiles;
+            if (more) {
+                if (!wait_q(i + 1)) { fail(); ok = false; break; }
+                tc_fence_after();
+                issue_st(qs);
+            }
+            if (!mbar_wait(&bar.p_full[1], i & 1)) { fail(); ok = false; break; }
+            tc_fence_after();
+#pragma unroll
+            for (int k = 0; k < kT / 16; ++k) {
+                const uint32_t a = tmem + kT + (k >> 2) * 64 + (k & 3) * 8;
+                tc_mma_bf16_ts(tmem + 256 + HD, a, dqm + k * (2048 >> 4), idesc_g, (i | k) != 0 ? 1u : 0u);   // dK += dS^T Q
             }
             tc_commit(&bar.rel[i & 3]);   // Q_i, dO_i, lse_i and D_i read for the last time
-            if (i + 1 < ntiles) {
-                if (!wait_qd(i + 1)) { fail(); ok = false; break; }
+            if (more) {
+                if (!wait_do(i + 1)) { fail(); ok = false; break; }
                 tc_fence_after();
-                issue_sdp(i + 1);
+                issue_dpt(ds);
             }
         }
         if (ok) tc_commit(&bar.done);
@@ -535,59 +632,84 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_con
         const bool live = row < p.nk[seg];
         bool ok = true;
         for (int i = 0; i < ntiles; ++i) {
-            if (!mbar_wait(&bar.s0_full, i & 1)) { fail(); ok = false; break; }
-            tc_fence_after();
-            const int nd = 2 * i + 1;
-            const float* lse = sLD + ((nd % S_) >> 1) * 2 * kT + cg * 64;
-            const float* dl = lse + kT;
+            const float* nl = sL + (i % kQSlots) * kT + cg * 64;   // -lse of this warp's 64 queries
+            const float* nd = sD + (i % kDoSlots) * kT + cg * 64;  // -D
             const int qs = i < nt0 ? 0 : 1;
             // query columns < valid of this warp's 64 are real
             const int valid = p.nq[qs] - (i - (qs ? nt0 : 0)) * kT - cg * 64;
             const uint32_t tb = tS + cg * 64;
-            uint32_t sr[64], pr_[64];
-            tmem_ld_x32(tb, *reinterpret_cast<uint32_t(*)[32]>(&sr[0]));
-            tmem_ld_x32(tb + 32, *reinterpret_cast<uint32_t(*)[32]>(&sr[32]));
-            tmem_ld_x32(tb + kT, *reinterpret_cast<uint32_t(*)[32]>(&pr_[0]));
-            tmem_ld_x32(tb + kT + 32, *reinterpret_cast<uint32_t(*)[32]>(&pr_[32]));
+            // P^T = 2^(S^T log2(e) / sqrt(d) - lse), kept in fp32 for dS^T
+            float pf[64];
+            uint32_t u[64];
+            if (!mbar_wait(&bar.s0_full, i & 1)) { fail(); ok = false; break; }
+            tc_fence_after();
+            tmem_ld_x32(tb, *reinterpret_cast<uint32_t(*)[32]>(&u[0]));
+            tmem_ld_x32(tb + 32, *reinterpret_cast<uint32_t(*)[32]>(&u[32]));
             tmem_ld_wait();
             if (valid >= 64) {
                 // every query column real: paired fp32 arithmetic, no selects
                 const float2 c2 = make_float2(p.scale_log2, p.scale_log2);
 #pragma unroll
-                for (int c = 0; c < 64; c += 2) {
-                    const float2 l2 = *reinterpret_cast<const float2*>(lse + c);
-                    const float2 d2 = *reinterpret_cast<const float2*>(dl + c);
-                    const float2 x = __ffma2_rn(make_float2(__uint_as_float(sr[c]), __uint_as_float(sr[c + 1])), c2,
-                                                make_float2(-l2.x, -l2.y));
-                    const float2 pv = make_float2(ex2(x.x), ex2(x.y));
-                    const float2 dp = __fadd2_rn(make_float2(__uint_as_float(pr_[c]), __uint_as_float(pr_[c + 1])),
-                                                 make_float2(-d2.x, -d2.y));
-                    const float2 ds = __fmul2_rn(pv, dp);
-                    sr[c / 2] = pack_bf16x2(pv.x, pv.y);
-                    pr_[c / 2] = pack_bf16x2(ds.x, ds.y);
+                for (int c = 0; c < 64; c += 4) {
+                    const float4 l4 = *reinterpret_cast<const float4*>(nl + c);
+                    const float2 x0 = __ffma2_rn(make_float2(__uint_as_float(u[c]), __uint_as_float(u[c + 1])), c2,
+                                                 make_float2(l4.x, l4.y));
+                    const float2 x1 = __ffma2_rn(make_float2(__uint_as_float(u[c + 2]), __uint_as_float(u[c + 3])), c2,
+                                                 make_float2(l4.z, l4.w));
+                    pf[c] = ex2(x0.x);
+                    pf[c + 1] = ex2(x0.y);
+                    pf[c + 2] = ex2(x1.x);
+                    pf[c + 3] = ex2(x1.y);
                 }
             } else {
 #pragma unroll
-                for (int c = 0; c < 64; c += 2) {
-                    float pv[2], ds[2];
-#pragma unroll
-                    for (int e = 0; e < 2; ++e) {
-                        const bool real = c + e < valid;
-                        const float x = ex2(fmaf(__uint_as_float(sr[c + e]), p.scale_log2, -lse[c + e]));
-                        pv[e] = real ? x : 0.f;
-                        ds[e] = real ? x * (__uint_as_float(pr_[c + e]) - dl[c + e]) : 0.f;
-                    }
-                    sr[c / 2] = pack_bf16x2(pv[0], pv[1]);
-                    pr_[c / 2] = pack_bf16x2(ds[0], ds[1]);
+                for (int c = 0; c < 64; ++c) {
+                    const float x = ex2(fmaf(__uint_as_float(u[c]), p.scale_log2, nl[c]));
+                    pf[c] = c < valid ? x : 0.f;
                 }
             }
-            // packed over this warp's own (already read) S^T / dP^T columns
-            tmem_st_x32(tb, sr);
-            tmem_st_x32(tb + kT, pr_);
+#pragma unroll
+            for (int c = 0; c < 64; c += 2) u[c / 2] = pack_bf16x2(pf[c], pf[c + 1]);
+            // packed over this warp's own (already read) S^T columns
+            tmem_st_x32(tb, *reinterpret_cast<uint32_t(*)[32]>(&u[0]));
             tmem_st_wait();
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&bar.p_full[0]);
+            // dS^T = P^T (dP^T - D)
+            if (!mbar_wait(&bar.s1_full, i & 1)) { fail(); ok = false; break; }
+            tc_fence_after();
+            tmem_ld_x32(tb + kT, *reinterpret_cast<uint32_t(*)[32]>(&u[0]));
+            tmem_ld_x32(tb + kT + 32, *reinterpret_cast<uint32_t(*)[32]>(&u[32]));
+            tmem_ld_wait();
+            if (valid >= 64) {
+#pragma unroll
+                for (int c = 0; c < 64; c += 4) {
+                    const float4 d4 = *reinterpret_cast<const float4*>(nd + c);
+                    const float2 dp0 = __fadd2_rn(make_float2(__uint_as_float(u[c]), __uint_as_float(u[c + 1])),
+                                                  make_float2(d4.x, d4.y));
+                    const float2 dp1 = __fadd2_rn(make_float2(__uint_as_float(u[c + 2]), __uint_as_float(u[c + 3])),
+                                                  make_float2(d4.z, d4.w));
+                    const float2 ds0 = __fmul2_rn(make_float2(pf[c], pf[c + 1]), dp0);
+                    const float2 ds1 = __fmul2_rn(make_float2(pf[c + 2], pf[c + 3]), dp1);
+                    u[c / 2] = pack_bf16x2(ds0.x, ds0.y);
+                    u[c / 2 + 1] = pack_bf16x2(ds1.x, ds1.y);
+                }
+            } else {
+#pragma unroll
+                for (int c = 0; c < 64; c += 2) {
+                    float ds[2];
+#pragma unroll
+                    for (int e = 0; e < 2; ++e)
+                        ds[e] = c + e < valid ? pf[c + e] * (__uint_as_float(u[c + e]) + nd[c + e]) : 0.f;
+                    u[c / 2] = pack_bf16x2(ds[0], ds[1]);
+                }
+            }
+            tmem_st_x32(tb + kT, *reinterpret_cast<uint32_t(*)[32]>(&u[0]));
+            tmem_st_wait();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&bar.p_full[1]);
         }
         if (ok && mbar_wait(&bar.done, 0)) {
             tc_fence_after();
@@ -614,13 +736,14 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_con
 template <int HD>
 constexpr int smem_dq() { return 2 * kT * HD * 2 + kSlotsDq * kT * HD * 2 + kBarBytes; }
 template <int HD>
-constexpr int smem_dkdv() { return 2 * kT * HD * 2 + kSlotsDkdv * kT * HD * 2 + (kSlotsDkdv / 2) * 2 * kT * 4 + kBarBytes; }
+constexpr int smem_dkdv() { return (2 + kQSlots + kDoSlots) * kT * HD * 2 + (kQSlots + kDoSlots) * kT * 4 + kBarBytes; }
+static_assert(smem_dkdv<128>() <= 227 * 1024, "dK dV shared memory");
 static_assert(sizeof(Bars) <= kBarBytes, "barrier block too small");
 
 }  // namespace
 
 size_t attention_backward_ws_bytes(int B, int heads, int n0, int n1) {
-    return static_cast<size_t>(B) * heads * attn_lse_rows(n0, n1) * sizeof(float);
+    return 2 * static_cast<size_t>(B) * heads * attn_lse_rows(n0, n1) * sizeof(float);   // -D, then -lse
 }
 
 namespace {
@@ -633,6 +756,9 @@ int attention_backward_hd(const AttnBwdSpec& a, void* ws, size_t ws_bytes, cudaS
     if (B <= 0 || heads <= 0 || B > 65535 || heads > 65535 || nq0 < 0 || nq1 < 0 || nk0 < 0 || nk1 < 0 ||
         nq0 + nq1 <= 0 || nk0 + nk1 <= 0)
         return set_error(FF_ERR_INVALID_ARG, "attention backward: bad shape");
+    const int64_t qrows = static_cast<int64_t>(B) * (static_cast<int64_t>(nq0) + nq1);
+    if (qrows >= (int64_t{1} << 31))
+        return set_error(FF_ERR_INVALID_ARG, "attention backward: too many query rows");
     if (!a.lse || !ws) return set_error(FF_ERR_INVALID_ARG, "attention backward: null lse or workspace");
     const int H = heads * HD;
     if (a.q_col < 0 || a.k_col < 0 || a.v_col < 0 || a.q_col % 8 || a.k_col % 8 || a.v_col % 8)
@@ -642,7 +768,7 @@ int attention_backward_hd(const AttnBwdSpec& a, void* ws, size_t ws_bytes, cudaS
         const AttnBwdQuerySeg& q = a.q[i];
         if (q.n && (!q.q || !q.o || !q.dout || !q.dq || !aligned16(q.q) || !aligned16(q.o) || !aligned16(q.dout) ||
                     !aligned16(q.dq) || q.ld % 8 || q.ldo % 8 || q.ldg % 8 || q.ldq % 8 || q.ld < a.q_col + H ||
-                    q.ldo < H || q.ldg < H || q.ldq < H))
+                    q.ldo < H || q.ldg < H || q.ldq < H || (q.o_lo && (!aligned16(q.o_lo) || q.ldo_lo % 8 || q.ldo_lo < H))))
             return set_error(FF_ERR_INVALID_ARG, "attention backward: bad query segment %d", i);
         const AttnBwdKvSeg& k = a.kv[i];
         if (k.n && (!k.kv || !k.dk || !k.dv || !aligned16(k.kv) || !aligned16(k.dk) || !aligned16(k.dv) ||
@@ -666,15 +792,19 @@ int attention_backward_hd(const AttnBwdSpec& a, void* ws, size_t ws_bytes, cudaS
         const AttnBwdKvSeg& k = a.kv[i].n > 0 ? a.kv[i] : a.kv[1 - i];
         FF_TRY(make_tmap_bf16(&tkv[i], k.kv, static_cast<int64_t>(B) * k.n, kv_cols, k.ld, kT));
     }
-    float* delta = static_cast<float*>(ws);
+    float* ndelta = static_cast<float*>(ws);                            // -D
+    float* nlse = ndelta + static_cast<size_t>(B) * heads * attn_lse_rows(nq0, nq1);   // -lse
     const int rows = attn_lse_rows(nq0, nq1);
     {
-        const int64_t warps = (static_cast<int64_t>(B) * (nq0 + nq1)) * heads;
+        const int64_t heads_rows = (static_cast<int64_t>(B) * (nq0 + nq1)) * heads;
         const bool lo = a.q[0].o_lo || a.q[1].o_lo;
-        ProfScope prof(stream, "attn_bwd_delta", 0.0, (lo ? 6.0 : 4.0) * warps * HD);
-        attn_bwd_delta_kernel<HD><<<static_cast<unsigned>((warps + 7) / 8), 256, 0, stream>>>(
+        constexpr int R = delta_rows<HD>();
+        const int64_t blocks = static_cast<int64_t>(B) * ((nq0 + R - 1) / R + (nq1 + R - 1) / R);
+        ProfScope prof(stream, "attn_bwd_delta", 0.0, (lo ? 6.0 : 4.0) * heads_rows * HD);
+        attn_bwd_delta_kernel<HD><<<dim3(static_cast<unsigned>(blocks), heads), 256, 0, stream>>>(
             B, heads, nq0, nq1, a.q[0].o, a.q[0].dout, a.q[1].o, a.q[1].dout, a.q[0].ldo, a.q[1].ldo, a.q[0].ldg,
-            a.q[1].ldg, a.q[0].o_lo, a.q[1].o_lo, a.q[0].ldo_lo, a.q[1].ldo_lo, rows, attn_pad128(nq0), delta);
+            a.q[1].ldg, a.q[0].o_lo, a.q[1].o_lo, a.q[0].ldo_lo, a.q[1].ldo_lo, rows, attn_pad128(nq0), a.lse, ndelta,
+            nlse);
         FF_TRY(check_launch("attn_bwd_delta_kernel"));
     }
     BwdParams p;
@@ -690,7 +820,8 @@ int attention_backward_hd(const AttnBwdSpec& a, void* ws, size_t ws_bytes, cudaS
     p.scale_log2 = static_cast<float>(1.4426950408889634 / sqrt(static_cast<double>(HD)));
     p.scale = static_cast<float>(1.0 / sqrt(static_cast<double>(HD)));
     p.lse = a.lse;
-    p.delta = delta;
+    p.nlse = nlse;
+    p.ndelta = ndelta;
     p.lse_rows = rows;
     p.lse_base[0] = 0;
     p.lse_base[1] = attn_pad128(nq0);

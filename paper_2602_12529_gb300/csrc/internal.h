@@ -226,7 +226,8 @@ int attention_general(const AttnSpec& a, cudaStream_t stream);
 // Backward of joint attention (d = 64 or 128): from dO (bf16, the layout of the
 // forward's output) and the forward's lse, the gradients of q, k and v are
 // written into dqkv buffers laid out like the qkv inputs.  ws holds
-// D = rowsum(dO * O) in the lse layout (attention_backward_ws_bytes).
+// -D = -rowsum(dO * O) and a copy of -lse, both in the lse layout
+// (attention_backward_ws_bytes).
 struct AttnBwdSeg {
     const __nv_bfloat16* qkv; int64_t ld;   // q, k, v at columns 0, H, 2H
     const __nv_bfloat16* o;                  // forward output, row pitch ldo

@@ -87,6 +87,11 @@ def test_workspace_queries(L):
     assert ffi.ff_sde_workspace_size(4, 1 << 26) == 256 * 1024 + 4 * 1024 * 4
     with pytest.raises(ffi.FFError):
         ffi.ff_sde_workspace_size(0, 16)
+    # attention backward: -D and a copy of -lse, each fp32 [B, heads, L] with
+    # L = pad128(n0) + pad128(n1)
+    sz = ffi._SZ()
+    assert L.ff_attention_backward_workspace_size(2, 3, 100, 200, C.byref(sz)) == 0
+    assert sz.value == 2 * 2 * 3 * (128 + 256) * 4
 
 
 def test_host_validation_without_gpu(L):
