@@ -89,6 +89,17 @@ __device__ __forceinline__ void bulk_load_1d(void* dst, const void* src, uint32_
                  : "memory");
 }
 
+// Lane 0 waits for the barrier phase (when `need`), the warp learns the
+// outcome.  The elementwise warps check the next tile's operand barriers
+// this way before their own arrival, so the MMA thread's wait on that
+// arrival also covers the operands (TMA completion observed here, then
+// release by the arrival and acquire by the MMA thread's wait).
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, bool need, int lane) {
+    bool good = true;
+    if (need && lane == 0) good = mbar_wait(bar, parity);
+    return __shfl_sync(0xffffffffu, good ? 1 : 0, 0) != 0;
+}
+
 // Stores `cols` fp32 TMEM columns of this thread's row as bf16 (times mul).
 __device__ __forceinline__ void store_row_bf16(uint32_t taddr, float mul, __nv_bfloat16* dst, bool live,
                                                int cols) {
@@ -318,8 +329,7 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_const
             vs = vs + 1 == kVSlots ? 0 : vs + 1;
             // the elementwise warps hold S_j / dP_j in registers: the next tile's may go in
             if (!mbar_wait(&bar.p_full[0], j & 1)) { fail(); ok = false; break; }
-            if (j + 1 < ntiles) {
-                if (!wait_kv(j + 1)) { fail(); ok = false; break; }
+            if (j + 1 < ntiles) {   // the arrival also covers K_j+1 / V_j+1
                 tc_fence_after();
                 issue_sdp(j + 1, ks, vs);
             }
@@ -359,7 +369,12 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_const
             tmem_ld_x32(tS + kColP + cg * 64 + 32, *reinterpret_cast<uint32_t(*)[32]>(&pr_[32]));
             tmem_ld_wait();
             tc_fence_before();
-            __syncwarp();
+            // K_j+1 and V_j+1 landed too: the MMA thread issues S_j+1 / dP_j+1 on this arrival alone
+            if (!warp_wait(&bar.grp_full[(j + 1) & 3], ((j + 1) >> 2) & 1, j + 1 < ntiles, lane)) {
+                fail();
+                ok = false;
+                break;
+            }
             if (lane == 0) mbar_arrive(&bar.p_full[0]);   // S_j / dP_j consumed: the buffer may be refilled
             const int ks = j < nt0 ? 0 : 1;
             // key columns < valid of this warp's 64 are real
@@ -599,11 +614,7 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_con
                 tc_mma_bf16_ts(tmem + 256, a, ddom + k * (2048 >> 4), idesc_g, (i | k) != 0 ? 1u : 0u);   // dV += P^T dO
             }
             const bool more = i + 1 < ntiles;
-            if (more) {
-                if (!wait_q(i + 1)) { fail(); ok = false; break; }
-                tc_fence_after();
-                issue_st(qs);
-            }
+            if (more) issue_st(qs);   // the P^T arrival also covers Q_i+1
             if (!mbar_wait(&bar.p_full[1], i & 1)) { fail(); ok = false; break; }
             tc_fence_after();
 #pragma unroll
@@ -612,11 +623,7 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_con
                 tc_mma_bf16_ts(tmem + 256 + HD, a, dqm + k * (2048 >> 4), idesc_g, (i | k) != 0 ? 1u : 0u);   // dK += dS^T Q
             }
             tc_commit(&bar.rel[i & 3]);   // Q_i, dO_i, lse_i and D_i read for the last time
-            if (more) {
-                if (!wait_do(i + 1)) { fail(); ok = false; break; }
-                tc_fence_after();
-                issue_dpt(ds);
-            }
+            if (more) issue_dpt(ds);   // the dS^T arrival also covers dO_i+1
         }
         if (ok) tc_commit(&bar.done);
         tc_commit(&bar.drain);
@@ -674,7 +681,12 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_con
             tmem_st_x32(tb, *reinterpret_cast<uint32_t(*)[32]>(&u[0]));
             tmem_st_wait();
             tc_fence_before();
-            __syncwarp();
+            // Q_i+1 and lse_i+1 landed too: S^T_i+1 follows dV_i on this arrival alone
+            if (!warp_wait(&bar.grp_full[(i + 1) & 3], ((i + 1) >> 2) & 1, i + 1 < ntiles, lane)) {
+                fail();
+                ok = false;
+                break;
+            }
             if (lane == 0) mbar_arrive(&bar.p_full[0]);
             // dS^T = P^T (dP^T - D)
             if (!mbar_wait(&bar.s1_full, i & 1)) { fail(); ok = false; break; }
@@ -708,7 +720,12 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_con
             tmem_st_x32(tb + kT, *reinterpret_cast<uint32_t(*)[32]>(&u[0]));
             tmem_st_wait();
             tc_fence_before();
-            __syncwarp();
+            // dO_i+1 and D_i+1 landed too: dP^T_i+1 follows dK_i on this arrival alone
+            if (!warp_wait(&bar.do_full[(i + 1) & 3], ((i + 1) >> 2) & 1, i + 1 < ntiles, lane)) {
+                fail();
+                ok = false;
+                break;
+            }
             if (lane == 0) mbar_arrive(&bar.p_full[1]);
         }
         if (ok && mbar_wait(&bar.done, 0)) {
