@@ -6,8 +6,14 @@
 // h*d, k at H + h*d, v at 2H + h*d) by TMA; the segments may live in
 // different buffers.
 //
-// One CTA = two 128-row query tiles (256 query rows) of one segment of one
-// (sample, head), sharing every K/V tile.  Warp roles (10 warps):
+// Work item = two 128-row query tiles (256 query rows) of one segment of one
+// (sample, head), sharing every K/V tile.  The kernel is persistent: one CTA
+// per SM takes items blockIdx.x, blockIdx.x + gridDim.x, ... and runs their
+// K/V steps as one stream (global step g), so the ring, the operand groups
+// and the per-step barriers carry on across items without a restart; the
+// next item's query tile t is loaded as soon as the last S_t of the current
+// item is done, and its epilogue (O / l out of TMEM) overlaps the next
+// item's first S MMAs.  Warp roles (10 warps):
 //   warp 0      TMA producer: both Q tiles once, then the 128-token K and V
 //               tiles in the order K_0, V_0, K_1, V_1, ... into a ring of
 //               single-operand slots (5 at d = 128), so the operands of the
@@ -31,13 +37,14 @@
 // between MMA batches leaves the pipe idle unless it is short.  Hence:
 //   * the K/V ring is signalled in groups: group 0 = K_0, group j + 1 =
 //     (V_j, K_j+1), the operands of step j's MMAs, one barrier arrival pair
-//     per group (ring of four barriers), so the MMA thread waits once per
-//     step for its operands;
+//     per group (ring of four barriers); tile 0's softmax warps check group
+//     j + 1 before they publish P_0,j, so the MMA thread's wait for P_0,j
+//     covers the operands too;
 //   * slots are released by the commit that already publishes S_1,j+1 to
 //     tile 1's softmax (a ring of four barriers, one per step): when S_1,j+1
 //     is done, every MMA of step j is done, so V_j and K_j+1 may be
-//     overwritten.  Step j's MMA thread work is two waits for P, one wait
-//     for the operand group and two commits;
+//     overwritten.  Step j's MMA thread work is two waits for P and two
+//     commits;
 //   * the softmax keeps its first tile's row maximum m as the reference for
 //     every later tile (softmax does not depend on the reference, and P in
 //     bf16 / l in fp32 lose nothing when later scores exceed m), so only
@@ -64,8 +71,13 @@ struct ACfg {
     static constexpr int kQBytes = kBM * HD * 2;        // one query tile
     static constexpr int kKBytes = kBN * HD * 2;        // one K or V tile = one ring slot
     static constexpr int kBarBytes = 256;
-    static constexpr int kSlots = (232448 - 2 * kQBytes - kBarBytes) / kKBytes < 8
-                                      ? (232448 - 2 * kQBytes - kBarBytes) / kKBytes : 8;
+    // At most seven slots: ring item n arrives on group (n + 1) / 2, whose
+    // barrier entry it shares with group (n + 1) / 2 - 4, and only the wait
+    // for slot n % kSlots (for S_1 of step (n - kSlots + 1) / 2) guarantees
+    // that group has completed; with eight slots item 7 (V_3, group 4)
+    // would need no wait and could arrive while group 0 still waits for K_0.
+    static constexpr int kSlots = (232448 - 2 * kQBytes - kBarBytes) / kKBytes < 7
+                                      ? (232448 - 2 * kQBytes - kBarBytes) / kKBytes : 7;
     static constexpr int kSmemBytes = 2 * kQBytes + kSlots * kKBytes + kBarBytes;
     static constexpr int kTmemCols = 512;
     // TMEM columns of query tile t: S (fp32, kBN columns) at t*256, with P
@@ -77,6 +89,9 @@ struct AttnParams {
     int nq[2];           // query tokens per sample in each query segment
     int nkv[2];          // key/value tokens per sample in each key/value segment
     int qpairs0;         // 256-row query blocks of query segment 0 (segment 1's follow)
+    int qpairs;          // 256-row query blocks of both segments
+    int heads;
+    int items;           // B * heads * qpairs work items, item = (b * heads + h) * qpairs + block
     int q_col, k_col, v_col;
     float scale_log2;
     __nv_bfloat16* out[2];
@@ -94,15 +109,15 @@ struct AttnParams {
 // barriers below are waited in lockstep with their producer, and the rings
 // of four are waited at most one step behind (ring item n = 2 j (K_j) or
 // 2 j + 1 (V_j) lives in slot n % kSlots and belongs to group (n + 1) / 2).
-constexpr int kMaxSlots = 8;
+constexpr int kMaxSlots = 7;
 struct Bars {
-    uint64_t q_full;
+    uint64_t q_full[2];       // producer -> MMA: query tile t of the current item landed (one phase per item)
     uint64_t grp_full[4];     // producer -> MMA: K/V group g landed (ring entry g % 4; two arrivals)
     uint64_t s0_full;         // MMA -> softmax 0: S_0,j is in TMEM (and O_0 += P V_{j-1} done)
     uint64_t s1_ring[4];      // MMA -> softmax 1 and producer: S_1,j done (ring entry j % 4), so
                               // every MMA up to step j - 1 is done and its K/V slots are free
     uint64_t p_full[2];       // softmax -> MMA: P_t,j is in TMEM, O_t rescaled if needed
-    uint64_t o_last[2];       // MMA -> softmax: the last O += P V has landed
+    uint64_t o_last[2];       // MMA -> softmax: the item's last O += P V has landed (one phase per item)
     uint64_t drain;
     uint32_t tmem_slot;
     int abort_flag;
@@ -125,12 +140,26 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    const int b = blockIdx.z;
-    const int h = blockIdx.y;
-    const int seg = blockIdx.x < p.qpairs0 ? 0 : 1;
-    const int q0 = (blockIdx.x - (seg ? p.qpairs0 : 0)) * (2 * kBM);   // first query row within the segment
     const int nt0 = (p.nkv[0] + kBN - 1) / kBN;
-    const int ntiles = nt0 + (p.nkv[1] + kBN - 1) / kBN;
+    const int ntiles = nt0 + (p.nkv[1] + kBN - 1) / kBN;   // K/V steps per item
+    // persistent: this CTA takes items blockIdx.x, blockIdx.x + gridDim.x, ...
+    // and runs their K/V steps as one stream, global step g = k ntiles + j
+    // for local step j of its k-th item
+    const int nitems = p.items > static_cast<int>(blockIdx.x)
+                           ? (p.items - 1 - static_cast<int>(blockIdx.x)) / static_cast<int>(gridDim.x) + 1 : 0;
+    const int nsteps = nitems * ntiles;
+    struct Item { int b, h, seg, q0; };   // q0: first query row within the segment
+    auto item_of = [&](int k) {
+        const int it = static_cast<int>(blockIdx.x) + k * static_cast<int>(gridDim.x);
+        const int qp = it % p.qpairs;
+        const int bh = it / p.qpairs;
+        Item r;
+        r.h = bh % p.heads;
+        r.b = bh / p.heads;
+        r.seg = qp < p.qpairs0 ? 0 : 1;
+        r.q0 = (qp - (r.seg ? p.qpairs0 : 0)) * (2 * kBM);
+        return r;
+    };
 
     if (threadIdx.x == 0) {
         *abort_flag = 0;
@@ -138,7 +167,7 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
             report_status(status, kStatusBadArgument);
             *abort_flag = 1;
         }
-        mbar_init(&bar.q_full, 1);
+        for (int t = 0; t < 2; ++t) mbar_init(&bar.q_full[t], 1);
         for (int g = 0; g < 4; ++g) {
             mbar_init(&bar.grp_full[g], 2);
             mbar_init(&bar.s1_ring[g], 1);
@@ -150,7 +179,8 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
         }
         mbar_init(&bar.drain, 1);
         fence_mbar_init();
-        prefetch_tmap(seg ? &tm_q1 : &tm_q0);
+        prefetch_tmap(&tm_q0);
+        prefetch_tmap(&tm_q1);
         prefetch_tmap(&tm_kv0);
         prefetch_tmap(&tm_kv1);
     }
@@ -162,7 +192,7 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = bar.tmem_slot;
-    const bool aborted_at_start = *abort_flag;
+    const bool aborted_at_start = *abort_flag || nsteps == 0;
 
     auto fail = [&]() {
         report_status(status, kStatusWaitTimeout);
@@ -173,33 +203,60 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
         // nothing issued
     } else if (warp == 0 && lane == 0) {
         // ------------------------------------------------------------ producer
-        const CUtensorMap* tq = seg ? &tm_q1 : &tm_q0;
-        mbar_arrive_expect_tx(&bar.q_full, 2 * C::kQBytes);
-        for (int t = 0; t < 2; ++t)
+        auto load_q = [&](int t, const Item& it) {
+            mbar_arrive_expect_tx(&bar.q_full[t], C::kQBytes);
             for (int c = 0; c < HD / 64; ++c)
-                tma_load_2d(sQ + t * C::kQBytes + c * (kBM * 128), tq, &bar.q_full, p.q_col + h * HD + c * 64,
-                            b * p.nq[seg] + q0 + t * kBM);
-        for (int n = 0; n < 2 * ntiles && !*abort_flag; ++n) {
+                tma_load_2d(sQ + t * C::kQBytes + c * (kBM * 128), it.seg ? &tm_q1 : &tm_q0, &bar.q_full[t],
+                            p.q_col + it.h * HD + c * 64, it.b * p.nq[it.seg] + it.q0 + t * kBM);
+        };
+        // S_1 of the steps up to c is done: the ring entries are confirmed in
+        // step order, so each parity wait is for the entry's current phase
+        int seen = -1;
+        auto s1_done_upto = [&](int c) {
+            for (; seen < c; ++seen)
+                if (!mbar_wait(&bar.s1_ring[(seen + 1) & 3], ((seen + 1) >> 2) & 1)) return false;
+            return true;
+        };
+        Item cur = item_of(0);
+        load_q(0, cur);
+        load_q(1, cur);
+        for (int n = 0, k = 0, j = 0; n < 2 * nsteps; ++n) {
             const int s = n % S;
+            const int g = n >> 1;                 // global step of this K or V tile: item k, local step j
             // item n - S (group c = (n - S + 1) / 2) leaves slot s once the
             // MMAs of group c are done, i.e. once S_1,c is done (S_1,c is the
             // last MMA of step c - 1, and K_0's only readers are S_0,0 and
             // S_1,0)
-            if (n >= S) {
-                const int c = (n - S + 1) >> 1;
-                if (!mbar_wait(&bar.s1_ring[c & 3], (c >> 2) & 1)) { fail(); break; }
-            }
+            if (n >= S && !s1_done_upto((n - S + 1) >> 1)) { fail(); break; }
+            const bool new_item = !(n & 1) && j == 0 && k > 0;
+            if (new_item) cur = item_of(k);
             uint64_t* fb = &bar.grp_full[((n + 1) >> 1) & 3];
-            const int j = n >> 1;
             const int ks = j < nt0 ? 0 : 1;
-            const int row = b * p.nkv[ks] + (j - (ks ? nt0 : 0)) * kBN;
+            const int row = cur.b * p.nkv[ks] + (j - (ks ? nt0 : 0)) * kBN;
             const CUtensorMap* tkv = ks ? &tm_kv1 : &tm_kv0;
-            const int col = ((n & 1) ? p.v_col : p.k_col) + h * HD;
+            const int col = ((n & 1) ? p.v_col : p.k_col) + cur.h * HD;
             uint8_t* dst = sKV + s * C::kKBytes;
             mbar_arrive_expect_tx(fb, C::kKBytes);
             for (int c = 0; c < HD / 64; ++c)
                 tma_load_2d(dst + c * (kBN * 128), tkv, fb, col + c * 64, row);
-            if (n == 0 || n == 2 * ntiles - 1) mbar_arrive(fb);   // one-item groups: the second arrival
+            if (n == 0 || n == 2 * nsteps - 1) mbar_arrive(fb);   // one-item groups: the second arrival
+            if (new_item) {
+                // the new item's K_0 is on its way; its query tile t is free
+                // once S_t of step g - 1 (the previous item's last) is done.
+                // With S_1,g-2 (hence S_0,g-2) seen done, the two-phase
+                // s0_full stands at step g - 1, and it cannot pass it: S_0,g
+                // needs the tile loaded here.
+                if (!s1_done_upto(g - 2) || !mbar_wait(&bar.s0_full, (g - 1) & 1)) { fail(); break; }
+                load_q(0, cur);
+                if (!s1_done_upto(g - 1)) { fail(); break; }
+                load_q(1, cur);
+            }
+            if (n & 1) {
+                if (++j == ntiles) {
+                    j = 0;
+                    ++k;
+                }
+            }
         }
     } else if (warp == 1 && lane == 0) {
         // ------------------------------------------------------------ MMA issuer
@@ -211,7 +268,7 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
         // is awaited once per step, before O_0 += P_0,j V_j.
         constexpr uint32_t idesc_s = idesc_bf16_f32(kBM, kBN);
         constexpr uint32_t idesc_o = idesc_bf16_f32(kBM, HD) | (1u << 16);   // B (V) is MN-major
-        bool ok = mbar_wait(&bar.q_full, 0);
+        bool ok = mbar_wait(&bar.q_full[0], 0) && mbar_wait(&bar.q_full[1], 0);
         if (!ok) fail();
         auto group_ready = [&](int g) {
             if (!mbar_wait(&bar.grp_full[g & 3], (g >> 2) & 1)) return false;
@@ -223,9 +280,10 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
         // below 256 KB, so the field never carries), which keeps the issue
         // cost per MMA to a few instructions.
         const uint64_t desc_q[2] = {smem_desc_k_sw128(smem_u32(sQ)), smem_desc_k_sw128(smem_u32(sQ + C::kQBytes))};
-        auto issue_s = [&](int t, int j) {
+        // S_t,g for global step g
+        auto issue_s = [&](int t, int g) {
             const uint64_t dq = desc_q[t];
-            const uint64_t dk = smem_desc_k_sw128(smem_u32(sKV + ((2 * j) % S) * C::kKBytes));
+            const uint64_t dk = smem_desc_k_sw128(smem_u32(sKV + ((2 * g) % S) * C::kKBytes));
             const uint32_t dS = tmem + t * 256;
 #pragma unroll
             for (int k = 0; k < HD / 16; ++k) {
@@ -233,13 +291,14 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
                 const uint32_t off_k = ((k / 4) * (kBN * 128) + (k % 4) * 32) >> 4;
                 tc_mma_bf16(dS, dq + off_q, dk + off_k, idesc_s, k != 0 ? 1u : 0u);
             }
-            tc_commit(t == 0 ? &bar.s0_full : &bar.s1_ring[j & 3]);
+            tc_commit(t == 0 ? &bar.s0_full : &bar.s1_ring[g & 3]);
         };
-        auto issue_pv = [&](int t, int j) -> bool {
-            if (t == 0 && !group_ready(j + 1)) return false;   // V_j and K_j+1
-            if (!mbar_wait(&bar.p_full[t], j & 1)) return false;
+        // O_t += P_t,g V_g (local step j: the item's first step overwrites O_t)
+        auto issue_pv = [&](int t, int g, int j) -> bool {
+            // P_0,g's arrival also covers operand group g + 1 (V_g and K_g+1)
+            if (!mbar_wait(&bar.p_full[t], g & 1)) return false;
             tc_fence_after();
-            const uint64_t dv = smem_desc_mn_sw128(smem_u32(sKV + ((2 * j + 1) % S) * C::kKBytes), kBN * 128);
+            const uint64_t dv = smem_desc_mn_sw128(smem_u32(sKV + ((2 * g + 1) % S) * C::kKBytes), kBN * 128);
             const uint32_t dO = tmem + t * 256 + C::kColO;
             const uint32_t aP = tmem + t * 256;
 #pragma unroll
@@ -248,24 +307,38 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
                                (j | k) != 0 ? 1u : 0u);
             return true;
         };
-        if (ok && ntiles > 0) {
+        if (ok) {
             if (!group_ready(0)) { fail(); ok = false; }
             else {
                 issue_s(0, 0);
                 issue_s(1, 0);
             }
         }
-        for (int j = 0; ok && j < ntiles; ++j) {
-            const bool more = j + 1 < ntiles;
+        // Across items the order stays PV_t,g ; S_t,g+1: the next item's
+        // S_t,0 overwrites P_t of the last step only after PV has read it,
+        // and its first PV (which overwrites O_t) waits for P_t,0, which the
+        // softmax warps publish only after their epilogue has read O_t.
+        for (int g = 0, k = 0, j = 0; ok && g < nsteps; ++g) {
+            const bool more = g + 1 < nsteps;
+            const bool last = j == ntiles - 1;   // the item's last step
             for (int t = 0; t < 2; ++t) {
-                if (!issue_pv(t, j)) { fail(); ok = false; break; }
-                if (more) issue_s(t, j + 1);
+                if (!issue_pv(t, g, j)) { fail(); ok = false; break; }
+                if (last) tc_commit(&bar.o_last[t]);   // O_t of item k final once this lands
+                if (more) {
+                    if (last) {   // query tile t of item k + 1
+                        if (!mbar_wait(&bar.q_full[t], (k + 1) & 1)) { fail(); ok = false; break; }
+                        tc_fence_after();
+                    }
+                    issue_s(t, g + 1);
+                }
             }
             if (!ok) break;
-        }
-        if (ok) {
-            tc_commit(&bar.o_last[0]);
-            tc_commit(&bar.o_last[1]);
+            if (last) {
+                j = 0;
+                ++k;
+            } else {
+                ++j;
+            }
         }
         tc_commit(&bar.drain);
         if (!mbar_wait(&bar.drain, 0)) report_status(status, kStatusWaitTimeout);
@@ -276,137 +349,155 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
         const int r = q * 32 + lane;                     // query row within the tile = TMEM lane
         const uint32_t tS = tmem + (static_cast<uint32_t>(q * 32) << 16) + t * 256;
         const uint32_t tO = tS + C::kColO;
-        float m_used = -INFINITY;
-        float l = 0.f;
         bool ok = true;
-        for (int j = 0; j < ntiles; ++j) {
-            // S_t,j ready; O_t += P_t,j-1 V_j-1 has completed as well
-            if (!(t == 0 ? mbar_wait(&bar.s0_full, j & 1) : mbar_wait(&bar.s1_ring[j & 3], (j >> 2) & 1))) {
-                fail();
-                ok = false;
-                break;
-            }
-            tc_fence_after();
-            uint32_t sr[kBN];
-            tmem_ld_x128(tS, sr);
-            tmem_ld_wait();
-
-            const int ks = j < nt0 ? 0 : 1;
-            const int valid = p.nkv[ks] - (j - (ks ? nt0 : 0)) * kBN;   // columns < valid are real tokens
-            if (valid < kBN) {
-#pragma unroll
-                for (int i = 0; i < kBN; ++i)
-                    if (i >= valid) sr[i] = __float_as_uint(-INFINITY);
-            }
-            auto row_max = [&]() {
-                float mc[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-#pragma unroll
-                for (int i = 0; i < kBN; i += 8) {
-#pragma unroll
-                    for (int k = 0; k < 4; ++k)
-                        mc[k] = max3(mc[k], __uint_as_float(sr[i + 2 * k]), __uint_as_float(sr[i + 2 * k + 1]));
+        for (int k = 0; ok && k < nitems; ++k) {
+            const Item it = item_of(k);
+            float m_used = -INFINITY;
+            float l = 0.f;
+            for (int j = 0; j < ntiles; ++j) {
+                const int g = k * ntiles + j;   // global step
+                // S_t,g ready; O_t += P_t,g-1 V_g-1 has completed as well
+                if (!(t == 0 ? mbar_wait(&bar.s0_full, g & 1) : mbar_wait(&bar.s1_ring[g & 3], (g >> 2) & 1))) {
+                    fail();
+                    ok = false;
+                    break;
                 }
-                return max3(mc[0], mc[1], fmaxf(mc[2], mc[3])) * p.scale_log2;
-            };
-            // P = exp2(S scale - m) packed over the front of sr; returns the row sum
-            auto exps = [&](float m) {
-                const float2 c2 = make_float2(p.scale_log2, p.scale_log2);
-                const float2 nm2 = make_float2(-m, -m);
-                float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
-                                 make_float2(0.f, 0.f)};
-#pragma unroll
-                for (int i = 0; i < kBN; i += 2) {
-                    const float2 x = __ffma2_rn(make_float2(__uint_as_float(sr[i]), __uint_as_float(sr[i + 1])), c2, nm2);
-                    const float2 e = make_float2(ex2(x.x), ex2(x.y));
-                    acc[(i >> 1) & 3] = __fadd2_rn(acc[(i >> 1) & 3], e);
-                    sr[i / 2] = pack_bf16x2(e.x, e.y);
-                }
-                const float2 a01 = __fadd2_rn(acc[0], acc[1]);
-                const float2 a23 = __fadd2_rn(acc[2], acc[3]);
-                return (a01.x + a01.y) + (a23.x + a23.y);
-            };
-            // Softmax is unchanged by the reference m subtracted before the
-            // exponentials, so after the first tile the row keeps its first
-            // maximum as the reference and skips the max pass.  Later scores
-            // may exceed it: P up to 2^40 is exact enough in bf16 / fp32, and
-            // a tile whose row sum passes 2^40 (or overflows) is redone with
-            // the true maximum, rescaling l and O.
-            if (j == 0) m_used = row_max();
-            float lt = exps(m_used);
-            if (j > 0 && __any_sync(0xffffffffu, !(lt <= 0x1p40f))) {
+                tc_fence_after();
+                uint32_t sr[kBN];
                 tmem_ld_x128(tS, sr);
                 tmem_ld_wait();
+
+                const int ks = j < nt0 ? 0 : 1;
+                const int valid = p.nkv[ks] - (j - (ks ? nt0 : 0)) * kBN;   // columns < valid are real tokens
                 if (valid < kBN) {
 #pragma unroll
                     for (int i = 0; i < kBN; ++i)
                         if (i >= valid) sr[i] = __float_as_uint(-INFINITY);
                 }
-                const float m_new = fmaxf(m_used, row_max());
-                const float alpha = ex2(m_used - m_new);
-                lt = exps(m_new);
-                l *= alpha;
-                m_used = m_new;
+                auto row_max = [&]() {
+                    float mc[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+                    for (int i = 0; i < kBN; i += 8) {
+#pragma unroll
+                        for (int k = 0; k < 4; ++k)
+                            mc[k] = max3(mc[k], __uint_as_float(sr[i + 2 * k]), __uint_as_float(sr[i + 2 * k + 1]));
+                    }
+                    return max3(mc[0], mc[1], fmaxf(mc[2], mc[3])) * p.scale_log2;
+                };
+                // P = exp2(S scale - m) packed over the front of sr; returns the row sum
+                auto exps = [&](float m) {
+                    const float2 c2 = make_float2(p.scale_log2, p.scale_log2);
+                    const float2 nm2 = make_float2(-m, -m);
+                    float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                                     make_float2(0.f, 0.f)};
+#pragma unroll
+                    for (int i = 0; i < kBN; i += 2) {
+                        const float2 x = __ffma2_rn(make_float2(__uint_as_float(sr[i]), __uint_as_float(sr[i + 1])), c2, nm2);
+                        const float2 e = make_float2(ex2(x.x), ex2(x.y));
+                        acc[(i >> 1) & 3] = __fadd2_rn(acc[(i >> 1) & 3], e);
+                        sr[i / 2] = pack_bf16x2(e.x, e.y);
+                    }
+                    const float2 a01 = __fadd2_rn(acc[0], acc[1]);
+                    const float2 a23 = __fadd2_rn(acc[2], acc[3]);
+                    return (a01.x + a01.y) + (a23.x + a23.y);
+                };
+                // Softmax is unchanged by the reference m subtracted before the
+                // exponentials, so after the first tile the row keeps its first
+                // maximum as the reference and skips the max pass.  Later scores
+                // may exceed it: P up to 2^40 is exact enough in bf16 / fp32, and
+                // a tile whose row sum passes 2^40 (or overflows) is redone with
+                // the true maximum, rescaling l and O.
+                if (j == 0) m_used = row_max();
+                float lt = exps(m_used);
+                if (j > 0 && __any_sync(0xffffffffu, !(lt <= 0x1p40f))) {
+                    tmem_ld_x128(tS, sr);
+                    tmem_ld_wait();
+                    if (valid < kBN) {
+#pragma unroll
+                        for (int i = 0; i < kBN; ++i)
+                            if (i >= valid) sr[i] = __float_as_uint(-INFINITY);
+                    }
+                    const float m_new = fmaxf(m_used, row_max());
+                    const float alpha = ex2(m_used - m_new);
+                    lt = exps(m_new);
+                    l *= alpha;
+                    m_used = m_new;
+#pragma unroll 1
+                    for (int c = 0; c < HD; c += 32) {
+                        uint32_t o[32];
+                        tmem_ld_x32(tO + c, o);
+                        tmem_ld_wait();
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+                        tmem_st_x32(tO + c, o);
+                    }
+                }
+                l += lt;
+                // P_t,j (bf16 pairs) over the first kBN/2 columns of S_t
+#pragma unroll
+                for (int c = 0; c < kBN / 2; c += 32) tmem_st_x32(tS + c, &sr[c]);
+                tmem_st_wait();
+                tc_fence_before();
+                // tile 0 also checks operand group g + 1 (V_g, K_g+1): the MMA
+                // thread issues O_0 += P_0,g V_g and S_0,g+1 on this arrival alone
+                if (!warp_wait(&bar.grp_full[(g + 1) & 3], ((g + 1) >> 2) & 1, t == 0, lane)) {
+                    fail();
+                    ok = false;
+                    break;
+                }
+                if (lane == 0) mbar_arrive(&bar.p_full[t]);
+            }
+            if (!ok) break;
+            // ---- epilogue: O / l -> bf16, after the item's last O += P V, and
+            // the row's log-sum-exp m + log2(l) (base 2) when it is asked for.
+            // The next item's first O += P V waits for this warpgroup's P, so it
+            // cannot overwrite O_t before these loads.
+            if (mbar_wait(&bar.o_last[t], k & 1)) {
+                tc_fence_after();
+                const float inv = 1.f / l;
+                const int row = it.q0 + t * kBM + r;
+                const bool live = row < p.nq[it.seg];
+                if (p.lse && live)
+                    p.lse[(static_cast<int64_t>(it.b) * p.heads + it.h) * p.lse_rows + p.lse_base[it.seg] + row] =
+                        m_used + log2f(l);
+                const int64_t grow = static_cast<int64_t>(it.b) * p.nq[it.seg] + row;
+                __nv_bfloat16* dst = p.out[it.seg] + grow * p.ldo[it.seg] + it.h * HD;
+                __nv_bfloat16* dst_lo =
+                    p.out_lo[it.seg] ? p.out_lo[it.seg] + grow * p.ldo_lo[it.seg] + it.h * HD : nullptr;
 #pragma unroll 1
                 for (int c = 0; c < HD; c += 32) {
                     uint32_t o[32];
                     tmem_ld_x32(tO + c, o);
                     tmem_ld_wait();
+                    if (live) {
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
-                    tmem_st_x32(tO + c, o);
-                }
-            }
-            l += lt;
-            // P_t,j (bf16 pairs) over the first kBN/2 columns of S_t
+                        for (int w = 0; w < 4; ++w) {
+                            float f[8];
 #pragma unroll
-            for (int c = 0; c < kBN / 2; c += 32) tmem_st_x32(tS + c, &sr[c]);
-            tmem_st_wait();
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&bar.p_full[t]);
-        }
-        // ---- epilogue: O / l -> bf16, after the last O += P V, and the
-        // row's log-sum-exp m + log2(l) (base 2) when it is asked for
-        if (ok && ntiles > 0 && mbar_wait(&bar.o_last[t], 0)) {
-            tc_fence_after();
-            const float inv = 1.f / l;
-            const int row = q0 + t * kBM + r;
-            const bool live = row < p.nq[seg];
-            if (p.lse && live)
-                p.lse[(static_cast<int64_t>(b) * gridDim.y + h) * p.lse_rows + p.lse_base[seg] + row] = m_used + log2f(l);
-            const int64_t grow = static_cast<int64_t>(b) * p.nq[seg] + row;
-            __nv_bfloat16* dst = p.out[seg] + grow * p.ldo[seg] + h * HD;
-            __nv_bfloat16* dst_lo = p.out_lo[seg] ? p.out_lo[seg] + grow * p.ldo_lo[seg] + h * HD : nullptr;
-#pragma unroll 1
-            for (int c = 0; c < HD; c += 32) {
-                uint32_t o[32];
-                tmem_ld_x32(tO + c, o);
-                tmem_ld_wait();
-                if (live) {
+                            for (int i = 0; i < 8; ++i) f[i] = __uint_as_float(o[8 * w + i]) * inv;
+                            const uint4 hi = make_uint4(pack_bf16x2(f[0], f[1]), pack_bf16x2(f[2], f[3]),
+                                                        pack_bf16x2(f[4], f[5]), pack_bf16x2(f[6], f[7]));
+                            *reinterpret_cast<uint4*>(dst + c + 8 * w) = hi;
+                            if (dst_lo) {
+                                // what bf16 dropped, itself in bf16
+                                const uint32_t hw[4] = {hi.x, hi.y, hi.z, hi.w};
+                                uint32_t lw[4];
 #pragma unroll
-                    for (int k = 0; k < 4; ++k) {
-                        float f[8];
-#pragma unroll
-                        for (int i = 0; i < 8; ++i) f[i] = __uint_as_float(o[8 * k + i]) * inv;
-                        const uint4 hi = make_uint4(pack_bf16x2(f[0], f[1]), pack_bf16x2(f[2], f[3]),
-                                                    pack_bf16x2(f[4], f[5]), pack_bf16x2(f[6], f[7]));
-                        *reinterpret_cast<uint4*>(dst + c + 8 * k) = hi;
-                        if (dst_lo) {
-                            // what bf16 dropped, itself in bf16
-                            const uint32_t hw[4] = {hi.x, hi.y, hi.z, hi.w};
-                            uint32_t lw[4];
-#pragma unroll
-                            for (int i = 0; i < 4; ++i) {
-                                const float2 r = unpack_bf16x2(hw[i]);
-                                lw[i] = pack_bf16x2(f[2 * i] - r.x, f[2 * i + 1] - r.y);
+                                for (int i = 0; i < 4; ++i) {
+                                    const float2 r = unpack_bf16x2(hw[i]);
+                                    lw[i] = pack_bf16x2(f[2 * i] - r.x, f[2 * i + 1] - r.y);
+                                }
+                                *reinterpret_cast<uint4*>(dst_lo + c + 8 * w) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
                             }
-                            *reinterpret_cast<uint4*>(dst_lo + c + 8 * k) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
                         }
                     }
                 }
+                tmem_ld_wait();
+                tc_fence_before();
+            } else {
+                fail();
+                ok = false;
             }
-        } else if (ok && ntiles > 0) {
-            fail();
         }
     }
 
@@ -449,6 +540,11 @@ int launch_attn(const AttnSpec& a, cudaStream_t stream) {
         p.ldo_lo[i] = a.q[i].ldo_lo;
     }
     p.qpairs0 = (a.q[0].n + 2 * kBM - 1) / (2 * kBM);
+    p.qpairs = p.qpairs0 + (a.q[1].n + 2 * kBM - 1) / (2 * kBM);
+    p.heads = a.heads;
+    const int64_t items = static_cast<int64_t>(p.qpairs) * a.heads * a.B;
+    if (items >= (int64_t{1} << 31)) return set_error(FF_ERR_INVALID_ARG, "attention: too many query blocks");
+    p.items = static_cast<int>(items);
     p.lse = a.lse;
     p.lse_rows = attn_lse_rows(a.q[0].n, a.q[1].n);
     p.lse_base[0] = 0;
@@ -457,7 +553,9 @@ int launch_attn(const AttnSpec& a, cudaStream_t stream) {
     p.k_col = a.k_col;
     p.v_col = a.v_col;
     p.scale_log2 = static_cast<float>(1.4426950408889634 / sqrt(static_cast<double>(HD)));
-    const dim3 grid(p.qpairs0 + (a.q[1].n + 2 * kBM - 1) / (2 * kBM), a.heads, a.B);
+    // persistent: one CTA per SM (the kernel takes the whole shared memory), each
+    // running a strided share of the items
+    const int grid = static_cast<int>(items < num_sms() ? items : num_sms());
     const double nkv = static_cast<double>(a.kv[0].n + a.kv[1].n);
     const double nq = static_cast<double>(a.q[0].n + a.q[1].n);
     ProfScope prof(stream, "attention", 4.0 * a.B * a.heads * nq * nkv * HD,

@@ -89,17 +89,6 @@ __device__ __forceinline__ void bulk_load_1d(void* dst, const void* src, uint32_
                  : "memory");
 }
 
-// Lane 0 waits for the barrier phase (when `need`), the warp learns the
-// outcome.  The elementwise warps check the next tile's operand barriers
-// this way before their own arrival, so the MMA thread's wait on that
-// arrival also covers the operands (TMA completion observed here, then
-// release by the arrival and acquire by the MMA thread's wait).
-__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, bool need, int lane) {
-    bool good = true;
-    if (need && lane == 0) good = mbar_wait(bar, parity);
-    return __shfl_sync(0xffffffffu, good ? 1 : 0, 0) != 0;
-}
-
 // Stores `cols` fp32 TMEM columns of this thread's row as bf16 (times mul).
 __device__ __forceinline__ void store_row_bf16(uint32_t taddr, float mul, __nv_bfloat16* dst, bool live,
                                                int cols) {

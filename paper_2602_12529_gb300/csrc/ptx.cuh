@@ -78,6 +78,17 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
     return true;
 }
 
+// Lane 0 waits for the barrier phase (when `need`), the whole warp learns
+// the outcome.  Consumer warps check the next step's operand barriers this
+// way before their own arrival, so the MMA thread's wait on that arrival
+// also covers the operands (TMA completion observed here, then release by
+// the arrival and acquire by the MMA thread's wait).
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, bool need, int lane) {
+    bool good = true;
+    if (need && lane == 0) good = mbar_wait(bar, parity);
+    return __shfl_sync(0xffffffffu, good ? 1 : 0, 0) != 0;
+}
+
 // --------------------------------------------------------------------- TMA
 __device__ __forceinline__ void prefetch_tmap(const CUtensorMap* tm) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tm)) : "memory");

@@ -90,7 +90,11 @@ def test_gemm_gated_residual_parity(cuda, M, N, K, rps):
                                              (1, 2, 128, 512, 1024),
                                              # d = 128 runs on CTA pairs owning 512 query rows: partial
                                              # blocks, a second pair tile past the segment end, ragged K/V
-                                             (2, 2, 128, 300, 777), (1, 1, 128, 1000, 24), (3, 1, 128, 130, 513)])
+                                             (2, 2, 128, 300, 777), (1, 1, 128, 1000, 24), (3, 1, 128, 130, 513),
+                                             # more 256-row query blocks than SMs: each persistent CTA
+                                             # runs several blocks back to back (one K/V step per block,
+                                             # ragged segments, d = 64)
+                                             (8, 40, 128, 0, 256), (6, 40, 128, 0, 100), (3, 64, 64, 77, 300)])
 def test_attention_parity(cuda, B, heads, d, n0, n1):
     import torch
     from paper_2602_12529_gb300 import ffi
