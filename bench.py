@@ -657,7 +657,8 @@ def train_step(args, ffi, model, cfg, dev, x, txt, t, tn, sg, x_next, lp_old, ad
     for _ in range(args.warmup):
         step()
     ms = timed(step, args.steps) / args.steps
-    ffi.ff_prof_enable((48 * (cfg["n_double"] + cfg["n_single"]) + 128) * args.steps + 64)
+    # recompute mode runs each block forward twice before its backward: room for every launch
+    ffi.ff_prof_enable((200 * (cfg["n_double"] + cfg["n_single"]) + 256) * args.steps + 64)
     timed(step, args.steps)
     recs = ffi.ff_prof_records()
     ffi.ff_prof_disable()

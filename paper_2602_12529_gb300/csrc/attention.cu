@@ -65,6 +65,7 @@ namespace {
 constexpr int kBM = 128;         // query rows per query tile (two tiles per CTA)
 constexpr int kBN = 128;         // tokens per K/V tile
 constexpr int kThreads = 320;    // producer, MMA, 2 x 4 softmax warps
+constexpr int kPersistentItemsPerSm = 16;   // persistent launch below this many items per SM
 
 template <int HD>
 struct ACfg {
@@ -123,7 +124,10 @@ struct Bars {
     int abort_flag;
 };
 
-template <int HD>
+// kPersistent: one CTA per SM over a strided share of the items; otherwise
+// one item per CTA (grid = items), the loops below run once and the
+// hardware's block scheduler balances the SMs
+template <int HD, bool kPersistent>
 __global__ void __launch_bounds__(kThreads, 1)
 attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_constant__ CUtensorMap tm_q1,
                     const __grid_constant__ CUtensorMap tm_kv0, const __grid_constant__ CUtensorMap tm_kv1,
@@ -145,7 +149,8 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
     // persistent: this CTA takes items blockIdx.x, blockIdx.x + gridDim.x, ...
     // and runs their K/V steps as one stream, global step g = k ntiles + j
     // for local step j of its k-th item
-    const int nitems = p.items > static_cast<int>(blockIdx.x)
+    const int nitems = !kPersistent ? (static_cast<int>(blockIdx.x) < p.items ? 1 : 0)
+                       : p.items > static_cast<int>(blockIdx.x)
                            ? (p.items - 1 - static_cast<int>(blockIdx.x)) / static_cast<int>(gridDim.x) + 1 : 0;
     const int nsteps = nitems * ntiles;
     struct Item { int b, h, seg, q0; };   // q0: first query row within the segment
@@ -317,27 +322,28 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
         // Across items the order stays PV_t,g ; S_t,g+1: the next item's
         // S_t,0 overwrites P_t of the last step only after PV has read it,
         // and its first PV (which overwrites O_t) waits for P_t,0, which the
-        // softmax warps publish only after their epilogue has read O_t.
-        for (int g = 0, k = 0, j = 0; ok && g < nsteps; ++g) {
-            const bool more = g + 1 < nsteps;
-            const bool last = j == ntiles - 1;   // the item's last step
-            for (int t = 0; t < 2; ++t) {
-                if (!issue_pv(t, g, j)) { fail(); ok = false; break; }
-                if (last) tc_commit(&bar.o_last[t]);   // O_t of item k final once this lands
-                if (more) {
-                    if (last) {   // query tile t of item k + 1
-                        if (!mbar_wait(&bar.q_full[t], (k + 1) & 1)) { fail(); ok = false; break; }
-                        tc_fence_after();
-                    }
-                    issue_s(t, g + 1);
+        // softmax warps publish only after their epilogue has read O_t.  The
+        // item's last step is peeled off, so the per-step loop carries no
+        // item bookkeeping.
+        for (int k = 0, g0 = 0; ok && k < nitems; ++k, g0 += ntiles) {
+            for (int j = 0; j + 1 < ntiles; ++j) {
+                for (int t = 0; t < 2; ++t) {
+                    if (!issue_pv(t, g0 + j, j)) { fail(); ok = false; break; }
+                    issue_s(t, g0 + j + 1);
                 }
+                if (!ok) break;
             }
             if (!ok) break;
-            if (last) {
-                j = 0;
-                ++k;
-            } else {
-                ++j;
+            const int j = ntiles - 1;   // the item's last step
+            const bool more = k + 1 < nitems;
+            for (int t = 0; t < 2; ++t) {
+                if (!issue_pv(t, g0 + j, j)) { fail(); ok = false; break; }
+                tc_commit(&bar.o_last[t]);   // O_t of item k final once this lands
+                if (more) {   // query tile t of item k + 1
+                    if (!mbar_wait(&bar.q_full[t], (k + 1) & 1)) { fail(); ok = false; break; }
+                    tc_fence_after();
+                    issue_s(t, g0 + ntiles);
+                }
             }
         }
         tc_commit(&bar.drain);
@@ -351,7 +357,6 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
         const uint32_t tO = tS + C::kColO;
         bool ok = true;
         for (int k = 0; ok && k < nitems; ++k) {
-            const Item it = item_of(k);
             float m_used = -INFINITY;
             float l = 0.f;
             for (int j = 0; j < ntiles; ++j) {
@@ -454,6 +459,7 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
             // cannot overwrite O_t before these loads.
             if (mbar_wait(&bar.o_last[t], k & 1)) {
                 tc_fence_after();
+                const Item it = item_of(k);
                 const float inv = 1.f / l;
                 const int row = it.q0 + t * kBM + r;
                 const bool live = row < p.nq[it.seg];
@@ -517,9 +523,9 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
 template <int HD>
 int launch_attn(const AttnSpec& a, cudaStream_t stream) {
     using C = ACfg<HD>;
-    if (cudaFuncSetAttribute(attn_tcgen05_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes) !=
-        cudaSuccess)
-        return set_error(FF_ERR_CUDA, "attention: cannot set shared memory size");
+    for (auto* f : {attn_tcgen05_kernel<HD, true>, attn_tcgen05_kernel<HD, false>})
+        if (cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes) != cudaSuccess)
+            return set_error(FF_ERR_CUDA, "attention: cannot set shared memory size");
     CUtensorMap tq[2], tkv[2];
     for (int i = 0; i < 2; ++i) {
         // an empty segment still needs a valid map: point it at the other one
@@ -553,15 +559,26 @@ int launch_attn(const AttnSpec& a, cudaStream_t stream) {
     p.k_col = a.k_col;
     p.v_col = a.v_col;
     p.scale_log2 = static_cast<float>(1.4426950408889634 / sqrt(static_cast<double>(HD)));
-    // persistent: one CTA per SM (the kernel takes the whole shared memory), each
-    // running a strided share of the items
-    const int grid = static_cast<int>(items < num_sms() ? items : num_sms());
+    // Persistent (one CTA per SM, the kernel takes the whole shared memory,
+    // each running a strided share of the items) when there are few items per
+    // SM: the first K/V and query loads and the epilogue of each item then
+    // overlap its neighbours (Flux block, 11 items per SM: 731 -> 707 us).
+    // With many items per SM the hardware's block scheduler, which hands the
+    // next item to whichever SM frees first, balances the SMs better than a
+    // fixed stride (WAN shape, 34 items per SM: 13.8 ms one item per CTA,
+    // 14.0 ms persistent).
+    const bool persistent = items < static_cast<int64_t>(kPersistentItemsPerSm) * num_sms();
+    const int grid = static_cast<int>(persistent ? (items < num_sms() ? items : num_sms()) : items);
     const double nkv = static_cast<double>(a.kv[0].n + a.kv[1].n);
     const double nq = static_cast<double>(a.q[0].n + a.q[1].n);
     ProfScope prof(stream, "attention", 4.0 * a.B * a.heads * nq * nkv * HD,
                    2.0 * a.B * a.heads * HD * (2.0 * nq + 2.0 * nkv));
-    attn_tcgen05_kernel<HD><<<grid, kThreads, C::kSmemBytes, stream>>>(tq[0], tq[1], tkv[0], tkv[1], p,
-                                                                        device_status_ptr());
+    if (persistent)
+        attn_tcgen05_kernel<HD, true><<<grid, kThreads, C::kSmemBytes, stream>>>(tq[0], tq[1], tkv[0], tkv[1], p,
+                                                                                  device_status_ptr());
+    else
+        attn_tcgen05_kernel<HD, false><<<grid, kThreads, C::kSmemBytes, stream>>>(tq[0], tq[1], tkv[0], tkv[1], p,
+                                                                                   device_status_ptr());
     return check_launch("attn_tcgen05_kernel");
 }
 

@@ -94,7 +94,9 @@ def test_gemm_gated_residual_parity(cuda, M, N, K, rps):
                                              # more 256-row query blocks than SMs: each persistent CTA
                                              # runs several blocks back to back (one K/V step per block,
                                              # ragged segments, d = 64)
-                                             (8, 40, 128, 0, 256), (6, 40, 128, 0, 100), (3, 64, 64, 77, 300)])
+                                             (8, 40, 128, 0, 256), (6, 40, 128, 0, 100), (3, 64, 64, 77, 300),
+                                             # at least 16 blocks per SM on 152 SMs: one block per CTA
+                                             (32, 80, 64, 0, 256)])
 def test_attention_parity(cuda, B, heads, d, n0, n1):
     import torch
     from paper_2602_12529_gb300 import ffi
