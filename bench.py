@@ -57,7 +57,7 @@ def parse_args():
                    help="skip the extra measurements (other workloads, training, sweeps)")
     p.add_argument("--profile-kernel", default=None,
                    choices=["sde_step", "sde_step_philox", "grpo_loss", "group_advantage", "ln_modulate",
-                            "attention", "velocity"],
+                            "attention", "attention_backward", "velocity"],
                    help="launch only this kernel (a few times, no timing) for an ncu capture")
     p.add_argument("--elements", type=int, default=1 << 24, help="problem size of --profile-kernel's HBM kernels")
     return p.parse_args()
@@ -1152,7 +1152,7 @@ def profile_kernel(args):
         for _ in range(reps):
             ffi.ff_debug_ln_modulate(x, mods, 0, H, rows // cfg["batch"], out)
         what = f"ln_modulate: {rows} rows x {H} fp32 -> bf16 ({6 * rows * H / 1e6:.0f} MB per launch)"
-    elif k == "attention":
+    elif k in ("attention", "attention_backward"):
         B, heads, d = cfg["batch"], cfg["heads"], cfg["head_dim"]
         H = heads * d
         if cfg.get("arch") == "wan":
@@ -1163,9 +1163,17 @@ def profile_kernel(args):
         q1 = rnd(B * n1, 3 * H).to(torch.bfloat16)
         o0 = torch.empty(max(B * n0, 1), H, dtype=torch.bfloat16, device=dev)
         o1 = torch.empty(B * n1, H, dtype=torch.bfloat16, device=dev)
-        for _ in range(reps):
-            ffi.ff_attention_forward(B, heads, d, q0, o0, n0, q1, o1, n1)
-        what = f"attention: B {B}, {heads} x {d} heads, {n0} + {n1} tokens"
+        if k == "attention":
+            for _ in range(reps):
+                ffi.ff_attention_forward(B, heads, d, q0, o0, n0, q1, o1, n1)
+        else:   # the backward (D, dQ, dK / dV kernels) after one forward that keeps lse
+            lse = torch.empty(B * heads * ffi.lib().ff_attention_lse_rows(n0, n1), device=dev)
+            ffi.ff_attention_forward(B, heads, d, q0, o0, n0, q1, o1, n1, lse=lse)
+            g0, g1 = rnd(max(B * n0, 1), H).to(torch.bfloat16), rnd(B * n1, H).to(torch.bfloat16)
+            dq0, dq1 = torch.empty_like(q0), torch.empty_like(q1)
+            for _ in range(reps):
+                ffi.ff_attention_backward(B, heads, d, (n0, q0, o0, g0, dq0), (n1, q1, o1, g1, dq1), lse)
+        what = f"{k}: B {B}, {heads} x {d} heads, {n0} + {n1} tokens"
     else:
         model, blob, _ = make_model(ffi, cfg, dev)
         si = StepInputs(ffi, cfg, dev, 0)
