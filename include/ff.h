@@ -444,13 +444,17 @@ int ff_dit_velocity(const ff_dit* model, int B, const float* x_t, const void* tx
  * single-stream block, R = B (N_t + N_i), plus scratch; per WAN block
  * R_i (42 H + 4 F) + 8 R_t H bytes (R_i = B N_i, R_t = B N_t).
  * ------------------------------------------------------------------------ */
-/* Recompute mode of the training pass: ff_dit_forward_train keeps only every
- * block's input residual (fp32, 4 H bytes per residual row) and the backward
- * re-runs block l's forward into one shared activation set (one per block
- * kind) just before that block's backward.  One more forward of the blocks;
- * 4 H bytes per row and block instead of the stored activations.  The
- * gradient is bit-identical to the stored-activation pass (every kernel is
- * deterministic).  Set it before ff_dit_train_workspace_size and keep it
+/* Recompute mode of the training pass (on = 1 or 2; 0 stores every
+ * activation): ff_dit_forward_train keeps every block's input residual (fp32,
+ * 4 H bytes per residual row) and the backward re-runs block l's forward into
+ * one shared activation set (one per block kind) just before that block's
+ * backward.  on = 1 also keeps the self-attention output of every WAN block
+ * and the joint-attention output of every double-stream MMDiT block (O and
+ * its low part in bf16 and lse: 4 H + 4 heads bytes per query row), and the
+ * re-run skips that attention, the most expensive kernel of a block; on = 2
+ * keeps the block inputs only and re-runs everything.  The gradient is
+ * bit-identical to the stored-activation pass in both modes (every kernel is
+ * deterministic).  Other values of on: FF_ERR_INVALID_ARG.  Set it before ff_dit_train_workspace_size and keep it
  * unchanged until the matching ff_dit_backward: ff_dit_backward returns
  * FF_ERR_INVALID_ARG when the mode differs from that of the model's latest
  * ff_dit_forward_train (or when there was none). */

@@ -29,7 +29,10 @@ struct ff_dit {
     const __nv_bfloat16* w;
     std::unordered_map<std::string, int64_t> off;
     int64_t mod_width;
-    int train_recompute = 0;   // training pass: keep block inputs only, re-run each block before its backward
+    // training pass: 0 keeps every activation; 1 keeps the block inputs and
+    // the attention outputs, re-running the rest of each block before its
+    // backward; 2 keeps the block inputs only
+    int train_recompute = 0;
     mutable int fwd_recompute = -1;   // the mode of the latest ff_dit_forward_train (-1: none yet)
 };
 
@@ -307,7 +310,7 @@ int wan_forward_block(const ff_dit* m, int B, int l, const DitBlockIo& io, const
             set_qk_norm(e, c, 2 * H, W(p + "q_norm.scale"), W(p + "k_norm.scale"), f.rope, 0);
             FF_TRY(gemm_bf16(io.h1, H, W(p + "qkv.w"), H, Ri, 3 * H, H, e, stream));
         }
-        {
+        if (!io.attn_kept) {   // a re-run in recompute mode 1 finds O, its low part and lse kept
             AttnSpec a{};
             a.q[0] = AttnQuerySeg{nullptr, 0, 0, nullptr, 0};
             a.q[1] = AttnQuerySeg{io.qkv, 3 * H, Ni, io.o, H, io.o_lo, H};
@@ -516,7 +519,7 @@ int mmdit_forward_double(const ff_dit* m, int B, int l, const DitBlockIo& io, co
             }
             FF_TRY(gemm_bf16_group(g, 2, stream));
         }
-        {
+        if (!io.attn_kept) {   // a re-run in recompute mode 1 finds O, its low part and lse kept
             AttnSegment a0{io.qkv, 3 * H, io.o, H, Nt, io.o_lo, H};
             AttnSegment a1{io.qkv + static_cast<int64_t>(Rt) * 3 * H, 3 * H, io.o + static_cast<int64_t>(Rt) * H, H, Ni,
                            io.o_lo ? io.o_lo + static_cast<int64_t>(Rt) * H : nullptr, H};
@@ -731,7 +734,8 @@ int ff_dit_destroy(ff_dit* m) {
 int ff_dit_set_train_recompute(ff_dit* m, int on) {
     using namespace ff;
     if (!m) return set_error(FF_ERR_INVALID_ARG, "model is null");
-    m->train_recompute = on ? 1 : 0;
+    if (on < 0 || on > 2) return set_error(FF_ERR_INVALID_ARG, "recompute mode %d (0, 1 or 2)", on);
+    m->train_recompute = on;
     return FF_OK;
 }
 

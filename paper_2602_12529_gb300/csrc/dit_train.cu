@@ -30,9 +30,11 @@
 //   residual; lse;
 //   the final residual and LN-modulate output; then the backward's scratch.
 // In recompute mode (ff_dit_set_train_recompute) the blocks of each kind
-// share one set of those activations and only the block inputs are kept;
-// the backward re-runs each block's forward (bit-identical: every kernel is
-// deterministic) just before its backward.
+// share one set of those activations and only the block inputs are kept,
+// with (mode 1) each double block's joint-attention output, its low part and
+// lse; the backward re-runs each block's forward (bit-identical: every kernel
+// is deterministic) just before its backward, a double block's without its
+// attention in mode 1.
 #include <initializer_list>
 #include <string>
 #include <vector>
@@ -60,7 +62,7 @@ struct TrainPlan {
     size_t bytes;
 };
 
-TrainPlan plan(const ff_dit_config& c, int64_t Wm, int B, uint8_t* base, bool recompute) {
+TrainPlan plan(const ff_dit_config& c, int64_t Wm, int B, uint8_t* base, int recompute) {
     const size_t H = c.hidden, F = c.mlp, P = c.patch_dim, tf = c.time_freq_dim, d = c.head_dim;
     const size_t Nt = c.n_txt, Ni = static_cast<size_t>(c.grid_f) * c.grid_h * c.grid_w;
     const size_t Rt = B * Nt, Ri = B * Ni, R = Rt + Ri;
@@ -87,7 +89,8 @@ TrainPlan plan(const ff_dit_config& c, int64_t Wm, int B, uint8_t* base, bool re
     float* x = f32(R * H);
     f.x0 = x;
     // recompute: one activation set per block kind, shared by the blocks of
-    // that kind (re-filled by the backward); only the block inputs kept
+    // that kind (re-filled by the backward); kept per block: the input and,
+    // in mode 1, a double block's joint-attention O, its low part and lse
     DitBlockIo shared_dbl{}, shared_sgl{};
     bool have_dbl = false, have_sgl = false;
     for (int l = 0; l < L; ++l) {
@@ -97,6 +100,11 @@ TrainPlan plan(const ff_dit_config& c, int64_t Wm, int B, uint8_t* base, bool re
             io = dbl ? shared_dbl : shared_sgl;
             io.xin = x;
             if (!dbl) io.xmid = x;
+            if (dbl && recompute == 1) {
+                io.o = b16(R * H);
+                io.o_lo = b16(R * H);
+                io.lse = f32(lse_n);
+            }
             x = f32(R * H);
             io.xout = x;
             continue;
@@ -187,7 +195,7 @@ int ff_dit_train_workspace_size(const ff_dit* m, int B, size_t* bytes) {
     if (!bytes) return set_error(FF_ERR_INVALID_ARG, "bytes is null");
     *bytes = model_config(m).arch == FF_ARCH_WAN
                  ? wan_train_workspace_bytes(m, B)
-                 : plan(model_config(m), model_mod_width(m), B, nullptr, model_train_recompute(m) != 0).bytes;
+                 : plan(model_config(m), model_mod_width(m), B, nullptr, model_train_recompute(m)).bytes;
     return FF_OK;
 }
 
@@ -201,7 +209,7 @@ int ff_dit_forward_train(const ff_dit* m, int B, const float* x_t, const void* t
     const ff_dit_config& c = model_config(m);
     model_note_forward_train(m);
     if (c.arch == FF_ARCH_WAN) return wan_forward_train(m, B, x_t, txt, t, v_out, ws, ws_bytes, stream);
-    TrainPlan p = plan(c, model_mod_width(m), B, static_cast<uint8_t*>(ws), model_train_recompute(m) != 0);
+    TrainPlan p = plan(c, model_mod_width(m), B, static_cast<uint8_t*>(ws), model_train_recompute(m));
     if (ws_bytes < p.bytes) return set_error(FF_ERR_WORKSPACE, "workspace %zu B < %zu B needed", ws_bytes, p.bytes);
     p.f.blocks = p.blk.data();
     // the time-MLP operands' padding rows (the weight-gradient products read them)
@@ -230,7 +238,7 @@ int ff_dit_backward(const ff_dit* m, int B, const void* txt, const float* dv, fl
                                                  : "backward: recompute mode changed since ff_dit_forward_train");
     if (c.arch == FF_ARCH_WAN) return wan_backward(m, B, txt, dv, grad, dx_t, ws, ws_bytes, stream);
     const int64_t Wm = model_mod_width(m);
-    const bool recompute = model_train_recompute(m) != 0;
+    const int recompute = model_train_recompute(m);
     TrainPlan p = plan(c, Wm, B, static_cast<uint8_t*>(ws), recompute);
     if (ws_bytes < p.bytes) return set_error(FF_ERR_WORKSPACE, "workspace %zu B < %zu B needed", ws_bytes, p.bytes);
     const FwdBufs& f = p.f;
@@ -356,7 +364,11 @@ int ff_dit_backward(const ff_dit* m, int B, const void* txt, const float* dv, fl
     struct Stream { const char* name; int row0, rows, tokens, mod, first, cps; };
     for (int l = c.n_double - 1; l >= 0; --l) {
         const DitBlockIo& io = p.blk[l];
-        if (recompute) FF_TRY(mmdit_forward_double(m, B, l, io, f, stream));
+        if (recompute) {
+            DitBlockIo r = io;
+            r.attn_kept = recompute == 1;   // mode 1: the joint attention's outputs were kept
+            FF_TRY(mmdit_forward_double(m, B, l, r, f, stream));
+        }
         const int base = l * 12 * H;
         const int first_img = B * cps_t;
         const Stream st[2] = {{"img", Rt, Ri, Ni, base, first_img, cps_i}, {"txt", 0, Rt, Nt, base + 6 * H, 0, cps_t}};

@@ -370,6 +370,10 @@ struct DitBlockIo {
     float* x3;
     __nv_bfloat16 *hc, *qc, *qc_raw, *kv, *kv_raw, *oc;
     float* lse_c;
+    // training, recompute mode 1: o, o_lo and lse of the self / joint
+    // attention already hold this block's values (kept by the first
+    // forward), so a re-run of the block skips that attention
+    bool attn_kept = false;
 };
 struct FwdBufs {
     float* mods;

@@ -24,9 +24,10 @@
 //   text (+ raw) [R_t, 2H]; a1, u [R_i, F]; both attentions' log-sum-exp;
 //   the final residual and LN-modulate output; then the backward's scratch.
 // In recompute mode (ff_dit_set_train_recompute) the blocks share one set of
-// those activations and only their input residuals are kept; the backward
+// those activations and only their input residuals are kept, with (mode 1)
+// each block's self-attention output, its low part and lse; the backward
 // re-runs block l's forward (bit-identical, every kernel is deterministic)
-// just before its backward.
+// just before its backward, skipping the self-attention in mode 1.
 #include <initializer_list>
 #include <string>
 #include <vector>
@@ -54,7 +55,7 @@ struct WanPlan {
     size_t bytes;
 };
 
-WanPlan plan(const ff_dit_config& c, int64_t Wm, int B, uint8_t* base, bool recompute) {
+WanPlan plan(const ff_dit_config& c, int64_t Wm, int B, uint8_t* base, int recompute) {
     const size_t H = c.hidden, F = c.mlp, P = c.patch_dim, tf = c.time_freq_dim, d = c.head_dim;
     const size_t Nt = c.n_txt, Ni = static_cast<size_t>(c.grid_f) * c.grid_h * c.grid_w;
     const size_t Rt = B * Nt, Ri = B * Ni;
@@ -86,13 +87,19 @@ WanPlan plan(const ff_dit_config& c, int64_t Wm, int B, uint8_t* base, bool reco
     float* x = f32(Ri * H);
     f.x0 = x;
     // recompute: one activation set shared by every block (re-filled by the
-    // backward), only the block inputs kept
+    // backward); kept per block: the input and, in mode 1, the
+    // self-attention's O, its low part and lse
     DitBlockIo shared{};
     for (int l = 0; l < L; ++l) {
         DitBlockIo& io = p.blk[l];
         if (recompute && l > 0) {
             io = shared;
             io.xin = x;
+            if (recompute == 1) {
+                io.o = b16(Ri * H);
+                io.o_lo = b16(Ri * H);
+                io.lse = f32(lse_n);
+            }
             x = f32(Ri * H);
             io.xout = x;
             continue;
@@ -164,13 +171,13 @@ WanPlan plan(const ff_dit_config& c, int64_t Wm, int B, uint8_t* base, bool reco
 }  // namespace
 
 size_t wan_train_workspace_bytes(const ff_dit* m, int B) {
-    return plan(model_config(m), model_mod_width(m), B, nullptr, model_train_recompute(m) != 0).bytes;
+    return plan(model_config(m), model_mod_width(m), B, nullptr, model_train_recompute(m)).bytes;
 }
 
 int wan_forward_train(const ff_dit* m, int B, const float* x_t, const void* txt, const float* t, float* v_out,
                       void* ws, size_t ws_bytes, cudaStream_t stream) {
     const ff_dit_config& c = model_config(m);
-    WanPlan p = plan(c, model_mod_width(m), B, static_cast<uint8_t*>(ws), model_train_recompute(m) != 0);
+    WanPlan p = plan(c, model_mod_width(m), B, static_cast<uint8_t*>(ws), model_train_recompute(m));
     if (ws_bytes < p.bytes) return set_error(FF_ERR_WORKSPACE, "workspace %zu B < %zu B needed", ws_bytes, p.bytes);
     p.f.blocks = p.blk.data();
     // the time-MLP operands' padding rows (the weight-gradient products read them)
@@ -188,7 +195,7 @@ int wan_backward(const ff_dit* m, int B, const void* txt, const float* dv, float
                  size_t ws_bytes, cudaStream_t stream) {
     const ff_dit_config& c = model_config(m);
     const int64_t Wm = model_mod_width(m);
-    const bool recompute = model_train_recompute(m) != 0;
+    const int recompute = model_train_recompute(m);
     WanPlan p = plan(c, Wm, B, static_cast<uint8_t*>(ws), recompute);
     if (ws_bytes < p.bytes) return set_error(FF_ERR_WORKSPACE, "workspace %zu B < %zu B needed", ws_bytes, p.bytes);
     const FwdBufs& f = p.f;
@@ -250,7 +257,11 @@ int wan_backward(const ff_dit* m, int B, const void* txt, const float* dv, float
     for (int l = L - 1; l >= 0; --l) {
         const DitBlockIo& io = p.blk[l];
         // recompute: this block's activations again, from its kept input
-        if (recompute) FF_TRY(wan_forward_block(m, B, l, io, f, stream));
+        if (recompute) {
+            DitBlockIo r = io;
+            r.attn_kept = recompute == 1;   // mode 1: the self-attention's outputs were kept
+            FF_TRY(wan_forward_block(m, B, l, r, f, stream));
+        }
         const int base = l * 6 * H;
         const std::string pre = "blocks." + std::to_string(l) + ".";
         // FFN half: x_out = x3 + g2 (GELU(LNmod2(x3) W1^T + b1) W2^T + b2)

@@ -500,9 +500,11 @@ class Dit:
         _call("ff_dit_backward", self._h, B, _ptr(txt), _ptr(dv), _ptr(grad), _ptr(dx_t), _ptr(ws), ws.numel(),
               _stream(stream))
 
-    def set_train_recompute(self, on: bool):
-        """Training pass keeps only block inputs and re-runs each block in the backward (WAN-style models)."""
-        _call("ff_dit_set_train_recompute", self._h, 1 if on else 0)
+    def set_train_recompute(self, on):
+        """Training pass keeps the block inputs (and, for True or 1, the attention outputs; 2: the inputs
+        only) and re-runs each block in the backward."""
+        mode = (1 if on else 0) if isinstance(on, bool) else int(on)
+        _call("ff_dit_set_train_recompute", self._h, mode)
 
     def rollout_workspace_size(self, B: int, S: int) -> int:
         n = _SZ()

@@ -199,14 +199,21 @@ def test_training_pass_host_validation(L):
     Ri, Rt = 4 * 32, 4 * wcfg["n_txt"]
     assert n.value >= 2 * (Ri * (42 * 256 + 4 * 512) + Rt * 8 * 256)
     assert L.ff_dit_destroy(h) == 0
-    # recompute mode keeps only the block inputs: a smaller workspace
+    # recompute mode 2 keeps only the block inputs: a smaller workspace; mode 1
+    # also keeps the second block's self-attention O, its low part and lse
     full = n.value
     wan2 = ffi.make_config(wcfg)
     hr = C.c_void_p()
     assert L.ff_dit_create(C.byref(wan2), C.c_void_p(256), C.byref(hr)) == 0
+    assert L.ff_dit_set_train_recompute(hr, 2) == 0
+    assert L.ff_dit_train_workspace_size(hr, 4, C.byref(n)) == 0
+    only_inputs = n.value
+    assert only_inputs < full - Ri * (38 * 256 + 4 * 512)
     assert L.ff_dit_set_train_recompute(hr, 1) == 0
     assert L.ff_dit_train_workspace_size(hr, 4, C.byref(n)) == 0
-    assert n.value < full - Ri * (38 * 256 + 4 * 512)
+    assert only_inputs + Ri * 4 * 256 <= n.value < full - Ri * (34 * 256 + 4 * 512)
+    assert L.ff_dit_set_train_recompute(hr, 3) == 1
+    assert L.ff_dit_set_train_recompute(hr, -1) == 1
     assert L.ff_dit_destroy(hr) == 0
     c64b = ffi.make_config(synth.config("tiny_mmdit"))                 # 2 double blocks
     assert L.ff_dit_create(C.byref(c64b), C.c_void_p(256), C.byref(hr)) == 0

@@ -188,17 +188,19 @@ def test_wan_forward_train_equals_velocity_and_backward_is_deterministic(cuda):
 @pytest.mark.parametrize("cfg", [dict(WAN_TRAIN, n_double=1), dict(WAN_TRAIN, n_double=3),
                                  _cfg(n_double=2, n_single=0), _cfg(n_double=0, n_single=3),
                                  _cfg(n_double=2, n_single=2, grid=(1, 3, 5), n_txt=5, batch=8)])
-def test_recompute_gives_the_same_gradient(cuda, cfg):
+@pytest.mark.parametrize("mode", [1, 2])
+def test_recompute_gives_the_same_gradient(cuda, cfg, mode):
     """Recompute mode (block inputs kept, each block re-run before its
-    backward) gives bit for bit the stored-activation pass's v and gradients,
-    for WAN-style and MMDiT models."""
+    backward; mode 1 also keeps the self / joint attention outputs and the
+    re-run skips that attention) gives bit for bit the stored-activation
+    pass's v and gradients, for WAN-style and MMDiT models."""
     import torch
     from paper_2602_12529_gb300 import ffi
     L = cfg["n_double"] + cfg["n_single"]
     run = Run(cfg, cuda, seed=3)
     dv = np.random.default_rng(10).standard_normal(tuple(run.v.shape)).astype(np.float32)
     g1, d1 = run.backward(dv)
-    run.model.set_train_recompute(True)
+    run.model.set_train_recompute(mode)
     ws = torch.empty(run.model.train_workspace_size(run.B), dtype=torch.uint8, device=cuda)
     assert ws.numel() < run.ws.numel() or L == 1
     v2 = torch.empty_like(run.v)
