@@ -39,6 +39,13 @@ int ff_debug_attention(int B, int heads, int head_dim, int n0, const void* qkv0,
                        int64_t ldo0, int n1, const void* qkv1, int64_t ld1, void* out1, int64_t ldo1,
                        cudaStream_t stream);
 
+/* Which variant of the attention kernel every later forward launch takes,
+ * process-wide (for tests): 0 the launcher's own choice by item count and
+ * length, 1 the persistent one (one CTA per SM), 2 one 256-row query block
+ * per CTA.  Returns the previous setting; FF_ERR_INVALID_ARG (and no change)
+ * for other values.  The output does not depend on the variant. */
+int ff_debug_attention_launch(int mode);
+
 /* out[r] = LN(x[r]) * (1 + mods[b, scale_off:]) + mods[b, shift_off:] for
  * rows r of x (fp32 [rows, H]); b = r / tokens_per_sample; out bf16 [rows, H]. */
 int ff_debug_ln_modulate(int rows, int H, const float* x, const float* mods, int64_t ld_mods, int shift_off,

@@ -55,6 +55,8 @@
 // drains its tensor-core work, frees TMEM and returns.  The MMA and softmax
 // loops do not poll the abort flag: a role that gave up stops signalling, so
 // the others run into their own bounded waits.
+#include <atomic>
+
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -65,7 +67,9 @@ namespace {
 constexpr int kBM = 128;         // query rows per query tile (two tiles per CTA)
 constexpr int kBN = 128;         // tokens per K/V tile
 constexpr int kThreads = 320;    // producer, MMA, 2 x 4 softmax warps
-constexpr int kPersistentItemsPerSm = 16;   // persistent launch below this many items per SM
+constexpr int kPersistentItemsPerSm = 16;   // persistent launch below this many items per SM,
+constexpr int kPersistentMaxSteps = 128;    // or with at most this many K/V steps per item
+std::atomic<int> g_launch_override{0};      // tests: 1 forces the persistent variant, 2 one item per CTA
 
 template <int HD>
 struct ACfg {
@@ -561,13 +565,19 @@ int launch_attn(const AttnSpec& a, cudaStream_t stream) {
     p.scale_log2 = static_cast<float>(1.4426950408889634 / sqrt(static_cast<double>(HD)));
     // Persistent (one CTA per SM, the kernel takes the whole shared memory,
     // each running a strided share of the items) when there are few items per
-    // SM: the first K/V and query loads and the epilogue of each item then
-    // overlap its neighbours (Flux block, 11 items per SM: 731 -> 707 us).
-    // With many items per SM the hardware's block scheduler, which hands the
-    // next item to whichever SM frees first, balances the SMs better than a
-    // fixed stride (WAN shape, 34 items per SM: 13.8 ms one item per CTA,
-    // 14.0 ms persistent).
-    const bool persistent = items < static_cast<int64_t>(kPersistentItemsPerSm) * num_sms();
+    // SM or the items are short: the first K/V and query loads and the
+    // epilogue of each item then overlap its neighbours (Flux block, 11 items
+    // of 36 steps per SM: 731 -> 707 us; 24-block Flux rollout, 30 items of
+    // 12 steps per SM: 762 -> 723 us).  With many long items per SM the
+    // hardware's block scheduler, which hands the next item to whichever SM
+    // frees first, balances the SMs better than a fixed stride and the
+    // overlap is worth little (WAN self-attention, 34 items of 256 steps per
+    // SM: 13.8 ms one item per CTA, 14.0 ms persistent).
+    const int steps = (a.kv[0].n + kBN - 1) / kBN + (a.kv[1].n + kBN - 1) / kBN;
+    const int forced = g_launch_override.load(std::memory_order_relaxed);
+    const bool persistent = forced ? forced == 1
+                                   : items < static_cast<int64_t>(kPersistentItemsPerSm) * num_sms() ||
+                                         steps <= kPersistentMaxSteps;
     const int grid = static_cast<int>(persistent ? (items < num_sms() ? items : num_sms()) : items);
     const double nkv = static_cast<double>(a.kv[0].n + a.kv[1].n);
     const double nq = static_cast<double>(a.q[0].n + a.q[1].n);
@@ -583,6 +593,8 @@ int launch_attn(const AttnSpec& a, cudaStream_t stream) {
 }
 
 }  // namespace
+
+int attention_launch_override(int mode) { return g_launch_override.exchange(mode); }
 
 int attention_general(const AttnSpec& a, cudaStream_t stream) {
     if (a.B <= 0 || a.heads <= 0 || a.B > 65535 || a.heads > 65535)

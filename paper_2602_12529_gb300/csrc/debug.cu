@@ -156,6 +156,12 @@ int ff_debug_attention(int B, int heads, int head_dim, int n0, const void* qkv0,
     return attention(s0, s1, B, heads, head_dim, heads * head_dim, stream);
 }
 
+int ff_debug_attention_launch(int mode) {
+    using namespace ff;
+    if (mode < 0 || mode > 2) return set_error(FF_ERR_INVALID_ARG, "attention launch mode %d (0, 1 or 2)", mode);
+    return attention_launch_override(mode);
+}
+
 int ff_debug_ln_modulate(int rows, int H, const float* x, const float* mods, int64_t ld_mods, int shift_off,
                          int scale_off, int tokens_per_sample, void* out, cudaStream_t stream) {
     using namespace ff;

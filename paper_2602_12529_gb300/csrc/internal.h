@@ -222,6 +222,8 @@ struct AttnSpec {
 inline int attn_pad128(int n) { return (n + 127) / 128 * 128; }
 inline int attn_lse_rows(int n0, int n1) { return attn_pad128(n0) + attn_pad128(n1); }
 int attention_general(const AttnSpec& a, cudaStream_t stream);
+// forward launch variant for tests: 0 automatic, 1 persistent, 2 one item per CTA; returns the previous
+int attention_launch_override(int mode);
 
 // Backward of joint attention (d = 64 or 128): from dO (bf16, the layout of the
 // forward's output) and the forward's lse, the gradients of q, k and v are

@@ -96,6 +96,9 @@ def test_workspace_queries(L):
 
 def test_host_validation_without_gpu(L):
     # every one of these is rejected before any CUDA call is made
+    assert L.ff_debug_attention_launch(3) == 1          # variants are 0, 1, 2
+    assert L.ff_debug_attention_launch(2) == 0          # returns the previous setting
+    assert L.ff_debug_attention_launch(0) == 2
     rc = L.ff_sde_step_logprob(0, 16, None, None, None, None, None, None, None, 0, 0, None, 1, None, 0, None)
     assert rc == 1
     rc = L.ff_sde_step_logprob(2, 18, 16, 16, 16, 16, 16, 16, 16, 0, 0, 16, 1, 16, 1 << 20, None)

@@ -94,12 +94,23 @@ def test_gemm_gated_residual_parity(cuda, M, N, K, rps):
                                              # more 256-row query blocks than SMs: each persistent CTA
                                              # runs several blocks back to back (one K/V step per block,
                                              # ragged segments, d = 64)
-                                             (8, 40, 128, 0, 256), (6, 40, 128, 0, 100), (3, 64, 64, 77, 300),
-                                             # at least 16 blocks per SM on 152 SMs: one block per CTA
-                                             (32, 80, 64, 0, 256)])
-def test_attention_parity(cuda, B, heads, d, n0, n1):
+                                             (8, 40, 128, 0, 256), (6, 40, 128, 0, 100), (3, 64, 64, 77, 300)])
+@pytest.mark.parametrize("launch", [1, 2])
+def test_attention_parity(cuda, B, heads, d, n0, n1, launch):
+    """Both kernel variants (1: persistent CTAs over strided query blocks;
+    2: one 256-row query block per CTA) against the fp64 attention."""
     import torch
     from paper_2602_12529_gb300 import ffi
+    lib = ffi.lib()
+    assert lib.ff_debug_attention_launch(launch) == 0
+    try:
+        _attention_case(ffi, cuda, B, heads, d, n0, n1)
+    finally:
+        lib.ff_debug_attention_launch(0)
+
+
+def _attention_case(ffi, cuda, B, heads, d, n0, n1):
+    import torch
     H = heads * d
     ld0, ld1, ldo = 3 * H + 64, 3 * H, H + 128    # non-trivial pitches
     q0 = _bf((max(B * n0, 1), ld0), 11, 1.0, "q0")
@@ -121,6 +132,36 @@ def test_attention_parity(cuda, B, heads, d, n0, n1):
         assert rms_rel(got, want) <= 1e-2, (b, rms_rel(got, want))
     # columns beyond H of the outputs are untouched
     assert float(o1[:, H:].float().abs().max()) == 0.0
+
+
+@pytest.mark.parametrize("d", [64, 128])
+def test_attention_variants_bit_identical(cuda, d):
+    """The persistent variant (one CTA per SM running several query blocks
+    as one K/V stream) and the one-block-per-CTA variant compute every block
+    the same way: O and lse agree bit for bit (400 query blocks, two ragged
+    segments)."""
+    import torch
+    from paper_2602_12529_gb300 import ffi
+    lib = ffi.lib()
+    B, heads, n0, n1 = 2, 40, 77, 1000
+    H = heads * d
+    q0 = _dev_bf16(_bf((B * n0, 3 * H), 21, 1.0, "q0"), cuda)
+    q1 = _dev_bf16(_bf((B * n1, 3 * H), 22, 1.0, "q1"), cuda)
+    outs = []
+    for launch in (1, 2):
+        o0 = torch.zeros((B * n0, H), dtype=torch.bfloat16, device=cuda)
+        o1 = torch.zeros((B * n1, H), dtype=torch.bfloat16, device=cuda)
+        lse = torch.zeros(B * heads * lib.ff_attention_lse_rows(n0, n1), device=cuda)
+        assert lib.ff_debug_attention_launch(launch) == 0
+        try:
+            ffi.ff_attention_forward(B, heads, d, q0, o0, n0, q1, o1, n1, lse=lse)
+            torch.cuda.synchronize()
+        finally:
+            lib.ff_debug_attention_launch(0)
+        outs.append((o0, o1, lse))
+    assert ffi.ff_check_device_status() == 0
+    for a, b in zip(*outs):
+        assert torch.equal(a, b)
 
 
 @pytest.mark.parametrize("rows,H,tps", [(96, 256, 32), (1000, 3072, 250)])
