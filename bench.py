@@ -53,6 +53,8 @@ def parse_args():
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default=WORKLOAD)
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--train-only", action="store_true",
+                   help="of the extra measurements, only the training step (on this workload)")
     p.add_argument("--no-sweep", action="store_true",
                    help="skip the extra measurements (other workloads, training, sweeps)")
     p.add_argument("--profile-kernel", default=None,
@@ -627,15 +629,18 @@ def train_step(args, ffi, model, cfg, dev, x, txt, t, tn, sg, x_next, lp_old, ad
     need = model.train_workspace_size(B)
     _, total = ffi.ff_dit_weight_layout(cfg)
     free, _ = torch.cuda.mem_get_info(dev)
-    recompute = False
+    recompute = 0
     if need + 4 * total > 0.9 * free:
-        # keep only the block inputs and re-run each block in the backward
-        model.set_train_recompute(True)
-        recompute = True
-        need = model.train_workspace_size(B)
-        if need + 4 * total > 0.9 * free:
+        # keep the block inputs (mode 1: and the attention outputs) and re-run
+        # each block in the backward
+        for recompute in (1, 2):
+            model.set_train_recompute(recompute)
+            need = model.train_workspace_size(B)
+            if need + 4 * total <= 0.9 * free:
+                break
+        else:
             model.set_train_recompute(False)
-            return {"skipped": f"training workspace {need / 1e9:.1f} GB (recompute mode) + fp32 gradients "
+            return {"skipped": f"training workspace {need / 1e9:.1f} GB (recompute mode 2) + fp32 gradients "
                                f"{4 * total / 1e9:.1f} GB exceed the free device memory ({free / 1e9:.1f} GB)"}
     ws_t = torch.empty(need, dtype=torch.uint8, device=dev)
     grad = torch.empty(total, dtype=torch.float32, device=dev)
@@ -1023,13 +1028,14 @@ def run_ours(args):
     ms_e2e_serial = timed(e2e_serial, K_ser) / K_ser
     del pipe
 
-    extras = not args.no_sweep and rank == 0 and world == 1
+    want_train = (not args.no_sweep or args.train_only) and rank == 0 and world == 1
+    extras = want_train and not args.train_only
     light = argparse.Namespace(steps=min(args.steps, 3), warmup=min(args.warmup, 2))
     awm = awm_step(light, ffi, model, cfg, dev, si.x, si.txt, torch.randn_like(si.x), si.r, timed, world) \
         if extras else None
     train = train_step(argparse.Namespace(steps=2, warmup=1) if ms_step > 200 else light, ffi, model, cfg, dev,
                        si.x, si.txt, si.t, si.tn, si.sg, ctx["x_next"], ctx["lp_old"], ctx["adv"], ctx["dit_flops"],
-                       timed, world) if extras else None
+                       timed, world) if want_train else None
     model.close()
     del ctx, model, step
     torch.cuda.empty_cache()
