@@ -668,6 +668,151 @@ int silu_backward(const float* dy, int64_t ld_dy, const __nv_bfloat16* pre, int 
     return check_launch("silu_backward_kernel");
 }
 
+namespace {
+
+// dW[m, n] = sum_{b < B} dy[b, m] x[b, n], b in order: the weight gradient of
+// a Linear applied to B rows (the adaLN modulation, the time MLP).  A thread
+// writes four consecutive columns of kRowsW rows; x's slice stays in L1.
+constexpr int kRowsW = 8;
+__global__ void __launch_bounds__(256) rows_wgrad_kernel(int B, int M, int N, const float* __restrict__ dy,
+                                                         int64_t ldy, const __nv_bfloat16* __restrict__ x,
+                                                         int64_t ldx, float* __restrict__ dw, int64_t ldw) {
+    const int n = (blockIdx.y * 256 + threadIdx.x) * 4;
+    if (n >= N) return;
+    const int m0 = blockIdx.x * kRowsW;   // row groups on x: M reaches millions of rows
+    for (int m = m0; m < m0 + kRowsW && m < M; ++m) {
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int b = 0; b < B; ++b) {
+            const float g = dy[static_cast<int64_t>(b) * ldy + m];
+            const uint2 u = *reinterpret_cast<const uint2*>(x + static_cast<int64_t>(b) * ldx + n);
+            const float2 x01 = unpack_bf16x2(u.x), x23 = unpack_bf16x2(u.y);
+            acc.x = fmaf(g, x01.x, acc.x);
+            acc.y = fmaf(g, x01.y, acc.y);
+            acc.z = fmaf(g, x23.x, acc.z);
+            acc.w = fmaf(g, x23.y, acc.w);
+        }
+        *reinterpret_cast<float4*>(dw + static_cast<int64_t>(m) * ldw + n) = acc;
+    }
+}
+
+// dx[b, n] = sum_{m < M} dy[b, m] w[m, n]: the input gradient of a Linear
+// applied to B <= kRowsDgrad rows.  Stage 1: a block takes a chunk of rows of
+// w (a multiple of 8 rows) for 512 columns; a thread issues the loads of 8
+// rows (a warp reads 256 contiguous bytes of each) before their arithmetic,
+// and writes the chunk's partial sums; stage 2 sums the chunks in order.
+constexpr int kRowsDgrad = 16;
+// BMAX: accumulators for up to BMAX batch rows (4, 8 or 16), so a small batch
+// keeps the registers low and more rows' loads in flight per SM
+template <int BMAX>
+__global__ void __launch_bounds__(128) rows_dgrad_partial_kernel(int B, int M, int N, int rows_per_chunk,
+                                                                 const float* __restrict__ dy, int64_t ldy,
+                                                                 const __nv_bfloat16* __restrict__ w, int64_t ldw,
+                                                                 float* __restrict__ part) {
+    const int n = (blockIdx.x * 128 + threadIdx.x) * 4;
+    const int c = blockIdx.y;
+    const int m0 = c * rows_per_chunk;
+    const int m1 = min(M, m0 + rows_per_chunk);
+    if (n >= N) return;
+    float4 acc[BMAX];
+#pragma unroll
+    for (int b = 0; b < BMAX; ++b) acc[b] = make_float4(0.f, 0.f, 0.f, 0.f);
+    // rows m0 .. m1 in groups of 8 (m1 - m0 a multiple of 8): group g + 1's
+    // loads are in flight while group g is used
+    auto load8 = [&](int m, uint2 (&u)[8]) {
+#pragma unroll
+        for (int r = 0; r < 8; ++r) u[r] = *reinterpret_cast<const uint2*>(w + static_cast<int64_t>(m + r) * ldw + n);
+    };
+    uint2 cur[8], nxt[8];
+    if (m0 < m1) load8(m0, cur);
+    for (int m = m0; m < m1; m += 8) {
+        if (m + 8 < m1) load8(m + 8, nxt);
+        float2 wv[8][2];
+#pragma unroll
+        for (int r = 0; r < 8; ++r) {
+            wv[r][0] = unpack_bf16x2(cur[r].x);
+            wv[r][1] = unpack_bf16x2(cur[r].y);
+        }
+#pragma unroll
+        for (int b = 0; b < BMAX; ++b) {
+            if (b < B) {
+                // dy[b, m .. m + 7] (m and ldy multiples of 4)
+                const float* g = dy + static_cast<int64_t>(b) * ldy + m;
+                const float4 g0 = *reinterpret_cast<const float4*>(g);
+                const float4 g1 = *reinterpret_cast<const float4*>(g + 4);
+                const float gv[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+#pragma unroll
+                for (int r = 0; r < 8; ++r) {
+                    acc[b].x = fmaf(gv[r], wv[r][0].x, acc[b].x);
+                    acc[b].y = fmaf(gv[r], wv[r][0].y, acc[b].y);
+                    acc[b].z = fmaf(gv[r], wv[r][1].x, acc[b].z);
+                    acc[b].w = fmaf(gv[r], wv[r][1].y, acc[b].w);
+                }
+            }
+        }
+#pragma unroll
+        for (int r = 0; r < 8; ++r) cur[r] = nxt[r];
+    }
+#pragma unroll
+    for (int b = 0; b < BMAX; ++b)
+        if (b < B) *reinterpret_cast<float4*>(part + (static_cast<int64_t>(c) * B + b) * N + n) = acc[b];
+}
+
+__global__ void __launch_bounds__(256) rows_dgrad_sum_kernel(int B, int N, int chunks, const float* __restrict__ part,
+                                                             float* __restrict__ dx, int64_t ldx) {
+    const int n = (blockIdx.x * 256 + threadIdx.x) * 4;
+    const int b = blockIdx.y;
+    if (n >= N) return;
+    float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int c = 0; c < chunks; ++c) {
+        const float4 v = *reinterpret_cast<const float4*>(part + (static_cast<int64_t>(c) * B + b) * N + n);
+        s.x += v.x;
+        s.y += v.y;
+        s.z += v.z;
+        s.w += v.w;
+    }
+    *reinterpret_cast<float4*>(dx + static_cast<int64_t>(b) * ldx + n) = s;
+}
+
+}  // namespace
+
+int rows_wgrad(int B, int M, int N, const float* dy, int64_t ldy, const __nv_bfloat16* x, int64_t ldx, float* dw,
+               int64_t ldw, cudaStream_t stream) {
+    if (B <= 0 || M <= 0 || N <= 0 || N % 4 || ldx % 4 || ldw % 4 || ldy < M || ldx < N || ldw < N)
+        return set_error(FF_ERR_INVALID_ARG, "rows_wgrad: B=%d M=%d N=%d", B, M, N);
+    ProfScope prof(stream, "rows_wgrad", 2.0 * B * M * N, 4.0 * M * N + 2.0 * B * N + 4.0 * B * M);
+    if (N / 4 > 255 * 65535) return set_error(FF_ERR_INVALID_ARG, "rows_wgrad: N=%d", N);
+    const dim3 grid((M + kRowsW - 1) / kRowsW, (N / 4 + 255) / 256);
+    rows_wgrad_kernel<<<grid, 256, 0, stream>>>(B, M, N, dy, ldy, x, ldx, dw, ldw);
+    return check_launch("rows_wgrad_kernel");
+}
+
+int rows_dgrad_chunks(int M) {
+    const int by_rows = (M + 31) / 32;              // at least 32 rows per chunk
+    return by_rows < kRowsDgradMaxChunks ? by_rows : kRowsDgradMaxChunks;
+}
+
+int rows_dgrad(int B, int M, int N, const float* dy, int64_t ldy, const __nv_bfloat16* w, int64_t ldw, float* dx,
+               int64_t ldx, float* part, size_t part_floats, cudaStream_t stream) {
+    const int chunks = rows_dgrad_chunks(M);
+    if (B <= 0 || B > kRowsDgrad || M <= 0 || M % 8 || N <= 0 || N % 4 || ldw % 4 || ldx % 4 || ldy % 4 ||
+        ldy < M || ldw < N || ldx < N)
+        return set_error(FF_ERR_INVALID_ARG, "rows_dgrad: B=%d M=%d N=%d", B, M, N);
+    if (part_floats < static_cast<size_t>(chunks) * B * N)
+        return set_error(FF_ERR_WORKSPACE, "rows_dgrad: %zu partial floats < %zu", part_floats,
+                         static_cast<size_t>(chunks) * B * N);
+    const int rows_per_chunk = ((M + chunks - 1) / chunks + 7) / 8 * 8;   // chunks start on 8-row boundaries
+    {
+        ProfScope prof(stream, "rows_dgrad", 2.0 * B * M * N, 2.0 * M * N + 4.0 * B * M + 4.0 * chunks * B * N);
+        const dim3 grid((N / 4 + 127) / 128, chunks);
+        if (B <= 4) rows_dgrad_partial_kernel<4><<<grid, 128, 0, stream>>>(B, M, N, rows_per_chunk, dy, ldy, w, ldw, part);
+        else if (B <= 8) rows_dgrad_partial_kernel<8><<<grid, 128, 0, stream>>>(B, M, N, rows_per_chunk, dy, ldy, w, ldw, part);
+        else rows_dgrad_partial_kernel<16><<<grid, 128, 0, stream>>>(B, M, N, rows_per_chunk, dy, ldy, w, ldw, part);
+        FF_TRY(check_launch("rows_dgrad_partial_kernel"));
+    }
+    rows_dgrad_sum_kernel<<<dim3((N / 4 + 255) / 256, B), 256, 0, stream>>>(B, N, chunks, part, dx, ldx);
+    return check_launch("rows_dgrad_sum_kernel");
+}
+
 int wan_modulation_backward(const float* dmods, int64_t ld, int B, int rows_pad, int H, int L, float* gbias0,
                             int64_t stride, float* gfinal, float* de0, __nv_bfloat16* de0b, float* de_fin,
                             cudaStream_t stream) {

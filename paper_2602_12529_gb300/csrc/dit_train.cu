@@ -58,6 +58,8 @@ struct TrainPlan {
     void* attn_ws;
     size_t attn_ws_bytes;
     float *dmods, *dtc, *dth, *dc, *da;
+    float* rows_part;          // rows_dgrad's partial sums
+    size_t rows_part_floats;
     __nv_bfloat16 *dmods_b, *dc_b, *da_b;
     size_t bytes;
 };
@@ -162,6 +164,8 @@ TrainPlan plan(const ff_dit_config& c, int64_t Wm, int B, uint8_t* base, int rec
     p.da = f32(B * H);
     p.dc_b = b16(Kp * H);
     p.da_b = b16(Kp * H);
+    p.rows_part_floats = B <= kRowsMaxB ? static_cast<size_t>(rows_dgrad_chunks(static_cast<int>(Wm))) * B * H : 0;
+    p.rows_part = f32(p.rows_part_floats);
     p.bytes = o;
     return p;
 }
@@ -515,34 +519,50 @@ int ff_dit_backward(const ff_dit* m, int B, const void* txt, const float* dv, fl
         FF_TRY(group(&g, 1));
     }
 
-    // ---- modulation and the timestep MLP (B rows, padded to Kp for the products)
-    FF_TRY(f32_to_bf16(p.dmods, p.dmods_b, static_cast<int64_t>(B) * Wm, stream));
-    if (Kp > B && cudaMemsetAsync(p.dmods_b + static_cast<int64_t>(B) * Wm, 0,
-                                  static_cast<size_t>(Kp - B) * Wm * 2, stream) != cudaSuccess)
-        return set_error(FF_ERR_CUDA, "backward: memset failed");
-    {
+    // ---- modulation and the timestep MLP: Linears of B rows.  Up to
+    // kRowsMaxB rows their products run on HBM-bound kernels (the weight
+    // gradient is a write of M N fp32, the input gradient a read of the
+    // weight); larger batches take the tensor-core GEMM over Kp padded rows.
+    const bool few = B <= kRowsMaxB;
+    if (few) {
+        FF_TRY(rows_wgrad(B, static_cast<int>(Wm), H, p.dmods, Wm, f.tc, H, G("mod.w"), H, stream));
+    } else {
+        FF_TRY(f32_to_bf16(p.dmods, p.dmods_b, static_cast<int64_t>(B) * Wm, stream));
+        if (Kp > B && cudaMemsetAsync(p.dmods_b + static_cast<int64_t>(B) * Wm, 0,
+                                      static_cast<size_t>(Kp - B) * Wm * 2, stream) != cudaSuccess)
+            return set_error(FF_ERR_CUDA, "backward: memset failed");
         GemmArgs g = wgrad(p.dmods_b, Wm, f.tc, H, static_cast<int>(Wm), H, Kp, G("mod.w"));
         FF_TRY(group(&g, 1));
     }
     FF_TRY(colsum(p.dmods, true, Wm, B, static_cast<int>(Wm), G("mod.b"), p.cs_ws, stream));
-    {
+    if (few) {
+        FF_TRY(rows_dgrad(B, static_cast<int>(Wm), H, p.dmods, Wm, W("mod.w"), H, p.dtc, H, p.rows_part,
+                          p.rows_part_floats, stream));
+    } else {
         GemmArgs g = dgrad(p.dmods_b, Wm, W("mod.w"), Kp, H, static_cast<int>(Wm));
         g.epi.out_f32 = 1; g.epi.out0 = p.dtc; g.epi.ld0 = H;
         FF_TRY(group(&g, 1));
     }
     FF_TRY(silu_backward(p.dtc, H, f.pre_c, B, Kp, H, p.dc, p.dc_b, stream));
-    {
+    if (few) {
+        FF_TRY(rows_wgrad(B, H, H, p.dc, H, f.th, H, G("t_embed.fc2.w"), H, stream));
+    } else {
         GemmArgs g = wgrad(p.dc_b, H, f.th, H, H, H, Kp, G("t_embed.fc2.w"));
         FF_TRY(group(&g, 1));
     }
     FF_TRY(colsum(p.dc, true, H, B, H, G("t_embed.fc2.b"), p.cs_ws, stream));
-    {
+    if (few) {
+        FF_TRY(rows_dgrad(B, H, H, p.dc, H, W("t_embed.fc2.w"), H, p.dth, H, p.rows_part, p.rows_part_floats,
+                          stream));
+    } else {
         GemmArgs g = dgrad(p.dc_b, H, W("t_embed.fc2.w"), Kp, H, H);
         g.epi.out_f32 = 1; g.epi.out0 = p.dth; g.epi.ld0 = H;
         FF_TRY(group(&g, 1));
     }
     FF_TRY(silu_backward(p.dth, H, f.pre_fc1, B, Kp, H, p.da, p.da_b, stream));
-    {
+    if (few) {
+        FF_TRY(rows_wgrad(B, H, tf, p.da, H, f.temb, tf, G("t_embed.fc1.w"), tf, stream));
+    } else {
         GemmArgs g = wgrad(p.da_b, H, f.temb, tf, H, tf, Kp, G("t_embed.fc1.w"));
         FF_TRY(group(&g, 1));
     }

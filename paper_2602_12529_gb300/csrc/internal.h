@@ -332,6 +332,21 @@ int reduce_chunks(const float* part, int64_t ld_part, int ncols, const ChunkSpan
 // its bf16 copy [rows_pad, n], zero-padded.
 int silu_backward(const float* dy, int64_t ld_dy, const __nv_bfloat16* pre, int B, int rows_pad, int n, float* dx,
                   __nv_bfloat16* dxb, cudaStream_t stream, const float* add = nullptr);
+// The two products of a Linear applied to B rows (the adaLN modulation and
+// the time MLP), HBM-bound kernels in place of the tensor-core GEMM:
+//   rows_wgrad  dw[m, n] = sum_b dy[b, m] x[b, n]  (fp32 dy [B, ldy], bf16 x
+//               [B, ldx], fp32 dw [M, ldw]; the sum over b in order);
+//   rows_dgrad  dx[b, n] = sum_m dy[b, m] w[m, n]  (bf16 w [M, ldw], fp32 dx
+//               [B, ldx]; rows_dgrad_chunks(M) fixed chunks of rows, summed in
+//               order; B <= 16; part: rows_dgrad_chunks(M) B N floats).
+// N, ldx and ldw multiples of 4, 16-byte aligned rows.
+constexpr int kRowsDgradMaxChunks = 256;
+constexpr int kRowsMaxB = 16;   // batches up to this size use rows_wgrad / rows_dgrad
+int rows_wgrad(int B, int M, int N, const float* dy, int64_t ldy, const __nv_bfloat16* x, int64_t ldx, float* dw,
+               int64_t ldw, cudaStream_t stream);
+int rows_dgrad_chunks(int M);
+int rows_dgrad(int B, int M, int N, const float* dy, int64_t ldy, const __nv_bfloat16* w, int64_t ldw, float* dx,
+               int64_t ldx, float* part, size_t part_floats, cudaStream_t stream);
 // Backward of wan_modulation: from dmods [B, ld] (block l's 6H at l 6H, the
 // final layer's shift | scale at L 6H) the bias gradients (blocks.l.mod.b at
 // gbias0 + l stride, final.mod.b at gfinal; sums over the batch), d e0 =

@@ -51,6 +51,8 @@ struct WanPlan {
     void* attn_ws;
     size_t attn_ws_bytes;
     float *dmods, *de0, *de_fin, *dtc, *dc, *dth, *da;
+    float* rows_part;          // rows_dgrad's partial sums
+    size_t rows_part_floats;
     __nv_bfloat16 *de0_b, *dc_b, *da_b;
     size_t bytes;
 };
@@ -164,6 +166,8 @@ WanPlan plan(const ff_dit_config& c, int64_t Wm, int B, uint8_t* base, int recom
     p.dth = f32(Kp * H);
     p.da = f32(B * H);
     p.da_b = b16(Kp * H);
+    p.rows_part_floats = B <= kRowsMaxB ? static_cast<size_t>(rows_dgrad_chunks(static_cast<int>(6 * H))) * B * H : 0;
+    p.rows_part = f32(p.rows_part_floats);
     p.bytes = o;
     return p;
 }
@@ -410,24 +414,36 @@ int wan_backward(const ff_dit* m, int B, const void* txt, const float* dv, float
         FF_TRY(wan_modulation_backward(p.dmods, Wm, B, Kp, H, L, G("blocks.0.mod.b"), stride, G("final.mod.b"), p.de0,
                                        p.de0_b, p.de_fin, stream));
     }
-    FF_TRY(gemm1(gemm_wgrad(p.de0_b, 6 * H, f.tc, H, 6 * H, H, Kp, G("mod.w"))));
+    // Linears of B rows: HBM-bound kernels up to kRowsMaxB rows, the
+    // tensor-core GEMM over Kp padded rows beyond
+    const bool few = B <= kRowsMaxB;
+    if (few) FF_TRY(rows_wgrad(B, 6 * H, H, p.de0, 6 * H, f.tc, H, G("mod.w"), H, stream));
+    else FF_TRY(gemm1(gemm_wgrad(p.de0_b, 6 * H, f.tc, H, 6 * H, H, Kp, G("mod.w"))));
     FF_TRY(colsum(p.de0, true, 6 * H, B, 6 * H, G("mod.b"), p.cs_ws, stream));
-    {
+    if (few) {
+        FF_TRY(rows_dgrad(B, 6 * H, H, p.de0, 6 * H, W("mod.w"), H, p.dtc, H, p.rows_part, p.rows_part_floats,
+                          stream));
+    } else {
         GemmArgs g = gemm_dgrad(p.de0_b, 6 * H, W("mod.w"), Kp, H, 6 * H);
         g.epi.out_f32 = 1; g.epi.out0 = p.dtc; g.epi.ld0 = H;
         FF_TRY(gemm1(g));
     }
     // d e = d SiLU(e) SiLU'(e) + the final layer's shift and scale gradients
     FF_TRY(silu_backward(p.dtc, H, f.pre_c, B, Kp, H, p.dc, p.dc_b, stream, p.de_fin));
-    FF_TRY(gemm1(gemm_wgrad(p.dc_b, H, f.th, H, H, H, Kp, G("t_embed.fc2.w"))));
+    if (few) FF_TRY(rows_wgrad(B, H, H, p.dc, H, f.th, H, G("t_embed.fc2.w"), H, stream));
+    else FF_TRY(gemm1(gemm_wgrad(p.dc_b, H, f.th, H, H, H, Kp, G("t_embed.fc2.w"))));
     FF_TRY(colsum(p.dc, true, H, B, H, G("t_embed.fc2.b"), p.cs_ws, stream));
-    {
+    if (few) {
+        FF_TRY(rows_dgrad(B, H, H, p.dc, H, W("t_embed.fc2.w"), H, p.dth, H, p.rows_part, p.rows_part_floats,
+                          stream));
+    } else {
         GemmArgs g = gemm_dgrad(p.dc_b, H, W("t_embed.fc2.w"), Kp, H, H);
         g.epi.out_f32 = 1; g.epi.out0 = p.dth; g.epi.ld0 = H;
         FF_TRY(gemm1(g));
     }
     FF_TRY(silu_backward(p.dth, H, f.pre_fc1, B, Kp, H, p.da, p.da_b, stream));
-    FF_TRY(gemm1(gemm_wgrad(p.da_b, H, f.temb, tf, H, tf, Kp, G("t_embed.fc1.w"))));
+    if (few) FF_TRY(rows_wgrad(B, H, tf, p.da, H, f.temb, tf, G("t_embed.fc1.w"), tf, stream));
+    else FF_TRY(gemm1(gemm_wgrad(p.da_b, H, f.temb, tf, H, tf, Kp, G("t_embed.fc1.w"))));
     return colsum(p.da, true, H, B, H, G("t_embed.fc1.b"), p.cs_ws, stream);
 }
 

@@ -96,7 +96,10 @@ TINY64 = {k: v for k, v in synth.config("tiny_mmdit").items() if k in SMALL}
                                   {"grid": (1, 3, 5), "n_txt": 5, "batch": 8},
                                   {"batch": 3, "n_txt": 8, "grid": (1, 4, 6)},
                                   dict(TINY64),
-                                  dict(TINY64, n_double=1, n_single=1, grid=(1, 3, 5), n_txt=5, batch=8)])
+                                  dict(TINY64, n_double=1, n_single=1, grid=(1, 3, 5), n_txt=5, batch=8),
+                                  # more than 16 samples: the B-row products (modulation, time MLP) on the
+                                  # tensor-core GEMM instead of the row kernels
+                                  {"batch": 20, "n_txt": 8, "grid": (1, 2, 4)}])
 def test_backward_matches_oracle(cuda, over):
     cfg = _cfg(**over)
     run = Run(cfg, cuda)
@@ -130,7 +133,8 @@ WAN_TRAIN = dict(name="wan_train", arch="wan", hidden=256, heads=2, head_dim=128
 @pytest.mark.parametrize("over", [{}, {"n_double": 2},
                                   {"heads": 4, "head_dim": 64, "rope_axes": (20, 22, 22)},
                                   {"grid": (1, 3, 5), "n_txt": 5, "batch": 8},
-                                  {"batch": 3, "n_txt": 8, "grid": (2, 2, 6), "n_double": 2}])
+                                  {"batch": 3, "n_txt": 8, "grid": (2, 2, 6), "n_double": 2},
+                                  {"batch": 20, "n_txt": 8, "grid": (1, 2, 4)}])
 def test_wan_backward_matches_oracle(cuda, over):
     """The WAN-style block's backward (affine LN, ungated cross-attention with
     text keys / values, shared modulation) against wan_velocity_vjp."""
