@@ -578,7 +578,8 @@ def backward_kernels(args, ffi, cfg, dev):
     g0, g1 = rnd(B * n0, H), rnd(B * n1, H)
     dq0, dq1 = torch.empty_like(q0), torch.empty_like(q1)
     lse = torch.empty(B * heads * ffi.lib().ff_attention_lse_rows(n0, n1), device=dev)
-    ffi.ff_attention_forward(B, heads, d, q0, o0, n0, q1, o1, n1, lse=lse)
+    aws = torch.empty(ffi.ff_attention_forward_workspace_size(d), dtype=torch.uint8, device=dev)
+    ffi.ff_attention_forward(B, heads, d, q0, o0, n0, q1, o1, n1, lse=lse, ws=aws)
     T = B * (n0 + n1)
     x, W, dy = rnd(T, H), rnd(3 * H, H), rnd(T, 3 * H)
     y = torch.empty(T, 3 * H, device=dev, dtype=torch.bfloat16)
@@ -586,7 +587,8 @@ def backward_kernels(args, ffi, cfg, dev):
     dW = torch.empty(3 * H, H, device=dev, dtype=torch.float32)
     N = n0 + n1
     cases = {
-        "attention_forward_lse": (lambda: ffi.ff_attention_forward(B, heads, d, q0, o0, n0, q1, o1, n1, lse=lse),
+        "attention_forward_lse": (lambda: ffi.ff_attention_forward(B, heads, d, q0, o0, n0, q1, o1, n1, lse=lse,
+                                                                   ws=aws),
                                   4.0 * B * heads * N * N * d),
         "attention_backward": (lambda: ffi.ff_attention_backward(B, heads, d, (n0, q0, o0, g0, dq0),
                                                                  (n1, q1, o1, g1, dq1), lse),
@@ -1180,12 +1182,13 @@ def profile_kernel(args):
         q1 = rnd(B * n1, 3 * H).to(torch.bfloat16)
         o0 = torch.empty(max(B * n0, 1), H, dtype=torch.bfloat16, device=dev)
         o1 = torch.empty(B * n1, H, dtype=torch.bfloat16, device=dev)
+        aws = torch.empty(ffi.ff_attention_forward_workspace_size(d), dtype=torch.uint8, device=dev)
         if k == "attention":
             for _ in range(reps):
-                ffi.ff_attention_forward(B, heads, d, q0, o0, n0, q1, o1, n1)
+                ffi.ff_attention_forward(B, heads, d, q0, o0, n0, q1, o1, n1, ws=aws)
         else:   # the backward (D, dQ, dK / dV kernels) after one forward that keeps lse
             lse = torch.empty(B * heads * ffi.lib().ff_attention_lse_rows(n0, n1), device=dev)
-            ffi.ff_attention_forward(B, heads, d, q0, o0, n0, q1, o1, n1, lse=lse)
+            ffi.ff_attention_forward(B, heads, d, q0, o0, n0, q1, o1, n1, lse=lse, ws=aws)
             g0, g1 = rnd(max(B * n0, 1), H).to(torch.bfloat16), rnd(B * n1, H).to(torch.bfloat16)
             dq0, dq1 = torch.empty_like(q0), torch.empty_like(q1)
             for _ in range(reps):

@@ -408,6 +408,19 @@ int ff_dit_weight_layout(const ff_dit_config* cfg, ff_tensor_desc* out, int capa
 int ff_dit_create(const ff_dit_config* cfg, const void* weights_dev, ff_dit** out);
 int ff_dit_destroy(ff_dit* model);
 
+/* Whether the model's attention launches may split the query blocks of
+ * their last, at most half-full round over the SMs into two halves of the
+ * keys (see ff_attention_forward's ws): on = 1 (the default) or 0.  A split
+ * block's output agrees with the unsplit one to fp32 rounding, and which
+ * blocks split depends on the batch size, so with on = 1 a sample's
+ * velocity can differ in its last bits between calls on different batches.
+ * With on = 0 a sample's velocity (and every training-pass result) is bit
+ * for bit independent of the other samples in the batch.  Applies to the
+ * velocity, rollout and training entries; set it before a training
+ * pass's forward and keep it until its backward.  The workspace sizes do
+ * not depend on it.  Other values of on: FF_ERR_INVALID_ARG. */
+int ff_dit_set_attention_split(ff_dit* model, int on);
+
 /* Workspace bytes for a velocity call on a batch of B samples. */
 int ff_dit_workspace_size(const ff_dit* model, int B, size_t* bytes);
 
@@ -501,11 +514,21 @@ int ff_gemm(int M, int N, int K, const void* A, int64_t lda, int a_layout, const
  * not touched).  ws: ff_attention_backward_workspace_size bytes (holds
  * -D = -rowsum(dO * O) and a copy of -lse, each [B, heads, L]).  A segment
  * with n = 0 may pass NULL buffers.
+ * ff_attention_forward's ws is optional (NULL: none): with at least
+ * ff_attention_forward_workspace_size(head_dim) bytes, 16-byte aligned, a
+ * launch whose work items (256 query rows of one sample and head) leave the
+ * last round over the SMs at most half full runs those items as two halves
+ * of their keys on two SMs each and merges the halves' partial softmaxes
+ * (the online-softmax rescale, exact up to rounding).  The results agree
+ * with the unsplit launch to fp32 rounding, not bit for bit.  Calls that
+ * share ws must not overlap on the GPU; ws needs no initial contents.
  * ------------------------------------------------------------------------ */
 int ff_attention_lse_rows(int n0, int n1);
+int ff_attention_forward_workspace_size(int head_dim, size_t* bytes);
 int ff_attention_forward(int B, int heads, int head_dim, int n0, const void* qkv0, int64_t ld0,
                          void* out0, int64_t ldo0, int n1, const void* qkv1, int64_t ld1,
-                         void* out1, int64_t ldo1, float* lse, cudaStream_t stream);
+                         void* out1, int64_t ldo1, float* lse, void* ws, size_t ws_bytes,
+                         cudaStream_t stream);
 int ff_attention_backward_workspace_size(int B, int heads, int n0, int n1, size_t* bytes);
 int ff_attention_backward(int B, int heads, int head_dim, int n0, const void* qkv0, int64_t ld0,
                           const void* out0, const void* dout0, int64_t ldo0, void* dqkv0,

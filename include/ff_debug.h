@@ -41,9 +41,12 @@ int ff_debug_attention(int B, int heads, int head_dim, int n0, const void* qkv0,
 
 /* Which variant of the attention kernel every later forward launch takes,
  * process-wide (for tests): 0 the launcher's own choice by item count and
- * length, 1 the persistent one (one CTA per SM), 2 one 256-row query block
- * per CTA.  Returns the previous setting; FF_ERR_INVALID_ARG (and no change)
- * for other values.  The output does not depend on the variant. */
+ * length, 1 the persistent one (one CTA per SM) without the split of the
+ * last round's items, 2 one 256-row query block per CTA, 3 the persistent
+ * one with the split wherever the launch has a scratch and its last round
+ * is at most half full.  Returns the previous setting; FF_ERR_INVALID_ARG
+ * (and no change) for other values.  Variants 0, 1 and 2 give bit-identical
+ * output when no split is taken; a split launch agrees to fp32 rounding. */
 int ff_debug_attention_launch(int mode);
 
 /* out[r] = LN(x[r]) * (1 + mods[b, scale_off:]) + mods[b, shift_off:] for

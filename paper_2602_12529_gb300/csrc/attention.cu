@@ -66,10 +66,11 @@ namespace {
 
 constexpr int kBM = 128;         // query rows per query tile (two tiles per CTA)
 constexpr int kBN = 128;         // tokens per K/V tile
+constexpr int kSplitMaxItems = 96;   // split items per launch (half of 192 SMs)
 constexpr int kThreads = 320;    // producer, MMA, 2 x 4 softmax warps
 constexpr int kPersistentItemsPerSm = 16;   // persistent launch below this many items per SM,
 constexpr int kPersistentMaxSteps = 128;    // or with at most this many K/V steps per item
-std::atomic<int> g_launch_override{0};      // tests: 1 forces the persistent variant, 2 one item per CTA
+std::atomic<int> g_launch_override{0};   // tests: 1 persistent unsplit, 2 one item per CTA, 3 persistent split
 
 template <int HD>
 struct ACfg {
@@ -97,6 +98,14 @@ struct AttnParams {
     int qpairs;          // 256-row query blocks of both segments
     int heads;
     int items;           // B * heads * qpairs work items, item = (b * heads + h) * qpairs + block
+    // persistent launch only: items split_first .. split_first + split_n - 1
+    // run as two halves of their K/V steps, half h of item split_first + i on
+    // CTA 2 i + h; each half leaves O (unnormalised), m and l of its rows in
+    // part / part_ml, and the second to finish a row group combines them
+    int split_first, split_n;
+    float* part;         // [split_n][2 halves][2 tiles][128 rows][d]
+    float2* part_ml;     // [split_n][2][2][128]: (m, l)
+    unsigned* tickets;   // [split_n][2 tiles][4 lane quarters], zero at launch
     int q_col, k_col, v_col;
     float scale_log2;
     __nv_bfloat16* out[2];
@@ -151,15 +160,25 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
     const int nt0 = (p.nkv[0] + kBN - 1) / kBN;
     const int ntiles = nt0 + (p.nkv[1] + kBN - 1) / kBN;   // K/V steps per item
     // persistent: this CTA takes items blockIdx.x, blockIdx.x + gridDim.x, ...
-    // and runs their K/V steps as one stream, global step g = k ntiles + j
-    // for local step j of its k-th item
-    const int nitems = !kPersistent ? (static_cast<int>(blockIdx.x) < p.items ? 1 : 0)
-                       : p.items > static_cast<int>(blockIdx.x)
-                           ? (p.items - 1 - static_cast<int>(blockIdx.x)) / static_cast<int>(gridDim.x) + 1 : 0;
-    const int nsteps = nitems * ntiles;
+    // and runs their K/V steps as one stream; the global step g counts the
+    // CTA's steps over its items in order.  A split launch gives every CTA
+    // split_first / gridDim.x whole items and CTAs 0 .. 2 split_n - 1 one half
+    // item after them (CTA 2 i + h: half h of item split_first + i)
+    const int c_ = static_cast<int>(blockIdx.x), g_ = static_cast<int>(gridDim.x);
+    const bool split = kPersistent && p.split_n > 0;
+    const int nfull = !kPersistent ? (c_ < p.items ? 1 : 0)
+                      : split ? p.split_first / g_
+                      : p.items > c_ ? (p.items - 1 - c_) / g_ + 1 : 0;
+    const bool has_half = split && c_ < 2 * p.split_n;
+    const int nitems = nfull + (has_half ? 1 : 0);
+    const int half_at = ntiles >> 1;   // the first half covers steps 0 .. half_at - 1
+    // K/V steps [j0, j1) of the CTA's k-th item
+    auto seg_j0 = [&](int k) { return k < nfull || !(c_ & 1) ? 0 : half_at; };
+    auto seg_j1 = [&](int k) { return k < nfull || (c_ & 1) ? ntiles : half_at; };
+    const int nsteps = nfull * ntiles + (has_half ? ((c_ & 1) ? ntiles - half_at : half_at) : 0);
     struct Item { int b, h, seg, q0; };   // q0: first query row within the segment
     auto item_of = [&](int k) {
-        const int it = static_cast<int>(blockIdx.x) + k * static_cast<int>(gridDim.x);
+        const int it = k < nfull ? c_ + k * g_ : p.split_first + (c_ >> 1);
         const int qp = it % p.qpairs;
         const int bh = it / p.qpairs;
         Item r;
@@ -229,7 +248,7 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
         Item cur = item_of(0);
         load_q(0, cur);
         load_q(1, cur);
-        for (int n = 0, k = 0, j = 0; n < 2 * nsteps; ++n) {
+        for (int n = 0, k = 0, j = seg_j0(0); n < 2 * nsteps; ++n) {
             const int s = n % S;
             const int g = n >> 1;                 // global step of this K or V tile: item k, local step j
             // item n - S (group c = (n - S + 1) / 2) leaves slot s once the
@@ -237,7 +256,7 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
             // last MMA of step c - 1, and K_0's only readers are S_0,0 and
             // S_1,0)
             if (n >= S && !s1_done_upto((n - S + 1) >> 1)) { fail(); break; }
-            const bool new_item = !(n & 1) && j == 0 && k > 0;
+            const bool new_item = !(n & 1) && j == seg_j0(k) && k > 0;
             if (new_item) cur = item_of(k);
             uint64_t* fb = &bar.grp_full[((n + 1) >> 1) & 3];
             const int ks = j < nt0 ? 0 : 1;
@@ -261,9 +280,9 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
                 load_q(1, cur);
             }
             if (n & 1) {
-                if (++j == ntiles) {
-                    j = 0;
+                if (++j == seg_j1(k)) {
                     ++k;
+                    j = seg_j0(k);
                 }
             }
         }
@@ -329,8 +348,10 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
         // softmax warps publish only after their epilogue has read O_t.  The
         // item's last step is peeled off, so the per-step loop carries no
         // item bookkeeping.
-        for (int k = 0, g0 = 0; ok && k < nitems; ++k, g0 += ntiles) {
-            for (int j = 0; j + 1 < ntiles; ++j) {
+        // j counts the item's steps from its first (a half item has fewer)
+        for (int k = 0, g0 = 0; ok && k < nitems; ++k) {
+            const int nk = seg_j1(k) - seg_j0(k);
+            for (int j = 0; j + 1 < nk; ++j) {
                 for (int t = 0; t < 2; ++t) {
                     if (!issue_pv(t, g0 + j, j)) { fail(); ok = false; break; }
                     issue_s(t, g0 + j + 1);
@@ -338,7 +359,7 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
                 if (!ok) break;
             }
             if (!ok) break;
-            const int j = ntiles - 1;   // the item's last step
+            const int j = nk - 1;   // the item's last step
             const bool more = k + 1 < nitems;
             for (int t = 0; t < 2; ++t) {
                 if (!issue_pv(t, g0 + j, j)) { fail(); ok = false; break; }
@@ -346,9 +367,10 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
                 if (more) {   // query tile t of item k + 1
                     if (!mbar_wait(&bar.q_full[t], (k + 1) & 1)) { fail(); ok = false; break; }
                     tc_fence_after();
-                    issue_s(t, g0 + ntiles);
+                    issue_s(t, g0 + nk);
                 }
             }
+            g0 += nk;
         }
         tc_commit(&bar.drain);
         if (!mbar_wait(&bar.drain, 0)) report_status(status, kStatusWaitTimeout);
@@ -360,11 +382,12 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
         const uint32_t tS = tmem + (static_cast<uint32_t>(q * 32) << 16) + t * 256;
         const uint32_t tO = tS + C::kColO;
         bool ok = true;
-        for (int k = 0; ok && k < nitems; ++k) {
+        for (int k = 0, g0 = 0; ok && k < nitems; ++k) {
             float m_used = -INFINITY;
             float l = 0.f;
-            for (int j = 0; j < ntiles; ++j) {
-                const int g = k * ntiles + j;   // global step
+            const int j0 = seg_j0(k), j1 = seg_j1(k);
+            for (int j = j0; j < j1; ++j) {
+                const int g = g0 + (j - j0);   // global step
                 // S_t,g ready; O_t += P_t,g-1 V_g-1 has completed as well
                 if (!(t == 0 ? mbar_wait(&bar.s0_full, g & 1) : mbar_wait(&bar.s1_ring[g & 3], (g >> 2) & 1))) {
                     fail();
@@ -416,9 +439,9 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
                 // may exceed it: P up to 2^40 is exact enough in bf16 / fp32, and
                 // a tile whose row sum passes 2^40 (or overflows) is redone with
                 // the true maximum, rescaling l and O.
-                if (j == 0) m_used = row_max();
+                if (j == j0) m_used = row_max();
                 float lt = exps(m_used);
-                if (j > 0 && __any_sync(0xffffffffu, !(lt <= 0x1p40f))) {
+                if (j > j0 && __any_sync(0xffffffffu, !(lt <= 0x1p40f))) {
                     tmem_ld_x128(tS, sr);
                     tmem_ld_wait();
                     if (valid < kBN) {
@@ -457,23 +480,48 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
                 if (lane == 0) mbar_arrive(&bar.p_full[t]);
             }
             if (!ok) break;
+            g0 += j1 - j0;
             // ---- epilogue: O / l -> bf16, after the item's last O += P V, and
             // the row's log-sum-exp m + log2(l) (base 2) when it is asked for.
             // The next item's first O += P V waits for this warpgroup's P, so it
             // cannot overwrite O_t before these loads.
-            if (mbar_wait(&bar.o_last[t], k & 1)) {
-                tc_fence_after();
-                const Item it = item_of(k);
+            if (!mbar_wait(&bar.o_last[t], k & 1)) {
+                fail();
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            const Item it = item_of(k);
+            const int row = it.q0 + t * kBM + r;
+            const bool live = row < p.nq[it.seg];
+            const int64_t grow = static_cast<int64_t>(it.b) * p.nq[it.seg] + row;
+            __nv_bfloat16* dst = p.out[it.seg] + grow * p.ldo[it.seg] + it.h * HD;
+            __nv_bfloat16* dst_lo =
+                p.out_lo[it.seg] ? p.out_lo[it.seg] + grow * p.ldo_lo[it.seg] + it.h * HD : nullptr;
+            float* lse_at = p.lse && live
+                                ? p.lse + (static_cast<int64_t>(it.b) * p.heads + it.h) * p.lse_rows +
+                                      p.lse_base[it.seg] + row
+                                : nullptr;
+            // eight outputs from column c0 as bf16, and what bf16 dropped (itself
+            // in bf16) when the low part is asked for
+            auto put8 = [&](int c0, const float* f) {
+                const uint4 hi = make_uint4(pack_bf16x2(f[0], f[1]), pack_bf16x2(f[2], f[3]),
+                                            pack_bf16x2(f[4], f[5]), pack_bf16x2(f[6], f[7]));
+                *reinterpret_cast<uint4*>(dst + c0) = hi;
+                if (dst_lo) {
+                    const uint32_t hw[4] = {hi.x, hi.y, hi.z, hi.w};
+                    uint32_t lw[4];
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const float2 rr = unpack_bf16x2(hw[i]);
+                        lw[i] = pack_bf16x2(f[2 * i] - rr.x, f[2 * i + 1] - rr.y);
+                    }
+                    *reinterpret_cast<uint4*>(dst_lo + c0) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+                }
+            };
+            if (k < nfull) {
                 const float inv = 1.f / l;
-                const int row = it.q0 + t * kBM + r;
-                const bool live = row < p.nq[it.seg];
-                if (p.lse && live)
-                    p.lse[(static_cast<int64_t>(it.b) * p.heads + it.h) * p.lse_rows + p.lse_base[it.seg] + row] =
-                        m_used + log2f(l);
-                const int64_t grow = static_cast<int64_t>(it.b) * p.nq[it.seg] + row;
-                __nv_bfloat16* dst = p.out[it.seg] + grow * p.ldo[it.seg] + it.h * HD;
-                __nv_bfloat16* dst_lo =
-                    p.out_lo[it.seg] ? p.out_lo[it.seg] + grow * p.ldo_lo[it.seg] + it.h * HD : nullptr;
+                if (lse_at) *lse_at = m_used + log2f(l);
 #pragma unroll 1
                 for (int c = 0; c < HD; c += 32) {
                     uint32_t o[32];
@@ -485,29 +533,74 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
                             float f[8];
 #pragma unroll
                             for (int i = 0; i < 8; ++i) f[i] = __uint_as_float(o[8 * w + i]) * inv;
-                            const uint4 hi = make_uint4(pack_bf16x2(f[0], f[1]), pack_bf16x2(f[2], f[3]),
-                                                        pack_bf16x2(f[4], f[5]), pack_bf16x2(f[6], f[7]));
-                            *reinterpret_cast<uint4*>(dst + c + 8 * w) = hi;
-                            if (dst_lo) {
-                                // what bf16 dropped, itself in bf16
-                                const uint32_t hw[4] = {hi.x, hi.y, hi.z, hi.w};
-                                uint32_t lw[4];
+                            put8(c + 8 * w, f);
+                        }
+                    }
+                }
+            } else {
+                // half of a split item: publish this half's unnormalised O_t
+                // rows with their (m, l); the warp that finds the other half
+                // already published merges the two (the partial softmaxes of
+                // two key ranges: weights 2^(m_h - max(m_0, m_1)), always in
+                // half order, so the result does not depend on which came last)
+                const int si = c_ >> 1, hh = c_ & 1;
+                const size_t prow = (static_cast<size_t>(si * 2 + hh) * 2 + t) * kBM + r;
+                float* mine = p.part + prow * HD;
+#pragma unroll 1
+                for (int c = 0; c < HD; c += 32) {
+                    uint32_t o[32];
+                    tmem_ld_x32(tO + c, o);
+                    tmem_ld_wait();
 #pragma unroll
-                                for (int i = 0; i < 4; ++i) {
-                                    const float2 r = unpack_bf16x2(hw[i]);
-                                    lw[i] = pack_bf16x2(f[2 * i] - r.x, f[2 * i + 1] - r.y);
+                    for (int w = 0; w < 8; ++w)
+                        *reinterpret_cast<float4*>(mine + c + 4 * w) =
+                            make_float4(__uint_as_float(o[4 * w]), __uint_as_float(o[4 * w + 1]),
+                                        __uint_as_float(o[4 * w + 2]), __uint_as_float(o[4 * w + 3]));
+                }
+                p.part_ml[prow] = make_float2(m_used, l);
+                __threadfence();
+                __syncwarp();
+                unsigned prev = 0;
+                if (lane == 0) prev = atomicAdd(&p.tickets[(si * 2 + t) * 4 + q], 1u);
+                prev = __shfl_sync(0xffffffffu, prev, 0);
+                if (prev == 1u) {
+                    __threadfence();
+                    const size_t orow = (static_cast<size_t>(si * 2 + (hh ^ 1)) * 2 + t) * kBM + r;
+                    const float* other = p.part + orow * HD;
+                    const float2 mo = __ldcg(p.part_ml + orow);
+                    const float m0 = hh ? mo.x : m_used, l0 = hh ? mo.y : l;
+                    const float m1 = hh ? m_used : mo.x, l1 = hh ? l : mo.y;
+                    const float mm = fmaxf(m0, m1);
+                    const float w0 = ex2(m0 - mm), w1 = ex2(m1 - mm);
+                    const float lsum = __fmaf_rn(l1, w1, __fmul_rn(l0, w0));
+                    const float inv = 1.f / lsum;
+                    if (lse_at) *lse_at = mm + log2f(lsum);
+#pragma unroll 1
+                    for (int c = 0; c < HD; c += 32) {
+                        uint32_t o[32];
+                        tmem_ld_x32(tO + c, o);
+                        tmem_ld_wait();
+                        if (live) {
+#pragma unroll
+                            for (int w = 0; w < 4; ++w) {
+                                const float4 a = __ldcg(reinterpret_cast<const float4*>(other + c + 8 * w));
+                                const float4 b = __ldcg(reinterpret_cast<const float4*>(other + c + 8 * w + 4));
+                                const float ot[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+                                float f[8];
+#pragma unroll
+                                for (int i = 0; i < 8; ++i) {
+                                    const float own = __uint_as_float(o[8 * w + i]);
+                                    const float o0 = hh ? ot[i] : own, o1 = hh ? own : ot[i];
+                                    f[i] = __fmul_rn(__fmaf_rn(o1, w1, __fmul_rn(o0, w0)), inv);
                                 }
-                                *reinterpret_cast<uint4*>(dst_lo + c + 8 * w) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+                                put8(c + 8 * w, f);
                             }
                         }
                     }
                 }
-                tmem_ld_wait();
-                tc_fence_before();
-            } else {
-                fail();
-                ok = false;
             }
+            tmem_ld_wait();
+            tc_fence_before();
         }
     }
 
@@ -523,6 +616,11 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
         tmem_dealloc(tmem, C::kTmemCols);
     }
 }
+
+// Scratch of a split launch: per split item, both halves' unnormalised O of
+// both query tiles (fp32), their (m, l), and 8 tickets.
+size_t split_part_bytes(int hd) { return static_cast<size_t>(kSplitMaxItems) * 2 * 2 * kBM * hd * sizeof(float); }
+size_t split_ml_bytes() { return static_cast<size_t>(kSplitMaxItems) * 2 * 2 * kBM * sizeof(float2); }
 
 template <int HD>
 int launch_attn(const AttnSpec& a, cudaStream_t stream) {
@@ -573,12 +671,38 @@ int launch_attn(const AttnSpec& a, cudaStream_t stream) {
     // frees first, balances the SMs better than a fixed stride and the
     // overlap is worth little (WAN self-attention, 34 items of 256 steps per
     // SM: 13.8 ms one item per CTA, 14.0 ms persistent).
+    //
+    // A persistent launch whose items do not fill a whole last round (L of
+    // the G SMs busy, 2 L <= G) runs those L items as 2 L halves of their K/V
+    // steps on 2 L CTAs, given the caller's scratch: Flux block, 1728 items =
+    // 11 rounds + 56, so the last round ends after half an item.
     const int steps = (a.kv[0].n + kBN - 1) / kBN + (a.kv[1].n + kBN - 1) / kBN;
     const int forced = g_launch_override.load(std::memory_order_relaxed);
-    const bool persistent = forced ? forced == 1
-                                   : items < static_cast<int64_t>(kPersistentItemsPerSm) * num_sms() ||
+    const int sms = num_sms();
+    const bool persistent = forced ? forced == 1 || forced == 3
+                                   : items < static_cast<int64_t>(kPersistentItemsPerSm) * sms ||
                                          steps <= kPersistentMaxSteps;
-    const int grid = static_cast<int>(persistent ? (items < num_sms() ? items : num_sms()) : items);
+    int64_t grid64 = persistent ? (items < sms ? items : sms) : items;
+    p.split_first = p.split_n = 0;
+    p.part = nullptr;
+    p.part_ml = nullptr;
+    p.tickets = nullptr;
+    if (persistent && (forced == 0 || forced == 3) && a.split_ws && steps >= 2 &&
+        a.split_ws_bytes >= attention_split_ws_bytes(HD)) {
+        const int64_t rounds = items / sms, rest = items % sms;
+        if (rest > 0 && 2 * rest <= sms && rest <= kSplitMaxItems) {
+            uint8_t* ws = static_cast<uint8_t*>(a.split_ws);
+            p.split_first = static_cast<int>(rounds * sms);
+            p.split_n = static_cast<int>(rest);
+            p.part = reinterpret_cast<float*>(ws);
+            p.part_ml = reinterpret_cast<float2*>(ws + split_part_bytes(HD));
+            p.tickets = reinterpret_cast<unsigned*>(ws + split_part_bytes(HD) + split_ml_bytes());
+            grid64 = rounds > 0 ? sms : 2 * rest;
+            if (cudaMemsetAsync(p.tickets, 0, static_cast<size_t>(rest) * 8 * sizeof(unsigned), stream) != cudaSuccess)
+                return set_error(FF_ERR_CUDA, "attention: cannot clear the split tickets");
+        }
+    }
+    const int grid = static_cast<int>(grid64);
     const double nkv = static_cast<double>(a.kv[0].n + a.kv[1].n);
     const double nq = static_cast<double>(a.q[0].n + a.q[1].n);
     ProfScope prof(stream, "attention", 4.0 * a.B * a.heads * nq * nkv * HD,
@@ -595,6 +719,10 @@ int launch_attn(const AttnSpec& a, cudaStream_t stream) {
 }  // namespace
 
 int attention_launch_override(int mode) { return g_launch_override.exchange(mode); }
+
+size_t attention_split_ws_bytes(int head_dim) {
+    return split_part_bytes(head_dim) + split_ml_bytes() + static_cast<size_t>(kSplitMaxItems) * 8 * sizeof(unsigned);
+}
 
 int attention_general(const AttnSpec& a, cudaStream_t stream) {
     if (a.B <= 0 || a.heads <= 0 || a.B > 65535 || a.heads > 65535)
@@ -618,15 +746,18 @@ int attention_general(const AttnSpec& a, cudaStream_t stream) {
         if (a.kv[i].n && (a.k_col + hd > a.kv[i].ld || a.v_col + hd > a.kv[i].ld))
             return set_error(FF_ERR_INVALID_ARG, "attention: k/v columns exceed ld");
     }
+    if (a.split_ws && !aligned16(a.split_ws)) return set_error(FF_ERR_INVALID_ARG, "attention: misaligned split scratch");
     if (a.head_dim == 128) return launch_attn<128>(a, stream);
     if (a.head_dim == 64) return launch_attn<64>(a, stream);
     return set_error(FF_ERR_UNSUPPORTED, "attention: head_dim %d", a.head_dim);
 }
 
 int attention(const AttnSegment& s0, const AttnSegment& s1, int B, int heads, int head_dim, int H,
-              cudaStream_t stream, float* lse) {
+              cudaStream_t stream, float* lse, void* split_ws, size_t split_ws_bytes) {
     AttnSpec a;
     a.lse = lse;
+    a.split_ws = split_ws;
+    a.split_ws_bytes = split_ws_bytes;
     const AttnSegment* seg[2] = {&s0, &s1};
     for (int i = 0; i < 2; ++i) {
         a.q[i] = AttnQuerySeg{seg[i]->qkv, seg[i]->ld, seg[i]->n, seg[i]->out, seg[i]->ldo, seg[i]->out_lo,

@@ -43,9 +43,10 @@ int ff_attention_lse_rows(int n0, int n1) { return ff::attn_lse_rows(n0 < 0 ? 0 
 
 int ff_attention_forward(int B, int heads, int head_dim, int n0, const void* qkv0, int64_t ld0, void* out0,
                          int64_t ldo0, int n1, const void* qkv1, int64_t ld1, void* out1, int64_t ldo1, float* lse,
-                         cudaStream_t stream) {
+                         void* ws, size_t ws_bytes, cudaStream_t stream) {
     using namespace ff;
     if (lse && !aligned16(lse)) return set_error(FF_ERR_INVALID_ARG, "attention: lse must be 16-byte aligned");
+    if (ws && !aligned16(ws)) return set_error(FF_ERR_INVALID_ARG, "attention: ws must be 16-byte aligned");
     AttnSpec a;
     const int H = heads * head_dim;
     const void* qkv[2] = {qkv0, qkv1};
@@ -64,7 +65,17 @@ int ff_attention_forward(int B, int heads, int head_dim, int n0, const void* qkv
     a.heads = heads;
     a.head_dim = head_dim;
     a.lse = lse;
+    a.split_ws = ws;
+    a.split_ws_bytes = ws ? ws_bytes : 0;
     return attention_general(a, stream);
+}
+
+int ff_attention_forward_workspace_size(int head_dim, size_t* bytes) {
+    using namespace ff;
+    if (!bytes) return set_error(FF_ERR_INVALID_ARG, "bytes is null");
+    if (head_dim != 64 && head_dim != 128) return set_error(FF_ERR_UNSUPPORTED, "attention: head_dim %d", head_dim);
+    *bytes = attention_split_ws_bytes(head_dim);
+    return FF_OK;
 }
 
 int ff_attention_backward_workspace_size(int B, int heads, int n0, int n1, size_t* bytes) {
@@ -158,7 +169,7 @@ int ff_debug_attention(int B, int heads, int head_dim, int n0, const void* qkv0,
 
 int ff_debug_attention_launch(int mode) {
     using namespace ff;
-    if (mode < 0 || mode > 2) return set_error(FF_ERR_INVALID_ARG, "attention launch mode %d (0, 1 or 2)", mode);
+    if (mode < 0 || mode > 3) return set_error(FF_ERR_INVALID_ARG, "attention launch mode %d (0 to 3)", mode);
     return attention_launch_override(mode);
 }
 

@@ -33,6 +33,7 @@ struct ff_dit {
     // the attention outputs, re-running the rest of each block before its
     // backward; 2 keeps the block inputs only
     int train_recompute = 0;
+    int attn_split = 1;   // attention launches may split their last round (ff_dit_set_attention_split)
     mutable int fwd_recompute = -1;   // the mode of the latest ff_dit_forward_train (-1: none yet)
 };
 
@@ -149,6 +150,7 @@ struct Workspace {
     float *e, *e0;
     __nv_bfloat16 *txt1, *txth, *kvc;
     float2* rope;   // cos / sin table of every rotation angle
+    void* attn_ws;  // the attention launches' split scratch
     size_t bytes;
 };
 
@@ -175,6 +177,7 @@ Workspace plan(const ff_dit_config& c, int B, uint8_t* base) {
     w.u = reinterpret_cast<__nv_bfloat16*>(take(R * (H + F) * 2));
     w.rope = reinterpret_cast<float2*>(take(static_cast<size_t>(rope_table_size(
         c.grid_f, c.grid_h, c.grid_w, c.rope_axes[0], c.rope_axes[1], c.rope_axes[2])) * sizeof(float2)));
+    w.attn_ws = take(attention_split_ws_bytes(c.head_dim));
     if (wan) {
         w.e = reinterpret_cast<float*>(take(B * H * 4));
         w.e0 = reinterpret_cast<float*>(take(B * 6 * H * 4));
@@ -319,6 +322,7 @@ int wan_forward_block(const ff_dit* m, int B, int l, const DitBlockIo& io, const
             a.q_col = 0; a.k_col = H; a.v_col = 2 * H;
             a.B = B; a.heads = c.heads; a.head_dim = d;
             a.lse = io.lse;
+            a.split_ws = f.attn_ws; a.split_ws_bytes = f.attn_ws_bytes;
             FF_TRY(attention_general(a, stream));
         }
         {
@@ -358,6 +362,7 @@ int wan_forward_block(const ff_dit* m, int B, int l, const DitBlockIo& io, const
             a.q_col = 0; a.k_col = 0; a.v_col = H;
             a.B = B; a.heads = c.heads; a.head_dim = d;
             a.lse = io.lse_c;
+            a.split_ws = f.attn_ws; a.split_ws_bytes = f.attn_ws_bytes;
             FF_TRY(attention_general(a, stream));
         }
         {
@@ -523,7 +528,7 @@ int mmdit_forward_double(const ff_dit* m, int B, int l, const DitBlockIo& io, co
             AttnSegment a0{io.qkv, 3 * H, io.o, H, Nt, io.o_lo, H};
             AttnSegment a1{io.qkv + static_cast<int64_t>(Rt) * 3 * H, 3 * H, io.o + static_cast<int64_t>(Rt) * H, H, Ni,
                            io.o_lo ? io.o_lo + static_cast<int64_t>(Rt) * H : nullptr, H};
-            FF_TRY(attention(a0, a1, B, c.heads, c.head_dim, H, stream, io.lse));
+            FF_TRY(attention(a0, a1, B, c.heads, c.head_dim, H, stream, io.lse, f.attn_ws, f.attn_ws_bytes));
         }
         // projection + gated residual (gate1)
         {
@@ -612,7 +617,7 @@ int mmdit_forward_single(const ff_dit* m, int B, int l, const DitBlockIo& io, co
             AttnSegment a0{io.qkv, 3 * H, io.u, H + F, Nt, io.o_lo, H};
             AttnSegment a1{io.qkv + static_cast<int64_t>(Rt) * 3 * H, 3 * H, io.u + static_cast<int64_t>(Rt) * (H + F),
                            H + F, Ni, io.o_lo ? io.o_lo + static_cast<int64_t>(Rt) * H : nullptr, H};
-            FF_TRY(attention(a0, a1, B, c.heads, c.head_dim, H, stream, io.lse));
+            FF_TRY(attention(a0, a1, B, c.heads, c.head_dim, H, stream, io.lse, f.attn_ws, f.attn_ws_bytes));
         }
         // linear2 + gated residual: one launch, the two segments as two
         // problems (the sample index of a row differs per segment)
@@ -675,6 +680,7 @@ int64_t model_offset(const ff_dit* m, const char* name) {
 }
 int64_t model_mod_width(const ff_dit* m) { return m->mod_width; }
 int model_train_recompute(const ff_dit* m) { return m->train_recompute; }
+int model_attention_split(const ff_dit* m) { return m->attn_split; }
 void model_note_forward_train(const ff_dit* m) { m->fwd_recompute = m->train_recompute; }
 int model_forward_train_mode(const ff_dit* m) { return m->fwd_recompute; }
 
@@ -739,6 +745,14 @@ int ff_dit_set_train_recompute(ff_dit* m, int on) {
     return FF_OK;
 }
 
+int ff_dit_set_attention_split(ff_dit* m, int on) {
+    using namespace ff;
+    if (!m) return set_error(FF_ERR_INVALID_ARG, "model is null");
+    if (on != 0 && on != 1) return set_error(FF_ERR_INVALID_ARG, "attention split %d (0 or 1)", on);
+    m->attn_split = on;
+    return FF_OK;
+}
+
 int ff_dit_workspace_size(const ff_dit* m, int B, size_t* bytes) {
     using namespace ff;
     if (!m || !bytes) return set_error(FF_ERR_INVALID_ARG, "model/bytes is null");
@@ -763,6 +777,8 @@ int ff_dit_velocity(const ff_dit* m, int B, const float* x_t, const void* txt, c
     f.mods = w.mods; f.temb = w.temb; f.th = w.th; f.tc = w.tc; f.xb = w.xb; f.rope = w.rope;
     f.x0 = f.xfin = w.x;
     f.hf = w.h;
+    f.attn_ws = m->attn_split ? w.attn_ws : nullptr;
+    f.attn_ws_bytes = attention_split_ws_bytes(c.head_dim);
     f.shared = DitBlockIo{w.x, w.x, w.x, w.h, w.qkv, nullptr, w.o, nullptr, w.h, nullptr, w.u, nullptr, nullptr};
     if (c.arch == FF_ARCH_WAN) {
         // one buffer per role, reused by every block: the residual in place,

@@ -35,6 +35,7 @@ const __nv_bfloat16* model_weights(const ff_dit* m);
 int64_t model_offset(const ff_dit* m, const char* name);
 int64_t model_mod_width(const ff_dit* m);
 int model_train_recompute(const ff_dit* m);
+int model_attention_split(const ff_dit* m);   // 0: the attention launches get no split scratch
 // The training forward records its recompute mode on the handle; the
 // backward refuses to run in another mode (the workspace layouts differ).
 void model_note_forward_train(const ff_dit* m);
@@ -197,7 +198,7 @@ struct AttnSegment {
     __nv_bfloat16* out_lo = nullptr; int64_t ldo_lo = 0;
 };
 int attention(const AttnSegment& s0, const AttnSegment& s1, int B, int heads, int head_dim, int H,
-              cudaStream_t stream, float* lse = nullptr);
+              cudaStream_t stream, float* lse = nullptr, void* split_ws = nullptr, size_t split_ws_bytes = 0);
 
 // General form: queries from up to two query segments, keys/values from up
 // to two key/value segments (concatenated per sample), head h of q / k / v
@@ -218,11 +219,20 @@ struct AttnSpec {
     // (lse2 = log2 sum_j 2^(s_j log2(e) / sqrt(d))), kept for the backward:
     // lse[(b * heads + h) * attn_lse_rows(q0, q1) + (seg ? pad128(q0) : 0) + row]
     float* lse = nullptr;
+    // optional scratch of attention_split_ws_bytes(head_dim) bytes (16-byte
+    // aligned, not shared by launches that overlap on the GPU): lets a
+    // persistent launch whose last round is at most half full split those
+    // items' K/V steps over two CTAs each.  Without it the launch is unsplit.
+    void* split_ws = nullptr;
+    size_t split_ws_bytes = 0;
 };
+size_t attention_split_ws_bytes(int head_dim);
 inline int attn_pad128(int n) { return (n + 127) / 128 * 128; }
 inline int attn_lse_rows(int n0, int n1) { return attn_pad128(n0) + attn_pad128(n1); }
 int attention_general(const AttnSpec& a, cudaStream_t stream);
-// forward launch variant for tests: 0 automatic, 1 persistent, 2 one item per CTA; returns the previous
+// forward launch variant for tests: 0 automatic, 1 persistent without the
+// split, 2 one item per CTA, 3 persistent with the split where it applies;
+// returns the previous
 int attention_launch_override(int mode);
 
 // Backward of joint attention (d = 64 or 128): from dO (bf16, the layout of the
@@ -407,6 +417,10 @@ struct FwdBufs {
     // output and the embedded text (bf16 [B N_t, H])
     float *e, *e0;
     __nv_bfloat16 *txt_pre, *txt1, *txth;
+    // the attention launches' split scratch (AttnSpec::split_ws), shared by
+    // every block: the launches run one after another on the stream
+    void* attn_ws = nullptr;
+    size_t attn_ws_bytes = 0;
 };
 int mmdit_forward(const ff_dit* m, int B, const float* x_t, const void* txt, const float* t, float* v_out,
                   const FwdBufs& f, cudaStream_t stream);

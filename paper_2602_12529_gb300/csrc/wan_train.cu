@@ -83,6 +83,8 @@ WanPlan plan(const ff_dit_config& c, int64_t Wm, int B, uint8_t* base, int recom
     f.txth = b16(Rt * H);
     f.rope = reinterpret_cast<float2*>(take(static_cast<size_t>(rope_table_size(
         c.grid_f, c.grid_h, c.grid_w, c.rope_axes[0], c.rope_axes[1], c.rope_axes[2])) * sizeof(float2)));
+    f.attn_ws_bytes = attention_split_ws_bytes(c.head_dim);
+    f.attn_ws = take(f.attn_ws_bytes);
     const int L = c.n_double;
     const size_t lse_n = static_cast<size_t>(B) * c.heads * attn_lse_rows(0, static_cast<int>(Ni));
     p.blk.resize(L);
@@ -182,6 +184,7 @@ int wan_forward_train(const ff_dit* m, int B, const float* x_t, const void* txt,
                       void* ws, size_t ws_bytes, cudaStream_t stream) {
     const ff_dit_config& c = model_config(m);
     WanPlan p = plan(c, model_mod_width(m), B, static_cast<uint8_t*>(ws), model_train_recompute(m));
+    if (!model_attention_split(m)) p.f.attn_ws = nullptr;
     if (ws_bytes < p.bytes) return set_error(FF_ERR_WORKSPACE, "workspace %zu B < %zu B needed", ws_bytes, p.bytes);
     p.f.blocks = p.blk.data();
     // the time-MLP operands' padding rows (the weight-gradient products read them)
@@ -201,6 +204,7 @@ int wan_backward(const ff_dit* m, int B, const void* txt, const float* dv, float
     const int64_t Wm = model_mod_width(m);
     const int recompute = model_train_recompute(m);
     WanPlan p = plan(c, Wm, B, static_cast<uint8_t*>(ws), recompute);
+    if (!model_attention_split(m)) p.f.attn_ws = nullptr;
     if (ws_bytes < p.bytes) return set_error(FF_ERR_WORKSPACE, "workspace %zu B < %zu B needed", ws_bytes, p.bytes);
     const FwdBufs& f = p.f;
     const int H = c.hidden, F = c.mlp, P = c.patch_dim, d = c.head_dim, heads = c.heads, tf = c.time_freq_dim;

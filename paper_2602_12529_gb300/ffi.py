@@ -84,13 +84,15 @@ _SIGS = {
     "ff_dit_velocity": ([_P, _I, _P, _P, _P, _P, _P, _SZ, _P], _I),
     "ff_rollout_workspace_size": ([_P, _I, _I, C.POINTER(_SZ)], _I),
     "ff_dit_set_train_recompute": ([_P, _I], _I),
+    "ff_dit_set_attention_split": ([_P, _I], _I),
     "ff_dit_train_workspace_size": ([_P, _I, C.POINTER(_SZ)], _I),
     "ff_dit_forward_train": ([_P, _I, _P, _P, _P, _P, _P, _SZ, _P], _I),
     "ff_dit_backward": ([_P, _I, _P, _P, _P, _P, _P, _SZ, _P], _I),
     "ff_sde_logprob_backward": ([_I, _I64, _P, _P, _P, _P, _P, _P, _I, _P, _I, _P, _P], _I),
     "ff_gemm": ([_I, _I, _I, _P, _I64, _I, _P, _I64, _I, _P, _I, _I, _P, _I64, _P], _I),
     "ff_attention_lse_rows": ([_I, _I], _I),
-    "ff_attention_forward": ([_I, _I, _I, _I, _P, _I64, _P, _I64, _I, _P, _I64, _P, _I64, _P, _P], _I),
+    "ff_attention_forward_workspace_size": ([_I, C.POINTER(_SZ)], _I),
+    "ff_attention_forward": ([_I, _I, _I, _I, _P, _I64, _P, _I64, _I, _P, _I64, _P, _I64, _P, _P, _SZ, _P], _I),
     "ff_attention_backward_workspace_size": ([_I, _I, _I, _I, C.POINTER(_SZ)], _I),
     "ff_attention_backward": ([_I, _I, _I, _I, _P, _I64, _P, _P, _I64, _P, _I64, _I, _P, _I64, _P, _P, _I64, _P,
                                _I64, _P, _P, _SZ, _P], _I),
@@ -507,6 +509,11 @@ class Dit:
         mode = (1 if on else 0) if isinstance(on, bool) else int(on)
         _call("ff_dit_set_train_recompute", self._h, mode)
 
+    def set_attention_split(self, on: bool):
+        """Attention launches may split their last round's query blocks (True, the default); False makes
+        every sample's results independent of the rest of the batch, bit for bit."""
+        _call("ff_dit_set_attention_split", self._h, 1 if on else 0)
+
     def rollout_workspace_size(self, B: int, S: int) -> int:
         n = _SZ()
         _call("ff_rollout_workspace_size", self._h, B, S, C.byref(n))
@@ -594,10 +601,25 @@ def ff_gemm(A, a_layout: int, B, b_layout: int, out, bias=None, act=FF_ACT_NONE,
           act, 1 if out.dtype == torch.float32 else 0, _ptr_rows(out), out.stride(0), _stream(stream))
 
 
-def ff_attention_forward(B, heads, head_dim, qkv0, out0, n0, qkv1, out1, n1, lse=None, stream=None):
-    """Joint attention over [segment 0; segment 1]; lse: [B, heads, ff_attention_lse_rows(n0, n1)] fp32 or None."""
+def ff_attention_forward_workspace_size(head_dim: int) -> int:
+    n = _SZ()
+    _call("ff_attention_forward_workspace_size", head_dim, C.byref(n))
+    return n.value
+
+
+def ff_attention_forward(B, heads, head_dim, qkv0, out0, n0, qkv1, out1, n1, lse=None, ws=None, stream=None):
+    """Joint attention over [segment 0; segment 1]; lse: [B, heads, ff_attention_lse_rows(n0, n1)] fp32 or None.
+    ws: the optional scratch that lets the launch split its last round's items (None: a fresh one of
+    ff_attention_forward_workspace_size bytes; False: none, the unsplit launch)."""
+    import torch
+    if ws is None:
+        dev = (qkv0 if n0 else qkv1).device
+        ws = torch.empty(ff_attention_forward_workspace_size(head_dim), dtype=torch.uint8, device=dev)
+    elif ws is False:
+        ws = None
     _call("ff_attention_forward", B, heads, head_dim, n0, _ptr(qkv0), qkv0.shape[-1], _ptr(out0), out0.shape[-1],
-          n1, _ptr(qkv1), qkv1.shape[-1], _ptr(out1), out1.shape[-1], _ptr(lse), _stream(stream))
+          n1, _ptr(qkv1), qkv1.shape[-1], _ptr(out1), out1.shape[-1], _ptr(lse), _ptr(ws),
+          0 if ws is None else ws.numel(), _stream(stream))
 
 
 def ff_attention_backward(B, heads, head_dim, seg0, seg1, lse, ws=None, stream=None):

@@ -92,13 +92,19 @@ def test_workspace_queries(L):
     sz = ffi._SZ()
     assert L.ff_attention_backward_workspace_size(2, 3, 100, 200, C.byref(sz)) == 0
     assert sz.value == 2 * 2 * 3 * (128 + 256) * 4
+    # attention forward's optional split scratch: per split query block (at
+    # most 96) both halves' fp32 O of both 128-row tiles, their (m, l), 8 tickets
+    for d in (64, 128):
+        assert ffi.ff_attention_forward_workspace_size(d) == 96 * (2 * 2 * 128 * d * 4 + 2 * 2 * 128 * 8 + 8 * 4)
+    with pytest.raises(ffi.FFError):
+        ffi.ff_attention_forward_workspace_size(96)
 
 
 def test_host_validation_without_gpu(L):
     # every one of these is rejected before any CUDA call is made
-    assert L.ff_debug_attention_launch(3) == 1          # variants are 0, 1, 2
-    assert L.ff_debug_attention_launch(2) == 0          # returns the previous setting
-    assert L.ff_debug_attention_launch(0) == 2
+    assert L.ff_debug_attention_launch(4) == 1          # variants are 0 to 3
+    assert L.ff_debug_attention_launch(3) == 0          # returns the previous setting
+    assert L.ff_debug_attention_launch(0) == 3
     rc = L.ff_sde_step_logprob(0, 16, None, None, None, None, None, None, None, 0, 0, None, 1, None, 0, None)
     assert rc == 1
     rc = L.ff_sde_step_logprob(2, 18, 16, 16, 16, 16, 16, 16, 16, 0, 0, 16, 1, 16, 1 << 20, None)

@@ -108,9 +108,18 @@ def test_full_depth_properties(cuda, name, sub, batch):
     assert torch.isfinite(v1).all()
     assert torch.equal(v1, v2)
     assert float(v1.float().std()) > 1e-3
-    # the last `sub` samples alone give bit-identical velocities
-    vs = _run(cfg, model, x[B - sub:].contiguous(), txt[B - sub:].contiguous(), t[B - sub:].contiguous(), cuda)
-    assert torch.equal(vs, v1[B - sub:])
+    tail = (x[B - sub:].contiguous(), txt[B - sub:].contiguous(), t[B - sub:].contiguous())
+    # the last `sub` samples alone: with the attention split allowed (the
+    # default) the split blocks depend on the batch, so the velocities agree
+    # to rounding; without it they are bit-identical
+    vs = _run(cfg, model, *tail, cuda)
+    assert float((vs - v1[B - sub:]).norm() / v1[B - sub:].norm()) <= 1e-2
+    model.set_attention_split(False)
+    vb = _run(cfg, model, x, txt, t, cuda)
+    vs = _run(cfg, model, *tail, cuda)
+    model.set_attention_split(True)
+    assert torch.equal(vs, vb[B - sub:])
+    assert float((vb - v1).norm() / v1.norm()) <= 1e-2
     assert ffi.ff_check_device_status() == 0
     del model, blob
     torch.cuda.empty_cache()

@@ -164,6 +164,122 @@ def test_attention_variants_bit_identical(cuda, d):
         assert torch.equal(a, b)
 
 
+def _split_applies(items, sms):
+    rest = items % sms
+    return 0 < rest and 2 * rest <= sms
+
+
+@pytest.mark.parametrize("B,heads,d,n0,n1", [
+    (1, 52, 128, 0, 1024),    # 208 blocks: one full round, 56 blocks split in two halves of 4 steps
+    (1, 20, 64, 77, 300),     # 60 blocks, all split; the halves meet inside segment 1
+    (2, 12, 128, 100, 420),   # 72 blocks, 5 steps: halves of 2 and 3 steps
+    (1, 30, 128, 0, 200),     # 2 steps: halves of one step each
+])
+def test_attention_split_parity(cuda, B, heads, d, n0, n1):
+    """The persistent launch that runs its last round's query blocks as two
+    halves of their K/V steps (launch 3, with a scratch): O and lse against
+    the fp64 attention and its log-sum-exp, and against the unsplit launch."""
+    import math
+    import torch
+    from paper_2602_12529_gb300 import ffi
+    lib = ffi.lib()
+    H = heads * d
+    sms = torch.cuda.get_device_properties(cuda).multi_processor_count
+    items = B * heads * ((n0 + 255) // 256 + (n1 + 255) // 256)
+    assert _split_applies(items, sms), (items, sms)
+    q0 = _bf((max(B * n0, 1), 3 * H), 31, 1.0, "q0")
+    q1 = _bf((B * n1, 3 * H), 32, 1.0, "q1")
+    qg0, qg1 = _dev_bf16(q0, cuda), _dev_bf16(q1, cuda)
+    L = lib.ff_attention_lse_rows(n0, n1)
+    ws = torch.full((ffi.ff_attention_forward_workspace_size(d),), 0xA5, dtype=torch.uint8, device=cuda)
+    res = {}
+    for launch in (3, 1):
+        o0 = torch.zeros((max(B * n0, 1), H), dtype=torch.bfloat16, device=cuda)
+        o1 = torch.zeros((B * n1, H), dtype=torch.bfloat16, device=cuda)
+        lse = torch.zeros(B * heads * L, device=cuda)
+        assert lib.ff_debug_attention_launch(launch) == 0
+        try:
+            for _ in range(2):   # a second call finds the tickets as the first left them
+                ffi.ff_attention_forward(B, heads, d, qg0, o0, n0, qg1, o1, n1, lse=lse, ws=ws)
+            torch.cuda.synchronize()
+        finally:
+            lib.ff_debug_attention_launch(0)
+        res[launch] = (_host_bf16(o0), _host_bf16(o1), lse.cpu().numpy().reshape(B, heads, L))
+    assert ffi.ff_check_device_status() == 0
+    w0, w1 = odit.widen(q0), odit.widen(q1)
+    g0, g1, lse_h = res[3]
+    for b in range(B):
+        rows = np.concatenate([w0[b * n0:(b + 1) * n0, :3 * H], w1[b * n1:(b + 1) * n1, :3 * H]])
+        q = rows[:, :H].reshape(-1, heads, d)
+        k = rows[:, H:2 * H].reshape(-1, heads, d)
+        v = rows[:, 2 * H:].reshape(-1, heads, d)
+        want = odit.attention(q, k, v).reshape(-1, H)
+        got = np.concatenate([g0[b * n0:(b + 1) * n0], g1[b * n1:(b + 1) * n1]])
+        assert rms_rel(got, want) <= 1e-2, (b, rms_rel(got, want))
+        want_lse = odit.attention_lse(q, k) / math.log(2.0)
+        got_lse = np.concatenate([lse_h[b, :, :n0], lse_h[b, :, (n0 + 127) // 128 * 128:][:, :n1]], axis=1).T
+        np.testing.assert_allclose(got_lse, want_lse, rtol=2e-4, atol=2e-4)
+    # split and unsplit: the same attention up to fp32 rounding before the bf16 output
+    u0, u1, ulse = res[1]
+    got = np.concatenate([g0[:B * n0], g1])
+    ref = np.concatenate([u0[:B * n0], u1])
+    assert rms_rel(got, ref) <= 4e-3
+    np.testing.assert_allclose(lse_h, ulse, rtol=1e-5, atol=1e-5)
+
+
+def test_attention_split_flux_block_sampled(cuda):
+    """The Flux double-block shape (4 samples, 24 heads of 128, 512 text +
+    4096 image tokens: 1728 query blocks) in the launch the velocity network
+    takes (automatic choice, with a scratch): 56 blocks past the 11 full
+    rounds run split on 152 SMs.  Sampled rows of split and unsplit blocks
+    against the fp64 attention and log-sum-exp."""
+    import math
+    import torch
+    from paper_2602_12529_gb300 import ffi
+    lib = ffi.lib()
+    B, heads, d, n0, n1 = 4, 24, 128, 512, 4096
+    H = heads * d
+    N = n0 + n1
+    q0 = _bf((B * n0, 3 * H), 41, 1.0, "q0")
+    q1 = _bf((B * n1, 3 * H), 42, 1.0, "q1")
+    o0 = torch.zeros((B * n0, H), dtype=torch.bfloat16, device=cuda)
+    o1 = torch.zeros((B * n1, H), dtype=torch.bfloat16, device=cuda)
+    L = lib.ff_attention_lse_rows(n0, n1)
+    lse = torch.zeros(B * heads * L, device=cuda)
+    ffi.ff_attention_forward(B, heads, d, _dev_bf16(q0, cuda), o0, n0, _dev_bf16(q1, cuda), o1, n1, lse=lse)
+    torch.cuda.synchronize()
+    assert ffi.ff_check_device_status() == 0
+    g0, g1 = _host_bf16(o0), _host_bf16(o1)
+    lse_h = lse.cpu().numpy().reshape(B, heads, L)
+    w0, w1 = odit.widen(q0), odit.widen(q1)
+    qpairs = n0 // 256 + n1 // 256
+    sms = torch.cuda.get_device_properties(cuda).multi_processor_count
+    items = B * heads * qpairs
+    split_first = items // sms * sms if _split_applies(items, sms) else items
+    rng = np.random.default_rng(7)
+    # (b, h, joint row): rows of the last (split) blocks, the first block and a middle one
+    picks = []
+    for it in (items - 1, items - 2, split_first, 0, items // 2):
+        qp, bh = it % qpairs, it // qpairs
+        b, h = bh // heads, bh % heads
+        base = qp * 256 if qp < n0 // 256 else n0 + (qp - n0 // 256) * 256
+        picks += [(b, h, base + int(r)) for r in rng.choice(256, 6, replace=False)]
+    for b in sorted({p[0] for p in picks}):
+        rows = np.concatenate([w0[b * n0:(b + 1) * n0, :3 * H], w1[b * n1:(b + 1) * n1, :3 * H]])
+        for bb, h, r in picks:
+            if bb != b:
+                continue
+            q = rows[r:r + 1, h * d:(h + 1) * d].reshape(1, 1, d)
+            k = rows[:, H + h * d:H + (h + 1) * d].reshape(N, 1, d)
+            v = rows[:, 2 * H + h * d:2 * H + (h + 1) * d].reshape(N, 1, d)
+            want = odit.attention(q, k, v).reshape(d)
+            got = (g0[b * n0 + r] if r < n0 else g1[b * n1 + r - n0])[h * d:(h + 1) * d]
+            assert rms_rel(got, want) <= 1e-2, (b, h, r)
+            want_lse = odit.attention_lse(q, k).reshape(()) / math.log(2.0)
+            got_lse = lse_h[b, h, r if r < n0 else (n0 + 127) // 128 * 128 + r - n0]
+            assert abs(got_lse - want_lse) <= 2e-4 * max(1.0, abs(want_lse)), (b, h, r)
+
+
 @pytest.mark.parametrize("rows,H,tps", [(96, 256, 32), (1000, 3072, 250)])
 def test_ln_modulate_parity(cuda, rows, H, tps):
     import torch
