@@ -49,6 +49,19 @@ int ff_debug_attention(int B, int heads, int head_dim, int n0, const void* qkv0,
  * output when no split is taken; a split launch agrees to fp32 rounding. */
 int ff_debug_attention_launch(int mode);
 
+/* The attention launcher's plan for `items` work items (256-row query
+ * blocks) of `steps` K/V steps each on a GPU of `sms` SMs, with (have_ws !=
+ * 0) or without the split scratch, under launch mode `mode` (as
+ * ff_debug_attention_launch).  Host arithmetic only: nothing is launched
+ * and no GPU is needed.  Writes (host pointers) *persistent (1: one CTA per
+ * SM runs a strided share of the items; 0: one item per CTA), *grid (CTAs),
+ * and *split_first, *split_n: items split_first .. split_first + split_n - 1
+ * run as two halves of their K/V steps on CTAs 0 .. 2 split_n - 1 (split_n
+ * = 0: no split).  FF_ERR_INVALID_ARG for items, sms or steps <= 0, a mode
+ * outside 0-3 or a null pointer. */
+int ff_debug_attention_plan(int64_t items, int sms, int steps, int have_ws, int mode, int* persistent,
+                            int64_t* grid, int64_t* split_first, int64_t* split_n);
+
 /* out[r] = LN(x[r]) * (1 + mods[b, scale_off:]) + mods[b, shift_off:] for
  * rows r of x (fp32 [rows, H]); b = r / tokens_per_sample; out bf16 [rows, H]. */
 int ff_debug_ln_modulate(int rows, int H, const float* x, const float* mods, int64_t ld_mods, int shift_off,

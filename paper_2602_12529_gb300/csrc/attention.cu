@@ -617,6 +617,29 @@ attn_tcgen05_kernel(const __grid_constant__ CUtensorMap tm_q0, const __grid_cons
     }
 }
 
+// The launch variant and grid for `items` work items of `steps` K/V steps
+// on `sms` SMs (forced: the test override, 0 for the launcher's own choice).
+struct LaunchPlan {
+    bool persistent;
+    int64_t grid;
+    int64_t split_first, split_n;   // split_n > 0: items split_first .. items - 1 run as two halves each
+};
+LaunchPlan launch_plan(int64_t items, int sms, int steps, int forced, bool have_ws) {
+    LaunchPlan r{};
+    r.persistent = forced ? forced == 1 || forced == 3
+                          : items < static_cast<int64_t>(kPersistentItemsPerSm) * sms || steps <= kPersistentMaxSteps;
+    r.grid = r.persistent ? (items < sms ? items : sms) : items;
+    if (r.persistent && (forced == 0 || forced == 3) && have_ws && steps >= 2) {
+        const int64_t rounds = items / sms, rest = items % sms;
+        if (rest > 0 && 2 * rest <= sms && rest <= kSplitMaxItems) {
+            r.split_first = rounds * sms;
+            r.split_n = rest;
+            r.grid = rounds > 0 ? sms : 2 * rest;
+        }
+    }
+    return r;
+}
+
 // Scratch of a split launch: per split item, both halves' unnormalised O of
 // both query tiles (fp32), their (m, l), and 8 tickets.
 size_t split_part_bytes(int hd) { return static_cast<size_t>(kSplitMaxItems) * 2 * 2 * kBM * hd * sizeof(float); }
@@ -677,32 +700,25 @@ int launch_attn(const AttnSpec& a, cudaStream_t stream) {
     // steps on 2 L CTAs, given the caller's scratch: Flux block, 1728 items =
     // 11 rounds + 56, so the last round ends after half an item.
     const int steps = (a.kv[0].n + kBN - 1) / kBN + (a.kv[1].n + kBN - 1) / kBN;
-    const int forced = g_launch_override.load(std::memory_order_relaxed);
-    const int sms = num_sms();
-    const bool persistent = forced ? forced == 1 || forced == 3
-                                   : items < static_cast<int64_t>(kPersistentItemsPerSm) * sms ||
-                                         steps <= kPersistentMaxSteps;
-    int64_t grid64 = persistent ? (items < sms ? items : sms) : items;
-    p.split_first = p.split_n = 0;
+    const bool have_ws = a.split_ws && a.split_ws_bytes >= attention_split_ws_bytes(HD);
+    const LaunchPlan plan =
+        launch_plan(items, num_sms(), steps, g_launch_override.load(std::memory_order_relaxed), have_ws);
+    const bool persistent = plan.persistent;
+    p.split_first = static_cast<int>(plan.split_first);
+    p.split_n = static_cast<int>(plan.split_n);
     p.part = nullptr;
     p.part_ml = nullptr;
     p.tickets = nullptr;
-    if (persistent && (forced == 0 || forced == 3) && a.split_ws && steps >= 2 &&
-        a.split_ws_bytes >= attention_split_ws_bytes(HD)) {
-        const int64_t rounds = items / sms, rest = items % sms;
-        if (rest > 0 && 2 * rest <= sms && rest <= kSplitMaxItems) {
-            uint8_t* ws = static_cast<uint8_t*>(a.split_ws);
-            p.split_first = static_cast<int>(rounds * sms);
-            p.split_n = static_cast<int>(rest);
-            p.part = reinterpret_cast<float*>(ws);
-            p.part_ml = reinterpret_cast<float2*>(ws + split_part_bytes(HD));
-            p.tickets = reinterpret_cast<unsigned*>(ws + split_part_bytes(HD) + split_ml_bytes());
-            grid64 = rounds > 0 ? sms : 2 * rest;
-            if (cudaMemsetAsync(p.tickets, 0, static_cast<size_t>(rest) * 8 * sizeof(unsigned), stream) != cudaSuccess)
-                return set_error(FF_ERR_CUDA, "attention: cannot clear the split tickets");
-        }
+    if (plan.split_n > 0) {
+        uint8_t* ws = static_cast<uint8_t*>(a.split_ws);
+        p.part = reinterpret_cast<float*>(ws);
+        p.part_ml = reinterpret_cast<float2*>(ws + split_part_bytes(HD));
+        p.tickets = reinterpret_cast<unsigned*>(ws + split_part_bytes(HD) + split_ml_bytes());
+        if (cudaMemsetAsync(p.tickets, 0, static_cast<size_t>(plan.split_n) * 8 * sizeof(unsigned), stream) !=
+            cudaSuccess)
+            return set_error(FF_ERR_CUDA, "attention: cannot clear the split tickets");
     }
-    const int grid = static_cast<int>(grid64);
+    const int grid = static_cast<int>(plan.grid);
     const double nkv = static_cast<double>(a.kv[0].n + a.kv[1].n);
     const double nq = static_cast<double>(a.q[0].n + a.q[1].n);
     ProfScope prof(stream, "attention", 4.0 * a.B * a.heads * nq * nkv * HD,
@@ -719,6 +735,26 @@ int launch_attn(const AttnSpec& a, cudaStream_t stream) {
 }  // namespace
 
 int attention_launch_override(int mode) { return g_launch_override.exchange(mode); }
+
+}  // namespace ff
+
+// The attention launcher's choice for a launch of `items` query blocks of
+// `steps` K/V steps on `sms` SMs (host arithmetic only; for tests).
+extern "C" int ff_debug_attention_plan(int64_t items, int sms, int steps, int have_ws, int mode, int* persistent,
+                                       int64_t* grid, int64_t* split_first, int64_t* split_n) {
+    using namespace ff;
+    if (items <= 0 || sms <= 0 || steps <= 0 || mode < 0 || mode > 3 || !persistent || !grid || !split_first ||
+        !split_n)
+        return set_error(FF_ERR_INVALID_ARG, "attention plan: bad arguments");
+    const LaunchPlan r = launch_plan(items, sms, steps, mode, have_ws != 0);
+    *persistent = r.persistent ? 1 : 0;
+    *grid = r.grid;
+    *split_first = r.split_first;
+    *split_n = r.split_n;
+    return FF_OK;
+}
+
+namespace ff {
 
 size_t attention_split_ws_bytes(int head_dim) {
     return split_part_bytes(head_dim) + split_ml_bytes() + static_cast<size_t>(kSplitMaxItems) * 8 * sizeof(unsigned);

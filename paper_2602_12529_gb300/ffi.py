@@ -105,6 +105,8 @@ _SIGS = {
     "ff_debug_gemm_gated": ([_I, _I, _I, _P, _I64, _P, _I64, _P, _P, _I64, _P, _I64, _I, _P], _I),
     "ff_debug_attention": ([_I, _I, _I, _I, _P, _I64, _P, _I64, _I, _P, _I64, _P, _I64, _P], _I),
     "ff_debug_attention_launch": ([_I], _I),
+    "ff_debug_attention_plan": ([_I64, _I, _I, _I, _I, C.POINTER(_I), C.POINTER(_I64), C.POINTER(_I64),
+                                 C.POINTER(_I64)], _I),
     "ff_debug_ln_modulate": ([_I, _I, _P, _P, _I64, _I, _I, _I, _P, _P], _I),
     "ff_debug_qk_norm_rope": ([_I, _I, _I, _I, _P, _I64, _P, _P, _I, _I, _I, C.POINTER(_I), _F, _P], _I),
     "ff_debug_reduce_chunks": ([_I, _I, _P, _P, C.POINTER(_I64), C.POINTER(_I64), C.POINTER(_I), C.POINTER(_I),

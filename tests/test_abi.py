@@ -100,6 +100,53 @@ def test_workspace_queries(L):
         ffi.ff_attention_forward_workspace_size(96)
 
 
+def _plan(L, items, sms, steps, have_ws, mode=0):
+    import ctypes as C
+    pers, grid, first, n = C.c_int(), C.c_int64(), C.c_int64(), C.c_int64()
+    rc = L.ff_debug_attention_plan(items, sms, steps, have_ws, mode, C.byref(pers), C.byref(grid), C.byref(first),
+                                   C.byref(n))
+    assert rc == 0, L.ff_last_error()
+    return pers.value, grid.value, first.value, n.value
+
+
+def test_attention_launch_plan(L):
+    """The attention launcher's choice of variant, grid and split (host
+    arithmetic, no GPU): persistent below 16 query blocks per SM or with at
+    most 128 K/V steps per block, one block per CTA otherwise; a persistent
+    launch with the scratch splits a last round that is at most half full."""
+    # Flux block (B 4, 24 heads, 512 + 4096 tokens): 1728 blocks of 36 steps
+    # on 152 SMs, 11 rounds + 56 -> 56 blocks split over CTAs 0 .. 111
+    assert _plan(L, 1728, 152, 36, 1) == (1, 152, 1672, 56)
+    assert _plan(L, 1728, 152, 36, 0) == (1, 152, 0, 0)           # no scratch: unsplit
+    assert _plan(L, 1728, 152, 36, 1, mode=1) == (1, 152, 0, 0)   # forced unsplit
+    assert _plan(L, 1728, 152, 36, 1, mode=2) == (0, 1728, 0, 0)  # forced one block per CTA
+    # WAN self-attention (32760 tokens, 40 heads): 5120 blocks of 256 steps
+    assert _plan(L, 5120, 152, 256, 1) == (0, 5120, 0, 0)
+    # forced persistent with the split: 104 left over, more than half of 152
+    assert _plan(L, 5120, 152, 256, 1, mode=3) == (1, 152, 0, 0)
+    # WAN cross-attention (512 text keys): 4 steps, persistent, 104 left over
+    assert _plan(L, 5120, 152, 4, 1) == (1, 152, 0, 0)
+    # fewer blocks than SMs: every block split, two CTAs each
+    assert _plan(L, 60, 152, 4, 1) == (1, 120, 0, 60)
+    assert _plan(L, 76, 152, 4, 1) == (1, 152, 0, 76)
+    assert _plan(L, 77, 152, 4, 1) == (1, 77, 0, 0)               # 154 halves do not fit
+    # a single K/V step cannot be halved
+    assert _plan(L, 60, 152, 1, 1) == (1, 60, 0, 0)
+    # an exact number of rounds leaves nothing to split
+    assert _plan(L, 304, 152, 36, 1) == (1, 152, 0, 0)
+    # at most 96 split blocks (the scratch's capacity), even on a larger GPU
+    assert _plan(L, 256 + 96, 256, 36, 1) == (1, 256, 256, 96)
+    assert _plan(L, 256 + 100, 256, 36, 1) == (1, 256, 0, 0)
+    # 16 blocks per SM and more than 128 steps: one block per CTA
+    assert _plan(L, 16 * 152, 152, 129, 1) == (0, 16 * 152, 0, 0)
+    assert _plan(L, 16 * 152 - 1, 152, 129, 1)[0] == 1
+    import ctypes as C
+    x = C.c_int(); y = C.c_int64()
+    assert L.ff_debug_attention_plan(0, 152, 4, 1, 0, C.byref(x), C.byref(y), C.byref(y), C.byref(y)) == 1
+    assert L.ff_debug_attention_plan(10, 152, 4, 1, 4, C.byref(x), C.byref(y), C.byref(y), C.byref(y)) == 1
+    assert L.ff_debug_attention_plan(10, 152, 4, 1, 0, None, C.byref(y), C.byref(y), C.byref(y)) == 1
+
+
 def test_host_validation_without_gpu(L):
     # every one of these is rejected before any CUDA call is made
     assert L.ff_debug_attention_launch(4) == 1          # variants are 0 to 3
