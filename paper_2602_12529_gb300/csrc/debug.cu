@@ -47,6 +47,10 @@ int ff_attention_forward(int B, int heads, int head_dim, int n0, const void* qkv
     using namespace ff;
     if (lse && !aligned16(lse)) return set_error(FF_ERR_INVALID_ARG, "attention: lse must be 16-byte aligned");
     if (ws && !aligned16(ws)) return set_error(FF_ERR_INVALID_ARG, "attention: ws must be 16-byte aligned");
+    // head h of O lands at columns h d .. h d + d - 1 of its row
+    if ((n0 > 0 && ldo0 < static_cast<int64_t>(heads) * head_dim) ||
+        (n1 > 0 && ldo1 < static_cast<int64_t>(heads) * head_dim))
+        return set_error(FF_ERR_INVALID_ARG, "attention: output pitch below heads * head_dim");
     AttnSpec a;
     const int H = heads * head_dim;
     const void* qkv[2] = {qkv0, qkv1};
@@ -104,6 +108,8 @@ int ff_cross_attention_forward(int B, int heads, int head_dim, int nq, const voi
     using namespace ff;
     if (nq <= 0 || nk <= 0) return set_error(FF_ERR_INVALID_ARG, "cross-attention: nq and nk must be positive");
     if (lse && !aligned16(lse)) return set_error(FF_ERR_INVALID_ARG, "cross-attention: lse must be 16-byte aligned");
+    if (ldo < static_cast<int64_t>(heads) * head_dim)
+        return set_error(FF_ERR_INVALID_ARG, "cross-attention: output pitch below heads * head_dim");
     AttnSpec a;
     a.q[0] = AttnQuerySeg{static_cast<const __nv_bfloat16*>(q), ldq, nq, static_cast<__nv_bfloat16*>(out), ldo};
     a.q[1] = AttnQuerySeg{nullptr, 0, 0, nullptr, 0};
@@ -162,6 +168,9 @@ int ff_debug_attention(int B, int heads, int head_dim, int n0, const void* qkv0,
                        int64_t ldo0, int n1, const void* qkv1, int64_t ld1, void* out1, int64_t ldo1,
                        cudaStream_t stream) {
     using namespace ff;
+    if ((n0 > 0 && ldo0 < static_cast<int64_t>(heads) * head_dim) ||
+        (n1 > 0 && ldo1 < static_cast<int64_t>(heads) * head_dim))
+        return set_error(FF_ERR_INVALID_ARG, "attention: output pitch below heads * head_dim");
     AttnSegment s0{static_cast<const __nv_bfloat16*>(qkv0), ld0, static_cast<__nv_bfloat16*>(out0), ldo0, n0};
     AttnSegment s1{static_cast<const __nv_bfloat16*>(qkv1), ld1, static_cast<__nv_bfloat16*>(out1), ldo1, n1};
     return attention(s0, s1, B, heads, head_dim, heads * head_dim, stream);

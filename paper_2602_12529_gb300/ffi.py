@@ -180,6 +180,17 @@ def _need(t, n: int, name: str):
         raise ValueError(f"{name}: {t.numel()} elements, the call touches {n}")
 
 
+def _rows(t, rows: int, cols: int, name: str):
+    """Raise unless t (row pitch t.shape[-1]) holds `rows` rows of at least
+    `cols` columns: the attention kernels address row r at r * pitch."""
+    if rows <= 0:
+        return
+    if t is None:
+        raise ValueError(f"{name}: missing, {rows} rows needed")
+    if t.dim() < 2 or t.shape[-1] < cols or t.numel() // t.shape[-1] < rows:
+        raise ValueError(f"{name}: shape {tuple(t.shape)}, the call touches {rows} rows of {cols} columns")
+
+
 def _sde_args(x_t, v, eps, x_next, t, t_next, sigma, logp, ld, need_eps):
     """dtype and size checks shared by the SDE step wrappers: [B, D] arrays,
     [B] times and sigmas, logp read at b * ld."""
@@ -614,6 +625,16 @@ def ff_attention_forward(B, heads, head_dim, qkv0, out0, n0, qkv1, out1, n1, lse
     ws: the optional scratch that lets the launch split its last round's items (None: a fresh one of
     ff_attention_forward_workspace_size bytes; False: none, the unsplit launch)."""
     import torch
+    H = heads * head_dim
+    for n_, q_, o_, tag in ((n0, qkv0, out0, "0"), (n1, qkv1, out1, "1")):
+        _rows(q_, B * n_, 3 * H, "qkv" + tag)
+        _rows(o_, B * n_, H, "out" + tag)
+        if n_ > 0:
+            _check(q_, torch.bfloat16, "qkv" + tag)
+            _check(o_, torch.bfloat16, "out" + tag)
+    if lse is not None:
+        _check(lse, torch.float32, "lse")
+        _need(lse, B * heads * lib().ff_attention_lse_rows(n0, n1), "lse")
     if ws is None:
         dev = (qkv0 if n0 else qkv1).device
         ws = torch.empty(ff_attention_forward_workspace_size(head_dim), dtype=torch.uint8, device=dev)
@@ -629,6 +650,15 @@ def ff_attention_backward(B, heads, head_dim, seg0, seg1, lse, ws=None, stream=N
     import torch
     n0, q0, o0, g0, d0 = seg0
     n1, q1, o1, g1, d1 = seg1
+    H = heads * head_dim
+    for n_, q_, o_, g_, d_, tag in ((n0, q0, o0, g0, d0, "0"), (n1, q1, o1, g1, d1, "1")):
+        _rows(q_, B * n_, 3 * H, "qkv" + tag)
+        _rows(o_, B * n_, H, "out" + tag)
+        _rows(g_, B * n_, H, "dout" + tag)
+        _rows(d_, B * n_, 3 * H, "dqkv" + tag)
+        if n_ > 0 and g_ is not None and o_ is not None and g_.shape[-1] != o_.shape[-1]:
+            raise ValueError(f"dout{tag} and out{tag} share one row pitch")
+    _need(lse, B * heads * lib().ff_attention_lse_rows(n0, n1), "lse")
     if ws is None:
         sz = _SZ()
         _call("ff_attention_backward_workspace_size", B, heads, n0, n1, C.byref(sz))
@@ -641,6 +671,12 @@ def ff_attention_backward(B, heads, head_dim, seg0, seg1, lse, ws=None, stream=N
 def ff_cross_attention_forward(B, heads, head_dim, q, nq, kv, nk, out, lse=None, stream=None):
     """Cross-attention: q [B nq, >= H] (q at columns h d), kv [B nk, >= 2H] (k at
     h d, v at H + h d), out [B nq, >= H]; lse [B, heads, ff_attention_lse_rows(nq, 0)] or None."""
+    H = heads * head_dim
+    _rows(q, B * nq, H, "q")
+    _rows(kv, B * nk, 2 * H, "kv")
+    _rows(out, B * nq, H, "out")
+    if lse is not None:
+        _need(lse, B * heads * lib().ff_attention_lse_rows(nq, 0), "lse")
     _call("ff_cross_attention_forward", B, heads, head_dim, nq, _ptr(q), q.shape[-1], nk, _ptr(kv), kv.shape[-1],
           _ptr(out), out.shape[-1], _ptr(lse), _stream(stream))
 
@@ -648,6 +684,16 @@ def ff_cross_attention_forward(B, heads, head_dim, q, nq, kv, nk, out, lse=None,
 def ff_cross_attention_backward(B, heads, head_dim, q, nq, out, dout, dq, kv, nk, dkv, lse, ws=None, stream=None):
     """Writes dq (like q) and dk | dv (like kv) from dO (like out) and the forward's lse."""
     import torch
+    H = heads * head_dim
+    _rows(q, B * nq, H, "q")
+    _rows(out, B * nq, H, "out")
+    _rows(dout, B * nq, H, "dout")
+    _rows(dq, B * nq, H, "dq")
+    _rows(kv, B * nk, 2 * H, "kv")
+    _rows(dkv, B * nk, 2 * H, "dkv")
+    if dout.shape[-1] != out.shape[-1]:
+        raise ValueError("dout and out share one row pitch")
+    _need(lse, B * heads * lib().ff_attention_lse_rows(nq, 0), "lse")
     if ws is None:
         sz = _SZ()
         _call("ff_attention_backward_workspace_size", B, heads, nq, 0, C.byref(sz))
@@ -665,6 +711,10 @@ def ff_debug_gemm_gated(A, B, bias, resid, gate, rows_per_sample, stream=None):
 
 
 def ff_debug_attention(B, heads, head_dim, qkv0, out0, n0, qkv1, out1, n1, stream=None):
+    H = heads * head_dim
+    for n_, q_, o_, tag in ((n0, qkv0, out0, "0"), (n1, qkv1, out1, "1")):
+        _rows(q_, B * n_, 3 * H, "qkv" + tag)
+        _rows(o_, B * n_, H, "out" + tag)
     _call("ff_debug_attention", B, heads, head_dim, n0, _ptr(qkv0), qkv0.shape[-1], _ptr(out0), out0.shape[-1],
           n1, _ptr(qkv1), qkv1.shape[-1], _ptr(out1), out1.shape[-1], _stream(stream))
 

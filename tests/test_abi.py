@@ -147,6 +147,37 @@ def test_attention_launch_plan(L):
     assert L.ff_debug_attention_plan(10, 152, 4, 1, 0, None, C.byref(y), C.byref(y), C.byref(y)) == 1
 
 
+def test_attention_entries_reject_short_buffers(L):
+    """Buffers too small for the launch are refused before anything runs:
+    in the Python binding by shape (host tensors suffice, nothing reaches
+    the library), and in the C entries by the output pitch (null pointers:
+    nothing could be launched even past the check)."""
+    import torch
+    from paper_2602_12529_gb300 import ffi
+    B, heads, d, n0, n1 = 2, 2, 64, 0, 100
+    H = heads * d
+    q1 = torch.zeros(B * n1, 3 * H, dtype=torch.bfloat16)
+    o1 = torch.zeros(B * n1, H, dtype=torch.bfloat16)
+    dummy = torch.zeros(1, 3 * H, dtype=torch.bfloat16)
+    with pytest.raises(ValueError, match="out1"):
+        ffi.ff_attention_forward(B, heads, d, dummy, dummy, n0, q1, o1[:B * n1 - 1], n1)
+    with pytest.raises(ValueError, match="out1"):
+        ffi.ff_attention_forward(B, heads, d, dummy, dummy, n0, q1, o1[:, :H - 8].contiguous(), n1)
+    with pytest.raises(ValueError, match="qkv1"):
+        ffi.ff_attention_forward(B, heads, d, dummy, dummy, n0, q1[:, :2 * H].contiguous(), o1, n1)
+    with pytest.raises(ValueError, match="lse"):
+        ffi.ff_attention_forward(B, heads, d, dummy, dummy, n0, q1, o1, n1, lse=torch.zeros(10))
+    with pytest.raises(ValueError, match="kv"):
+        ffi.ff_cross_attention_forward(B, heads, d, o1, n1, o1[:8], 8, o1)
+    with pytest.raises(ValueError, match="dqkv1"):
+        ffi.ff_attention_backward(B, heads, d, (0, None, None, None, None), (n1, q1, o1, o1, o1), torch.zeros(1))
+    # C entries: an output pitch below heads * head_dim
+    rc = L.ff_attention_forward(B, heads, d, 0, None, 0, None, 0, n1, None, 3 * H, None, H - 8, None, None, 0, None)
+    assert rc == 1 and b"pitch" in L.ff_last_error()
+    rc = L.ff_cross_attention_forward(B, heads, d, n1, None, H, 8, None, 2 * H, None, H - 8, None, None)
+    assert rc == 1 and b"pitch" in L.ff_last_error()
+
+
 def test_host_validation_without_gpu(L):
     # every one of these is rejected before any CUDA call is made
     assert L.ff_debug_attention_launch(4) == 1          # variants are 0 to 3
