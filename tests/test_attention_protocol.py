@@ -25,6 +25,10 @@ TMEM, ordered only by mbarrier phases:
 A split launch gives a CTA one half item after its whole items: steps
 [0, h) or [h, T) of an item of T steps.
 
+The backward's two kernels (csrc/attention_bwd.cu: dQ over key tiles, dK / dV
+over query tiles, each with a ring of three and a ring of two operand slots)
+get models of the same kind below.
+
 The model executes random interleavings and checks every hazard: a slot,
 query tile or TMEM region overwritten while a reader is pending, an operand
 read before its copy landed, a barrier receiving more arrivals than its
@@ -252,6 +256,275 @@ def _simulate(S, steps, items, seed, half=None, defect=None, max_events=10 ** 6)
     raise _Hazard("no progress: deadlock")
 
 
+def _run(agents, pipe, tma, execute, land, rng, max_events=10 ** 6):
+    """Random interleaving of the agents (generators), the in-order tensor
+    pipe and the TMA engine (copies land in any order) until all finish."""
+    done = set()
+    for _ in range(max_events):
+        live = [a for a in agents if a not in done]
+        hardware = (["pipe"] if pipe else []) + (["tma"] if tma else [])
+        if not live and not hardware:
+            return
+        choice = rng.choice(live + hardware * 2)
+        if choice == "pipe":
+            execute(pipe.pop(0))
+        elif choice == "tma":
+            land(tma.pop(rng.randrange(len(tma))))
+        else:
+            try:
+                next(agents[choice])
+            except StopIteration:
+                done.add(choice)
+    raise _Hazard("no progress: deadlock")
+
+
+def _waiter(bars):
+    def wait(name, parity, need_phases):
+        while not bars[name].passes(parity):
+            yield "blocked"
+        if bars[name].phases < need_phases:
+            raise _Hazard(f"{name}: parity wait passed on an older phase")
+    return wait
+
+
+def _ring_wait(wait, name, j):
+    """Wait for phase j of a four-entry barrier ring (entry j % 4)."""
+    return wait(f"{name}{j & 3}", (j >> 2) & 1, (j >> 2) + 1)
+
+
+def _simulate_dq(T, seed, defect=None):
+    """The backward's dQ kernel (csrc/attention_bwd.cu) for one 128-row query
+    tile against T key tiles: K_j into K slot j % 3 once dQ_j-3 is done
+    (rel ring), V_j into V slot j % 2 once S / dP of tile j - 2 are done
+    (s0 ring), both on operand barrier j % 4 (two arrivals); the MMA thread
+    issues S_j+1 / dP_j+1 once both elementwise warps hold S_j / dP_j, and
+    dQ += dS_j K_j once both have written dS_j; an elementwise warp writes
+    dS_j only after dQ_j-1 (rel ring).  defect: "no_v_wait" drops the
+    producer's wait before reusing a V slot; "no_ds_wait" drops the
+    elementwise warps' wait before writing dS."""
+    rng = random.Random(seed)
+    bars = {"p0": _Bar("p0", 2), "p1": _Bar("p1", 2), "done": _Bar("done", 1)}
+    for i in range(4):
+        bars[f"grp{i}"] = _Bar(f"grp{i}", 2)
+        bars[f"rel{i}"] = _Bar(f"rel{i}", 1)
+        bars[f"sring{i}"] = _Bar(f"sring{i}", 1)
+    wait = _waiter(bars)
+    kslot, vslot = [[None, False] for _ in range(3)], [[None, False] for _ in range(2)]
+    kread, vread = [set() for _ in range(3)], [set() for _ in range(2)]
+    tma, pipe = [], []
+    st = {"sp": None, "sp_read": [-1, -1], "ds": [-1, -1], "dq": -1}
+
+    def producer():
+        for j in range(T):
+            if j >= 3:
+                yield from _ring_wait(wait, "rel", j - 3)
+            if kread[j % 3]:
+                raise _Hazard(f"K slot {j % 3} reused with reads pending")
+            bars[f"grp{j & 3}"].arrive(tx=1)
+            kslot[j % 3][:] = [j, False]
+            kread[j % 3] |= {("SDP", j), ("DQ", j)}
+            tma.append(("k", j % 3, j, f"grp{j & 3}"))
+            if j >= 2 and defect != "no_v_wait":
+                yield from _ring_wait(wait, "sring", j - 2)
+            if vread[j % 2]:
+                raise _Hazard(f"V slot {j % 2} reused with reads pending")
+            bars[f"grp{j & 3}"].arrive(tx=1)
+            vslot[j % 2][:] = [j, False]
+            vread[j % 2] |= {("SDP", j)}
+            tma.append(("v", j % 2, j, f"grp{j & 3}"))
+            yield "step"
+
+    def mma():
+        yield from _ring_wait(wait, "grp", 0)
+        pipe.extend([("SDP", 0), ("commit", "sring0")])
+        for j in range(T):
+            yield from wait("p0", j & 1, j + 1)
+            if j + 1 < T:
+                pipe.extend([("SDP", j + 1), ("commit", f"sring{(j + 1) & 3}")])
+            yield from wait("p1", j & 1, j + 1)
+            pipe.extend([("DQ", j), ("commit", f"rel{j & 3}")])
+            yield "step"
+        pipe.append(("commit", "done"))
+
+    def elementwise(cg):
+        for j in range(T):
+            yield from _ring_wait(wait, "sring", j)
+            for _ in range(2):   # the TMEM loads span two events
+                if st["sp"] != j:
+                    raise _Hazard(f"warp {cg} read S / dP {st['sp']} for tile {j}")
+                yield "step"
+            st["sp_read"][cg] = j
+            if j + 1 < T:
+                yield from _ring_wait(wait, "grp", j + 1)
+            bars["p0"].arrive()
+            yield "step"
+            if j > 0 and defect != "no_ds_wait":
+                yield from _ring_wait(wait, "rel", j - 1)
+            if st["dq"] < j - 1:
+                raise _Hazard(f"warp {cg} wrote dS_{j} before dQ_{j - 1} read dS_{j - 1}")
+            st["ds"][cg] = j
+            bars["p1"].arrive()
+            yield "step"
+        yield from wait("done", 0, 1)
+        if st["dq"] != T - 1:
+            raise _Hazard("dQ read before its last product")
+
+    def execute(op):
+        if op[0] == "SDP":
+            j = op[1]
+            if kslot[j % 3] != [j, True] or vslot[j % 2] != [j, True]:
+                raise _Hazard(f"S / dP of tile {j} read K or V before it landed")
+            if j > 0 and min(st["sp_read"]) < j - 1:
+                raise _Hazard(f"S / dP of tile {j} overwrote tile {j - 1}'s before both warps read them")
+            st["sp"] = j
+            kread[j % 3].discard(("SDP", j))
+            vread[j % 2].discard(("SDP", j))
+        elif op[0] == "DQ":
+            j = op[1]
+            if st["ds"] != [j, j]:
+                raise _Hazard(f"dQ_{j} read dS {st['ds']}")
+            if kslot[j % 3] != [j, True] or st["dq"] != j - 1:
+                raise _Hazard(f"dQ_{j} out of order or before K_{j} landed")
+            st["dq"] = j
+            kread[j % 3].discard(("DQ", j))
+        else:
+            bars[op[1]].arrive()
+
+    def land(copy):
+        kind, idx, owner, bar = copy
+        ring = kslot if kind == "k" else vslot
+        if ring[idx][0] == owner:
+            ring[idx][1] = True
+        bars[bar].complete_tx(1)
+
+    agents = {"producer": producer(), "mma": mma(), "ew0": elementwise(0), "ew1": elementwise(1)}
+    _run(agents, pipe, tma, execute, land, rng)
+
+
+def _simulate_dkdv(T, seed, defect=None):
+    """The backward's dK / dV kernel for one 128-key tile against T query
+    tiles: Q_i (with lse_i) into Q slot i % 3 on barrier ring grp, dO_i (with
+    D_i) into dO slot i % 2 on ring do; before step n the producer waits for
+    step n - 2's last MMA (rel ring), then loads Q_n+1 and dO_n.  The MMA
+    thread: dV += P^T_i dO_i once both elementwise warps wrote P^T_i, S^T_i+1
+    over it, dK += dS^T_i Q_i once both wrote dS^T_i, release, dP^T_i+1 over
+    it.  The elementwise warps check Q_i+1 (dO_i+1) before publishing P^T_i
+    (dS^T_i).  defect: "no_release_wait" drops the producer's wait."""
+    rng = random.Random(seed)
+    bars = {"s0": _Bar("s0", 1), "s1": _Bar("s1", 1), "p0": _Bar("p0", 2), "p1": _Bar("p1", 2),
+            "done": _Bar("done", 1)}
+    for i in range(4):
+        bars[f"grp{i}"] = _Bar(f"grp{i}", 1)
+        bars[f"do{i}"] = _Bar(f"do{i}", 1)
+        bars[f"rel{i}"] = _Bar(f"rel{i}", 1)
+    wait = _waiter(bars)
+    qslot, doslot = [[None, False] for _ in range(3)], [[None, False] for _ in range(2)]
+    qread, doread = [set() for _ in range(3)], [set() for _ in range(2)]
+    tma, pipe = [], []
+    st = {"a": None, "pt": [-1, -1], "b": None, "dst": [-1, -1], "dv": -1, "dk": -1}
+
+    def producer():
+        def load(ring, reads, i, tag, bar, slots):
+            if reads[i % slots]:
+                raise _Hazard(f"{tag} slot {i % slots} reused with reads pending")
+            bars[bar].arrive(tx=1)
+            ring[i % slots][:] = [i, False]
+            reads[i % slots] |= {(tag, i, "mma"), (tag, i, 0), (tag, i, 1), (tag, i, "acc")}
+            tma.append((tag, i % slots, i, bar))
+
+        load(qslot, qread, 0, "q", "grp0", 3)
+        for n in range(T):
+            if n >= 2 and defect != "no_release_wait":
+                yield from _ring_wait(wait, "rel", n - 2)
+            if n + 1 < T:
+                load(qslot, qread, n + 1, "q", f"grp{(n + 1) & 3}", 3)
+            load(doslot, doread, n, "do", f"do{n & 3}", 2)
+            yield "step"
+
+    def mma():
+        yield from _ring_wait(wait, "grp", 0)
+        pipe.extend([("ST", 0), ("commit", "s0")])
+        yield from _ring_wait(wait, "do", 0)
+        pipe.extend([("DPT", 0), ("commit", "s1")])
+        for i in range(T):
+            yield from wait("p0", i & 1, i + 1)
+            pipe.append(("DV", i))
+            if i + 1 < T:
+                pipe.extend([("ST", i + 1), ("commit", "s0")])
+            yield from wait("p1", i & 1, i + 1)
+            pipe.extend([("DK", i), ("commit", f"rel{i & 3}")])
+            if i + 1 < T:
+                pipe.extend([("DPT", i + 1), ("commit", "s1")])
+            yield "step"
+        pipe.append(("commit", "done"))
+
+    def elementwise(cg):
+        for i in range(T):
+            yield from wait("s0", i & 1, i + 1)
+            if st["a"] != i or qslot[i % 3] != [i, True]:
+                raise _Hazard(f"warp {cg} read S^T {st['a']} / lse of Q slot {qslot[i % 3]} for tile {i}")
+            yield "step"
+            if st["a"] != i:
+                raise _Hazard(f"S^T_{i} overwritten while warp {cg} read it")
+            st["pt"][cg] = i
+            qread[i % 3].discard(("q", i, cg))
+            if i + 1 < T:
+                yield from _ring_wait(wait, "grp", i + 1)
+            bars["p0"].arrive()
+            yield from wait("s1", i & 1, i + 1)
+            if st["b"] != i or doslot[i % 2] != [i, True]:
+                raise _Hazard(f"warp {cg} read dP^T {st['b']} / D of dO slot {doslot[i % 2]} for tile {i}")
+            yield "step"
+            st["dst"][cg] = i
+            doread[i % 2].discard(("do", i, cg))
+            if i + 1 < T:
+                yield from _ring_wait(wait, "do", i + 1)
+            bars["p1"].arrive()
+            yield "step"
+        yield from wait("done", 0, 1)
+        if st["dv"] != T - 1 or st["dk"] != T - 1:
+            raise _Hazard("dK / dV read before their last products")
+
+    def execute(op):
+        kind, i = op
+        if kind == "ST":
+            if qslot[i % 3] != [i, True]:
+                raise _Hazard(f"S^T_{i} read Q_{i} before it landed")
+            if i > 0 and st["dv"] < i - 1:
+                raise _Hazard(f"S^T_{i} overwrote P^T_{i - 1} before dV read it")
+            st["a"] = i
+            qread[i % 3].discard(("q", i, "mma"))
+        elif kind == "DPT":
+            if doslot[i % 2] != [i, True]:
+                raise _Hazard(f"dP^T_{i} read dO_{i} before it landed")
+            if i > 0 and st["dk"] < i - 1:
+                raise _Hazard(f"dP^T_{i} overwrote dS^T_{i - 1} before dK read it")
+            st["b"] = i
+            doread[i % 2].discard(("do", i, "mma"))
+        elif kind == "DV":
+            if st["pt"] != [i, i] or st["a"] != i or doslot[i % 2] != [i, True] or st["dv"] != i - 1:
+                raise _Hazard(f"dV_{i} read P^T {st['pt']} / dO slot {doslot[i % 2]}")
+            st["dv"] = i
+            doread[i % 2].discard(("do", i, "acc"))
+        elif kind == "DK":
+            if st["dst"] != [i, i] or st["b"] != i or qslot[i % 3] != [i, True] or st["dk"] != i - 1:
+                raise _Hazard(f"dK_{i} read dS^T {st['dst']} / Q slot {qslot[i % 3]}")
+            st["dk"] = i
+            qread[i % 3].discard(("q", i, "acc"))
+        else:
+            bars[i].arrive()
+
+    def land(copy):
+        tag, idx, owner, bar = copy
+        ring = qslot if tag == "q" else doslot
+        if ring[idx][0] == owner:
+            ring[idx][1] = True
+        bars[bar].complete_tx(1)
+
+    agents = {"producer": producer(), "mma": mma(), "ew0": elementwise(0), "ew1": elementwise(1)}
+    _run(agents, pipe, tma, execute, land, rng)
+
+
 CASES = [(7, 4, 4, None), (7, 4, 3, 0), (7, 4, 3, 1), (5, 2, 3, 0), (5, 2, 3, 1), (5, 2, 1, 0), (5, 2, 1, 1),
          (7, 3, 2, 1), (7, 3, 2, 0), (5, 36, 3, 1), (5, 36, 1, 0), (5, 5, 4, 1), (5, 1, 6, None), (3, 4, 3, None),
          (6, 4, 3, None)]
@@ -283,3 +556,20 @@ def test_eight_slots_overfill_an_operand_group_barrier():
     with pytest.raises(_Hazard, match="more arrivals"):
         for seed in range(400):
             _simulate(8, 4, 3, seed)
+
+
+@pytest.mark.parametrize("T", [1, 2, 3, 5, 9])
+def test_backward_protocols_are_hazard_free(T):
+    """The backward's dQ kernel (K ring of 3, V ring of 2) and dK / dV
+    kernel (Q ring of 3, dO ring of 2) over 1 to 9 tiles."""
+    for seed in range(120):
+        _simulate_dq(T, seed)
+        _simulate_dkdv(T, seed)
+
+
+@pytest.mark.parametrize("sim,defect", [(_simulate_dq, "no_v_wait"), (_simulate_dq, "no_ds_wait"),
+                                        (_simulate_dkdv, "no_release_wait")])
+def test_backward_planted_mistakes_are_caught(sim, defect):
+    with pytest.raises(_Hazard):
+        for seed in range(400):
+            sim(6, seed, defect=defect)
