@@ -1,6 +1,7 @@
-"""A randomised model of the forward attention kernel's synchronisation
-protocol (paper_2602_12529_gb300/csrc/attention.cu, persistent variant),
-run on the CPU.
+"""Randomised models of the tcgen05 kernels' synchronisation protocols, run
+on the CPU: the forward attention kernel (paper_2602_12529_gb300/csrc/
+attention.cu, persistent variant) first, then the attention backward's two
+kernels and the pair GEMM's main pipeline.
 
 The kernel has four agents sharing shared-memory slots, two query tiles and
 TMEM, ordered only by mbarrier phases:
@@ -573,3 +574,118 @@ def test_backward_planted_mistakes_are_caught(sim, defect):
     with pytest.raises(_Hazard):
         for seed in range(400):
             sim(6, seed, defect=defect)
+
+
+def _simulate_gemm_pair(tiles, kblocks, seed, stages=5, defect=None):
+    """The pair GEMM's main pipeline (csrc/gemm.cu, gemm_pair_kernel): two
+    CTAs each load their half of a K block's A and B into stage s of a ring;
+    both halves complete on the leader's full[s] (the leader alone announces
+    the bytes); the leader's MMA thread consumes the stage and its commit
+    arrives on both CTAs' empty[s]; after a tile's last K block it commits
+    tfull[a] to both CTAs for accumulator a (two, alternating); each CTA's
+    epilogue reads its half and arrives on the leader's tempty[a] (one
+    arrival per CTA here, eight warps each in the kernel).  defect:
+    "no_tempty_wait" drops the MMA thread's wait for a free accumulator,
+    "no_empty_wait" the producers' wait for a free stage."""
+    rng = random.Random(seed)
+    bars = {}
+    for s in range(stages):
+        bars[f"full{s}"] = _Bar(f"full{s}", 1)
+        for r in range(2):
+            bars[f"empty{s}.{r}"] = _Bar(f"empty{s}.{r}", 1)
+    for a in range(2):
+        bars[f"tempty{a}"] = _Bar(f"tempty{a}", 2)
+        for r in range(2):
+            bars[f"tfull{a}.{r}"] = _Bar(f"tfull{a}.{r}", 1)
+    wait = _waiter(bars)
+    stage = [[None, [False, False]] for _ in range(stages)]   # (round, both halves landed)
+    pending_reads = [None] * stages                           # round an MMA has yet to read
+    tma, pipe = [], []
+    acc = [{"tile": None, "k": -1, "read": [True, True]} for _ in range(2)]
+
+    def producer(rank):
+        n = 0
+        for _ in range(tiles):
+            for _ in range(kblocks):
+                s, rnd = n % stages, n // stages
+                if defect != "no_empty_wait":
+                    yield from wait(f"empty{s}.{rank}", (rnd & 1) ^ 1, rnd)
+                if pending_reads[s] is not None and pending_reads[s] != rnd:
+                    raise _Hazard(f"stage {s} refilled before the MMA read round {pending_reads[s]}")
+                if rank == 0:
+                    bars[f"full{s}"].arrive(tx=2)
+                if stage[s][0] != rnd:
+                    stage[s][0], stage[s][1] = rnd, [False, False]
+                    pending_reads[s] = rnd
+                tma.append((s, rnd, rank))
+                n += 1
+                yield "step"
+
+    def mma():
+        n = 0
+        for t in range(tiles):
+            a, use = t & 1, t >> 1
+            if defect != "no_tempty_wait":
+                yield from wait(f"tempty{a}", (use & 1) ^ 1, use)
+            for kb in range(kblocks):
+                s, rnd = n % stages, n // stages
+                yield from wait(f"full{s}", rnd & 1, rnd + 1)
+                pipe.append(("MMA", s, rnd, t, kb, a))
+                pipe.append(("commit", [f"empty{s}.0", f"empty{s}.1"]))
+                n += 1
+                yield "step"
+            pipe.append(("commit", [f"tfull{a}.0", f"tfull{a}.1"]))
+
+    def epilogue(rank):
+        for t in range(tiles):
+            a, use = t & 1, t >> 1
+            yield from wait(f"tfull{a}.{rank}", use & 1, use + 1)
+            for _ in range(2):
+                if acc[a]["tile"] != t or acc[a]["k"] != kblocks - 1:
+                    raise _Hazard(f"epilogue {rank} read accumulator {a} holding {acc[a]} for tile {t}")
+                yield "step"
+            acc[a]["read"][rank] = True
+            bars[f"tempty{a}"].arrive()
+
+    def execute(op):
+        if op[0] == "commit":
+            for name in op[1]:
+                bars[name].arrive()
+            return
+        _, s, rnd, t, kb, a = op
+        if stage[s][0] != rnd or stage[s][1] != [True, True]:
+            raise _Hazard(f"MMA of tile {t} block {kb} read stage {s} before both halves landed")
+        pending_reads[s] = None
+        if kb == 0:
+            if not all(acc[a]["read"]):
+                raise _Hazard(f"tile {t} overwrote accumulator {a} before both epilogues read it")
+            acc[a].update(tile=t, k=0, read=[False, False])
+        else:
+            if acc[a]["tile"] != t or acc[a]["k"] != kb - 1:
+                raise _Hazard(f"MMA of tile {t} block {kb} accumulated onto {acc[a]}")
+            acc[a]["k"] = kb
+
+    def land(copy):
+        s, rnd, rank = copy
+        if stage[s][0] == rnd:
+            stage[s][1][rank] = True
+        bars[f"full{s}"].complete_tx(1)
+
+    agents = {"prod0": producer(0), "prod1": producer(1), "mma": mma(), "epi0": epilogue(0), "epi1": epilogue(1)}
+    _run(agents, pipe, tma, execute, land, rng)
+
+
+@pytest.mark.parametrize("tiles,kblocks", [(1, 1), (3, 2), (5, 7), (4, 48), (9, 3)])
+def test_gemm_pair_pipeline_is_hazard_free(tiles, kblocks):
+    """Five stages, two accumulators, K blocks from 1 to 48 (K = 3072 at
+    BK 64), several tiles per CTA pair."""
+    for seed in range(100):
+        _simulate_gemm_pair(tiles, kblocks, seed)
+
+
+@pytest.mark.parametrize("defect,match", [("no_tempty_wait", "accumulator"),
+                                          ("no_empty_wait", "stage|landed|more arrivals")])
+def test_gemm_pair_planted_mistakes_are_caught(defect, match):
+    with pytest.raises(_Hazard, match=match):
+        for seed in range(400):
+            _simulate_gemm_pair(6, 4, seed, defect=defect)
