@@ -1,7 +1,7 @@
 """Randomised models of the tcgen05 kernels' synchronisation protocols, run
 on the CPU: the forward attention kernel (paper_2602_12529_gb300/csrc/
 attention.cu, persistent variant) first, then the attention backward's two
-kernels and the pair GEMM's main pipeline.
+kernels, the pair GEMM's main pipeline and its gated-residual epilogue.
 
 The kernel has four agents sharing shared-memory slots, two query tiles and
 TMEM, ordered only by mbarrier phases:
@@ -689,3 +689,105 @@ def test_gemm_pair_planted_mistakes_are_caught(defect, match):
     with pytest.raises(_Hazard, match=match):
         for seed in range(400):
             _simulate_gemm_pair(6, 4, seed, defect=defect)
+
+
+def _simulate_gated_epilogue(tiles, chunks, seed, workers=3, defect=None):
+    """The gated-residual epilogue's chunk ring (csrc/gemm.cu, epilogue_tile):
+    per column group two shared-memory buffers; chunk c of a tile uses
+    buffer c % 2.  The group's leader loads the fp32 residual chunk by TMA
+    (rfull[b]: its own arrival plus the bytes), every thread waits for it,
+    updates its row, arrives on rdone[b]; the leader waits for all arrivals,
+    stores the chunk by TMA and, before reloading the buffer with chunk
+    c + 2 (or the next tile's first chunks), waits until its stores have
+    read shared memory (bulk_wait_read).  Worker 0 is the leader.  defect:
+    "no_store_wait" drops the bulk_wait_read, "no_rdone_wait" the leader's
+    wait for every thread's update."""
+    rng = random.Random(seed)
+    bars = {}
+    for b in range(2):
+        bars[f"rfull{b}"] = _Bar(f"rfull{b}", 1)
+        bars[f"rdone{b}"] = _Bar(f"rdone{b}", workers)
+    wait = _waiter(bars)
+    buf = [{"chunk": None, "landed": False, "updated": set()} for _ in range(2)]
+    stores, loads = [], []   # the TMA engine: stores reading a buffer, loads filling one
+
+    def store_free():
+        while stores:
+            yield "blocked"
+
+    def load(b, chunk):
+        if any(sb == b for sb, _ in stores):
+            raise _Hazard(f"buffer {b} reloaded while a store still reads it")
+        if buf[b]["chunk"] is not None and len(buf[b]["updated"]) < workers:
+            raise _Hazard(f"buffer {b} reloaded before every thread updated chunk {buf[b]['chunk']}")
+        bars[f"rfull{b}"].arrive(tx=1)
+        buf[b].update(chunk=chunk, landed=False, updated=set())
+        loads.append((b, chunk))
+
+    def worker(w):
+        ruse = [0, 0]
+        for t in range(tiles):
+            if w == 0:
+                for c in range(min(2, chunks)):
+                    if defect != "no_store_wait":
+                        yield from store_free()
+                    load(c, (t, c))
+            for c in range(chunks):
+                b = c & 1
+                yield from wait(f"rfull{b}", ruse[b] & 1, ruse[b] + 1)
+                for _ in range(2):   # the row update spans two events
+                    if buf[b]["chunk"] != (t, c) or not buf[b]["landed"]:
+                        raise _Hazard(f"thread {w} updated buffer {b} holding {buf[b]['chunk']} for {(t, c)}")
+                    yield "step"
+                buf[b]["updated"].add(w)
+                bars[f"rdone{b}"].arrive()
+                if w == 0 and defect != "no_rdone_wait":
+                    yield from wait(f"rdone{b}", ruse[b] & 1, ruse[b] + 1)
+                ruse[b] += 1
+                if w == 0:
+                    if len(buf[b]["updated"]) < workers:
+                        raise _Hazard(f"chunk {(t, c)} stored before every thread updated it")
+                    stores.append((b, (t, c)))
+                    if c + 2 < chunks:
+                        if defect != "no_store_wait":
+                            yield from store_free()
+                        load(b, (t, c + 2))
+                yield "step"
+
+    agents = {f"w{w}": worker(w) for w in range(workers)}
+    done = set()
+    for _ in range(10 ** 6):
+        live = [a for a in agents if a not in done]
+        hw = (["store"] if stores else []) + (["load"] if loads else [])
+        if not live and not hw:
+            return
+        choice = rng.choice(live + hw * 2)
+        if choice == "store":
+            stores.pop(rng.randrange(len(stores)))
+        elif choice == "load":
+            b, chunk = loads.pop(rng.randrange(len(loads)))
+            if buf[b]["chunk"] == chunk:
+                buf[b]["landed"] = True
+            bars[f"rfull{b}"].complete_tx(1)
+        else:
+            try:
+                next(agents[choice])
+            except StopIteration:
+                done.add(choice)
+    raise _Hazard("no progress: deadlock")
+
+
+@pytest.mark.parametrize("tiles,chunks", [(1, 1), (1, 2), (3, 4), (4, 3), (2, 8)])
+def test_gated_epilogue_ring_is_hazard_free(tiles, chunks):
+    """Four chunks per column group (256-column pair tiles, eight epilogue
+    warps), and other counts; several tiles in a row."""
+    for seed in range(100):
+        _simulate_gated_epilogue(tiles, chunks, seed)
+
+
+@pytest.mark.parametrize("defect,match", [("no_store_wait", "store still reads"),
+                                          ("no_rdone_wait", "every thread")])
+def test_gated_epilogue_planted_mistakes_are_caught(defect, match):
+    with pytest.raises(_Hazard, match=match):
+        for seed in range(400):
+            _simulate_gated_epilogue(3, 4, seed, defect=defect)
